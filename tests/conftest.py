@@ -1,0 +1,17 @@
+"""Shared pytest configuration.
+
+Marker ``gpu``: the test needs a CUDA device (a GB300) and the compiled CUDA
+library.  The CPU suite runs with ``-m "not gpu"``.
+"""
+import os
+import sys
+
+import pytest
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+if ROOT not in sys.path:
+    sys.path.insert(0, ROOT)
+
+
+def pytest_configure(config):
+    config.addinivalue_line("markers", "gpu: needs a CUDA device and the compiled sm_103a library")

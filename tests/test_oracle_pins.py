@@ -1,0 +1,380 @@
+"""Pins of the CPU oracle against things other than itself (CPU only).
+
+Each test checks the oracle against what the paper or the mathematics fixes:
+printed values of the Appendix A.1 microcase, library routines (torch's E4M3
+cast, numpy's IEEE fp32 division and fp64 sums), closed forms, invariants the
+paper states (h = 1 reduces to plain MSE search; the shift 0 is always in the
+window so the chosen error never exceeds the initial one; a window covering the
+ladder equals the full E4M3 grid), and brute force on tiny inputs written as a
+different method (nearest-value search instead of midpoint comparisons).
+"""
+import json
+import math
+import os
+
+import numpy as np
+import pytest
+import torch
+
+import oracle
+
+GOLDEN = os.path.join(os.path.dirname(__file__), "golden")
+E2M1_GRID = [0.0, 0.5, 1.0, 1.5, 2.0, 3.0, 4.0, 6.0]  # OCP FP4 E2M1 magnitudes
+
+
+def to_bf16_bits(a) -> np.ndarray:
+    t = torch.as_tensor(np.asarray(a, dtype=np.float32)).to(torch.bfloat16)
+    return t.view(torch.int16).numpy().view(np.uint16)
+
+
+def bits_to_f64(b: np.ndarray) -> np.ndarray:
+    return torch.from_numpy(b.view(np.int16).copy()).view(torch.bfloat16).double().numpy()
+
+
+def random_weights(rng, m, n, sigma=0.02):
+    w = rng.standard_t(4, size=(m, n)) * sigma
+    k = max(1, int(round(1e-3 * m * n)))
+    idx = rng.choice(m * n, size=k, replace=False)
+    w.reshape(-1)[idx] *= 20
+    return to_bf16_bits(w)
+
+
+def random_h(rng, n):
+    return (np.exp(rng.standard_normal(n)) ** 2 * 2048).astype(np.float32)
+
+
+# ---------------------------------------------------------------- formats
+
+def test_e4m3_table_matches_torch_view_cast():
+    ours = oracle.e4m3_decode_table()
+    ref = torch.arange(256, dtype=torch.uint8).view(torch.float8_e4m3fn).double().numpy()
+    nan = np.isnan(ref)
+    assert np.array_equal(np.isnan(ours), nan)
+    assert np.array_equal(ours[~nan], ref[~nan])
+    assert list(np.nonzero(nan)[0]) == [0x7F, 0xFF]
+
+
+def test_e4m3_ladder_shape():
+    t = oracle.e4m3_decode_table()
+    ladder = t[1:127]  # bytes 0x01..0x7E: the sorted positive finite values L+ (Eq. 8)
+    assert ladder.size == 126
+    assert np.all(np.diff(ladder) > 0)
+    assert ladder[0] == 2.0 ** -9 and ladder[-1] == 448.0
+    assert t[0] == 0.0
+
+
+def test_e2m1_table_is_the_ocp_grid():
+    t = oracle.e2m1_decode_table()
+    assert list(t[:8]) == E2M1_GRID
+    assert list(t[8:]) == [-v for v in E2M1_GRID]
+    # the paper's Clip range and its outer codes {+-4, +-6} (Sec. 3.1, Sec. 3.3)
+    assert t.max() == 6.0 and t.min() == -6.0 and 4.0 in t
+
+
+def nearest_e2m1(a: float, s: float) -> int:
+    """Brute force: nearest grid value to a/s by distance a - v*s; ties to even code."""
+    d = [abs(a - v * s) for v in E2M1_GRID]
+    best = min(d)
+    ks = [k for k in range(8) if d[k] == best]
+    return ks[0] if len(ks) == 1 else [k for k in ks if k % 2 == 0][0]
+
+
+def test_e2m1_rounding_against_brute_force_including_midpoints():
+    s = 0.8125  # exact binary scale so midpoints are exactly representable
+    vals = []
+    for i in range(1, 8):
+        mid = 0.5 * (E2M1_GRID[i - 1] + E2M1_GRID[i]) * s
+        vals += [mid, np.nextafter(mid, 0), np.nextafter(mid, 10)]
+    vals += list(np.linspace(0, 9 * s, 997)) + [6 * s, 7 * s, 100.0, 0.0]
+    w = np.array(vals + [-v for v in vals])
+    _, codes = oracle.quantize_at_scale(w, s)
+    expect = [nearest_e2m1(abs(v), s) for v in w]
+    assert list(np.abs(codes)) == expect
+    # ties go to the even code: 0.25->0, 0.75->1, 1.25->1, 1.75->2, 2.5->2, 3.5->4, 5->4
+    ties = np.array([0.25, 0.75, 1.25, 1.75, 2.5, 3.5, 5.0]) * s
+    _, c = oracle.quantize_at_scale(ties, s)
+    assert [E2M1_GRID[k] for k in c] == [0.0, 1.0, 1.0, 2.0, 2.0, 4.0, 4.0]
+
+
+# ---------------------------------------------------------------- microcase (App. A.1)
+
+def test_calibration_microcase_from_the_paper():
+    g = json.load(open(os.path.join(GOLDEN, "microcase.json")))
+    w = np.array(g["w"])
+    X = np.array(g["X"])
+    for row in g["rows"]:
+        s = np.abs(w).max() / 6.0 if row.get("scale_exact") == "max|w|/6" else row["scale"]
+        w_hat, codes = oracle.quantize_at_scale(w, s)
+        np.testing.assert_allclose(w_hat, row["w_hat"], atol=0.01)
+        werr = oracle.output_error(np.eye(4), w - w_hat)        # sum_j (w_j - w_hat_j)^2
+        oerr = oracle.output_error(X, w - w_hat)                # ||X (w - w_hat)^T||^2, Eq. 3
+        assert abs(werr - row["weight_error"]) <= 0.01, row["name"]
+        assert abs(oerr - row["output_error"]) <= 0.01, row["name"]
+        if "codes" in row:
+            signed = [np.sign(c) * E2M1_GRID[abs(c)] for c in codes]
+            assert signed == row["codes"]
+    # the min-max row is printed at its exact scale: 3 decimals agree exactly
+    s = 4.88 / 6.0
+    w_hat, _ = oracle.quantize_at_scale(w, s)
+    assert round(oracle.output_error(np.eye(4), w - w_hat), 3) == 0.573
+    assert round(oracle.output_error(X, w - w_hat), 3) == 3.927
+
+
+# ---------------------------------------------------------------- Hessian diagonal (Eq. 4)
+
+def test_hessian_constant_input_closed_form():
+    for c in (0.5, -1.5, 3.0):
+        x = to_bf16_bits(np.full((37, 48), c))
+        h = np.zeros(48)
+        oracle.hessian_accumulate(x, h)
+        assert np.all(h == 37 * c * c)
+
+
+def test_hessian_one_hot_rows_and_chunking():
+    T, n = 50, 32
+    x = np.zeros((T, n))
+    cols = np.arange(T) % n
+    x[np.arange(T), cols] = 2.0
+    bits = to_bf16_bits(x)
+    h = np.zeros(n)
+    oracle.hessian_accumulate(bits[:17], h)  # two chunks accumulate into one h
+    oracle.hessian_accumulate(bits[17:], h)
+    expect = np.bincount(cols, minlength=n) * 4.0
+    assert np.array_equal(h, expect)
+
+
+def test_hessian_random_against_numpy_and_strided_rows():
+    rng = np.random.default_rng(3)
+    x = to_bf16_bits(rng.standard_normal((300, 80)) * np.exp(rng.standard_normal(80)))
+    ref = (bits_to_f64(x) ** 2).sum(axis=0)
+    h = np.zeros(80)
+    oracle.hessian_accumulate(x, h)
+    np.testing.assert_allclose(h, ref, rtol=1e-13)
+    # leading dimension: use the first 48 columns of a wider buffer
+    h2 = np.zeros(48)
+    oracle.hessian_accumulate(x, h2, ld=80, n=48)
+    np.testing.assert_allclose(h2, ref[:48], rtol=1e-13)
+
+
+# ---------------------------------------------------------------- global scale and RTN codes
+
+def test_global_scale_is_ieee_fp32_division():
+    rng = np.random.default_rng(4)
+    for _ in range(200):
+        w = random_weights(rng, 4, 64, sigma=float(np.exp(rng.normal(-3, 2))))
+        s, amax = oracle.global_scale(w)
+        assert amax == np.abs(bits_to_f64(w)).max()
+        assert s == np.float32(amax) / np.float32(2688.0)   # numpy: correctly rounded fp32
+    s, amax = oracle.global_scale(np.zeros((2, 16), np.uint16))
+    assert amax == 0.0 and s == np.float32(1.0)
+
+
+def e4m3_code_by_torch(q: np.ndarray) -> np.ndarray:
+    """torch's round-to-nearest-even E4M3 cast of float32 values (overflow -> NaN byte)."""
+    return torch.from_numpy(q.astype(np.float32)).to(torch.float8_e4m3fn).view(torch.uint8).numpy()
+
+
+def test_rtn_codes_against_torch_cast_on_exact_quotients():
+    # amax = 2688 * 2^-10 makes s_g = 2^-10 exactly; a group whose max is 6*v*2^-10 then has
+    # the exact quotient v, so torch's cast of v is the E4M3 round-to-nearest-even of Eq. 7.
+    ladder = oracle.e4m3_decode_table()[0:127]
+    mids = 0.5 * (ladder[:-1] + ladder[1:])
+    vs = [v for v in np.concatenate([ladder[1:], mids]) if v <= 448]
+    rows = []
+    for v in vs:
+        g = np.zeros(16)
+        g[3] = 6 * v * 2.0 ** -10
+        rows.append(g)
+    w = np.stack(rows).reshape(len(rows), 16)
+    w[0, 0] = 2688 * 2.0 ** -10                          # sets amax, s_g = 2^-10
+    bits = to_bf16_bits(w)
+    assert np.array_equal(bits_to_f64(bits), w)          # all values are exact in bf16
+    s_g, _ = oracle.global_scale(bits)
+    assert s_g == np.float32(2.0 ** -10)
+    codes = oracle.rtn_codes(bits, s_g).reshape(-1)
+    amax_g = np.abs(w).max(axis=1)
+    expect = e4m3_code_by_torch(amax_g / (6 * 2.0 ** -10))
+    expect = np.maximum(expect, 1)                        # code 0 clamps to 1
+    assert np.array_equal(codes, expect)
+
+
+def test_rtn_codes_against_torch_cast_on_random_groups():
+    rng = np.random.default_rng(5)
+    w = random_weights(rng, 64, 256)
+    s_g, _ = oracle.global_scale(w)
+    codes = oracle.rtn_codes(w, s_g)
+    amax_g = np.abs(bits_to_f64(w)).reshape(64, 16, 16).max(axis=2)
+    q = amax_g / (6.0 * float(s_g))
+    expect = np.maximum(e4m3_code_by_torch(q), 1)
+    expect = np.where(expect == 127, 126, expect)         # saturate instead of NaN
+    assert np.array_equal(codes, expect)
+    assert codes.max() == 126                             # the group holding amax hits 448
+
+
+# ---------------------------------------------------------------- scale search (Algorithm 1)
+
+def brute_force_group(g_bits, h, s_g, c0, down, up):
+    """Algorithm 1 by brute force: nearest-value FP4 search, exhaustive window, tie rule
+    (E, |shift|, shift).  Returns (best code, magnitude codes, errors by code)."""
+    a = np.abs(bits_to_f64(g_bits))
+    ladder = oracle.e4m3_decode_table()
+    errs = {}
+    for d in range(-down, up + 1):
+        c = min(max(c0 + d, 1), 126)
+        if c in errs:
+            continue
+        s = float(s_g) * ladder[c]
+        ks = [nearest_e2m1(v, s) for v in a]
+        errs[c] = (math.fsum((1.0 if h is None else float(h[j])) * (a[j] - E2M1_GRID[ks[j]] * s) ** 2
+                             for j in range(16)), ks)
+    best = min(errs, key=lambda c: (errs[c][0], abs(c - c0), c - c0))
+    return best, errs[best][1], {c: e for c, (e, _) in errs.items()}
+
+
+def test_refine_matches_brute_force_on_tiny_inputs():
+    rng = np.random.default_rng(6)
+    checked = 0
+    for trial in range(6):
+        m, n = 4, 64
+        w = random_weights(rng, m, n)
+        h = random_h(rng, n)
+        down, up = [(4, 4), (9, 6), (2, 7), (0, 3), (5, 0), (1, 1)][trial]
+        s_g, _ = oracle.global_scale(w)
+        out = oracle.refine(w, h, s_g, None, down, up)
+        rtn = oracle.rtn_codes(w, s_g)
+        for r in range(m):
+            for i in range(n // 16):
+                g = w[r, 16 * i:16 * i + 16]
+                best, ks, errs = brute_force_group(g, h[16 * i:16 * i + 16], s_g, int(rtn[r, i]),
+                                                   down, up)
+                assert math.isclose(out["e_best"][r, i], errs[best], rel_tol=1e-12)
+                assert math.isclose(out["e_init"][r, i], errs[int(rtn[r, i])], rel_tol=1e-12)
+                if out["near_tie"][r, i]:
+                    continue
+                assert out["codes"][r, i] == best
+                assert out["delta"][r, i] == best - int(rtn[r, i])
+                signs = (g >> 15).astype(np.uint8)
+                nib = (signs << 3) | np.array(ks, np.uint8)
+                assert np.array_equal(out["packed"][r, 8 * i:8 * i + 8], nib[0::2] | (nib[1::2] << 4))
+                checked += 1
+    assert checked > 80
+
+
+def test_h_one_reduces_to_plain_mse_search():
+    rng = np.random.default_rng(7)
+    w = random_weights(rng, 8, 128)
+    s_g, _ = oracle.global_scale(w)
+    a = oracle.refine(w, None, s_g, None, 4, 4)
+    b = oracle.refine(w, np.ones(128, np.float32), s_g, None, 4, 4)
+    for k in ("codes", "packed", "e_best"):
+        assert np.array_equal(a[k], b[k])
+    rtn = oracle.rtn_codes(w, s_g)
+    for r in range(8):
+        for i in range(8):
+            g = w[r, 16 * i:16 * i + 16]
+            best, _, _ = brute_force_group(g, None, s_g, int(rtn[r, i]), 4, 4)
+            if not a["near_tie"][r, i]:
+                assert a["codes"][r, i] == best
+
+
+def test_chosen_error_never_exceeds_initial_error():
+    rng = np.random.default_rng(8)
+    w = random_weights(rng, 32, 256)
+    h = random_h(rng, 256)
+    s_g, _ = oracle.global_scale(w)
+    for down, up in ((4, 4), (9, 6), (0, 0), (16, 16)):
+        out = oracle.refine(w, h, s_g, None, down, up)
+        assert np.all(out["e_best"] <= out["e_init"])
+        assert np.all(out["delta"] >= -down) and np.all(out["delta"] <= up)
+        assert out["codes"].min() >= 1 and out["codes"].max() <= 126
+    out = oracle.refine(w, h, s_g, None, 0, 0)
+    assert np.array_equal(out["codes"], oracle.rtn_codes(w, s_g))   # empty window = RTN
+
+
+def test_full_window_equals_full_e4m3_grid():
+    rng = np.random.default_rng(9)
+    w = random_weights(rng, 6, 64)
+    h = random_h(rng, 64)
+    s_g, _ = oracle.global_scale(w)
+    small = oracle.refine(w, h, s_g, None, 4, 4)
+    full = oracle.refine(w, h, s_g, None, 125, 125)
+    assert np.all(full["e_best"] <= small["e_best"])
+    all_codes = np.arange(1, 127, dtype=np.uint8)
+    for r in range(6):
+        for i in range(4):
+            errs = oracle.group_errors(w[r, 16 * i:16 * i + 16], h[16 * i:16 * i + 16], s_g, all_codes)
+            assert full["e_best"][r, i] == errs.min()
+            if not full["near_tie"][r, i]:
+                assert full["codes"][r, i] == all_codes[np.argmin(errs)]
+
+
+def test_codes_invariant_under_h_power_of_two_scaling_and_row_permutation():
+    rng = np.random.default_rng(10)
+    w = random_weights(rng, 16, 128)
+    h = random_h(rng, 128)
+    s_g, _ = oracle.global_scale(w)
+    base = oracle.refine(w, h, s_g, None, 4, 4)
+    for k in (-7, 3, 20):
+        other = oracle.refine(w, (h * np.float32(2.0 ** k)).astype(np.float32), s_g, None, 4, 4)
+        assert np.array_equal(base["codes"], other["codes"])
+        assert np.array_equal(base["packed"], other["packed"])
+    perm = rng.permutation(16)
+    other = oracle.refine(w[perm], h, s_g, None, 4, 4)
+    assert np.array_equal(base["codes"][perm], other["codes"])
+    assert np.array_equal(base["packed"][perm], other["packed"])
+
+
+def test_init_codes_path_and_window_clipping_at_both_ends():
+    rng = np.random.default_rng(11)
+    w = random_weights(rng, 8, 64)
+    h = random_h(rng, 64)
+    s_g, _ = oracle.global_scale(w)
+    rtn = oracle.rtn_codes(w, s_g)
+    a = oracle.refine(w, h, s_g, None, 4, 4)
+    b = oracle.refine(w, h, s_g, rtn, 4, 4)
+    for k in a:
+        assert np.array_equal(a[k], b[k])
+    # init codes at the ladder ends: the walk clips to [1, 126]
+    lo = np.ones_like(rtn)
+    hi = np.full_like(rtn, 126)
+    out_lo = oracle.refine(w, h, s_g, lo, 4, 4)
+    out_hi = oracle.refine(w, h, s_g, hi, 4, 4)
+    assert out_lo["codes"].max() <= 5 and out_lo["delta"].min() >= 0
+    assert out_hi["codes"].min() >= 122 and out_hi["delta"].max() <= 0
+
+
+def test_pack_matches_refine_and_decodes_to_the_quantized_weights():
+    rng = np.random.default_rng(12)
+    w = random_weights(rng, 8, 96)
+    h = random_h(rng, 96)
+    s_g, _ = oracle.global_scale(w)
+    out = oracle.refine(w, h, s_g, None, 4, 4)
+    packed = oracle.pack(w, s_g, out["codes"])
+    assert np.array_equal(packed, out["packed"])
+    # decode: nibble value * s_g * lambda(code) is the FP4 projection of w (Eq. 12)
+    e2 = oracle.e2m1_decode_table()
+    e4 = oracle.e4m3_decode_table()
+    lo, hi = packed & 15, packed >> 4
+    nib = np.empty((8, 96), np.uint8)
+    nib[:, 0::2], nib[:, 1::2] = lo, hi
+    scale = float(s_g) * e4[np.repeat(out["codes"], 16, axis=1)]
+    wq = e2[nib] * scale
+    wf = bits_to_f64(w)
+    for r in range(8):
+        for j in range(96):
+            k = nearest_e2m1(abs(wf[r, j]), scale[r, j])
+            assert abs(wq[r, j]) == E2M1_GRID[k] * scale[r, j]
+            assert (nib[r, j] >> 3) == (w[r, j] >> 15)
+
+
+def test_zero_groups_and_negative_zero():
+    w = np.zeros((2, 32))
+    w[1, 20] = 0.5                                           # second group of row 1 non-zero
+    bits = to_bf16_bits(w)
+    bits[0, 5] = 0x8000                                      # -0.0
+    s_g, _ = oracle.global_scale(bits)
+    out = oracle.refine(bits, None, s_g, None, 4, 4)
+    # all-zero groups: every candidate has E = 0, the tie rule keeps the RTN code (1)
+    assert out["codes"][0, 0] == 1 and out["delta"][0, 0] == 0 and out["near_tie"][0, 0] == 1
+    assert out["packed"][0, 2] == 0x80                       # -0 (odd element: high nibble) keeps its sign
+    assert out["codes"][1, 1] == 126 or out["e_best"][1, 1] == 0.0
