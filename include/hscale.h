@@ -1,0 +1,152 @@
+/*
+ * hscale.h -- C ABI of the GB300 (sm_103a) H-Scale hot path.
+ *
+ * H-Scale ("Hessian-Guided Scale Refinement for NVFP4 Sub-Byte LLM Inference")
+ * picks each 16-element NVFP4 group's E4M3 local scale by a windowed search that
+ * minimises a diagonal-Hessian weighted reconstruction error.  The data-parallel
+ * hot path has two parts, both exposed here:
+ *
+ *   1. hscale_hessian_diag_accumulate   h_j += sum_t x_tj^2 over a token chunk
+ *                                       (Sec. 3.2, Eq. 4: h = diag(X^T X))
+ *   2. hscale_rtn_scales                global scale s_g and the RTN local-scale codes
+ *                                       (Sec. 3.3 "Initialization", Eq. 7)
+ *      hscale_refine_scales             Algorithm 1: walk the E4M3 ladder around the
+ *                                       initial code (Eqs. 8-10), quantize the group to
+ *                                       E2M1 under each candidate (Eqs. 11-12), keep the
+ *                                       code with the smallest sum_j h_j (w_j - s q_j)^2
+ *                                       (Eqs. 6, 13), then re-quantize and pack
+ *      hscale_pack_nvfp4                final FP4 quantization with given codes
+ *                                       (Sec. 3.3 "Final re-quantization", Eq. 2)
+ *
+ * Equation numbers count the paper's displayed equations in order (Eq. 1 is the
+ * effective scale s = s_g * l).
+ *
+ * Conventions shared by every entry point
+ * ---------------------------------------
+ * - All pointers except `stream` are DEVICE pointers owned by the caller; the
+ *   library allocates and frees nothing.  Work is enqueued on `stream` (a
+ *   cudaStream_t passed as void*, NULL = legacy default stream) and nothing
+ *   synchronises: results are ready when the stream reaches them.
+ * - Matrices are row-major.  W is [m, n] bfloat16 with contiguous rows; groups of 16
+ *   run along n (the input-channel axis), so n must be a multiple of 16.
+ * - Local-scale codes are E4M3 bytes in [1, 126] (the index iota of Algorithm 1 is
+ *   the byte itself), stored [m, n/16] row-major, one byte per group.
+ * - Packed FP4 is [m, n/2] bytes: element 2j of a row in the low nibble of byte j,
+ *   element 2j+1 in the high nibble.  A nibble is sign<<3 | E2M1 magnitude code; the
+ *   sign is the sign bit of w, also when the magnitude rounds to zero.
+ * - The effective scale of a group is s_g * E4M3(code); dequantized weight =
+ *   E2M1(nibble) * s_g * E4M3(code).
+ * - Rounding is round-to-nearest-even on the exact real quotients w / (s_g * l) and
+ *   amax_group / (6 s_g), decided exactly in the kernels; E2M1 saturates at 6, E4M3
+ *   at 448.
+ * - Inputs are assumed finite; NaN or Inf in W, X or h gives unspecified codes.
+ *   s_g must be a positive normal fp32 number.
+ * - Zero-sized inputs (m, n or tokens == 0) return HSCALE_OK and launch nothing.
+ * - Every argument is checked before anything is enqueued; a failed check returns
+ *   its status and enqueues nothing.  A launch failure returns HSCALE_ERR_CUDA
+ *   (cudaGetLastError after the launch).  No C++ exception crosses the ABI.
+ * - Results are deterministic: the same inputs on the same GPU model give the same
+ *   bits on every run.
+ */
+#ifndef HSCALE_H
+#define HSCALE_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef enum hscale_status {
+  HSCALE_OK = 0,
+  HSCALE_ERR_NULL = 1,      /* a required pointer is NULL                            */
+  HSCALE_ERR_SHAPE = 2,     /* negative size, n not a multiple of 16, ld < n, ...    */
+  HSCALE_ERR_ALIGN = 3,     /* a pointer or leading dimension breaks the alignment   */
+  HSCALE_ERR_ARG = 4,       /* an out-of-range scalar argument (window half-widths)  */
+  HSCALE_ERR_CUDA = 5,      /* the CUDA runtime reported an error for a launch       */
+  HSCALE_ERR_WORKSPACE = 6  /* workspace missing or smaller than the query says      */
+} hscale_status;
+
+/* Static, NUL-terminated description of a status code (unknown codes included). */
+const char* hscale_status_string(int status);
+
+/* ABI version of this header (incremented on any signature change). */
+int hscale_abi_version(void);
+
+/*
+ * Hessian diagonal, one token chunk (Sec. 3.2, Eq. 4).
+ *
+ *   h[j] += sum_{t < tokens} x[t * ld_x + j]^2      for j < n
+ *
+ * x      [tokens, ld_x] bfloat16, 16-byte aligned; only the first n columns are read.
+ * h      [n] fp32, read and written (accumulated in place).  Zero it before the first
+ *        chunk; streaming a calibration set is one call per chunk on the same h.
+ * n      multiple of 8; ld_x >= n and a multiple of 8.
+ * Arithmetic: x^2 is exact in fp32; sums are fp32 in a fixed order (per-thread runs of
+ * at most 1024 tokens, then fixed-order trees inside the CTA and across a thread-block
+ * cluster), so each call adds a relative error of at most about 1100 * 2^-24 to h.
+ * Nothing else is touched: the call needs no workspace.
+ */
+int hscale_hessian_diag_accumulate(const void* x_bf16, int64_t tokens, int64_t n, int64_t ld_x,
+                                   float* h, void* stream);
+
+/*
+ * Global scale and RTN local-scale codes (Sec. 3.3 "Initialization", Eq. 7).
+ *
+ *   s_g      = fl32(amax|W| / (6 * 448))          (1.0 when W is all zero)
+ *   codes[g] = max(1, RNE_E4M3_sat(amax_g / (6 s_g)))   for every group g
+ *
+ * w             [m, n] bfloat16, 16-byte aligned, n % 16 == 0.
+ * global_scale  device fp32 scalar, written.
+ * codes         [m, n/16] bytes, written; may be NULL to compute only s_g.
+ * workspace     at least hscale_rtn_workspace_bytes() bytes of device memory, 4-byte
+ *               aligned; its contents on entry do not matter (the call clears it on
+ *               the stream before use).
+ */
+size_t hscale_rtn_workspace_bytes(void);
+int hscale_rtn_scales(const void* w_bf16, int64_t m, int64_t n, float* global_scale,
+                      uint8_t* codes, void* workspace, size_t workspace_bytes, void* stream);
+
+/*
+ * H-Scale refinement, Algorithm 1 (Eqs. 6-13), fused with the final re-quantization.
+ *
+ * For every group with initial code c (init_codes[g] with its sign bit cleared and
+ * clamped to [1, 126]; or, when init_codes is NULL, the RTN code of Eq. 7 computed in
+ * place), the candidates are the distinct codes clip(c + delta, 1, 126) for
+ * delta = -down .. up; each candidate's error is sum_j h_j (|w_j| - s q_j)^2 with
+ * s = s_g * E4M3(code) and q_j the E2M1 round-to-nearest-even of |w_j| / s.  The code
+ * with the smallest error wins; exact ties keep the smaller |delta|, then the smaller
+ * delta.  Codes whose errors differ by less than about 1e-6 relative may be ordered
+ * either way (fp32 error sums).
+ *
+ * w             [m, n] bfloat16, 16-byte aligned, n % 16 == 0.
+ * h             [n] fp32, 16-byte aligned; NULL means h = 1 (plain weight MSE search).
+ * global_scale  device fp32 scalar s_g (e.g. from hscale_rtn_scales).
+ * init_codes    [m, n/16] bytes or NULL.
+ * down, up      window half-widths, 0 <= down, up <= 125 (the paper's default is
+ *               down = 9, up = 6, i.e. K = 16 candidates).
+ * codes_out     [m, n/16] bytes, written; may alias init_codes.
+ * packed_out    [m, n/2] bytes, 8-byte aligned, written; may be NULL.
+ */
+int hscale_refine_scales(const void* w_bf16, const float* h, int64_t m, int64_t n,
+                         const float* global_scale, const uint8_t* init_codes, int32_t down,
+                         int32_t up, uint8_t* codes_out, uint8_t* packed_out, void* stream);
+
+/*
+ * Final FP4 quantization with given codes (Sec. 3.3 "Final re-quantization", Eq. 2):
+ * packed nibble of w = sign(w) << 3 | RNE_E2M1_sat(|w| / (s_g * E4M3(code))).
+ *
+ * w             [m, n] bfloat16, 16-byte aligned, n % 16 == 0.
+ * codes         [m, n/16] bytes; the sign bit is ignored and a code is read as
+ *               clamp(code, 1, 126), the clip of Eq. 10.
+ * packed_out    [m, n/2] bytes, 8-byte aligned, written.
+ */
+int hscale_pack_nvfp4(const void* w_bf16, int64_t m, int64_t n, const float* global_scale,
+                      const uint8_t* codes, uint8_t* packed_out, void* stream);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* HSCALE_H */

@@ -333,7 +333,8 @@ void oracle_pack(const uint16_t* w, int64_t m, int64_t n, float s_g, const uint8
     for (int64_t i = 0; i < ng; ++i) {
       const int64_t gi = r * ng + i;
       uint8_t q[16];
-      int c = codes[gi] & 0x7F;
+      int c = codes[gi] & 0x7F;  /* a code off the ladder is read as its clipped index (Eq. 10) */
+      if (c < 1) c = 1;
       if (c > E4M3_MAX_CODE) c = E4M3_MAX_CODE;
       group_error(w + r * n + i * 16, NULL, (double)s_g, c, q);
       pack_group(w + r * n + i * 16, q, packed_out + gi * 8);

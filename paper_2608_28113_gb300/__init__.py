@@ -1,1 +1,188 @@
-"""GB300-native H-Scale hot path (placeholder; the binding is added with the CUDA library)."""
+"""GB300-native (sm_103a) H-Scale hot path: Python binding of ``libhscale.so``.
+
+The functions here have the names of the C entry points in ``include/hscale.h`` and
+only marshal arguments: they take torch CUDA tensors, check dtype/shape/device, pass
+raw device pointers and the current CUDA stream through ctypes, and raise
+``HScaleError`` on a non-zero status.  Every step of the path runs in the CUDA
+kernels; there is no CPU fallback: if the compiled library is missing, loading it
+raises.
+
+Paper map: ``hscale_hessian_diag_accumulate`` is h = diag(X^T X) (Sec. 3.2, Eq. 4);
+``hscale_rtn_scales`` the global scale and RTN codes (Sec. 3.3, Eq. 7);
+``hscale_refine_scales`` Algorithm 1 (Eqs. 6-13); ``hscale_pack_nvfp4`` the final
+re-quantization (Sec. 3.3).
+"""
+from __future__ import annotations
+
+import ctypes
+import pathlib
+import threading
+
+import torch
+
+__all__ = [
+    "HScaleError", "load", "library_path", "hscale_status_string", "hscale_abi_version",
+    "hscale_hessian_diag_accumulate", "hscale_rtn_workspace_bytes", "hscale_rtn_scales",
+    "hscale_refine_scales", "hscale_pack_nvfp4", "EXPORTED_SYMBOLS",
+]
+
+_PKG = pathlib.Path(__file__).resolve().parent
+_LIB_PATH = _PKG / "_build" / "libhscale.so"
+_lock = threading.Lock()
+_lib = None
+
+# every entry point of include/hscale.h, with its ctypes signature
+_P, _I64, _I32, _SZ = ctypes.c_void_p, ctypes.c_int64, ctypes.c_int32, ctypes.c_size_t
+_SIGNATURES = {
+    "hscale_status_string": (ctypes.c_char_p, [ctypes.c_int]),
+    "hscale_abi_version": (ctypes.c_int, []),
+    "hscale_hessian_diag_accumulate": (ctypes.c_int, [_P, _I64, _I64, _I64, _P, _P]),
+    "hscale_rtn_workspace_bytes": (_SZ, []),
+    "hscale_rtn_scales": (ctypes.c_int, [_P, _I64, _I64, _P, _P, _P, _SZ, _P]),
+    "hscale_refine_scales": (ctypes.c_int, [_P, _P, _I64, _I64, _P, _P, _I32, _I32, _P, _P, _P]),
+    "hscale_pack_nvfp4": (ctypes.c_int, [_P, _I64, _I64, _P, _P, _P, _P]),
+}
+EXPORTED_SYMBOLS = tuple(_SIGNATURES)
+
+
+class HScaleError(RuntimeError):
+    def __init__(self, fn: str, status: int):
+        super().__init__(f"{fn} failed with status {status}: {hscale_status_string(status)}")
+        self.status = status
+
+
+def library_path() -> pathlib.Path:
+    return _LIB_PATH
+
+
+def load(build_if_missing: bool = False) -> ctypes.CDLL:
+    """The loaded CUDA library.  Raises if it has not been built."""
+    global _lib
+    with _lock:
+        if _lib is not None:
+            return _lib
+        if not _LIB_PATH.exists():
+            if not build_if_missing:
+                raise ImportError(f"{_LIB_PATH} is missing: build it with "
+                                  "`python -c 'import __graft_entry__ as g; g.build()'`")
+            from . import build as _build
+            _build.build()
+        lib = ctypes.CDLL(str(_LIB_PATH))
+        for name, (res, args) in _SIGNATURES.items():
+            fn = getattr(lib, name)
+            fn.restype = res
+            fn.argtypes = args
+        _lib = lib
+        return lib
+
+
+def hscale_status_string(status: int) -> str:
+    return load().hscale_status_string(int(status)).decode()
+
+
+def hscale_abi_version() -> int:
+    return int(load().hscale_abi_version())
+
+
+def _stream_ptr(stream) -> int:
+    if stream is None:
+        stream = torch.cuda.current_stream()
+    return int(stream.cuda_stream) if hasattr(stream, "cuda_stream") else int(stream)
+
+
+def _check(fn: str, status: int) -> None:
+    if status != 0:
+        raise HScaleError(fn, status)
+
+
+def _ptr(t: torch.Tensor | None):
+    return None if t is None else t.data_ptr()
+
+
+def _need(t: torch.Tensor, dtype, name: str):
+    if not isinstance(t, torch.Tensor) or t.dtype != dtype or not t.is_cuda:
+        raise TypeError(f"{name} must be a CUDA tensor of dtype {dtype}")
+
+
+def hscale_hessian_diag_accumulate(x: torch.Tensor, h: torch.Tensor, stream=None) -> torch.Tensor:
+    """h[j] += sum_t x[t, j]^2 for a bf16 chunk x [tokens, n] (row stride >= n)."""
+    _need(x, torch.bfloat16, "x")
+    _need(h, torch.float32, "h")
+    if x.dim() != 2 or x.stride(1) != 1:
+        raise ValueError("x must be 2-D with unit column stride")
+    tokens, n = x.shape
+    if h.numel() != n or not h.is_contiguous():
+        raise ValueError("h must be a contiguous float32 vector of length n")
+    ld = x.stride(0) if tokens > 1 else n
+    _check("hscale_hessian_diag_accumulate",
+           load().hscale_hessian_diag_accumulate(_ptr(x), tokens, n, ld, _ptr(h), _stream_ptr(stream)))
+    return h
+
+
+def hscale_rtn_workspace_bytes() -> int:
+    return int(load().hscale_rtn_workspace_bytes())
+
+
+def hscale_rtn_scales(w: torch.Tensor, global_scale: torch.Tensor, codes: torch.Tensor | None,
+                      workspace: torch.Tensor, stream=None) -> None:
+    """s_g = amax|W| / 2688 into global_scale[0]; RTN codes [m, n/16] into codes."""
+    _need(w, torch.bfloat16, "w")
+    _need(global_scale, torch.float32, "global_scale")
+    if not w.is_contiguous() or w.dim() != 2:
+        raise ValueError("w must be a contiguous 2-D tensor")
+    m, n = w.shape
+    if codes is not None:
+        _need(codes, torch.uint8, "codes")
+        if codes.numel() != m * (n // 16) or not codes.is_contiguous():
+            raise ValueError("codes must be contiguous [m, n/16]")
+    if not workspace.is_cuda:
+        raise TypeError("workspace must live on the GPU")
+    nbytes = workspace.numel() * workspace.element_size()
+    _check("hscale_rtn_scales",
+           load().hscale_rtn_scales(_ptr(w), m, n, _ptr(global_scale), _ptr(codes),
+                                    _ptr(workspace), nbytes, _stream_ptr(stream)))
+
+
+def hscale_refine_scales(w: torch.Tensor, h: torch.Tensor | None, global_scale: torch.Tensor,
+                         init_codes: torch.Tensor | None, down: int, up: int,
+                         codes_out: torch.Tensor, packed_out: torch.Tensor | None,
+                         stream=None) -> None:
+    """Algorithm 1 over every group of W, with the final re-quantization and packing."""
+    _need(w, torch.bfloat16, "w")
+    _need(global_scale, torch.float32, "global_scale")
+    _need(codes_out, torch.uint8, "codes_out")
+    if not w.is_contiguous() or w.dim() != 2:
+        raise ValueError("w must be a contiguous 2-D tensor")
+    m, n = w.shape
+    if h is not None:
+        _need(h, torch.float32, "h")
+        if h.numel() != n or not h.is_contiguous():
+            raise ValueError("h must be a contiguous float32 vector of length n")
+    for name, t, size in (("init_codes", init_codes, m * (n // 16)),
+                          ("codes_out", codes_out, m * (n // 16)),
+                          ("packed_out", packed_out, m * (n // 2))):
+        if t is not None:
+            _need(t, torch.uint8, name)
+            if t.numel() != size or not t.is_contiguous():
+                raise ValueError(f"{name} must be contiguous with {size} bytes")
+    _check("hscale_refine_scales",
+           load().hscale_refine_scales(_ptr(w), _ptr(h), m, n, _ptr(global_scale), _ptr(init_codes),
+                                       int(down), int(up), _ptr(codes_out), _ptr(packed_out),
+                                       _stream_ptr(stream)))
+
+
+def hscale_pack_nvfp4(w: torch.Tensor, global_scale: torch.Tensor, codes: torch.Tensor,
+                      packed_out: torch.Tensor, stream=None) -> None:
+    """FP4 nibbles of W under the given codes."""
+    _need(w, torch.bfloat16, "w")
+    _need(global_scale, torch.float32, "global_scale")
+    _need(codes, torch.uint8, "codes")
+    _need(packed_out, torch.uint8, "packed_out")
+    if not w.is_contiguous() or w.dim() != 2:
+        raise ValueError("w must be a contiguous 2-D tensor")
+    m, n = w.shape
+    if codes.numel() != m * (n // 16) or packed_out.numel() != m * (n // 2):
+        raise ValueError("codes must be [m, n/16] and packed_out [m, n/2]")
+    _check("hscale_pack_nvfp4",
+           load().hscale_pack_nvfp4(_ptr(w), m, n, _ptr(global_scale), _ptr(codes),
+                                    _ptr(packed_out), _stream_ptr(stream)))

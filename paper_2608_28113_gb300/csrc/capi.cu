@@ -1,0 +1,134 @@
+// capi.cu -- the extern "C" boundary declared in include/hscale.h.
+//
+// Every entry point validates its arguments on the host before enqueueing anything,
+// then calls the launchers in hessian.cu / scales.cu.  No exception crosses the ABI.
+#include <cuda_runtime.h>
+
+#include <cstdint>
+#include <mutex>
+
+#include "../../include/hscale.h"
+#include "hscale_internal.h"
+
+namespace hscale {
+
+cudaError_t current_device_info(DeviceInfo* out) {
+  static std::mutex mu;
+  static int sms[64] = {0};
+  int dev = 0;
+  cudaError_t err = cudaGetDevice(&dev);
+  if (err != cudaSuccess) return err;
+  if (dev < 0 || dev >= 64) return cudaErrorInvalidDevice;
+  std::lock_guard<std::mutex> lock(mu);
+  if (sms[dev] == 0) {
+    int v = 0;
+    err = cudaDeviceGetAttribute(&v, cudaDevAttrMultiProcessorCount, dev);
+    if (err != cudaSuccess) return err;
+    sms[dev] = v;
+  }
+  out->device = dev;
+  out->sm_count = sms[dev];
+  return cudaSuccess;
+}
+
+}  // namespace hscale
+
+namespace {
+
+inline bool aligned(const void* p, uintptr_t a) { return (reinterpret_cast<uintptr_t>(p) & (a - 1)) == 0; }
+
+inline int from_cuda(cudaError_t e) { return e == cudaSuccess ? HSCALE_OK : HSCALE_ERR_CUDA; }
+
+inline cudaStream_t as_stream(void* s) { return static_cast<cudaStream_t>(s); }
+
+// common checks of a weight matrix argument
+inline int check_weight(const void* w, int64_t m, int64_t n) {
+  if (m < 0 || n < 0) return HSCALE_ERR_SHAPE;
+  if (n % 16 != 0) return HSCALE_ERR_SHAPE;
+  if (m > 0 && n > 0 && (m > INT64_MAX / n || n / 16 > INT32_MAX)) return HSCALE_ERR_SHAPE;
+  if (m == 0 || n == 0) return HSCALE_OK;
+  if (w == nullptr) return HSCALE_ERR_NULL;
+  if (!aligned(w, 16)) return HSCALE_ERR_ALIGN;
+  return HSCALE_OK;
+}
+
+}  // namespace
+
+extern "C" {
+
+const char* hscale_status_string(int status) {
+  switch (status) {
+    case HSCALE_OK: return "ok";
+    case HSCALE_ERR_NULL: return "a required pointer is NULL";
+    case HSCALE_ERR_SHAPE: return "invalid shape (negative size, n not a multiple of 16/8, ld < n, or too large)";
+    case HSCALE_ERR_ALIGN: return "misaligned pointer or leading dimension";
+    case HSCALE_ERR_ARG: return "scalar argument out of range";
+    case HSCALE_ERR_CUDA: return "CUDA runtime error";
+    case HSCALE_ERR_WORKSPACE: return "workspace missing or too small";
+    default: return "unknown status";
+  }
+}
+
+int hscale_abi_version(void) { return 1; }
+
+int hscale_hessian_diag_accumulate(const void* x_bf16, int64_t tokens, int64_t n, int64_t ld_x,
+                                   float* h, void* stream) {
+  if (tokens < 0 || n < 0 || ld_x < n) return HSCALE_ERR_SHAPE;
+  if (n % 8 != 0) return HSCALE_ERR_SHAPE;
+  if (n > (int64_t)65535 * 64) return HSCALE_ERR_SHAPE;  // 64-channel tiles on grid.y
+  if (tokens == 0 || n == 0) return HSCALE_OK;
+  if (x_bf16 == nullptr || h == nullptr) return HSCALE_ERR_NULL;
+  if (ld_x % 8 != 0) return HSCALE_ERR_ALIGN;
+  if (!aligned(x_bf16, 16) || !aligned(h, 4)) return HSCALE_ERR_ALIGN;
+  if (tokens > INT64_MAX / ld_x) return HSCALE_ERR_SHAPE;
+  return from_cuda(hscale::launch_hessian(x_bf16, tokens, n, ld_x, h, as_stream(stream)));
+}
+
+size_t hscale_rtn_workspace_bytes(void) { return 256; }
+
+int hscale_rtn_scales(const void* w_bf16, int64_t m, int64_t n, float* global_scale,
+                      uint8_t* codes, void* workspace, size_t workspace_bytes, void* stream) {
+  int st = check_weight(w_bf16, m, n);
+  if (st != HSCALE_OK) return st;
+  if (m == 0 || n == 0) return HSCALE_OK;
+  if (global_scale == nullptr) return HSCALE_ERR_NULL;
+  if (!aligned(global_scale, 4)) return HSCALE_ERR_ALIGN;
+  if (workspace == nullptr || workspace_bytes < hscale_rtn_workspace_bytes()) return HSCALE_ERR_WORKSPACE;
+  if (!aligned(workspace, 4)) return HSCALE_ERR_ALIGN;
+  cudaStream_t s = as_stream(stream);
+  uint32_t* amax = static_cast<uint32_t*>(workspace);
+  cudaError_t err = cudaMemsetAsync(amax, 0, sizeof(uint32_t), s);
+  if (err != cudaSuccess) return HSCALE_ERR_CUDA;
+  err = hscale::launch_amax(w_bf16, m * n, amax, s);
+  if (err != cudaSuccess) return HSCALE_ERR_CUDA;
+  return from_cuda(hscale::launch_rtn_codes(w_bf16, m, n, amax, global_scale, codes, s));
+}
+
+int hscale_refine_scales(const void* w_bf16, const float* h, int64_t m, int64_t n,
+                         const float* global_scale, const uint8_t* init_codes, int32_t down,
+                         int32_t up, uint8_t* codes_out, uint8_t* packed_out, void* stream) {
+  int st = check_weight(w_bf16, m, n);
+  if (st != HSCALE_OK) return st;
+  if (down < 0 || up < 0 || down > 125 || up > 125) return HSCALE_ERR_ARG;
+  if (m == 0 || n == 0) return HSCALE_OK;
+  if (global_scale == nullptr || codes_out == nullptr) return HSCALE_ERR_NULL;
+  if (!aligned(global_scale, 4)) return HSCALE_ERR_ALIGN;
+  if (h != nullptr && !aligned(h, 16)) return HSCALE_ERR_ALIGN;
+  if (packed_out != nullptr && !aligned(packed_out, 8)) return HSCALE_ERR_ALIGN;
+  return from_cuda(hscale::launch_refine(w_bf16, h, m, n, global_scale, init_codes, down, up,
+                                         codes_out, packed_out, as_stream(stream)));
+}
+
+int hscale_pack_nvfp4(const void* w_bf16, int64_t m, int64_t n, const float* global_scale,
+                      const uint8_t* codes, uint8_t* packed_out, void* stream) {
+  int st = check_weight(w_bf16, m, n);
+  if (st != HSCALE_OK) return st;
+  if (m == 0 || n == 0) return HSCALE_OK;
+  if (global_scale == nullptr || codes == nullptr || packed_out == nullptr) return HSCALE_ERR_NULL;
+  if (!aligned(global_scale, 4)) return HSCALE_ERR_ALIGN;
+  if (!aligned(packed_out, 8)) return HSCALE_ERR_ALIGN;
+  return from_cuda(hscale::launch_pack(w_bf16, m, n, global_scale, codes, packed_out,
+                                       as_stream(stream)));
+}
+
+}  // extern "C"

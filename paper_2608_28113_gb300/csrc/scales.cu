@@ -1,0 +1,381 @@
+// scales.cu -- global scale, RTN codes, H-Scale search and NVFP4 packing on sm_103a.
+//
+//   amax_kernel         amax|W| (integer max of |bf16| bit patterns; order-free)
+//   rtn_codes_kernel    s_g = amax / 2688 and the RTN code of every group (Eq. 7)
+//   refine_kernel       Algorithm 1: per group, every distinct E4M3 code in the window
+//                       (Eqs. 8-11) is scored by sum_j h_j (|w_j| - s q_j)^2 (Eqs. 6, 12,
+//                       13); the best code is re-quantized exactly and packed
+//   pack_kernel         exact FP4 quantization with given codes (Eq. 2)
+//
+// The search (one group per thread, no shuffles in the hot loop)
+//   Per element and candidate the fast score costs one multiply for the quotient, an
+//   integer add + and + min for the E2M1 rounding (see hscale_device.cuh), one FMA for
+//   the residual, and a multiply + FMA for h * r^2.  The fast scores differ from the
+//   exact-decision scores only through roundings near E2M1 midpoints and fp32 error,
+//   which together stay below
+//        B(E) = 2^-13 E + 32 * 2^-24 * s_max * sqrt(H E)     (H = sum of the group's h)
+//   so when runner-up - best > B(runner-up) the fast winner is the exact winner.
+//   Otherwise the group is "ambiguous" and the whole warp rescores it cooperatively with
+//   exact rounding decisions (16 lanes per candidate, one element each, a fixed
+//   pairwise shuffle tree per error: relative error <= 8 * 2^-24), applying the tie
+//   rule (smaller error, then smaller |shift|, then smaller shift).  The winner's
+//   nibbles are always produced with exact round-to-nearest-even decisions.
+#include <algorithm>
+
+#include "hscale_device.cuh"
+#include "hscale_internal.h"
+
+namespace hscale {
+namespace {
+
+constexpr int kRefineThreads = 128;
+constexpr int kWarpsPerRefineBlock = kRefineThreads / 32;
+constexpr float kInf = __builtin_huge_valf();
+
+// ---------------------------------------------------------------- amax
+__global__ void __launch_bounds__(256) amax_kernel(const uint4* __restrict__ w, int64_t nvec,
+                                                   uint32_t* __restrict__ amax_bits) {
+  __shared__ uint32_t warp_max[8];
+  uint32_t m2 = 0;  // two packed 16-bit maxima
+  const int64_t stride = (int64_t)gridDim.x * blockDim.x;
+  for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < nvec; i += stride) {
+    const uint4 v = ld_stream_v4(w + i);
+    m2 = __vmaxu2(m2, v.x & 0x7FFF7FFFu);
+    m2 = __vmaxu2(m2, v.y & 0x7FFF7FFFu);
+    m2 = __vmaxu2(m2, v.z & 0x7FFF7FFFu);
+    m2 = __vmaxu2(m2, v.w & 0x7FFF7FFFu);
+  }
+  uint32_t m = max(m2 & 0xFFFFu, m2 >> 16);
+  m = __reduce_max_sync(0xFFFFFFFFu, m);
+  if ((threadIdx.x & 31) == 0) warp_max[threadIdx.x >> 5] = m;
+  __syncthreads();
+  if (threadIdx.x < 32) {
+    m = threadIdx.x < (blockDim.x >> 5) ? warp_max[threadIdx.x] : 0u;
+    m = __reduce_max_sync(0xFFFFFFFFu, m);
+    if (threadIdx.x == 0 && m) atomicMax(amax_bits, m);
+  }
+}
+
+__device__ __forceinline__ float global_scale_of(uint32_t amax_bits) {
+  const float amax = __uint_as_float(amax_bits << 16);
+  return amax == 0.0f ? 1.0f : __fdiv_rn(amax, 2688.0f);  // 6 * 448
+}
+
+__device__ __forceinline__ uint32_t group_abs_max_bits(const uint4& a, const uint4& b) {
+  uint32_t m = __vmaxu2(a.x & 0x7FFF7FFFu, a.y & 0x7FFF7FFFu);
+  m = __vmaxu2(m, a.z & 0x7FFF7FFFu);
+  m = __vmaxu2(m, a.w & 0x7FFF7FFFu);
+  m = __vmaxu2(m, b.x & 0x7FFF7FFFu);
+  m = __vmaxu2(m, b.y & 0x7FFF7FFFu);
+  m = __vmaxu2(m, b.z & 0x7FFF7FFFu);
+  m = __vmaxu2(m, b.w & 0x7FFF7FFFu);
+  return max(m & 0xFFFFu, m >> 16);
+}
+
+// ---------------------------------------------------------------- RTN codes
+__global__ void __launch_bounds__(256) rtn_codes_kernel(const uint4* __restrict__ w, int64_t groups,
+                                                        const uint32_t* __restrict__ amax_bits,
+                                                        float* __restrict__ global_scale,
+                                                        uint8_t* __restrict__ codes) {
+  const float sg = global_scale_of(*amax_bits);
+  if (blockIdx.x == 0 && threadIdx.x == 0) *global_scale = sg;
+  if (codes == nullptr) return;
+  const ScaleDomain d = make_scale_domain(sg);
+  const float inv6 = rtn_inv6_raw(d.sgk);
+  const int64_t stride = (int64_t)gridDim.x * blockDim.x;
+  for (int64_t g = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; g < groups; g += stride) {
+    const uint4 a = ld_stream_v4(w + 2 * g);
+    const uint4 b = ld_stream_v4(w + 2 * g + 1);
+    const float amax_k = __fmul_rn(__uint_as_float(group_abs_max_bits(a, b) << 16), d.pw);
+    codes[g] = (uint8_t)rtn_code(amax_k, d.sgk, inv6);
+  }
+}
+
+// ---------------------------------------------------------------- search helpers
+struct Group {
+  uint32_t wb[8];  // raw bf16 pairs (element 2i in the low half of wb[i])
+  float a[16];     // |w| * 2^-K
+};
+
+__device__ __forceinline__ void load_group(const uint4* w, int64_t g, float pw, Group& G) {
+  const uint4 p = ld_stream_v4(w + 2 * g);
+  const uint4 q = ld_stream_v4(w + 2 * g + 1);
+  G.wb[0] = p.x; G.wb[1] = p.y; G.wb[2] = p.z; G.wb[3] = p.w;
+  G.wb[4] = q.x; G.wb[5] = q.y; G.wb[6] = q.z; G.wb[7] = q.w;
+#pragma unroll
+  for (int i = 0; i < 8; ++i) {
+    G.a[2 * i] = __fmul_rn(fabsf(bf16_lo(G.wb[i])), pw);
+    G.a[2 * i + 1] = __fmul_rn(fabsf(bf16_hi(G.wb[i])), pw);
+  }
+}
+
+// tie rule of the search: smaller error, then smaller |shift|, then smaller shift
+__device__ __forceinline__ bool better(float e, int c, float be, int bc, int c0) {
+  if (e != be) return e < be;
+  const int s = c - c0, bs = bc - c0;
+  const int as = s < 0 ? -s : s, abs_ = bs < 0 ? -bs : bs;
+  return as < abs_ || (as == abs_ && s < bs);
+}
+
+// Exact-decision score of one element under code c (scaled domain, one rounding in the
+// residual: q * l is exact and the FMA rounds once).
+__device__ __forceinline__ float exact_term(float a_k, float hj, uint32_t c, float sgk) {
+  const float l = e4m3_mag(c);
+  const float inv = inv_raw_of(__fmul_rn(l, sgk));
+  const uint32_t k = e2m1_code(a_k, inv, l, sgk);
+  const float ql = __fmul_rn(e2m1_from_raw(k << 22), l);
+  const float r = __fmaf_rn(-ql, sgk, a_k);
+  return __fmul_rn(hj, __fmul_rn(r, r));
+}
+
+// The whole warp rescores the group of lane `owner` with exact rounding decisions and
+// returns its winning code (in every lane).  Lanes 0-15 take the candidates lo, lo+2,
+// ..., lanes 16-31 lo+1, lo+3, ...; lane j of each half scores element j & 15.
+__device__ int warp_exact_search(int owner, const uint4* w, int64_t g_own, const float* h,
+                                 int64_t hcol_own, int c0, int lo, int hi, float sgk, float pw) {
+  const int lane = threadIdx.x & 31;
+  const int j = lane & 15, half = lane >> 4;
+  const uint16_t wb = reinterpret_cast<const uint16_t*>(w)[g_own * 16 + j];
+  const float a_k = __fmul_rn(fabsf(__uint_as_float((uint32_t)wb << 16)), pw);
+  const float hj = h ? h[hcol_own * 16 + j] : 1.0f;
+  const unsigned mask = 0xFFFFu << (16 * half);
+  float be = kInf;
+  int bc = -1;
+  for (int c = lo + half; c <= hi; c += 2) {
+    float e = exact_term(a_k, hj, (uint32_t)c, sgk);
+    e = __fadd_rn(e, __shfl_xor_sync(mask, e, 1));
+    e = __fadd_rn(e, __shfl_xor_sync(mask, e, 2));
+    e = __fadd_rn(e, __shfl_xor_sync(mask, e, 4));
+    e = __fadd_rn(e, __shfl_xor_sync(mask, e, 8));
+    if (bc < 0 || better(e, c, be, bc, c0)) { be = e; bc = c; }
+  }
+  __syncwarp();
+  const float oe = __shfl_xor_sync(0xFFFFFFFFu, be, 16);
+  const int oc = __shfl_xor_sync(0xFFFFFFFFu, bc, 16);
+  if (oc >= 0 && (bc < 0 || better(oe, oc, be, bc, c0))) { be = oe; bc = oc; }
+  (void)owner;
+  return bc;
+}
+
+// Exact final re-quantization of one group under code c: 8 bytes of packed nibbles.
+__device__ __forceinline__ uint2 quantize_pack(const Group& G, uint32_t c, float sgk) {
+  const float l = e4m3_mag(c);
+  const float inv = inv_raw_of(__fmul_rn(l, sgk));
+  uint32_t out[2] = {0u, 0u};
+#pragma unroll
+  for (int j = 0; j < 16; ++j) {
+    const uint32_t k = e2m1_code(G.a[j], inv, l, sgk);
+    const uint32_t sign = (j & 1) ? (G.wb[j >> 1] >> 31) : ((G.wb[j >> 1] >> 15) & 1u);
+    out[j >> 3] |= ((sign << 3) | k) << (4 * (j & 7));
+  }
+  return make_uint2(out[0], out[1]);
+}
+
+// ---------------------------------------------------------------- refine (Algorithm 1)
+// Work unit: one warp, 32 consecutive groups of one row (a "row chunk"); warps stride
+// over (row, chunk) units so the h slice of a lane is reloaded only when its chunk
+// changes.
+__global__ void __launch_bounds__(kRefineThreads)
+refine_kernel(const uint4* __restrict__ w, const float* __restrict__ h, int64_t m, int ng,
+              const float* __restrict__ global_scale, const uint8_t* init_codes,
+              int down, int up, uint8_t* codes_out, uint2* __restrict__ packed_out) {
+  const int lane = threadIdx.x & 31;
+  const int64_t warp_global = ((int64_t)blockIdx.x * blockDim.x + threadIdx.x) >> 5;
+  const int64_t warps_total = ((int64_t)gridDim.x * blockDim.x) >> 5;
+  const int chunks = (ng + 31) / 32;
+  const int64_t units = m * chunks;
+
+  const ScaleDomain d = make_scale_domain(*global_scale);
+  const float inv6 = rtn_inv6_raw(d.sgk);
+
+  int cur_chunk = -1;
+  float hv[16];
+  float H = 0.0f;
+#pragma unroll
+  for (int j = 0; j < 16; ++j) hv[j] = 1.0f;
+
+  for (int64_t u = warp_global; u < units; u += warps_total) {
+    const int64_t row = u / chunks;
+    const int chunk = (int)(u - row * chunks);
+    const int gcol = chunk * 32 + lane;
+    const bool active = gcol < ng;
+    const int64_t g = row * ng + gcol;
+
+    if (chunk != cur_chunk) {
+      cur_chunk = chunk;
+      H = 0.0f;
+      if (h != nullptr && active) {
+        const float4* hp = reinterpret_cast<const float4*>(h + (int64_t)gcol * 16);
+#pragma unroll
+        for (int i = 0; i < 4; ++i) {
+          const float4 t = hp[i];
+          hv[4 * i] = t.x; hv[4 * i + 1] = t.y; hv[4 * i + 2] = t.z; hv[4 * i + 3] = t.w;
+        }
+      }
+#pragma unroll
+      for (int j = 0; j < 16; ++j) H = __fadd_rn(H, hv[j]);
+    }
+
+    Group G;
+    int c0 = 1, lo = 1, hi = 1;
+    if (active) {
+      load_group(w, g, d.pw, G);
+      if (init_codes != nullptr) {
+        c0 = init_codes[g] & 0x7F;
+        c0 = c0 < 1 ? 1 : (c0 > (int)kE4M3MaxCode ? (int)kE4M3MaxCode : c0);
+      } else {
+        const uint32_t amax = group_abs_max_bits(make_uint4(G.wb[0], G.wb[1], G.wb[2], G.wb[3]),
+                                                 make_uint4(G.wb[4], G.wb[5], G.wb[6], G.wb[7]));
+        c0 = (int)rtn_code(__fmul_rn(__uint_as_float(amax << 16), d.pw), d.sgk, inv6);
+      }
+      lo = max(1, c0 - down);
+      hi = min((int)kE4M3MaxCode, c0 + up);
+    }
+
+    // ---- fast scores of every distinct candidate
+    float e1 = kInf, e2 = kInf;
+    int best = c0;
+    if (active) {
+      for (int c = lo; c <= hi; ++c) {
+        const float l = e4m3_mag((uint32_t)c);
+        const float sp = __fmul_rn(l, d.sgk);
+        const float S = __fmul_rn(sp, 0x1p126f);
+        const float inv = inv_raw_of(sp);
+        float acc0 = 0.f, acc1 = 0.f, acc2 = 0.f, acc3 = 0.f;
+#pragma unroll
+        for (int j = 0; j < 16; j += 4) {
+          float y, r;
+          uint32_t q;
+          y = __fmul_rn(G.a[j], inv);
+          q = min((__float_as_uint(y) + kE2M1Half) & kE2M1Keep, kE2M1SixRaw);
+          r = __fmaf_rn(-__uint_as_float(q), S, G.a[j]);
+          acc0 = __fmaf_rn(hv[j], __fmul_rn(r, r), acc0);
+          y = __fmul_rn(G.a[j + 1], inv);
+          q = min((__float_as_uint(y) + kE2M1Half) & kE2M1Keep, kE2M1SixRaw);
+          r = __fmaf_rn(-__uint_as_float(q), S, G.a[j + 1]);
+          acc1 = __fmaf_rn(hv[j + 1], __fmul_rn(r, r), acc1);
+          y = __fmul_rn(G.a[j + 2], inv);
+          q = min((__float_as_uint(y) + kE2M1Half) & kE2M1Keep, kE2M1SixRaw);
+          r = __fmaf_rn(-__uint_as_float(q), S, G.a[j + 2]);
+          acc2 = __fmaf_rn(hv[j + 2], __fmul_rn(r, r), acc2);
+          y = __fmul_rn(G.a[j + 3], inv);
+          q = min((__float_as_uint(y) + kE2M1Half) & kE2M1Keep, kE2M1SixRaw);
+          r = __fmaf_rn(-__uint_as_float(q), S, G.a[j + 3]);
+          acc3 = __fmaf_rn(hv[j + 3], __fmul_rn(r, r), acc3);
+        }
+        const float e = __fadd_rn(__fadd_rn(acc0, acc1), __fadd_rn(acc2, acc3));
+        if (e < e1) { e2 = e1; e1 = e; best = c; }
+        else if (e < e2) { e2 = e; }
+      }
+    }
+
+    // ---- is the fast winner certain?
+    bool ambiguous = false;
+    if (active && hi > lo) {
+      const float smax = __fmul_rn(e4m3_mag((uint32_t)hi), d.sgk);
+      const float bound = __fmaf_rn(0x1p-13f, e2,
+                                    __fmul_rn(32.0f * 0x1p-24f, __fmul_rn(smax, sqrtf(__fmul_rn(H, e2)))));
+      ambiguous = !(__fsub_rn(e2, e1) > bound) || !(e2 >= 0x1p-100f);
+    }
+    unsigned amb = __ballot_sync(0xFFFFFFFFu, ambiguous);
+    while (amb) {
+      const int owner = __ffs(amb) - 1;
+      amb &= amb - 1;
+      const int64_t g_own = __shfl_sync(0xFFFFFFFFu, g, owner);
+      const int gcol_own = __shfl_sync(0xFFFFFFFFu, gcol, owner);
+      const int c0o = __shfl_sync(0xFFFFFFFFu, c0, owner);
+      const int loo = __shfl_sync(0xFFFFFFFFu, lo, owner);
+      const int hio = __shfl_sync(0xFFFFFFFFu, hi, owner);
+      const int bc = warp_exact_search(owner, w, g_own, h, gcol_own, c0o, loo, hio, d.sgk, d.pw);
+      if (lane == owner) best = bc;
+    }
+
+    if (active) {
+      codes_out[g] = (uint8_t)best;
+      if (packed_out != nullptr) packed_out[g] = quantize_pack(G, (uint32_t)best, d.sgk);
+    }
+  }
+}
+
+// ---------------------------------------------------------------- pack with given codes
+__global__ void __launch_bounds__(256) pack_kernel(const uint4* __restrict__ w, int64_t groups,
+                                                   const float* __restrict__ global_scale,
+                                                   const uint8_t* __restrict__ codes,
+                                                   uint2* __restrict__ packed_out) {
+  const ScaleDomain d = make_scale_domain(*global_scale);
+  const int64_t stride = (int64_t)gridDim.x * blockDim.x;
+  for (int64_t g = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; g < groups; g += stride) {
+    Group G;
+    load_group(w, g, d.pw, G);
+    uint32_t c = codes[g] & 0x7Fu;
+    c = c < 1 ? 1u : (c > kE4M3MaxCode ? kE4M3MaxCode : c);
+    packed_out[g] = quantize_pack(G, c, d.sgk);
+  }
+}
+
+template <typename K>
+int occupancy_blocks(K kernel, int threads) {
+  int blocks = 0;
+  if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&blocks, kernel, threads, 0) != cudaSuccess ||
+      blocks < 1)
+    blocks = 1;
+  return blocks;
+}
+
+}  // namespace
+
+cudaError_t launch_amax(const void* w, int64_t count, uint32_t* amax_bits, cudaStream_t stream) {
+  DeviceInfo info;
+  cudaError_t err = current_device_info(&info);
+  if (err != cudaSuccess) return err;
+  const int64_t nvec = count / 8;
+  int64_t blocks = (nvec + 255) / 256;
+  blocks = std::min<int64_t>(blocks, (int64_t)info.sm_count * occupancy_blocks(amax_kernel, 256));
+  amax_kernel<<<(unsigned)blocks, 256, 0, stream>>>(static_cast<const uint4*>(w), nvec, amax_bits);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_rtn_codes(const void* w, int64_t m, int64_t n, const uint32_t* amax_bits,
+                             float* global_scale, uint8_t* codes, cudaStream_t stream) {
+  DeviceInfo info;
+  cudaError_t err = current_device_info(&info);
+  if (err != cudaSuccess) return err;
+  const int64_t groups = m * (n / 16);
+  int64_t blocks = codes ? (groups + 255) / 256 : 1;
+  blocks = std::max<int64_t>(1, std::min<int64_t>(blocks, (int64_t)info.sm_count * occupancy_blocks(rtn_codes_kernel, 256)));
+  rtn_codes_kernel<<<(unsigned)blocks, 256, 0, stream>>>(static_cast<const uint4*>(w), groups,
+                                                          amax_bits, global_scale, codes);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_refine(const void* w, const float* h, int64_t m, int64_t n,
+                          const float* global_scale, const uint8_t* init_codes, int down, int up,
+                          uint8_t* codes_out, uint8_t* packed_out, cudaStream_t stream) {
+  DeviceInfo info;
+  cudaError_t err = current_device_info(&info);
+  if (err != cudaSuccess) return err;
+  const int ng = (int)(n / 16);
+  const int64_t units = m * ((ng + 31) / 32);
+  const int64_t resident = (int64_t)info.sm_count * occupancy_blocks(refine_kernel, kRefineThreads);
+  const int64_t blocks = std::max<int64_t>(1, std::min<int64_t>((units + kWarpsPerRefineBlock - 1) / kWarpsPerRefineBlock, resident));
+  refine_kernel<<<(unsigned)blocks, kRefineThreads, 0, stream>>>(
+      static_cast<const uint4*>(w), h, m, ng, global_scale, init_codes, down, up, codes_out,
+      reinterpret_cast<uint2*>(packed_out));
+  return cudaGetLastError();
+}
+
+cudaError_t launch_pack(const void* w, int64_t m, int64_t n, const float* global_scale,
+                        const uint8_t* codes, uint8_t* packed_out, cudaStream_t stream) {
+  DeviceInfo info;
+  cudaError_t err = current_device_info(&info);
+  if (err != cudaSuccess) return err;
+  const int64_t groups = m * (n / 16);
+  int64_t blocks = (groups + 255) / 256;
+  blocks = std::max<int64_t>(1, std::min<int64_t>(blocks, (int64_t)info.sm_count * occupancy_blocks(pack_kernel, 256)));
+  pack_kernel<<<(unsigned)blocks, 256, 0, stream>>>(static_cast<const uint4*>(w), groups,
+                                                     global_scale, codes,
+                                                     reinterpret_cast<uint2*>(packed_out));
+  return cudaGetLastError();
+}
+
+}  // namespace hscale

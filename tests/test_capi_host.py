@@ -1,0 +1,116 @@
+"""Host-side checks of the C ABI (CPU only: no kernel is launched).
+
+The library must build for sm_103a, load, export every entry point that
+include/hscale.h declares, and reject bad arguments with a status code before it
+enqueues anything.
+"""
+import ctypes
+import pathlib
+import re
+
+import pytest
+
+import paper_2608_28113_gb300 as hs
+from paper_2608_28113_gb300 import build
+
+HEADER = pathlib.Path(__file__).resolve().parent.parent / "include" / "hscale.h"
+
+OK, ERR_NULL, ERR_SHAPE, ERR_ALIGN, ERR_ARG, ERR_CUDA, ERR_WS = range(7)
+
+
+@pytest.fixture(scope="module")
+def lib():
+    build.build()
+    return hs.load()
+
+
+def declared_functions():
+    text = HEADER.read_text()
+    text = re.sub(r"/\*.*?\*/", "", text, flags=re.S)
+    return sorted(set(re.findall(r"^\s*(?:const\s+)?\w+\*?\s+\*?(hscale_\w+)\s*\(", text, flags=re.M)))
+
+
+def test_header_declares_the_boundary():
+    names = declared_functions()
+    for required in ("hscale_hessian_diag_accumulate", "hscale_rtn_scales",
+                     "hscale_refine_scales", "hscale_pack_nvfp4"):
+        assert required in names
+    assert set(names) == set(hs.EXPORTED_SYMBOLS)
+
+
+def test_library_exports_every_declared_symbol(lib):
+    for name in declared_functions():
+        assert hasattr(lib, name), name
+    assert hs.hscale_abi_version() == 1
+    assert hs.library_path().exists()
+
+
+def test_status_strings(lib):
+    for s in range(7):
+        assert hs.hscale_status_string(s)
+    assert hs.hscale_status_string(99) == "unknown status"
+
+
+FAKE = ctypes.c_void_p(0x10000)  # 64 KiB-aligned; never dereferenced: checks fail or no-op first
+MIS = ctypes.c_void_p(0x10002)
+
+
+def test_hessian_argument_errors(lib):
+    f = lib.hscale_hessian_diag_accumulate
+    assert f(None, 4, 64, 64, FAKE, None) == ERR_NULL
+    assert f(FAKE, 4, 64, 64, None, None) == ERR_NULL
+    assert f(FAKE, -1, 64, 64, FAKE, None) == ERR_SHAPE
+    assert f(FAKE, 4, 60, 64, FAKE, None) == ERR_SHAPE        # n % 8
+    assert f(FAKE, 4, 64, 32, FAKE, None) == ERR_SHAPE        # ld < n
+    assert f(FAKE, 4, 64, 68, FAKE, None) == ERR_ALIGN        # ld % 8
+    assert f(MIS, 4, 64, 64, FAKE, None) == ERR_ALIGN
+    assert f(FAKE, 0, 64, 64, FAKE, None) == OK               # empty chunk: no-op
+    assert f(None, 0, 0, 0, None, None) == OK
+
+
+def test_rtn_argument_errors(lib):
+    f = lib.hscale_rtn_scales
+    ws = hs.hscale_rtn_workspace_bytes()
+    assert ws >= 4
+    assert f(FAKE, 4, 24, FAKE, FAKE, FAKE, ws, None) == ERR_SHAPE   # n % 16
+    assert f(None, 4, 32, FAKE, FAKE, FAKE, ws, None) == ERR_NULL
+    assert f(FAKE, 4, 32, None, FAKE, FAKE, ws, None) == ERR_NULL
+    assert f(FAKE, 4, 32, FAKE, FAKE, None, ws, None) == ERR_WS
+    assert f(FAKE, 4, 32, FAKE, FAKE, FAKE, 2, None) == ERR_WS
+    assert f(MIS, 4, 32, FAKE, FAKE, FAKE, ws, None) == ERR_ALIGN
+    assert f(FAKE, -4, 32, FAKE, FAKE, FAKE, ws, None) == ERR_SHAPE
+    assert f(None, 0, 32, None, None, None, 0, None) == OK
+
+
+def test_refine_argument_errors(lib):
+    f = lib.hscale_refine_scales
+    assert f(FAKE, FAKE, 4, 32, FAKE, None, -1, 4, FAKE, FAKE, None) == ERR_ARG
+    assert f(FAKE, FAKE, 4, 32, FAKE, None, 4, 126, FAKE, FAKE, None) == ERR_ARG
+    assert f(FAKE, FAKE, 4, 40, FAKE, None, 4, 4, FAKE, FAKE, None) == ERR_SHAPE
+    assert f(FAKE, FAKE, 4, 32, None, None, 4, 4, FAKE, FAKE, None) == ERR_NULL
+    assert f(FAKE, FAKE, 4, 32, FAKE, None, 4, 4, None, FAKE, None) == ERR_NULL
+    assert f(FAKE, MIS, 4, 32, FAKE, None, 4, 4, FAKE, FAKE, None) == ERR_ALIGN   # h 16-B
+    assert f(FAKE, FAKE, 4, 32, FAKE, None, 4, 4, FAKE, ctypes.c_void_p(0x10004), None) == ERR_ALIGN
+    assert f(None, None, 0, 32, None, None, 4, 4, None, None, None) == OK
+
+
+def test_pack_argument_errors(lib):
+    f = lib.hscale_pack_nvfp4
+    assert f(FAKE, 4, 32, FAKE, None, FAKE, None) == ERR_NULL
+    assert f(FAKE, 4, 32, FAKE, FAKE, None, None) == ERR_NULL
+    assert f(FAKE, 4, 33, FAKE, FAKE, FAKE, None) == ERR_SHAPE
+    assert f(FAKE, 4, 32, FAKE, FAKE, ctypes.c_void_p(0x10004), None) == ERR_ALIGN
+    assert f(None, 4, 0, None, None, None, None) == OK
+
+
+def test_binding_refuses_cpu_tensors(lib):
+    import torch
+    x = torch.zeros(4, 16, dtype=torch.bfloat16)
+    h = torch.zeros(16)
+    with pytest.raises(TypeError):
+        hs.hscale_hessian_diag_accumulate(x, h)
+
+
+def test_build_flags_target_sm103a_only():
+    assert build.ARCH == ["-gencode", "arch=compute_103a,code=sm_103a"]
+    assert not any("fast_math" in f or "ftz=true" in f for f in build.NVCC_FLAGS)

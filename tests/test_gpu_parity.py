@@ -1,0 +1,401 @@
+"""GPU parity: the sm_103a kernels (through the C ABI) against the fp64 CPU oracle.
+
+Pass rules:
+  * h: |h_gpu - h_oracle| <= 1e-4 * h_oracle element-wise (exact zero where the oracle
+    has zero).
+  * s_g, RTN codes, packed nibbles: bit-exact.
+  * refined codes and nibbles: bit-exact in every group except the oracle's near-ties
+    (best and runner-up errors within 1e-6 relative); near-ties are counted and
+    reported.  The search gets one fp32 h on both sides (the oracle's h rounded to
+    fp32), so the comparison isolates the search.
+"""
+import os
+
+import numpy as np
+import pytest
+import torch
+
+import oracle
+import paper_2608_28113_gb300 as hs
+from paper_2608_28113_gb300 import workloads as wl
+
+pytestmark = pytest.mark.gpu
+
+H_RTOL = 1e-4
+
+
+@pytest.fixture(scope="module", autouse=True)
+def _setup():
+    if not torch.cuda.is_available():
+        pytest.skip("no CUDA device")
+    hs.load()
+    oracle.set_threads(os.cpu_count() or 1)
+
+
+def dev():
+    return torch.device("cuda", 0)
+
+
+def bits(t):
+    return wl.bf16_bits(t)
+
+
+def from_bits(b: np.ndarray) -> torch.Tensor:
+    return torch.from_numpy(np.ascontiguousarray(b).view(np.int16)).view(torch.bfloat16)
+
+
+def gpu_hessian(chunks, n):
+    h = torch.zeros(n, dtype=torch.float32, device=dev())
+    for x in chunks:
+        hs.hscale_hessian_diag_accumulate(x, h)
+    torch.cuda.synchronize()
+    return h.cpu().numpy()
+
+
+def oracle_hessian(chunks, n):
+    h = np.zeros(n)
+    for x in chunks:
+        xb = bits(x)
+        oracle.hessian_accumulate(xb, h, ld=xb.shape[1], n=n)
+    return h
+
+
+def assert_h_close(h_gpu, h_ref):
+    h_gpu = h_gpu.astype(np.float64)
+    zero = h_ref == 0
+    assert np.all(h_gpu[zero] == 0)
+    rel = np.abs(h_gpu[~zero] - h_ref[~zero]) / h_ref[~zero]
+    assert rel.max(initial=0.0) <= H_RTOL, f"max rel err {rel.max():.3e}"
+    return rel.max(initial=0.0)
+
+
+def gpu_rtn(w):
+    m, n = w.shape
+    sg = torch.empty(1, dtype=torch.float32, device=dev())
+    codes = torch.empty(m, n // 16, dtype=torch.uint8, device=dev())
+    ws = torch.empty(hs.hscale_rtn_workspace_bytes(), dtype=torch.uint8, device=dev())
+    hs.hscale_rtn_scales(w, sg, codes, ws)
+    torch.cuda.synchronize()
+    return sg, codes
+
+
+def gpu_refine(w, h32, sg, init, down, up, with_packed=True):
+    m, n = w.shape
+    codes = torch.empty(m, n // 16, dtype=torch.uint8, device=dev())
+    packed = torch.empty(m, n // 2, dtype=torch.uint8, device=dev()) if with_packed else None
+    h = None if h32 is None else torch.from_numpy(np.ascontiguousarray(h32, np.float32)).to(dev())
+    hs.hscale_refine_scales(w, h, sg, init, down, up, codes, packed)
+    torch.cuda.synchronize()
+    return codes.cpu().numpy(), (packed.cpu().numpy() if with_packed else None)
+
+
+def compare_search(ref, codes, packed, label=""):
+    """Bit-exact outside near-ties.  Returns (groups, near_ties, mismatches_in_near_ties)."""
+    nt = ref["near_tie"].astype(bool)
+    diff_code = codes != ref["codes"]
+    bad = diff_code & ~nt
+    assert not bad.any(), f"{label}: {bad.sum()} code mismatches outside near-ties at {np.argwhere(bad)[:5]}"
+    if packed is not None:
+        m, ng = codes.shape
+        pdiff = (packed.reshape(m, ng, 8) != ref["packed"].reshape(m, ng, 8)).any(axis=2)
+        badp = pdiff & ~nt
+        assert not badp.any(), f"{label}: {badp.sum()} nibble mismatches outside near-ties"
+        # where the codes agree, the nibbles must agree too (final re-quantization is exact)
+        assert not (pdiff & ~diff_code).any(), f"{label}: nibbles differ under an equal code"
+    print(f"[parity] {label}: groups={codes.size} near_ties={int(nt.sum())} "
+          f"near_tie_code_mismatches={int((diff_code & nt).sum())}")
+    return codes.size, int(nt.sum()), int((diff_code & nt).sum())
+
+
+def small_layer(seed=0, m=512, n=1024, sigma=0.02):
+    w = wl.weight(m, n, sigma, seed, device="cpu")
+    return w
+
+
+# ------------------------------------------------------------------ Hessian pass
+
+def test_hessian_single_chunk_small_layer():
+    W = wl.WORKLOADS["layer-512x1024"]
+    a = wl.channel_magnitudes(1024, W.sigma_a, W.outlier_channels, W.outlier_channel_mult, W.seed)
+    x = wl.activation_chunk(2048, a, W.seed, 0)
+    h_gpu = gpu_hessian([x.to(dev())], 1024)
+    h_ref = oracle_hessian([x], 1024)
+    print(f"[parity] hessian 2048x1024 max rel err {assert_h_close(h_gpu, h_ref):.3e}")
+
+
+@pytest.mark.parametrize("n,tokens,chunk,pad", [
+    (1040, 5000, 1536, 0),     # ragged column tile (1040 = 16 tiles + 16), chunk does not divide N
+    (64, 300000, 300000, 0),   # one call longer than a launch's token limit
+    (8, 3, 3, 8),              # minimum width, strided rows (ld = 16)
+    (4096, 777, 256, 64),      # wide rows, ld = n + 64, ragged last chunk
+    (14336, 4096, 4096, 0),    # MLP width
+])
+def test_hessian_chunking_ragged_and_strided(n, tokens, chunk, pad):
+    g = torch.Generator().manual_seed(n * 7 + tokens)
+    base = (torch.randn(tokens, n + pad, generator=g) * torch.exp(torch.randn(n + pad, generator=g)))
+    xb = base.to(torch.bfloat16)
+    chunks_cpu = [xb[t:t + chunk, :n] for t in range(0, tokens, chunk)]
+    xd = xb.to(dev())
+    chunks_gpu = [xd[t:t + chunk, :n] for t in range(0, tokens, chunk)]
+    h_gpu = gpu_hessian(chunks_gpu, n)
+    h_ref = np.zeros(n)
+    for c in chunks_cpu:
+        cb = bits(c.contiguous())
+        oracle.hessian_accumulate(cb, h_ref)
+    assert_h_close(h_gpu, h_ref)
+
+
+def test_hessian_closed_forms_and_empty_chunk():
+    n = 192
+    x = torch.full((1000, n), -1.5, dtype=torch.bfloat16, device=dev())
+    h = torch.zeros(n, device=dev())
+    hs.hscale_hessian_diag_accumulate(x, h)
+    hs.hscale_hessian_diag_accumulate(x[:0], h)          # empty chunk: no-op
+    torch.cuda.synchronize()
+    assert torch.all(h == 1000 * 2.25)
+    one_hot = torch.zeros(3 * n, n, dtype=torch.bfloat16, device=dev())
+    idx = torch.arange(3 * n, device=dev())
+    one_hot[idx, idx % n] = 2.0
+    h.zero_()
+    hs.hscale_hessian_diag_accumulate(one_hot, h)
+    torch.cuda.synchronize()
+    assert torch.all(h == 12.0)
+
+
+def test_hessian_is_deterministic():
+    g = torch.Generator().manual_seed(5)
+    x = (torch.randn(20000, 4096, generator=g) * 3).to(torch.bfloat16).to(dev())
+    outs = []
+    for _ in range(3):
+        h = torch.zeros(4096, device=dev())
+        hs.hscale_hessian_diag_accumulate(x, h)
+        outs.append(h.cpu())
+    assert torch.equal(outs[0], outs[1]) and torch.equal(outs[1], outs[2])
+
+
+# ------------------------------------------------------------------ global scale and RTN codes
+
+def test_rtn_scales_match_oracle_bit_exact():
+    for seed in range(4):
+        w = small_layer(seed)
+        sg, codes = gpu_rtn(w.to(dev()))
+        s_ref, _ = oracle.global_scale(bits(w))
+        assert sg.cpu().numpy()[0] == s_ref
+        assert np.array_equal(codes.cpu().numpy(), oracle.rtn_codes(bits(w), s_ref))
+
+
+def exact_tie_matrix():
+    """Groups whose max sits exactly on each E4M3 ladder value and midpoint, under
+    s_g = 2^-10 (amax = 2688 * 2^-10): RTN ties are decided by round-half-even."""
+    ladder = oracle.e4m3_decode_table()[0:127]
+    mids = 0.5 * (ladder[:-1] + ladder[1:])
+    vs = [v for v in np.concatenate([ladder[1:], mids]) if v <= 448]
+    w = np.zeros((len(vs), 32), np.float32)
+    for i, v in enumerate(vs):
+        w[i, 3] = 6 * v * 2.0 ** -10
+        w[i, 17] = -w[i, 3] / 3.0
+        w[i, 20:28] = np.linspace(-w[i, 3], w[i, 3], 8)
+    w[0, 0] = 2688 * 2.0 ** -10
+    return torch.from_numpy(w).to(torch.bfloat16)
+
+
+def test_rtn_codes_exact_ties_and_saturation():
+    w = exact_tie_matrix()
+    sg, codes = gpu_rtn(w.to(dev()))
+    s_ref, _ = oracle.global_scale(bits(w))
+    assert sg.cpu().numpy()[0] == s_ref == np.float32(2.0 ** -10)
+    assert np.array_equal(codes.cpu().numpy(), oracle.rtn_codes(bits(w), s_ref))
+    sg_only = torch.empty(1, device=dev())
+    ws = torch.empty(hs.hscale_rtn_workspace_bytes(), dtype=torch.uint8, device=dev())
+    hs.hscale_rtn_scales(w.to(dev()), sg_only, None, ws)   # codes = NULL: s_g only
+    torch.cuda.synchronize()
+    assert sg_only.item() == float(s_ref)
+
+
+# ------------------------------------------------------------------ search (Algorithm 1)
+
+def oracle_h32(seed, n, tokens=2048, sigma_a=1.0):
+    a = wl.channel_magnitudes(n, sigma_a, 8, 50.0, seed)
+    x = wl.activation_chunk(tokens, a, seed, 0)
+    h = np.zeros(n)
+    oracle.hessian_accumulate(bits(x), h)
+    return h.astype(np.float32)
+
+
+@pytest.mark.parametrize("down,up", [(4, 4), (9, 6), (0, 0), (1, 1), (8, 8), (16, 16), (0, 7), (125, 125)])
+def test_refine_matches_oracle_small_layer(down, up):
+    m, n = (512, 1024) if down + up < 40 else (64, 1024)
+    w = small_layer(0, m, n)
+    h32 = oracle_h32(0, n)
+    wd = w.to(dev())
+    sg, _ = gpu_rtn(wd)
+    s_ref, _ = oracle.global_scale(bits(w))
+    ref = oracle.refine(bits(w), h32, s_ref, None, down, up)
+    codes, packed = gpu_refine(wd, h32, sg, None, down, up)
+    compare_search(ref, codes, packed, f"layer {m}x{n} window -{down}/+{up}")
+
+
+def test_refine_with_init_codes_aliasing_and_no_packed_output():
+    w = small_layer(1, 256, 512)
+    h32 = oracle_h32(1, 512)
+    wd = w.to(dev())
+    sg, rtn = gpu_rtn(wd)
+    s_ref, _ = oracle.global_scale(bits(w))
+    # arbitrary baseline codes (sign bits and off-ladder values included)
+    g = np.random.default_rng(3)
+    init = g.integers(0, 256, size=(256, 32)).astype(np.uint8)
+    ref = oracle.refine(bits(w), h32, s_ref, init, 4, 4)
+    buf = torch.from_numpy(init).to(dev())
+    h = torch.from_numpy(h32).to(dev())
+    packed = torch.empty(256, 256, dtype=torch.uint8, device=dev())
+    hs.hscale_refine_scales(wd, h, sg, buf, 4, 4, buf, packed)   # codes_out aliases init_codes
+    torch.cuda.synchronize()
+    compare_search(ref, buf.cpu().numpy(), packed.cpu().numpy(), "init codes, in place")
+    codes_np, _ = gpu_refine(wd, h32, sg, rtn, 4, 4, with_packed=False)
+    ref2 = oracle.refine(bits(w), h32, s_ref, None, 4, 4)
+    compare_search(ref2, codes_np, None, "rtn init codes, no packed output")
+
+
+def test_refine_h_none_is_plain_mse_search():
+    w = small_layer(2, 256, 1024)
+    wd = w.to(dev())
+    sg, _ = gpu_rtn(wd)
+    s_ref, _ = oracle.global_scale(bits(w))
+    ref = oracle.refine(bits(w), None, s_ref, None, 9, 6)
+    codes, packed = gpu_refine(wd, None, sg, None, 9, 6)
+    compare_search(ref, codes, packed, "h = 1")
+
+
+def test_refine_edge_groups():
+    """All-zero groups, h = 0 on whole groups, the group holding amax (code 126, the
+    upward walk clips), tiny groups near code 1 (the downward walk clips), -0."""
+    rng = np.random.default_rng(11)
+    m, n = 64, 256
+    w = (rng.standard_t(4, size=(m, n)) * 0.02).astype(np.float32)
+    w[0, :16] = 0.0                       # all-zero group
+    w[1, :16] = -0.0                      # all negative zeros
+    w[2, 16:32] *= 1e-4                   # tiny group near the bottom of the ladder
+    w[3, 32:48] = 0.0
+    w[3, 40] = 1e-6                       # one tiny non-zero
+    w[5, 100] = 40.0                      # the tensor's amax: code 126
+    w[6, 3] = 39.0
+    wb = torch.from_numpy(w).to(torch.bfloat16)
+    b = bits(wb)
+    b[1, :16] = 0x8000
+    wb = from_bits(b)
+    h32 = oracle_h32(4, n)
+    h32[48:64] = 0.0                      # h = 0 on a whole group column
+    h32[64:80] = np.float32(1e-30)        # vanishing channel energy
+    wd = wb.to(dev())
+    sg, _ = gpu_rtn(wd)
+    s_ref, _ = oracle.global_scale(b)
+    assert sg.cpu().numpy()[0] == s_ref
+    for down, up in ((4, 4), (9, 6)):
+        ref = oracle.refine(b, h32, s_ref, None, down, up)
+        codes, packed = gpu_refine(wd, h32, sg, None, down, up)
+        compare_search(ref, codes, packed, f"edge groups -{down}/+{up}")
+        assert codes[5, 6] == ref["codes"][5, 6]
+
+
+@pytest.mark.parametrize("m,n", [(1, 16), (3, 48), (33, 16 * 33), (1, 4096 * 4)])
+def test_refine_tiny_and_ragged_shapes(m, n):
+    w = wl.weight(m, n, 0.02, m * 1000 + n)
+    h32 = oracle_h32(7, n)
+    wd = w.to(dev())
+    sg, _ = gpu_rtn(wd)
+    s_ref, _ = oracle.global_scale(bits(w))
+    ref = oracle.refine(bits(w), h32, s_ref, None, 4, 4)
+    codes, packed = gpu_refine(wd, h32, sg, None, 4, 4)
+    compare_search(ref, codes, packed, f"shape {m}x{n}")
+
+
+def test_refine_short_global_scale_exact_midpoint_ties():
+    """amax = 2688 * 2^-7 gives s_g = 2^-7 exactly, so many |w| / (s_g l) land exactly on
+    E2M1 midpoints: nibbles must follow round-half-even bit-exactly."""
+    rng = np.random.default_rng(12)
+    m, n = 128, 512
+    grid = np.array([0.25, 0.75, 1.25, 1.75, 2.5, 3.5, 5.0, 1.0, 3.0, 0.5])
+    lad = oracle.e4m3_decode_table()[1:127]
+    l = lad[rng.integers(40, 60, size=(m, n // 16))]
+    q = grid[rng.integers(0, grid.size, size=(m, n))]
+    w = (q * np.repeat(l, 16, axis=1) * 2.0 ** -7 * rng.choice([-1, 1], size=(m, n))).astype(np.float32)
+    w[0, 0] = 2688 * 2.0 ** -7
+    wb = torch.from_numpy(w).to(torch.bfloat16)
+    b = bits(wb)
+    s_ref, _ = oracle.global_scale(b)
+    assert s_ref == np.float32(2.0 ** -7)
+    h32 = oracle_h32(8, n)
+    wd = wb.to(dev())
+    sg, codes_rtn = gpu_rtn(wd)
+    for down, up in ((4, 4), (0, 0)):
+        ref = oracle.refine(b, h32, s_ref, None, down, up)
+        codes, packed = gpu_refine(wd, h32, sg, None, down, up)
+        compare_search(ref, codes, packed, f"exact midpoints -{down}/+{up}")
+
+
+def test_pack_matches_oracle_bit_exact():
+    w = small_layer(9, 256, 1024)
+    wd = w.to(dev())
+    sg, codes = gpu_rtn(wd)
+    s_ref, _ = oracle.global_scale(bits(w))
+    rng = np.random.default_rng(9)
+    for c in (codes.cpu().numpy(), rng.integers(0, 256, size=(256, 64)).astype(np.uint8)):
+        ct = torch.from_numpy(c).to(dev())
+        packed = torch.empty(256, 512, dtype=torch.uint8, device=dev())
+        hs.hscale_pack_nvfp4(wd, sg, ct, packed)
+        torch.cuda.synchronize()
+        assert np.array_equal(packed.cpu().numpy(), oracle.pack(bits(w), s_ref, c))
+
+
+def test_refine_is_deterministic():
+    w = small_layer(3, 512, 1024)
+    h32 = oracle_h32(3, 1024)
+    wd = w.to(dev())
+    sg, _ = gpu_rtn(wd)
+    a = gpu_refine(wd, h32, sg, None, 8, 8)
+    b = gpu_refine(wd, h32, sg, None, 8, 8)
+    assert np.array_equal(a[0], b[0]) and np.array_equal(a[1], b[1])
+
+
+# ------------------------------------------------------------------ full-size workloads
+
+def full_size_check(name, sample_rows):
+    """The workload at its full size in the launch configuration bench.py times: h over
+    every streamed chunk (all columns, against the oracle fed the same chunks), s_g and
+    RTN codes over the whole matrix, and the search on a seeded sample of rows."""
+    W = wl.WORKLOADS[name]
+    L = W.layers[0]
+    n, m = L.in_features, L.out_features
+    chunk = W.chunk_tokens[n]
+    a = wl.channel_magnitudes(n, W.sigma_a, W.outlier_channels, W.outlier_channel_mult, W.seed,
+                              device=dev())
+    h = torch.zeros(n, device=dev())
+    h_ref = np.zeros(n)
+    for c in range(0, W.tokens // chunk):
+        x = wl.activation_chunk(chunk, a, W.seed, c)
+        hs.hscale_hessian_diag_accumulate(x, h)
+        oracle.hessian_accumulate(bits(x), h_ref)
+        del x
+    torch.cuda.synchronize()
+    err = assert_h_close(h.cpu().numpy(), h_ref)
+    print(f"[parity] {name}: h over {W.tokens} tokens x {n}: max rel err {err:.3e}")
+    w = wl.weight(m, n, W.sigma_w, W.seed, device=dev())
+    sg, codes = gpu_rtn(w)
+    wb = bits(w)
+    s_ref, _ = oracle.global_scale(wb)
+    assert sg.cpu().numpy()[0] == s_ref
+    assert np.array_equal(codes.cpu().numpy(), oracle.rtn_codes(wb, s_ref))
+    h32 = h_ref.astype(np.float32)
+    rows = np.sort(np.random.default_rng(W.seed).choice(m, size=min(sample_rows, m), replace=False))
+    for k in W.window:
+        codes_g, packed_g = gpu_refine(w, h32, sg, None, k, k)
+        ref = oracle.refine(wb[rows], h32, s_ref, None, k, k)
+        compare_search(ref, codes_g[rows], packed_g[rows], f"{name} k={k} ({rows.size} sampled rows)")
+
+
+def test_full_size_llama8b_q_proj():
+    full_size_check("llama8b-q_proj", sample_rows=512)
+
+
+def test_full_size_mlp_down_proj():
+    full_size_check("mlp-down_proj", sample_rows=128)
