@@ -26,7 +26,6 @@ import argparse
 import json
 import os
 import statistics
-import subprocess
 import sys
 import time
 
@@ -47,11 +46,13 @@ FALLBACK_HBM_GBS = 6800.0
 def parse():
     p = argparse.ArgumentParser()
     p.add_argument("--gpus", type=int, default=1)
-    p.add_argument("--steps", type=int, default=10)
+    p.add_argument("--steps", type=int, default=50)
     p.add_argument("--warmup", type=int, default=3)
     p.add_argument("--impl", choices=["hscale", "reference"], default="hscale")
     p.add_argument("--workload", default="llama8b-q_proj", choices=sorted(wl.WORKLOADS))
     p.add_argument("--k", type=int, default=None, help="window half-width (default: workload's)")
+    p.add_argument("--tokens", type=int, default=None,
+                   help="calibration tokens per step (default: the workload's; smaller for ncu captures)")
     p.add_argument("--no-cpu-baseline", action="store_true")
     p.add_argument("--no-e2e", action="store_true")
     return p.parse_args()
@@ -102,65 +103,88 @@ def measured_peaks():
 
 
 class ClockSampler:
-    """nvidia-smi clock/throttle samples during the timed region."""
-    FIELDS = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
-              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
-              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+    """SM clock and clock-event (throttle) reasons, read through NVML every ~2 ms on a
+    background thread during the timed region (nothing is recorded without NVML)."""
+    REASONS = {0x4: "sw_power_cap", 0x8: "hw_slowdown", 0x20: "sw_thermal_slowdown",
+               0x40: "hw_thermal_slowdown", 0x80: "hw_power_brake_slowdown"}
 
-    def __init__(self, index: int):
-        self.index = index
-        self.proc = None
+    def __init__(self, device_index: int):
+        self.device_index = device_index
+        self.samples, self.max_mhz, self.reasons = [], None, set()
+        self._nvml = None
+        self._handle = None
+        self._stop = False
+        try:
+            import ctypes
+            nv = ctypes.CDLL("libnvidia-ml.so.1")
+            if nv.nvmlInit_v2() != 0:
+                raise OSError("nvmlInit failed")
+            h = ctypes.c_void_p()
+            ok = False
+            try:
+                bus = torch.cuda.get_device_properties(device_index)
+                bus_id = "%08x:%02x:%02x.0" % (bus.pci_domain_id, bus.pci_bus_id, bus.pci_device_id)
+                ok = nv.nvmlDeviceGetHandleByPciBusId_v2(bus_id.encode(), ctypes.byref(h)) == 0
+            except AttributeError:
+                pass
+            if not ok:
+                vis = os.environ.get("CUDA_VISIBLE_DEVICES", "").split(",")
+                idx = int(vis[device_index]) if device_index < len(vis) and vis[device_index].strip().isdigit() else device_index
+                if nv.nvmlDeviceGetHandleByIndex_v2(idx, ctypes.byref(h)) != 0:
+                    raise OSError("no NVML handle")
+            self._nvml, self._handle, self._ct = nv, h, ctypes
+            v = ctypes.c_uint()
+            if nv.nvmlDeviceGetMaxClockInfo(h, 1, ctypes.byref(v)) == 0:
+                self.max_mhz = float(v.value)
+        except Exception:
+            self._nvml = None
+
+    def _sample(self):
+        ct, nv, h = self._ct, self._nvml, self._handle
+        v = ct.c_uint()
+        r = ct.c_ulonglong()
+        if nv.nvmlDeviceGetClockInfo(h, 1, ct.byref(v)) == 0:
+            self.samples.append(float(v.value))
+        if nv.nvmlDeviceGetCurrentClocksEventReasons(h, ct.byref(r)) == 0:
+            for bit, name in self.REASONS.items():
+                if r.value & bit:
+                    self.reasons.add(name)
+
+    def _loop(self):
+        while not self._stop:
+            self._sample()
+            time.sleep(0.002)
 
     def __enter__(self):
-        try:
-            self.proc = subprocess.Popen(
-                ["nvidia-smi", f"--id={self.index}", f"--query-gpu={self.FIELDS}",
-                 "--format=csv,noheader,nounits", "-lms", "100"],
-                stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
-        except Exception:
-            self.proc = None
+        if self._nvml is not None:
+            import threading
+            self._sample()
+            self._thread = threading.Thread(target=self._loop, daemon=True)
+            self._thread.start()
         return self
 
     def __exit__(self, *a):
-        self.lines = []
-        if self.proc:
-            self.proc.terminate()
-            try:
-                out, _ = self.proc.communicate(timeout=5)
-            except Exception:
-                self.proc.kill()
-                out = ""
-            self.lines = [l for l in out.splitlines() if l.strip()]
+        if self._nvml is not None:
+            self._stop = True
+            self._thread.join()
+            self._sample()
 
     def summary(self):
-        sm, mx, reasons = [], None, set()
-        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
-        for l in getattr(self, "lines", []):
-            f = [x.strip() for x in l.split(",")]
-            if len(f) < 9:
-                continue
-            try:
-                sm.append(float(f[1]))
-                mx = float(f[2])
-            except ValueError:
-                continue
-            for name, v in zip(names, f[5:9]):
-                if v.lower() == "active":
-                    reasons.add(name)
-        return {"sm_mhz": statistics.median(sm) if sm else None, "sm_max_mhz": mx,
-                "reasons": sorted(reasons), "samples": len(sm)}
+        return {"sm_mhz": statistics.median(self.samples) if self.samples else None,
+                "sm_max_mhz": self.max_mhz, "reasons": sorted(self.reasons),
+                "samples": len(self.samples), "source": "nvml" if self._nvml else "none"}
 
 
 # ------------------------------------------------------------------ workload
 class Layer:
     """Device-resident inputs and outputs of one layer of a workload."""
 
-    def __init__(self, W: wl.Workload, rank: int, k: int, device):
+    def __init__(self, W: wl.Workload, rank: int, k: int, device, tokens=None):
         L = W.layers[0]
         self.W, self.k = W, k
         self.m, self.n = L.out_features, L.in_features
         self.chunk = W.chunk_tokens[self.n]
-        self.nchunks = W.tokens // self.chunk
+        self.nchunks = max(1, (tokens or W.tokens) // self.chunk)
         self.tokens = self.nchunks * self.chunk
         seed = W.seed + 7919 * rank
         self.seed = seed
@@ -178,23 +202,48 @@ class Layer:
         self.packed = torch.empty(self.m, self.n // 2, dtype=torch.uint8, device=device)
 
 
-def run_step(hs, L: Layer, x=None, w=None, ev=None):
-    """One pass of the hot path.  ev: optional 4 events (start, after h, after rtn, end)."""
+def hessian_phase(hs, L: Layer, x=None):
+    """h = 0, then one hscale_hessian_diag_accumulate per calibration chunk."""
     x = L.x if x is None else x
-    w = L.w if w is None else w
-    if ev:
-        ev[0].record()
     L.h.zero_()
     for c in range(L.nchunks):
         hs.hscale_hessian_diag_accumulate(x[c * L.chunk:(c + 1) * L.chunk], L.h)
+
+
+def scale_phase(hs, L: Layer, w=None):
+    """Global scale + RTN codes, then the H-Scale search with the final packing."""
+    w = L.w if w is None else w
+    hs.hscale_rtn_scales(w, L.sg, L.codes0, L.ws)
+    hs.hscale_refine_scales(w, L.h, L.sg, L.codes0, L.k, L.k, L.codes, L.packed)
+
+
+def run_step(hs, L: Layer, ev=None):
+    """One eager pass of the hot path.  ev: optional 3 events (start, after h, end)."""
+    if ev:
+        ev[0].record()
+    hessian_phase(hs, L)
     if ev:
         ev[1].record()
-    hs.hscale_rtn_scales(w, L.sg, L.codes0, L.ws)
+    scale_phase(hs, L)
     if ev:
         ev[2].record()
-    hs.hscale_refine_scales(w, L.h, L.sg, L.codes0, L.k, L.k, L.codes, L.packed)
-    if ev:
-        ev[3].record()
+
+
+def capture_graphs(hs, L: Layer):
+    """The step's launch sequence captured as two CUDA graphs (Hessian pass; scales)."""
+    side = torch.cuda.Stream()
+    side.wait_stream(torch.cuda.current_stream())
+    with torch.cuda.stream(side):
+        run_step(hs, L)
+    torch.cuda.current_stream().wait_stream(side)
+    torch.cuda.synchronize()
+    gh, gs = torch.cuda.CUDAGraph(), torch.cuda.CUDAGraph()
+    with torch.cuda.graph(gh):
+        hessian_phase(hs, L)
+    with torch.cuda.graph(gs):
+        scale_phase(hs, L)
+    torch.cuda.synchronize()
+    return gh, gs
 
 
 KERNELS_PER_STEP_FIXED = 3  # amax, rtn codes, refine
@@ -291,15 +340,29 @@ def gpu_arm(args, d: Dist):
     dev = torch.device("cuda", d.local)
     W = wl.WORKLOADS[args.workload]
     k = args.k if args.k is not None else W.window[0]
-    L = Layer(W, d.rank, k, dev)
+    L = Layer(W, d.rank, k, dev, tokens=args.tokens)
     L.ws = torch.empty(hs.hscale_rtn_workspace_bytes(), dtype=torch.uint8, device=dev)
     torch.cuda.synchronize()
 
-    for _ in range(max(args.warmup, 3)):
+    warm = max(args.warmup, 3)
+    for _ in range(warm):
         run_step(hs, L)
     torch.cuda.synchronize()
 
-    evs = [[torch.cuda.Event(enable_timing=True) for _ in range(4)] for _ in range(args.steps)]
+    # eager launches (one API call per chunk), for reference
+    ev_e = [[torch.cuda.Event(enable_timing=True) for _ in range(3)] for _ in range(args.steps)]
+    torch.cuda.synchronize()
+    for s in range(args.steps):
+        run_step(hs, L, ev=ev_e[s])
+    torch.cuda.synchronize()
+    ms_eager = sum(e[0].elapsed_time(e[2]) for e in ev_e) / args.steps
+
+    # timed region: the same launches replayed from CUDA graphs
+    gh, gs = capture_graphs(hs, L)
+    for _ in range(warm):
+        gh.replay()
+        gs.replay()
+    evs = [[torch.cuda.Event(enable_timing=True) for _ in range(3)] for _ in range(args.steps)]
     d.barrier()
     torch.cuda.synchronize()
     with ClockSampler(d.local) as clk:
@@ -307,16 +370,32 @@ def gpu_arm(args, d: Dist):
         t1 = torch.cuda.Event(enable_timing=True)
         t0.record()
         for s in range(args.steps):
-            run_step(hs, L, ev=evs[s])
+            evs[s][0].record()
+            gh.replay()
+            evs[s][1].record()
+            gs.replay()
+            evs[s][2].record()
         t1.record()
         torch.cuda.synchronize()
     d.barrier()
     ms_total = t0.elapsed_time(t1)
     ms_h = sum(e[0].elapsed_time(e[1]) for e in evs) / args.steps
-    ms_rtn = sum(e[1].elapsed_time(e[2]) for e in evs) / args.steps
-    ms_ref = sum(e[2].elapsed_time(e[3]) for e in evs) / args.steps
+    ms_sc = sum(e[1].elapsed_time(e[2]) for e in evs) / args.steps
     ms_step = d.max(ms_total / args.steps)
     value = L.groups * d.world / (ms_step * 1e-3)
+
+    # per-kernel times of the scale phase (rtn_scales; refine) from an eager loop
+    ev_k = [[torch.cuda.Event(enable_timing=True) for _ in range(3)] for _ in range(args.steps)]
+    for s in range(args.steps):
+        hs.hscale_rtn_scales(L.w, L.sg, L.codes0, L.ws)
+        ev_k[s][0].record()
+        hs.hscale_rtn_scales(L.w, L.sg, L.codes0, L.ws)
+        ev_k[s][1].record()
+        hs.hscale_refine_scales(L.w, L.h, L.sg, L.codes0, L.k, L.k, L.codes, L.packed)
+        ev_k[s][2].record()
+    torch.cuda.synchronize()
+    ms_rtn = sum(e[0].elapsed_time(e[1]) for e in ev_k) / args.steps
+    ms_ref = sum(e[1].elapsed_time(e[2]) for e in ev_k) / args.steps
 
     # ---- roofline of the dominant kernel (the Hessian pass)
     hbm_peak, peak_kind, peaks = measured_peaks()
@@ -352,7 +431,9 @@ def gpu_arm(args, d: Dist):
                      "peak_kind": f"{peak_kind} HBM copy bandwidth",
                      "frac_of_8TBs_spec": h_gbs / HBM_SPEC_GBS, "traffic": None,
                      "bytes_per_launch": h_bytes_launch, "ms_per_launch": ms_h_launch},
-        "phases_ms": {"hessian": ms_h, "rtn_scales": ms_rtn, "refine": ms_ref},
+        "phases_ms": {"hessian": ms_h, "scales": ms_sc, "rtn_scales": ms_rtn, "refine": ms_ref},
+        "ms_per_step_eager": ms_eager,
+        "timed_launch": "CUDA graphs of the step's API calls (Hessian pass; scales)",
         "hessian": {"gbs": h_gbs, "tokens_channels_per_s": L.chunk * L.n / (ms_h_launch * 1e-3),
                     "frac_of_measured_hbm": h_gbs / hbm_peak, "frac_of_8TBs": h_gbs / HBM_SPEC_GBS},
         "search": {"groups_per_s": L.groups / (ms_ref * 1e-3), "candidates": C,

@@ -75,18 +75,29 @@ const char* hscale_status_string(int status);
 int hscale_abi_version(void);
 
 /*
+ * Device-side failure report.  Kernels never hang: every wait on an asynchronous copy
+ * is bounded, and a wait that runs out sets a sticky flag on the current device (and
+ * the affected h entries become NaN).  This call synchronises with the device, stores
+ * the flags in *flags (0 = no failure; bit 0 = a bounded wait ran out) and clears them.
+ */
+int hscale_device_error_flags(uint32_t* flags);
+
+/*
  * Hessian diagonal, one token chunk (Sec. 3.2, Eq. 4).
  *
  *   h[j] += sum_{t < tokens} x[t * ld_x + j]^2      for j < n
  *
- * x      [tokens, ld_x] bfloat16, 16-byte aligned; only the first n columns are read.
+ * x      [tokens, ld_x] bfloat16, 16-byte aligned; only the first n columns are read;
+ *        tokens < 2^31.
  * h      [n] fp32, read and written (accumulated in place).  Zero it before the first
  *        chunk; streaming a calibration set is one call per chunk on the same h.
  * n      multiple of 8; ld_x >= n and a multiple of 8.
  * Arithmetic: x^2 is exact in fp32; sums are fp32 in a fixed order (per-thread runs of
  * at most 1024 tokens, then fixed-order trees inside the CTA and across a thread-block
  * cluster), so each call adds a relative error of at most about 1100 * 2^-24 to h.
- * Nothing else is touched: the call needs no workspace.
+ * Nothing else is touched: the call needs no workspace.  Consecutive calls on one
+ * stream overlap (programmatic dependent launch): a call starts reading its chunk
+ * while the previous one finishes, and waits for it before it updates h.
  */
 int hscale_hessian_diag_accumulate(const void* x_bf16, int64_t tokens, int64_t n, int64_t ld_x,
                                    float* h, void* stream);

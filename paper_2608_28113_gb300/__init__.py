@@ -22,6 +22,7 @@ import torch
 
 __all__ = [
     "HScaleError", "load", "library_path", "hscale_status_string", "hscale_abi_version",
+    "hscale_device_error_flags",
     "hscale_hessian_diag_accumulate", "hscale_rtn_workspace_bytes", "hscale_rtn_scales",
     "hscale_refine_scales", "hscale_pack_nvfp4", "EXPORTED_SYMBOLS",
 ]
@@ -36,6 +37,7 @@ _P, _I64, _I32, _SZ = ctypes.c_void_p, ctypes.c_int64, ctypes.c_int32, ctypes.c_
 _SIGNATURES = {
     "hscale_status_string": (ctypes.c_char_p, [ctypes.c_int]),
     "hscale_abi_version": (ctypes.c_int, []),
+    "hscale_device_error_flags": (ctypes.c_int, [_P]),
     "hscale_hessian_diag_accumulate": (ctypes.c_int, [_P, _I64, _I64, _I64, _P, _P]),
     "hscale_rtn_workspace_bytes": (_SZ, []),
     "hscale_rtn_scales": (ctypes.c_int, [_P, _I64, _I64, _P, _P, _P, _SZ, _P]),
@@ -82,6 +84,13 @@ def hscale_status_string(status: int) -> str:
 
 def hscale_abi_version() -> int:
     return int(load().hscale_abi_version())
+
+
+def hscale_device_error_flags() -> int:
+    """Synchronise and return (then clear) the device failure flags; 0 = none."""
+    v = ctypes.c_uint32(0)
+    _check("hscale_device_error_flags", load().hscale_device_error_flags(ctypes.byref(v)))
+    return int(v.value)
 
 
 def _stream_ptr(stream) -> int:

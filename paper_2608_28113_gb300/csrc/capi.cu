@@ -71,6 +71,11 @@ const char* hscale_status_string(int status) {
 
 int hscale_abi_version(void) { return 1; }
 
+int hscale_device_error_flags(uint32_t* flags) {
+  if (flags == nullptr) return HSCALE_ERR_NULL;
+  return from_cuda(hscale::read_and_clear_device_error(flags));
+}
+
 int hscale_hessian_diag_accumulate(const void* x_bf16, int64_t tokens, int64_t n, int64_t ld_x,
                                    float* h, void* stream) {
   if (tokens < 0 || n < 0 || ld_x < n) return HSCALE_ERR_SHAPE;
@@ -80,7 +85,7 @@ int hscale_hessian_diag_accumulate(const void* x_bf16, int64_t tokens, int64_t n
   if (x_bf16 == nullptr || h == nullptr) return HSCALE_ERR_NULL;
   if (ld_x % 8 != 0) return HSCALE_ERR_ALIGN;
   if (!aligned(x_bf16, 16) || !aligned(h, 4)) return HSCALE_ERR_ALIGN;
-  if (tokens > INT64_MAX / ld_x) return HSCALE_ERR_SHAPE;
+  if (tokens > INT32_MAX || tokens > INT64_MAX / ld_x) return HSCALE_ERR_SHAPE;
   return from_cuda(hscale::launch_hessian(x_bf16, tokens, n, ld_x, h, as_stream(stream)));
 }
 

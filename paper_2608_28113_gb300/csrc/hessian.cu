@@ -3,37 +3,57 @@
 // HBM-bound column sum of squares over a bf16 token chunk X[tokens, ld].
 //
 // Layout of the work
-//   * A CTA owns a 64-channel column tile (eight 16-byte vectors per row) and a
-//     contiguous run of tokens.  Its 256 threads are 32 row phases x 8 vectors: a warp
-//     reads 4 rows x 128 contiguous bytes per load instruction, and each thread keeps
-//     8 loads of 16 bytes in flight (rows r, r+32, ..., r+224).
+//   * A CTA owns a 64-channel column tile (128 bytes of every row) and a contiguous
+//     run of tokens.  One thread streams the run into a ring of shared-memory stages
+//     with 2-D TMA tensor loads (64 channels x 64 rows = 8 KB per stage, 6 stages in
+//     flight per CTA, L2 evict-first); the CTA's 256 threads (32 row phases x 8
+//     16-byte vectors) read each stage back with conflict-free 128-bit shared loads
+//     and accumulate in fp32.  mbarriers order the ring; every wait is bounded.
 //   * The token range of a tile is split over the CTAs of one thread-block cluster
-//     (1, 2, 4 or 8 CTAs, picked so the grid is about one wave of resident CTAs).  The
-//     CTAs of a cluster reduce their partial sums through distributed shared memory, so
-//     the kernel needs no global scratch, no atomics and no second launch.
+//     (1, 2, 4 or 8 CTAs, so the grid is about one wave of resident CTAs).  The CTAs
+//     of a cluster reduce their partial sums through distributed shared memory: the
+//     kernel needs no global scratch, no atomics and no second launch.
+//   * Launches use programmatic dependent launch: the next chunk's kernel may start
+//     streaming X while this one finishes; it waits (griddepcontrol.wait) only before
+//     it reads and writes h.
+//   * Rows past the end of the chunk read as zero (TMA out-of-bounds fill), so ragged
+//     chunks and ragged column tiles need no special cases.
 // Determinism and accuracy
 //   x^2 of a bf16 value is exact in fp32.  Each thread adds at most 1024 squares in
 //   token order; partials then meet in fixed-order pairwise trees (4 phases in a warp,
 //   8 warps in the CTA, the cluster's CTAs), and the total is added to h once.  Every
 //   run gives the same bits, and a call adds a relative error of at most
 //   (1024 + 2 + 3 + 3 + 1) * 2^-24 to h.
+// Failure reporting
+//   A wait that runs out of polls (it cannot on a healthy GPU) sets the library's
+//   device error flag and turns the affected h entries into NaN instead of hanging.
 #include <cooperative_groups.h>
+#include <cuda.h>
+
+#include <algorithm>
+#include <mutex>
 
 #include "hscale_device.cuh"
 #include "hscale_internal.h"
+#include "tma.cuh"
 
 namespace cg = cooperative_groups;
 
 namespace hscale {
+
+__device__ uint32_t g_device_error = 0;
+
 namespace {
 
-constexpr int kVecPerRow = 8;                      // 16-byte vectors per tile row
-constexpr int kTileCols = kVecPerRow * 8;          // 64 channels
+constexpr int kTileCols = 64;                       // channels per CTA tile (128 bytes)
 constexpr int kThreads = 256;
-constexpr int kPhases = kThreads / kVecPerRow;     // 32 rows read side by side
-constexpr int kUnroll = 8;                         // rows in flight per thread
+constexpr int kPhases = 32;                         // rows read side by side
 constexpr int kWarps = kThreads / 32;
-constexpr int64_t kMaxRunPerThread = 1024;         // longest sequential fp32 run
+constexpr int kStageRows = 64;
+constexpr int kStages = 6;
+constexpr uint32_t kStageBytes = kStageRows * kTileCols * 2;
+constexpr size_t kRingBytes = (size_t)kStages * kStageBytes;
+constexpr int64_t kMaxRowsPerCta = 1024 * kPhases;  // <= 1024 sequential adds per thread
 constexpr int kMaxCluster = 8;
 
 __device__ __forceinline__ void accum_sq8(float (&acc)[8], const uint4& v) {
@@ -50,33 +70,81 @@ __device__ __forceinline__ void accum_sq8(float (&acc)[8], const uint4& v) {
 }
 
 template <int CS>
-__global__ void __launch_bounds__(kThreads)
-hessian_colsumsq_kernel(const uint4* __restrict__ x, int64_t tokens, int64_t ld_vec, int nvec,
+__global__ void __launch_bounds__(kThreads, 4)
+hessian_colsumsq_kernel(const __grid_constant__ CUtensorMap xmap, int64_t row0, int64_t rows,
                         int n, float* __restrict__ h, int64_t rows_per_cta) {
+  extern __shared__ __align__(1024) uint8_t ring[];
+  __shared__ __align__(8) uint64_t full_bar[kStages];
+  __shared__ __align__(8) uint64_t empty_bar[kStages];
   __shared__ float warp_part[kWarps][kTileCols];
   __shared__ float cta_part[kTileCols];
+  __shared__ int s_bad;
 
   cg::cluster_group cluster = cg::this_cluster();
   const unsigned crank = cluster.block_rank();
-  const int tid = threadIdx.x;
-  const int v = tid & (kVecPerRow - 1);
-  const int phase = tid / kVecPerRow;
-  const int vec = blockIdx.y * kVecPerRow + v;
-  const int64_t r0 = (int64_t)crank * rows_per_cta;
-  const int64_t r1 = min(tokens, r0 + rows_per_cta);
+  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+  const int v = tid & 7, p = tid >> 3;
+  const int64_t r0 = row0 + (int64_t)crank * rows_per_cta;
+  const int64_t r1 = min(row0 + rows, r0 + rows_per_cta);
+  const int nst = r1 > r0 ? (int)((r1 - r0 + kStageRows - 1) / kStageRows) : 0;
+  const int x0 = blockIdx.y * kTileCols;
+
+  uint64_t policy = 0;
+  int issued = 0;
+  if (tid == 0) {
+    prefetch_tensormap(&xmap);
+    for (int s = 0; s < kStages; ++s) {
+      mbar_init(&full_bar[s], 1);
+      mbar_init(&empty_bar[s], kWarps);
+    }
+    mbar_fence_init();
+    s_bad = 0;
+  }
+  __syncthreads();
+  if (tid == 0) {
+    policy = l2_evict_first_policy();
+    for (; issued < kStages && issued < nst; ++issued) {
+      mbar_arrive_expect_tx(&full_bar[issued], kStageBytes);
+      tma_load_2d(ring + (size_t)issued * kStageBytes, &xmap, x0, (int32_t)(r0 + issued * kStageRows),
+                  &full_bar[issued], policy);
+    }
+  }
+  pdl_launch_dependents();
 
   float acc[8] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};
-  if (vec < nvec) {
-    const uint4* p = x + vec;
-    int64_t r = r0 + phase;
-    for (; r + (int64_t)(kUnroll - 1) * kPhases < r1; r += (int64_t)kUnroll * kPhases) {
-      uint4 q[kUnroll];
-#pragma unroll
-      for (int u = 0; u < kUnroll; ++u) q[u] = ld_stream_v4(p + (r + (int64_t)u * kPhases) * ld_vec);
-#pragma unroll
-      for (int u = 0; u < kUnroll; ++u) accum_sq8(acc, q[u]);
+  int waited = 0;  // tid 0: stages whose full barrier it has seen complete
+  for (int i = 0; i < nst; ++i) {
+    const int s = i % kStages;
+    const uint32_t par = (uint32_t)(i / kStages) & 1u;
+    bool ok = !*(volatile int*)&s_bad;
+    if (ok && !mbar_wait(&full_bar[s], par)) {
+      ok = false;
+      s_bad = 1;
     }
-    for (; r < r1; r += kPhases) accum_sq8(acc, ld_stream_v4(p + r * ld_vec));
+    if (ok) {
+      if (tid == 0) waited = i + 1;
+      const uint8_t* st = ring + (size_t)s * kStageBytes + p * 128 + v * 16;
+#pragma unroll
+      for (int rr = 0; rr < kStageRows / kPhases; ++rr)
+        accum_sq8(acc, *reinterpret_cast<const uint4*>(st + rr * kPhases * 128));
+    }
+    __syncwarp();
+    if (lane == 0) mbar_arrive(&empty_bar[s]);
+    if (tid == 0 && issued < nst && issued == i + kStages) {
+      if (!*(volatile int*)&s_bad && mbar_wait(&empty_bar[s], par)) {
+        mbar_arrive_expect_tx(&full_bar[s], kStageBytes);
+        tma_load_2d(ring + (size_t)s * kStageBytes, &xmap, x0, (int32_t)(r0 + issued * kStageRows),
+                    &full_bar[s], policy);
+        ++issued;
+      } else {
+        s_bad = 1;
+      }
+    }
+  }
+  if (tid == 0 && s_bad) {
+    // let copies still in flight land before the CTA's shared memory goes away
+    for (int j = waited; j < issued; ++j) mbar_wait(&full_bar[j % kStages], (uint32_t)(j / kStages) & 1u);
+    atomicOr(&g_device_error, kErrMbarTimeout);
   }
 
   // phases 4w..4w+3 of a warp: lane bit 3 is phase bit 0, lane bit 4 is phase bit 1
@@ -87,8 +155,7 @@ hessian_colsumsq_kernel(const uint4* __restrict__ x, int64_t tokens, int64_t ld_
     t = __fadd_rn(t, __shfl_xor_sync(0xFFFFFFFFu, t, 16));
     acc[k] = t;
   }
-  const int lane = tid & 31, warp = tid >> 5;
-  if (lane < kVecPerRow) {
+  if (lane < 8) {
 #pragma unroll
     for (int k = 0; k < 8; ++k) warp_part[warp][lane * 8 + k] = acc[k];
   }
@@ -101,13 +168,14 @@ hessian_colsumsq_kernel(const uint4* __restrict__ x, int64_t tokens, int64_t ld_
     for (int step = 1; step < kWarps; step <<= 1)
 #pragma unroll
       for (int w = 0; w + step < kWarps; w += 2 * step) s[w] = __fadd_rn(s[w], s[w + step]);
-    cta_part[tid] = s[0];
+    cta_part[tid] = s_bad ? __int_as_float(0x7FC00000) : s[0];
   }
 
+  pdl_wait_primary();  // the previous chunk's kernel has finished writing h
   if constexpr (CS == 1) {
     __syncthreads();
     if (tid < kTileCols) {
-      const int col = blockIdx.y * kTileCols + tid;
+      const int col = x0 + tid;
       if (col < n) h[col] = __fadd_rn(h[col], cta_part[tid]);
     }
   } else {
@@ -120,35 +188,65 @@ hessian_colsumsq_kernel(const uint4* __restrict__ x, int64_t tokens, int64_t ld_
       for (int step = 1; step < CS; step <<= 1)
 #pragma unroll
         for (int r = 0; r + step < CS; r += 2 * step) s[r] = __fadd_rn(s[r], s[r + step]);
-      const int col = blockIdx.y * kTileCols + tid;
+      const int col = x0 + tid;
       if (col < n) h[col] = __fadd_rn(h[col], s[0]);
     }
     cluster.sync();  // keep every CTA's shared memory alive until rank 0 has read it
   }
 }
 
+// ---------------------------------------------------------------- host side
+using EncodeTiledFn = CUresult (*)(CUtensorMap*, CUtensorMapDataType, cuuint32_t, void*,
+                                   const cuuint64_t*, const cuuint64_t*, const cuuint32_t*,
+                                   const cuuint32_t*, CUtensorMapInterleave, CUtensorMapSwizzle,
+                                   CUtensorMapL2promotion, CUtensorMapFloatOOBfill);
+
+cudaError_t encode_tiled_fn(EncodeTiledFn* out) {
+  static std::once_flag once;
+  static EncodeTiledFn fn = nullptr;
+  static cudaError_t status = cudaSuccess;
+  std::call_once(once, [] {
+    void* p = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    status = cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &p, 12000, cudaEnableDefault, &q);
+    if (status == cudaSuccess && q != cudaDriverEntryPointSuccess) status = cudaErrorNotSupported;
+    fn = reinterpret_cast<EncodeTiledFn>(p);
+  });
+  *out = fn;
+  return status;
+}
+
 template <int CS>
-cudaError_t launch_cs(const uint4* x, int64_t tokens, int64_t ld_vec, int nvec, int n, float* h,
-                      int tiles, cudaStream_t stream) {
-  const int64_t max_rows_per_cta = kMaxRunPerThread * kPhases;
-  const int64_t rows_per_launch = max_rows_per_cta * CS;
+cudaError_t launch_cs(const CUtensorMap& map, int64_t tokens, int n, float* h, int tiles,
+                      cudaStream_t stream) {
+  static std::once_flag once;
+  static cudaError_t attr_status = cudaSuccess;
+  std::call_once(once, [] {
+    attr_status = cudaFuncSetAttribute(hessian_colsumsq_kernel<CS>,
+                                       cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kRingBytes);
+  });
+  if (attr_status != cudaSuccess) return attr_status;
+  const int64_t rows_per_launch = kMaxRowsPerCta * CS;
   for (int64_t t0 = 0; t0 < tokens; t0 += rows_per_launch) {
-    const int64_t t = min(tokens - t0, rows_per_launch);
+    const int64_t t = std::min(tokens - t0, rows_per_launch);
     int64_t rows_per_cta = (t + CS - 1) / CS;
+    rows_per_cta = (rows_per_cta + kStageRows - 1) / kStageRows * kStageRows;
     cudaLaunchConfig_t cfg = {};
     cfg.gridDim = dim3(CS, tiles, 1);
     cfg.blockDim = dim3(kThreads, 1, 1);
-    cfg.dynamicSmemBytes = 0;
+    cfg.dynamicSmemBytes = kRingBytes;
     cfg.stream = stream;
-    cudaLaunchAttribute attr[1];
+    cudaLaunchAttribute attr[2];
     attr[0].id = cudaLaunchAttributeClusterDimension;
     attr[0].val.clusterDim.x = CS;
     attr[0].val.clusterDim.y = 1;
     attr[0].val.clusterDim.z = 1;
+    attr[1].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[1].val.programmaticStreamSerializationAllowed = 1;
     cfg.attrs = attr;
-    cfg.numAttrs = 1;
-    cudaError_t err = cudaLaunchKernelEx(&cfg, hessian_colsumsq_kernel<CS>, x + t0 * ld_vec, t,
-                                         ld_vec, nvec, n, h, rows_per_cta);
+    cfg.numAttrs = 2;
+    cudaError_t err = cudaLaunchKernelEx(&cfg, hessian_colsumsq_kernel<CS>, map, t0, t, n, h,
+                                         rows_per_cta);
     if (err != cudaSuccess) return err;
   }
   return cudaGetLastError();
@@ -161,21 +259,44 @@ cudaError_t launch_hessian(const void* x, int64_t tokens, int64_t n, int64_t ld_
   DeviceInfo info;
   cudaError_t err = current_device_info(&info);
   if (err != cudaSuccess) return err;
-  const int nvec = (int)(n / 8);
-  const int tiles = (nvec + kVecPerRow - 1) / kVecPerRow;
-  // about one wave: 256-thread CTAs, 4 resident per SM
+  EncodeTiledFn encode = nullptr;
+  err = encode_tiled_fn(&encode);
+  if (err != cudaSuccess) return err;
+
+  CUtensorMap map;
+  const cuuint64_t dims[2] = {(cuuint64_t)n, (cuuint64_t)tokens};
+  const cuuint64_t strides[1] = {(cuuint64_t)ld_x * 2};
+  const cuuint32_t box[2] = {(cuuint32_t)kTileCols, (cuuint32_t)kStageRows};
+  const cuuint32_t estr[2] = {1, 1};
+  CUresult r = encode(&map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(x), dims, strides,
+                      box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_NONE,
+                      CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+  if (r != CUDA_SUCCESS) return cudaErrorInvalidValue;
+
+  const int tiles = (int)((n + kTileCols - 1) / kTileCols);
+  // about one wave: 4 resident CTAs per SM
   const int64_t target = (int64_t)info.sm_count * 4;
   int cs = 1;
-  while (cs < kMaxCluster && (int64_t)tiles * cs * 2 <= target && (int64_t)cs * 2 * kPhases * 4 <= tokens)
+  while (cs < kMaxCluster && (int64_t)tiles * cs * 2 <= target && (int64_t)cs * 2 * kStageRows * 4 <= tokens)
     cs *= 2;
-  const uint4* xv = static_cast<const uint4*>(x);
-  const int64_t ld_vec = ld_x / 8;
   switch (cs) {
-    case 1: return launch_cs<1>(xv, tokens, ld_vec, nvec, (int)n, h, tiles, stream);
-    case 2: return launch_cs<2>(xv, tokens, ld_vec, nvec, (int)n, h, tiles, stream);
-    case 4: return launch_cs<4>(xv, tokens, ld_vec, nvec, (int)n, h, tiles, stream);
-    default: return launch_cs<8>(xv, tokens, ld_vec, nvec, (int)n, h, tiles, stream);
+    case 1: return launch_cs<1>(map, tokens, (int)n, h, tiles, stream);
+    case 2: return launch_cs<2>(map, tokens, (int)n, h, tiles, stream);
+    case 4: return launch_cs<4>(map, tokens, (int)n, h, tiles, stream);
+    default: return launch_cs<8>(map, tokens, (int)n, h, tiles, stream);
   }
+}
+
+cudaError_t read_and_clear_device_error(uint32_t* flags) {
+  uint32_t v = 0;
+  cudaError_t err = cudaMemcpyFromSymbol(&v, g_device_error, sizeof v);
+  if (err != cudaSuccess) return err;
+  *flags = v;
+  if (v) {
+    const uint32_t zero = 0;
+    err = cudaMemcpyToSymbol(g_device_error, &zero, sizeof zero);
+  }
+  return err;
 }
 
 }  // namespace hscale

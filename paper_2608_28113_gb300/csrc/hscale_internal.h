@@ -29,6 +29,9 @@ cudaError_t launch_refine(const void* w, const float* h, int64_t m, int64_t n,
                           const float* global_scale, const uint8_t* init_codes, int down, int up,
                           uint8_t* codes_out, uint8_t* packed_out, cudaStream_t stream);
 
+// Sticky device error flags of this library (bit 0: a bounded wait ran out); cleared on read.
+cudaError_t read_and_clear_device_error(uint32_t* flags);
+
 cudaError_t launch_pack(const void* w, int64_t m, int64_t n, const float* global_scale,
                         const uint8_t* codes, uint8_t* packed_out, cudaStream_t stream);
 

@@ -94,7 +94,7 @@ __global__ void __launch_bounds__(256) rtn_codes_kernel(const uint4* __restrict_
 // ---------------------------------------------------------------- search helpers
 struct Group {
   uint32_t wb[8];  // raw bf16 pairs (element 2i in the low half of wb[i])
-  float a[16];     // |w| * 2^-K
+  float2 a[8];     // |w| * 2^-K, elements (2i, 2i+1)
 };
 
 __device__ __forceinline__ void load_group(const uint4* w, int64_t g, float pw, Group& G) {
@@ -103,10 +103,76 @@ __device__ __forceinline__ void load_group(const uint4* w, int64_t g, float pw, 
   G.wb[0] = p.x; G.wb[1] = p.y; G.wb[2] = p.z; G.wb[3] = p.w;
   G.wb[4] = q.x; G.wb[5] = q.y; G.wb[6] = q.z; G.wb[7] = q.w;
 #pragma unroll
+  for (int i = 0; i < 8; ++i)
+    G.a[i] = make_float2(__fmul_rn(fabsf(bf16_lo(G.wb[i])), pw), __fmul_rn(fabsf(bf16_hi(G.wb[i])), pw));
+}
+
+// Per-block table of the candidate constants of every E4M3 code c (1..126), filled once
+// per CTA: x = -(s' * 2^126) and y = 2^-126 / s' (fast reciprocal), with s' = l(c) * sgk.
+// Reading it costs one shared load per candidate instead of a decode, two multiplies and
+// a reciprocal on the candidate's critical path.
+__device__ __forceinline__ float2 candidate_constants(uint32_t c, float sgk) {
+  const float sp = __fmul_rn(e4m3_mag(c), sgk);
+  return make_float2(-__fmul_rn(sp, 0x1p126f), c ? inv_raw_of(sp) : 0.0f);
+}
+
+// Fast score of one candidate from its table entry (see the file comment): per pair of
+// elements one packed multiply for the quotients, integer rounding of each raw pattern
+// (plus the saturation when SAT), one packed FMA for the residuals, a packed square and a
+// packed FMA into the h-weighted sum.
+template <bool SAT>
+__device__ __forceinline__ float fast_score(const Group& G, const float2 (&hv2)[8], float2 t) {
+  const float2 inv2 = make_float2(t.y, t.y);
+  const float2 nS2 = make_float2(t.x, t.x);
+  float2 acc0 = make_float2(0.f, 0.f), acc1 = make_float2(0.f, 0.f);
+#pragma unroll
   for (int i = 0; i < 8; ++i) {
-    G.a[2 * i] = __fmul_rn(fabsf(bf16_lo(G.wb[i])), pw);
-    G.a[2 * i + 1] = __fmul_rn(fabsf(bf16_hi(G.wb[i])), pw);
+    const float2 y = __fmul2_rn(G.a[i], inv2);
+    uint32_t q0 = (__float_as_uint(y.x) + kE2M1Half) & kE2M1Keep;
+    uint32_t q1 = (__float_as_uint(y.y) + kE2M1Half) & kE2M1Keep;
+    if (SAT) {
+      q0 = min(q0, kE2M1SixRaw);
+      q1 = min(q1, kE2M1SixRaw);
+    }
+    const float2 r = __ffma2_rn(make_float2(__uint_as_float(q0), __uint_as_float(q1)), nS2, G.a[i]);
+    const float2 rr = __fmul2_rn(r, r);
+    if (i & 1) acc1 = __ffma2_rn(hv2[i], rr, acc1);
+    else acc0 = __ffma2_rn(hv2[i], rr, acc0);
   }
+  const float2 t2 = __fadd2_rn(acc0, acc1);
+  return __fadd_rn(t2.x, t2.y);
+}
+
+__device__ __forceinline__ void keep_best(float e, int c, float& e1, float& e2, int& best) {
+  if (e < e1) { e2 = e1; e1 = e; best = c; }
+  else if (e < e2) { e2 = e; }
+}
+
+// Scores the codes [a, b) two at a time (independent chains interleave).
+template <bool SAT>
+__device__ __forceinline__ void score_range(const Group& G, const float2 (&hv2)[8],
+                                            const float2* tab, int a, int b, float& e1, float& e2,
+                                            int& best) {
+  int c = a;
+  for (; c + 1 < b; c += 2) {
+    const float2 t0 = tab[c], t1 = tab[c + 1];
+    const float ea = fast_score<SAT>(G, hv2, t0);
+    const float eb = fast_score<SAT>(G, hv2, t1);
+    keep_best(ea, c, e1, e2, best);
+    keep_best(eb, c + 1, e1, e2, best);
+  }
+  if (c < b) keep_best(fast_score<SAT>(G, hv2, tab[c]), c, e1, e2, best);
+}
+
+// True when some quotient of the group under code c rounds to 7 or more in the fast
+// path, i.e. when candidates from c upwards still need the E2M1 saturation.  The test
+// uses the same fp32 product as the fast path on the group's largest magnitude, and
+// quotients only shrink as the code grows, so it is exact for every code >= c.
+__device__ __forceinline__ bool needs_saturation_from(const Group& G, float2 t) {
+  float amax = 0.f;
+#pragma unroll
+  for (int i = 0; i < 8; ++i) amax = fmaxf(amax, fmaxf(G.a[i].x, G.a[i].y));
+  return __fmul_rn(amax, t.y) >= 7.0f * 0x1p-126f;
 }
 
 // tie rule of the search: smaller error, then smaller |shift|, then smaller shift
@@ -157,18 +223,54 @@ __device__ int warp_exact_search(int owner, const uint4* w, int64_t g_own, const
   return bc;
 }
 
-// Exact final re-quantization of one group under code c: 8 bytes of packed nibbles.
-__device__ __forceinline__ uint2 quantize_pack(const Group& G, uint32_t c, float sgk) {
-  const float l = e4m3_mag(c);
-  const float inv = inv_raw_of(__fmul_rn(l, sgk));
-  uint32_t out[2] = {0u, 0u};
+// Hardware E2M1 conversion of two fp32 values (round-to-nearest-even, saturating at
+// +-6, sign kept, also for a result of zero): one byte, `hi` in the upper nibble.
+__device__ __forceinline__ uint32_t cvt_e2m1x2(float hi, float lo) {
+  uint32_t r;
+  asm("{\n\t.reg .b8 t;\n\tcvt.rn.satfinite.e2m1x2.f32 t, %1, %2;\n\tcvt.u32.u8 %0, t;\n\t}"
+      : "=r"(r)
+      : "f"(hi), "f"(lo));
+  return r;
+}
+
+// Exact final re-quantization of one group under code c (table entry t): 8 bytes of
+// packed nibbles.  The raw-domain quotients y_raw = |w| * 2^-126 / s' are rescaled
+// exactly to real units, given the sign of w, and converted by the hardware E2M1
+// conversion (round-to-nearest-even).  That equals the exact rounding of |w| / s unless
+// some y_raw lies within 16 ulps of a midpoint; then every element is redone with the
+// exact midpoint test.
+__device__ __forceinline__ uint2 quantize_pack(const Group& G, uint32_t c, float2 t, float sgk) {
+  const float2 ir2 = make_float2(t.y, t.y);
+  const float2 up2 = make_float2(0x1p126f, 0x1p126f);
+  uint32_t word[2] = {0u, 0u};
+  uint32_t near = 0xFFFFFFFFu;
 #pragma unroll
-  for (int j = 0; j < 16; ++j) {
-    const uint32_t k = e2m1_code(G.a[j], inv, l, sgk);
-    const uint32_t sign = (j & 1) ? (G.wb[j >> 1] >> 31) : ((G.wb[j >> 1] >> 15) & 1u);
-    out[j >> 3] |= ((sign << 3) | k) << (4 * (j & 7));
+  for (int i = 0; i < 8; ++i) {
+    const float2 yr = __fmul2_rn(G.a[i], ir2);
+    near = min(near, (__float_as_uint(yr.x) - 0x1FFFF0u) & 0x3FFFFFu);
+    near = min(near, (__float_as_uint(yr.y) - 0x1FFFF0u) & 0x3FFFFFu);
+    const float2 yv = __fmul2_rn(yr, up2);
+    const float y0 = __uint_as_float(__float_as_uint(yv.x) | ((G.wb[i] << 16) & 0x80000000u));
+    const float y1 = __uint_as_float(__float_as_uint(yv.y) | (G.wb[i] & 0x80000000u));
+    word[i >> 2] |= cvt_e2m1x2(y1, y0) << (8 * (i & 3));
   }
-  return make_uint2(out[0], out[1]);
+  if (near <= 0x20u) {
+    // rare: redo only the flagged elements with the exact midpoint test (static indices
+    // keep the group in registers)
+    const float l = e4m3_mag(c);
+#pragma unroll
+    for (int j = 0; j < 16; ++j) {
+      const float a = (j & 1) ? G.a[j >> 1].y : G.a[j >> 1].x;
+      const float y = __fmul_rn(a, t.y);
+      if (e2m1_uncertain(y)) {
+        const uint32_t k = e2m1_exact_code(y, a, l, sgk);
+        const uint32_t sign = (j & 1) ? (G.wb[j >> 1] >> 31) : ((G.wb[j >> 1] >> 15) & 1u);
+        const int sh = 4 * (j & 7);
+        word[j >> 3] = (word[j >> 3] & ~(0xFu << sh)) | (((sign << 3) | k) << sh);
+      }
+    }
+  }
+  return make_uint2(word[0], word[1]);
 }
 
 // ---------------------------------------------------------------- refine (Algorithm 1)
@@ -185,14 +287,17 @@ refine_kernel(const uint4* __restrict__ w, const float* __restrict__ h, int64_t 
   const int chunks = (ng + 31) / 32;
   const int64_t units = m * chunks;
 
+  __shared__ float2 tab[128];
   const ScaleDomain d = make_scale_domain(*global_scale);
   const float inv6 = rtn_inv6_raw(d.sgk);
+  for (int c = threadIdx.x; c < 128; c += blockDim.x) tab[c] = candidate_constants((uint32_t)c, d.sgk);
+  __syncthreads();
 
   int cur_chunk = -1;
-  float hv[16];
+  float2 hv2[8];
   float H = 0.0f;
 #pragma unroll
-  for (int j = 0; j < 16; ++j) hv[j] = 1.0f;
+  for (int j = 0; j < 8; ++j) hv2[j] = make_float2(1.0f, 1.0f);
 
   for (int64_t u = warp_global; u < units; u += warps_total) {
     const int64_t row = u / chunks;
@@ -209,11 +314,12 @@ refine_kernel(const uint4* __restrict__ w, const float* __restrict__ h, int64_t 
 #pragma unroll
         for (int i = 0; i < 4; ++i) {
           const float4 t = hp[i];
-          hv[4 * i] = t.x; hv[4 * i + 1] = t.y; hv[4 * i + 2] = t.z; hv[4 * i + 3] = t.w;
+          hv2[2 * i] = make_float2(t.x, t.y);
+          hv2[2 * i + 1] = make_float2(t.z, t.w);
         }
       }
 #pragma unroll
-      for (int j = 0; j < 16; ++j) H = __fadd_rn(H, hv[j]);
+      for (int j = 0; j < 8; ++j) H = __fadd_rn(H, __fadd_rn(hv2[j].x, hv2[j].y));
     }
 
     Group G;
@@ -232,41 +338,17 @@ refine_kernel(const uint4* __restrict__ w, const float* __restrict__ h, int64_t 
       hi = min((int)kE4M3MaxCode, c0 + up);
     }
 
-    // ---- fast scores of every distinct candidate
+    // ---- fast scores of every distinct candidate.  Codes below c0 run with the E2M1
+    // saturation; codes from c0 up skip it unless some lane of the warp needs it there
+    // (never for an RTN start on a normal E4M3 code, whose quotients stay below 6.375).
+    // Splitting every lane at its own c0 keeps the loop trip counts uniform in the warp.
     float e1 = kInf, e2 = kInf;
     int best = c0;
+    const bool sat_hi = __any_sync(0xFFFFFFFFu, active && needs_saturation_from(G, tab[c0]));
     if (active) {
-      for (int c = lo; c <= hi; ++c) {
-        const float l = e4m3_mag((uint32_t)c);
-        const float sp = __fmul_rn(l, d.sgk);
-        const float S = __fmul_rn(sp, 0x1p126f);
-        const float inv = inv_raw_of(sp);
-        float acc0 = 0.f, acc1 = 0.f, acc2 = 0.f, acc3 = 0.f;
-#pragma unroll
-        for (int j = 0; j < 16; j += 4) {
-          float y, r;
-          uint32_t q;
-          y = __fmul_rn(G.a[j], inv);
-          q = min((__float_as_uint(y) + kE2M1Half) & kE2M1Keep, kE2M1SixRaw);
-          r = __fmaf_rn(-__uint_as_float(q), S, G.a[j]);
-          acc0 = __fmaf_rn(hv[j], __fmul_rn(r, r), acc0);
-          y = __fmul_rn(G.a[j + 1], inv);
-          q = min((__float_as_uint(y) + kE2M1Half) & kE2M1Keep, kE2M1SixRaw);
-          r = __fmaf_rn(-__uint_as_float(q), S, G.a[j + 1]);
-          acc1 = __fmaf_rn(hv[j + 1], __fmul_rn(r, r), acc1);
-          y = __fmul_rn(G.a[j + 2], inv);
-          q = min((__float_as_uint(y) + kE2M1Half) & kE2M1Keep, kE2M1SixRaw);
-          r = __fmaf_rn(-__uint_as_float(q), S, G.a[j + 2]);
-          acc2 = __fmaf_rn(hv[j + 2], __fmul_rn(r, r), acc2);
-          y = __fmul_rn(G.a[j + 3], inv);
-          q = min((__float_as_uint(y) + kE2M1Half) & kE2M1Keep, kE2M1SixRaw);
-          r = __fmaf_rn(-__uint_as_float(q), S, G.a[j + 3]);
-          acc3 = __fmaf_rn(hv[j + 3], __fmul_rn(r, r), acc3);
-        }
-        const float e = __fadd_rn(__fadd_rn(acc0, acc1), __fadd_rn(acc2, acc3));
-        if (e < e1) { e2 = e1; e1 = e; best = c; }
-        else if (e < e2) { e2 = e; }
-      }
+      score_range<true>(G, hv2, tab, lo, c0, e1, e2, best);
+      if (sat_hi) score_range<true>(G, hv2, tab, c0, hi + 1, e1, e2, best);
+      else score_range<false>(G, hv2, tab, c0, hi + 1, e1, e2, best);
     }
 
     // ---- is the fast winner certain?
@@ -292,7 +374,7 @@ refine_kernel(const uint4* __restrict__ w, const float* __restrict__ h, int64_t 
 
     if (active) {
       codes_out[g] = (uint8_t)best;
-      if (packed_out != nullptr) packed_out[g] = quantize_pack(G, (uint32_t)best, d.sgk);
+      if (packed_out != nullptr) packed_out[g] = quantize_pack(G, (uint32_t)best, tab[best], d.sgk);
     }
   }
 }
@@ -309,17 +391,25 @@ __global__ void __launch_bounds__(256) pack_kernel(const uint4* __restrict__ w, 
     load_group(w, g, d.pw, G);
     uint32_t c = codes[g] & 0x7Fu;
     c = c < 1 ? 1u : (c > kE4M3MaxCode ? kE4M3MaxCode : c);
-    packed_out[g] = quantize_pack(G, c, d.sgk);
+    packed_out[g] = quantize_pack(G, c, candidate_constants(c, d.sgk), d.sgk);
   }
 }
 
+// Resident CTAs per SM of a kernel, queried once per kernel and device (the query is
+// not repeated under stream capture).
 template <typename K>
 int occupancy_blocks(K kernel, int threads) {
-  int blocks = 0;
-  if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&blocks, kernel, threads, 0) != cudaSuccess ||
-      blocks < 1)
-    blocks = 1;
-  return blocks;
+  static int cache[64] = {0};
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) dev = 0;
+  if (cache[dev] == 0) {
+    int blocks = 0;
+    if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&blocks, kernel, threads, 0) != cudaSuccess ||
+        blocks < 1)
+      blocks = 1;
+    cache[dev] = blocks;
+  }
+  return cache[dev];
 }
 
 }  // namespace
