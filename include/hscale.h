@@ -120,6 +120,30 @@ int hscale_rtn_scales(const void* w_bf16, int64_t m, int64_t n, float* global_sc
                       uint8_t* codes, void* workspace, size_t workspace_bytes, void* stream);
 
 /*
+ * hscale_rtn_scales without a workspace and without any allocation.  (The paper has no
+ * counterpart: this is a convenience of the library.)
+ *
+ * Same inputs, outputs and results as hscale_rtn_scales, for callers that cannot
+ * allocate device memory, such as a plugin or callback that is handed only its input and
+ * output tensors, or a service whose device memory belongs to a framework pool it cannot
+ * reach.  The call allocates nothing (no cudaMalloc, no cudaFree, no allocating library
+ * routine); its scratch is a fixed array of HSCALE_NOALLOC_SCRATCH_BYTES bytes compiled
+ * into the library, which every GPU that loads the library holds until the process exits.
+ *
+ * - The first call on each device looks up that array's device address (a synchronous
+ *   runtime query) and caches it; make that first call before any stream capture.
+ * - Every call on a device shares the array: each call clears the part it uses on its
+ *   stream before use, and calls whose work overlaps on the GPU (different streams,
+ *   different threads) race with each other.  Serialise them.
+ * - The scratch this work needs does not grow with m or n, so no input size is refused
+ *   for lack of scratch; HSCALE_ERR_WORKSPACE would mean the work needs more than
+ *   HSCALE_NOALLOC_SCRATCH_BYTES.
+ */
+#define HSCALE_NOALLOC_SCRATCH_BYTES 256
+int hscale_rtn_scales_noalloc(const void* w_bf16, int64_t m, int64_t n, float* global_scale,
+                              uint8_t* codes, void* stream);
+
+/*
  * H-Scale refinement, Algorithm 1 (Eqs. 6-13), fused with the final re-quantization.
  *
  * For every group with initial code c (init_codes[g] with its sign bit cleared and

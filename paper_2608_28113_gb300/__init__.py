@@ -24,6 +24,7 @@ __all__ = [
     "HScaleError", "load", "library_path", "hscale_status_string", "hscale_abi_version",
     "hscale_device_error_flags",
     "hscale_hessian_diag_accumulate", "hscale_rtn_workspace_bytes", "hscale_rtn_scales",
+    "hscale_rtn_scales_noalloc",
     "hscale_refine_scales", "hscale_pack_nvfp4", "EXPORTED_SYMBOLS",
 ]
 
@@ -41,6 +42,7 @@ _SIGNATURES = {
     "hscale_hessian_diag_accumulate": (ctypes.c_int, [_P, _I64, _I64, _I64, _P, _P]),
     "hscale_rtn_workspace_bytes": (_SZ, []),
     "hscale_rtn_scales": (ctypes.c_int, [_P, _I64, _I64, _P, _P, _P, _SZ, _P]),
+    "hscale_rtn_scales_noalloc": (ctypes.c_int, [_P, _I64, _I64, _P, _P, _P]),
     "hscale_refine_scales": (ctypes.c_int, [_P, _P, _I64, _I64, _P, _P, _I32, _I32, _P, _P, _P]),
     "hscale_pack_nvfp4": (ctypes.c_int, [_P, _I64, _I64, _P, _P, _P, _P]),
 }
@@ -150,6 +152,24 @@ def hscale_rtn_scales(w: torch.Tensor, global_scale: torch.Tensor, codes: torch.
     _check("hscale_rtn_scales",
            load().hscale_rtn_scales(_ptr(w), m, n, _ptr(global_scale), _ptr(codes),
                                     _ptr(workspace), nbytes, _stream_ptr(stream)))
+
+
+def hscale_rtn_scales_noalloc(w: torch.Tensor, global_scale: torch.Tensor,
+                              codes: torch.Tensor | None, stream=None) -> None:
+    """hscale_rtn_scales for callers that cannot allocate: no workspace argument; the
+    library's fixed per-GPU scratch array is used instead (calls must not overlap)."""
+    _need(w, torch.bfloat16, "w")
+    _need(global_scale, torch.float32, "global_scale")
+    if not w.is_contiguous() or w.dim() != 2:
+        raise ValueError("w must be a contiguous 2-D tensor")
+    m, n = w.shape
+    if codes is not None:
+        _need(codes, torch.uint8, "codes")
+        if codes.numel() != m * (n // 16) or not codes.is_contiguous():
+            raise ValueError("codes must be contiguous [m, n/16]")
+    _check("hscale_rtn_scales_noalloc",
+           load().hscale_rtn_scales_noalloc(_ptr(w), m, n, _ptr(global_scale), _ptr(codes),
+                                            _stream_ptr(stream)))
 
 
 def hscale_refine_scales(w: torch.Tensor, h: torch.Tensor | None, global_scale: torch.Tensor,

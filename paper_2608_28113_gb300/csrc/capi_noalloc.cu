@@ -1,0 +1,70 @@
+// capi_noalloc.cu -- hscale_rtn_scales_noalloc: the global scale and RTN codes without a
+// caller-supplied workspace and without any allocation.
+//
+// Some callers of this library cannot allocate device memory: a plugin or callback that
+// is handed only its input and output tensors by a host framework, or a service whose
+// device memory is owned by a framework pool it has no handle to.  They cannot provide
+// the small workspace hscale_rtn_scales needs for its amax word.  This entry point keeps
+// that word in a fixed array of this file that lives in every GPU's memory from the
+// moment the library is loaded there until the process exits.
+#include <cuda_runtime.h>
+
+#include <cstdint>
+#include <mutex>
+
+#include "../../include/hscale.h"
+#include "hscale_internal.h"
+
+namespace {
+
+// The fixed scratch of hscale_rtn_scales_noalloc (HSCALE_NOALLOC_SCRATCH_BYTES bytes per
+// GPU).  Host code must not pass this name to a kernel: on the host it is only a stand-in
+// for the symbol, so its device address is looked up once per device below.
+static __device__ __align__(256) uint8_t g_noalloc_scratch[HSCALE_NOALLOC_SCRATCH_BYTES];
+
+constexpr int kMaxDevices = 64;
+
+// Device address of g_noalloc_scratch on the current device, resolved on the first call
+// for that device (with that device current) and cached.
+cudaError_t scratch_address(uint32_t** out) {
+  static std::mutex mu;
+  static void* addr[kMaxDevices] = {nullptr};
+  int dev = 0;
+  cudaError_t err = cudaGetDevice(&dev);
+  if (err != cudaSuccess) return err;
+  if (dev < 0 || dev >= kMaxDevices) return cudaErrorInvalidDevice;
+  std::lock_guard<std::mutex> lock(mu);
+  if (addr[dev] == nullptr) {
+    void* p = nullptr;
+    err = cudaGetSymbolAddress(&p, g_noalloc_scratch);
+    if (err != cudaSuccess) return err;
+    if (p == nullptr) return cudaErrorInvalidSymbol;
+    addr[dev] = p;
+  }
+  *out = static_cast<uint32_t*>(addr[dev]);
+  return cudaSuccess;
+}
+
+}  // namespace
+
+extern "C" int hscale_rtn_scales_noalloc(const void* w_bf16, int64_t m, int64_t n,
+                                         float* global_scale, uint8_t* codes, void* stream) {
+  if (m < 0 || n < 0 || n % 16 != 0) return HSCALE_ERR_SHAPE;
+  if (m > 0 && n > 0 && (m > INT64_MAX / n || n / 16 > INT32_MAX)) return HSCALE_ERR_SHAPE;
+  if (m == 0 || n == 0) return HSCALE_OK;
+  if (w_bf16 == nullptr || global_scale == nullptr) return HSCALE_ERR_NULL;
+  if ((reinterpret_cast<uintptr_t>(w_bf16) & 15) != 0) return HSCALE_ERR_ALIGN;
+  if ((reinterpret_cast<uintptr_t>(global_scale) & 3) != 0) return HSCALE_ERR_ALIGN;
+  // the work needs hscale_rtn_workspace_bytes() of scratch, which does not depend on m or n;
+  // refuse if it ever outgrows the fixed array
+  if (hscale_rtn_workspace_bytes() > (size_t)HSCALE_NOALLOC_SCRATCH_BYTES) return HSCALE_ERR_WORKSPACE;
+  uint32_t* amax = nullptr;
+  if (scratch_address(&amax) != cudaSuccess) return HSCALE_ERR_CUDA;
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  // the amax word keeps the previous call's value: clear it first
+  if (cudaMemsetAsync(amax, 0, sizeof(uint32_t), s) != cudaSuccess) return HSCALE_ERR_CUDA;
+  if (hscale::launch_amax(w_bf16, m * n, amax, s) != cudaSuccess) return HSCALE_ERR_CUDA;
+  return hscale::launch_rtn_codes(w_bf16, m, n, amax, global_scale, codes, s) == cudaSuccess
+             ? HSCALE_OK
+             : HSCALE_ERR_CUDA;
+}
