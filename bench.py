@@ -175,6 +175,25 @@ class ClockSampler:
                 "samples": len(self.samples), "source": "nvml" if self._nvml else "none"}
 
 
+def profiled_traffic(workload: str, chunk: int, n: int):
+    """DRAM bytes per Hessian launch from the committed ncu summary, if the kernel's sources
+    are unchanged since that capture and the launch shape matches; else None."""
+    import hashlib
+    path = os.path.join(ROOT, "profiles", f"hessian_colsumsq_{workload}.traffic.json")
+    try:
+        with open(path) as f:
+            d = json.load(f)
+        h = hashlib.sha256()
+        for src in d["kernel_sources"]:
+            with open(os.path.join(ROOT, src), "rb") as f:
+                h.update(f.read())
+        if h.hexdigest() != d["kernel_sources_sha256"] or d["chunk_tokens"] != chunk or d["n"] != n:
+            return None
+        return int(d["dram_bytes_per_launch"])
+    except Exception:
+        return None
+
+
 # ------------------------------------------------------------------ workload
 class Layer:
     """Device-resident inputs and outputs of one layer of a workload."""
@@ -429,7 +448,8 @@ def gpu_arm(args, d: Dist):
         "roofline": {"bound": "hbm", "kernel": "hessian_colsumsq", "achieved": h_gbs,
                      "peak": hbm_peak, "unit": "GB/s", "frac": h_gbs / hbm_peak,
                      "peak_kind": f"{peak_kind} HBM copy bandwidth",
-                     "frac_of_8TBs_spec": h_gbs / HBM_SPEC_GBS, "traffic": None,
+                     "frac_of_8TBs_spec": h_gbs / HBM_SPEC_GBS,
+                     "traffic": profiled_traffic(W.name, L.chunk, L.n),
                      "bytes_per_launch": h_bytes_launch, "ms_per_launch": ms_h_launch},
         "phases_ms": {"hessian": ms_h, "scales": ms_sc, "rtn_scales": ms_rtn, "refine": ms_ref},
         "ms_per_step_eager": ms_eager,

@@ -5,12 +5,12 @@
 // Layout of the work
 //   * A CTA owns a 64-channel column tile (128 bytes of every row) and a contiguous
 //     run of tokens.  One thread streams the run into a ring of shared-memory stages
-//     with 2-D TMA tensor loads (64 channels x 64 rows = 8 KB per stage, 6 stages in
+//     with 2-D TMA tensor loads (64 channels x 128 rows = 16 KB per stage, 3 stages in
 //     flight per CTA, L2 evict-first); the CTA's 256 threads (32 row phases x 8
 //     16-byte vectors) read each stage back with conflict-free 128-bit shared loads
 //     and accumulate in fp32.  mbarriers order the ring; every wait is bounded.
 //   * The token range of a tile is split over the CTAs of one thread-block cluster
-//     (1, 2, 4 or 8 CTAs, so the grid is about one wave of resident CTAs).  The CTAs
+//     (1, 2, 4 or 8 CTAs, so a launch holds about two CTAs per SM).  The CTAs
 //     of a cluster reduce their partial sums through distributed shared memory: the
 //     kernel needs no global scratch, no atomics and no second launch.
 //   * Launches use programmatic dependent launch: the next chunk's kernel may start
@@ -49,8 +49,8 @@ constexpr int kTileCols = 64;                       // channels per CTA tile (12
 constexpr int kThreads = 256;
 constexpr int kPhases = 32;                         // rows read side by side
 constexpr int kWarps = kThreads / 32;
-constexpr int kStageRows = 64;
-constexpr int kStages = 6;
+constexpr int kStageRows = 128;
+constexpr int kStages = 3;
 constexpr uint32_t kStageBytes = kStageRows * kTileCols * 2;
 constexpr size_t kRingBytes = (size_t)kStages * kStageBytes;
 constexpr int64_t kMaxRowsPerCta = 1024 * kPhases;  // <= 1024 sequential adds per thread
@@ -274,8 +274,9 @@ cudaError_t launch_hessian(const void* x, int64_t tokens, int64_t n, int64_t ld_
   if (r != CUDA_SUCCESS) return cudaErrorInvalidValue;
 
   const int tiles = (int)((n + kTileCols - 1) / kTileCols);
-  // about one wave: 4 resident CTAs per SM
-  const int64_t target = (int64_t)info.sm_count * 4;
+  // about two CTAs per SM: two consecutive chunk launches fit side by side, so with
+  // programmatic dependent launch the next chunk streams while this one drains
+  const int64_t target = (int64_t)info.sm_count * 2;
   int cs = 1;
   while (cs < kMaxCluster && (int64_t)tiles * cs * 2 <= target && (int64_t)cs * 2 * kStageRows * 4 <= tokens)
     cs *= 2;
