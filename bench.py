@@ -2,19 +2,20 @@
 """Benchmark of the H-Scale hot path on GB300 (one JSON line on rank 0).
 
 A step is one pass of the whole hot path over one synthetic layer with its inputs
-resident in HBM: the Hessian-diagonal pass over every calibration chunk
-(h_j += sum_t x_tj^2, Sec. 3.2), the global scale + RTN codes (Eq. 7), and the
-H-Scale window search fused with the final re-quantization and packing
-(Algorithm 1).  Default workload: Llama-style 8B q_proj, W [4096, 4096] bf16,
-262144 calibration tokens of width 4096 streamed in 8192-token chunks, window
-k = +-4.
+resident in HBM: for every input space the Hessian-diagonal pass over all calibration
+chunks (h_j += sum_t x_tj^2, Sec. 3.2), and for every weight matrix the global scale +
+RTN codes (Eq. 7) and the H-Scale window search fused with the final re-quantization and
+packing (Algorithm 1).  Default workload: Llama-style 8B q_proj, W [4096, 4096] bf16,
+262144 calibration tokens of width 4096 streamed in 8192-token chunks, window k = +-4.
+Other workloads: the full 8B decoder layer (per-layer and per-model seconds), the MLP
+down_proj, and the 70B MLP block with its window sweep.
 
 value      groups quantized per second by the whole step (all ranks), inputs in HBM
-e2e        the same through the public API with host buffers: the step's X chunks
-           and W copied from pinned host memory (chunk copies overlap the Hessian
-           pass on a second stream) and the codes + nibbles copied back
-roofline   the dominant kernel (the Hessian pass): algorithmic bytes per launch over
-           its CUDA-event time, against the measured HBM copy bandwidth
+e2e        the same through the public API with host buffers: the X chunks and W copied
+           from pinned host memory (chunk copies overlap the Hessian pass on a second
+           stream) and the codes + nibbles copied back
+roofline   the dominant kernel (the Hessian pass): algorithmic bytes per launch over its
+           CUDA-event time, against the measured HBM copy bandwidth
 cpu_baseline  the fp64 CPU oracle on a bounded sample of the same workload
 
 Multi-GPU: every rank quantizes its own layer (independent problems, no data-path
@@ -50,9 +51,9 @@ def parse():
     p.add_argument("--warmup", type=int, default=3)
     p.add_argument("--impl", choices=["hscale", "reference"], default="hscale")
     p.add_argument("--workload", default="llama8b-q_proj", choices=sorted(wl.WORKLOADS))
-    p.add_argument("--k", type=int, default=None, help="window half-width (default: workload's)")
+    p.add_argument("--k", type=int, default=None, help="window half-width (default: workload's first)")
     p.add_argument("--tokens", type=int, default=None,
-                   help="calibration tokens per step (default: the workload's; smaller for ncu captures)")
+                   help="calibration tokens per input space (default: the workload's; smaller for ncu captures)")
     p.add_argument("--no-cpu-baseline", action="store_true")
     p.add_argument("--no-e2e", action="store_true")
     return p.parse_args()
@@ -100,6 +101,25 @@ def measured_peaks():
         return float(d["hbm_gbs"]), "measured", d
     except Exception:
         return FALLBACK_HBM_GBS, "fallback", {}
+
+
+def profiled_traffic(workload: str, chunk: int, n: int):
+    """DRAM bytes per Hessian launch from the committed ncu summary, if the kernel's sources
+    are unchanged since that capture and the launch shape matches; else None."""
+    import hashlib
+    path = os.path.join(ROOT, "profiles", f"hessian_colsumsq_{workload}.traffic.json")
+    try:
+        with open(path) as f:
+            d = json.load(f)
+        h = hashlib.sha256()
+        for src in d["kernel_sources"]:
+            with open(os.path.join(ROOT, src), "rb") as f:
+                h.update(f.read())
+        if h.hexdigest() != d["kernel_sources_sha256"] or d["chunk_tokens"] != chunk or d["n"] != n:
+            return None
+        return int(d["dram_bytes_per_launch"])
+    except Exception:
+        return None
 
 
 class ClockSampler:
@@ -175,149 +195,175 @@ class ClockSampler:
                 "samples": len(self.samples), "source": "nvml" if self._nvml else "none"}
 
 
-def profiled_traffic(workload: str, chunk: int, n: int):
-    """DRAM bytes per Hessian launch from the committed ncu summary, if the kernel's sources
-    are unchanged since that capture and the launch shape matches; else None."""
-    import hashlib
-    path = os.path.join(ROOT, "profiles", f"hessian_colsumsq_{workload}.traffic.json")
-    try:
-        with open(path) as f:
-            d = json.load(f)
-        h = hashlib.sha256()
-        for src in d["kernel_sources"]:
-            with open(os.path.join(ROOT, src), "rb") as f:
-                h.update(f.read())
-        if h.hexdigest() != d["kernel_sources_sha256"] or d["chunk_tokens"] != chunk or d["n"] != n:
-            return None
-        return int(d["dram_bytes_per_launch"])
-    except Exception:
-        return None
-
-
 # ------------------------------------------------------------------ workload
-class Layer:
-    """Device-resident inputs and outputs of one layer of a workload."""
+class Space:
+    """One input space: resident calibration activations X [tokens, n] and its h."""
 
-    def __init__(self, W: wl.Workload, rank: int, k: int, device, tokens=None):
-        L = W.layers[0]
-        self.W, self.k = W, k
-        self.m, self.n = L.out_features, L.in_features
-        self.chunk = W.chunk_tokens[self.n]
+    def __init__(self, W: wl.Workload, name: str, n: int, seed: int, device, tokens=None):
+        self.name, self.n = name, n
+        self.chunk = W.chunk_tokens[n]
         self.nchunks = max(1, (tokens or W.tokens) // self.chunk)
         self.tokens = self.nchunks * self.chunk
-        seed = W.seed + 7919 * rank
-        self.seed = seed
-        a = wl.channel_magnitudes(self.n, W.sigma_a, W.outlier_channels, W.outlier_channel_mult,
-                                  seed, device=device)
-        self.x = torch.empty(self.tokens, self.n, dtype=torch.bfloat16, device=device)
+        a = wl.channel_magnitudes(n, W.sigma_a, W.outlier_channels, W.outlier_channel_mult,
+                                  wl.chunk_seed(seed, name, 0) & 0xFFFFFFFF, device=device)
+        self.x = torch.empty(self.tokens, n, dtype=torch.bfloat16, device=device)
         for c in range(self.nchunks):
-            wl.activation_chunk(self.chunk, a, seed, c, out=self.x[c * self.chunk:(c + 1) * self.chunk])
-        self.w = wl.weight(self.m, self.n, W.sigma_w, seed, device=device)
+            wl.activation_chunk(self.chunk, a, wl.chunk_seed(seed, name, 1) & 0xFFFFFFFF, c,
+                                out=self.x[c * self.chunk:(c + 1) * self.chunk])
+        self.h = torch.zeros(n, dtype=torch.float32, device=device)
+
+
+class Matrix:
+    """One weight matrix with its outputs; uses the h of its input space."""
+
+    def __init__(self, W: wl.Workload, L: wl.LayerShape, space: Space, seed: int, device):
+        self.name, self.m, self.n, self.space = L.name, L.out_features, L.in_features, space
+        self.w = wl.weight(self.m, self.n, W.sigma_w, wl.chunk_seed(seed, L.name, 0) & 0xFFFFFFFF,
+                           device=device)
         self.groups = self.m * self.n // 16
-        self.h = torch.zeros(self.n, dtype=torch.float32, device=device)
         self.sg = torch.empty(1, dtype=torch.float32, device=device)
         self.codes0 = torch.empty(self.m, self.n // 16, dtype=torch.uint8, device=device)
         self.codes = torch.empty_like(self.codes0)
         self.packed = torch.empty(self.m, self.n // 2, dtype=torch.uint8, device=device)
 
 
-def hessian_phase(hs, L: Layer, x=None):
-    """h = 0, then one hscale_hessian_diag_accumulate per calibration chunk."""
-    x = L.x if x is None else x
-    L.h.zero_()
-    for c in range(L.nchunks):
-        hs.hscale_hessian_diag_accumulate(x[c * L.chunk:(c + 1) * L.chunk], L.h)
+class Work:
+    """Device-resident inputs and outputs of one layer of a workload."""
+
+    def __init__(self, W: wl.Workload, rank: int, k: int, device, tokens=None):
+        self.W, self.k = W, k
+        self.seed = W.layer_seed(0) + 7919 * rank
+        self.spaces = {name: Space(W, name, n, self.seed, device, tokens) for name, n in W.input_spaces()}
+        self.mats = [Matrix(W, L, self.spaces[L.input_space], self.seed, device) for L in W.layers]
+        self.groups = sum(M.groups for M in self.mats)
+        self.h_bytes = sum(2 * S.tokens * S.n + 8 * S.n * S.nchunks for S in self.spaces.values())
+        self.h_launches = sum(S.nchunks for S in self.spaces.values())
+        self.ws = None
 
 
-def scale_phase(hs, L: Layer, w=None):
-    """Global scale + RTN codes, then the H-Scale search with the final packing."""
-    w = L.w if w is None else w
-    hs.hscale_rtn_scales(w, L.sg, L.codes0, L.ws)
-    hs.hscale_refine_scales(w, L.h, L.sg, L.codes0, L.k, L.k, L.codes, L.packed)
+def hessian_phase(hs, work: Work, xs=None):
+    """For every input space: h = 0, then one hscale_hessian_diag_accumulate per chunk."""
+    for S in work.spaces.values():
+        x = S.x if xs is None else xs[S.name]
+        S.h.zero_()
+        for c in range(S.nchunks):
+            hs.hscale_hessian_diag_accumulate(x[c * S.chunk:(c + 1) * S.chunk], S.h)
 
 
-def run_step(hs, L: Layer, ev=None):
+def scale_phase(hs, work: Work, k=None, ws=None):
+    """For every matrix: global scale + RTN codes, then the H-Scale search with packing."""
+    k = work.k if k is None else k
+    for M in work.mats:
+        w = M.w if ws is None else ws[M.name]
+        hs.hscale_rtn_scales(w, M.sg, M.codes0, work.ws)
+        hs.hscale_refine_scales(w, M.space.h, M.sg, M.codes0, k, k, M.codes, M.packed)
+
+
+def run_step(hs, work: Work, ev=None):
     """One eager pass of the hot path.  ev: optional 3 events (start, after h, end)."""
     if ev:
         ev[0].record()
-    hessian_phase(hs, L)
+    hessian_phase(hs, work)
     if ev:
         ev[1].record()
-    scale_phase(hs, L)
+    scale_phase(hs, work)
     if ev:
         ev[2].record()
 
 
-def capture_graphs(hs, L: Layer):
+def capture_graphs(hs, work: Work):
     """The step's launch sequence captured as two CUDA graphs (Hessian pass; scales)."""
     side = torch.cuda.Stream()
     side.wait_stream(torch.cuda.current_stream())
     with torch.cuda.stream(side):
-        run_step(hs, L)
+        run_step(hs, work)
     torch.cuda.current_stream().wait_stream(side)
     torch.cuda.synchronize()
     gh, gs = torch.cuda.CUDAGraph(), torch.cuda.CUDAGraph()
     with torch.cuda.graph(gh):
-        hessian_phase(hs, L)
+        hessian_phase(hs, work)
     with torch.cuda.graph(gs):
-        scale_phase(hs, L)
+        scale_phase(hs, work)
     torch.cuda.synchronize()
     return gh, gs
 
 
-KERNELS_PER_STEP_FIXED = 3  # amax, rtn codes, refine
+KERNELS_PER_MATRIX = 3  # amax, RTN codes, refine
+
+
+def timed(fn, reps):
+    """Average CUDA-event time (ms) of fn over reps calls on the current stream."""
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    e0.record()
+    for _ in range(reps):
+        fn()
+    e1.record()
+    torch.cuda.synchronize()
+    return e0.elapsed_time(e1) / reps
 
 
 # ------------------------------------------------------------------ CPU oracle baseline
 def cpu_baseline(W: wl.Workload, k: int, budget_s: float = 12.0):
     """Time the fp64 oracle on a bounded sample of the workload and extrapolate the
-    whole-step time: Hessian over sampled tokens, RTN over the whole W, search over
-    sampled rows."""
+    whole-step time: Hessian over sampled tokens of every input space, global scale + RTN
+    over every matrix, search over sampled rows of every matrix."""
     import oracle
     oracle.build()
     cores = len(os.sched_getaffinity(0)) if hasattr(os, "sched_getaffinity") else os.cpu_count()
     oracle.set_threads(cores)
-    L = W.layers[0]
-    m, n = L.out_features, L.in_features
-    a = wl.channel_magnitudes(n, W.sigma_a, W.outlier_channels, W.outlier_channel_mult, W.seed)
-    tok = min(W.chunk_tokens[n], 4096)
-    xb = wl.bf16_bits(wl.activation_chunk(tok, a, W.seed, 0))
-    wb = wl.bf16_bits(wl.weight(m, n, W.sigma_w, W.seed))
-    h = np.zeros(n)
-    t0 = time.perf_counter()
-    reps = 0
-    while True:
-        oracle.hessian_accumulate(xb, h)
-        reps += 1
-        if time.perf_counter() - t0 > budget_s / 3:
-            break
-    t_h = (time.perf_counter() - t0) / (reps * tok * n)        # seconds per token*channel
-    t0 = time.perf_counter()
-    s_g, _ = oracle.global_scale(wb)
-    oracle.rtn_codes(wb, s_g)
-    t_rtn = time.perf_counter() - t0
-    h32 = h.astype(np.float32)
-    rows = max(8, min(m, 64))
-    t0 = time.perf_counter()
-    done = 0
-    while True:
-        r0 = (done * rows) % m
-        oracle.refine(wb[r0:r0 + rows], h32, s_g, None, k, k)
-        done += 1
-        if time.perf_counter() - t0 > budget_s / 3:
-            break
-    t_g = (time.perf_counter() - t0) / (done * rows * n // 16)  # seconds per group
-    groups = m * n // 16
-    step = t_h * W.tokens * n + t_rtn + t_g * groups
+    per_part = budget_s / (len(W.input_spaces()) + len(W.layers))
+    step = 0.0
+    groups = 0
+    h_tc = 0
+    samples = []
+    hs_of = {}
+    for name, n in W.input_spaces():
+        a = wl.channel_magnitudes(n, W.sigma_a, W.outlier_channels, W.outlier_channel_mult, W.seed)
+        tok = min(W.chunk_tokens[n], 4096)
+        xb = wl.bf16_bits(wl.activation_chunk(tok, a, W.seed, 0))
+        h = np.zeros(n)
+        t0 = time.perf_counter()
+        reps = 0
+        while True:
+            oracle.hessian_accumulate(xb, h)
+            reps += 1
+            if time.perf_counter() - t0 > per_part:
+                break
+        t_tc = (time.perf_counter() - t0) / (reps * tok * n)
+        step += t_tc * W.tokens * n
+        h_tc += W.tokens * n
+        hs_of[name] = (h / reps * (W.tokens / tok)).astype(np.float32)
+        samples.append(f"Hessian {name}: {reps} x {tok}x{n}")
+    t_rtn_total = 0.0
+    for L in W.layers:
+        m, n = L.out_features, L.in_features
+        wb = wl.bf16_bits(wl.weight(m, n, W.sigma_w, W.seed))
+        t0 = time.perf_counter()
+        s_g, _ = oracle.global_scale(wb)
+        oracle.rtn_codes(wb, s_g)
+        t_rtn_total += time.perf_counter() - t0
+        rows = max(8, min(m, 64))
+        t0 = time.perf_counter()
+        done = 0
+        while True:
+            r0 = (done * rows) % m
+            oracle.refine(wb[r0:r0 + rows], hs_of[L.input_space], s_g, None, k, k)
+            done += 1
+            if time.perf_counter() - t0 > per_part:
+                break
+        t_g = (time.perf_counter() - t0) / (done * rows * n // 16)
+        G = m * n // 16
+        step += t_g * G
+        groups += G
+        samples.append(f"search {L.name}: {done}x{rows} rows")
+    step += t_rtn_total
     return {
         "value": groups / step, "unit": UNIT, "cores": cores, "kind": "oracle",
-        "sample": (f"fp64 C oracle, {cores} threads: Hessian over {tok}x{n} tokens*channels "
-                   f"x{reps}, global scale + RTN over the whole {m}x{n} W, search over "
-                   f"{done}x{rows} rows (k={k}); step time extrapolated to {W.tokens} tokens "
-                   f"and {groups} groups"),
+        "sample": (f"fp64 C oracle, {cores} threads, bounded sample extrapolated to the step "
+                   f"({W.tokens} tokens per input space, {groups} groups, k={k}): "
+                   + "; ".join(samples) + "; global scale + RTN over every whole matrix"),
         "seconds_per_step": step,
-        "hessian_tokens_channels_per_s": 1.0 / t_h,
-        "search_groups_per_s": 1.0 / t_g,
+        "hessian_tokens_channels_per_s": h_tc / max(step, 1e-30),
     }
 
 
@@ -333,8 +379,7 @@ def reference_arm(args, d: Dist):
         cb = cpu_baseline(W, k, budget_s=3.0)
         if i >= args.warmup:
             vals.append(cb["seconds_per_step"])
-    L = W.layers[0]
-    groups = L.out_features * L.in_features // 16
+    groups = sum(L.out_features * L.in_features // 16 for L in W.layers)
     sec = statistics.mean(vals)
     value = groups / sec
     line = {
@@ -342,7 +387,7 @@ def reference_arm(args, d: Dist):
         "steps": args.steps, "warmup": args.warmup, "ms_per_step": sec * 1e3,
         "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
         "data": "synthetic",
-        "config": {"workload": W.name, "m": L.out_features, "n": L.in_features,
+        "config": {"workload": W.name, "matrices": [[L.name, L.out_features, L.in_features] for L in W.layers],
                    "tokens": W.tokens, "k": k},
         "cpu_baseline": {"value": value, "unit": UNIT, "cores": cb["cores"], "kind": "oracle",
                          "sample": cb["sample"]},
@@ -359,25 +404,20 @@ def gpu_arm(args, d: Dist):
     dev = torch.device("cuda", d.local)
     W = wl.WORKLOADS[args.workload]
     k = args.k if args.k is not None else W.window[0]
-    L = Layer(W, d.rank, k, dev, tokens=args.tokens)
-    L.ws = torch.empty(hs.hscale_rtn_workspace_bytes(), dtype=torch.uint8, device=dev)
+    work = Work(W, d.rank, k, dev, tokens=args.tokens)
+    work.ws = torch.empty(hs.hscale_rtn_workspace_bytes(), dtype=torch.uint8, device=dev)
     torch.cuda.synchronize()
 
     warm = max(args.warmup, 3)
     for _ in range(warm):
-        run_step(hs, L)
+        run_step(hs, work)
     torch.cuda.synchronize()
 
-    # eager launches (one API call per chunk), for reference
-    ev_e = [[torch.cuda.Event(enable_timing=True) for _ in range(3)] for _ in range(args.steps)]
-    torch.cuda.synchronize()
-    for s in range(args.steps):
-        run_step(hs, L, ev=ev_e[s])
-    torch.cuda.synchronize()
-    ms_eager = sum(e[0].elapsed_time(e[2]) for e in ev_e) / args.steps
+    # eager launches (one API call per chunk and matrix), for reference
+    ms_eager = timed(lambda: run_step(hs, work), args.steps)
 
     # timed region: the same launches replayed from CUDA graphs
-    gh, gs = capture_graphs(hs, L)
+    gh, gs = capture_graphs(hs, work)
     for _ in range(warm):
         gh.replay()
         gs.replay()
@@ -401,70 +441,78 @@ def gpu_arm(args, d: Dist):
     ms_h = sum(e[0].elapsed_time(e[1]) for e in evs) / args.steps
     ms_sc = sum(e[1].elapsed_time(e[2]) for e in evs) / args.steps
     ms_step = d.max(ms_total / args.steps)
-    value = L.groups * d.world / (ms_step * 1e-3)
+    value = work.groups * d.world / (ms_step * 1e-3)
 
-    # per-kernel times of the scale phase (rtn_scales; refine) from an eager loop
-    ev_k = [[torch.cuda.Event(enable_timing=True) for _ in range(3)] for _ in range(args.steps)]
-    for s in range(args.steps):
-        hs.hscale_rtn_scales(L.w, L.sg, L.codes0, L.ws)
-        ev_k[s][0].record()
-        hs.hscale_rtn_scales(L.w, L.sg, L.codes0, L.ws)
-        ev_k[s][1].record()
-        hs.hscale_refine_scales(L.w, L.h, L.sg, L.codes0, L.k, L.k, L.codes, L.packed)
-        ev_k[s][2].record()
-    torch.cuda.synchronize()
-    ms_rtn = sum(e[0].elapsed_time(e[1]) for e in ev_k) / args.steps
-    ms_ref = sum(e[1].elapsed_time(e[2]) for e in ev_k) / args.steps
-
-    # ---- roofline of the dominant kernel (the Hessian pass)
+    # ---- per-kernel times of the scale phase, every matrix, every window of the workload
     hbm_peak, peak_kind, peaks = measured_peaks()
-    h_bytes_launch = 2 * L.chunk * L.n + 8 * L.n          # X read + h read/write
-    ms_h_launch = ms_h / L.nchunks
-    h_gbs = h_bytes_launch / (ms_h_launch * 1e-3) / 1e9
-    # ---- search roofline: max(42 B/group over HBM, 80*C ops/group over the FP32 peak)
     props = torch.cuda.get_device_properties(dev)
     sm_max_mhz = float(peaks.get("sm_max_mhz", 2070.0))
     fp32_peak = props.multi_processor_count * 128 * sm_max_mhz * 1e6
-    C = 2 * k + 1
-    t_bytes = 42 * L.groups / (hbm_peak * 1e9)
-    t_ops = 80 * C * L.groups / fp32_peak
-    t_search_roof = max(t_bytes, t_ops)
-    search_frac = t_search_roof / (ms_ref * 1e-3)
+    reps = max(3, min(args.steps, 20))
+    ms_rtn = sum(timed(lambda M=M: hs.hscale_rtn_scales(M.w, M.sg, M.codes0, work.ws), reps) for M in work.mats)
+    sweep = []
+    for kk in sorted(set([k] + list(W.window))):
+        ms_ref = 0.0
+        for M in work.mats:
+            ms_ref += timed(lambda M=M: hs.hscale_refine_scales(M.w, M.space.h, M.sg, M.codes0, kk, kk,
+                                                                 M.codes, M.packed), reps)
+        C = 2 * kk + 1
+        t_bytes = 42 * work.groups / (hbm_peak * 1e9)
+        t_ops = 80 * C * work.groups / fp32_peak
+        sweep.append({"k": kk, "candidates": C, "ms": ms_ref, "groups_per_s": work.groups / (ms_ref * 1e-3),
+                      "bound": "alu" if t_ops > t_bytes else "hbm", "roofline_ms": max(t_bytes, t_ops) * 1e3,
+                      "frac": max(t_bytes, t_ops) / (ms_ref * 1e-3)})
+    # restore the outputs of the step's own window
+    scale_phase(hs, work)
+    torch.cuda.synchronize()
+    main = [s for s in sweep if s["k"] == k][0]
+
+    # ---- roofline of the dominant kernel (the Hessian pass)
+    h_bytes_launch = work.h_bytes / work.h_launches
+    ms_h_launch = ms_h / work.h_launches
+    h_gbs = work.h_bytes / (ms_h * 1e-3) / 1e9
+    first = next(iter(work.spaces.values()))
+    traffic = profiled_traffic(W.name, first.chunk, first.n) if len(work.spaces) == 1 else None
 
     # ---- end to end through the public API with host buffers
-    e2e = None
-    if not args.no_e2e:
-        e2e = e2e_leg(hs, L, args)
+    e2e = None if args.no_e2e else e2e_leg(hs, work, args)
 
+    n_layers = W.n_layers
     line = {
         "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": d.world, "steps": args.steps,
-        "warmup": max(args.warmup, 3), "ms_per_step": ms_step, "higher_is_better": True,
+        "warmup": warm, "ms_per_step": ms_step, "higher_is_better": True,
         "scaling": "weak", "vs_baseline": None, "dtype": "f32", "input_dtype": "bf16",
         "data": "synthetic",
-        "config": {"workload": W.name, "m": L.m, "n": L.n, "tokens": L.tokens,
-                   "chunk_tokens": L.chunk, "k": k, "groups": L.groups,
-                   "l2": f"inputs larger than L2: {L.tokens * L.n * 2 / 1e9:.2f} GB of X streamed per step",
+        "config": {"workload": W.name,
+                   "matrices": [[M.name, M.m, M.n] for M in work.mats],
+                   "input_spaces": [[S.name, S.tokens, S.n, S.chunk] for S in work.spaces.values()],
+                   "k": k, "groups": work.groups,
+                   "l2": "inputs larger than L2: %.2f GB of X streamed per step" %
+                         (sum(S.tokens * S.n * 2 for S in work.spaces.values()) / 1e9),
                    "parallelism": f"independent layer per GPU x{d.world}"},
         "roofline": {"bound": "hbm", "kernel": "hessian_colsumsq", "achieved": h_gbs,
                      "peak": hbm_peak, "unit": "GB/s", "frac": h_gbs / hbm_peak,
                      "peak_kind": f"{peak_kind} HBM copy bandwidth",
-                     "frac_of_8TBs_spec": h_gbs / HBM_SPEC_GBS,
-                     "traffic": profiled_traffic(W.name, L.chunk, L.n),
+                     "frac_of_8TBs_spec": h_gbs / HBM_SPEC_GBS, "traffic": traffic,
                      "bytes_per_launch": h_bytes_launch, "ms_per_launch": ms_h_launch},
-        "phases_ms": {"hessian": ms_h, "scales": ms_sc, "rtn_scales": ms_rtn, "refine": ms_ref},
+        "phases_ms": {"hessian": ms_h, "scales": ms_sc, "rtn_scales": ms_rtn, "refine": main["ms"]},
         "ms_per_step_eager": ms_eager,
         "timed_launch": "CUDA graphs of the step's API calls (Hessian pass; scales)",
-        "hessian": {"gbs": h_gbs, "tokens_channels_per_s": L.chunk * L.n / (ms_h_launch * 1e-3),
+        "hessian": {"gbs": h_gbs, "tokens_channels_per_s": work.h_bytes / 2 / (ms_h * 1e-3),
                     "frac_of_measured_hbm": h_gbs / hbm_peak, "frac_of_8TBs": h_gbs / HBM_SPEC_GBS},
-        "search": {"groups_per_s": L.groups / (ms_ref * 1e-3), "candidates": C,
-                   "bound": "alu" if t_ops > t_bytes else "hbm",
-                   "roofline_s": t_search_roof, "frac": search_frac,
+        "search": {"groups_per_s": main["groups_per_s"], "candidates": main["candidates"],
+                   "bound": main["bound"], "roofline_s": main["roofline_ms"] * 1e-3, "frac": main["frac"],
                    "fp32_peak_ops": fp32_peak, "sm_count": props.multi_processor_count,
                    "clock_mhz_for_peak": sm_max_mhz},
         "seconds_per_layer": ms_step * 1e-3,
         "clocks": clk.summary(),
-        "gpu_launches": args.steps * (L.nchunks + KERNELS_PER_STEP_FIXED),
+        "gpu_launches": args.steps * (work.h_launches + KERNELS_PER_MATRIX * len(work.mats)),
     }
+    if len(sweep) > 1:
+        line["search_sweep"] = sweep
+    if n_layers > 1:
+        line["seconds_per_model"] = ms_step * 1e-3 * n_layers
+        line["seconds_per_model_note"] = f"{n_layers} layers of identical shapes: per-layer step x {n_layers}"
     if e2e:
         line["e2e"] = e2e
     if d.rank == 0 and d.world == 1 and not args.no_cpu_baseline:
@@ -474,63 +522,58 @@ def gpu_arm(args, d: Dist):
         print(json.dumps(line), flush=True)
 
 
-def e2e_leg(hs, L: Layer, args):
+def e2e_leg(hs, work: Work, args):
     """Whole step through the public API with host buffers: X chunks and W copied from
     pinned host memory inside the timed region (chunk copies on a copy stream overlap
     the Hessian pass), codes and nibbles copied back."""
-    dev = L.x.device
-    x_host = torch.empty(L.x.shape, dtype=L.x.dtype, pin_memory=True)
-    x_host.copy_(L.x)
-    w_host = torch.empty(L.w.shape, dtype=L.w.dtype, pin_memory=True)
-    w_host.copy_(L.w)
-    codes_host = torch.empty(L.codes.shape, dtype=torch.uint8, pin_memory=True)
-    packed_host = torch.empty(L.packed.shape, dtype=torch.uint8, pin_memory=True)
+    dev = next(iter(work.spaces.values())).x.device
+    x_host, xbuf = {}, {}
     nbuf = 3
-    xbuf = [torch.empty(L.chunk, L.n, dtype=torch.bfloat16, device=dev) for _ in range(nbuf)]
-    wdev = torch.empty_like(L.w)
+    for S in work.spaces.values():
+        x_host[S.name] = torch.empty(S.x.shape, dtype=S.x.dtype, pin_memory=True)
+        x_host[S.name].copy_(S.x)
+        xbuf[S.name] = [torch.empty(S.chunk, S.n, dtype=torch.bfloat16, device=dev) for _ in range(nbuf)]
+    w_host = {M.name: torch.empty(M.w.shape, dtype=M.w.dtype, pin_memory=True).copy_(M.w) for M in work.mats}
+    w_dev = {M.name: torch.empty_like(M.w) for M in work.mats}
+    out_host = {M.name: (torch.empty(M.codes.shape, dtype=torch.uint8, pin_memory=True),
+                         torch.empty(M.packed.shape, dtype=torch.uint8, pin_memory=True)) for M in work.mats}
     copy = torch.cuda.Stream(device=dev)
     comp = torch.cuda.current_stream(dev)
 
     def step():
-        done = [torch.cuda.Event() for _ in range(nbuf)]
-        ready = [torch.cuda.Event() for _ in range(L.nchunks)]
-        L.h.zero_()
-        for c in range(L.nchunks):
-            b = c % nbuf
-            with torch.cuda.stream(copy):
-                if c >= nbuf:
-                    copy.wait_event(done[b])
-                xbuf[b].copy_(x_host[c * L.chunk:(c + 1) * L.chunk], non_blocking=True)
-                ready[c].record(copy)
-            comp.wait_event(ready[c])
-            hs.hscale_hessian_diag_accumulate(xbuf[b], L.h)
-            done[b].record(comp)
+        for S in work.spaces.values():
+            done = [torch.cuda.Event() for _ in range(nbuf)]
+            S.h.zero_()
+            for c in range(S.nchunks):
+                b = c % nbuf
+                with torch.cuda.stream(copy):
+                    if c >= nbuf:
+                        copy.wait_event(done[b])
+                    xbuf[S.name][b].copy_(x_host[S.name][c * S.chunk:(c + 1) * S.chunk], non_blocking=True)
+                    ready = torch.cuda.Event()
+                    ready.record(copy)
+                comp.wait_event(ready)
+                hs.hscale_hessian_diag_accumulate(xbuf[S.name][b], S.h)
+                done[b].record(comp)
         with torch.cuda.stream(copy):
-            wdev.copy_(w_host, non_blocking=True)
+            for M in work.mats:
+                w_dev[M.name].copy_(w_host[M.name], non_blocking=True)
             wr = torch.cuda.Event()
             wr.record(copy)
         comp.wait_event(wr)
-        hs.hscale_rtn_scales(wdev, L.sg, L.codes0, L.ws)
-        hs.hscale_refine_scales(wdev, L.h, L.sg, L.codes0, L.k, L.k, L.codes, L.packed)
-        codes_host.copy_(L.codes, non_blocking=True)
-        packed_host.copy_(L.packed, non_blocking=True)
+        scale_phase(hs, work, ws=w_dev)
+        for M in work.mats:
+            out_host[M.name][0].copy_(M.codes, non_blocking=True)
+            out_host[M.name][1].copy_(M.packed, non_blocking=True)
 
     for _ in range(2):
         step()
     torch.cuda.synchronize()
     reps = max(3, min(args.steps, 10))
-    t0 = torch.cuda.Event(enable_timing=True)
-    t1 = torch.cuda.Event(enable_timing=True)
-    t0.record()
-    for _ in range(reps):
-        step()
-    t1.record()
-    torch.cuda.synchronize()
-    ms = t0.elapsed_time(t1) / reps
-    h2d = L.tokens * L.n * 2 + L.m * L.n * 2
-    d2h = L.codes.numel() + L.packed.numel()
-    del x_host
-    return {"value": L.groups / (ms * 1e-3), "unit": UNIT, "ms_per_step": ms,
+    ms = timed(step, reps)
+    h2d = sum(S.tokens * S.n * 2 for S in work.spaces.values()) + sum(M.m * M.n * 2 for M in work.mats)
+    d2h = sum(M.codes.numel() + M.packed.numel() for M in work.mats)
+    return {"value": work.groups / (ms * 1e-3), "unit": UNIT, "ms_per_step": ms,
             "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h}
 
 

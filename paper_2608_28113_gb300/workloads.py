@@ -86,13 +86,13 @@ WORKLOADS = {
          LayerShape("down_proj", 4096, 14336, "down_in")),
         tokens=131072, chunk_tokens={4096: 8192, 14336: 4096}, sigma_w=0.02, sigma_a=1.5,
         outlier_channels=32, outlier_channel_mult=100.0, window=(4,), seed=3, n_layers=32),
-    # 70B-class MLP block at wide shapes; window sweep k in {1, 2, 4, 8, 16}
+    # 70B-class MLP block at wide shapes; k = 4 first, then the sweep k in {1, 2, 8, 16}
     "llama70b-mlp": Workload(
         "llama70b-mlp",
         (LayerShape("gate_proj", 28672, 8192, "mlp_in"), LayerShape("up_proj", 28672, 8192, "mlp_in"),
          LayerShape("down_proj", 8192, 28672, "down_in")),
         tokens=65536, chunk_tokens={8192: 4096, 28672: 2048}, sigma_w=0.015, sigma_a=1.5,
-        outlier_channels=32, outlier_channel_mult=100.0, window=(1, 2, 4, 8, 16), seed=4),
+        outlier_channels=32, outlier_channel_mult=100.0, window=(4, 1, 2, 8, 16), seed=4),
 }
 
 

@@ -359,38 +359,44 @@ def test_refine_is_deterministic():
 
 # ------------------------------------------------------------------ full-size workloads
 
-def full_size_check(name, sample_rows):
-    """The workload at its full size in the launch configuration bench.py times: h over
-    every streamed chunk (all columns, against the oracle fed the same chunks), s_g and
-    RTN codes over the whole matrix, and the search on a seeded sample of rows."""
+def full_size_check(name, sample_rows, layer_index=0):
+    """A workload at its full size in the launch configuration bench.py times: h of every
+    input space over every streamed chunk (all columns, against the oracle fed the same
+    chunks), s_g and RTN codes over every whole matrix, and the search with packing on a
+    seeded sample of rows of every matrix, for every window of the workload."""
     W = wl.WORKLOADS[name]
-    L = W.layers[0]
-    n, m = L.in_features, L.out_features
-    chunk = W.chunk_tokens[n]
-    a = wl.channel_magnitudes(n, W.sigma_a, W.outlier_channels, W.outlier_channel_mult, W.seed,
-                              device=dev())
-    h = torch.zeros(n, device=dev())
-    h_ref = np.zeros(n)
-    for c in range(0, W.tokens // chunk):
-        x = wl.activation_chunk(chunk, a, W.seed, c)
-        hs.hscale_hessian_diag_accumulate(x, h)
-        oracle.hessian_accumulate(bits(x), h_ref)
-        del x
-    torch.cuda.synchronize()
-    err = assert_h_close(h.cpu().numpy(), h_ref)
-    print(f"[parity] {name}: h over {W.tokens} tokens x {n}: max rel err {err:.3e}")
-    w = wl.weight(m, n, W.sigma_w, W.seed, device=dev())
-    sg, codes = gpu_rtn(w)
-    wb = bits(w)
-    s_ref, _ = oracle.global_scale(wb)
-    assert sg.cpu().numpy()[0] == s_ref
-    assert np.array_equal(codes.cpu().numpy(), oracle.rtn_codes(wb, s_ref))
-    h32 = h_ref.astype(np.float32)
-    rows = np.sort(np.random.default_rng(W.seed).choice(m, size=min(sample_rows, m), replace=False))
-    for k in W.window:
-        codes_g, packed_g = gpu_refine(w, h32, sg, None, k, k)
-        ref = oracle.refine(wb[rows], h32, s_ref, None, k, k)
-        compare_search(ref, codes_g[rows], packed_g[rows], f"{name} k={k} ({rows.size} sampled rows)")
+    seed = W.layer_seed(layer_index)
+    h_ref = {}
+    for space, n in W.input_spaces():
+        chunk = W.chunk_tokens[n]
+        a = wl.channel_magnitudes(n, W.sigma_a, W.outlier_channels, W.outlier_channel_mult,
+                                  wl.chunk_seed(seed, space, 0) & 0xFFFFFFFF, device=dev())
+        h = torch.zeros(n, device=dev())
+        href = np.zeros(n)
+        for c in range(W.tokens // chunk):
+            x = wl.activation_chunk(chunk, a, wl.chunk_seed(seed, space, 1) & 0xFFFFFFFF, c)
+            hs.hscale_hessian_diag_accumulate(x, h)
+            oracle.hessian_accumulate(bits(x), href)
+            del x
+        torch.cuda.synchronize()
+        err = assert_h_close(h.cpu().numpy(), href)
+        print(f"[parity] {name} {space}: h over {W.tokens} tokens x {n}: max rel err {err:.3e}")
+        h_ref[space] = href.astype(np.float32)
+    for L in W.layers:
+        m, n = L.out_features, L.in_features
+        w = wl.weight(m, n, W.sigma_w, wl.chunk_seed(seed, L.name, 0) & 0xFFFFFFFF, device=dev())
+        sg, codes = gpu_rtn(w)
+        wb = bits(w)
+        s_ref, _ = oracle.global_scale(wb)
+        assert sg.cpu().numpy()[0] == s_ref
+        assert np.array_equal(codes.cpu().numpy(), oracle.rtn_codes(wb, s_ref))
+        rows = np.sort(np.random.default_rng(seed).choice(m, size=min(sample_rows, m), replace=False))
+        for k in W.window:
+            codes_g, packed_g = gpu_refine(w, h_ref[L.input_space], sg, None, k, k)
+            ref = oracle.refine(wb[rows], h_ref[L.input_space], s_ref, None, k, k)
+            compare_search(ref, codes_g[rows], packed_g[rows],
+                           f"{name} {L.name} {m}x{n} k={k} ({rows.size} sampled rows)")
+        del w
 
 
 def test_full_size_llama8b_q_proj():
@@ -399,3 +405,11 @@ def test_full_size_llama8b_q_proj():
 
 def test_full_size_mlp_down_proj():
     full_size_check("mlp-down_proj", sample_rows=128)
+
+
+def test_full_size_llama8b_decoder_layer():
+    full_size_check("llama8b-decoder", sample_rows=64, layer_index=7)
+
+
+def test_full_size_llama70b_mlp_window_sweep():
+    full_size_check("llama70b-mlp", sample_rows=24)
