@@ -51,7 +51,9 @@ def parse():
     p.add_argument("--warmup", type=int, default=3)
     p.add_argument("--impl", choices=["hscale", "reference"], default="hscale")
     p.add_argument("--workload", default="llama8b-q_proj", choices=sorted(wl.WORKLOADS))
-    p.add_argument("--k", type=int, default=None, help="window half-width (default: workload's first)")
+    p.add_argument("--k", type=int, default=None, help="symmetric window half-width (default: workload's first)")
+    p.add_argument("--window", default=None,
+                   help="asymmetric window 'D,U' (codes c0-D .. c0+U); e.g. 9,6 is the paper's K = 16 default")
     p.add_argument("--tokens", type=int, default=None,
                    help="calibration tokens per input space (default: the workload's; smaller for ncu captures)")
     p.add_argument("--no-cpu-baseline", action="store_true")
@@ -230,8 +232,8 @@ class Matrix:
 class Work:
     """Device-resident inputs and outputs of one layer of a workload."""
 
-    def __init__(self, W: wl.Workload, rank: int, k: int, device, tokens=None):
-        self.W, self.k = W, k
+    def __init__(self, W: wl.Workload, rank: int, win, device, tokens=None):
+        self.W, self.win = W, tuple(win)
         self.seed = W.layer_seed(0) + 7919 * rank
         self.spaces = {name: Space(W, name, n, self.seed, device, tokens) for name, n in W.input_spaces()}
         self.mats = [Matrix(W, L, self.spaces[L.input_space], self.seed, device) for L in W.layers]
@@ -250,13 +252,14 @@ def hessian_phase(hs, work: Work, xs=None):
             hs.hscale_hessian_diag_accumulate(x[c * S.chunk:(c + 1) * S.chunk], S.h)
 
 
-def scale_phase(hs, work: Work, k=None, ws=None):
-    """For every matrix: global scale + RTN codes, then the H-Scale search with packing."""
-    k = work.k if k is None else k
+def scale_phase(hs, work: Work, win=None, ws=None):
+    """For every matrix: global scale + RTN codes, then the H-Scale search with packing
+    over the window win = (down, up)."""
+    down, up = work.win if win is None else win
     for M in work.mats:
         w = M.w if ws is None else ws[M.name]
         hs.hscale_rtn_scales(w, M.sg, M.codes0, work.ws)
-        hs.hscale_refine_scales(w, M.space.h, M.sg, M.codes0, k, k, M.codes, M.packed)
+        hs.hscale_refine_scales(w, M.space.h, M.sg, M.codes0, down, up, M.codes, M.packed)
 
 
 def run_step(hs, work: Work, ev=None):
@@ -303,7 +306,16 @@ def timed(fn, reps):
 
 
 # ------------------------------------------------------------------ CPU oracle baseline
-def cpu_baseline(W: wl.Workload, k: int, budget_s: float = 12.0):
+def window_of(args, W: wl.Workload):
+    """(down, up) of the run: --window D,U, else --k, else the workload's first k."""
+    if args.window:
+        d, u = (int(v) for v in args.window.split(","))
+        return (d, u)
+    k = args.k if args.k is not None else W.window[0]
+    return (k, k)
+
+
+def cpu_baseline(W: wl.Workload, win, budget_s: float = 12.0):
     """Time the fp64 oracle on a bounded sample of the workload and extrapolate the
     whole-step time: Hessian over sampled tokens of every input space, global scale + RTN
     over every matrix, search over sampled rows of every matrix."""
@@ -347,7 +359,7 @@ def cpu_baseline(W: wl.Workload, k: int, budget_s: float = 12.0):
         done = 0
         while True:
             r0 = (done * rows) % m
-            oracle.refine(wb[r0:r0 + rows], hs_of[L.input_space], s_g, None, k, k)
+            oracle.refine(wb[r0:r0 + rows], hs_of[L.input_space], s_g, None, win[0], win[1])
             done += 1
             if time.perf_counter() - t0 > per_part:
                 break
@@ -360,7 +372,7 @@ def cpu_baseline(W: wl.Workload, k: int, budget_s: float = 12.0):
     return {
         "value": groups / step, "unit": UNIT, "cores": cores, "kind": "oracle",
         "sample": (f"fp64 C oracle, {cores} threads, bounded sample extrapolated to the step "
-                   f"({W.tokens} tokens per input space, {groups} groups, k={k}): "
+                   f"({W.tokens} tokens per input space, {groups} groups, window -{win[0]}/+{win[1]}): "
                    + "; ".join(samples) + "; global scale + RTN over every whole matrix"),
         "seconds_per_step": step,
         "hessian_tokens_channels_per_s": h_tc / max(step, 1e-30),
@@ -372,11 +384,11 @@ def reference_arm(args, d: Dist):
     if d.rank != 0:
         return
     W = wl.WORKLOADS[args.workload]
-    k = args.k if args.k is not None else W.window[0]
+    win = window_of(args, W)
     vals = []
     cb = None
     for i in range(args.warmup + args.steps):
-        cb = cpu_baseline(W, k, budget_s=3.0)
+        cb = cpu_baseline(W, win, budget_s=3.0)
         if i >= args.warmup:
             vals.append(cb["seconds_per_step"])
     groups = sum(L.out_features * L.in_features // 16 for L in W.layers)
@@ -388,12 +400,50 @@ def reference_arm(args, d: Dist):
         "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
         "data": "synthetic",
         "config": {"workload": W.name, "matrices": [[L.name, L.out_features, L.in_features] for L in W.layers],
-                   "tokens": W.tokens, "k": k},
+                   "tokens": W.tokens, "window": list(win)},
         "cpu_baseline": {"value": value, "unit": UNIT, "cores": cb["cores"], "kind": "oracle",
                          "sample": cb["sample"]},
         "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
     }
     print(json.dumps(line), flush=True)
+
+
+def shift_statistics(work: Work, win, sample_rows: int = 16):
+    """Selected shifts delta = chosen code - initial code over every group of the step
+    (from the GPU outputs), and the mean reduction of the Hessian-weighted error per
+    delta relative to delta = 0 on a sample of rows (from the CPU oracle).  The paper
+    reports the same statistics for real weights (Sec. 4, selected scale shifts)."""
+    down, up = win
+    hist = torch.zeros(down + up + 1, dtype=torch.int64)
+    for M in work.mats:
+        delta = M.codes.to(torch.int16) - M.codes0.to(torch.int16)
+        hist += torch.bincount((delta.flatten() + down).clamp(0, down + up).to(torch.int64).cpu(),
+                               minlength=down + up + 1)
+    total = int(hist.sum())
+    out = {"window": [down, up], "groups": total,
+           "delta_hist": {str(i - down): int(v) for i, v in enumerate(hist.tolist())},
+           "keep": float(hist[down]) / total, "larger": float(hist[down + 1:].sum()) / total,
+           "smaller": float(hist[:down].sum()) / total}
+    try:
+        import oracle
+        M = work.mats[0]
+        rows = np.linspace(0, M.m - 1, num=min(sample_rows, M.m)).astype(int)
+        ref = oracle.refine(wl.bf16_bits(M.w[rows]), M.space.h.cpu().numpy(), M.sg.item(),
+                            M.codes0[rows].cpu().numpy(), down, up)
+        red = {}
+        for dlt in range(-down, up + 1):
+            sel = ref["delta"] == dlt
+            if sel.any() and dlt != 0:
+                e0, e1 = ref["e_init"][sel], ref["e_best"][sel]
+                ok = e0 > 0
+                red[str(dlt)] = float(np.mean(1.0 - e1[ok] / e0[ok])) if ok.any() else None
+        tot0, tot1 = ref["e_init"].sum(), ref["e_best"].sum()
+        out["mean_error_reduction_by_delta"] = red
+        out["error_removed"] = float(1.0 - tot1 / tot0) if tot0 > 0 else None
+        out["error_sample"] = f"oracle on {rows.size} rows of {M.name}"
+    except Exception as e:  # the statistics are context; never fail the run for them
+        out["error_sample"] = f"unavailable: {e}"
+    return out
 
 
 # ------------------------------------------------------------------ GPU arm
@@ -403,8 +453,8 @@ def gpu_arm(args, d: Dist):
     torch.cuda.set_device(d.local)
     dev = torch.device("cuda", d.local)
     W = wl.WORKLOADS[args.workload]
-    k = args.k if args.k is not None else W.window[0]
-    work = Work(W, d.rank, k, dev, tokens=args.tokens)
+    win = window_of(args, W)
+    work = Work(W, d.rank, win, dev, tokens=args.tokens)
     work.ws = torch.empty(hs.hscale_rtn_workspace_bytes(), dtype=torch.uint8, device=dev)
     torch.cuda.synchronize()
 
@@ -451,21 +501,24 @@ def gpu_arm(args, d: Dist):
     reps = max(3, min(args.steps, 20))
     ms_rtn = sum(timed(lambda M=M: hs.hscale_rtn_scales(M.w, M.sg, M.codes0, work.ws), reps) for M in work.mats)
     sweep = []
-    for kk in sorted(set([k] + list(W.window))):
+    windows = sorted(set([win] + [(kk, kk) for kk in W.window]))
+    for dn, upw in windows:
         ms_ref = 0.0
         for M in work.mats:
-            ms_ref += timed(lambda M=M: hs.hscale_refine_scales(M.w, M.space.h, M.sg, M.codes0, kk, kk,
+            ms_ref += timed(lambda M=M: hs.hscale_refine_scales(M.w, M.space.h, M.sg, M.codes0, dn, upw,
                                                                  M.codes, M.packed), reps)
-        C = 2 * kk + 1
+        C = dn + upw + 1
         t_bytes = 42 * work.groups / (hbm_peak * 1e9)
         t_ops = 80 * C * work.groups / fp32_peak
-        sweep.append({"k": kk, "candidates": C, "ms": ms_ref, "groups_per_s": work.groups / (ms_ref * 1e-3),
+        sweep.append({"window": [dn, upw], "candidates": C, "ms": ms_ref,
+                      "groups_per_s": work.groups / (ms_ref * 1e-3),
                       "bound": "alu" if t_ops > t_bytes else "hbm", "roofline_ms": max(t_bytes, t_ops) * 1e3,
                       "frac": max(t_bytes, t_ops) / (ms_ref * 1e-3)})
     # restore the outputs of the step's own window
     scale_phase(hs, work)
     torch.cuda.synchronize()
-    main = [s for s in sweep if s["k"] == k][0]
+    main = [s for s in sweep if tuple(s["window"]) == tuple(win)][0]
+    shifts = shift_statistics(work, win)
 
     # ---- roofline of the dominant kernel (the Hessian pass)
     h_bytes_launch = work.h_bytes / work.h_launches
@@ -486,7 +539,7 @@ def gpu_arm(args, d: Dist):
         "config": {"workload": W.name,
                    "matrices": [[M.name, M.m, M.n] for M in work.mats],
                    "input_spaces": [[S.name, S.tokens, S.n, S.chunk] for S in work.spaces.values()],
-                   "k": k, "groups": work.groups,
+                   "window": list(win), "groups": work.groups,
                    "l2": "inputs larger than L2: %.2f GB of X streamed per step" %
                          (sum(S.tokens * S.n * 2 for S in work.spaces.values()) / 1e9),
                    "parallelism": f"independent layer per GPU x{d.world}"},
@@ -510,13 +563,14 @@ def gpu_arm(args, d: Dist):
     }
     if len(sweep) > 1:
         line["search_sweep"] = sweep
+    line["shift_statistics"] = shifts
     if n_layers > 1:
         line["seconds_per_model"] = ms_step * 1e-3 * n_layers
         line["seconds_per_model_note"] = f"{n_layers} layers of identical shapes: per-layer step x {n_layers}"
     if e2e:
         line["e2e"] = e2e
     if d.rank == 0 and d.world == 1 and not args.no_cpu_baseline:
-        cb = cpu_baseline(W, k)
+        cb = cpu_baseline(W, win)
         line["cpu_baseline"] = {k2: cb[k2] for k2 in ("value", "unit", "cores", "kind", "sample")}
     if d.rank == 0:
         print(json.dumps(line), flush=True)

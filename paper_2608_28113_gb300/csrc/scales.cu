@@ -197,7 +197,7 @@ __device__ __forceinline__ float exact_term(float a_k, float hj, uint32_t c, flo
 // The whole warp rescores the group of lane `owner` with exact rounding decisions and
 // returns its winning code (in every lane).  Lanes 0-15 take the candidates lo, lo+2,
 // ..., lanes 16-31 lo+1, lo+3, ...; lane j of each half scores element j & 15.
-__device__ int warp_exact_search(int owner, const uint4* w, int64_t g_own, const float* h,
+__device__ __noinline__ int warp_exact_search(int owner, const uint4* w, int64_t g_own, const float* h,
                                  int64_t hcol_own, int c0, int lo, int hi, float sgk, float pw) {
   const int lane = threadIdx.x & 31;
   const int j = lane & 15, half = lane >> 4;
@@ -237,38 +237,36 @@ __device__ __forceinline__ uint32_t cvt_e2m1x2(float hi, float lo) {
 // packed nibbles.  The raw-domain quotients y_raw = |w| * 2^-126 / s' are rescaled
 // exactly to real units, given the sign of w, and converted by the hardware E2M1
 // conversion (round-to-nearest-even).  That equals the exact rounding of |w| / s unless
-// some y_raw lies within 16 ulps of a midpoint; then every element is redone with the
-// exact midpoint test.
-__device__ __forceinline__ uint2 quantize_pack(const Group& G, uint32_t c, float2 t, float sgk) {
+// y_raw lies within 16 ulps of a midpoint; such elements are flagged and redone one by
+// one with the exact midpoint test, reading the weight back from `wg` (the group's 16
+// bf16 values in global memory).
+__device__ __forceinline__ uint2 quantize_pack(const Group& G, uint32_t c, float2 t, float sgk,
+                                               float pw, const uint16_t* wg) {
   const float2 ir2 = make_float2(t.y, t.y);
   const float2 up2 = make_float2(0x1p126f, 0x1p126f);
   uint32_t word[2] = {0u, 0u};
-  uint32_t near = 0xFFFFFFFFu;
+  uint32_t flagged = 0u;
 #pragma unroll
   for (int i = 0; i < 8; ++i) {
     const float2 yr = __fmul2_rn(G.a[i], ir2);
-    near = min(near, (__float_as_uint(yr.x) - 0x1FFFF0u) & 0x3FFFFFu);
-    near = min(near, (__float_as_uint(yr.y) - 0x1FFFF0u) & 0x3FFFFFu);
+    flagged |= (uint32_t)(((__float_as_uint(yr.x) - 0x1FFFF0u) & 0x3FFFFFu) <= 0x20u) << (2 * i);
+    flagged |= (uint32_t)(((__float_as_uint(yr.y) - 0x1FFFF0u) & 0x3FFFFFu) <= 0x20u) << (2 * i + 1);
     const float2 yv = __fmul2_rn(yr, up2);
     const float y0 = __uint_as_float(__float_as_uint(yv.x) | ((G.wb[i] << 16) & 0x80000000u));
     const float y1 = __uint_as_float(__float_as_uint(yv.y) | (G.wb[i] & 0x80000000u));
     word[i >> 2] |= cvt_e2m1x2(y1, y0) << (8 * (i & 3));
   }
-  if (near <= 0x20u) {
-    // rare: redo only the flagged elements with the exact midpoint test (static indices
-    // keep the group in registers)
+  if (flagged) {
     const float l = e4m3_mag(c);
-#pragma unroll
-    for (int j = 0; j < 16; ++j) {
-      const float a = (j & 1) ? G.a[j >> 1].y : G.a[j >> 1].x;
-      const float y = __fmul_rn(a, t.y);
-      if (e2m1_uncertain(y)) {
-        const uint32_t k = e2m1_exact_code(y, a, l, sgk);
-        const uint32_t sign = (j & 1) ? (G.wb[j >> 1] >> 31) : ((G.wb[j >> 1] >> 15) & 1u);
-        const int sh = 4 * (j & 7);
-        word[j >> 3] = (word[j >> 3] & ~(0xFu << sh)) | (((sign << 3) | k) << sh);
-      }
-    }
+    do {
+      const int j = __ffs(flagged) - 1;
+      flagged &= flagged - 1;
+      const uint32_t b = wg[j];
+      const float a = __fmul_rn(__uint_as_float((b & 0x7FFFu) << 16), pw);
+      const uint32_t k = e2m1_exact_code(__fmul_rn(a, t.y), a, l, sgk);
+      const int sh = 4 * (j & 7);
+      word[j >> 3] = (word[j >> 3] & ~(0xFu << sh)) | ((((b >> 15) << 3) | k) << sh);
+    } while (flagged);
   }
   return make_uint2(word[0], word[1]);
 }
@@ -276,8 +274,9 @@ __device__ __forceinline__ uint2 quantize_pack(const Group& G, uint32_t c, float
 // ---------------------------------------------------------------- refine (Algorithm 1)
 // Work unit: one warp, 32 consecutive groups of one row (a "row chunk"); warps stride
 // over (row, chunk) units so the h slice of a lane is reloaded only when its chunk
-// changes.
-__global__ void __launch_bounds__(kRefineThreads)
+// changes.  7 resident CTAs of 4 warps per SM (72 registers); the rarely taken
+// warp-cooperative rescoring is a separate call so it does not raise that.
+__global__ void __launch_bounds__(kRefineThreads, 7)
 refine_kernel(const uint4* __restrict__ w, const float* __restrict__ h, int64_t m, int ng,
               const float* __restrict__ global_scale, const uint8_t* init_codes,
               int down, int up, uint8_t* codes_out, uint2* __restrict__ packed_out) {
@@ -374,7 +373,9 @@ refine_kernel(const uint4* __restrict__ w, const float* __restrict__ h, int64_t 
 
     if (active) {
       codes_out[g] = (uint8_t)best;
-      if (packed_out != nullptr) packed_out[g] = quantize_pack(G, (uint32_t)best, tab[best], d.sgk);
+      if (packed_out != nullptr)
+        packed_out[g] = quantize_pack(G, (uint32_t)best, tab[best], d.sgk, d.pw,
+                                      reinterpret_cast<const uint16_t*>(w) + g * 16);
     }
   }
 }
@@ -391,7 +392,8 @@ __global__ void __launch_bounds__(256) pack_kernel(const uint4* __restrict__ w, 
     load_group(w, g, d.pw, G);
     uint32_t c = codes[g] & 0x7Fu;
     c = c < 1 ? 1u : (c > kE4M3MaxCode ? kE4M3MaxCode : c);
-    packed_out[g] = quantize_pack(G, c, candidate_constants(c, d.sgk), d.sgk);
+    packed_out[g] = quantize_pack(G, c, candidate_constants(c, d.sgk), d.sgk, d.pw,
+                                  reinterpret_cast<const uint16_t*>(w) + g * 16);
   }
 }
 

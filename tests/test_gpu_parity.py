@@ -359,7 +359,7 @@ def test_refine_is_deterministic():
 
 # ------------------------------------------------------------------ full-size workloads
 
-def full_size_check(name, sample_rows, layer_index=0):
+def full_size_check(name, sample_rows, layer_index=0, windows=None):
     """A workload at its full size in the launch configuration bench.py times: h of every
     input space over every streamed chunk (all columns, against the oracle fed the same
     chunks), s_g and RTN codes over every whole matrix, and the search with packing on a
@@ -391,16 +391,21 @@ def full_size_check(name, sample_rows, layer_index=0):
         assert sg.cpu().numpy()[0] == s_ref
         assert np.array_equal(codes.cpu().numpy(), oracle.rtn_codes(wb, s_ref))
         rows = np.sort(np.random.default_rng(seed).choice(m, size=min(sample_rows, m), replace=False))
-        for k in W.window:
-            codes_g, packed_g = gpu_refine(w, h_ref[L.input_space], sg, None, k, k)
-            ref = oracle.refine(wb[rows], h_ref[L.input_space], s_ref, None, k, k)
+        for down, up in (windows or [(k, k) for k in W.window]):
+            codes_g, packed_g = gpu_refine(w, h_ref[L.input_space], sg, None, down, up)
+            ref = oracle.refine(wb[rows], h_ref[L.input_space], s_ref, None, down, up)
             compare_search(ref, codes_g[rows], packed_g[rows],
-                           f"{name} {L.name} {m}x{n} k={k} ({rows.size} sampled rows)")
+                           f"{name} {L.name} {m}x{n} window -{down}/+{up} ({rows.size} sampled rows)")
         del w
 
 
 def test_full_size_llama8b_q_proj():
     full_size_check("llama8b-q_proj", sample_rows=512)
+
+
+def test_full_size_q_proj_paper_window_and_full_grid():
+    """The paper's default window (D = 9, U = 6, K = 16) and the whole E4M3 ladder."""
+    full_size_check("llama8b-q_proj", sample_rows=64, windows=[(9, 6), (125, 125)])
 
 
 def test_full_size_mlp_down_proj():
