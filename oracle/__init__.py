@@ -11,6 +11,7 @@ Function map (paper equations in their order of appearance):
   global_scale         s_g = amax|W| / (6*448)               Sec. 3.1 (formula is a reading)
   rtn_codes            iota(Q_fp8(amax_group / (6 s_g)))     Sec. 3.3, Eq. 7
   refine               Algorithm 1 with diagnostics          Eqs. 8-13
+  fourover6_codes      Algorithm 2's 4over6 initialization   Sec. 3.5, Algorithm 2
   pack                 final FP4 quantization                Sec. 3.3, Eq. 2
   quantize_at_scale    Eq. 2 at a real scale (App. A.1 microcase)
   output_error         ||X dW^T||_F^2                        Eq. 3
@@ -67,6 +68,7 @@ def _load():
             "oracle_refine": (None, [P, P, i64, i64, f32, P, i32, i32, P, P, P, P, P, P, P]),
             "oracle_group_errors": (None, [P, P, f32, P, i32, P]),
             "oracle_pack": (None, [P, i64, i64, f32, P, P]),
+            "oracle_fourover6_codes": (None, [P, i64, i64, f32, P, P]),
             "oracle_quantize_at_scale": (None, [P, i64, f64, P, P]),
             "oracle_output_error": (f64, [P, i64, i64, P, i64]),
         }
@@ -180,6 +182,16 @@ def group_errors(g16_u16: np.ndarray, h16: np.ndarray | None, s_g, codes) -> np.
     _load().oracle_group_errors(_ptr(g), _ptr(h), float(np.float32(s_g)), _ptr(c), c.size,
                                 _ptr(err))
     return err
+
+
+def fourover6_codes(w_u16: np.ndarray, s_g) -> tuple[np.ndarray, np.ndarray]:
+    """Algorithm 2's initial codes [m, n/16] and the anchor near-tie flags."""
+    w = _u16(w_u16)
+    m, n = w.shape
+    codes = np.empty((m, n // 16), np.uint8)
+    nt = np.empty((m, n // 16), np.uint8)
+    _load().oracle_fourover6_codes(_ptr(w), m, n, float(np.float32(s_g)), _ptr(codes), _ptr(nt))
+    return codes, nt
 
 
 def pack(w_u16: np.ndarray, s_g, codes: np.ndarray) -> np.ndarray:

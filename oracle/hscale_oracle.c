@@ -27,6 +27,8 @@
  *                               E4M3 ladder (Eqs. 8-10), candidate set (Eq. 11), FP4
  *                               projection (Eq. 12), argmin of the diagonal-Hessian
  *                               weighted error (Eqs. 6 and 13), final re-quantization
+ *   oracle_fourover6_codes      Algorithm 2's initialization: the better of the anchors
+ *                               m/4 and m/6 by plain MSE (Sec. 3.5, Algorithm 2)
  *   oracle_pack                 final FP4 quantization with given local scales (Sec. 3.3
  *                               "Final re-quantization"; quantizer of Eq. 2)
  *   oracle_quantize_at_scale    Eq. 2 at a real scale s (calibration microcase, App. A.1)
@@ -320,6 +322,49 @@ void oracle_refine(const uint16_t* w, const float* h, int64_t m, int64_t n, floa
 void oracle_group_errors(const uint16_t* g16, const float* h16, float s_g, const uint8_t* codes,
                          int count, double* err) {
   for (int k = 0; k < count; ++k) err[k] = group_error(g16, h16, (double)s_g, codes[k], NULL);
+}
+
+/* ------------------------------------------------------------------ */
+/* Algorithm 2, 4over6 initialization (the part before HScaleGroupQuantize) */
+/* ------------------------------------------------------------------ */
+/* For every group: m = max|w|; for each anchor c in C = {4, 6}, in that order,
+ *   l_c = Q_fp8(m / (c s_g))   (round-to-nearest-even, saturating; code 0 clamps to 1,
+ *                               the same reading as Eq. 7)
+ *   L(c) = || w - Q_fp4(w / (s_g l_c)) s_g l_c ||^2      (plain weight MSE)
+ * and the initial code is the code of argmin_c L(c); the first anchor in the order of C
+ * wins an exact tie (a reading: the paper writes argmin over C without a tie rule).
+ * near_tie (may be NULL): 1 iff the two anchors give different codes whose errors are
+ * within 1e-6 relative of each other. */
+void oracle_fourover6_codes(const uint16_t* w, int64_t m, int64_t n, float s_g_f,
+                            uint8_t* codes_out, uint8_t* near_tie) {
+  const int64_t ng = n / 16;
+  const double s_g = (double)s_g_f;
+#pragma omp parallel for schedule(static)
+  for (int64_t r = 0; r < m; ++r) {
+    for (int64_t i = 0; i < ng; ++i) {
+      const uint16_t* g = w + r * n + i * 16;
+      double mx = 0.0;
+      for (int j = 0; j < 16; ++j) {
+        double a = fabs(bf16_value(g[j]));
+        if (a > mx) mx = a;
+      }
+      const double anchors[2] = {4.0, 6.0};
+      int code[2];
+      double err[2];
+      for (int k = 0; k < 2; ++k) {
+        int c = e4m3_rne_sat_quotient(mx, anchors[k], s_g);
+        code[k] = c < 1 ? 1 : c;
+        err[k] = group_error(g, NULL, s_g, code[k], NULL);
+      }
+      const int pick = err[1] < err[0] ? 1 : 0;
+      codes_out[r * ng + i] = (uint8_t)code[pick];
+      if (near_tie) {
+        const double hi = err[0] > err[1] ? err[0] : err[1];
+        const double lo = err[0] > err[1] ? err[1] : err[0];
+        near_tie[r * ng + i] = (uint8_t)(code[0] != code[1] && hi - lo <= 1e-6 * hi);
+      }
+    }
+  }
 }
 
 /* ------------------------------------------------------------------ */

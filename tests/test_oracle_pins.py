@@ -378,3 +378,52 @@ def test_zero_groups_and_negative_zero():
     assert out["codes"][0, 0] == 1 and out["delta"][0, 0] == 0 and out["near_tie"][0, 0] == 1
     assert out["packed"][0, 2] == 0x80                       # -0 (odd element: high nibble) keeps its sign
     assert out["codes"][1, 1] == 126 or out["e_best"][1, 1] == 0.0
+
+
+# ---------------------------------------------------------------- Algorithm 2 (4over6 initialization)
+
+def brute_force_fourover6(g_bits, s_g):
+    """Algorithm 2's initialization by brute force: torch's E4M3 cast of the fp64 quotient
+    (valid away from midpoints), nearest-value FP4 search, anchors in the order 4, 6."""
+    a = np.abs(bits_to_f64(g_bits))
+    mx = a.max()
+    ladder = oracle.e4m3_decode_table()
+    best = None
+    for c in (4.0, 6.0):
+        q = mx / (c * float(s_g))
+        code = int(e4m3_code_by_torch(np.array([q]))[0])
+        code = 126 if code == 127 else max(code, 1)
+        s = float(s_g) * ladder[code]
+        err = math.fsum((v - E2M1_GRID[nearest_e2m1(v, s)] * s) ** 2 for v in a)
+        if best is None or err < best[1]:
+            best = (code, err)
+    return best[0]
+
+
+def test_fourover6_codes_against_brute_force_and_rtn():
+    rng = np.random.default_rng(13)
+    w = random_weights(rng, 16, 256)
+    s_g, _ = oracle.global_scale(w)
+    codes, nt = oracle.fourover6_codes(w, s_g)
+    rtn = oracle.rtn_codes(w, s_g)
+    for r in range(16):
+        for i in range(16):
+            if nt[r, i]:
+                continue
+            assert codes[r, i] == brute_force_fourover6(w[r, 16 * i:16 * i + 16], s_g)
+    # the anchor 6 is the RTN code of Eq. 7; 4over6 never has a larger MSE than RTN
+    e_fo6 = oracle.refine(w, None, s_g, codes, 0, 0)["e_best"]
+    e_rtn = oracle.refine(w, None, s_g, rtn, 0, 0)["e_best"]
+    assert np.all(e_fo6 <= e_rtn * (1 + 1e-12))
+    assert (codes != rtn).any() and (codes == rtn).any()
+
+
+def test_fourover6_saturated_group_keeps_the_top_code():
+    # the group holding amax: m/(6 s_g) = 448 and m/(4 s_g) = 672 both saturate to 448
+    w = np.zeros((1, 32))
+    w[0, 5] = 2688 * 2.0 ** -10
+    w[0, 20] = 0.01
+    bits = to_bf16_bits(w)
+    s_g, _ = oracle.global_scale(bits)
+    codes, nt = oracle.fourover6_codes(bits, s_g)
+    assert codes[0, 0] == 126 and nt[0, 0] == 0
