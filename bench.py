@@ -56,6 +56,8 @@ def parse():
                    help="asymmetric window 'D,U' (codes c0-D .. c0+U); e.g. 9,6 is the paper's K = 16 default")
     p.add_argument("--tokens", type=int, default=None,
                    help="calibration tokens per input space (default: the workload's; smaller for ncu captures)")
+    p.add_argument("--init", choices=["rtn", "4over6"], default="rtn",
+                   help="initial codes of the search: max-abs RTN (Eq. 7) or 4over6 (Algorithm 2)")
     p.add_argument("--no-cpu-baseline", action="store_true")
     p.add_argument("--no-e2e", action="store_true")
     return p.parse_args()
@@ -232,8 +234,8 @@ class Matrix:
 class Work:
     """Device-resident inputs and outputs of one layer of a workload."""
 
-    def __init__(self, W: wl.Workload, rank: int, win, device, tokens=None):
-        self.W, self.win = W, tuple(win)
+    def __init__(self, W: wl.Workload, rank: int, win, device, tokens=None, init="rtn"):
+        self.W, self.win, self.init = W, tuple(win), init
         self.seed = W.layer_seed(0) + 7919 * rank
         self.spaces = {name: Space(W, name, n, self.seed, device, tokens) for name, n in W.input_spaces()}
         self.mats = [Matrix(W, L, self.spaces[L.input_space], self.seed, device) for L in W.layers]
@@ -252,13 +254,24 @@ def hessian_phase(hs, work: Work, xs=None):
             hs.hscale_hessian_diag_accumulate(x[c * S.chunk:(c + 1) * S.chunk], S.h)
 
 
+def init_codes(hs, work: Work, M, w=None):
+    """Global scale and the search's initial codes of one matrix: max-abs RTN codes
+    (Eq. 7), or, with 4over6 init, s_g alone followed by Algorithm 2's codes."""
+    w = M.w if w is None else w
+    if work.init == "4over6":
+        hs.hscale_rtn_scales(w, M.sg, None, work.ws)
+        hs.hscale_fourover6_codes(w, M.sg, M.codes0)
+    else:
+        hs.hscale_rtn_scales(w, M.sg, M.codes0, work.ws)
+
+
 def scale_phase(hs, work: Work, win=None, ws=None):
-    """For every matrix: global scale + RTN codes, then the H-Scale search with packing
-    over the window win = (down, up)."""
+    """For every matrix: global scale + initial codes, then the H-Scale search with
+    packing over the window win = (down, up)."""
     down, up = work.win if win is None else win
     for M in work.mats:
         w = M.w if ws is None else ws[M.name]
-        hs.hscale_rtn_scales(w, M.sg, M.codes0, work.ws)
+        init_codes(hs, work, M, w)
         hs.hscale_refine_scales(w, M.space.h, M.sg, M.codes0, down, up, M.codes, M.packed)
 
 
@@ -291,7 +304,7 @@ def capture_graphs(hs, work: Work):
     return gh, gs
 
 
-KERNELS_PER_MATRIX = 3  # amax, RTN codes, refine
+KERNELS_PER_MATRIX = 3  # amax, RTN or 4over6 codes, refine
 
 
 def timed(fn, reps):
@@ -315,10 +328,11 @@ def window_of(args, W: wl.Workload):
     return (k, k)
 
 
-def cpu_baseline(W: wl.Workload, win, budget_s: float = 12.0):
+def cpu_baseline(W: wl.Workload, win, budget_s: float = 12.0, init: str = "rtn"):
     """Time the fp64 oracle on a bounded sample of the workload and extrapolate the
-    whole-step time: Hessian over sampled tokens of every input space, global scale + RTN
-    over every matrix, search over sampled rows of every matrix."""
+    whole-step time: Hessian over sampled tokens of every input space, global scale +
+    initial codes (RTN or 4over6) over every matrix, search over sampled rows of every
+    matrix."""
     import oracle
     oracle.build()
     cores = len(os.sched_getaffinity(0)) if hasattr(os, "sched_getaffinity") else os.cpu_count()
@@ -352,14 +366,14 @@ def cpu_baseline(W: wl.Workload, win, budget_s: float = 12.0):
         wb = wl.bf16_bits(wl.weight(m, n, W.sigma_w, W.seed))
         t0 = time.perf_counter()
         s_g, _ = oracle.global_scale(wb)
-        oracle.rtn_codes(wb, s_g)
+        c0 = oracle.fourover6_codes(wb, s_g)[0] if init == "4over6" else oracle.rtn_codes(wb, s_g)
         t_rtn_total += time.perf_counter() - t0
         rows = max(8, min(m, 64))
         t0 = time.perf_counter()
         done = 0
         while True:
             r0 = (done * rows) % m
-            oracle.refine(wb[r0:r0 + rows], hs_of[L.input_space], s_g, None, win[0], win[1])
+            oracle.refine(wb[r0:r0 + rows], hs_of[L.input_space], s_g, c0[r0:r0 + rows], win[0], win[1])
             done += 1
             if time.perf_counter() - t0 > per_part:
                 break
@@ -373,7 +387,7 @@ def cpu_baseline(W: wl.Workload, win, budget_s: float = 12.0):
         "value": groups / step, "unit": UNIT, "cores": cores, "kind": "oracle",
         "sample": (f"fp64 C oracle, {cores} threads, bounded sample extrapolated to the step "
                    f"({W.tokens} tokens per input space, {groups} groups, window -{win[0]}/+{win[1]}): "
-                   + "; ".join(samples) + "; global scale + RTN over every whole matrix"),
+                   + "; ".join(samples) + f"; global scale + {init} codes over every whole matrix"),
         "seconds_per_step": step,
         "hessian_tokens_channels_per_s": h_tc / max(step, 1e-30),
     }
@@ -388,7 +402,7 @@ def reference_arm(args, d: Dist):
     vals = []
     cb = None
     for i in range(args.warmup + args.steps):
-        cb = cpu_baseline(W, win, budget_s=3.0)
+        cb = cpu_baseline(W, win, budget_s=3.0, init=args.init)
         if i >= args.warmup:
             vals.append(cb["seconds_per_step"])
     groups = sum(L.out_features * L.in_features // 16 for L in W.layers)
@@ -400,7 +414,7 @@ def reference_arm(args, d: Dist):
         "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
         "data": "synthetic",
         "config": {"workload": W.name, "matrices": [[L.name, L.out_features, L.in_features] for L in W.layers],
-                   "tokens": W.tokens, "window": list(win)},
+                   "tokens": W.tokens, "window": list(win), "init": args.init},
         "cpu_baseline": {"value": value, "unit": UNIT, "cores": cb["cores"], "kind": "oracle",
                          "sample": cb["sample"]},
         "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
@@ -454,7 +468,7 @@ def gpu_arm(args, d: Dist):
     dev = torch.device("cuda", d.local)
     W = wl.WORKLOADS[args.workload]
     win = window_of(args, W)
-    work = Work(W, d.rank, win, dev, tokens=args.tokens)
+    work = Work(W, d.rank, win, dev, tokens=args.tokens, init=args.init)
     work.ws = torch.empty(hs.hscale_rtn_workspace_bytes(), dtype=torch.uint8, device=dev)
     torch.cuda.synchronize()
 
@@ -499,7 +513,7 @@ def gpu_arm(args, d: Dist):
     sm_max_mhz = float(peaks.get("sm_max_mhz", 2070.0))
     fp32_peak = props.multi_processor_count * 128 * sm_max_mhz * 1e6
     reps = max(3, min(args.steps, 20))
-    ms_rtn = sum(timed(lambda M=M: hs.hscale_rtn_scales(M.w, M.sg, M.codes0, work.ws), reps) for M in work.mats)
+    ms_init = sum(timed(lambda M=M: init_codes(hs, work, M), reps) for M in work.mats)
     sweep = []
     windows = sorted(set([win] + [(kk, kk) for kk in W.window]))
     for dn, upw in windows:
@@ -539,7 +553,7 @@ def gpu_arm(args, d: Dist):
         "config": {"workload": W.name,
                    "matrices": [[M.name, M.m, M.n] for M in work.mats],
                    "input_spaces": [[S.name, S.tokens, S.n, S.chunk] for S in work.spaces.values()],
-                   "window": list(win), "groups": work.groups,
+                   "window": list(win), "init": work.init, "groups": work.groups,
                    "l2": "inputs larger than L2: %.2f GB of X streamed per step" %
                          (sum(S.tokens * S.n * 2 for S in work.spaces.values()) / 1e9),
                    "parallelism": f"independent layer per GPU x{d.world}"},
@@ -548,7 +562,7 @@ def gpu_arm(args, d: Dist):
                      "peak_kind": f"{peak_kind} HBM copy bandwidth",
                      "frac_of_8TBs_spec": h_gbs / HBM_SPEC_GBS, "traffic": traffic,
                      "bytes_per_launch": h_bytes_launch, "ms_per_launch": ms_h_launch},
-        "phases_ms": {"hessian": ms_h, "scales": ms_sc, "rtn_scales": ms_rtn, "refine": main["ms"]},
+        "phases_ms": {"hessian": ms_h, "scales": ms_sc, "init_codes": ms_init, "refine": main["ms"]},
         "ms_per_step_eager": ms_eager,
         "timed_launch": "CUDA graphs of the step's API calls (Hessian pass; scales)",
         "hessian": {"gbs": h_gbs, "tokens_channels_per_s": work.h_bytes / 2 / (ms_h * 1e-3),
@@ -570,7 +584,7 @@ def gpu_arm(args, d: Dist):
     if e2e:
         line["e2e"] = e2e
     if d.rank == 0 and d.world == 1 and not args.no_cpu_baseline:
-        cb = cpu_baseline(W, win)
+        cb = cpu_baseline(W, win, init=args.init)
         line["cpu_baseline"] = {k2: cb[k2] for k2 in ("value", "unit", "cores", "kind", "sample")}
     if d.rank == 0:
         print(json.dumps(line), flush=True)

@@ -17,6 +17,8 @@
  *                                       (Eqs. 6, 13), then re-quantize and pack
  *      hscale_pack_nvfp4                final FP4 quantization with given codes
  *                                       (Sec. 3.3 "Final re-quantization", Eq. 2)
+ *      hscale_fourover6_codes           the 4over6 initial codes of Algorithm 2, an
+ *                                       alternative start for the refinement (Sec. 3.5)
  *
  * Equation numbers count the paper's displayed equations in order (Eq. 1 is the
  * effective scale s = s_g * l).
@@ -142,6 +144,23 @@ int hscale_rtn_scales(const void* w_bf16, int64_t m, int64_t n, float* global_sc
 #define HSCALE_NOALLOC_SCRATCH_BYTES 256
 int hscale_rtn_scales_noalloc(const void* w_bf16, int64_t m, int64_t n, float* global_scale,
                               uint8_t* codes, void* stream);
+
+/*
+ * 4over6 initial codes (Algorithm 2, the part before HScaleGroupQuantize), to be refined
+ * by hscale_refine_scales as its init_codes.
+ *
+ * For every group with m = max|w|, the anchors c in C = {4, 6} give the codes
+ * max(1, RNE_E4M3_sat(m / (c s_g))) (each as in Eq. 7); the code whose group has the
+ * smaller plain weight MSE sum_j (|w_j| - q_j s)^2 (exact E2M1 round-to-nearest-even
+ * decisions) is written.  The anchor 4, first in C, wins an exact tie; errors within about
+ * 1e-6 relative may be ordered either way (fp32 sums).
+ *
+ * w             [m, n] bfloat16, 16-byte aligned, n % 16 == 0.
+ * global_scale  device fp32 scalar s_g (e.g. from hscale_rtn_scales with codes = NULL).
+ * codes         [m, n/16] bytes, written.
+ */
+int hscale_fourover6_codes(const void* w_bf16, int64_t m, int64_t n, const float* global_scale,
+                           uint8_t* codes, void* stream);
 
 /*
  * H-Scale refinement, Algorithm 1 (Eqs. 6-13), fused with the final re-quantization.

@@ -10,7 +10,7 @@ raises.
 Paper map: ``hscale_hessian_diag_accumulate`` is h = diag(X^T X) (Sec. 3.2, Eq. 4);
 ``hscale_rtn_scales`` the global scale and RTN codes (Sec. 3.3, Eq. 7);
 ``hscale_refine_scales`` Algorithm 1 (Eqs. 6-13); ``hscale_pack_nvfp4`` the final
-re-quantization (Sec. 3.3).
+re-quantization (Sec. 3.3); ``hscale_fourover6_codes`` the 4over6 start of Algorithm 2.
 """
 from __future__ import annotations
 
@@ -25,7 +25,7 @@ __all__ = [
     "hscale_device_error_flags",
     "hscale_hessian_diag_accumulate", "hscale_rtn_workspace_bytes", "hscale_rtn_scales",
     "hscale_rtn_scales_noalloc",
-    "hscale_refine_scales", "hscale_pack_nvfp4", "EXPORTED_SYMBOLS",
+    "hscale_refine_scales", "hscale_pack_nvfp4", "hscale_fourover6_codes", "EXPORTED_SYMBOLS",
 ]
 
 _PKG = pathlib.Path(__file__).resolve().parent
@@ -45,6 +45,7 @@ _SIGNATURES = {
     "hscale_rtn_scales_noalloc": (ctypes.c_int, [_P, _I64, _I64, _P, _P, _P]),
     "hscale_refine_scales": (ctypes.c_int, [_P, _P, _I64, _I64, _P, _P, _I32, _I32, _P, _P, _P]),
     "hscale_pack_nvfp4": (ctypes.c_int, [_P, _I64, _I64, _P, _P, _P, _P]),
+    "hscale_fourover6_codes": (ctypes.c_int, [_P, _I64, _I64, _P, _P, _P]),
 }
 EXPORTED_SYMBOLS = tuple(_SIGNATURES)
 
@@ -215,3 +216,19 @@ def hscale_pack_nvfp4(w: torch.Tensor, global_scale: torch.Tensor, codes: torch.
     _check("hscale_pack_nvfp4",
            load().hscale_pack_nvfp4(_ptr(w), m, n, _ptr(global_scale), _ptr(codes),
                                     _ptr(packed_out), _stream_ptr(stream)))
+
+
+def hscale_fourover6_codes(w: torch.Tensor, global_scale: torch.Tensor, codes: torch.Tensor,
+                           stream=None) -> None:
+    """Algorithm 2's 4over6 initial codes [m, n/16] (input to hscale_refine_scales)."""
+    _need(w, torch.bfloat16, "w")
+    _need(global_scale, torch.float32, "global_scale")
+    _need(codes, torch.uint8, "codes")
+    if not w.is_contiguous() or w.dim() != 2:
+        raise ValueError("w must be a contiguous 2-D tensor")
+    m, n = w.shape
+    if codes.numel() != m * (n // 16) or not codes.is_contiguous():
+        raise ValueError("codes must be contiguous [m, n/16]")
+    _check("hscale_fourover6_codes",
+           load().hscale_fourover6_codes(_ptr(w), m, n, _ptr(global_scale), _ptr(codes),
+                                         _stream_ptr(stream)))

@@ -124,6 +124,16 @@ int hscale_refine_scales(const void* w_bf16, const float* h, int64_t m, int64_t 
                                          codes_out, packed_out, as_stream(stream)));
 }
 
+int hscale_fourover6_codes(const void* w_bf16, int64_t m, int64_t n, const float* global_scale,
+                           uint8_t* codes, void* stream) {
+  int st = check_weight(w_bf16, m, n);
+  if (st != HSCALE_OK) return st;
+  if (m == 0 || n == 0) return HSCALE_OK;
+  if (global_scale == nullptr || codes == nullptr) return HSCALE_ERR_NULL;
+  if (!aligned(global_scale, 4)) return HSCALE_ERR_ALIGN;
+  return from_cuda(hscale::launch_fourover6(w_bf16, m, n, global_scale, codes, as_stream(stream)));
+}
+
 int hscale_pack_nvfp4(const void* w_bf16, int64_t m, int64_t n, const float* global_scale,
                       const uint8_t* codes, uint8_t* packed_out, void* stream) {
   int st = check_weight(w_bf16, m, n);

@@ -85,32 +85,38 @@ __device__ __forceinline__ ScaleDomain make_scale_domain(float sg) {
 }
 
 // ---------------------------------------------------------------- RTN code (Eq. 7)
-// code = max(1, RNE_E4M3_sat(amax_g / (6 s_g))), decided exactly.  amax_k = amax_g * 2^-K.
-// An fp32 estimate of the quotient picks a code within one step; the two midpoints
-// next to it are then checked exactly: 6 * mu has <= 7 significant bits and one FMA
-// rounds once, so the sign of fma(-6 mu, sgk, amax_k) is the sign of amax_g - 6 mu s_g.
-// Ties go to the even code.
-__device__ __forceinline__ uint32_t rtn_code(float amax_k, float sgk, float inv6_raw) {
-  const float r_raw = __fmul_rn(amax_k, inv6_raw);  // ~ amax_g / (6 s_g) * 2^-120
+// code = max(1, RNE_E4M3_sat(amax_g / (c s_g))) for an anchor c = 2 * half_c (6 for the
+// max-abs RTN scale of Eq. 7; 4 and 6 for the 4over6 anchors of Algorithm 2), decided
+// exactly.  amax_k = amax_g * 2^-K, inv_raw = 2^-120 / (c sgk).  An fp32 estimate of the
+// quotient picks a code within one step; the two midpoints next to it are then checked
+// exactly: c * mu has <= 7 significant bits and one FMA rounds once, so the sign of
+// fma(-c mu, sgk, amax_k) is the sign of amax_g - c mu s_g.  Ties go to the even code.
+__device__ __forceinline__ uint32_t anchored_code(float amax_k, float sgk, float inv_raw, float half_c) {
+  const float r_raw = __fmul_rn(amax_k, inv_raw);  // ~ amax_g / (c s_g) * 2^-120
   uint32_t c = (__float_as_uint(r_raw) + (1u << 19)) >> 20;
   c = min(c, kE4M3MaxCode);
   if (c < kE4M3MaxCode) {
-    const float mu6 = __fmul_rn(3.0f, __fadd_rn(e4m3_mag(c), e4m3_mag(c + 1)));
-    const float t = __fmaf_rn(-mu6, sgk, amax_k);
+    const float muc = __fmul_rn(half_c, __fadd_rn(e4m3_mag(c), e4m3_mag(c + 1)));
+    const float t = __fmaf_rn(-muc, sgk, amax_k);
     if (t > 0.0f || (t == 0.0f && ((c + 1) & 1u) == 0)) c += 1;
   }
   if (c > 0) {
-    const float mu6 = __fmul_rn(3.0f, __fadd_rn(e4m3_mag(c - 1), e4m3_mag(c)));
-    const float t = __fmaf_rn(-mu6, sgk, amax_k);
+    const float muc = __fmul_rn(half_c, __fadd_rn(e4m3_mag(c - 1), e4m3_mag(c)));
+    const float t = __fmaf_rn(-muc, sgk, amax_k);
     if (t < 0.0f || (t == 0.0f && ((c - 1) & 1u) == 0)) c -= 1;
   }
   return c < 1 ? 1u : c;
 }
 
-// 2^-120 / (6 sgk): the factor rtn_code multiplies amax_k by (a normal number).
-__device__ __forceinline__ float rtn_inv6_raw(float sgk) {
-  return __fdiv_rn(0x1p-120f, __fmul_rn(6.0f, sgk));
+__device__ __forceinline__ uint32_t rtn_code(float amax_k, float sgk, float inv6_raw) {
+  return anchored_code(amax_k, sgk, inv6_raw, 3.0f);
 }
+
+// 2^-120 / (c sgk): the factor anchored_code multiplies amax_k by (a normal number).
+__device__ __forceinline__ float anchor_inv_raw(float sgk, float c) {
+  return __fdiv_rn(0x1p-120f, __fmul_rn(c, sgk));
+}
+__device__ __forceinline__ float rtn_inv6_raw(float sgk) { return anchor_inv_raw(sgk, 6.0f); }
 
 // ---------------------------------------------------------------- E2M1 projection (Eq. 12)
 // Fast rounding of y_raw = (|w| / s) * 2^-126 to the E2M1 grid: round-half-up on the

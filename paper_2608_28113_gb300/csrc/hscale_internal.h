@@ -29,6 +29,10 @@ cudaError_t launch_refine(const void* w, const float* h, int64_t m, int64_t n,
                           const float* global_scale, const uint8_t* init_codes, int down, int up,
                           uint8_t* codes_out, uint8_t* packed_out, cudaStream_t stream);
 
+// Algorithm 2's initial codes (the better of the anchors m/4, m/6 by plain MSE).
+cudaError_t launch_fourover6(const void* w, int64_t m, int64_t n, const float* global_scale,
+                             uint8_t* codes, cudaStream_t stream);
+
 // Sticky device error flags of this library (bit 0: a bounded wait ran out); cleared on read.
 cudaError_t read_and_clear_device_error(uint32_t* flags);
 

@@ -399,6 +399,52 @@ __global__ void __launch_bounds__(256) pack_kernel(const uint4* __restrict__ w, 
 
 // Resident CTAs per SM of a kernel, queried once per kernel and device (the query is
 // not repeated under stream capture).
+// ---------------------------------------------------------------- 4over6 init (Algorithm 2)
+// Plain-MSE error of one group under code c with exact rounding decisions: one rounding
+// in each residual (q * l is exact inside the FMA), the square, and a fixed pairwise
+// 16-term sum; relative error <= 7 * 2^-24.
+__device__ __forceinline__ float exact_group_mse(const Group& G, uint32_t c, float sgk) {
+  const float l = e4m3_mag(c);
+  const float inv = inv_raw_of(__fmul_rn(l, sgk));
+  float t[16];
+#pragma unroll
+  for (int j = 0; j < 16; ++j) {
+    const float a = (j & 1) ? G.a[j >> 1].y : G.a[j >> 1].x;
+    const uint32_t k = e2m1_code(a, inv, l, sgk);
+    const float r = __fmaf_rn(-__fmul_rn(e2m1_from_raw(k << 22), l), sgk, a);
+    t[j] = __fmul_rn(r, r);
+  }
+#pragma unroll
+  for (int step = 1; step < 16; step <<= 1)
+#pragma unroll
+    for (int j = 0; j + step < 16; j += 2 * step) t[j] = __fadd_rn(t[j], t[j + step]);
+  return t[0];
+}
+
+// Initial codes of Algorithm 2: for m = max|w| of the group, the E4M3 codes of m / (4 s_g)
+// and m / (6 s_g) (each as in Eq. 7), and the one whose group has the smaller plain MSE;
+// the anchor 4 (first in C = {4, 6}) wins an exact tie.
+__global__ void __launch_bounds__(256) fourover6_codes_kernel(const uint4* __restrict__ w, int64_t groups,
+                                                              const float* __restrict__ global_scale,
+                                                              uint8_t* __restrict__ codes) {
+  const ScaleDomain d = make_scale_domain(*global_scale);
+  const float inv4 = anchor_inv_raw(d.sgk, 4.0f);
+  const float inv6 = anchor_inv_raw(d.sgk, 6.0f);
+  const int64_t stride = (int64_t)gridDim.x * blockDim.x;
+  for (int64_t g = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; g < groups; g += stride) {
+    Group G;
+    load_group(w, g, d.pw, G);
+    const uint32_t amax = group_abs_max_bits(make_uint4(G.wb[0], G.wb[1], G.wb[2], G.wb[3]),
+                                             make_uint4(G.wb[4], G.wb[5], G.wb[6], G.wb[7]));
+    const float amax_k = __fmul_rn(__uint_as_float(amax << 16), d.pw);
+    const uint32_t c4 = anchored_code(amax_k, d.sgk, inv4, 2.0f);
+    const uint32_t c6 = anchored_code(amax_k, d.sgk, inv6, 3.0f);
+    uint32_t c = c4;
+    if (c6 != c4 && exact_group_mse(G, c6, d.sgk) < exact_group_mse(G, c4, d.sgk)) c = c6;
+    codes[g] = (uint8_t)c;
+  }
+}
+
 template <typename K>
 int occupancy_blocks(K kernel, int threads) {
   static int cache[64] = {0};
@@ -453,6 +499,19 @@ cudaError_t launch_refine(const void* w, const float* h, int64_t m, int64_t n,
   refine_kernel<<<(unsigned)blocks, kRefineThreads, 0, stream>>>(
       static_cast<const uint4*>(w), h, m, ng, global_scale, init_codes, down, up, codes_out,
       reinterpret_cast<uint2*>(packed_out));
+  return cudaGetLastError();
+}
+
+cudaError_t launch_fourover6(const void* w, int64_t m, int64_t n, const float* global_scale,
+                             uint8_t* codes, cudaStream_t stream) {
+  DeviceInfo info;
+  cudaError_t err = current_device_info(&info);
+  if (err != cudaSuccess) return err;
+  const int64_t groups = m * (n / 16);
+  int64_t blocks = (groups + 255) / 256;
+  blocks = std::max<int64_t>(1, std::min<int64_t>(blocks, (int64_t)info.sm_count * occupancy_blocks(fourover6_codes_kernel, 256)));
+  fourover6_codes_kernel<<<(unsigned)blocks, 256, 0, stream>>>(static_cast<const uint4*>(w), groups,
+                                                                global_scale, codes);
   return cudaGetLastError();
 }
 

@@ -357,13 +357,111 @@ def test_refine_is_deterministic():
     assert np.array_equal(a[0], b[0]) and np.array_equal(a[1], b[1])
 
 
+# ------------------------------------------------------------------ 4over6 initialization (Algorithm 2)
+
+def gpu_fourover6(w, sg):
+    m, n = w.shape
+    codes = torch.empty(m, n // 16, dtype=torch.uint8, device=dev())
+    hs.hscale_fourover6_codes(w, sg, codes)
+    torch.cuda.synchronize()
+    return codes.cpu().numpy()
+
+
+def compare_init(ref_codes, near_tie, codes, label=""):
+    """4over6 codes: bit-exact except where the two anchors' errors are a near-tie."""
+    nt = near_tie.astype(bool)
+    diff = codes != ref_codes
+    bad = diff & ~nt
+    assert not bad.any(), f"{label}: {bad.sum()} 4over6 code mismatches at {np.argwhere(bad)[:5]}"
+    print(f"[parity] 4over6 {label}: groups={codes.size} anchor_near_ties={int(nt.sum())} "
+          f"near_tie_mismatches={int((diff & nt).sum())}")
+    return diff
+
+
+@pytest.mark.parametrize("seed,m,n", [(0, 512, 1024), (1, 512, 1024), (2, 256, 4096),
+                                      (5, 1, 16), (6, 3, 48), (7, 33, 16 * 33)])
+def test_fourover6_codes_match_oracle(seed, m, n):
+    w = wl.weight(m, n, 0.02, seed)
+    wd = w.to(dev())
+    sg, _ = gpu_rtn(wd)
+    s_ref, _ = oracle.global_scale(bits(w))
+    ref, nt = oracle.fourover6_codes(bits(w), s_ref)
+    codes = gpu_fourover6(wd, sg)
+    diff = compare_init(ref, nt, codes, f"{m}x{n} seed {seed}")
+    # both anchors are used on real-looking weights
+    if m * n >= 512 * 1024:
+        rtn = oracle.rtn_codes(bits(w), s_ref)
+        assert 0.05 < float(np.mean(codes == rtn)) < 0.95
+    assert not diff.all()
+
+
+def test_fourover6_exact_ties_and_edge_groups():
+    """s_g = 2^-7; groups whose elements sit on both anchors' grids (zero error at both
+    codes: the tie keeps anchor 4), all-zero and -0 groups, tiny groups (both codes clip
+    to 1), the saturated group that holds amax (both codes 126)."""
+    rng = np.random.default_rng(21)
+    m, n = 96, 256
+    lad = oracle.e4m3_decode_table()[1:127]
+    pairs = [(l6, 1.5 * l6) for l6 in lad if 1.5 * l6 in set(lad)]
+    w = (rng.standard_t(4, size=(m, n)) * 0.05).astype(np.float32)
+    both = np.array([0.0, 1.5, 3.0, 6.0])
+    for i in range(m):
+        l6, _ = pairs[i % len(pairs)]
+        q = both[rng.integers(0, 4, size=16)] * rng.choice([-1, 1], size=16)
+        q[rng.integers(0, 16)] = 6.0
+        w[i, 16:32] = q * l6 * 2.0 ** -7
+    w[0, 0] = 2688 * 2.0 ** -7            # tensor amax: s_g = 2^-7, code 126 at both anchors
+    w[1, 32:48] = 0.0
+    w[2, 48:64] = 1e-7                    # tiny: both anchors clip to code 1
+    w[3, 64:80] = 0.0
+    w[3, 70] = -3e-6
+    wb = torch.from_numpy(w).to(torch.bfloat16)
+    b = bits(wb)
+    b[4, 32:48] = 0x8000                  # -0
+    wb = from_bits(b)
+    s_ref, _ = oracle.global_scale(b)
+    assert s_ref == np.float32(2.0 ** -7)
+    ref, nt = oracle.fourover6_codes(b, s_ref)
+    wd = wb.to(dev())
+    sg, _ = gpu_rtn(wd)
+    codes = gpu_fourover6(wd, sg)
+    compare_init(ref, nt, codes, "exact ties and edge groups")
+    col = codes[:, 1]
+    l6s = np.array([pairs[i % len(pairs)][0] for i in range(m)])
+    expect = np.array([np.flatnonzero(lad == 1.5 * v)[0] + 1 for v in l6s])
+    assert np.array_equal(col, expect), "an exact zero-error tie must keep anchor 4"
+    assert codes[0, 0] == 126 and codes[1, 2] == 1 and codes[4, 2] == 1 and codes[2, 3] == 1
+
+
+@pytest.mark.parametrize("down,up", [(4, 4), (9, 6), (0, 0)])
+def test_fourover6_then_refine_matches_oracle(down, up):
+    """Algorithm 2 end to end: 4over6 initial codes, then the search around them."""
+    w = small_layer(4, 512, 1024)
+    h32 = oracle_h32(4, 1024)
+    wd = w.to(dev())
+    sg, _ = gpu_rtn(wd)
+    s_ref, _ = oracle.global_scale(bits(w))
+    init_ref, nt = oracle.fourover6_codes(bits(w), s_ref)
+    init = torch.empty(512, 64, dtype=torch.uint8, device=dev())
+    hs.hscale_fourover6_codes(wd, sg, init)
+    diff = compare_init(init_ref, nt, init.cpu().numpy(), "512x1024 seed 4")
+    codes, packed = gpu_refine(wd, h32, sg, init, down, up)
+    ref = oracle.refine(bits(w), h32, s_ref, init_ref, down, up)
+    ref["near_tie"] = ref["near_tie"] | diff.astype(np.uint8)
+    compare_search(ref, codes, packed, f"4over6 init, window -{down}/+{up}")
+    if (down, up) == (0, 0):
+        assert np.array_equal(codes[~diff], init_ref[~diff])
+
+
 # ------------------------------------------------------------------ full-size workloads
 
-def full_size_check(name, sample_rows, layer_index=0, windows=None):
+def full_size_check(name, sample_rows, layer_index=0, windows=None, fourover6=False):
     """A workload at its full size in the launch configuration bench.py times: h of every
     input space over every streamed chunk (all columns, against the oracle fed the same
     chunks), s_g and RTN codes over every whole matrix, and the search with packing on a
-    seeded sample of rows of every matrix, for every window of the workload."""
+    seeded sample of rows of every matrix, for every window of the workload.  With
+    ``fourover6`` the search starts from Algorithm 2's codes, checked over every whole
+    matrix first."""
     W = wl.WORKLOADS[name]
     seed = W.layer_seed(layer_index)
     h_ref = {}
@@ -391,9 +489,18 @@ def full_size_check(name, sample_rows, layer_index=0, windows=None):
         assert sg.cpu().numpy()[0] == s_ref
         assert np.array_equal(codes.cpu().numpy(), oracle.rtn_codes(wb, s_ref))
         rows = np.sort(np.random.default_rng(seed).choice(m, size=min(sample_rows, m), replace=False))
+        init = init_ref = None
+        exclude = np.zeros((rows.size, n // 16), np.uint8)
+        if fourover6:
+            init_ref, nt = oracle.fourover6_codes(wb, s_ref)
+            init = torch.empty(m, n // 16, dtype=torch.uint8, device=dev())
+            hs.hscale_fourover6_codes(w, sg, init)
+            diff = compare_init(init_ref, nt, init.cpu().numpy(), f"{name} {L.name} {m}x{n}")
+            init_ref, exclude = init_ref[rows], diff[rows].astype(np.uint8)
         for down, up in (windows or [(k, k) for k in W.window]):
-            codes_g, packed_g = gpu_refine(w, h_ref[L.input_space], sg, None, down, up)
-            ref = oracle.refine(wb[rows], h_ref[L.input_space], s_ref, None, down, up)
+            codes_g, packed_g = gpu_refine(w, h_ref[L.input_space], sg, init, down, up)
+            ref = oracle.refine(wb[rows], h_ref[L.input_space], s_ref, init_ref, down, up)
+            ref["near_tie"] = ref["near_tie"] | exclude
             compare_search(ref, codes_g[rows], packed_g[rows],
                            f"{name} {L.name} {m}x{n} window -{down}/+{up} ({rows.size} sampled rows)")
         del w
@@ -406,6 +513,12 @@ def test_full_size_llama8b_q_proj():
 def test_full_size_q_proj_paper_window_and_full_grid():
     """The paper's default window (D = 9, U = 6, K = 16) and the whole E4M3 ladder."""
     full_size_check("llama8b-q_proj", sample_rows=64, windows=[(9, 6), (125, 125)])
+
+
+def test_full_size_q_proj_fourover6_init():
+    """Algorithm 2 at full size: 4over6 codes over the whole matrix, then the search
+    around them with the paper's default window."""
+    full_size_check("llama8b-q_proj", sample_rows=128, windows=[(9, 6), (4, 4)], fourover6=True)
 
 
 def test_full_size_mlp_down_proj():
