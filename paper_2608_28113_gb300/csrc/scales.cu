@@ -8,13 +8,20 @@
 //   pack_kernel         exact FP4 quantization with given codes (Eq. 2)
 //
 // The search (one group per thread, no shuffles in the hot loop)
-//   Per element and candidate the fast score costs one multiply for the quotient, an
-//   integer add + and + min for the E2M1 rounding (see hscale_device.cuh), one FMA for
-//   the residual, and a multiply + FMA for h * r^2.  The fast scores differ from the
-//   exact-decision scores only through roundings near E2M1 midpoints and fp32 error,
-//   which together stay below
-//        B(E) = 2^-13 E + 32 * 2^-24 * s_max * sqrt(H E)     (H = sum of the group's h)
-//   so when runner-up - best > B(runner-up) the fast winner is the exact winner.
+//   A candidate scale s' = l sgk is scored as E = s'^2 sum_j h_j (q_j - y_j)^2 with
+//   y_j = |a_j| / s' (one packed multiply by a tabulated reciprocal) and q_j = RNE_sat(y_j)
+//   from the hardware E2M1 conversion (saturation included) converted back to f16; the
+//   residual q - y is one mixed f16/f32 subtract.  That is five lane operations per
+//   element and candidate.  With y within a relative 2^-21 of the exact quotient, every
+//   element's term differs from its exact-decision term by at most
+//   4 * 2^-21 y* |q* - y*| + 8 * 2^-42 y*^2 (also where a midpoint falls between y and
+//   y*), so by Cauchy-Schwarz the fast score is within
+//        4 * 2^-21 sqrt(A E*) + 8 * 2^-42 A + 13 * 2^-24 E*    (A = sum_j h_j a_j^2)
+//   of the exact score E*; in terms of the fast score E that is at most
+//   4.01 * 2^-21 sqrt(A E) + 33 * 2^-42 A + 13 * 2^-24 E.  When
+//        runner-up - best > 2^-13 E2 + 2^-17 sqrt(A E2) + 2^-35 A
+//   (more than the two errors together) and E2 >= 2^-36 A (so the bound grows slower
+//   than the score for every other candidate), the fast winner is the exact winner.
 //   Otherwise the group is "ambiguous" and the whole warp rescores it cooperatively with
 //   exact rounding decisions (16 lanes per candidate, one element each, a fixed
 //   pairwise shuffle tree per error: relative error <= 8 * 2^-24), applying the tie
@@ -108,39 +115,46 @@ __device__ __forceinline__ void load_group(const uint4* w, int64_t g, float pw, 
 }
 
 // Per-block table of the candidate constants of every E4M3 code c (1..126), filled once
-// per CTA: x = -(s' * 2^126) and y = 2^-126 / s' (fast reciprocal), with s' = l(c) * sgk.
-// Reading it costs one shared load per candidate instead of a decode, two multiplies and
-// a reciprocal on the candidate's critical path.
-__device__ __forceinline__ float2 candidate_constants(uint32_t c, float sgk) {
+// per CTA and stored pre-splatted for the packed arithmetic: x = y = s'^2 and
+// z = w = 1 / s' (fast reciprocal), with s' = l(c) * sgk in [2^-21, 2^-2], so both are
+// normal numbers.  One 16-byte shared load per candidate replaces a decode, a multiply
+// and a reciprocal on the candidate's critical path.
+__device__ __forceinline__ float4 candidate_constants(uint32_t c, float sgk) {
   const float sp = __fmul_rn(e4m3_mag(c), sgk);
-  return make_float2(-__fmul_rn(sp, 0x1p126f), c ? inv_raw_of(sp) : 0.0f);
+  const float s2 = __fmul_rn(sp, sp), inv = c ? rcp_approx(sp) : 0.0f;
+  return make_float4(s2, s2, inv, inv);
 }
 
-// Fast score of one candidate from its table entry (see the file comment): per pair of
-// elements one packed multiply for the quotients, integer rounding of each raw pattern
-// (plus the saturation when SAT), one packed FMA for the residuals, a packed square and a
-// packed FMA into the h-weighted sum.
-template <bool SAT>
-__device__ __forceinline__ float fast_score(const Group& G, const float2 (&hv2)[8], float2 t) {
-  const float2 inv2 = make_float2(t.y, t.y);
-  const float2 nS2 = make_float2(t.x, t.x);
+// q - y for a pair of quotients y (real units): q = RNE_sat(y) by the hardware E2M1
+// conversion, back to f16 (exact), and one mixed f16 - f32 subtract per element.
+__device__ __forceinline__ float2 e2m1_residual2(float2 y) {
+  float d0, d1;
+  asm("{\n\t.reg .b8 c;\n\t.reg .b32 q;\n\t.reg .f16 lo, hi;\n\t"
+      "cvt.rn.satfinite.e2m1x2.f32 c, %3, %2;\n\t"
+      "cvt.rn.f16x2.e2m1x2 q, c;\n\t"
+      "mov.b32 {lo, hi}, q;\n\t"
+      "sub.rn.f32.f16 %0, lo, %2;\n\t"
+      "sub.rn.f32.f16 %1, hi, %3;\n\t}"
+      : "=f"(d0), "=f"(d1)
+      : "f"(y.x), "f"(y.y));
+  return make_float2(d0, d1);
+}
+
+// Fast score of one candidate from its table entry t (see the file comment): per pair of
+// elements one packed multiply for the quotients, the hardware rounding and residuals,
+// a packed square and a packed FMA into the h-weighted sum; then one multiply by s'^2.
+__device__ __forceinline__ float fast_score(const Group& G, const float2 (&hv2)[8], float4 t) {
+  const float2 inv2 = make_float2(t.z, t.w);
   float2 acc0 = make_float2(0.f, 0.f), acc1 = make_float2(0.f, 0.f);
 #pragma unroll
   for (int i = 0; i < 8; ++i) {
-    const float2 y = __fmul2_rn(G.a[i], inv2);
-    uint32_t q0 = (__float_as_uint(y.x) + kE2M1Half) & kE2M1Keep;
-    uint32_t q1 = (__float_as_uint(y.y) + kE2M1Half) & kE2M1Keep;
-    if (SAT) {
-      q0 = min(q0, kE2M1SixRaw);
-      q1 = min(q1, kE2M1SixRaw);
-    }
-    const float2 r = __ffma2_rn(make_float2(__uint_as_float(q0), __uint_as_float(q1)), nS2, G.a[i]);
-    const float2 rr = __fmul2_rn(r, r);
-    if (i & 1) acc1 = __ffma2_rn(hv2[i], rr, acc1);
-    else acc0 = __ffma2_rn(hv2[i], rr, acc0);
+    const float2 d = e2m1_residual2(__fmul2_rn(G.a[i], inv2));
+    const float2 dd = __fmul2_rn(d, d);
+    if (i & 1) acc1 = __ffma2_rn(hv2[i], dd, acc1);
+    else acc0 = __ffma2_rn(hv2[i], dd, acc0);
   }
   const float2 t2 = __fadd2_rn(acc0, acc1);
-  return __fadd_rn(t2.x, t2.y);
+  return __fmul_rn(t.x, __fadd_rn(t2.x, t2.y));
 }
 
 __device__ __forceinline__ void keep_best(float e, int c, float& e1, float& e2, int& best) {
@@ -149,30 +163,26 @@ __device__ __forceinline__ void keep_best(float e, int c, float& e1, float& e2, 
 }
 
 // Scores the codes [a, b) two at a time (independent chains interleave).
-template <bool SAT>
 __device__ __forceinline__ void score_range(const Group& G, const float2 (&hv2)[8],
-                                            const float2* tab, int a, int b, float& e1, float& e2,
+                                            const float4* tab, int a, int b, float& e1, float& e2,
                                             int& best) {
   int c = a;
   for (; c + 1 < b; c += 2) {
-    const float2 t0 = tab[c], t1 = tab[c + 1];
-    const float ea = fast_score<SAT>(G, hv2, t0);
-    const float eb = fast_score<SAT>(G, hv2, t1);
+    const float4 t0 = tab[c], t1 = tab[c + 1];
+    const float ea = fast_score(G, hv2, t0);
+    const float eb = fast_score(G, hv2, t1);
     keep_best(ea, c, e1, e2, best);
     keep_best(eb, c + 1, e1, e2, best);
   }
-  if (c < b) keep_best(fast_score<SAT>(G, hv2, tab[c]), c, e1, e2, best);
+  if (c < b) keep_best(fast_score(G, hv2, tab[c]), c, e1, e2, best);
 }
 
-// True when some quotient of the group under code c rounds to 7 or more in the fast
-// path, i.e. when candidates from c upwards still need the E2M1 saturation.  The test
-// uses the same fp32 product as the fast path on the group's largest magnitude, and
-// quotients only shrink as the code grows, so it is exact for every code >= c.
-__device__ __forceinline__ bool needs_saturation_from(const Group& G, float2 t) {
-  float amax = 0.f;
+// A = sum_j h_j a_j^2 of a group (scaled domain), the scale of the fast-score error bound.
+__device__ __forceinline__ float group_energy(const Group& G, const float2 (&hv2)[8]) {
+  float2 acc = make_float2(0.f, 0.f);
 #pragma unroll
-  for (int i = 0; i < 8; ++i) amax = fmaxf(amax, fmaxf(G.a[i].x, G.a[i].y));
-  return __fmul_rn(amax, t.y) >= 7.0f * 0x1p-126f;
+  for (int i = 0; i < 8; ++i) acc = __ffma2_rn(hv2[i], __fmul2_rn(G.a[i], G.a[i]), acc);
+  return __fadd_rn(acc.x, acc.y);
 }
 
 // tie rule of the search: smaller error, then smaller |shift|, then smaller shift
@@ -233,16 +243,16 @@ __device__ __forceinline__ uint32_t cvt_e2m1x2(float hi, float lo) {
   return r;
 }
 
-// Exact final re-quantization of one group under code c (table entry t): 8 bytes of
+// Exact final re-quantization of one group under code c (inv_raw = 2^-126 / s'): 8 bytes of
 // packed nibbles.  The raw-domain quotients y_raw = |w| * 2^-126 / s' are rescaled
 // exactly to real units, given the sign of w, and converted by the hardware E2M1
 // conversion (round-to-nearest-even).  That equals the exact rounding of |w| / s unless
 // y_raw lies within 16 ulps of a midpoint; such elements are flagged and redone one by
 // one with the exact midpoint test, reading the weight back from `wg` (the group's 16
 // bf16 values in global memory).
-__device__ __forceinline__ uint2 quantize_pack(const Group& G, uint32_t c, float2 t, float sgk,
+__device__ __forceinline__ uint2 quantize_pack(const Group& G, uint32_t c, float inv_raw, float sgk,
                                                float pw, const uint16_t* wg) {
-  const float2 ir2 = make_float2(t.y, t.y);
+  const float2 ir2 = make_float2(inv_raw, inv_raw);
   const float2 up2 = make_float2(0x1p126f, 0x1p126f);
   uint32_t word[2] = {0u, 0u};
   uint32_t flagged = 0u;
@@ -263,7 +273,7 @@ __device__ __forceinline__ uint2 quantize_pack(const Group& G, uint32_t c, float
       flagged &= flagged - 1;
       const uint32_t b = wg[j];
       const float a = __fmul_rn(__uint_as_float((b & 0x7FFFu) << 16), pw);
-      const uint32_t k = e2m1_exact_code(__fmul_rn(a, t.y), a, l, sgk);
+      const uint32_t k = e2m1_exact_code(__fmul_rn(a, inv_raw), a, l, sgk);
       const int sh = 4 * (j & 7);
       word[j >> 3] = (word[j >> 3] & ~(0xFu << sh)) | ((((b >> 15) << 3) | k) << sh);
     } while (flagged);
@@ -286,7 +296,7 @@ refine_kernel(const uint4* __restrict__ w, const float* __restrict__ h, int64_t 
   const int chunks = (ng + 31) / 32;
   const int64_t units = m * chunks;
 
-  __shared__ float2 tab[128];
+  __shared__ float4 tab[128];
   const ScaleDomain d = make_scale_domain(*global_scale);
   const float inv6 = rtn_inv6_raw(d.sgk);
   for (int c = threadIdx.x; c < 128; c += blockDim.x) tab[c] = candidate_constants((uint32_t)c, d.sgk);
@@ -294,7 +304,6 @@ refine_kernel(const uint4* __restrict__ w, const float* __restrict__ h, int64_t 
 
   int cur_chunk = -1;
   float2 hv2[8];
-  float H = 0.0f;
 #pragma unroll
   for (int j = 0; j < 8; ++j) hv2[j] = make_float2(1.0f, 1.0f);
 
@@ -307,7 +316,6 @@ refine_kernel(const uint4* __restrict__ w, const float* __restrict__ h, int64_t 
 
     if (chunk != cur_chunk) {
       cur_chunk = chunk;
-      H = 0.0f;
       if (h != nullptr && active) {
         const float4* hp = reinterpret_cast<const float4*>(h + (int64_t)gcol * 16);
 #pragma unroll
@@ -317,8 +325,6 @@ refine_kernel(const uint4* __restrict__ w, const float* __restrict__ h, int64_t 
           hv2[2 * i + 1] = make_float2(t.z, t.w);
         }
       }
-#pragma unroll
-      for (int j = 0; j < 8; ++j) H = __fadd_rn(H, __fadd_rn(hv2[j].x, hv2[j].y));
     }
 
     Group G;
@@ -337,26 +343,19 @@ refine_kernel(const uint4* __restrict__ w, const float* __restrict__ h, int64_t 
       hi = min((int)kE4M3MaxCode, c0 + up);
     }
 
-    // ---- fast scores of every distinct candidate.  Codes below c0 run with the E2M1
-    // saturation; codes from c0 up skip it unless some lane of the warp needs it there
-    // (never for an RTN start on a normal E4M3 code, whose quotients stay below 6.375).
-    // Splitting every lane at its own c0 keeps the loop trip counts uniform in the warp.
+    // ---- fast scores of every distinct candidate (the same trip count in every lane
+    // unless the window is clipped at the ends of the ladder)
     float e1 = kInf, e2 = kInf;
     int best = c0;
-    const bool sat_hi = __any_sync(0xFFFFFFFFu, active && needs_saturation_from(G, tab[c0]));
-    if (active) {
-      score_range<true>(G, hv2, tab, lo, c0, e1, e2, best);
-      if (sat_hi) score_range<true>(G, hv2, tab, c0, hi + 1, e1, e2, best);
-      else score_range<false>(G, hv2, tab, c0, hi + 1, e1, e2, best);
-    }
+    if (active) score_range(G, hv2, tab, lo, hi + 1, e1, e2, best);
 
     // ---- is the fast winner certain?
     bool ambiguous = false;
     if (active && hi > lo) {
-      const float smax = __fmul_rn(e4m3_mag((uint32_t)hi), d.sgk);
-      const float bound = __fmaf_rn(0x1p-13f, e2,
-                                    __fmul_rn(32.0f * 0x1p-24f, __fmul_rn(smax, sqrtf(__fmul_rn(H, e2)))));
-      ambiguous = !(__fsub_rn(e2, e1) > bound) || !(e2 >= 0x1p-100f);
+      const float A = group_energy(G, hv2);
+      const float bound = __fmaf_rn(0x1p-13f, e2, __fmaf_rn(0x1p-17f, __fsqrt_rn(__fmul_rn(A, e2)),
+                                                             __fmul_rn(0x1p-35f, A)));
+      ambiguous = !(__fsub_rn(e2, e1) > bound) || !(e2 >= __fmul_rn(0x1p-36f, A)) || !(A > 0.0f);
     }
     unsigned amb = __ballot_sync(0xFFFFFFFFu, ambiguous);
     while (amb) {
@@ -374,7 +373,7 @@ refine_kernel(const uint4* __restrict__ w, const float* __restrict__ h, int64_t 
     if (active) {
       codes_out[g] = (uint8_t)best;
       if (packed_out != nullptr)
-        packed_out[g] = quantize_pack(G, (uint32_t)best, tab[best], d.sgk, d.pw,
+        packed_out[g] = quantize_pack(G, (uint32_t)best, __fmul_rn(tab[best].z, 0x1p-126f), d.sgk, d.pw,
                                       reinterpret_cast<const uint16_t*>(w) + g * 16);
     }
   }
@@ -392,7 +391,7 @@ __global__ void __launch_bounds__(256) pack_kernel(const uint4* __restrict__ w, 
     load_group(w, g, d.pw, G);
     uint32_t c = codes[g] & 0x7Fu;
     c = c < 1 ? 1u : (c > kE4M3MaxCode ? kE4M3MaxCode : c);
-    packed_out[g] = quantize_pack(G, c, candidate_constants(c, d.sgk), d.sgk, d.pw,
+    packed_out[g] = quantize_pack(G, c, inv_raw_of(__fmul_rn(e4m3_mag(c), d.sgk)), d.sgk, d.pw,
                                   reinterpret_cast<const uint16_t*>(w) + g * 16);
   }
 }
