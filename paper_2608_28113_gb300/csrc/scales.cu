@@ -19,9 +19,10 @@
 //        4 * 2^-21 sqrt(A E*) + 8 * 2^-42 A + 13 * 2^-24 E*    (A = sum_j h_j a_j^2)
 //   of the exact score E*; in terms of the fast score E that is at most
 //   4.01 * 2^-21 sqrt(A E) + 33 * 2^-42 A + 13 * 2^-24 E.  When
-//        runner-up - best > 2^-13 E2 + 2^-17 sqrt(A E2) + 2^-35 A
-//   (more than the two errors together) and E2 >= 2^-36 A (so the bound grows slower
-//   than the score for every other candidate), the fast winner is the exact winner.
+//        runner-up - best > 2^-18 E2 + 2^-17 sqrt(A E2) + 2^-35 A
+//   (more than the two errors together, with at least 2x slack on every term) and
+//   E2 >= 2^-36 A (so the bound grows slower than the score for every other candidate),
+//   the fast winner is the exact winner.
 //   Otherwise the group is "ambiguous" and the whole warp rescores it cooperatively with
 //   exact rounding decisions (16 lanes per candidate, one element each, a fixed
 //   pairwise shuffle tree per error: relative error <= 8 * 2^-24), applying the tie
@@ -352,10 +353,15 @@ refine_kernel(const uint4* __restrict__ w, const float* __restrict__ h, int64_t 
     // ---- is the fast winner certain?
     bool ambiguous = false;
     if (active && hi > lo) {
+      // In units of E2 (no underflow or overflow for 2^-36 A <= E2 <= A-ish):
+      //   g = (E2 - E1) / E2 - 2^-18 - 2^-35 A / E2 > 2^-17 sqrt(A / E2), tested on squares.
+      // A zero, denormal or non-finite E2 makes the reciprocal infinite or NaN and g fails.
       const float A = group_energy(G, hv2);
-      const float bound = __fmaf_rn(0x1p-13f, e2, __fmaf_rn(0x1p-17f, __fsqrt_rn(__fmul_rn(A, e2)),
-                                                             __fmul_rn(0x1p-35f, A)));
-      ambiguous = !(__fsub_rn(e2, e1) > bound) || !(e2 >= __fmul_rn(0x1p-36f, A)) || !(A > 0.0f);
+      const float r = rcp_approx(e2);
+      const float ratio = __fmul_rn(A, r);
+      const float g = __fsub_rn(__fsub_rn(__fmul_rn(__fsub_rn(e2, e1), r), 0x1p-18f), __fmul_rn(0x1p-35f, ratio));
+      const bool certain = g > 0.0f && __fmul_rn(g, g) > __fmul_rn(0x1p-34f, ratio);
+      ambiguous = !certain || !(ratio <= 0x1p36f) || !(A > 0.0f);
     }
     unsigned amb = __ballot_sync(0xFFFFFFFFu, ambiguous);
     while (amb) {
