@@ -58,6 +58,9 @@ def parse():
                    help="calibration tokens per input space (default: the workload's; smaller for ncu captures)")
     p.add_argument("--init", choices=["rtn", "4over6"], default="rtn",
                    help="initial codes of the search: max-abs RTN (Eq. 7) or 4over6 (Algorithm 2)")
+    p.add_argument("--overlap-ctas", type=int, default=4,
+                   help="resident search CTAs per SM while the next input space's Hessian pass "
+                        "runs alongside (0: run every search after the last Hessian pass)")
     p.add_argument("--no-cpu-baseline", action="store_true")
     p.add_argument("--no-e2e", action="store_true")
     return p.parse_args()
@@ -245,9 +248,12 @@ class Work:
         self.ws = None
 
 
-def hessian_phase(hs, work: Work, xs=None):
-    """For every input space: h = 0, then one hscale_hessian_diag_accumulate per chunk."""
+def hessian_phase(hs, work: Work, xs=None, only=None):
+    """For every input space (or the one named `only`): h = 0, then one
+    hscale_hessian_diag_accumulate per chunk."""
     for S in work.spaces.values():
+        if only is not None and S.name != only:
+            continue
         x = S.x if xs is None else xs[S.name]
         S.h.zero_()
         for c in range(S.nchunks):
@@ -255,56 +261,128 @@ def hessian_phase(hs, work: Work, xs=None):
 
 
 def init_codes(hs, work: Work, M, w=None):
-    """Global scale and the search's initial codes of one matrix: max-abs RTN codes
-    (Eq. 7), or, with 4over6 init, s_g alone followed by Algorithm 2's codes."""
+    """The weight-only part of one matrix: the global scale s_g, and with 4over6 init
+    Algorithm 2's codes.  With RTN init the search computes the RTN codes (Eq. 7) itself
+    (init_codes = NULL), which saves a pass over W."""
     w = M.w if w is None else w
+    hs.hscale_rtn_scales(w, M.sg, None, work.ws)
     if work.init == "4over6":
-        hs.hscale_rtn_scales(w, M.sg, None, work.ws)
         hs.hscale_fourover6_codes(w, M.sg, M.codes0)
-    else:
-        hs.hscale_rtn_scales(w, M.sg, M.codes0, work.ws)
+
+
+def init_phase(hs, work: Work, ws=None):
+    for M in work.mats:
+        init_codes(hs, work, M, None if ws is None else ws[M.name])
+
+
+def refine(hs, work: Work, M, down, up, w=None, ctas_per_sm=0):
+    """The H-Scale search with packing of one matrix over the window (down, up)."""
+    init = M.codes0 if work.init == "4over6" else None
+    hs.hscale_refine_scales_ex(M.w if w is None else w, M.space.h, M.sg, init, down, up, M.codes,
+                               M.packed, ctas_per_sm)
+
+
+def refine_phase(hs, work: Work, win=None, ws=None):
+    down, up = work.win if win is None else win
+    for M in work.mats:
+        refine(hs, work, M, down, up, None if ws is None else ws[M.name])
 
 
 def scale_phase(hs, work: Work, win=None, ws=None):
-    """For every matrix: global scale + initial codes, then the H-Scale search with
-    packing over the window win = (down, up)."""
-    down, up = work.win if win is None else win
-    for M in work.mats:
-        w = M.w if ws is None else ws[M.name]
-        init_codes(hs, work, M, w)
-        hs.hscale_refine_scales(w, M.space.h, M.sg, M.codes0, down, up, M.codes, M.packed)
+    """For every matrix: the weight-only part, then the search."""
+    init_phase(hs, work, ws)
+    refine_phase(hs, work, win, ws)
 
 
-def run_step(hs, work: Work, ev=None):
-    """One eager pass of the hot path.  ev: optional 3 events (start, after h, end)."""
-    if ev:
-        ev[0].record()
+def run_step(hs, work: Work):
+    """One eager pass of the hot path on the current stream."""
     hessian_phase(hs, work)
-    if ev:
-        ev[1].record()
     scale_phase(hs, work)
-    if ev:
-        ev[2].record()
 
 
-def capture_graphs(hs, work: Work):
-    """The step's launch sequence captured as two CUDA graphs (Hessian pass; scales)."""
-    side = torch.cuda.Stream()
-    side.wait_stream(torch.cuda.current_stream())
-    with torch.cuda.stream(side):
-        run_step(hs, work)
-    torch.cuda.current_stream().wait_stream(side)
-    torch.cuda.synchronize()
-    gh, gs = torch.cuda.CUDAGraph(), torch.cuda.CUDAGraph()
-    with torch.cuda.graph(gh):
-        hessian_phase(hs, work)
-    with torch.cuda.graph(gs):
-        scale_phase(hs, work)
-    torch.cuda.synchronize()
-    return gh, gs
+class StepGraphs:
+    """The step's launches as CUDA graphs on three streams.
+
+    main:   the Hessian pass of each input space in turn (HBM-bound);
+    side:   the weight-only calls of every matrix (s_g, 4over6 codes), alongside;
+    search: the searches of an input space's matrices (ALU-bound), started as soon as
+            that space's h is complete and the weight-only calls are done, so that they
+            run alongside the next space's Hessian pass.  Those searches keep at most
+            `overlap_ctas` CTAs resident per SM, which leaves registers for the Hessian
+            CTAs; the last space's searches fill the GPU.  overlap_ctas = 0 runs every
+            search after the last Hessian pass instead."""
+
+    def __init__(self, hs, work: Work, overlap_ctas: int):
+        self.work, self.overlap = work, overlap_ctas > 0
+        spaces = list(work.spaces.values())
+        warm = torch.cuda.Stream()
+        warm.wait_stream(torch.cuda.current_stream())
+        with torch.cuda.stream(warm):
+            run_step(hs, work)
+        torch.cuda.current_stream().wait_stream(warm)
+        torch.cuda.synchronize()
+        down, up = work.win
+        self.gh, self.gr = [], []
+        for i, S in enumerate(spaces):
+            g = torch.cuda.CUDAGraph()
+            with torch.cuda.graph(g):
+                hessian_phase(hs, work, only=S.name)
+            self.gh.append(g)
+            ctas = overlap_ctas if (self.overlap and i + 1 < len(spaces)) else 0
+            g = torch.cuda.CUDAGraph()
+            with torch.cuda.graph(g):
+                for M in work.mats:
+                    if M.space is S:
+                        refine(hs, work, M, down, up, ctas_per_sm=ctas)
+            self.gr.append(g)
+        self.gi = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(self.gi):
+            init_phase(hs, work)
+        torch.cuda.synchronize()
+        self.side, self.search = torch.cuda.Stream(), torch.cuda.Stream()
+        self.ev_init = torch.cuda.Event()
+        self.ev_h = [torch.cuda.Event() for _ in spaces]
+
+    def replay(self, ev=None):
+        """One step.  ev: optional (start, after the last Hessian pass, end) timing events
+        recorded on the current stream, which runs the Hessian passes."""
+        main = torch.cuda.current_stream()
+        if ev:
+            ev[0].record()
+        self.side.wait_stream(main)
+        self.search.wait_stream(main)
+        with torch.cuda.stream(self.side):
+            self.gi.replay()
+            self.ev_init.record(self.side)
+        self.search.wait_event(self.ev_init)
+        for i, g in enumerate(self.gh):
+            g.replay()
+            self.ev_h[i].record(main)
+            if self.overlap:
+                self.search.wait_event(self.ev_h[i])
+                with torch.cuda.stream(self.search):
+                    self.gr[i].replay()
+        if ev:
+            ev[1].record()
+        if not self.overlap:
+            self.search.wait_stream(main)
+            with torch.cuda.stream(self.search):
+                for g in self.gr:
+                    g.replay()
+        main.wait_stream(self.search)
+        main.wait_stream(self.side)
+        if ev:
+            ev[2].record()
 
 
-KERNELS_PER_MATRIX = 3  # amax, RTN or 4over6 codes, refine
+# algorithmic bytes per group of the search: W 32, nibbles 8, code out 1, code in 1 (none
+# when the search computes the RTN codes itself)
+SEARCH_BYTES = {"rtn": 41, "4over6": 42}
+
+
+def kernels_per_matrix(work: Work) -> int:
+    """Library kernels per matrix and step: amax, (4over6 codes,) refine."""
+    return 3 if work.init == "4over6" else 2
 
 
 def timed(fn, reps):
@@ -481,10 +559,9 @@ def gpu_arm(args, d: Dist):
     ms_eager = timed(lambda: run_step(hs, work), args.steps)
 
     # timed region: the same launches replayed from CUDA graphs
-    gh, gs = capture_graphs(hs, work)
+    graphs = StepGraphs(hs, work, args.overlap_ctas)
     for _ in range(warm):
-        gh.replay()
-        gs.replay()
+        graphs.replay()
     evs = [[torch.cuda.Event(enable_timing=True) for _ in range(3)] for _ in range(args.steps)]
     d.barrier()
     torch.cuda.synchronize()
@@ -493,11 +570,7 @@ def gpu_arm(args, d: Dist):
         t1 = torch.cuda.Event(enable_timing=True)
         t0.record()
         for s in range(args.steps):
-            evs[s][0].record()
-            gh.replay()
-            evs[s][1].record()
-            gs.replay()
-            evs[s][2].record()
+            graphs.replay(evs[s])
         t1.record()
         torch.cuda.synchronize()
     d.barrier()
@@ -514,22 +587,26 @@ def gpu_arm(args, d: Dist):
     fp32_peak = props.multi_processor_count * 128 * sm_max_mhz * 1e6
     reps = max(3, min(args.steps, 20))
     ms_init = sum(timed(lambda M=M: init_codes(hs, work, M), reps) for M in work.mats)
+    ms_h_alone = timed(lambda: [g.replay() for g in graphs.gh], reps)
     sweep = []
     windows = sorted(set([win] + [(kk, kk) for kk in W.window]))
     for dn, upw in windows:
         ms_ref = 0.0
         for M in work.mats:
-            ms_ref += timed(lambda M=M: hs.hscale_refine_scales(M.w, M.space.h, M.sg, M.codes0, dn, upw,
-                                                                 M.codes, M.packed), reps)
+            ms_ref += timed(lambda M=M: refine(hs, work, M, dn, upw), reps)
         C = dn + upw + 1
-        t_bytes = 42 * work.groups / (hbm_peak * 1e9)
+        t_bytes = SEARCH_BYTES[work.init] * work.groups / (hbm_peak * 1e9)
         t_ops = 80 * C * work.groups / fp32_peak
         sweep.append({"window": [dn, upw], "candidates": C, "ms": ms_ref,
                       "groups_per_s": work.groups / (ms_ref * 1e-3),
                       "bound": "alu" if t_ops > t_bytes else "hbm", "roofline_ms": max(t_bytes, t_ops) * 1e3,
                       "frac": max(t_bytes, t_ops) / (ms_ref * 1e-3)})
-    # restore the outputs of the step's own window
+    # restore the outputs of the step's own window; materialize the RTN codes the search
+    # computed inline, for the shift statistics
     scale_phase(hs, work)
+    if work.init == "rtn":
+        for M in work.mats:
+            hs.hscale_rtn_scales(M.w, M.sg, M.codes0, work.ws)
     torch.cuda.synchronize()
     main = [s for s in sweep if tuple(s["window"]) == tuple(win)][0]
     shifts = shift_statistics(work, win)
@@ -562,9 +639,14 @@ def gpu_arm(args, d: Dist):
                      "peak_kind": f"{peak_kind} HBM copy bandwidth",
                      "frac_of_8TBs_spec": h_gbs / HBM_SPEC_GBS, "traffic": traffic,
                      "bytes_per_launch": h_bytes_launch, "ms_per_launch": ms_h_launch},
-        "phases_ms": {"hessian": ms_h, "scales": ms_sc, "init_codes": ms_init, "refine": main["ms"]},
+        "phases_ms": {"hessian": ms_h, "after_hessian": ms_sc, "hessian_alone": ms_h_alone,
+                      "weight_only": ms_init, "refine": main["ms"]},
         "ms_per_step_eager": ms_eager,
-        "timed_launch": "CUDA graphs of the step's API calls (Hessian pass; scales)",
+        "timed_launch": ("CUDA graphs of the step's API calls on three streams: the Hessian pass of "
+                         "each input space; alongside it the weight-only calls (s_g, 4over6 codes); the "
+                         "searches of each input space as soon as its h is complete"
+                         + (f" (at most {args.overlap_ctas} search CTAs per SM while a Hessian pass runs)"
+                            if args.overlap_ctas > 0 and len(work.spaces) > 1 else "")),
         "hessian": {"gbs": h_gbs, "tokens_channels_per_s": work.h_bytes / 2 / (ms_h * 1e-3),
                     "frac_of_measured_hbm": h_gbs / hbm_peak, "frac_of_8TBs": h_gbs / HBM_SPEC_GBS},
         "search": {"groups_per_s": main["groups_per_s"], "candidates": main["candidates"],
@@ -573,7 +655,7 @@ def gpu_arm(args, d: Dist):
                    "clock_mhz_for_peak": sm_max_mhz},
         "seconds_per_layer": ms_step * 1e-3,
         "clocks": clk.summary(),
-        "gpu_launches": args.steps * (work.h_launches + KERNELS_PER_MATRIX * len(work.mats)),
+        "gpu_launches": args.steps * (work.h_launches + kernels_per_matrix(work) * len(work.mats)),
     }
     if len(sweep) > 1:
         line["search_sweep"] = sweep

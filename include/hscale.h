@@ -17,6 +17,7 @@
  *                                       (Eqs. 6, 13), then re-quantize and pack
  *      hscale_pack_nvfp4                final FP4 quantization with given codes
  *                                       (Sec. 3.3 "Final re-quantization", Eq. 2)
+ *      hscale_refine_scales_ex          the same with a cap on resident CTAs per SM
  *      hscale_fourover6_codes           the 4over6 initial codes of Algorithm 2, an
  *                                       alternative start for the refinement (Sec. 3.5)
  *
@@ -186,6 +187,20 @@ int hscale_fourover6_codes(const void* w_bf16, int64_t m, int64_t n, const float
 int hscale_refine_scales(const void* w_bf16, const float* h, int64_t m, int64_t n,
                          const float* global_scale, const uint8_t* init_codes, int32_t down,
                          int32_t up, uint8_t* codes_out, uint8_t* packed_out, void* stream);
+
+/*
+ * hscale_refine_scales with an explicit launch shape; the results are identical.
+ * The paper has no counterpart: this is a scheduling knob for callers that run the
+ * search alongside another kernel (e.g. the next input space's Hessian pass on another
+ * stream).  ctas_per_sm = 0 fills every SM as hscale_refine_scales does; k > 0 keeps at
+ * most k of the search's CTAs (128 threads, 72 registers each) resident per SM, leaving
+ * the rest of the register file to concurrent work.  Negative values return
+ * HSCALE_ERR_ARG.
+ */
+int hscale_refine_scales_ex(const void* w_bf16, const float* h, int64_t m, int64_t n,
+                            const float* global_scale, const uint8_t* init_codes, int32_t down,
+                            int32_t up, uint8_t* codes_out, uint8_t* packed_out,
+                            int32_t ctas_per_sm, void* stream);
 
 /*
  * Final FP4 quantization with given codes (Sec. 3.3 "Final re-quantization", Eq. 2):

@@ -25,7 +25,8 @@ __all__ = [
     "hscale_device_error_flags",
     "hscale_hessian_diag_accumulate", "hscale_rtn_workspace_bytes", "hscale_rtn_scales",
     "hscale_rtn_scales_noalloc",
-    "hscale_refine_scales", "hscale_pack_nvfp4", "hscale_fourover6_codes", "EXPORTED_SYMBOLS",
+    "hscale_refine_scales", "hscale_refine_scales_ex", "hscale_pack_nvfp4", "hscale_fourover6_codes",
+    "EXPORTED_SYMBOLS",
 ]
 
 _PKG = pathlib.Path(__file__).resolve().parent
@@ -44,6 +45,7 @@ _SIGNATURES = {
     "hscale_rtn_scales": (ctypes.c_int, [_P, _I64, _I64, _P, _P, _P, _SZ, _P]),
     "hscale_rtn_scales_noalloc": (ctypes.c_int, [_P, _I64, _I64, _P, _P, _P]),
     "hscale_refine_scales": (ctypes.c_int, [_P, _P, _I64, _I64, _P, _P, _I32, _I32, _P, _P, _P]),
+    "hscale_refine_scales_ex": (ctypes.c_int, [_P, _P, _I64, _I64, _P, _P, _I32, _I32, _P, _P, _I32, _P]),
     "hscale_pack_nvfp4": (ctypes.c_int, [_P, _I64, _I64, _P, _P, _P, _P]),
     "hscale_fourover6_codes": (ctypes.c_int, [_P, _I64, _I64, _P, _P, _P]),
 }
@@ -178,6 +180,14 @@ def hscale_refine_scales(w: torch.Tensor, h: torch.Tensor | None, global_scale: 
                          codes_out: torch.Tensor, packed_out: torch.Tensor | None,
                          stream=None) -> None:
     """Algorithm 1 over every group of W, with the final re-quantization and packing."""
+    hscale_refine_scales_ex(w, h, global_scale, init_codes, down, up, codes_out, packed_out, 0, stream)
+
+
+def hscale_refine_scales_ex(w: torch.Tensor, h: torch.Tensor | None, global_scale: torch.Tensor,
+                            init_codes: torch.Tensor | None, down: int, up: int,
+                            codes_out: torch.Tensor, packed_out: torch.Tensor | None,
+                            ctas_per_sm: int, stream=None) -> None:
+    """hscale_refine_scales with at most ``ctas_per_sm`` resident CTAs per SM (0: all)."""
     _need(w, torch.bfloat16, "w")
     _need(global_scale, torch.float32, "global_scale")
     _need(codes_out, torch.uint8, "codes_out")
@@ -195,10 +205,10 @@ def hscale_refine_scales(w: torch.Tensor, h: torch.Tensor | None, global_scale: 
             _need(t, torch.uint8, name)
             if t.numel() != size or not t.is_contiguous():
                 raise ValueError(f"{name} must be contiguous with {size} bytes")
-    _check("hscale_refine_scales",
-           load().hscale_refine_scales(_ptr(w), _ptr(h), m, n, _ptr(global_scale), _ptr(init_codes),
-                                       int(down), int(up), _ptr(codes_out), _ptr(packed_out),
-                                       _stream_ptr(stream)))
+    _check("hscale_refine_scales_ex",
+           load().hscale_refine_scales_ex(_ptr(w), _ptr(h), m, n, _ptr(global_scale), _ptr(init_codes),
+                                          int(down), int(up), _ptr(codes_out), _ptr(packed_out),
+                                          int(ctas_per_sm), _stream_ptr(stream)))
 
 
 def hscale_pack_nvfp4(w: torch.Tensor, global_scale: torch.Tensor, codes: torch.Tensor,

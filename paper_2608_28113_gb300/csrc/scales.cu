@@ -493,13 +493,15 @@ cudaError_t launch_rtn_codes(const void* w, int64_t m, int64_t n, const uint32_t
 
 cudaError_t launch_refine(const void* w, const float* h, int64_t m, int64_t n,
                           const float* global_scale, const uint8_t* init_codes, int down, int up,
-                          uint8_t* codes_out, uint8_t* packed_out, cudaStream_t stream) {
+                          uint8_t* codes_out, uint8_t* packed_out, int ctas_per_sm, cudaStream_t stream) {
   DeviceInfo info;
   cudaError_t err = current_device_info(&info);
   if (err != cudaSuccess) return err;
   const int ng = (int)(n / 16);
   const int64_t units = m * ((ng + 31) / 32);
-  const int64_t resident = (int64_t)info.sm_count * occupancy_blocks(refine_kernel, kRefineThreads);
+  int per_sm = occupancy_blocks(refine_kernel, kRefineThreads);
+  if (ctas_per_sm > 0) per_sm = std::min(per_sm, ctas_per_sm);
+  const int64_t resident = (int64_t)info.sm_count * per_sm;
   const int64_t blocks = std::max<int64_t>(1, std::min<int64_t>((units + kWarpsPerRefineBlock - 1) / kWarpsPerRefineBlock, resident));
   refine_kernel<<<(unsigned)blocks, kRefineThreads, 0, stream>>>(
       static_cast<const uint4*>(w), h, m, ng, global_scale, init_codes, down, up, codes_out,

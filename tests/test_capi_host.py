@@ -94,6 +94,15 @@ def test_refine_argument_errors(lib):
     assert f(None, None, 0, 32, None, None, 4, 4, None, None, None) == OK
 
 
+def test_refine_ex_argument_errors(lib):
+    f = lib.hscale_refine_scales_ex
+    assert f(FAKE, FAKE, 4, 32, FAKE, None, 4, 4, FAKE, FAKE, -1, None) == ERR_ARG
+    assert f(FAKE, FAKE, 4, 32, FAKE, None, -1, 4, FAKE, FAKE, 0, None) == ERR_ARG
+    assert f(FAKE, FAKE, 4, 40, FAKE, None, 4, 4, FAKE, FAKE, 5, None) == ERR_SHAPE
+    assert f(FAKE, FAKE, 4, 32, None, None, 4, 4, FAKE, FAKE, 5, None) == ERR_NULL
+    assert f(None, None, 0, 32, None, None, 4, 4, None, None, 5, None) == OK
+
+
 def test_pack_argument_errors(lib):
     f = lib.hscale_pack_nvfp4
     assert f(FAKE, 4, 32, FAKE, None, FAKE, None) == ERR_NULL

@@ -347,6 +347,24 @@ def test_pack_matches_oracle_bit_exact():
         assert np.array_equal(packed.cpu().numpy(), oracle.pack(bits(w), s_ref, c))
 
 
+def test_refine_launch_shape_does_not_change_results():
+    """hscale_refine_scales_ex with 1, 2 or 5 resident CTAs per SM (more units per warp,
+    other unit-to-warp assignment) writes the same bytes as the full launch."""
+    w = small_layer(5, 512, 1024)
+    h = torch.from_numpy(oracle_h32(5, 1024)).to(dev())
+    wd = w.to(dev())
+    sg, _ = gpu_rtn(wd)
+    outs = []
+    for k in (0, 1, 2, 5):
+        codes = torch.empty(512, 64, dtype=torch.uint8, device=dev())
+        packed = torch.empty(512, 512, dtype=torch.uint8, device=dev())
+        hs.hscale_refine_scales_ex(wd, h, sg, None, 9, 6, codes, packed, k)
+        torch.cuda.synchronize()
+        outs.append((codes.cpu(), packed.cpu()))
+    for c, p in outs[1:]:
+        assert torch.equal(c, outs[0][0]) and torch.equal(p, outs[0][1])
+
+
 def test_refine_is_deterministic():
     w = small_layer(3, 512, 1024)
     h32 = oracle_h32(3, 1024)
