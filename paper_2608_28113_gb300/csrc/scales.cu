@@ -308,9 +308,16 @@ refine_kernel(const uint4* __restrict__ w, const float* __restrict__ h, int64_t 
 #pragma unroll
   for (int j = 0; j < 8; ++j) hv2[j] = make_float2(1.0f, 1.0f);
 
-  for (int64_t u = warp_global; u < units; u += warps_total) {
-    const int64_t row = u / chunks;
-    const int chunk = (int)(u - row * chunks);
+  // (row, chunk) of unit u, advanced by warps_total units per step without a division
+  const int row_step = (int)(warps_total / chunks);
+  const int chunk_step = (int)(warps_total - (int64_t)row_step * chunks);
+  int64_t row = warp_global / chunks;
+  int chunk = (int)(warp_global - row * chunks);
+  for (int64_t u = warp_global; u < units; u += warps_total, row += row_step, chunk += chunk_step) {
+    if (chunk >= chunks) {
+      chunk -= chunks;
+      ++row;
+    }
     const int gcol = chunk * 32 + lane;
     const bool active = gcol < ng;
     const int64_t g = row * ng + gcol;
