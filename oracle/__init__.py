@@ -14,6 +14,7 @@ Function map (paper equations in their order of appearance):
   fourover6_codes      Algorithm 2's 4over6 initialization   Sec. 3.5, Algorithm 2
   pack                 final FP4 quantization                Sec. 3.3, Eq. 2
   quantize_at_scale    Eq. 2 at a real scale (App. A.1 microcase)
+  dequant_residual     dW = W - W_hat of packed NVFP4         Eqs. 1-3
   output_error         ||X dW^T||_F^2                        Eq. 3
 """
 from __future__ import annotations
@@ -71,6 +72,7 @@ def _load():
             "oracle_fourover6_codes": (None, [P, i64, i64, f32, P, P]),
             "oracle_quantize_at_scale": (None, [P, i64, f64, P, P]),
             "oracle_output_error": (f64, [P, i64, i64, P, i64]),
+            "oracle_dequant_residual": (None, [P, i64, i64, f32, P, P, P]),
         }
         for name, (res, args) in sig.items():
             fn = getattr(lib, name)
@@ -210,6 +212,17 @@ def quantize_at_scale(w: np.ndarray, s: float) -> tuple[np.ndarray, np.ndarray]:
     codes = np.empty(ww.shape, np.int8)
     _load().oracle_quantize_at_scale(_ptr(ww), ww.size, float(s), _ptr(wh), _ptr(codes))
     return wh, codes
+
+
+def dequant_residual(w_u16: np.ndarray, s_g, codes: np.ndarray, packed: np.ndarray) -> np.ndarray:
+    """dW = W - W_hat (fp64 [m, n]) for packed NVFP4 weights with per-group codes."""
+    w = _u16(w_u16)
+    m, n = w.shape
+    c = np.ascontiguousarray(codes, dtype=np.uint8).reshape(m, n // 16)
+    p = np.ascontiguousarray(packed, dtype=np.uint8).reshape(m, n // 2)
+    out = np.empty((m, n), np.float64)
+    _load().oracle_dequant_residual(_ptr(w), m, n, float(np.float32(s_g)), _ptr(c), _ptr(p), _ptr(out))
+    return out
 
 
 def output_error(X: np.ndarray, dW: np.ndarray) -> float:

@@ -32,6 +32,8 @@
  *   oracle_pack                 final FP4 quantization with given local scales (Sec. 3.3
  *                               "Final re-quantization"; quantizer of Eq. 2)
  *   oracle_quantize_at_scale    Eq. 2 at a real scale s (calibration microcase, App. A.1)
+ *   oracle_dequant_residual     dW = W - W_hat of the packed NVFP4 weights (the dW of Eq. 3;
+ *                               W_hat = s_g * E4M3(code) * E2M1(nibble), Eqs. 1-2)
  *   oracle_output_error         ||X dW^T||_F^2 (Eq. 3)
  *
  * Parity unpinned: the paper does not fix these conventions, so no pin can check
@@ -44,6 +46,7 @@
  */
 #include <math.h>
 #include <stdint.h>
+#include <stdlib.h>
 #include <stddef.h>
 #include <string.h>
 #ifdef _OPENMP
@@ -406,12 +409,53 @@ void oracle_quantize_at_scale(const double* w, int64_t len, double s, double* w_
 /* ||X dW^T||_F^2 = sum_r sum_t (sum_j X_tj dW_rj)^2 (Eq. 3); X is [N, n], dW is [m, n],
  * both row-major fp64. */
 double oracle_output_error(const double* X, int64_t N, int64_t n, const double* dW, int64_t m) {
-  double total = 0.0;
-  for (int64_t r = 0; r < m; ++r)
+  /* one fp64 partial per output row, summed in row order afterwards, so the result does
+   * not depend on the thread count */
+  double* row_total = (double*)malloc((size_t)(m > 0 ? m : 1) * sizeof(double));
+  if (row_total == NULL) return NAN;
+#pragma omp parallel for schedule(static)
+  for (int64_t r = 0; r < m; ++r) {
+    double rt = 0.0;
     for (int64_t t = 0; t < N; ++t) {
       double acc = 0.0;
       for (int64_t j = 0; j < n; ++j) acc += X[t * n + j] * dW[r * n + j];
-      total += acc * acc;
+      rt += acc * acc;
     }
+    row_total[r] = rt;
+  }
+  double total = 0.0;
+  for (int64_t r = 0; r < m; ++r) total += row_total[r];
+  free(row_total);
   return total;
+}
+
+/* ------------------------------------------------------------------ */
+/* quantization residual dW = W - W_hat (the dW of Eq. 3)               */
+/* ------------------------------------------------------------------ */
+/* W_hat_j = sign(nibble_j) * s_g * E4M3(code of the group) * E2M1(magnitude of nibble_j),
+ * the value the packed NVFP4 format encodes (Eq. 1 scale times the Eq. 2 grid value).  A
+ * code off the ladder is read as its clipped index, as in oracle_pack.  s_g * l * q has at
+ * most 24 + 4 + 2 significant bits, so W_hat is exact in fp64; dW is the fp64 rounding of
+ * w - W_hat. */
+void oracle_dequant_residual(const uint16_t* w, int64_t m, int64_t n, float s_g_f,
+                             const uint8_t* codes, const uint8_t* packed, double* dw_out) {
+  const double s_g = (double)s_g_f;
+  const int64_t ng = n / 16;
+#pragma omp parallel for schedule(static)
+  for (int64_t r = 0; r < m; ++r) {
+    for (int64_t i = 0; i < ng; ++i) {
+      const int64_t gi = r * ng + i;
+      int c = codes[gi] & 0x7F;
+      if (c < 1) c = 1;
+      if (c > E4M3_MAX_CODE) c = E4M3_MAX_CODE;
+      const double s = s_g * oracle_e4m3_decode((uint8_t)c);
+      for (int j = 0; j < 16; ++j) {
+        const uint8_t nib = (uint8_t)((packed[gi * 8 + j / 2] >> (4 * (j & 1))) & 0xF);
+        const double mag = s * oracle_e2m1_decode((uint8_t)(nib & 0x7));
+        const double w_hat = (nib & 0x8) ? -mag : mag;
+        const int64_t e = r * n + i * 16 + j;
+        dw_out[e] = bf16_value(w[e]) - w_hat;
+      }
+    }
+  }
 }

@@ -427,3 +427,46 @@ def test_fourover6_saturated_group_keeps_the_top_code():
     s_g, _ = oracle.global_scale(bits)
     codes, nt = oracle.fourover6_codes(bits, s_g)
     assert codes[0, 0] == 126 and nt[0, 0] == 0
+
+
+# ---------------------------------------------------------------- residual and output error (Eq. 3)
+
+def test_dequant_residual_against_nearest_grid_value():
+    """dW = W - W_hat, with W_hat found by a brute-force nearest-grid search per element (a
+    different method from the oracle's decode of the packed nibbles), for RTN codes and for
+    arbitrary codes (off-ladder bytes are clipped, Eq. 10); -0 stays a zero residual."""
+    rng = np.random.default_rng(31)
+    w = random_weights(rng, 8, 64)
+    w[0, :16] = 0x8000                                   # -0
+    s_g, _ = oracle.global_scale(w)
+    ladder = oracle.e4m3_decode_table()
+    wv = bits_to_f64(w)
+    for codes in (oracle.rtn_codes(w, s_g), rng.integers(0, 256, size=(8, 4)).astype(np.uint8)):
+        packed = oracle.pack(w, s_g, codes)
+        dw = oracle.dequant_residual(w, s_g, codes, packed)
+        for r in range(8):
+            for i in range(4):
+                c = min(max(int(codes[r, i]) & 0x7F, 1), 126)
+                s = float(s_g) * ladder[c]
+                for j in range(16):
+                    v = wv[r, 16 * i + j]
+                    k = nearest_e2m1(abs(v), s)
+                    w_hat = math.copysign(E2M1_GRID[k] * s, v) if k else 0.0
+                    assert dw[r, 16 * i + j] == v - w_hat, (r, i, j)
+    assert np.all(dw[0, :16] == 0.0)
+
+
+def test_output_error_closed_forms():
+    """||X dW^T||_F^2: X = I gives ||dW||_F^2; one-hot rows scaled by c give
+    c^2 * sum over the selected columns of the column energies; E scales with c^2."""
+    rng = np.random.default_rng(32)
+    m, n = 5, 24
+    dW = rng.standard_normal((m, n))
+    assert math.isclose(oracle.output_error(np.eye(n), dW), math.fsum((dW ** 2).ravel()), rel_tol=1e-12)
+    cols = rng.integers(0, n, size=9)
+    X = np.zeros((9, n))
+    X[np.arange(9), cols] = 3.0
+    expect = 9.0 * math.fsum(math.fsum(dW[:, j] ** 2) for j in cols)
+    assert math.isclose(oracle.output_error(X, dW), expect, rel_tol=1e-12)
+    Xr = rng.standard_normal((7, n))
+    assert math.isclose(oracle.output_error(2.0 * Xr, dW), 4.0 * oracle.output_error(Xr, dW), rel_tol=1e-12)
