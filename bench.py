@@ -62,6 +62,8 @@ def parse():
                    help="resident search CTAs per SM while the next input space's Hessian pass "
                         "runs alongside (0: run every search after the last Hessian pass)")
     p.add_argument("--no-cpu-baseline", action="store_true")
+    p.add_argument("--no-output-error", action="store_true",
+                   help="skip the tensor-core layer-output error evaluation")
     p.add_argument("--no-e2e", action="store_true")
     return p.parse_args()
 
@@ -500,6 +502,44 @@ def reference_arm(args, d: Dist):
     print(json.dumps(line), flush=True)
 
 
+def output_error_eval(hs, work: Work, peaks: dict, tokens: int = 8192, reps: int = 5):
+    """Layer-output error ||X dW^T||_F^2 (Eq. 3) of the first matrix on one chunk of its
+    calibration tokens, for the RTN codes and for the searched codes of the step, on the
+    tensor cores; with the GEMM's throughput.  Outside the timed step."""
+    M = work.mats[0]
+    S = M.space
+    T = min(tokens, S.tokens)
+    x = S.x[:T]
+    dev = x.device
+    ld = hs.residual_ld(M.n)
+    dw2 = torch.empty(M.m, ld, dtype=torch.bfloat16, device=dev)
+    out = torch.zeros(1, dtype=torch.float64, device=dev)
+    ws = torch.empty(hs.hscale_output_error_workspace_bytes(T, M.m), dtype=torch.uint8, device=dev)
+    rtn_codes = torch.empty_like(M.codes)
+    rtn_packed = torch.empty_like(M.packed)
+    hs.hscale_rtn_scales(M.w, M.sg, rtn_codes, work.ws)
+    hs.hscale_pack_nvfp4(M.w, M.sg, rtn_codes, rtn_packed)
+    err = {}
+    for name, codes, packed in (("rtn", rtn_codes, rtn_packed), ("hscale", M.codes, M.packed)):
+        hs.hscale_dequant_residual(M.w, M.sg, codes, packed, dw2)
+        out.zero_()
+        hs.hscale_output_error(x, dw2, M.m, out, ws)
+        err[name] = float(out.item())
+    ms = timed(lambda: hs.hscale_output_error(x, dw2, M.m, out, ws), reps)
+    ms_res = timed(lambda: hs.hscale_dequant_residual(M.w, M.sg, M.codes, M.packed, dw2), reps)
+    n_pad = ld // 2
+    executed = 2.0 * T * M.m * (2 * n_pad)        # X [hi | lo]^T: K = 2 n_pad
+    useful = 2.0 * T * M.m * M.n                  # X dW^T
+    peak = float(peaks.get("bf16_tflops", 1900.0))
+    return {"matrix": M.name, "tokens": T, "error_rtn": err["rtn"], "error_hscale": err["hscale"],
+            "reduction": 1.0 - err["hscale"] / err["rtn"] if err["rtn"] > 0 else None,
+            "gemm_ms": ms, "gemm_tflops_executed": executed / (ms * 1e-3) / 1e12,
+            "gemm_tflops_useful": useful / (ms * 1e-3) / 1e12,
+            "frac_of_measured_bf16": executed / (ms * 1e-3) / 1e12 / peak, "bf16_peak_tflops": peak,
+            "residual_ms": ms_res,
+            "note": "tcgen05 bf16 GEMM of X with the [hi | lo] split of dW, fused sum of squares"}
+
+
 def shift_statistics(work: Work, win, sample_rows: int = 16):
     """Selected shifts delta = chosen code - initial code over every group of the step
     (from the GPU outputs), and the mean reduction of the Hessian-weighted error per
@@ -610,6 +650,7 @@ def gpu_arm(args, d: Dist):
     torch.cuda.synchronize()
     main = [s for s in sweep if tuple(s["window"]) == tuple(win)][0]
     shifts = shift_statistics(work, win)
+    out_err = None if args.no_output_error else output_error_eval(hs, work, peaks)
 
     # ---- roofline of the dominant kernel (the Hessian pass)
     h_bytes_launch = work.h_bytes / work.h_launches
@@ -660,6 +701,8 @@ def gpu_arm(args, d: Dist):
     if len(sweep) > 1:
         line["search_sweep"] = sweep
     line["shift_statistics"] = shifts
+    if out_err:
+        line["output_error"] = out_err
     if n_layers > 1:
         line["seconds_per_model"] = ms_step * 1e-3 * n_layers
         line["seconds_per_model_note"] = f"{n_layers} layers of identical shapes: per-layer step x {n_layers}"

@@ -17,6 +17,8 @@
  *                                       (Eqs. 6, 13), then re-quantize and pack
  *      hscale_pack_nvfp4                final FP4 quantization with given codes
  *                                       (Sec. 3.3 "Final re-quantization", Eq. 2)
+ *      hscale_dequant_residual          dW = W - W_hat of the packed weights (Eqs. 1-3)
+ *      hscale_output_error              ||X dW^T||_F^2 on the tensor cores (Eq. 3)
  *      hscale_refine_scales_ex          the same with a cap on resident CTAs per SM
  *      hscale_fourover6_codes           the 4over6 initial codes of Algorithm 2, an
  *                                       alternative start for the refinement (Sec. 3.5)
@@ -213,6 +215,41 @@ int hscale_refine_scales_ex(const void* w_bf16, const float* h, int64_t m, int64
  */
 int hscale_pack_nvfp4(const void* w_bf16, int64_t m, int64_t n, const float* global_scale,
                       const uint8_t* codes, uint8_t* packed_out, void* stream);
+
+/*
+ * Quantization residual dW = W - W_hat of packed NVFP4 weights (the dW of Eq. 3), for the
+ * layer-output evaluation below.  W_hat = sign * s_g * E4M3(code) * E2M1(magnitude) per
+ * nibble (Eqs. 1-2); dW is w - s_g * (l q) rounded once to fp32, then split into bf16
+ * hi = RN(dW) and lo = RN(dW - hi), so hi + lo equals dW to a relative 2^-17.
+ *
+ * w          [m, n] bfloat16, 16-byte aligned, n % 16 == 0.
+ * codes      [m, n/16] bytes (sign bit ignored, clamped to [1, 126] as in the pack).
+ * packed     [m, n/2] bytes, 8-byte aligned (the layout hscale_refine_scales writes).
+ * dw2        [m, ld_dw2] bfloat16, 16-byte aligned, written: with n_pad = 64 * ceil(n/64),
+ *            columns [0, n) hold hi, [n_pad, n_pad + n) hold lo, and [n, n_pad) and
+ *            [n_pad + n, 2 n_pad) are zero.  ld_dw2 >= 2 n_pad, ld_dw2 % 8 == 0.
+ */
+int hscale_dequant_residual(const void* w_bf16, int64_t m, int64_t n, const float* global_scale,
+                            const uint8_t* codes, const uint8_t* packed, void* dw2_bf16, int64_t ld_dw2,
+                            void* stream);
+
+/*
+ * Layer-output error of a quantization (Eq. 3): *out_sum += ||X dW^T||_F^2 over this chunk
+ * of calibration tokens, computed on the tensor cores as C = X hi^T + X lo^T (bf16
+ * operands, fp32 accumulation) with the sum of squares of C fused into the GEMM.  Tiles of
+ * 128 tokens x 256 outputs each give one fp64 partial; the partials are added in a fixed
+ * order, so the result is deterministic.
+ *
+ * x          [tokens, ld_x] bfloat16 row-major (first n columns used), 16-byte aligned,
+ *            ld_x % 8 == 0, tokens < 2^31.
+ * dw2        the [m, ld_dw2] output of hscale_dequant_residual for the same n.
+ * out_sum    device fp64 scalar, accumulated (the caller zeroes it once).
+ * workspace  device buffer of hscale_output_error_workspace_bytes(tokens, m) bytes.
+ */
+size_t hscale_output_error_workspace_bytes(int64_t tokens, int64_t m);
+int hscale_output_error(const void* x_bf16, int64_t tokens, int64_t n, int64_t ld_x, const void* dw2_bf16,
+                        int64_t ld_dw2, int64_t m, double* out_sum, void* workspace, size_t workspace_bytes,
+                        void* stream);
 
 #ifdef __cplusplus
 }

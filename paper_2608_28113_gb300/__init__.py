@@ -26,7 +26,8 @@ __all__ = [
     "hscale_hessian_diag_accumulate", "hscale_rtn_workspace_bytes", "hscale_rtn_scales",
     "hscale_rtn_scales_noalloc",
     "hscale_refine_scales", "hscale_refine_scales_ex", "hscale_pack_nvfp4", "hscale_fourover6_codes",
-    "EXPORTED_SYMBOLS",
+    "hscale_dequant_residual", "hscale_output_error_workspace_bytes", "hscale_output_error",
+    "residual_ld", "EXPORTED_SYMBOLS",
 ]
 
 _PKG = pathlib.Path(__file__).resolve().parent
@@ -48,6 +49,9 @@ _SIGNATURES = {
     "hscale_refine_scales_ex": (ctypes.c_int, [_P, _P, _I64, _I64, _P, _P, _I32, _I32, _P, _P, _I32, _P]),
     "hscale_pack_nvfp4": (ctypes.c_int, [_P, _I64, _I64, _P, _P, _P, _P]),
     "hscale_fourover6_codes": (ctypes.c_int, [_P, _I64, _I64, _P, _P, _P]),
+    "hscale_dequant_residual": (ctypes.c_int, [_P, _I64, _I64, _P, _P, _P, _P, _I64, _P]),
+    "hscale_output_error_workspace_bytes": (ctypes.c_size_t, [_I64, _I64]),
+    "hscale_output_error": (ctypes.c_int, [_P, _I64, _I64, _I64, _P, _I64, _I64, _P, _P, ctypes.c_size_t, _P]),
 }
 EXPORTED_SYMBOLS = tuple(_SIGNATURES)
 
@@ -242,3 +246,47 @@ def hscale_fourover6_codes(w: torch.Tensor, global_scale: torch.Tensor, codes: t
     _check("hscale_fourover6_codes",
            load().hscale_fourover6_codes(_ptr(w), m, n, _ptr(global_scale), _ptr(codes),
                                          _stream_ptr(stream)))
+
+
+def residual_ld(n: int) -> int:
+    """Row length (elements) of the [hi | lo] residual matrix for n input features."""
+    return 2 * 64 * ((int(n) + 63) // 64)
+
+
+def hscale_dequant_residual(w: torch.Tensor, global_scale: torch.Tensor, codes: torch.Tensor,
+                            packed: torch.Tensor, dw2: torch.Tensor, stream=None) -> None:
+    """dW = W - W_hat of packed NVFP4 weights into dw2 [m, ld] bf16 as [hi | lo] halves."""
+    _need(w, torch.bfloat16, "w")
+    _need(global_scale, torch.float32, "global_scale")
+    _need(codes, torch.uint8, "codes")
+    _need(packed, torch.uint8, "packed")
+    _need(dw2, torch.bfloat16, "dw2")
+    if not w.is_contiguous() or w.dim() != 2:
+        raise ValueError("w must be a contiguous 2-D tensor")
+    m, n = w.shape
+    if codes.numel() != m * (n // 16) or packed.numel() != m * (n // 2):
+        raise ValueError("codes must be [m, n/16] and packed [m, n/2]")
+    if dw2.dim() != 2 or dw2.shape[0] != m or dw2.stride(1) != 1 or dw2.shape[1] < residual_ld(n):
+        raise ValueError("dw2 must be [m, >= residual_ld(n)] with unit column stride")
+    _check("hscale_dequant_residual",
+           load().hscale_dequant_residual(_ptr(w), m, n, _ptr(global_scale), _ptr(codes), _ptr(packed),
+                                          _ptr(dw2), dw2.stride(0), _stream_ptr(stream)))
+
+
+def hscale_output_error_workspace_bytes(tokens: int, m: int) -> int:
+    return int(load().hscale_output_error_workspace_bytes(int(tokens), int(m)))
+
+
+def hscale_output_error(x: torch.Tensor, dw2: torch.Tensor, m: int, out_sum: torch.Tensor,
+                        workspace: torch.Tensor, stream=None) -> None:
+    """out_sum (fp64, device) += ||X dW^T||_F^2 for x [tokens, n] (row stride ld_x)."""
+    _need(x, torch.bfloat16, "x")
+    _need(dw2, torch.bfloat16, "dw2")
+    _need(out_sum, torch.float64, "out_sum")
+    if x.dim() != 2 or x.stride(1) != 1 or dw2.dim() != 2 or dw2.stride(1) != 1:
+        raise ValueError("x and dw2 must be 2-D with unit column stride")
+    tokens, n = x.shape
+    _check("hscale_output_error",
+           load().hscale_output_error(_ptr(x), tokens, n, x.stride(0), _ptr(dw2), dw2.stride(0), int(m),
+                                      _ptr(out_sum), _ptr(workspace), workspace.numel() * workspace.element_size(),
+                                      _stream_ptr(stream)))

@@ -73,7 +73,11 @@ int hscale_abi_version(void) { return 1; }
 
 int hscale_device_error_flags(uint32_t* flags) {
   if (flags == nullptr) return HSCALE_ERR_NULL;
-  return from_cuda(hscale::read_and_clear_device_error(flags));
+  uint32_t a = 0, b = 0;
+  cudaError_t err = hscale::read_hessian_device_error(&a);
+  if (err == cudaSuccess) err = hscale::read_output_error_device_error(&b);
+  *flags = a | b;
+  return from_cuda(err);
 }
 
 int hscale_hessian_diag_accumulate(const void* x_bf16, int64_t tokens, int64_t n, int64_t ld_x,
@@ -141,6 +145,50 @@ int hscale_fourover6_codes(const void* w_bf16, int64_t m, int64_t n, const float
   if (global_scale == nullptr || codes == nullptr) return HSCALE_ERR_NULL;
   if (!aligned(global_scale, 4)) return HSCALE_ERR_ALIGN;
   return from_cuda(hscale::launch_fourover6(w_bf16, m, n, global_scale, codes, as_stream(stream)));
+}
+
+int hscale_dequant_residual(const void* w_bf16, int64_t m, int64_t n, const float* global_scale,
+                            const uint8_t* codes, const uint8_t* packed, void* dw2_bf16, int64_t ld_dw2,
+                            void* stream) {
+  int st = check_weight(w_bf16, m, n);
+  if (st != HSCALE_OK) return st;
+  if (m == 0 || n == 0) return HSCALE_OK;
+  const int64_t n_pad = (n + 63) / 64 * 64;
+  if (ld_dw2 < 2 * n_pad || m > INT64_MAX / ld_dw2) return HSCALE_ERR_SHAPE;
+  if (global_scale == nullptr || codes == nullptr || packed == nullptr || dw2_bf16 == nullptr)
+    return HSCALE_ERR_NULL;
+  if (!aligned(global_scale, 4) || !aligned(packed, 8) || !aligned(dw2_bf16, 16) || ld_dw2 % 8 != 0)
+    return HSCALE_ERR_ALIGN;
+  return from_cuda(hscale::launch_residual(w_bf16, m, n, global_scale, codes, packed, dw2_bf16, ld_dw2,
+                                           as_stream(stream)));
+}
+
+size_t hscale_output_error_workspace_bytes(int64_t tokens, int64_t m) {
+  if (tokens <= 0 || m <= 0) return 0;
+  const int64_t tiles = hscale::output_error_tiles(tokens, m);
+  return (size_t)((tiles * 8 + 255) / 256 * 256);
+}
+
+int hscale_output_error(const void* x_bf16, int64_t tokens, int64_t n, int64_t ld_x, const void* dw2_bf16,
+                        int64_t ld_dw2, int64_t m, double* out_sum, void* workspace, size_t workspace_bytes,
+                        void* stream) {
+  if (tokens < 0 || n < 0 || m < 0 || ld_x < n) return HSCALE_ERR_SHAPE;
+  if (n % 16 != 0) return HSCALE_ERR_SHAPE;
+  const int64_t n_pad = (n + 63) / 64 * 64;
+  if (ld_dw2 < 2 * n_pad) return HSCALE_ERR_SHAPE;
+  if (tokens == 0 || n == 0 || m == 0) return HSCALE_OK;
+  if (tokens > INT32_MAX || m > INT32_MAX || tokens > INT64_MAX / ld_x || m > INT64_MAX / ld_dw2)
+    return HSCALE_ERR_SHAPE;
+  if (hscale::output_error_tiles(tokens, m) > INT32_MAX) return HSCALE_ERR_SHAPE;
+  if (x_bf16 == nullptr || dw2_bf16 == nullptr || out_sum == nullptr) return HSCALE_ERR_NULL;
+  if (!aligned(x_bf16, 16) || !aligned(dw2_bf16, 16) || !aligned(out_sum, 8) || ld_x % 8 != 0 ||
+      ld_dw2 % 8 != 0)
+    return HSCALE_ERR_ALIGN;
+  if (workspace == nullptr || workspace_bytes < hscale_output_error_workspace_bytes(tokens, m) ||
+      !aligned(workspace, 8))
+    return HSCALE_ERR_WORKSPACE;
+  return from_cuda(hscale::launch_output_error(x_bf16, tokens, n, ld_x, dw2_bf16, ld_dw2, m, out_sum,
+                                               static_cast<double*>(workspace), as_stream(stream)));
 }
 
 int hscale_pack_nvfp4(const void* w_bf16, int64_t m, int64_t n, const float* global_scale,

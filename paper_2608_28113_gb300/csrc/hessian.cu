@@ -196,26 +196,6 @@ hessian_colsumsq_kernel(const __grid_constant__ CUtensorMap xmap, int64_t row0, 
 }
 
 // ---------------------------------------------------------------- host side
-using EncodeTiledFn = CUresult (*)(CUtensorMap*, CUtensorMapDataType, cuuint32_t, void*,
-                                   const cuuint64_t*, const cuuint64_t*, const cuuint32_t*,
-                                   const cuuint32_t*, CUtensorMapInterleave, CUtensorMapSwizzle,
-                                   CUtensorMapL2promotion, CUtensorMapFloatOOBfill);
-
-cudaError_t encode_tiled_fn(EncodeTiledFn* out) {
-  static std::once_flag once;
-  static EncodeTiledFn fn = nullptr;
-  static cudaError_t status = cudaSuccess;
-  std::call_once(once, [] {
-    void* p = nullptr;
-    cudaDriverEntryPointQueryResult q;
-    status = cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &p, 12000, cudaEnableDefault, &q);
-    if (status == cudaSuccess && q != cudaDriverEntryPointSuccess) status = cudaErrorNotSupported;
-    fn = reinterpret_cast<EncodeTiledFn>(p);
-  });
-  *out = fn;
-  return status;
-}
-
 template <int CS>
 cudaError_t launch_cs(const CUtensorMap& map, int64_t tokens, int n, float* h, int tiles,
                       cudaStream_t stream) {
@@ -288,7 +268,22 @@ cudaError_t launch_hessian(const void* x, int64_t tokens, int64_t n, int64_t ld_
   }
 }
 
-cudaError_t read_and_clear_device_error(uint32_t* flags) {
+cudaError_t encode_tiled_fn(EncodeTiledFn* out) {
+  static std::once_flag once;
+  static EncodeTiledFn fn = nullptr;
+  static cudaError_t status = cudaSuccess;
+  std::call_once(once, [] {
+    void* p = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    status = cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &p, 12000, cudaEnableDefault, &q);
+    if (status == cudaSuccess && q != cudaDriverEntryPointSuccess) status = cudaErrorNotSupported;
+    fn = reinterpret_cast<EncodeTiledFn>(p);
+  });
+  *out = fn;
+  return status;
+}
+
+cudaError_t read_hessian_device_error(uint32_t* flags) {
   uint32_t v = 0;
   cudaError_t err = cudaMemcpyFromSymbol(&v, g_device_error, sizeof v);
   if (err != cudaSuccess) return err;

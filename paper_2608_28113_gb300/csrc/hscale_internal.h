@@ -2,6 +2,7 @@
 #pragma once
 #include <cstddef>
 #include <cstdint>
+#include <cuda.h>
 #include <cuda_runtime.h>
 
 namespace hscale {
@@ -35,8 +36,29 @@ cudaError_t launch_refine(const void* w, const float* h, int64_t m, int64_t n,
 cudaError_t launch_fourover6(const void* w, int64_t m, int64_t n, const float* global_scale,
                              uint8_t* codes, cudaStream_t stream);
 
-// Sticky device error flags of this library (bit 0: a bounded wait ran out); cleared on read.
-cudaError_t read_and_clear_device_error(uint32_t* flags);
+// cuTensorMapEncodeTiled, looked up once through the runtime's driver entry point.
+using EncodeTiledFn = CUresult (*)(CUtensorMap*, CUtensorMapDataType, cuuint32_t, void*,
+                                   const cuuint64_t*, const cuuint64_t*, const cuuint32_t*,
+                                   const cuuint32_t*, CUtensorMapInterleave, CUtensorMapSwizzle,
+                                   CUtensorMapL2promotion, CUtensorMapFloatOOBfill);
+cudaError_t encode_tiled_fn(EncodeTiledFn* out);
+
+// dW = W - W_hat of packed NVFP4 weights as a bf16 pair [hi | lo] per row, rows of ld
+// elements: hi in [0, n_pad), lo in [n_pad, 2 n_pad), zero padding, n_pad = 64 * ceil(n / 64).
+cudaError_t launch_residual(const void* w, int64_t m, int64_t n, const float* global_scale,
+                            const uint8_t* codes, const uint8_t* packed, void* dw2, int64_t ld_dw2,
+                            cudaStream_t stream);
+
+// *out += ||X dW^T||_F^2 on the tensor cores; partials holds one double per 128 x 256 tile.
+int64_t output_error_tiles(int64_t tokens, int64_t m);
+cudaError_t launch_output_error(const void* x, int64_t tokens, int64_t n, int64_t ld_x, const void* dw2,
+                                int64_t ld_dw2, int64_t m, double* out, double* partials,
+                                cudaStream_t stream);
+
+// Sticky device error flags of each translation unit (bit 0: a bounded wait ran out);
+// cleared on read.
+cudaError_t read_hessian_device_error(uint32_t* flags);
+cudaError_t read_output_error_device_error(uint32_t* flags);
 
 cudaError_t launch_pack(const void* w, int64_t m, int64_t n, const float* global_scale,
                         const uint8_t* codes, uint8_t* packed_out, cudaStream_t stream);

@@ -1,0 +1,316 @@
+// output_error.cu -- the layer-output error ||X dW^T||_F^2 of an NVFP4 quantization (Eq. 3)
+// on the tcgen05 tensor cores of sm_103a.
+//
+//   residual_kernel       dW = W - W_hat with W_hat = s_g * E4M3(code) * E2M1(nibble), as a
+//                         bf16 pair hi = bf16(dW), lo = bf16(dW - hi), written as one matrix
+//                         [hi | lo] per row (each half zero-padded to n_pad = 64 * ceil(n/64))
+//   output_error_kernel   C = [X | X] [hi | lo]^T = X (hi + lo)^T on the tensor cores (bf16
+//                         operands, fp32 accumulation in tensor memory), fused with the sum of
+//                         squares of C: one fp64 partial per 128 x 256 tile of C
+//   reduce_kernel         the partials summed in tile order, added to the caller's scalar
+//
+// The residual is rounded once (one FMA of the exact w - s_g * (l q)), and hi + lo carries
+// it to a relative 2^-17, so the GEMM sees dW, not a difference of two large products.
+//
+// GEMM tile: 128 tokens x 256 outputs, K in steps of 64 bf16 (one 128-byte swizzle atom
+// per row), a 4-stage ring of TMA loads (48 KB per stage).  Warp 0 issues the loads, warp 1
+// owns the tensor memory and issues the MMAs (M = 128, N = 256, K = 16 each), warps 2-5
+// read the 128 x 256 fp32 accumulator back (each warp its 32-lane quarter) and square and
+// sum it.  Every wait is bounded; one that runs out sets the error flag and the tile's
+// partial becomes NaN.
+#include <algorithm>
+#include <cuda_bf16.h>
+
+#include "hscale_device.cuh"
+#include "hscale_internal.h"
+#include "tcgen05.cuh"
+#include "tma.cuh"
+
+namespace hscale {
+namespace {
+
+constexpr int kBM = 128, kBN = 256, kBK = 64, kStages = 4;
+constexpr int kGemmThreads = 192;
+constexpr uint32_t kTileABytes = kBM * kBK * 2;  // 16 KB
+constexpr uint32_t kTileBBytes = kBN * kBK * 2;  // 32 KB
+constexpr uint32_t kStageBytes = kTileABytes + kTileBBytes;
+constexpr uint32_t kTmemCols = kBN;  // fp32 accumulator: 128 lanes x 256 columns
+constexpr uint32_t kGemmSmemBytes = kStages * kStageBytes + 1024 /* alignment */ + 256 /* barriers */;
+constexpr uint32_t kIdesc = idesc_bf16_f32(kBM, kBN);
+
+__device__ uint32_t g_output_error_flags = 0;
+
+// ---------------------------------------------------------------- residual
+__device__ __forceinline__ uint32_t bf16x2_pack(__nv_bfloat16 lo, __nv_bfloat16 hi) {
+  return (uint32_t)__bfloat16_as_ushort(lo) | ((uint32_t)__bfloat16_as_ushort(hi) << 16);
+}
+
+// One thread per 16-element slot of a [hi | lo] row: slots below ng hold a group, the rest
+// of the padded half is written with zeros.
+__global__ void __launch_bounds__(256) residual_kernel(const uint4* __restrict__ w, int64_t m, int ng,
+                                                       int ng_pad, const float* __restrict__ global_scale,
+                                                       const uint8_t* __restrict__ codes,
+                                                       const uint2* __restrict__ packed,
+                                                       uint4* __restrict__ dw2, int64_t ld_dw2) {
+  const float sg = *global_scale;
+  const int64_t slots = m * ng_pad;
+  for (int64_t t = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; t < slots;
+       t += (int64_t)gridDim.x * blockDim.x) {
+    const int64_t r = t / ng_pad;
+    const int i = (int)(t - r * ng_pad);
+    uint4* hi_dst = dw2 + (r * ld_dw2 + (int64_t)i * 16) / 8;
+    uint4* lo_dst = dw2 + (r * ld_dw2 + (int64_t)(ng_pad + i) * 16) / 8;
+    if (i >= ng) {
+      const uint4 z = make_uint4(0u, 0u, 0u, 0u);
+      hi_dst[0] = z; hi_dst[1] = z; lo_dst[0] = z; lo_dst[1] = z;
+      continue;
+    }
+    const int64_t g = r * ng + i;
+    const uint4 p0 = ld_stream_v4(w + 2 * g), p1 = ld_stream_v4(w + 2 * g + 1);
+    const uint32_t wb[8] = {p0.x, p0.y, p0.z, p0.w, p1.x, p1.y, p1.z, p1.w};
+    uint32_t c = codes[g] & 0x7Fu;
+    c = c < 1u ? 1u : (c > kE4M3MaxCode ? kE4M3MaxCode : c);
+    const float l = e4m3_mag(c);
+    const uint2 nib = packed[g];
+    uint32_t hw[8], lw[8];
+#pragma unroll
+    for (int k = 0; k < 8; ++k) {
+      __nv_bfloat16 h2[2], l2[2];
+#pragma unroll
+      for (int e = 0; e < 2; ++e) {
+        const int j = 2 * k + e;
+        const uint32_t nb = ((j < 8 ? nib.x : nib.y) >> (4 * (j & 7))) & 0xFu;
+        float lq = __fmul_rn(l, e2m1_from_raw((nb & 7u) << 22));  // exact: <= 6 significant bits
+        if (nb & 8u) lq = -lq;
+        const float wv = e ? bf16_hi(wb[k]) : bf16_lo(wb[k]);
+        const float d = __fmaf_rn(-sg, lq, wv);  // w - s_g * l * q, rounded once
+        h2[e] = __float2bfloat16_rn(d);
+        l2[e] = __float2bfloat16_rn(__fsub_rn(d, __bfloat162float(h2[e])));
+      }
+      hw[k] = bf16x2_pack(h2[0], h2[1]);
+      lw[k] = bf16x2_pack(l2[0], l2[1]);
+    }
+    hi_dst[0] = make_uint4(hw[0], hw[1], hw[2], hw[3]);
+    hi_dst[1] = make_uint4(hw[4], hw[5], hw[6], hw[7]);
+    lo_dst[0] = make_uint4(lw[0], lw[1], lw[2], lw[3]);
+    lo_dst[1] = make_uint4(lw[4], lw[5], lw[6], lw[7]);
+  }
+}
+
+// ---------------------------------------------------------------- GEMM + sum of squares
+__device__ __forceinline__ float sum_squares32(const uint32_t (&r)[32]) {
+  float t[16];
+#pragma unroll
+  for (int j = 0; j < 16; ++j) {
+    const float a = __uint_as_float(r[2 * j]), b = __uint_as_float(r[2 * j + 1]);
+    t[j] = __fmaf_rn(a, a, __fmul_rn(b, b));
+  }
+#pragma unroll
+  for (int step = 1; step < 16; step <<= 1)
+#pragma unroll
+    for (int j = 0; j + step < 16; j += 2 * step) t[j] = __fadd_rn(t[j], t[j + step]);
+  return t[0];
+}
+
+__global__ void __launch_bounds__(kGemmThreads, 1)
+output_error_kernel(const __grid_constant__ CUtensorMap xmap, const __grid_constant__ CUtensorMap wmap,
+                    int kb_half, int tiles_n, double* __restrict__ partials) {
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+  uint8_t* tile_a = smem;
+  uint8_t* tile_b = smem + kStages * kTileABytes;
+  uint64_t* full = reinterpret_cast<uint64_t*>(smem + kStages * kStageBytes);
+  uint64_t* empty = full + kStages;
+  uint64_t* acc_ready = empty + kStages;
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(acc_ready + 1);
+  uint32_t* failed = tmem_slot + 1;
+  double* warp_sum = reinterpret_cast<double*>(smem + kStages * kStageBytes + 128);
+
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int tile_m = blockIdx.x / tiles_n, tile_n = blockIdx.x - tile_m * tiles_n;
+  const int kb_total = 2 * kb_half;
+
+  if (threadIdx.x == 0) {
+    for (int s = 0; s < kStages; ++s) {
+      mbar_init(&full[s], 1);
+      mbar_init(&empty[s], 1);
+    }
+    mbar_init(acc_ready, 1);
+    *failed = 0u;
+    mbar_fence_init();
+    prefetch_tensormap(&xmap);
+    prefetch_tensormap(&wmap);
+  }
+  if (warp == 1) {
+    tmem_alloc(smem_addr(tmem_slot), kTmemCols);
+    tmem_relinquish();
+  }
+  tc_fence_before_sync();
+  __syncthreads();
+  tc_fence_after_sync();
+  const uint32_t tmem_d = *tmem_slot;
+
+  if (warp == 0) {
+    if (lane == 0) {
+      uint64_t policy;
+      asm volatile("createpolicy.fractional.L2::evict_last.b64 %0, 1.0;" : "=l"(policy));
+      for (int kb = 0; kb < kb_total; ++kb) {
+        const int s = kb % kStages;
+        const uint32_t round = (uint32_t)(kb / kStages);
+        if (!mbar_wait(&empty[s], (round & 1u) ^ 1u)) {
+          atomicOr(failed, 1u);
+          break;
+        }
+        mbar_arrive_expect_tx(&full[s], kStageBytes);
+        const int xk = (kb < kb_half ? kb : kb - kb_half) * kBK;
+        tma_load_2d(tile_a + s * kTileABytes, &xmap, xk, tile_m * kBM, &full[s], policy);
+        tma_load_2d(tile_b + s * kTileBBytes, &wmap, kb * kBK, tile_n * kBN, &full[s], policy);
+      }
+    }
+  } else if (warp == 1) {
+    if (lane == 0) {
+      int issued = 0;
+      for (int kb = 0; kb < kb_total; ++kb) {
+        const int s = kb % kStages;
+        const uint32_t round = (uint32_t)(kb / kStages);
+        if (!mbar_wait(&full[s], round & 1u)) {
+          atomicOr(failed, 1u);
+          break;
+        }
+        tc_fence_after_sync();
+        const uint64_t ad = smem_desc_k_sw128(smem_addr(tile_a + s * kTileABytes));
+        const uint64_t bd = smem_desc_k_sw128(smem_addr(tile_b + s * kTileBBytes));
+#pragma unroll
+        for (int kk = 0; kk < kBK / 16; ++kk)
+          umma_bf16(tmem_d, ad + 2 * kk, bd + 2 * kk, kIdesc, (uint32_t)(issued++ > 0));
+        umma_commit(smem_addr(&empty[s]));
+      }
+      umma_commit(smem_addr(acc_ready));  // fires once every MMA issued above has completed
+    }
+    __syncwarp();
+  } else {
+    const uint32_t quarter = (uint32_t)(warp & 3);
+    double acc = 0.0;
+    if (mbar_wait(acc_ready, 0u)) {
+      tc_fence_after_sync();
+#pragma unroll 1
+      for (int c0 = 0; c0 < kBN; c0 += 32) {
+        uint32_t r[32];
+        tmem_ld_32x32b_x32(tmem_d + ((quarter * 32u) << 16) + (uint32_t)c0, r);
+        tmem_ld_wait();
+        acc += (double)sum_squares32(r);
+      }
+    } else {
+      atomicOr(failed, 1u);
+    }
+#pragma unroll
+    for (int off = 16; off > 0; off >>= 1) acc += __shfl_xor_sync(0xFFFFFFFFu, acc, off);
+    if (lane == 0) warp_sum[quarter] = acc;
+  }
+  tc_fence_before_sync();
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    double total = (warp_sum[0] + warp_sum[1]) + (warp_sum[2] + warp_sum[3]);
+    if (*failed) {
+      atomicOr(&g_output_error_flags, kErrMbarTimeout);
+      total = __longlong_as_double(0x7FF8000000000000ll);
+    }
+    partials[blockIdx.x] = total;
+  }
+  if (warp == 1) {
+    tc_fence_after_sync();
+    tmem_dealloc(tmem_d, kTmemCols);
+  }
+}
+
+// The partials summed in index order by one block (fixed tree), added to *out.
+__global__ void __launch_bounds__(256) reduce_kernel(const double* __restrict__ partials, int64_t count,
+                                                     double* __restrict__ out) {
+  __shared__ double part[256];
+  double s = 0.0;
+  for (int64_t i = threadIdx.x; i < count; i += blockDim.x) s += partials[i];
+  part[threadIdx.x] = s;
+  __syncthreads();
+  for (int step = 128; step > 0; step >>= 1) {
+    if ((int)threadIdx.x < step) part[threadIdx.x] += part[threadIdx.x + step];
+    __syncthreads();
+  }
+  if (threadIdx.x == 0) *out += part[0];
+}
+
+}  // namespace
+
+cudaError_t launch_residual(const void* w, int64_t m, int64_t n, const float* global_scale,
+                            const uint8_t* codes, const uint8_t* packed, void* dw2, int64_t ld_dw2,
+                            cudaStream_t stream) {
+  DeviceInfo info;
+  cudaError_t err = current_device_info(&info);
+  if (err != cudaSuccess) return err;
+  const int ng = (int)(n / 16);
+  const int ng_pad = (int)((n + 63) / 64 * 4);
+  const int64_t slots = m * ng_pad;
+  const int64_t blocks = std::max<int64_t>(1, std::min<int64_t>((slots + 255) / 256, (int64_t)info.sm_count * 8));
+  residual_kernel<<<(unsigned)blocks, 256, 0, stream>>>(static_cast<const uint4*>(w), m, ng, ng_pad, global_scale,
+                                                        codes, reinterpret_cast<const uint2*>(packed),
+                                                        static_cast<uint4*>(dw2), ld_dw2);
+  return cudaGetLastError();
+}
+
+int64_t output_error_tiles(int64_t tokens, int64_t m) {
+  return ((tokens + kBM - 1) / kBM) * ((m + kBN - 1) / kBN);
+}
+
+cudaError_t launch_output_error(const void* x, int64_t tokens, int64_t n, int64_t ld_x, const void* dw2,
+                                int64_t ld_dw2, int64_t m, double* out, double* partials,
+                                cudaStream_t stream) {
+  EncodeTiledFn encode = nullptr;
+  cudaError_t err = encode_tiled_fn(&encode);
+  if (err != cudaSuccess) return err;
+  const int64_t n_pad = (n + kBK - 1) / kBK * kBK;
+  CUtensorMap xmap, wmap;
+  {
+    const cuuint64_t dims[2] = {(cuuint64_t)n, (cuuint64_t)tokens};
+    const cuuint64_t strides[1] = {(cuuint64_t)ld_x * 2};
+    const cuuint32_t box[2] = {(cuuint32_t)kBK, (cuuint32_t)kBM};
+    const cuuint32_t estr[2] = {1, 1};
+    if (encode(&xmap, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(x), dims, strides, box, estr,
+               CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+               CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) != CUDA_SUCCESS)
+      return cudaErrorInvalidValue;
+  }
+  {
+    const cuuint64_t dims[2] = {(cuuint64_t)(2 * n_pad), (cuuint64_t)m};
+    const cuuint64_t strides[1] = {(cuuint64_t)ld_dw2 * 2};
+    const cuuint32_t box[2] = {(cuuint32_t)kBK, (cuuint32_t)kBN};
+    const cuuint32_t estr[2] = {1, 1};
+    if (encode(&wmap, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(dw2), dims, strides, box, estr,
+               CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+               CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) != CUDA_SUCCESS)
+      return cudaErrorInvalidValue;
+  }
+  static cudaError_t attr_status = cudaFuncSetAttribute(output_error_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                                        (int)kGemmSmemBytes);
+  if (attr_status != cudaSuccess) return attr_status;
+  const int64_t tiles_n = (m + kBN - 1) / kBN;
+  const int64_t tiles = output_error_tiles(tokens, m);
+  output_error_kernel<<<(unsigned)tiles, kGemmThreads, kGemmSmemBytes, stream>>>(
+      xmap, wmap, (int)(n_pad / kBK), (int)tiles_n, partials);
+  err = cudaGetLastError();
+  if (err != cudaSuccess) return err;
+  reduce_kernel<<<1, 256, 0, stream>>>(partials, tiles, out);
+  return cudaGetLastError();
+}
+
+cudaError_t read_output_error_device_error(uint32_t* flags) {
+  uint32_t v = 0;
+  cudaError_t err = cudaMemcpyFromSymbol(&v, g_output_error_flags, sizeof v);
+  if (err != cudaSuccess) return err;
+  *flags = v;
+  if (v) {
+    const uint32_t zero = 0;
+    err = cudaMemcpyToSymbol(g_output_error_flags, &zero, sizeof zero);
+  }
+  return err;
+}
+
+}  // namespace hscale

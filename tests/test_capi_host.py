@@ -103,6 +103,26 @@ def test_refine_ex_argument_errors(lib):
     assert f(None, None, 0, 32, None, None, 4, 4, None, None, 5, None) == OK
 
 
+def test_residual_and_output_error_argument_errors(lib):
+    r = lib.hscale_dequant_residual
+    assert r(FAKE, 4, 24, FAKE, FAKE, FAKE, FAKE, 128, None) == ERR_SHAPE       # n % 16
+    assert r(FAKE, 4, 80, FAKE, FAKE, FAKE, FAKE, 200, None) == ERR_SHAPE       # ld < 2 * 128
+    assert r(FAKE, 4, 64, FAKE, None, FAKE, FAKE, 128, None) == ERR_NULL
+    assert r(FAKE, 4, 64, FAKE, FAKE, FAKE, MIS, 128, None) == ERR_ALIGN
+    assert r(FAKE, 4, 64, FAKE, FAKE, FAKE, FAKE, 132, None) == ERR_ALIGN       # ld % 8
+    assert r(None, 0, 64, None, None, None, None, 0, None) == OK
+    ws = lib.hscale_output_error_workspace_bytes
+    assert ws(0, 256) == 0 and ws(128, 256) == 256 and ws(129, 257) == 256 and ws(128 * 64, 256 * 40) == 20480
+    f = lib.hscale_output_error
+    assert f(FAKE, 128, 64, 64, FAKE, 100, 256, FAKE, FAKE, 256, None) == ERR_SHAPE   # ld_dw2 < 128
+    assert f(FAKE, 128, 40, 40, FAKE, 128, 256, FAKE, FAKE, 256, None) == ERR_SHAPE   # n % 16
+    assert f(FAKE, 128, 64, 64, FAKE, 128, 256, None, FAKE, 256, None) == ERR_NULL
+    assert f(FAKE, 128, 64, 64, FAKE, 128, 256, FAKE, FAKE, 8, None) == ERR_WS
+    assert f(FAKE, 128, 64, 64, FAKE, 128, 256, FAKE, None, 256, None) == ERR_WS
+    assert f(MIS, 128, 64, 64, FAKE, 128, 256, FAKE, FAKE, 256, None) == ERR_ALIGN
+    assert f(None, 0, 64, 64, None, 128, 256, None, None, 0, None) == OK
+
+
 def test_pack_argument_errors(lib):
     f = lib.hscale_pack_nvfp4
     assert f(FAKE, 4, 32, FAKE, None, FAKE, None) == ERR_NULL

@@ -471,6 +471,100 @@ def test_fourover6_then_refine_matches_oracle(down, up):
         assert np.array_equal(codes[~diff], init_ref[~diff])
 
 
+# ------------------------------------------------------------------ output error (Eq. 3)
+
+def oracle_codes_packed(wb, h32, s_ref, window):
+    """Codes and nibbles from the CPU oracle (RTN for window None, else the search)."""
+    if window is None:
+        codes = oracle.rtn_codes(wb, s_ref)
+        return codes, oracle.pack(wb, s_ref, codes)
+    out = oracle.refine(wb, h32, s_ref, None, *window)
+    return out["codes"], out["packed"]
+
+
+def gpu_residual(wd, sg, codes, packed):
+    m, n = wd.shape
+    dw2 = torch.full((m, hs.residual_ld(n)), float("nan"), dtype=torch.bfloat16, device=dev())
+    hs.hscale_dequant_residual(wd, sg, torch.from_numpy(codes).to(dev()), torch.from_numpy(packed).to(dev()), dw2)
+    torch.cuda.synchronize()
+    return dw2
+
+
+@pytest.mark.parametrize("m,n,window", [(64, 1024, None), (48, 80, (4, 4)), (3, 16, (9, 6))])
+def test_dequant_residual_matches_oracle(m, n, window):
+    """hi + lo equals the oracle's dW = W - W_hat within a relative 2^-17 (one fp32 rounding
+    of dW, then the bf16 split), and the padding columns are zero."""
+    w = wl.weight(m, n, 0.02, 40 + n)
+    wb = bits(w)
+    s_ref, _ = oracle.global_scale(wb)
+    codes, packed = oracle_codes_packed(wb, oracle_h32(9, n), s_ref, window)
+    wd = w.to(dev())
+    sg = torch.tensor([s_ref], dtype=torch.float32, device=dev())
+    dw2 = gpu_residual(wd, sg, codes, packed).float().cpu().double().numpy()
+    n_pad = hs.residual_ld(n) // 2
+    hi, lo = dw2[:, :n], dw2[:, n_pad:n_pad + n]
+    ref = oracle.dequant_residual(wb, s_ref, codes, packed)
+    err = np.abs(hi + lo - ref)
+    assert np.all(err <= 2.0 ** -17 * np.abs(ref) + 1e-45), f"max rel {np.max(err / (np.abs(ref) + 1e-300)):.3e}"
+    assert np.all(dw2[:, n:n_pad] == 0) and np.all(dw2[:, n_pad + n:] == 0)
+
+
+def gpu_output_error(xd, dw2, m):
+    out = torch.zeros(1, dtype=torch.float64, device=dev())
+    ws = torch.empty(max(8, hs.hscale_output_error_workspace_bytes(xd.shape[0], m)), dtype=torch.uint8, device=dev())
+    hs.hscale_output_error(xd, dw2, m, out, ws)
+    torch.cuda.synchronize()
+    return float(out.item())
+
+
+OUTPUT_ERROR_RTOL = 1e-4
+
+
+@pytest.mark.parametrize("tokens,m,n", [(128, 256, 64), (300, 300, 80), (512, 512, 1024), (1000, 40, 4096)])
+def test_output_error_matches_oracle(tokens, m, n):
+    """||X dW^T||_F^2 on the tensor cores against the fp64 oracle: ragged tokens, outputs
+    and K (n not a multiple of 64), one tile and many.  Tolerance: the bf16 split of dW
+    (2^-17 relative per element) plus fp32 accumulation over 2 * n_pad products."""
+    w = wl.weight(m, n, 0.02, 50 + n)
+    wb = bits(w)
+    s_ref, _ = oracle.global_scale(wb)
+    codes, packed = oracle_codes_packed(wb, None, s_ref, None)
+    a = wl.channel_magnitudes(n, 1.0, 4, 50.0, 7)
+    x = wl.activation_chunk(tokens, a, 7, n)
+    ref = oracle.output_error(bits_to_f64(x), oracle.dequant_residual(wb, s_ref, codes, packed))
+    wd = w.to(dev())
+    sg = torch.tensor([s_ref], dtype=torch.float32, device=dev())
+    dw2 = gpu_residual(wd, sg, codes, packed)
+    got = gpu_output_error(x.to(dev()), dw2, m)
+    print(f"[parity] output error {tokens}x{n} -> {m}: gpu {got:.9e} oracle {ref:.9e} rel {abs(got - ref) / ref:.2e}")
+    assert abs(got - ref) <= OUTPUT_ERROR_RTOL * ref
+
+
+def test_output_error_strided_tokens_and_accumulation():
+    """x as a strided row slice of a wider buffer, two chunks accumulated into one sum."""
+    m, n = 256, 512
+    w = wl.weight(m, n, 0.02, 61)
+    wb = bits(w)
+    s_ref, _ = oracle.global_scale(wb)
+    codes, packed = oracle_codes_packed(wb, None, s_ref, None)
+    g = torch.Generator().manual_seed(62)
+    xf = (torch.randn(384, n + 64, generator=g)).to(torch.bfloat16)
+    dw = oracle.dequant_residual(wb, s_ref, codes, packed)
+    ref = oracle.output_error(bits_to_f64(xf[:, :n].contiguous()), dw)
+    dw2 = gpu_residual(w.to(dev()), torch.tensor([s_ref], dtype=torch.float32, device=dev()), codes, packed)
+    xd = xf.to(dev())
+    out = torch.zeros(1, dtype=torch.float64, device=dev())
+    ws = torch.empty(hs.hscale_output_error_workspace_bytes(384, m), dtype=torch.uint8, device=dev())
+    hs.hscale_output_error(xd[:200, :n], dw2, m, out, ws)
+    hs.hscale_output_error(xd[200:, :n], dw2, m, out, ws)
+    torch.cuda.synchronize()
+    assert abs(out.item() - ref) <= OUTPUT_ERROR_RTOL * ref
+
+
+def bits_to_f64(x):
+    return x.float().double().numpy()
+
+
 # ------------------------------------------------------------------ full-size workloads
 
 def full_size_check(name, sample_rows, layer_index=0, windows=None, fourover6=False):
