@@ -565,6 +565,33 @@ def bits_to_f64(x):
     return x.float().double().numpy()
 
 
+def test_full_size_output_error_q_proj():
+    """The 4096 x 4096 q_proj layer at full width: RTN and searched (k = 4) quantizations
+    from the oracle, ||X dW^T||^2 over 512 calibration tokens on both sides."""
+    W = wl.WORKLOADS["llama8b-q_proj"]
+    L = W.layers[0]
+    m, n = L.out_features, L.in_features
+    w = wl.weight(m, n, W.sigma_w, W.seed)
+    wb = bits(w)
+    s_ref, _ = oracle.global_scale(wb)
+    a = wl.channel_magnitudes(n, W.sigma_a, W.outlier_channels, W.outlier_channel_mult, W.seed)
+    x = wl.activation_chunk(2048, a, W.seed, 0)
+    h = np.zeros(n)
+    oracle.hessian_accumulate(bits(x), h)
+    xe = x[:512]
+    wd = w.to(dev())
+    sg = torch.tensor([s_ref], dtype=torch.float32, device=dev())
+    got = {}
+    for name, window in (("rtn", None), ("hscale", (4, 4))):
+        codes, packed = oracle_codes_packed(wb, h.astype(np.float32), s_ref, window)
+        ref = oracle.output_error(bits_to_f64(xe), oracle.dequant_residual(wb, s_ref, codes, packed))
+        g = gpu_output_error(xe.to(dev()), gpu_residual(wd, sg, codes, packed), m)
+        assert abs(g - ref) <= OUTPUT_ERROR_RTOL * ref, (name, g, ref)
+        got[name] = g
+    print(f"[parity] q_proj output error over 512 tokens: rtn {got['rtn']:.6e} hscale {got['hscale']:.6e} "
+          f"reduction {1 - got['hscale'] / got['rtn']:.1%}")
+
+
 # ------------------------------------------------------------------ full-size workloads
 
 def full_size_check(name, sample_rows, layer_index=0, windows=None, fourover6=False):
