@@ -77,8 +77,12 @@ class Dist:
         self.pg = None
         if self.world > 1:
             import torch.distributed as dist
+            from datetime import timedelta
             backend = "nccl" if torch.cuda.is_available() else "gloo"
-            dist.init_process_group(backend)
+            # a rank that dies or never arrives makes the others' next collective fail
+            # after this long instead of hanging
+            timeout = timedelta(seconds=float(os.environ.get("HSCALE_PG_TIMEOUT_S", "600")))
+            dist.init_process_group(backend, timeout=timeout)
             self.pg = dist
 
     def barrier(self):

@@ -88,6 +88,14 @@ int hscale_abi_version(void);
 int hscale_device_error_flags(uint32_t* flags);
 
 /*
+ * Self-test of that failure path (the paper has no counterpart): one CTA waits, at most
+ * `polls` polls, on an mbarrier that nothing arrives on, so the wait runs out and sets
+ * bit 0 of the device error flags the way a stalled copy pipeline would, without a fault
+ * or a hang.  The kernel then ends normally and the context stays usable.
+ */
+int hscale_selftest_bounded_wait(uint32_t polls, void* stream);
+
+/*
  * Hessian diagonal, one token chunk (Sec. 3.2, Eq. 4).
  *
  *   h[j] += sum_{t < tokens} x[t * ld_x + j]^2      for j < n

@@ -27,7 +27,7 @@ __all__ = [
     "hscale_rtn_scales_noalloc",
     "hscale_refine_scales", "hscale_refine_scales_ex", "hscale_pack_nvfp4", "hscale_fourover6_codes",
     "hscale_dequant_residual", "hscale_output_error_workspace_bytes", "hscale_output_error",
-    "residual_ld", "EXPORTED_SYMBOLS",
+    "residual_ld", "hscale_selftest_bounded_wait", "EXPORTED_SYMBOLS",
 ]
 
 _PKG = pathlib.Path(__file__).resolve().parent
@@ -41,6 +41,7 @@ _SIGNATURES = {
     "hscale_status_string": (ctypes.c_char_p, [ctypes.c_int]),
     "hscale_abi_version": (ctypes.c_int, []),
     "hscale_device_error_flags": (ctypes.c_int, [_P]),
+    "hscale_selftest_bounded_wait": (ctypes.c_int, [ctypes.c_uint32, _P]),
     "hscale_hessian_diag_accumulate": (ctypes.c_int, [_P, _I64, _I64, _I64, _P, _P]),
     "hscale_rtn_workspace_bytes": (_SZ, []),
     "hscale_rtn_scales": (ctypes.c_int, [_P, _I64, _I64, _P, _P, _P, _SZ, _P]),
@@ -93,6 +94,11 @@ def hscale_status_string(status: int) -> str:
 
 def hscale_abi_version() -> int:
     return int(load().hscale_abi_version())
+
+
+def hscale_selftest_bounded_wait(polls: int, stream=None) -> None:
+    """Launch the bounded-wait self-test (the wait runs out and sets device flag bit 0)."""
+    _check("hscale_selftest_bounded_wait", load().hscale_selftest_bounded_wait(int(polls), _stream_ptr(stream)))
 
 
 def hscale_device_error_flags() -> int:

@@ -73,11 +73,16 @@ int hscale_abi_version(void) { return 1; }
 
 int hscale_device_error_flags(uint32_t* flags) {
   if (flags == nullptr) return HSCALE_ERR_NULL;
-  uint32_t a = 0, b = 0;
+  uint32_t a = 0, b = 0, c = 0;
   cudaError_t err = hscale::read_hessian_device_error(&a);
   if (err == cudaSuccess) err = hscale::read_output_error_device_error(&b);
-  *flags = a | b;
+  if (err == cudaSuccess) err = hscale::read_selftest_device_error(&c);
+  *flags = a | b | c;
   return from_cuda(err);
+}
+
+int hscale_selftest_bounded_wait(uint32_t polls, void* stream) {
+  return from_cuda(hscale::launch_bounded_wait_selftest(polls, as_stream(stream)));
 }
 
 int hscale_hessian_diag_accumulate(const void* x_bf16, int64_t tokens, int64_t n, int64_t ld_x,

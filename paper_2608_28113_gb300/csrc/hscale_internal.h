@@ -59,6 +59,10 @@ cudaError_t launch_output_error(const void* x, int64_t tokens, int64_t n, int64_
 // cleared on read.
 cudaError_t read_hessian_device_error(uint32_t* flags);
 cudaError_t read_output_error_device_error(uint32_t* flags);
+cudaError_t read_selftest_device_error(uint32_t* flags);
+
+// One CTA waits at most `polls` polls on an mbarrier that nothing arrives on.
+cudaError_t launch_bounded_wait_selftest(uint32_t polls, cudaStream_t stream);
 
 cudaError_t launch_pack(const void* w, int64_t m, int64_t n, const float* global_scale,
                         const uint8_t* codes, uint8_t* packed_out, cudaStream_t stream);

@@ -45,6 +45,38 @@ def test_dist_barrier_and_max_over_ranks():
     assert out[0] == out[1] == 3.0
 
 
+def _rank_leaves(rank, world, port, out):
+    os.environ.update(MASTER_ADDR="127.0.0.1", MASTER_PORT=str(port), RANK=str(rank),
+                      WORLD_SIZE=str(world), LOCAL_RANK=str(rank), HSCALE_PG_TIMEOUT_S="5")
+    sys.path.insert(0, ROOT)
+    import bench
+    d = bench.Dist(world)
+    d.barrier()
+    if rank == 1:
+        out[1] = "left"
+        os._exit(0)                  # leaves between steps, with nothing in flight
+    try:
+        d.max(1.0)                   # the next collective of the surviving rank
+        out[0] = "no error"
+    except Exception as e:           # noqa: BLE001 -- any error is the expected outcome
+        out[0] = type(e).__name__
+    os._exit(0)
+
+
+def test_a_rank_that_leaves_makes_the_next_collective_fail_not_hang():
+    """Failure detection on the host: rank 1 exits between steps; rank 0's next
+    collective must end with an error within the process-group timeout."""
+    world = 2
+    out = mp.Manager().dict()
+    ctx = mp.start_processes(_rank_leaves, args=(world, free_port(), out), nprocs=world, join=False,
+                             start_method="spawn")
+    for _ in range(120):
+        if ctx.join(timeout=1):       # True once every process has been joined
+            break
+    assert out.get(1) == "left"
+    assert out.get(0) not in (None, "no error"), out.get(0)
+
+
 def test_rank_layers_are_independent_problems():
     sys.path.insert(0, ROOT)
     from paper_2608_28113_gb300 import workloads as wl
