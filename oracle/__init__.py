@@ -12,6 +12,10 @@ Function map (paper equations in their order of appearance):
   rtn_codes            iota(Q_fp8(amax_group / (6 s_g)))     Sec. 3.3, Eq. 7
   refine               Algorithm 1 with diagnostics          Eqs. 8-13
   fourover6_codes      Algorithm 2's 4over6 initialization   Sec. 3.5, Algorithm 2
+  refine_f64           Algorithm 1 on fp64 weights           (local quantizer of Algorithm 3)
+  hessian_full         H += X^T X                            GPTQ Hessian of Algorithm 3
+  gptq_factor          damped inverse-Cholesky factor        Algorithm 3 (as in GPTQ)
+  gptq_hscale          GPTQ with H-Scale as local quantizer  Algorithm 3
   pack                 final FP4 quantization                Sec. 3.3, Eq. 2
   quantize_at_scale    Eq. 2 at a real scale (App. A.1 microcase)
   dequant_residual     dW = W - W_hat of packed NVFP4         Eqs. 1-3
@@ -73,6 +77,8 @@ def _load():
             "oracle_quantize_at_scale": (None, [P, i64, f64, P, P]),
             "oracle_output_error": (f64, [P, i64, i64, P, i64]),
             "oracle_dequant_residual": (None, [P, i64, i64, f32, P, P, P]),
+            "oracle_refine_f64": (None, [P, P, i64, i64, f32, i32, i32, P, P, P, P]),
+            "oracle_hessian_full": (None, [P, i64, i64, i64, P]),
         }
         for name, (res, args) in sig.items():
             fn = getattr(lib, name)
@@ -231,3 +237,70 @@ def output_error(X: np.ndarray, dW: np.ndarray) -> float:
     D = np.ascontiguousarray(np.atleast_2d(dW), dtype=np.float64)
     return float(_load().oracle_output_error(_ptr(Xd), Xd.shape[0], Xd.shape[1], _ptr(D),
                                              D.shape[0]))
+
+
+def refine_f64(w: np.ndarray, h_f32: np.ndarray | None, s_g, down: int, up: int) -> dict:
+    """Algorithm 1 with RTN initial codes on fp64 weights [m, n]: codes, w_hat (signed
+    dequantized values), packed nibbles, near_tie flags."""
+    wv = np.ascontiguousarray(w, dtype=np.float64)
+    m, n = wv.shape
+    h = None if h_f32 is None else np.ascontiguousarray(h_f32, dtype=np.float32).reshape(n)
+    out = {"codes": np.empty((m, n // 16), np.uint8), "w_hat": np.empty((m, n), np.float64),
+           "packed": np.empty((m, n // 2), np.uint8), "near_tie": np.empty((m, n // 16), np.uint8)}
+    _load().oracle_refine_f64(_ptr(wv), _ptr(h), m, n, float(np.float32(s_g)), int(down), int(up),
+                              _ptr(out["codes"]), _ptr(out["w_hat"]), _ptr(out["packed"]), _ptr(out["near_tie"]))
+    return out
+
+
+def hessian_full(x_u16: np.ndarray, H: np.ndarray, ld: int | None = None, n: int | None = None) -> np.ndarray:
+    """H (fp64 [n, n], in place) += X^T X for x [tokens, ld] uint16 (first n columns)."""
+    x = _u16(x_u16)
+    nn = x.shape[1] if n is None else n
+    L = x.shape[1] if ld is None else ld
+    if H.dtype != np.float64 or not H.flags.c_contiguous or H.shape != (nn, nn):
+        raise ValueError("H must be a contiguous float64 [n, n] array")
+    _load().oracle_hessian_full(_ptr(x), x.shape[0], nn, L, _ptr(H))
+    return H
+
+
+def gptq_factor(H: np.ndarray, damp: float = 0.01) -> tuple[np.ndarray, np.ndarray]:
+    """The damped inverse-Cholesky factor of Algorithm 3, formed as GPTQ forms it: dead
+    columns (H_jj = 0) get H_jj = 1, the diagonal gets damp * mean(diag H), and U is the
+    upper Cholesky factor of (H + damp I)^-1, so U^T U = (H + damp I)^-1.  Returns
+    (U, dead-column mask).  numpy's Cholesky and inverse serve as library steps."""
+    Hd = np.array(H, dtype=np.float64, copy=True)
+    dead = np.diag(Hd) == 0
+    Hd[dead, dead] = 1.0
+    Hd[np.diag_indices_from(Hd)] += damp * float(np.mean(np.diag(Hd)))
+    Hinv = np.linalg.inv(Hd)
+    Hinv = 0.5 * (Hinv + Hinv.T)
+    U = np.linalg.cholesky(Hinv).T
+    return U, dead
+
+
+def gptq_hscale(w_u16: np.ndarray, U: np.ndarray, h_f32: np.ndarray, s_g, block: int, down: int, up: int,
+                dead: np.ndarray | None = None) -> dict:
+    """Algorithm 3 (GPTQ + H-Scale) on bf16 weights: for each block of B columns, quantize
+    the current weights with H-Scale (RTN start, window (down, up), h of the block), form
+    E = (W_b - W_hat_b) / diag(U_b), and update the later columns by
+    W[:, i+B:] -= E U[i:i+B, i+B:].  Returns codes, packed nibbles, w_hat (fp64) and the
+    near-tie flags of every block quantization."""
+    W = (_u16(w_u16).astype(np.uint32) << 16).view(np.float32).astype(np.float64)
+    m, n = W.shape
+    if dead is not None:
+        W[:, dead] = 0.0
+    if block % 16 or n % block:
+        raise ValueError("block must be a multiple of 16 dividing n")
+    h = np.ascontiguousarray(h_f32, dtype=np.float32).reshape(n)
+    out = {"codes": np.empty((m, n // 16), np.uint8), "packed": np.empty((m, n // 2), np.uint8),
+           "w_hat": np.empty((m, n), np.float64), "near_tie": np.empty((m, n // 16), np.uint8)}
+    for i in range(0, n, block):
+        q = refine_f64(W[:, i:i + block], h[i:i + block], s_g, down, up)
+        out["codes"][:, i // 16:(i + block) // 16] = q["codes"]
+        out["packed"][:, i // 2:(i + block) // 2] = q["packed"]
+        out["near_tie"][:, i // 16:(i + block) // 16] = q["near_tie"]
+        out["w_hat"][:, i:i + block] = q["w_hat"]
+        E = (W[:, i:i + block] - q["w_hat"]) / np.diag(U)[i:i + block]
+        if i + block < n:
+            W[:, i + block:] -= E @ U[i:i + block, i + block:]
+    return out

@@ -27,6 +27,9 @@
  *                               E4M3 ladder (Eqs. 8-10), candidate set (Eq. 11), FP4
  *                               projection (Eq. 12), argmin of the diagonal-Hessian
  *                               weighted error (Eqs. 6 and 13), final re-quantization
+ *   oracle_refine_f64           Algorithm 1 on fp64 weights: the local quantizer of
+ *                               Algorithm 3 (GPTQ + H-Scale), whose running weights are fp64
+ *   oracle_hessian_full         H += X^T X, the GPTQ Hessian of Algorithm 3
  *   oracle_fourover6_codes      Algorithm 2's initialization: the better of the anchors
  *                               m/4 and m/6 by plain MSE (Sec. 3.5, Algorithm 2)
  *   oracle_pack                 final FP4 quantization with given local scales (Sec. 3.3
@@ -197,14 +200,25 @@ float oracle_global_scale(const uint16_t* w, int64_t count, double* amax_out) {
  * round-to-nearest-even (saturating) of amax_group / (6 s_g).  A result of code 0
  * (value 0, not on the ladder L+) is clamped to code 1, as the walk of Eq. 10 clips
  * indices to [1, M]. */
-static int rtn_code_of_group(const uint16_t* g, double s_g) {
+static int rtn_code_of_values(const double* v, double s_g) {
   double amax = 0.0;
   for (int j = 0; j < 16; ++j) {
-    double a = fabs(bf16_value(g[j]));
+    double a = fabs(v[j]);
     if (a > amax) amax = a;
   }
   int c = e4m3_rne_sat_quotient(amax, 6.0, s_g);
   return c < 1 ? 1 : c;
+}
+
+/* the 16 values of a bf16 group (exact in fp64) */
+static void group_values(const uint16_t* g, double* v) {
+  for (int j = 0; j < 16; ++j) v[j] = bf16_value(g[j]);
+}
+
+static int rtn_code_of_group(const uint16_t* g, double s_g) {
+  double v[16];
+  group_values(g, v);
+  return rtn_code_of_values(v, s_g);
 }
 
 void oracle_rtn_codes(const uint16_t* w, int64_t m, int64_t n, float s_g, uint8_t* codes) {
@@ -222,11 +236,11 @@ void oracle_rtn_codes(const uint16_t* w, int64_t m, int64_t n, float s_g, uint8_
  * s (<= 28 bits), q_j * s (<= 30 bits) and the residual are exact in fp64; only the
  * squares and the sum round (relative error ~1e-16).  Returns E; writes the magnitude
  * codes if q != NULL. */
-static double group_error(const uint16_t* g, const float* h, double s_g, int code, uint8_t* q) {
+static double group_error_values(const double* v, const float* h, double s_g, int code, uint8_t* q) {
   const double scale = s_g * oracle_e4m3_decode((uint8_t)code);
   double e = 0.0;
   for (int j = 0; j < 16; ++j) {
-    double a = fabs(bf16_value(g[j]));
+    double a = fabs(v[j]);
     int k = e2m1_rne_sat_quotient(a, scale);
     double d = a - oracle_e2m1_decode((uint8_t)k) * scale;
     double hj = h ? (double)h[j] : 1.0;
@@ -234,6 +248,12 @@ static double group_error(const uint16_t* g, const float* h, double s_g, int cod
     if (q) q[j] = (uint8_t)k;
   }
   return e;
+}
+
+static double group_error(const uint16_t* g, const float* h, double s_g, int code, uint8_t* q) {
+  double v[16];
+  group_values(g, v);
+  return group_error_values(v, h, s_g, code, q);
 }
 
 /* nibble = sign(w) << 3 | magnitude code (E2M1 bit layout S.EE.M); the sign bit is
@@ -262,6 +282,45 @@ static void pack_group(const uint16_t* g, const uint8_t* q, uint8_t* out8) {
  *   near_tie: 1 iff the best and the runner-up among distinct codes satisfy
  *             E2 - E1 <= 1e-6 * E2 (both zero counts as a tie); 0 with one code.
  *   delta:    chosen code - c;  e_best, e_init (shift 0), e_second (runner-up or -1). */
+/* Algorithm 1 on one group of values (see above); returns the chosen code and writes the
+ * magnitude codes of the final quantization and the diagnostics. */
+static int refine_group(const double* v, const float* hg, double s_g, int c, int down, int up, uint8_t* q,
+                        uint8_t* near_tie, int16_t* delta_out, double* e_best, double* e_init,
+                        double* e_second) {
+  /* errors by code; a code repeated by the clip is evaluated once */
+  double err[E4M3_MAX_CODE + 1];
+  for (int k = 0; k <= E4M3_MAX_CODE; ++k) err[k] = -1.0;
+  int best = -1, best_shift = 0;
+  double best_e = 0.0;
+  for (int d = -down; d <= up; ++d) {
+    int cc = c + d;
+    if (cc < 1) cc = 1;
+    if (cc > E4M3_MAX_CODE) cc = E4M3_MAX_CODE;
+    if (err[cc] < 0.0) err[cc] = group_error_values(v, hg, s_g, cc, NULL);
+    double e = err[cc];
+    int shift = cc - c;
+    int better = 0;
+    if (best < 0 || e < best_e) better = 1;
+    else if (e == best_e && cc != best) {
+      int as = shift < 0 ? -shift : shift, ab = best_shift < 0 ? -best_shift : best_shift;
+      if (as < ab || (as == ab && shift < best_shift)) better = 1;
+    }
+    if (better) { best = cc; best_e = e; best_shift = shift; }
+  }
+  const double e0 = err[c];
+  /* runner-up over the distinct codes other than the winner */
+  double second = -1.0;
+  for (int cc = 1; cc <= E4M3_MAX_CODE; ++cc)
+    if (cc != best && err[cc] >= 0.0 && (second < 0.0 || err[cc] < second)) second = err[cc];
+  group_error_values(v, hg, s_g, best, q);
+  if (near_tie) *near_tie = (uint8_t)(second >= 0.0 && (second - best_e) <= 1e-6 * second);
+  if (delta_out) *delta_out = (int16_t)best_shift;
+  if (e_best) *e_best = best_e;
+  if (e_init) *e_init = e0;
+  if (e_second) *e_second = second;
+  return best;
+}
+
 void oracle_refine(const uint16_t* w, const float* h, int64_t m, int64_t n, float s_g_f,
                    const uint8_t* init_codes, int down, int up, uint8_t* codes_out,
                    uint8_t* packed_out, uint8_t* near_tie, int16_t* delta_out, double* e_best,
@@ -274,50 +333,71 @@ void oracle_refine(const uint16_t* w, const float* h, int64_t m, int64_t n, floa
       const int64_t gi = r * ng + i;
       const uint16_t* g = w + r * n + i * 16;
       const float* hg = h ? h + i * 16 : NULL;
+      double v[16];
+      group_values(g, v);
       int c;
       if (init_codes) {
         c = init_codes[gi] & 0x7F;
         if (c < 1) c = 1;
         if (c > E4M3_MAX_CODE) c = E4M3_MAX_CODE;
       } else {
-        c = rtn_code_of_group(g, s_g);
+        c = rtn_code_of_values(v, s_g);
       }
-      /* errors by code; a code repeated by the clip is evaluated once */
-      double err[E4M3_MAX_CODE + 1];
-      for (int k = 0; k <= E4M3_MAX_CODE; ++k) err[k] = -1.0;
-      int best = -1, best_shift = 0;
-      double best_e = 0.0;
-      for (int d = -down; d <= up; ++d) {
-        int cc = c + d;
-        if (cc < 1) cc = 1;
-        if (cc > E4M3_MAX_CODE) cc = E4M3_MAX_CODE;
-        if (err[cc] < 0.0) err[cc] = group_error(g, hg, s_g, cc, NULL);
-        double e = err[cc];
-        int shift = cc - c;
-        int better = 0;
-        if (best < 0 || e < best_e) better = 1;
-        else if (e == best_e && cc != best) {
-          int as = shift < 0 ? -shift : shift, ab = best_shift < 0 ? -best_shift : best_shift;
-          if (as < ab || (as == ab && shift < best_shift)) better = 1;
-        }
-        if (better) { best = cc; best_e = e; best_shift = shift; }
-      }
-      const double e0 = err[c];
-      /* runner-up over the distinct codes other than the winner */
-      double second = -1.0;
-      for (int cc = 1; cc <= E4M3_MAX_CODE; ++cc)
-        if (cc != best && err[cc] >= 0.0 && (second < 0.0 || err[cc] < second)) second = err[cc];
       uint8_t q[16];
-      group_error(g, hg, s_g, best, q);
+      const int best = refine_group(v, hg, s_g, c, down, up, q, near_tie ? near_tie + gi : NULL,
+                                    delta_out ? delta_out + gi : NULL, e_best ? e_best + gi : NULL,
+                                    e_init ? e_init + gi : NULL, e_second ? e_second + gi : NULL);
       if (codes_out) codes_out[gi] = (uint8_t)best;
       if (packed_out) pack_group(g, q, packed_out + gi * 8);
-      if (near_tie) near_tie[gi] = (uint8_t)(second >= 0.0 && (second - best_e) <= 1e-6 * second);
-      if (delta_out) delta_out[gi] = (int16_t)best_shift;
-      if (e_best) e_best[gi] = best_e;
-      if (e_init) e_init[gi] = e0;
-      if (e_second) e_second[gi] = second;
     }
   }
+}
+
+/* Algorithm 1 on real-valued (fp64) weights W [m, n] with the RTN initial codes of Eq. 7,
+ * the local quantizer inside GPTQ (Algorithm 3), where the running weights are no longer
+ * bf16.  Rounding decisions stay exact: |w| is compared with mid * s (<= 31 bits, exact)
+ * in fp64.  Writes the codes [m, n/16], the signed dequantized values
+ * W_hat = sign(w) s q [m, n], the packed nibbles [m, n/2] and the near-tie flags
+ * [m, n/16] (any output may be NULL). */
+void oracle_refine_f64(const double* w, const float* h, int64_t m, int64_t n, float s_g_f, int down, int up,
+                       uint8_t* codes_out, double* w_hat, uint8_t* packed_out, uint8_t* near_tie) {
+  const int64_t ng = n / 16;
+  const double s_g = (double)s_g_f;
+#pragma omp parallel for schedule(static)
+  for (int64_t r = 0; r < m; ++r) {
+    for (int64_t i = 0; i < ng; ++i) {
+      const int64_t gi = r * ng + i;
+      const double* v = w + r * n + i * 16;
+      const float* hg = h ? h + i * 16 : NULL;
+      uint8_t q[16];
+      const int best = refine_group(v, hg, s_g, rtn_code_of_values(v, s_g), down, up, q,
+                                    near_tie ? near_tie + gi : NULL, NULL, NULL, NULL, NULL);
+      if (codes_out) codes_out[gi] = (uint8_t)best;
+      const double scale = s_g * oracle_e4m3_decode((uint8_t)best);
+      for (int j = 0; j < 16; ++j) {
+        const double mag = oracle_e2m1_decode(q[j]) * scale;
+        if (w_hat) w_hat[r * n + i * 16 + j] = signbit(v[j]) ? -mag : mag;
+      }
+      if (packed_out)
+        for (int j = 0; j < 8; ++j) {
+          uint8_t lo = (uint8_t)(((signbit(v[2 * j]) ? 1 : 0) << 3) | q[2 * j]);
+          uint8_t hi = (uint8_t)(((signbit(v[2 * j + 1]) ? 1 : 0) << 3) | q[2 * j + 1]);
+          packed_out[gi * 8 + j] = (uint8_t)(lo | (hi << 4));
+        }
+    }
+  }
+}
+
+/* Full Hessian H += X^T X over a token chunk (the GPTQ Hessian of Algorithm 3; its
+ * diagonal is the h of Eq. 4): plain fp64 sums in token order. */
+void oracle_hessian_full(const uint16_t* x, int64_t tokens, int64_t n, int64_t ld, double* H) {
+#pragma omp parallel for schedule(static)
+  for (int64_t i = 0; i < n; ++i)
+    for (int64_t t = 0; t < tokens; ++t) {
+      const double xi = bf16_value(x[t * ld + i]);
+      if (xi == 0.0) continue;
+      for (int64_t j = 0; j < n; ++j) H[i * n + j] += xi * bf16_value(x[t * ld + j]);
+    }
 }
 
 /* All candidate errors of one group over an explicit code list (tests: full-grid and

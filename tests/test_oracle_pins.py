@@ -470,3 +470,108 @@ def test_output_error_closed_forms():
     assert math.isclose(oracle.output_error(X, dW), expect, rel_tol=1e-12)
     Xr = rng.standard_normal((7, n))
     assert math.isclose(oracle.output_error(2.0 * Xr, dW), 4.0 * oracle.output_error(Xr, dW), rel_tol=1e-12)
+
+
+# ---------------------------------------------------------------- GPTQ + H-Scale (Algorithm 3)
+
+def test_full_hessian_diagonal_symmetry_and_closed_form():
+    rng = np.random.default_rng(41)
+    x = to_bf16_bits(rng.standard_normal((37, 24)) * 2.0)
+    H = np.zeros((24, 24))
+    oracle.hessian_full(x, H)
+    h = np.zeros(24)
+    oracle.hessian_accumulate(x, h)
+    assert np.array_equal(np.diag(H), h)          # the diagonal is Eq. 4's h
+    assert np.array_equal(H, H.T)
+    onehot = np.zeros((5, 24))
+    onehot[np.arange(5), [3, 3, 7, 10, 3]] = 2.0
+    H1 = np.zeros((24, 24))
+    oracle.hessian_full(to_bf16_bits(onehot), H1)
+    expect = np.zeros((24, 24))
+    expect[3, 3], expect[7, 7], expect[10, 10] = 12.0, 4.0, 4.0
+    assert np.array_equal(H1, expect)
+
+
+def test_gptq_factor_inverts_the_damped_hessian():
+    rng = np.random.default_rng(42)
+    X = rng.standard_normal((64, 32))
+    X[:, 5] = 0.0                                   # a dead input channel
+    H = X.T @ X
+    U, dead = oracle.gptq_factor(H, damp=0.01)
+    assert dead[5] and dead.sum() == 1
+    Hd = H.copy()
+    Hd[5, 5] = 1.0
+    Hd[np.diag_indices(32)] += 0.01 * np.mean(np.diag(Hd))
+    assert np.allclose(np.triu(U), U) and np.all(np.diag(U) > 0)
+    assert np.allclose(Hd @ (U.T @ U), np.eye(32), atol=1e-9)
+
+
+def test_gptq_one_block_equals_the_search_and_fp64_path_equals_bf16_path():
+    rng = np.random.default_rng(43)
+    w = random_weights(rng, 8, 64)
+    h = random_h(rng, 64)
+    s_g, _ = oracle.global_scale(w)
+    U = np.triu(rng.standard_normal((64, 64))) + 8 * np.eye(64)
+    out = oracle.gptq_hscale(w, U, h, s_g, 64, 4, 4)
+    ref = oracle.refine(w, h, s_g, None, 4, 4)
+    assert np.array_equal(out["codes"], ref["codes"]) and np.array_equal(out["packed"], ref["packed"])
+
+
+def test_gptq_diagonal_factor_does_not_propagate():
+    rng = np.random.default_rng(44)
+    w = random_weights(rng, 8, 64)
+    h = random_h(rng, 64)
+    s_g, _ = oracle.global_scale(w)
+    U = np.diag(rng.uniform(0.5, 2.0, 64))
+    out = oracle.gptq_hscale(w, U, h, s_g, 16, 9, 6)
+    ref = oracle.refine(w, h, s_g, None, 9, 6)
+    assert np.array_equal(out["codes"], ref["codes"]) and np.array_equal(out["packed"], ref["packed"])
+
+
+def brute_force_block(Wb, hb, s_g, down, up):
+    """Brute-force H-Scale on real-valued rows: RTN start by torch's E4M3 cast, every code in
+    the window, nearest-grid FP4 values, math.fsum errors, the tie rule of the search."""
+    ladder = oracle.e4m3_decode_table()
+    codes, w_hat = [], np.zeros_like(Wb)
+    for r in range(Wb.shape[0]):
+        row = []
+        for i in range(Wb.shape[1] // 16):
+            g = Wb[r, 16 * i:16 * i + 16]
+            hg = hb[16 * i:16 * i + 16]
+            c0 = max(1, min(126, int(e4m3_code_by_torch(np.array([np.abs(g).max() / (6 * float(s_g))]))[0])))
+            best = None
+            for d in range(-down, up + 1):
+                c = min(max(c0 + d, 1), 126)
+                s = float(s_g) * ladder[c]
+                q = [E2M1_GRID[nearest_e2m1(abs(v), s)] * s for v in g]
+                e = math.fsum(float(hj) * (abs(v) - qv) ** 2 for v, hj, qv in zip(g, hg, q))
+                key = (e, abs(c - c0), c - c0)
+                if best is None or key < best[0]:
+                    best = (key, c, q)
+            row.append(best[1])
+            w_hat[r, 16 * i:16 * i + 16] = [math.copysign(qv, v) if qv else 0.0 for v, qv in zip(g, best[2])]
+        codes.append(row)
+    return np.array(codes, np.uint8), w_hat
+
+
+def test_gptq_error_propagation_against_brute_force():
+    """Three blocks of 16 columns: every block quantized by brute force on the running
+    weights, E = (W_b - W_hat_b) / U_jj and the later columns updated element by element."""
+    rng = np.random.default_rng(45)
+    m, n, B = 4, 48, 16
+    w = random_weights(rng, m, n)
+    X = rng.standard_normal((96, n)) * np.exp(rng.standard_normal(n))
+    H = X.T @ X
+    h = np.diag(H).astype(np.float32)
+    s_g, _ = oracle.global_scale(w)
+    U, dead = oracle.gptq_factor(H)
+    out = oracle.gptq_hscale(w, U, h, s_g, B, 2, 2, dead=dead)
+    W = bits_to_f64(w).copy()
+    for i in range(0, n, B):
+        codes, w_hat = brute_force_block(W[:, i:i + B], h[i:i + B], s_g, 2, 2)
+        keep = out["near_tie"][:, i // 16:(i + B) // 16] == 0
+        assert np.array_equal(codes[keep], out["codes"][:, i // 16:(i + B) // 16][keep]), i
+        for r in range(m):
+            for j in range(i + B, n):
+                W[r, j] -= math.fsum((W[r, i + k] - w_hat[r, k]) / U[i + k, i + k] * U[i + k, j]
+                                     for k in range(B))
