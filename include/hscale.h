@@ -19,6 +19,9 @@
  *                                       (Sec. 3.3 "Final re-quantization", Eq. 2)
  *      hscale_dequant_residual          dW = W - W_hat of the packed weights (Eqs. 1-3)
  *      hscale_output_error              ||X dW^T||_F^2 on the tensor cores (Eq. 3)
+ *      hscale_hessian_full_accumulate   H += X^T X on the tensor cores (Algorithm 3)
+ *      hscale_gptq_factor               damped inverse-Cholesky factor (Algorithm 3)
+ *      hscale_gptq_hscale               GPTQ with H-Scale as local quantizer (Algorithm 3)
  *      hscale_refine_scales_ex          the same with a cap on resident CTAs per SM
  *      hscale_fourover6_codes           the 4over6 initial codes of Algorithm 2, an
  *                                       alternative start for the refinement (Sec. 3.5)
@@ -258,6 +261,44 @@ size_t hscale_output_error_workspace_bytes(int64_t tokens, int64_t m);
 int hscale_output_error(const void* x_bf16, int64_t tokens, int64_t n, int64_t ld_x, const void* dw2_bf16,
                         int64_t ld_dw2, int64_t m, double* out_sum, void* workspace, size_t workspace_bytes,
                         void* stream);
+
+/*
+ * GPTQ with H-Scale as its local quantizer (Algorithm 3), in three calls.
+ *
+ * 1. hscale_hessian_full_accumulate: H[n, n] (fp32, row stride ld_h) += X^T X over a chunk
+ *    of calibration tokens, on the tensor cores (bf16 products, fp32 accumulation); its
+ *    diagonal is the h of Eq. 4.  x is [tokens, ld_x] bf16 row-major (2-byte aligned);
+ *    the workspace (hscale_hessian_full_workspace_bytes, 256-byte aligned) holds X^T.
+ *
+ * 2. hscale_gptq_factor: the damped inverse-Cholesky factor, formed as GPTQ forms it.
+ *    Channels with H_jj = 0 are dead (dead[j] = 1 if dead is not NULL; their weights are
+ *    zeroed in step 3) and get H_jj = 1; the diagonal gets damp * mean(diag H) (GPTQ uses
+ *    damp = 0.01); U [n, n] (fp32, row stride n) is upper triangular with
+ *    U^T U = (H + damp I)^-1.  Cholesky and the triangular inverse come from cuSOLVER,
+ *    loaded at run time: without it the call returns HSCALE_ERR_CUDA and the rest of the
+ *    library is unaffected.  info is a device int32[3], written with the status of the two
+ *    factorizations and the inverse (0 = success, > 0: not positive definite).  n < 46341.
+ *
+ * 3. hscale_gptq_hscale: for each block of `block` columns (a multiple of 16 dividing n)
+ *    of the running fp32 weights (W with dead columns zeroed): the RTN codes of Eq. 7 of
+ *    the current block weights, the H-Scale search over the window (down, up) with the
+ *    diagonal proxy h [n] (16-byte aligned) and the global scale s_g of the original W,
+ *    with exact E2M1 decisions and the tie rule of hscale_refine_scales; then
+ *    E = (W_b - W_hat_b) / diag(U_b) and W[:, i+B:] -= E U[i:i+B, i+B:] in fp32.  Writes
+ *    codes_out [m, n/16] and packed_out [m, n/2] (8-byte aligned) as hscale_refine_scales
+ *    does.  The workspace (hscale_gptq_workspace_bytes) holds the running weights and E.
+ */
+size_t hscale_hessian_full_workspace_bytes(int64_t tokens, int64_t n);
+int hscale_hessian_full_accumulate(const void* x_bf16, int64_t tokens, int64_t n, int64_t ld_x, float* H,
+                                   int64_t ld_h, void* workspace, size_t workspace_bytes, void* stream);
+size_t hscale_gptq_factor_workspace_bytes(int64_t n);
+int hscale_gptq_factor(const float* H, int64_t n, int64_t ld_h, float damp, float* U, uint8_t* dead,
+                       int32_t* info, void* workspace, size_t workspace_bytes, void* stream);
+size_t hscale_gptq_workspace_bytes(int64_t m, int64_t n, int32_t block);
+int hscale_gptq_hscale(const void* w_bf16, int64_t m, int64_t n, const float* U, const float* h,
+                       const float* global_scale, const uint8_t* dead, int32_t block, int32_t down, int32_t up,
+                       uint8_t* codes_out, uint8_t* packed_out, void* workspace, size_t workspace_bytes,
+                       void* stream);
 
 #ifdef __cplusplus
 }

@@ -27,7 +27,9 @@ __all__ = [
     "hscale_rtn_scales_noalloc",
     "hscale_refine_scales", "hscale_refine_scales_ex", "hscale_pack_nvfp4", "hscale_fourover6_codes",
     "hscale_dequant_residual", "hscale_output_error_workspace_bytes", "hscale_output_error",
-    "residual_ld", "hscale_selftest_bounded_wait", "EXPORTED_SYMBOLS",
+    "residual_ld", "hscale_selftest_bounded_wait", "hscale_hessian_full_workspace_bytes",
+    "hscale_hessian_full_accumulate", "hscale_gptq_factor_workspace_bytes", "hscale_gptq_factor",
+    "hscale_gptq_workspace_bytes", "hscale_gptq_hscale", "EXPORTED_SYMBOLS",
 ]
 
 _PKG = pathlib.Path(__file__).resolve().parent
@@ -53,6 +55,13 @@ _SIGNATURES = {
     "hscale_dequant_residual": (ctypes.c_int, [_P, _I64, _I64, _P, _P, _P, _P, _I64, _P]),
     "hscale_output_error_workspace_bytes": (ctypes.c_size_t, [_I64, _I64]),
     "hscale_output_error": (ctypes.c_int, [_P, _I64, _I64, _I64, _P, _I64, _I64, _P, _P, ctypes.c_size_t, _P]),
+    "hscale_hessian_full_workspace_bytes": (ctypes.c_size_t, [_I64, _I64]),
+    "hscale_hessian_full_accumulate": (ctypes.c_int, [_P, _I64, _I64, _I64, _P, _I64, _P, ctypes.c_size_t, _P]),
+    "hscale_gptq_factor_workspace_bytes": (ctypes.c_size_t, [_I64]),
+    "hscale_gptq_factor": (ctypes.c_int, [_P, _I64, _I64, ctypes.c_float, _P, _P, _P, _P, ctypes.c_size_t, _P]),
+    "hscale_gptq_workspace_bytes": (ctypes.c_size_t, [_I64, _I64, _I32]),
+    "hscale_gptq_hscale": (ctypes.c_int, [_P, _I64, _I64, _P, _P, _P, _P, _I32, _I32, _I32, _P, _P, _P,
+                                          ctypes.c_size_t, _P]),
 }
 EXPORTED_SYMBOLS = tuple(_SIGNATURES)
 
@@ -296,3 +305,62 @@ def hscale_output_error(x: torch.Tensor, dw2: torch.Tensor, m: int, out_sum: tor
            load().hscale_output_error(_ptr(x), tokens, n, x.stride(0), _ptr(dw2), dw2.stride(0), int(m),
                                       _ptr(out_sum), _ptr(workspace), workspace.numel() * workspace.element_size(),
                                       _stream_ptr(stream)))
+
+
+def _workspace(nbytes: int, device) -> torch.Tensor:
+    return torch.empty(max(int(nbytes), 256), dtype=torch.uint8, device=device)
+
+
+def hscale_hessian_full_accumulate(x: torch.Tensor, H: torch.Tensor, workspace: torch.Tensor | None = None,
+                                   stream=None) -> None:
+    """H (fp32 [n, n]) += X^T X for x [tokens, n] bf16 (row stride ld_x) on the tensor cores."""
+    _need(x, torch.bfloat16, "x")
+    _need(H, torch.float32, "H")
+    if x.dim() != 2 or x.stride(1) != 1 or H.dim() != 2 or H.stride(1) != 1:
+        raise ValueError("x and H must be 2-D with unit column stride")
+    tokens, n = x.shape
+    if workspace is None:
+        workspace = _workspace(load().hscale_hessian_full_workspace_bytes(tokens, n), x.device)
+    _check("hscale_hessian_full_accumulate",
+           load().hscale_hessian_full_accumulate(_ptr(x), tokens, n, x.stride(0), _ptr(H), H.stride(0), _ptr(workspace),
+                                                 workspace.numel(), _stream_ptr(stream)))
+
+
+def hscale_gptq_factor(H: torch.Tensor, damp: float, U: torch.Tensor, dead: torch.Tensor | None,
+                       info: torch.Tensor, workspace: torch.Tensor | None = None, stream=None) -> None:
+    """U (fp32 [n, n], upper) with U^T U = (H + damp * mean(diag H) I)^-1, as GPTQ forms it."""
+    _need(H, torch.float32, "H")
+    _need(U, torch.float32, "U")
+    _need(info, torch.int32, "info")
+    n = H.shape[0]
+    if U.shape != (n, n) or not U.is_contiguous() or info.numel() < 3:
+        raise ValueError("U must be contiguous [n, n] and info hold 3 int32")
+    if dead is not None:
+        _need(dead, torch.uint8, "dead")
+    if workspace is None:
+        nbytes = load().hscale_gptq_factor_workspace_bytes(n)
+        if nbytes == 0:
+            raise HScaleError("hscale_gptq_factor_workspace_bytes", 5)
+        workspace = _workspace(nbytes, H.device)
+    _check("hscale_gptq_factor",
+           load().hscale_gptq_factor(_ptr(H), n, H.stride(0), float(damp), _ptr(U), _ptr(dead), _ptr(info),
+                                     _ptr(workspace), workspace.numel(), _stream_ptr(stream)))
+
+
+def hscale_gptq_hscale(w: torch.Tensor, U: torch.Tensor, h: torch.Tensor, global_scale: torch.Tensor,
+                       dead: torch.Tensor | None, block: int, down: int, up: int, codes_out: torch.Tensor,
+                       packed_out: torch.Tensor, workspace: torch.Tensor | None = None, stream=None) -> None:
+    """Algorithm 3: GPTQ over blocks of `block` columns with H-Scale as the local quantizer."""
+    _need(w, torch.bfloat16, "w")
+    for name, t, dt in (("U", U, torch.float32), ("h", h, torch.float32), ("global_scale", global_scale, torch.float32),
+                        ("codes_out", codes_out, torch.uint8), ("packed_out", packed_out, torch.uint8)):
+        _need(t, dt, name)
+    if not w.is_contiguous() or w.dim() != 2:
+        raise ValueError("w must be a contiguous 2-D tensor")
+    m, n = w.shape
+    if workspace is None:
+        workspace = _workspace(load().hscale_gptq_workspace_bytes(m, n, block), w.device)
+    _check("hscale_gptq_hscale",
+           load().hscale_gptq_hscale(_ptr(w), m, n, _ptr(U), _ptr(h), _ptr(global_scale), _ptr(dead), int(block),
+                                     int(down), int(up), _ptr(codes_out), _ptr(packed_out), _ptr(workspace),
+                                     workspace.numel(), _stream_ptr(stream)))

@@ -196,6 +196,71 @@ int hscale_output_error(const void* x_bf16, int64_t tokens, int64_t n, int64_t l
                                                static_cast<double*>(workspace), as_stream(stream)));
 }
 
+size_t hscale_hessian_full_workspace_bytes(int64_t tokens, int64_t n) {
+  if (tokens <= 0 || n <= 0) return 0;
+  return (size_t)((n * hscale::hessian_full_ld(tokens) * 2 + 255) / 256 * 256);
+}
+
+int hscale_hessian_full_accumulate(const void* x_bf16, int64_t tokens, int64_t n, int64_t ld_x, float* H,
+                                   int64_t ld_h, void* workspace, size_t workspace_bytes, void* stream) {
+  if (tokens < 0 || n < 0 || ld_x < n || ld_h < n) return HSCALE_ERR_SHAPE;
+  if (tokens == 0 || n == 0) return HSCALE_OK;
+  if (tokens > INT32_MAX || n > INT32_MAX || tokens > INT64_MAX / ld_x || n > INT64_MAX / ld_h) return HSCALE_ERR_SHAPE;
+  if (x_bf16 == nullptr || H == nullptr) return HSCALE_ERR_NULL;
+  if (!aligned(x_bf16, 2) || !aligned(H, 4)) return HSCALE_ERR_ALIGN;
+  if (workspace == nullptr || workspace_bytes < hscale_hessian_full_workspace_bytes(tokens, n) ||
+      !aligned(workspace, 256))
+    return HSCALE_ERR_WORKSPACE;
+  return from_cuda(hscale::launch_hessian_full(x_bf16, tokens, n, ld_x, H, ld_h, workspace, as_stream(stream)));
+}
+
+size_t hscale_gptq_factor_workspace_bytes(int64_t n) {
+  if (n <= 0 || n > INT32_MAX) return 0;
+  const size_t floats = hscale::gptq_factor_solver_floats(n);
+  return floats ? (floats * 4 + 255) / 256 * 256 : 0;
+}
+
+int hscale_gptq_factor(const float* H, int64_t n, int64_t ld_h, float damp, float* U, uint8_t* dead,
+                       int32_t* info, void* workspace, size_t workspace_bytes, void* stream) {
+  if (n < 0 || ld_h < n || n > 46340) return HSCALE_ERR_SHAPE;  // n^2 < 2^31 (cuSOLVER's int sizes)
+  if (!(damp >= 0.0f)) return HSCALE_ERR_ARG;
+  if (n == 0) return HSCALE_OK;
+  if (H == nullptr || U == nullptr || info == nullptr) return HSCALE_ERR_NULL;
+  if (!aligned(H, 4) || !aligned(U, 4) || !aligned(info, 4)) return HSCALE_ERR_ALIGN;
+  if (!hscale::gptq_solver_available()) return HSCALE_ERR_CUDA;
+  const size_t need = hscale_gptq_factor_workspace_bytes(n);
+  if (workspace == nullptr || need == 0 || workspace_bytes < need || !aligned(workspace, 256))
+    return HSCALE_ERR_WORKSPACE;
+  return from_cuda(hscale::launch_gptq_factor(H, n, ld_h, damp, U, dead, info, static_cast<float*>(workspace),
+                                              workspace_bytes / 4, as_stream(stream)));
+}
+
+size_t hscale_gptq_workspace_bytes(int64_t m, int64_t n, int32_t block) {
+  if (m <= 0 || n <= 0 || block <= 0) return 0;
+  return (size_t)(((m * n + m * (int64_t)block) * 4 + 255) / 256 * 256);
+}
+
+int hscale_gptq_hscale(const void* w_bf16, int64_t m, int64_t n, const float* U, const float* h,
+                       const float* global_scale, const uint8_t* dead, int32_t block, int32_t down, int32_t up,
+                       uint8_t* codes_out, uint8_t* packed_out, void* workspace, size_t workspace_bytes,
+                       void* stream) {
+  int st = check_weight(w_bf16, m, n);
+  if (st != HSCALE_OK) return st;
+  if (block <= 0 || block % 16 != 0 || (n > 0 && n % block != 0)) return HSCALE_ERR_SHAPE;
+  if (down < 0 || up < 0 || down > 125 || up > 125) return HSCALE_ERR_ARG;
+  if (m == 0 || n == 0) return HSCALE_OK;
+  if (U == nullptr || h == nullptr || global_scale == nullptr || codes_out == nullptr || packed_out == nullptr)
+    return HSCALE_ERR_NULL;
+  if (!aligned(U, 4) || !aligned(h, 16) || !aligned(global_scale, 4) || !aligned(packed_out, 8))
+    return HSCALE_ERR_ALIGN;
+  if (workspace == nullptr || workspace_bytes < hscale_gptq_workspace_bytes(m, n, block) || !aligned(workspace, 256))
+    return HSCALE_ERR_WORKSPACE;
+  float* Wf = static_cast<float*>(workspace);
+  float* E = Wf + m * n;
+  return from_cuda(hscale::launch_gptq_hscale(w_bf16, m, n, U, h, global_scale, dead, block, down, up, codes_out,
+                                              packed_out, Wf, E, as_stream(stream)));
+}
+
 int hscale_pack_nvfp4(const void* w_bf16, int64_t m, int64_t n, const float* global_scale,
                       const uint8_t* codes, uint8_t* packed_out, void* stream) {
   int st = check_weight(w_bf16, m, n);

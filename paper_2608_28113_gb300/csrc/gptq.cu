@@ -1,0 +1,308 @@
+// gptq.cu -- GPTQ with H-Scale as the local quantizer (Algorithm 3) on sm_103a.
+//
+//   factor            the damped inverse-Cholesky factor U of GPTQ: dead channels (H_jj = 0)
+//                     get H_jj = 1, the diagonal gets damp * mean(diag), and U is upper
+//                     triangular with U^T U = (H + damp I)^-1.  Cholesky and the inverse come
+//                     from cuSOLVER, loaded at run time (column-major: its lower factor of
+//                     (H + damp I)^-1 is our row-major U).
+//   block_kernel      one thread per 16-element group of a block of B columns of the running
+//                     fp32 weights: the RTN code (Eq. 7) of the current weights, the exact
+//                     H-Scale search over the window (Algorithm 1, exact E2M1 decisions, the
+//                     tie rule of the search), the codes and packed nibbles, and the
+//                     propagated errors E = (W - W_hat) / U_jj
+//   update_kernel     W[:, i+B:] -= E U[i:i+B, i+B:] in fp32 (register-blocked SIMT GEMM)
+#include <dlfcn.h>
+
+#include <algorithm>
+#include <cstdio>
+#include <mutex>
+
+#include <cusolverDn.h>
+
+#include "hscale_device.cuh"
+#include "hscale_internal.h"
+
+namespace hscale {
+namespace {
+
+// ---------------------------------------------------------------- cuSOLVER at run time
+struct Solver {
+  decltype(&cusolverDnCreate) create = nullptr;
+  decltype(&cusolverDnSetStream) set_stream = nullptr;
+  decltype(&cusolverDnSpotrf_bufferSize) potrf_size = nullptr;
+  decltype(&cusolverDnSpotrf) potrf = nullptr;
+  decltype(&cusolverDnSpotri_bufferSize) potri_size = nullptr;
+  decltype(&cusolverDnSpotri) potri = nullptr;
+  bool ok = false;
+};
+
+const Solver& solver() {
+  static Solver s;
+  static std::once_flag once;
+  std::call_once(once, [] {
+    void* lib = nullptr;
+    for (const char* name : {"libcusolver.so.12", "libcusolver.so.11", "libcusolver.so"}) {
+      lib = dlopen(name, RTLD_NOW | RTLD_LOCAL);
+      if (lib) break;
+    }
+    if (!lib) return;
+    s.create = reinterpret_cast<decltype(s.create)>(dlsym(lib, "cusolverDnCreate"));
+    s.set_stream = reinterpret_cast<decltype(s.set_stream)>(dlsym(lib, "cusolverDnSetStream"));
+    s.potrf_size = reinterpret_cast<decltype(s.potrf_size)>(dlsym(lib, "cusolverDnSpotrf_bufferSize"));
+    s.potrf = reinterpret_cast<decltype(s.potrf)>(dlsym(lib, "cusolverDnSpotrf"));
+    s.potri_size = reinterpret_cast<decltype(s.potri_size)>(dlsym(lib, "cusolverDnSpotri_bufferSize"));
+    s.potri = reinterpret_cast<decltype(s.potri)>(dlsym(lib, "cusolverDnSpotri"));
+    s.ok = s.create && s.set_stream && s.potrf_size && s.potrf && s.potri_size && s.potri;
+  });
+  return s;
+}
+
+// one handle per device, created on first use
+cusolverDnHandle_t solver_handle() {
+  static std::mutex mu;
+  static cusolverDnHandle_t handles[64] = {};
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return nullptr;
+  std::lock_guard<std::mutex> lock(mu);
+  if (!handles[dev] && solver().create(&handles[dev]) != CUSOLVER_STATUS_SUCCESS) handles[dev] = nullptr;
+  return handles[dev];
+}
+
+// ---------------------------------------------------------------- factor helpers
+// One block: dead channels, the mean of the diagonal, and the damping added to it.
+__global__ void __launch_bounds__(1024) damp_diagonal_kernel(float* A, int64_t n, float damp, uint8_t* dead) {
+  __shared__ double part[1024];
+  double s = 0.0;
+  for (int64_t j = threadIdx.x; j < n; j += blockDim.x) {
+    float d = A[j * n + j];
+    const bool is_dead = (d == 0.0f);
+    if (is_dead) A[j * n + j] = d = 1.0f;
+    if (dead) dead[j] = (uint8_t)is_dead;
+    s += (double)d;
+  }
+  part[threadIdx.x] = s;
+  __syncthreads();
+  for (int step = 512; step > 0; step >>= 1) {
+    if ((int)threadIdx.x < step) part[threadIdx.x] += part[threadIdx.x + step];
+    __syncthreads();
+  }
+  const float add = (float)((double)damp * part[0] / (double)n);
+  for (int64_t j = threadIdx.x; j < n; j += blockDim.x) A[j * n + j] += add;
+}
+
+// row-major: A[r][c] = A[c][r] for r > c (mirror the upper triangle), or zero it (zero_lower)
+__global__ void __launch_bounds__(256) lower_kernel(float* A, int64_t n, int zero_lower) {
+  const int64_t total = n * n;
+  for (int64_t e = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; e < total; e += (int64_t)gridDim.x * blockDim.x) {
+    const int64_t r = e / n, c = e - r * n;
+    if (r > c) A[e] = zero_lower ? 0.0f : A[c * n + r];
+  }
+}
+
+// ---------------------------------------------------------------- block quantizer
+__device__ __forceinline__ bool better_code(float e, int c, float be, int bc, int c0) {
+  if (e != be) return e < be;
+  const int s = c - c0, bs = bc - c0;
+  const int as = s < 0 ? -s : s, abs_ = bs < 0 ? -bs : bs;
+  return as < abs_ || (as == abs_ && s < bs);
+}
+
+// sum_j h_j (a_j - s' q_j)^2 with exact E2M1 decisions, one rounding per residual and a
+// fixed pairwise sum (relative error <= 8 * 2^-24)
+__device__ float exact_group_score(const float (&a)[16], const float (&hj)[16], uint32_t c, float sgk) {
+  const float l = e4m3_mag(c);
+  const float inv = inv_raw_of(__fmul_rn(l, sgk));
+  float t[16];
+#pragma unroll
+  for (int j = 0; j < 16; ++j) {
+    const uint32_t k = e2m1_code(a[j], inv, l, sgk);
+    const float r = __fmaf_rn(-__fmul_rn(e2m1_from_raw(k << 22), l), sgk, a[j]);
+    t[j] = __fmul_rn(hj[j], __fmul_rn(r, r));
+  }
+#pragma unroll
+  for (int step = 1; step < 16; step <<= 1)
+#pragma unroll
+    for (int j = 0; j + step < 16; j += 2 * step) t[j] = __fadd_rn(t[j], t[j + step]);
+  return t[0];
+}
+
+__global__ void __launch_bounds__(128) block_kernel(const float* __restrict__ W, int64_t m, int64_t n, int64_t col0,
+                                                    int B, const float* __restrict__ h, const float* __restrict__ U,
+                                                    const float* __restrict__ global_scale, int down, int up,
+                                                    uint8_t* __restrict__ codes, uint2* __restrict__ packed,
+                                                    float* __restrict__ E) {
+  const int gpb = B / 16;
+  const int64_t groups = m * gpb;
+  const ScaleDomain d = make_scale_domain(*global_scale);
+  const float inv6 = rtn_inv6_raw(d.sgk);
+  for (int64_t g = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; g < groups; g += (int64_t)gridDim.x * blockDim.x) {
+    const int64_t r = g / gpb;
+    const int i = (int)(g - r * gpb);
+    const int64_t col = col0 + 16 * i;
+    float w[16], a[16], hj[16];
+    float amax = 0.0f;
+#pragma unroll
+    for (int q = 0; q < 4; ++q) {
+      const float4 v = reinterpret_cast<const float4*>(W + r * n + col)[q];
+      const float4 hv = reinterpret_cast<const float4*>(h + col)[q];
+      w[4 * q] = v.x; w[4 * q + 1] = v.y; w[4 * q + 2] = v.z; w[4 * q + 3] = v.w;
+      hj[4 * q] = hv.x; hj[4 * q + 1] = hv.y; hj[4 * q + 2] = hv.z; hj[4 * q + 3] = hv.w;
+    }
+#pragma unroll
+    for (int j = 0; j < 16; ++j) {
+      a[j] = __fmul_rn(fabsf(w[j]), d.pw);
+      amax = fmaxf(amax, a[j]);
+    }
+    const int c0 = (int)rtn_code(amax, d.sgk, inv6);
+    const int lo = max(1, c0 - down), hi = min((int)kE4M3MaxCode, c0 + up);
+    float be = 0.0f;
+    int bc = -1;
+    for (int c = lo; c <= hi; ++c) {
+      const float e = exact_group_score(a, hj, (uint32_t)c, d.sgk);
+      if (bc < 0 || better_code(e, c, be, bc, c0)) {
+        be = e;
+        bc = c;
+      }
+    }
+    const float l = e4m3_mag((uint32_t)bc);
+    const float inv = inv_raw_of(__fmul_rn(l, d.sgk));
+    uint32_t word[2] = {0u, 0u};
+#pragma unroll
+    for (int j = 0; j < 16; ++j) {
+      const uint32_t k = e2m1_code(a[j], inv, l, d.sgk);
+      const uint32_t neg = signbit(w[j]) ? 1u : 0u;
+      word[j >> 3] |= ((neg << 3) | k) << (4 * (j & 7));
+      float what = __fmul_rn(d.sg, __fmul_rn(e2m1_from_raw(k << 22), l));  // s_g (l q), l q exact
+      if (neg) what = -what;
+      E[r * B + 16 * i + j] = __fdiv_rn(__fsub_rn(w[j], what), U[(col + j) * n + col + j]);
+    }
+    codes[r * (n / 16) + col / 16] = (uint8_t)bc;
+    packed[r * (n / 16) + col / 16] = make_uint2(word[0], word[1]);
+  }
+}
+
+// W[r, c1 + c] -= sum_k E[r, k] U[col0 + k, c1 + c], k < B; 128 x 128 tiles, 8 x 8 per thread
+constexpr int kUT = 128, kUK = 8;
+__global__ void __launch_bounds__(256) update_kernel(float* __restrict__ W, int64_t m, int64_t n, int64_t col0, int B,
+                                                     const float* __restrict__ E, const float* __restrict__ U) {
+  __shared__ float As[kUK][kUT];
+  __shared__ float Bs[kUK][kUT];
+  const int64_t c1 = col0 + B;
+  const int64_t row0 = (int64_t)blockIdx.y * kUT, cb = c1 + (int64_t)blockIdx.x * kUT;
+  const int tr = threadIdx.x / 16, tc = threadIdx.x % 16;
+  float acc[8][8];
+#pragma unroll
+  for (int i = 0; i < 8; ++i)
+#pragma unroll
+    for (int j = 0; j < 8; ++j) acc[i][j] = 0.0f;
+  for (int k0 = 0; k0 < B; k0 += kUK) {
+    for (int e = threadIdx.x; e < kUK * kUT; e += 256) {
+      const int kk = e % kUK, rr = e / kUK;
+      const int64_t row = row0 + rr;
+      As[kk][rr] = row < m ? E[row * B + k0 + kk] : 0.0f;
+      const int cc = e % kUT, kb = e / kUT;
+      const int64_t col = cb + cc;
+      Bs[kb][cc] = col < n ? U[(col0 + k0 + kb) * n + col] : 0.0f;
+    }
+    __syncthreads();
+#pragma unroll
+    for (int kk = 0; kk < kUK; ++kk) {
+      float av[8], bv[8];
+#pragma unroll
+      for (int i = 0; i < 8; ++i) av[i] = As[kk][tr * 8 + i];
+#pragma unroll
+      for (int j = 0; j < 8; ++j) bv[j] = Bs[kk][tc * 8 + j];
+#pragma unroll
+      for (int i = 0; i < 8; ++i)
+#pragma unroll
+        for (int j = 0; j < 8; ++j) acc[i][j] = __fmaf_rn(av[i], bv[j], acc[i][j]);
+    }
+    __syncthreads();
+  }
+#pragma unroll
+  for (int i = 0; i < 8; ++i) {
+    const int64_t row = row0 + tr * 8 + i;
+    if (row >= m) continue;
+#pragma unroll
+    for (int j = 0; j < 8; ++j) {
+      const int64_t col = cb + tc * 8 + j;
+      if (col < n) W[row * n + col] -= acc[i][j];
+    }
+  }
+}
+
+__global__ void __launch_bounds__(256) to_fp32_kernel(const uint16_t* __restrict__ w, int64_t m, int64_t n,
+                                                      const uint8_t* __restrict__ dead, float* __restrict__ W) {
+  const int64_t total = m * n;
+  for (int64_t e = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; e < total; e += (int64_t)gridDim.x * blockDim.x) {
+    const int64_t c = e % n;
+    W[e] = (dead && dead[c]) ? 0.0f : __uint_as_float((uint32_t)w[e] << 16);
+  }
+}
+
+}  // namespace
+
+// ---------------------------------------------------------------- host side
+bool gptq_solver_available() { return solver().ok && solver_handle() != nullptr; }
+
+size_t gptq_factor_solver_floats(int64_t n) {
+  if (!gptq_solver_available()) return 0;
+  int a = 0, b = 0;
+  cusolverDnHandle_t hd = solver_handle();
+  if (solver().potrf_size(hd, CUBLAS_FILL_MODE_LOWER, (int)n, nullptr, (int)n, &a) != CUSOLVER_STATUS_SUCCESS ||
+      solver().potri_size(hd, CUBLAS_FILL_MODE_LOWER, (int)n, nullptr, (int)n, &b) != CUSOLVER_STATUS_SUCCESS)
+    return 0;
+  return (size_t)std::max(std::max(a, b), 1);
+}
+
+cudaError_t launch_gptq_factor(const float* H, int64_t n, int64_t ld_h, float damp, float* Uo, uint8_t* dead,
+                               int32_t* info, float* work, size_t work_floats, cudaStream_t stream) {
+  if (!gptq_solver_available()) return cudaErrorNotSupported;
+  const Solver& sv = solver();
+  cusolverDnHandle_t hd = solver_handle();
+  if (sv.set_stream(hd, stream) != CUSOLVER_STATUS_SUCCESS) return cudaErrorUnknown;
+  cudaError_t err = cudaMemcpy2DAsync(Uo, (size_t)n * 4, H, (size_t)ld_h * 4, (size_t)n * 4, (size_t)n,
+                                      cudaMemcpyDeviceToDevice, stream);
+  if (err != cudaSuccess) return err;
+  damp_diagonal_kernel<<<1, 1024, 0, stream>>>(Uo, n, damp, dead);
+  if ((err = cudaGetLastError()) != cudaSuccess) return err;
+  const int ni = (int)n, lw = (int)work_floats;
+  if (sv.potrf(hd, CUBLAS_FILL_MODE_LOWER, ni, Uo, ni, work, lw, info) != CUSOLVER_STATUS_SUCCESS) return cudaErrorUnknown;
+  if (sv.potri(hd, CUBLAS_FILL_MODE_LOWER, ni, Uo, ni, work, lw, info + 1) != CUSOLVER_STATUS_SUCCESS)
+    return cudaErrorUnknown;
+  DeviceInfo dinfo;
+  if ((err = current_device_info(&dinfo)) != cudaSuccess) return err;
+  const unsigned blocks = (unsigned)std::min<int64_t>((n * n + 255) / 256, (int64_t)dinfo.sm_count * 16);
+  lower_kernel<<<blocks, 256, 0, stream>>>(Uo, n, 0);
+  if ((err = cudaGetLastError()) != cudaSuccess) return err;
+  if (sv.potrf(hd, CUBLAS_FILL_MODE_LOWER, ni, Uo, ni, work, lw, info + 2) != CUSOLVER_STATUS_SUCCESS)
+    return cudaErrorUnknown;
+  lower_kernel<<<blocks, 256, 0, stream>>>(Uo, n, 1);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_gptq_hscale(const void* w, int64_t m, int64_t n, const float* U, const float* h,
+                               const float* global_scale, const uint8_t* dead, int block, int down, int up,
+                               uint8_t* codes, uint8_t* packed, float* Wf, float* E, cudaStream_t stream) {
+  DeviceInfo info;
+  cudaError_t err = current_device_info(&info);
+  if (err != cudaSuccess) return err;
+  const unsigned cvt_blocks = (unsigned)std::min<int64_t>((m * n + 255) / 256, (int64_t)info.sm_count * 16);
+  to_fp32_kernel<<<cvt_blocks, 256, 0, stream>>>(static_cast<const uint16_t*>(w), m, n, dead, Wf);
+  if ((err = cudaGetLastError()) != cudaSuccess) return err;
+  for (int64_t col0 = 0; col0 < n; col0 += block) {
+    const int64_t groups = m * (block / 16);
+    const unsigned qb = (unsigned)std::min<int64_t>((groups + 127) / 128, (int64_t)info.sm_count * 16);
+    block_kernel<<<qb, 128, 0, stream>>>(Wf, m, n, col0, block, h, U, global_scale, down, up, codes,
+                                         reinterpret_cast<uint2*>(packed), E);
+    if ((err = cudaGetLastError()) != cudaSuccess) return err;
+    if (col0 + block < n) {
+      const dim3 ug((unsigned)((n - col0 - block + kUT - 1) / kUT), (unsigned)((m + kUT - 1) / kUT));
+      update_kernel<<<ug, 256, 0, stream>>>(Wf, m, n, col0, block, E, U);
+      if ((err = cudaGetLastError()) != cudaSuccess) return err;
+    }
+  }
+  return cudaSuccess;
+}
+
+}  // namespace hscale

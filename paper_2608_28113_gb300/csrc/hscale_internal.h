@@ -55,6 +55,21 @@ cudaError_t launch_output_error(const void* x, int64_t tokens, int64_t n, int64_
                                 int64_t ld_dw2, int64_t m, double* out, double* partials,
                                 cudaStream_t stream);
 
+// H[n, n] (row stride ld_h) += X^T X on the tensor cores; xt is scratch for X^T
+// (n rows of hessian_full_ld(tokens) bf16).
+int64_t hessian_full_ld(int64_t tokens);
+cudaError_t launch_hessian_full(const void* x, int64_t tokens, int64_t n, int64_t ld_x, float* H, int64_t ld_h,
+                                void* xt, cudaStream_t stream);
+
+// Algorithm 3 (GPTQ + H-Scale).  The factor needs cuSOLVER, loaded at run time.
+bool gptq_solver_available();
+size_t gptq_factor_solver_floats(int64_t n);  // 0 if cuSOLVER is unavailable
+cudaError_t launch_gptq_factor(const float* H, int64_t n, int64_t ld_h, float damp, float* U, uint8_t* dead,
+                               int32_t* info, float* work, size_t work_floats, cudaStream_t stream);
+cudaError_t launch_gptq_hscale(const void* w, int64_t m, int64_t n, const float* U, const float* h,
+                               const float* global_scale, const uint8_t* dead, int block, int down, int up,
+                               uint8_t* codes, uint8_t* packed, float* Wf, float* E, cudaStream_t stream);
+
 // Sticky device error flags of each translation unit (bit 0: a bounded wait ran out);
 // cleared on read.
 cudaError_t read_hessian_device_error(uint32_t* flags);

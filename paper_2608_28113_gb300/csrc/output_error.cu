@@ -8,6 +8,10 @@
 //                         operands, fp32 accumulation in tensor memory), fused with the sum of
 //                         squares of C: one fp64 partial per 128 x 256 tile of C
 //   reduce_kernel         the partials summed in tile order, added to the caller's scalar
+//   transpose_kernel      X [tokens, n] -> X^T [n, tokens] (tokens contiguous per channel)
+//   gemm_kernel<true>     H += X^T X, the full Hessian of Algorithm 3, with the same tensor-
+//                         core pipeline over K = tokens and an epilogue that adds each
+//                         128 x 256 tile of the product into H
 //
 // The residual is rounded once (one FMA of the exact w - s_g * (l q)), and hi + lo carries
 // it to a relative 2^-17, so the GEMM sees dW, not a difference of two large products.
@@ -112,9 +116,14 @@ __device__ __forceinline__ float sum_squares32(const uint32_t (&r)[32]) {
   return t[0];
 }
 
+// kAccum = false: the sum-of-squares GEMM of the output error (K runs over [X | X], kb_half
+// blocks per half).  kAccum = true: H[rows, cols] += A B^T over kb_half K blocks, both
+// operands rows of X^T.
+template <bool kAccum>
 __global__ void __launch_bounds__(kGemmThreads, 1)
-output_error_kernel(const __grid_constant__ CUtensorMap xmap, const __grid_constant__ CUtensorMap wmap,
-                    int kb_half, int tiles_n, double* __restrict__ partials) {
+gemm_kernel(const __grid_constant__ CUtensorMap xmap, const __grid_constant__ CUtensorMap wmap,
+            int kb_half, int tiles_n, double* __restrict__ partials, float* __restrict__ H, int64_t h_rows,
+            int64_t h_cols, int64_t ld_h) {
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
   uint8_t* tile_a = smem;
@@ -128,7 +137,7 @@ output_error_kernel(const __grid_constant__ CUtensorMap xmap, const __grid_const
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int tile_m = blockIdx.x / tiles_n, tile_n = blockIdx.x - tile_m * tiles_n;
-  const int kb_total = 2 * kb_half;
+  const int kb_total = kAccum ? kb_half : 2 * kb_half;
 
   if (threadIdx.x == 0) {
     for (int s = 0; s < kStages; ++s) {
@@ -162,7 +171,7 @@ output_error_kernel(const __grid_constant__ CUtensorMap xmap, const __grid_const
           break;
         }
         mbar_arrive_expect_tx(&full[s], kStageBytes);
-        const int xk = (kb < kb_half ? kb : kb - kb_half) * kBK;
+        const int xk = (kAccum || kb < kb_half ? kb : kb - kb_half) * kBK;
         tma_load_2d(tile_a + s * kTileABytes, &xmap, xk, tile_m * kBM, &full[s], policy);
         tma_load_2d(tile_b + s * kTileBBytes, &wmap, kb * kBK, tile_n * kBN, &full[s], policy);
       }
@@ -188,6 +197,39 @@ output_error_kernel(const __grid_constant__ CUtensorMap xmap, const __grid_const
       umma_commit(smem_addr(acc_ready));  // fires once every MMA issued above has completed
     }
     __syncwarp();
+  } else if (kAccum) {
+    // row of H held by this thread (TMEM lane = row of the tile), 32 columns at a time
+    const uint32_t quarter = (uint32_t)(warp & 3);
+    const int64_t row = (int64_t)tile_m * kBM + quarter * 32 + lane;
+    const int64_t col0 = (int64_t)tile_n * kBN;
+    if (mbar_wait(acc_ready, 0u)) {
+      tc_fence_after_sync();
+#pragma unroll 1
+      for (int c0 = 0; c0 < kBN; c0 += 32) {
+        uint32_t r[32];
+        tmem_ld_32x32b_x32(tmem_d + ((quarter * 32u) << 16) + (uint32_t)c0, r);
+        tmem_ld_wait();
+        if (row < h_rows) {
+          float* dst = H + row * ld_h + col0 + c0;
+          if (col0 + c0 + 32 <= h_cols && ((ld_h | (col0 + c0)) & 3) == 0 &&
+              (reinterpret_cast<uintptr_t>(H) & 15) == 0) {
+#pragma unroll
+            for (int q = 0; q < 8; ++q) {
+              float4 v = reinterpret_cast<float4*>(dst)[q];
+              v.x += __uint_as_float(r[4 * q]);
+              v.y += __uint_as_float(r[4 * q + 1]);
+              v.z += __uint_as_float(r[4 * q + 2]);
+              v.w += __uint_as_float(r[4 * q + 3]);
+              reinterpret_cast<float4*>(dst)[q] = v;
+            }
+          } else {
+            for (int q = 0; q < 32 && col0 + c0 + q < h_cols; ++q) dst[q] += __uint_as_float(r[q]);
+          }
+        }
+      }
+    } else {
+      atomicOr(failed, 1u);
+    }
   } else {
     const uint32_t quarter = (uint32_t)(warp & 3);
     double acc = 0.0;
@@ -209,7 +251,17 @@ output_error_kernel(const __grid_constant__ CUtensorMap xmap, const __grid_const
   }
   tc_fence_before_sync();
   __syncthreads();
-  if (threadIdx.x == 0) {
+  if (kAccum) {
+    // a wait that ran out makes the whole tile NaN (written after the partial sums above)
+    if (*failed && warp >= 2) {
+      const uint32_t quarter = (uint32_t)(warp & 3);
+      const int64_t row = (int64_t)tile_m * kBM + quarter * 32 + lane;
+      if (row < h_rows)
+        for (int64_t c = (int64_t)tile_n * kBN; c < (int64_t)(tile_n + 1) * kBN && c < h_cols; ++c)
+          H[row * ld_h + c] = __int_as_float(0x7FC00000);
+      if (threadIdx.x == 64) atomicOr(&g_output_error_flags, kErrMbarTimeout);
+    }
+  } else if (threadIdx.x == 0) {
     double total = (warp_sum[0] + warp_sum[1]) + (warp_sum[2] + warp_sum[3]);
     if (*failed) {
       atomicOr(&g_output_error_flags, kErrMbarTimeout);
@@ -220,6 +272,24 @@ output_error_kernel(const __grid_constant__ CUtensorMap xmap, const __grid_const
   if (warp == 1) {
     tc_fence_after_sync();
     tmem_dealloc(tmem_d, kTmemCols);
+  }
+}
+
+// X [tokens, n] (row stride ld_x) -> Xt [n, tokens] (row stride ld_t), 32 x 32 tiles
+// through shared memory so both the reads and the writes are coalesced.
+__global__ void __launch_bounds__(256) transpose_kernel(const uint16_t* __restrict__ x, int64_t tokens, int64_t n,
+                                                        int64_t ld_x, uint16_t* __restrict__ xt, int64_t ld_t) {
+  __shared__ uint16_t tile[32][33];
+  const int64_t t0 = (int64_t)blockIdx.x * 32, c0 = (int64_t)blockIdx.y * 32;
+  const int tx = threadIdx.x & 31, ty = threadIdx.x >> 5;  // 8 rows of 32 per pass
+  for (int k = ty; k < 32; k += 8) {
+    const int64_t t = t0 + k, c = c0 + tx;
+    tile[k][tx] = (t < tokens && c < n) ? x[t * ld_x + c] : (uint16_t)0;
+  }
+  __syncthreads();
+  for (int k = ty; k < 32; k += 8) {
+    const int64_t c = c0 + k, t = t0 + tx;
+    if (c < n && t < tokens) xt[c * ld_t + t] = tile[tx][k];
   }
 }
 
@@ -288,16 +358,50 @@ cudaError_t launch_output_error(const void* x, int64_t tokens, int64_t n, int64_
                CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) != CUDA_SUCCESS)
       return cudaErrorInvalidValue;
   }
-  static cudaError_t attr_status = cudaFuncSetAttribute(output_error_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+  static cudaError_t attr_status = cudaFuncSetAttribute(gemm_kernel<false>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                                         (int)kGemmSmemBytes);
   if (attr_status != cudaSuccess) return attr_status;
   const int64_t tiles_n = (m + kBN - 1) / kBN;
   const int64_t tiles = output_error_tiles(tokens, m);
-  output_error_kernel<<<(unsigned)tiles, kGemmThreads, kGemmSmemBytes, stream>>>(
-      xmap, wmap, (int)(n_pad / kBK), (int)tiles_n, partials);
+  gemm_kernel<false><<<(unsigned)tiles, kGemmThreads, kGemmSmemBytes, stream>>>(
+      xmap, wmap, (int)(n_pad / kBK), (int)tiles_n, partials, nullptr, 0, 0, 0);
   err = cudaGetLastError();
   if (err != cudaSuccess) return err;
   reduce_kernel<<<1, 256, 0, stream>>>(partials, tiles, out);
+  return cudaGetLastError();
+}
+
+int64_t hessian_full_ld(int64_t tokens) { return (tokens + 7) / 8 * 8; }
+
+cudaError_t launch_hessian_full(const void* x, int64_t tokens, int64_t n, int64_t ld_x, float* H, int64_t ld_h,
+                                void* xt, cudaStream_t stream) {
+  const int64_t ld_t = hessian_full_ld(tokens);
+  const dim3 tgrid((unsigned)((tokens + 31) / 32), (unsigned)((n + 31) / 32));
+  transpose_kernel<<<tgrid, 256, 0, stream>>>(static_cast<const uint16_t*>(x), tokens, n, ld_x,
+                                              static_cast<uint16_t*>(xt), ld_t);
+  cudaError_t err = cudaGetLastError();
+  if (err != cudaSuccess) return err;
+  EncodeTiledFn encode = nullptr;
+  err = encode_tiled_fn(&encode);
+  if (err != cudaSuccess) return err;
+  CUtensorMap amap, bmap;
+  const cuuint64_t dims[2] = {(cuuint64_t)tokens, (cuuint64_t)n};
+  const cuuint64_t strides[1] = {(cuuint64_t)ld_t * 2};
+  const cuuint32_t estr[2] = {1, 1};
+  const cuuint32_t abox[2] = {(cuuint32_t)kBK, (cuuint32_t)kBM};
+  const cuuint32_t bbox[2] = {(cuuint32_t)kBK, (cuuint32_t)kBN};
+  if (encode(&amap, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, xt, dims, strides, abox, estr, CU_TENSOR_MAP_INTERLEAVE_NONE,
+             CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) != CUDA_SUCCESS ||
+      encode(&bmap, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, xt, dims, strides, bbox, estr, CU_TENSOR_MAP_INTERLEAVE_NONE,
+             CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) != CUDA_SUCCESS)
+    return cudaErrorInvalidValue;
+  static cudaError_t attr_status = cudaFuncSetAttribute(gemm_kernel<true>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                                        (int)kGemmSmemBytes);
+  if (attr_status != cudaSuccess) return attr_status;
+  const int64_t tiles_n = (n + kBN - 1) / kBN;
+  const int64_t tiles = ((n + kBM - 1) / kBM) * tiles_n;
+  gemm_kernel<true><<<(unsigned)tiles, kGemmThreads, kGemmSmemBytes, stream>>>(
+      amap, bmap, (int)((tokens + kBK - 1) / kBK), (int)tiles_n, nullptr, H, n, n, ld_h);
   return cudaGetLastError();
 }
 

@@ -123,6 +123,29 @@ def test_residual_and_output_error_argument_errors(lib):
     assert f(None, 0, 64, 64, None, 128, 256, None, None, 0, None) == OK
 
 
+def test_gptq_argument_errors(lib):
+    ws = lib.hscale_hessian_full_workspace_bytes
+    assert ws(0, 64) == 0 and ws(100, 64) == 13312    # 64 rows of 104 bf16, rounded to 256 B
+    f = lib.hscale_hessian_full_accumulate
+    assert f(FAKE, 100, 64, 32, FAKE, 64, FAKE, 1 << 20, None) == ERR_SHAPE      # ld_x < n
+    assert f(FAKE, 100, 64, 64, None, 64, FAKE, 1 << 20, None) == ERR_NULL
+    assert f(FAKE, 100, 64, 64, FAKE, 64, FAKE, 16, None) == ERR_WS
+    assert f(None, 0, 64, 64, None, 64, None, 0, None) == OK
+    g = lib.hscale_gptq_factor
+    assert g(FAKE, 64, 32, 0.01, FAKE, None, FAKE, FAKE, 1 << 20, None) == ERR_SHAPE   # ld < n
+    assert g(FAKE, 64, 64, -1.0, FAKE, None, FAKE, FAKE, 1 << 20, None) == ERR_ARG
+    assert g(FAKE, 64, 64, 0.01, None, None, FAKE, FAKE, 1 << 20, None) == ERR_NULL
+    assert g(None, 0, 0, 0.01, None, None, None, None, 0, None) == OK
+    assert lib.hscale_gptq_workspace_bytes(4, 64, 32) == 1536
+    q = lib.hscale_gptq_hscale
+    assert q(FAKE, 4, 64, FAKE, FAKE, FAKE, None, 24, 4, 4, FAKE, FAKE, FAKE, 1 << 20, None) == ERR_SHAPE
+    assert q(FAKE, 4, 64, FAKE, FAKE, FAKE, None, 48, 4, 4, FAKE, FAKE, FAKE, 1 << 20, None) == ERR_SHAPE
+    assert q(FAKE, 4, 64, FAKE, FAKE, FAKE, None, 32, -1, 4, FAKE, FAKE, FAKE, 1 << 20, None) == ERR_ARG
+    assert q(FAKE, 4, 64, None, FAKE, FAKE, None, 32, 4, 4, FAKE, FAKE, FAKE, 1 << 20, None) == ERR_NULL
+    assert q(FAKE, 4, 64, FAKE, FAKE, FAKE, None, 32, 4, 4, FAKE, FAKE, FAKE, 64, None) == ERR_WS
+    assert q(None, 0, 64, None, None, None, None, 32, 4, 4, None, None, None, 0, None) == OK
+
+
 def test_pack_argument_errors(lib):
     f = lib.hscale_pack_nvfp4
     assert f(FAKE, 4, 32, FAKE, None, FAKE, None) == ERR_NULL
