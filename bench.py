@@ -64,6 +64,8 @@ def parse():
     p.add_argument("--no-cpu-baseline", action="store_true")
     p.add_argument("--no-output-error", action="store_true",
                    help="skip the tensor-core layer-output error evaluation")
+    p.add_argument("--no-gptq", action="store_true",
+                   help="skip the GPTQ + H-Scale (Algorithm 3) evaluation")
     p.add_argument("--no-e2e", action="store_true")
     return p.parse_args()
 
@@ -544,6 +546,66 @@ def output_error_eval(hs, work: Work, peaks: dict, tokens: int = 8192, reps: int
             "note": "tcgen05 bf16 GEMM of X with the [hi | lo] split of dW, fused sum of squares"}
 
 
+def gptq_eval(hs, work: Work, peaks: dict, block: int = 128, reps: int = 3):
+    """Algorithm 3 (GPTQ + H-Scale) on the first matrix of the workload, outside the timed
+    step: the full Hessian X^T X over every calibration chunk of its input space on the
+    tensor cores, the damped inverse-Cholesky factor, and the block loop with H-Scale as the
+    local quantizer (blocks of `block` columns, the step's window); each timed, and the
+    layer-output error ||X dW^T||^2 on the first chunk for GPTQ + H-Scale, H-Scale and RTN."""
+    M = work.mats[0]
+    S = M.space
+    dev = S.x.device
+    n, m = M.n, M.m
+    down, up = work.win
+    H = torch.zeros(n, n, dtype=torch.float32, device=dev)
+    hws = torch.empty(max(256, hs.hscale_hessian_full_workspace_bytes(S.chunk, n)), dtype=torch.uint8, device=dev)
+
+    def hessian():
+        H.zero_()
+        for c in range(S.nchunks):
+            hs.hscale_hessian_full_accumulate(S.x[c * S.chunk:(c + 1) * S.chunk], H, hws)
+
+    ms_h = timed(hessian, reps)
+    U = torch.empty(n, n, dtype=torch.float32, device=dev)
+    dead = torch.empty(n, dtype=torch.uint8, device=dev)
+    info = torch.zeros(3, dtype=torch.int32, device=dev)
+    fws = torch.empty(max(256, hs.hscale_gptq_factor_workspace_bytes(n)), dtype=torch.uint8, device=dev)
+    ms_f = timed(lambda: hs.hscale_gptq_factor(H, 0.01, U, dead, info, fws), reps)
+    if int(info.abs().sum().item()) != 0:
+        return {"unavailable": f"factorization failed, info {info.tolist()}"}
+    h = torch.diagonal(H).contiguous()
+    codes = torch.empty_like(M.codes)
+    packed = torch.empty_like(M.packed)
+    gws = torch.empty(hs.hscale_gptq_workspace_bytes(m, n, block), dtype=torch.uint8, device=dev)
+    ms_q = timed(lambda: hs.hscale_gptq_hscale(M.w, U, h, M.sg, dead, block, down, up, codes, packed, gws), reps)
+    # output error on the first chunk: GPTQ + H-Scale, H-Scale (the step's outputs), RTN
+    T = S.chunk
+    x = S.x[:T]
+    dw2 = torch.empty(m, hs.residual_ld(n), dtype=torch.bfloat16, device=dev)
+    out = torch.zeros(1, dtype=torch.float64, device=dev)
+    ows = torch.empty(hs.hscale_output_error_workspace_bytes(T, m), dtype=torch.uint8, device=dev)
+    rtn_codes = torch.empty_like(M.codes)
+    rtn_packed = torch.empty_like(M.packed)
+    hs.hscale_rtn_scales(M.w, M.sg, rtn_codes, work.ws)
+    hs.hscale_pack_nvfp4(M.w, M.sg, rtn_codes, rtn_packed)
+    err = {}
+    for name, c, p in (("gptq_hscale", codes, packed), ("hscale", M.codes, M.packed), ("rtn", rtn_codes, rtn_packed)):
+        hs.hscale_dequant_residual(M.w, M.sg, c, p, dw2)
+        out.zero_()
+        hs.hscale_output_error(x, dw2, m, out, ows)
+        err[name] = float(out.item())
+    h_flop = 2.0 * S.tokens * n * n
+    upd_flop = sum(2.0 * m * block * (n - c0 - block) for c0 in range(0, n, block))
+    return {"matrix": M.name, "block": block, "window": [down, up], "tokens": S.tokens,
+            "hessian_full_ms": ms_h, "hessian_full_tflops": h_flop / (ms_h * 1e-3) / 1e12,
+            "hessian_full_note": "dense-equivalent 2 T n^2 FLOP; tiles wholly below the diagonal are skipped",
+            "hessian_full_frac_of_measured_bf16": h_flop / (ms_h * 1e-3) / 1e12 / float(peaks.get("bf16_tflops", 1900.0)),
+            "factor_ms": ms_f, "block_loop_ms": ms_q, "update_gemm_gflop": upd_flop / 1e9,
+            "output_error_chunk_tokens": T, "output_error": err,
+            "reduction_vs_rtn": 1.0 - err["gptq_hscale"] / err["rtn"],
+            "reduction_vs_hscale": 1.0 - err["gptq_hscale"] / err["hscale"]}
+
+
 def shift_statistics(work: Work, win, sample_rows: int = 16):
     """Selected shifts delta = chosen code - initial code over every group of the step
     (from the GPU outputs), and the mean reduction of the Hessian-weighted error per
@@ -655,6 +717,12 @@ def gpu_arm(args, d: Dist):
     main = [s for s in sweep if tuple(s["window"]) == tuple(win)][0]
     shifts = shift_statistics(work, win)
     out_err = None if args.no_output_error else output_error_eval(hs, work, peaks)
+    gptq = None
+    if not args.no_gptq:
+        try:
+            gptq = gptq_eval(hs, work, peaks)
+        except Exception as e:  # e.g. no cuSOLVER on the machine: report, keep the bench line
+            gptq = {"unavailable": f"{type(e).__name__}: {e}"}
 
     # ---- roofline of the dominant kernel (the Hessian pass)
     h_bytes_launch = work.h_bytes / work.h_launches
@@ -707,6 +775,8 @@ def gpu_arm(args, d: Dist):
     line["shift_statistics"] = shifts
     if out_err:
         line["output_error"] = out_err
+    if gptq:
+        line["gptq_hscale"] = gptq
     if n_layers > 1:
         line["seconds_per_model"] = ms_step * 1e-3 * n_layers
         line["seconds_per_model_note"] = f"{n_layers} layers of identical shapes: per-layer step x {n_layers}"

@@ -267,11 +267,14 @@ int hscale_output_error(const void* x_bf16, int64_t tokens, int64_t n, int64_t l
  *
  * 1. hscale_hessian_full_accumulate: H[n, n] (fp32, row stride ld_h) += X^T X over a chunk
  *    of calibration tokens, on the tensor cores (bf16 products, fp32 accumulation); its
- *    diagonal is the h of Eq. 4.  x is [tokens, ld_x] bf16 row-major (2-byte aligned);
- *    the workspace (hscale_hessian_full_workspace_bytes, 256-byte aligned) holds X^T.
+ *    diagonal is the h of Eq. 4.  H is symmetric and only its upper triangle (j >= i) is
+ *    accumulated and read later: 128 x 256 tiles wholly below the diagonal are not
+ *    written, those crossing it are written in full.  x is [tokens, ld_x] bf16 row-major
+ *    (2-byte aligned); the workspace (hscale_hessian_full_workspace_bytes, 256-byte
+ *    aligned) holds X^T.
  *
  * 2. hscale_gptq_factor: the damped inverse-Cholesky factor, formed as GPTQ forms it.
- *    Channels with H_jj = 0 are dead (dead[j] = 1 if dead is not NULL; their weights are
+ *    Only the upper triangle of H (j >= i) is read.  Channels with H_jj = 0 are dead (dead[j] = 1 if dead is not NULL; their weights are
  *    zeroed in step 3) and get H_jj = 1; the diagonal gets damp * mean(diag H) (GPTQ uses
  *    damp = 0.01); U [n, n] (fp32, row stride n) is upper triangular with
  *    U^T U = (H + damp I)^-1.  Cholesky and the triangular inverse come from cuSOLVER,

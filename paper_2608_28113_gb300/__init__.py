@@ -313,7 +313,7 @@ def _workspace(nbytes: int, device) -> torch.Tensor:
 
 def hscale_hessian_full_accumulate(x: torch.Tensor, H: torch.Tensor, workspace: torch.Tensor | None = None,
                                    stream=None) -> None:
-    """H (fp32 [n, n]) += X^T X for x [tokens, n] bf16 (row stride ld_x) on the tensor cores."""
+    """Upper triangle of H (fp32 [n, n]) += X^T X for x [tokens, n] bf16 on the tensor cores."""
     _need(x, torch.bfloat16, "x")
     _need(H, torch.float32, "H")
     if x.dim() != 2 or x.stride(1) != 1 or H.dim() != 2 or H.stride(1) != 1:
@@ -364,3 +364,15 @@ def hscale_gptq_hscale(w: torch.Tensor, U: torch.Tensor, h: torch.Tensor, global
            load().hscale_gptq_hscale(_ptr(w), m, n, _ptr(U), _ptr(h), _ptr(global_scale), _ptr(dead), int(block),
                                      int(down), int(up), _ptr(codes_out), _ptr(packed_out), _ptr(workspace),
                                      workspace.numel(), _stream_ptr(stream)))
+
+
+def hscale_hessian_full_workspace_bytes(tokens: int, n: int) -> int:
+    return int(load().hscale_hessian_full_workspace_bytes(int(tokens), int(n)))
+
+
+def hscale_gptq_factor_workspace_bytes(n: int) -> int:
+    return int(load().hscale_gptq_factor_workspace_bytes(int(n)))
+
+
+def hscale_gptq_workspace_bytes(m: int, n: int, block: int) -> int:
+    return int(load().hscale_gptq_workspace_bytes(int(m), int(n), int(block)))

@@ -11,7 +11,8 @@
 //   transpose_kernel      X [tokens, n] -> X^T [n, tokens] (tokens contiguous per channel)
 //   gemm_kernel<true>     H += X^T X, the full Hessian of Algorithm 3, with the same tensor-
 //                         core pipeline over K = tokens and an epilogue that adds each
-//                         128 x 256 tile of the product into H
+//                         128 x 256 tile of the product into H; tiles wholly below the
+//                         diagonal are skipped (the factor reads the upper triangle only)
 //
 // The residual is rounded once (one FMA of the exact w - s_g * (l q)), and hi + lo carries
 // it to a relative 2^-17, so the GEMM sees dW, not a difference of two large products.
@@ -138,6 +139,9 @@ gemm_kernel(const __grid_constant__ CUtensorMap xmap, const __grid_constant__ CU
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int tile_m = blockIdx.x / tiles_n, tile_n = blockIdx.x - tile_m * tiles_n;
   const int kb_total = kAccum ? kb_half : 2 * kb_half;
+  // H is symmetric and only its upper triangle is used: a tile wholly below the diagonal
+  // (every column index below every row index) is skipped, uniformly for the whole CTA
+  if (kAccum && (int64_t)(tile_n + 1) * kBN <= (int64_t)tile_m * kBM) return;
 
   if (threadIdx.x == 0) {
     for (int s = 0; s < kStages; ++s) {

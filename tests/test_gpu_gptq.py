@@ -63,7 +63,7 @@ def test_full_hessian_matches_oracle(tokens, n, chunks):
     torch.cuda.synchronize()
     got = H.cpu().double().numpy()
     scale = np.sqrt(np.outer(np.diag(ref), np.diag(ref)))
-    err = np.abs(got - ref)
+    err = np.triu(np.abs(got - ref))        # the upper triangle is the accumulated part
     assert np.all(err <= 1e-5 * scale + 1e-30), f"max scaled err {np.max(err / (scale + 1e-300)):.2e}"
     assert hs.hscale_device_error_flags() == 0
 
@@ -175,11 +175,15 @@ def test_full_size_gptq_q_proj_slice():
     hs.hscale_hessian_full_accumulate(x.to(dev()), Hg)
     torch.cuda.synchronize()
     scale = np.sqrt(np.outer(np.diag(H), np.diag(H)))
-    assert np.all(np.abs(Hg.cpu().double().numpy() - H) <= 1e-5 * scale + 1e-30)
+    assert np.all(np.triu(np.abs(Hg.cpu().double().numpy() - H)) <= 1e-5 * scale + 1e-30)
+    # the factor of the GPU's own H (upper triangle only) equals the factor of the oracle's
+    Ug, _, info_g = gpu_factor(Hg.cpu().numpy())
+    assert np.all(info_g == 0)
     U, dead, info = gpu_factor(H32)
     assert np.all(info == 0)
     Uref, dref = oracle.gptq_factor(H32.astype(np.float64))
     assert np.linalg.norm(U - Uref) / np.linalg.norm(Uref) <= 1e-3
+    assert np.linalg.norm(Ug - Uref) / np.linalg.norm(Uref) <= 1e-3
     h32 = np.diag(H32).copy()
     U32 = Uref.astype(np.float32)
     codes, packed = gpu_gptq(w, U32, h32, s_g, 128, 4, 4, dead=dref)
