@@ -56,8 +56,9 @@ def parse():
                    help="asymmetric window 'D,U' (codes c0-D .. c0+U); e.g. 9,6 is the paper's K = 16 default")
     p.add_argument("--tokens", type=int, default=None,
                    help="calibration tokens per input space (default: the workload's; smaller for ncu captures)")
-    p.add_argument("--init", choices=["rtn", "4over6"], default="rtn",
-                   help="initial codes of the search: max-abs RTN (Eq. 7) or 4over6 (Algorithm 2)")
+    p.add_argument("--init", choices=["rtn", "4over6", "4over6-2pass"], default="rtn",
+                   help="initial codes of the search: max-abs RTN (Eq. 7), or 4over6 (Algorithm 2) "
+                        "decided inside the search (one pass) or by a separate codes pass")
     p.add_argument("--overlap-ctas", type=int, default=4,
                    help="resident search CTAs per SM while the next input space's Hessian pass "
                         "runs alongside (0: run every search after the last Hessian pass)")
@@ -269,12 +270,12 @@ def hessian_phase(hs, work: Work, xs=None, only=None):
 
 
 def init_codes(hs, work: Work, M, w=None):
-    """The weight-only part of one matrix: the global scale s_g, and with 4over6 init
-    Algorithm 2's codes.  With RTN init the search computes the RTN codes (Eq. 7) itself
-    (init_codes = NULL), which saves a pass over W."""
+    """The weight-only part of one matrix: the global scale s_g, and with the two-pass
+    4over6 init Algorithm 2's codes.  With RTN or one-pass 4over6 init the search decides
+    the initial codes itself, which saves a pass over W."""
     w = M.w if w is None else w
     hs.hscale_rtn_scales(w, M.sg, None, work.ws)
-    if work.init == "4over6":
+    if work.init == "4over6-2pass":
         hs.hscale_fourover6_codes(w, M.sg, M.codes0)
 
 
@@ -285,9 +286,12 @@ def init_phase(hs, work: Work, ws=None):
 
 def refine(hs, work: Work, M, down, up, w=None, ctas_per_sm=0):
     """The H-Scale search with packing of one matrix over the window (down, up)."""
-    init = M.codes0 if work.init == "4over6" else None
-    hs.hscale_refine_scales_ex(M.w if w is None else w, M.space.h, M.sg, init, down, up, M.codes,
-                               M.packed, ctas_per_sm)
+    w = M.w if w is None else w
+    if work.init == "4over6":
+        hs.hscale_refine_scales_4over6(w, M.space.h, M.sg, down, up, M.codes, M.packed, ctas_per_sm)
+    else:
+        init = M.codes0 if work.init == "4over6-2pass" else None
+        hs.hscale_refine_scales_ex(w, M.space.h, M.sg, init, down, up, M.codes, M.packed, ctas_per_sm)
 
 
 def refine_phase(hs, work: Work, win=None, ws=None):
@@ -384,13 +388,13 @@ class StepGraphs:
 
 
 # algorithmic bytes per group of the search: W 32, nibbles 8, code out 1, code in 1 (none
-# when the search computes the RTN codes itself)
-SEARCH_BYTES = {"rtn": 41, "4over6": 42}
+# when the search decides the initial codes itself)
+SEARCH_BYTES = {"rtn": 41, "4over6": 41, "4over6-2pass": 42}
 
 
 def kernels_per_matrix(work: Work) -> int:
     """Library kernels per matrix and step: amax, (4over6 codes,) refine."""
-    return 3 if work.init == "4over6" else 2
+    return 3 if work.init == "4over6-2pass" else 2
 
 
 def timed(fn, reps):
@@ -452,7 +456,7 @@ def cpu_baseline(W: wl.Workload, win, budget_s: float = 12.0, init: str = "rtn")
         wb = wl.bf16_bits(wl.weight(m, n, W.sigma_w, W.seed))
         t0 = time.perf_counter()
         s_g, _ = oracle.global_scale(wb)
-        c0 = oracle.fourover6_codes(wb, s_g)[0] if init == "4over6" else oracle.rtn_codes(wb, s_g)
+        c0 = oracle.fourover6_codes(wb, s_g)[0] if init.startswith("4over6") else oracle.rtn_codes(wb, s_g)
         t_rtn_total += time.perf_counter() - t0
         rows = max(8, min(m, 64))
         t0 = time.perf_counter()
@@ -707,12 +711,14 @@ def gpu_arm(args, d: Dist):
                       "groups_per_s": work.groups / (ms_ref * 1e-3),
                       "bound": "alu" if t_ops > t_bytes else "hbm", "roofline_ms": max(t_bytes, t_ops) * 1e3,
                       "frac": max(t_bytes, t_ops) / (ms_ref * 1e-3)})
-    # restore the outputs of the step's own window; materialize the RTN codes the search
-    # computed inline, for the shift statistics
+    # restore the outputs of the step's own window; materialize the initial codes the
+    # search decided inline, for the shift statistics
     scale_phase(hs, work)
-    if work.init == "rtn":
-        for M in work.mats:
+    for M in work.mats:
+        if work.init == "rtn":
             hs.hscale_rtn_scales(M.w, M.sg, M.codes0, work.ws)
+        elif work.init == "4over6":
+            hs.hscale_fourover6_codes(M.w, M.sg, M.codes0)
     torch.cuda.synchronize()
     main = [s for s in sweep if tuple(s["window"]) == tuple(win)][0]
     shifts = shift_statistics(work, win)

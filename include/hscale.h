@@ -15,16 +15,18 @@
  *                                       E2M1 under each candidate (Eqs. 11-12), keep the
  *                                       code with the smallest sum_j h_j (w_j - s q_j)^2
  *                                       (Eqs. 6, 13), then re-quantize and pack
+ *      hscale_refine_scales_ex          the same with a cap on resident CTAs per SM
  *      hscale_pack_nvfp4                final FP4 quantization with given codes
  *                                       (Sec. 3.3 "Final re-quantization", Eq. 2)
+ *      hscale_fourover6_codes           the 4over6 initial codes of Algorithm 2, an
+ *                                       alternative start for the refinement (Sec. 3.5)
+ *      hscale_refine_scales_4over6      Algorithm 2 in one pass: those codes decided
+ *                                       inside the search
  *      hscale_dequant_residual          dW = W - W_hat of the packed weights (Eqs. 1-3)
  *      hscale_output_error              ||X dW^T||_F^2 on the tensor cores (Eq. 3)
  *      hscale_hessian_full_accumulate   H += X^T X on the tensor cores (Algorithm 3)
  *      hscale_gptq_factor               damped inverse-Cholesky factor (Algorithm 3)
  *      hscale_gptq_hscale               GPTQ with H-Scale as local quantizer (Algorithm 3)
- *      hscale_refine_scales_ex          the same with a cap on resident CTAs per SM
- *      hscale_fourover6_codes           the 4over6 initial codes of Algorithm 2, an
- *                                       alternative start for the refinement (Sec. 3.5)
  *
  * Equation numbers count the paper's displayed equations in order (Eq. 1 is the
  * effective scale s = s_g * l).
@@ -214,6 +216,26 @@ int hscale_refine_scales_ex(const void* w_bf16, const float* h, int64_t m, int64
                             const float* global_scale, const uint8_t* init_codes, int32_t down,
                             int32_t up, uint8_t* codes_out, uint8_t* packed_out,
                             int32_t ctas_per_sm, void* stream);
+
+/*
+ * 4over6 + H-Scale, Algorithm 2 in one pass: the 4over6 initial codes are decided inside
+ * the search, group by group, and the window is searched around them.
+ *
+ * The results equal hscale_fourover6_codes followed by hscale_refine_scales_ex with those
+ * codes as init_codes, bit for bit, in one read of W and one launch, and with no
+ * intermediate codes array.  The anchors are ordered by fast plain-MSE scores (the
+ * hardware E2M1 conversion) whenever a margin test shows that the fast order is the exact
+ * one; the few other groups take the exact comparison of hscale_fourover6_codes.
+ *
+ * Arguments as for hscale_refine_scales_ex without init_codes: w [m, n] bfloat16
+ * (16-byte aligned, n % 16 == 0); h [n] fp32 (16-byte aligned) or NULL for h = 1;
+ * global_scale a device fp32 scalar; 0 <= down, up <= 125; codes_out [m, n/16] bytes,
+ * written; packed_out [m, n/2] bytes (8-byte aligned) or NULL; ctas_per_sm >= 0 (0 fills
+ * every SM).  The same status codes as hscale_refine_scales_ex.
+ */
+int hscale_refine_scales_4over6(const void* w_bf16, const float* h, int64_t m, int64_t n,
+                                const float* global_scale, int32_t down, int32_t up, uint8_t* codes_out,
+                                uint8_t* packed_out, int32_t ctas_per_sm, void* stream);
 
 /*
  * Final FP4 quantization with given codes (Sec. 3.3 "Final re-quantization", Eq. 2):

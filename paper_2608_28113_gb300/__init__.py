@@ -25,7 +25,7 @@ __all__ = [
     "hscale_device_error_flags",
     "hscale_hessian_diag_accumulate", "hscale_rtn_workspace_bytes", "hscale_rtn_scales",
     "hscale_rtn_scales_noalloc",
-    "hscale_refine_scales", "hscale_refine_scales_ex", "hscale_pack_nvfp4", "hscale_fourover6_codes",
+    "hscale_refine_scales", "hscale_refine_scales_ex", "hscale_refine_scales_4over6", "hscale_pack_nvfp4", "hscale_fourover6_codes",
     "hscale_dequant_residual", "hscale_output_error_workspace_bytes", "hscale_output_error",
     "residual_ld", "hscale_selftest_bounded_wait", "hscale_hessian_full_workspace_bytes",
     "hscale_hessian_full_accumulate", "hscale_gptq_factor_workspace_bytes", "hscale_gptq_factor",
@@ -50,6 +50,7 @@ _SIGNATURES = {
     "hscale_rtn_scales_noalloc": (ctypes.c_int, [_P, _I64, _I64, _P, _P, _P]),
     "hscale_refine_scales": (ctypes.c_int, [_P, _P, _I64, _I64, _P, _P, _I32, _I32, _P, _P, _P]),
     "hscale_refine_scales_ex": (ctypes.c_int, [_P, _P, _I64, _I64, _P, _P, _I32, _I32, _P, _P, _I32, _P]),
+    "hscale_refine_scales_4over6": (ctypes.c_int, [_P, _P, _I64, _I64, _P, _I32, _I32, _P, _P, _I32, _P]),
     "hscale_pack_nvfp4": (ctypes.c_int, [_P, _I64, _I64, _P, _P, _P, _P]),
     "hscale_fourover6_codes": (ctypes.c_int, [_P, _I64, _I64, _P, _P, _P]),
     "hscale_dequant_residual": (ctypes.c_int, [_P, _I64, _I64, _P, _P, _P, _P, _I64, _P]),
@@ -228,6 +229,32 @@ def hscale_refine_scales_ex(w: torch.Tensor, h: torch.Tensor | None, global_scal
            load().hscale_refine_scales_ex(_ptr(w), _ptr(h), m, n, _ptr(global_scale), _ptr(init_codes),
                                           int(down), int(up), _ptr(codes_out), _ptr(packed_out),
                                           int(ctas_per_sm), _stream_ptr(stream)))
+
+
+def hscale_refine_scales_4over6(w: torch.Tensor, h: torch.Tensor | None, global_scale: torch.Tensor,
+                                down: int, up: int, codes_out: torch.Tensor, packed_out: torch.Tensor | None,
+                                ctas_per_sm: int = 0, stream=None) -> None:
+    """Algorithm 2 in one pass: 4over6 initial codes decided in the search, then the search."""
+    _need(w, torch.bfloat16, "w")
+    _need(global_scale, torch.float32, "global_scale")
+    _need(codes_out, torch.uint8, "codes_out")
+    if not w.is_contiguous() or w.dim() != 2:
+        raise ValueError("w must be a contiguous 2-D tensor")
+    m, n = w.shape
+    if h is not None:
+        _need(h, torch.float32, "h")
+        if h.numel() != n or not h.is_contiguous():
+            raise ValueError("h must be a contiguous float32 vector of length n")
+    for name, t, size in (("codes_out", codes_out, m * (n // 16)),
+                          ("packed_out", packed_out, m * (n // 2))):
+        if t is not None:
+            _need(t, torch.uint8, name)
+            if t.numel() != size or not t.is_contiguous():
+                raise ValueError(f"{name} must be contiguous with {size} bytes")
+    _check("hscale_refine_scales_4over6",
+           load().hscale_refine_scales_4over6(_ptr(w), _ptr(h), m, n, _ptr(global_scale), int(down), int(up),
+                                              _ptr(codes_out), _ptr(packed_out), int(ctas_per_sm),
+                                              _stream_ptr(stream)))
 
 
 def hscale_pack_nvfp4(w: torch.Tensor, global_scale: torch.Tensor, codes: torch.Tensor,

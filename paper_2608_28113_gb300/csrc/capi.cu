@@ -139,7 +139,23 @@ int hscale_refine_scales_ex(const void* w_bf16, const float* h, int64_t m, int64
   if (h != nullptr && !aligned(h, 16)) return HSCALE_ERR_ALIGN;
   if (packed_out != nullptr && !aligned(packed_out, 8)) return HSCALE_ERR_ALIGN;
   return from_cuda(hscale::launch_refine(w_bf16, h, m, n, global_scale, init_codes, down, up,
-                                         codes_out, packed_out, ctas_per_sm, as_stream(stream)));
+                                         codes_out, packed_out, ctas_per_sm, false, as_stream(stream)));
+}
+
+int hscale_refine_scales_4over6(const void* w_bf16, const float* h, int64_t m, int64_t n,
+                                const float* global_scale, int32_t down, int32_t up, uint8_t* codes_out,
+                                uint8_t* packed_out, int32_t ctas_per_sm, void* stream) {
+  int st = check_weight(w_bf16, m, n);
+  if (st != HSCALE_OK) return st;
+  if (down < 0 || up < 0 || down > 125 || up > 125) return HSCALE_ERR_ARG;
+  if (ctas_per_sm < 0) return HSCALE_ERR_ARG;
+  if (m == 0 || n == 0) return HSCALE_OK;
+  if (global_scale == nullptr || codes_out == nullptr) return HSCALE_ERR_NULL;
+  if (!aligned(global_scale, 4)) return HSCALE_ERR_ALIGN;
+  if (h != nullptr && !aligned(h, 16)) return HSCALE_ERR_ALIGN;
+  if (packed_out != nullptr && !aligned(packed_out, 8)) return HSCALE_ERR_ALIGN;
+  return from_cuda(hscale::launch_refine(w_bf16, h, m, n, global_scale, nullptr, down, up, codes_out,
+                                         packed_out, ctas_per_sm, true, as_stream(stream)));
 }
 
 int hscale_fourover6_codes(const void* w_bf16, int64_t m, int64_t n, const float* global_scale,

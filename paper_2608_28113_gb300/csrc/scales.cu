@@ -4,7 +4,9 @@
 //   rtn_codes_kernel    s_g = amax / 2688 and the RTN code of every group (Eq. 7)
 //   refine_kernel       Algorithm 1: per group, every distinct E4M3 code in the window
 //                       (Eqs. 8-11) is scored by sum_j h_j (|w_j| - s q_j)^2 (Eqs. 6, 12,
-//                       13); the best code is re-quantized exactly and packed
+//                       13); the best code is re-quantized exactly and packed.  Its
+//                       4over6 instance decides Algorithm 2's initial code in place
+//   fourover6_codes_kernel  Algorithm 2's initial codes as a separate pass
 //   pack_kernel         exact FP4 quantization with given codes (Eq. 2)
 //
 // The search (one group per thread, no shuffles in the hot loop)
@@ -282,11 +284,93 @@ __device__ __forceinline__ uint2 quantize_pack(const Group& G, uint32_t c, float
   return make_uint2(word[0], word[1]);
 }
 
+// ---------------------------------------------------------------- 4over6 scores (Algorithm 2)
+// Plain-MSE error of one group under code c with exact rounding decisions: one rounding
+// in each residual (q * l is exact inside the FMA), the square, and a fixed pairwise
+// 16-term sum; relative error <= 7 * 2^-24.
+__device__ __forceinline__ float exact_group_mse(const Group& G, uint32_t c, float sgk) {
+  const float l = e4m3_mag(c);
+  const float inv = inv_raw_of(__fmul_rn(l, sgk));
+  float t[16];
+#pragma unroll
+  for (int j = 0; j < 16; ++j) {
+    const float a = (j & 1) ? G.a[j >> 1].y : G.a[j >> 1].x;
+    const uint32_t k = e2m1_code(a, inv, l, sgk);
+    const float r = __fmaf_rn(-__fmul_rn(e2m1_from_raw(k << 22), l), sgk, a);
+    t[j] = __fmul_rn(r, r);
+  }
+#pragma unroll
+  for (int step = 1; step < 16; step <<= 1)
+#pragma unroll
+    for (int j = 0; j + step < 16; j += 2 * step) t[j] = __fadd_rn(t[j], t[j + step]);
+  return t[0];
+}
+
+// Fast plain-MSE score of one candidate (fast_score with every h_j = 1).
+__device__ __forceinline__ float fast_mse(const Group& G, float4 t) {
+  const float2 inv2 = make_float2(t.z, t.w);
+  float2 acc0 = make_float2(0.f, 0.f), acc1 = make_float2(0.f, 0.f);
+#pragma unroll
+  for (int i = 0; i < 8; ++i) {
+    const float2 d = e2m1_residual2(__fmul2_rn(G.a[i], inv2));
+    if (i & 1) acc1 = __ffma2_rn(d, d, acc1);
+    else acc0 = __ffma2_rn(d, d, acc0);
+  }
+  const float2 t2 = __fadd2_rn(acc0, acc1);
+  return __fmul_rn(t.x, __fadd_rn(t2.x, t2.y));
+}
+
+// Is the fast winner (fast score e1) certainly ahead of the runner-up (e2), given the
+// energy A = sum_j h_j a_j^2 of the group?  The test of the file comment, in units of e2
+// (no underflow or overflow for 2^-36 A <= e2 <= A-ish):
+//   g = (e2 - e1) / e2 - 2^-18 - 2^-35 A / e2 > 2^-17 sqrt(A / e2), tested on squares.
+// A zero, denormal or non-finite e2 makes the reciprocal infinite or NaN and g fails.
+__device__ __forceinline__ bool fast_winner_certain(float e1, float e2, float A) {
+  const float r = rcp_approx(e2);
+  const float ratio = __fmul_rn(A, r);
+  const float g = __fsub_rn(__fsub_rn(__fmul_rn(__fsub_rn(e2, e1), r), 0x1p-18f), __fmul_rn(0x1p-35f, ratio));
+  const bool certain = g > 0.0f && __fmul_rn(g, g) > __fmul_rn(0x1p-34f, ratio);
+  return certain && ratio <= 0x1p36f && A > 0.0f;
+}
+
+// The anchor choice of Algorithm 2 for one group with exact rounding decisions (the
+// group is read back from global memory); the anchor 4 code c4 wins an exact tie.  Kept
+// out of line: the search calls it only when the fast scores cannot order the anchors.
+__device__ __noinline__ uint32_t fourover6_exact_pick(const uint4* w, int64_t g, float pw, uint32_t c4,
+                                                      uint32_t c6, float sgk) {
+  Group G;
+  load_group(w, g, pw, G);
+  return exact_group_mse(G, c6, sgk) < exact_group_mse(G, c4, sgk) ? c6 : c4;
+}
+
+// Algorithm 2's initial code of one group, decided in the search kernel: the two
+// anchored codes, their fast plain-MSE scores from the candidate table and, only when
+// the margin test cannot order them, the exact comparison.  When the test passes, the
+// fast order is the order of the exact errors, and the exact fp32 sums (relative error
+// <= 7 * 2^-24, far inside the margin) order them the same way; so the result is always
+// the code fourover6_codes_kernel writes.
+__device__ __forceinline__ int fourover6_init_code(const Group& G, const uint4* w, int64_t g, const float4* tab,
+                                                   float amax_k, float sgk, float pw, float inv4, float inv6) {
+  const uint32_t c4 = anchored_code(amax_k, sgk, inv4, 2.0f);
+  const uint32_t c6 = anchored_code(amax_k, sgk, inv6, 3.0f);
+  if (c4 == c6) return (int)c4;
+  const float e4 = fast_mse(G, tab[c4]);
+  const float e6 = fast_mse(G, tab[c6]);
+  float2 acc = make_float2(0.f, 0.f);
+#pragma unroll
+  for (int i = 0; i < 8; ++i) acc = __ffma2_rn(G.a[i], G.a[i], acc);
+  const float A = __fadd_rn(acc.x, acc.y);
+  if (fast_winner_certain(fminf(e4, e6), fmaxf(e4, e6), A)) return (int)(e6 < e4 ? c6 : c4);
+  return (int)fourover6_exact_pick(w, g, pw, c4, c6, sgk);
+}
+
 // ---------------------------------------------------------------- refine (Algorithm 1)
 // Work unit: one warp, 32 consecutive groups of one row (a "row chunk"); warps stride
 // over (row, chunk) units so the h slice of a lane is reloaded only when its chunk
 // changes.  7 resident CTAs of 4 warps per SM (72 registers); the rarely taken
 // warp-cooperative rescoring is a separate call so it does not raise that.
+// kFourOverSix: the initial codes are Algorithm 2's, decided in place (init_codes unused).
+template <bool kFourOverSix>
 __global__ void __launch_bounds__(kRefineThreads, 7)
 refine_kernel(const uint4* __restrict__ w, const float* __restrict__ h, int64_t m, int ng,
               const float* __restrict__ global_scale, const uint8_t* init_codes,
@@ -300,6 +384,7 @@ refine_kernel(const uint4* __restrict__ w, const float* __restrict__ h, int64_t 
   __shared__ float4 tab[128];
   const ScaleDomain d = make_scale_domain(*global_scale);
   const float inv6 = rtn_inv6_raw(d.sgk);
+  const float inv4 = kFourOverSix ? anchor_inv_raw(d.sgk, 4.0f) : 0.0f;
   for (int c = threadIdx.x; c < 128; c += blockDim.x) tab[c] = candidate_constants((uint32_t)c, d.sgk);
   __syncthreads();
 
@@ -339,13 +424,15 @@ refine_kernel(const uint4* __restrict__ w, const float* __restrict__ h, int64_t 
     int c0 = 1, lo = 1, hi = 1;
     if (active) {
       load_group(w, g, d.pw, G);
-      if (init_codes != nullptr) {
+      if (!kFourOverSix && init_codes != nullptr) {
         c0 = init_codes[g] & 0x7F;
         c0 = c0 < 1 ? 1 : (c0 > (int)kE4M3MaxCode ? (int)kE4M3MaxCode : c0);
       } else {
         const uint32_t amax = group_abs_max_bits(make_uint4(G.wb[0], G.wb[1], G.wb[2], G.wb[3]),
                                                  make_uint4(G.wb[4], G.wb[5], G.wb[6], G.wb[7]));
-        c0 = (int)rtn_code(__fmul_rn(__uint_as_float(amax << 16), d.pw), d.sgk, inv6);
+        const float amax_k = __fmul_rn(__uint_as_float(amax << 16), d.pw);
+        c0 = kFourOverSix ? fourover6_init_code(G, w, g, tab, amax_k, d.sgk, d.pw, inv4, inv6)
+                          : (int)rtn_code(amax_k, d.sgk, inv6);
       }
       lo = max(1, c0 - down);
       hi = min((int)kE4M3MaxCode, c0 + up);
@@ -359,17 +446,7 @@ refine_kernel(const uint4* __restrict__ w, const float* __restrict__ h, int64_t 
 
     // ---- is the fast winner certain?
     bool ambiguous = false;
-    if (active && hi > lo) {
-      // In units of E2 (no underflow or overflow for 2^-36 A <= E2 <= A-ish):
-      //   g = (E2 - E1) / E2 - 2^-18 - 2^-35 A / E2 > 2^-17 sqrt(A / E2), tested on squares.
-      // A zero, denormal or non-finite E2 makes the reciprocal infinite or NaN and g fails.
-      const float A = group_energy(G, hv2);
-      const float r = rcp_approx(e2);
-      const float ratio = __fmul_rn(A, r);
-      const float g = __fsub_rn(__fsub_rn(__fmul_rn(__fsub_rn(e2, e1), r), 0x1p-18f), __fmul_rn(0x1p-35f, ratio));
-      const bool certain = g > 0.0f && __fmul_rn(g, g) > __fmul_rn(0x1p-34f, ratio);
-      ambiguous = !certain || !(ratio <= 0x1p36f) || !(A > 0.0f);
-    }
+    if (active && hi > lo) ambiguous = !fast_winner_certain(e1, e2, group_energy(G, hv2));
     unsigned amb = __ballot_sync(0xFFFFFFFFu, ambiguous);
     while (amb) {
       const int owner = __ffs(amb) - 1;
@@ -412,27 +489,6 @@ __global__ void __launch_bounds__(256) pack_kernel(const uint4* __restrict__ w, 
 // Resident CTAs per SM of a kernel, queried once per kernel and device (the query is
 // not repeated under stream capture).
 // ---------------------------------------------------------------- 4over6 init (Algorithm 2)
-// Plain-MSE error of one group under code c with exact rounding decisions: one rounding
-// in each residual (q * l is exact inside the FMA), the square, and a fixed pairwise
-// 16-term sum; relative error <= 7 * 2^-24.
-__device__ __forceinline__ float exact_group_mse(const Group& G, uint32_t c, float sgk) {
-  const float l = e4m3_mag(c);
-  const float inv = inv_raw_of(__fmul_rn(l, sgk));
-  float t[16];
-#pragma unroll
-  for (int j = 0; j < 16; ++j) {
-    const float a = (j & 1) ? G.a[j >> 1].y : G.a[j >> 1].x;
-    const uint32_t k = e2m1_code(a, inv, l, sgk);
-    const float r = __fmaf_rn(-__fmul_rn(e2m1_from_raw(k << 22), l), sgk, a);
-    t[j] = __fmul_rn(r, r);
-  }
-#pragma unroll
-  for (int step = 1; step < 16; step <<= 1)
-#pragma unroll
-    for (int j = 0; j + step < 16; j += 2 * step) t[j] = __fadd_rn(t[j], t[j + step]);
-  return t[0];
-}
-
 // Initial codes of Algorithm 2: for m = max|w| of the group, the E4M3 codes of m / (4 s_g)
 // and m / (6 s_g) (each as in Eq. 7), and the one whose group has the smaller plain MSE;
 // the anchor 4 (first in C = {4, 6}) wins an exact tie.
@@ -457,14 +513,14 @@ __global__ void __launch_bounds__(256) fourover6_codes_kernel(const uint4* __res
   }
 }
 
-template <typename K>
-int occupancy_blocks(K kernel, int threads) {
+template <auto kKernel>
+int occupancy_blocks(int threads) {
   static int cache[64] = {0};
   int dev = 0;
   if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) dev = 0;
   if (cache[dev] == 0) {
     int blocks = 0;
-    if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&blocks, kernel, threads, 0) != cudaSuccess ||
+    if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&blocks, kKernel, threads, 0) != cudaSuccess ||
         blocks < 1)
       blocks = 1;
     cache[dev] = blocks;
@@ -480,7 +536,7 @@ cudaError_t launch_amax(const void* w, int64_t count, uint32_t* amax_bits, cudaS
   if (err != cudaSuccess) return err;
   const int64_t nvec = count / 8;
   int64_t blocks = (nvec + 255) / 256;
-  blocks = std::min<int64_t>(blocks, (int64_t)info.sm_count * occupancy_blocks(amax_kernel, 256));
+  blocks = std::min<int64_t>(blocks, (int64_t)info.sm_count * occupancy_blocks<amax_kernel>(256));
   amax_kernel<<<(unsigned)blocks, 256, 0, stream>>>(static_cast<const uint4*>(w), nvec, amax_bits);
   return cudaGetLastError();
 }
@@ -492,7 +548,7 @@ cudaError_t launch_rtn_codes(const void* w, int64_t m, int64_t n, const uint32_t
   if (err != cudaSuccess) return err;
   const int64_t groups = m * (n / 16);
   int64_t blocks = codes ? (groups + 255) / 256 : 1;
-  blocks = std::max<int64_t>(1, std::min<int64_t>(blocks, (int64_t)info.sm_count * occupancy_blocks(rtn_codes_kernel, 256)));
+  blocks = std::max<int64_t>(1, std::min<int64_t>(blocks, (int64_t)info.sm_count * occupancy_blocks<rtn_codes_kernel>(256)));
   rtn_codes_kernel<<<(unsigned)blocks, 256, 0, stream>>>(static_cast<const uint4*>(w), groups,
                                                           amax_bits, global_scale, codes);
   return cudaGetLastError();
@@ -500,19 +556,22 @@ cudaError_t launch_rtn_codes(const void* w, int64_t m, int64_t n, const uint32_t
 
 cudaError_t launch_refine(const void* w, const float* h, int64_t m, int64_t n,
                           const float* global_scale, const uint8_t* init_codes, int down, int up,
-                          uint8_t* codes_out, uint8_t* packed_out, int ctas_per_sm, cudaStream_t stream) {
+                          uint8_t* codes_out, uint8_t* packed_out, int ctas_per_sm, bool fourover6,
+                          cudaStream_t stream) {
   DeviceInfo info;
   cudaError_t err = current_device_info(&info);
   if (err != cudaSuccess) return err;
   const int ng = (int)(n / 16);
   const int64_t units = m * ((ng + 31) / 32);
-  int per_sm = occupancy_blocks(refine_kernel, kRefineThreads);
+  int per_sm = fourover6 ? occupancy_blocks<refine_kernel<true>>(kRefineThreads)
+                         : occupancy_blocks<refine_kernel<false>>(kRefineThreads);
   if (ctas_per_sm > 0) per_sm = std::min(per_sm, ctas_per_sm);
   const int64_t resident = (int64_t)info.sm_count * per_sm;
   const int64_t blocks = std::max<int64_t>(1, std::min<int64_t>((units + kWarpsPerRefineBlock - 1) / kWarpsPerRefineBlock, resident));
-  refine_kernel<<<(unsigned)blocks, kRefineThreads, 0, stream>>>(
-      static_cast<const uint4*>(w), h, m, ng, global_scale, init_codes, down, up, codes_out,
-      reinterpret_cast<uint2*>(packed_out));
+  auto kernel = fourover6 ? refine_kernel<true> : refine_kernel<false>;
+  kernel<<<(unsigned)blocks, kRefineThreads, 0, stream>>>(static_cast<const uint4*>(w), h, m, ng, global_scale,
+                                                          fourover6 ? nullptr : init_codes, down, up, codes_out,
+                                                          reinterpret_cast<uint2*>(packed_out));
   return cudaGetLastError();
 }
 
@@ -523,7 +582,7 @@ cudaError_t launch_fourover6(const void* w, int64_t m, int64_t n, const float* g
   if (err != cudaSuccess) return err;
   const int64_t groups = m * (n / 16);
   int64_t blocks = (groups + 255) / 256;
-  blocks = std::max<int64_t>(1, std::min<int64_t>(blocks, (int64_t)info.sm_count * occupancy_blocks(fourover6_codes_kernel, 256)));
+  blocks = std::max<int64_t>(1, std::min<int64_t>(blocks, (int64_t)info.sm_count * occupancy_blocks<fourover6_codes_kernel>(256)));
   fourover6_codes_kernel<<<(unsigned)blocks, 256, 0, stream>>>(static_cast<const uint4*>(w), groups,
                                                                 global_scale, codes);
   return cudaGetLastError();
@@ -536,7 +595,7 @@ cudaError_t launch_pack(const void* w, int64_t m, int64_t n, const float* global
   if (err != cudaSuccess) return err;
   const int64_t groups = m * (n / 16);
   int64_t blocks = (groups + 255) / 256;
-  blocks = std::max<int64_t>(1, std::min<int64_t>(blocks, (int64_t)info.sm_count * occupancy_blocks(pack_kernel, 256)));
+  blocks = std::max<int64_t>(1, std::min<int64_t>(blocks, (int64_t)info.sm_count * occupancy_blocks<pack_kernel>(256)));
   pack_kernel<<<(unsigned)blocks, 256, 0, stream>>>(static_cast<const uint4*>(w), groups,
                                                      global_scale, codes,
                                                      reinterpret_cast<uint2*>(packed_out));

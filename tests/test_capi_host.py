@@ -103,6 +103,21 @@ def test_refine_ex_argument_errors(lib):
     assert f(None, None, 0, 32, None, None, 4, 4, None, None, 5, None) == OK
 
 
+def test_refine_4over6_argument_errors(lib):
+    f = lib.hscale_refine_scales_4over6
+    assert f(FAKE, FAKE, 4, 32, FAKE, 4, 4, FAKE, FAKE, -1, None) == ERR_ARG
+    assert f(FAKE, FAKE, 4, 32, FAKE, -1, 4, FAKE, FAKE, 0, None) == ERR_ARG
+    assert f(FAKE, FAKE, 4, 32, FAKE, 4, 126, FAKE, FAKE, 0, None) == ERR_ARG
+    assert f(FAKE, FAKE, 4, 40, FAKE, 4, 4, FAKE, FAKE, 0, None) == ERR_SHAPE
+    assert f(None, FAKE, 4, 32, FAKE, 4, 4, FAKE, FAKE, 0, None) == ERR_NULL
+    assert f(FAKE, FAKE, 4, 32, None, 4, 4, FAKE, FAKE, 0, None) == ERR_NULL
+    assert f(FAKE, FAKE, 4, 32, FAKE, 4, 4, None, FAKE, 0, None) == ERR_NULL
+    assert f(FAKE, MIS, 4, 32, FAKE, 4, 4, FAKE, FAKE, 0, None) == ERR_ALIGN      # h 16-B
+    assert f(FAKE, FAKE, 4, 32, FAKE, 4, 4, FAKE, ctypes.c_void_p(0x10004), 0, None) == ERR_ALIGN
+    assert f(MIS, FAKE, 4, 32, FAKE, 4, 4, FAKE, FAKE, 0, None) == ERR_ALIGN
+    assert f(None, None, 0, 32, None, 4, 4, None, None, 0, None) == OK
+
+
 def test_residual_and_output_error_argument_errors(lib):
     r = lib.hscale_dequant_residual
     assert r(FAKE, 4, 24, FAKE, FAKE, FAKE, FAKE, 128, None) == ERR_SHAPE       # n % 16

@@ -449,6 +449,9 @@ def test_fourover6_exact_ties_and_edge_groups():
     expect = np.array([np.flatnonzero(lad == 1.5 * v)[0] + 1 for v in l6s])
     assert np.array_equal(col, expect), "an exact zero-error tie must keep anchor 4"
     assert codes[0, 0] == 126 and codes[1, 2] == 1 and codes[4, 2] == 1 and codes[2, 3] == 1
+    # the fused pass decides the same anchors (window 0: its codes are the initial codes)
+    fused, _ = gpu_refine_4over6(wd, None, sg, 0, 0)
+    assert np.array_equal(fused, codes)
 
 
 @pytest.mark.parametrize("down,up", [(4, 4), (9, 6), (0, 0)])
@@ -469,6 +472,57 @@ def test_fourover6_then_refine_matches_oracle(down, up):
     compare_search(ref, codes, packed, f"4over6 init, window -{down}/+{up}")
     if (down, up) == (0, 0):
         assert np.array_equal(codes[~diff], init_ref[~diff])
+
+
+def gpu_refine_4over6(w, h32, sg, down, up, ctas_per_sm=0):
+    m, n = w.shape
+    codes = torch.empty(m, n // 16, dtype=torch.uint8, device=dev())
+    packed = torch.empty(m, n // 2, dtype=torch.uint8, device=dev())
+    h = None if h32 is None else torch.from_numpy(np.ascontiguousarray(h32, np.float32)).to(dev())
+    hs.hscale_refine_scales_4over6(w, h, sg, down, up, codes, packed, ctas_per_sm)
+    torch.cuda.synchronize()
+    return codes.cpu().numpy(), packed.cpu().numpy()
+
+
+@pytest.mark.parametrize("down,up,weighted,ctas", [(4, 4, True, 0), (9, 6, True, 4), (0, 0, True, 0),
+                                                   (16, 16, True, 0), (4, 4, False, 0)])
+def test_fused_fourover6_refine_matches_oracle(down, up, weighted, ctas):
+    """Algorithm 2 in one pass: the 4over6 codes decided inside the search.  Against the
+    oracle (its 4over6 codes, then its search), outside anchor and search near-ties; and
+    bit for bit against the two-pass chain of the same library."""
+    w = small_layer(4, 512, 1024)
+    h32 = oracle_h32(4, 1024) if weighted else None
+    wd = w.to(dev())
+    sg, _ = gpu_rtn(wd)
+    s_ref, _ = oracle.global_scale(bits(w))
+    init_ref, nt = oracle.fourover6_codes(bits(w), s_ref)
+    codes, packed = gpu_refine_4over6(wd, h32, sg, down, up, ctas)
+    ref = oracle.refine(bits(w), h32, s_ref, init_ref, down, up)
+    ref["near_tie"] = ref["near_tie"] | nt
+    compare_search(ref, codes, packed, f"fused 4over6, window -{down}/+{up}, h={'x' if weighted else '1'}")
+    if (down, up) == (0, 0):
+        keep = ~nt.astype(bool)
+        assert np.array_equal(codes[keep], init_ref[keep])
+    init = torch.empty(512, 64, dtype=torch.uint8, device=dev())
+    hs.hscale_fourover6_codes(wd, sg, init)
+    codes2, packed2 = gpu_refine(wd, h32, sg, init, down, up)
+    assert np.array_equal(codes, codes2) and np.array_equal(packed, packed2)
+
+
+@pytest.mark.parametrize("seed,m,n", [(5, 1, 16), (6, 3, 48), (7, 33, 16 * 33), (8, 2, 16 * 200)])
+def test_fused_fourover6_ragged_shapes(seed, m, n):
+    """One row, ragged row chunks (groups per row not a multiple of the 32 lanes)."""
+    w = wl.weight(m, n, 0.02, seed)
+    h32 = oracle_h32(seed, n, tokens=256)
+    wd = w.to(dev())
+    sg, _ = gpu_rtn(wd)
+    s_ref, _ = oracle.global_scale(bits(w))
+    init_ref, nt = oracle.fourover6_codes(bits(w), s_ref)
+    for down, up in ((4, 4), (0, 0)):
+        codes, packed = gpu_refine_4over6(wd, h32, sg, down, up)
+        ref = oracle.refine(bits(w), h32, s_ref, init_ref, down, up)
+        ref["near_tie"] = ref["near_tie"] | nt
+        compare_search(ref, codes, packed, f"fused 4over6 {m}x{n} window -{down}/+{up}")
 
 
 # ------------------------------------------------------------------ output error (Eq. 3)
@@ -642,6 +696,10 @@ def full_size_check(name, sample_rows, layer_index=0, windows=None, fourover6=Fa
             ref["near_tie"] = ref["near_tie"] | exclude
             compare_search(ref, codes_g[rows], packed_g[rows],
                            f"{name} {L.name} {m}x{n} window -{down}/+{up} ({rows.size} sampled rows)")
+            if fourover6:
+                # the one-pass form, at the launch shape the bench times it with (4 CTAs/SM)
+                codes_f, packed_f = gpu_refine_4over6(w, h_ref[L.input_space], sg, down, up, 4)
+                assert np.array_equal(codes_f, codes_g) and np.array_equal(packed_f, packed_g)
         del w
 
 
