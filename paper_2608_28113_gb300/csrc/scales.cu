@@ -11,7 +11,7 @@
 //
 // The search (one group per thread, no shuffles in the hot loop)
 //   A candidate scale s' = l sgk is scored as E = s'^2 sum_j h_j (q_j - y_j)^2 with
-//   y_j = |a_j| / s' (one packed multiply by a tabulated reciprocal) and q_j = RNE_sat(y_j)
+//   y_j = a_j / s' (one packed multiply by a tabulated reciprocal) and q_j = RNE_sat(y_j)
 //   from the hardware E2M1 conversion (saturation included) converted back to f16; the
 //   residual q - y is one mixed f16/f32 subtract.  That is five lane operations per
 //   element and candidate.  With y within a relative 2^-21 of the exact quotient, every
@@ -102,9 +102,12 @@ __global__ void __launch_bounds__(256) rtn_codes_kernel(const uint4* __restrict_
 }
 
 // ---------------------------------------------------------------- search helpers
+// a_j keeps the sign of w_j.  Every score is even in a_j (round-to-nearest-even and
+// saturation are symmetric, and only squares of residuals enter), so the search pays
+// nothing for the sign, and the pack converts the signed quotients directly.
 struct Group {
   uint32_t wb[8];  // raw bf16 pairs (element 2i in the low half of wb[i])
-  float2 a[8];     // |w| * 2^-K, elements (2i, 2i+1)
+  float2 a[8];     // w * 2^-K, elements (2i, 2i+1)
 };
 
 __device__ __forceinline__ void load_group(const uint4* w, int64_t g, float pw, Group& G) {
@@ -114,7 +117,7 @@ __device__ __forceinline__ void load_group(const uint4* w, int64_t g, float pw, 
   G.wb[4] = q.x; G.wb[5] = q.y; G.wb[6] = q.z; G.wb[7] = q.w;
 #pragma unroll
   for (int i = 0; i < 8; ++i)
-    G.a[i] = make_float2(__fmul_rn(fabsf(bf16_lo(G.wb[i])), pw), __fmul_rn(fabsf(bf16_hi(G.wb[i])), pw));
+    G.a[i] = __fmul2_rn(make_float2(bf16_lo(G.wb[i]), bf16_hi(G.wb[i])), make_float2(pw, pw));
 }
 
 // Per-block table of the candidate constants of every E4M3 code c (1..126), filled once
@@ -247,29 +250,33 @@ __device__ __forceinline__ uint32_t cvt_e2m1x2(float hi, float lo) {
 }
 
 // Exact final re-quantization of one group under code c (inv_raw = 2^-126 / s'): 8 bytes of
-// packed nibbles.  The raw-domain quotients y_raw = |w| * 2^-126 / s' are rescaled
-// exactly to real units, given the sign of w, and converted by the hardware E2M1
-// conversion (round-to-nearest-even).  That equals the exact rounding of |w| / s unless
-// y_raw lies within 16 ulps of a midpoint; such elements are flagged and redone one by
-// one with the exact midpoint test, reading the weight back from `wg` (the group's 16
-// bf16 values in global memory).
+// packed nibbles.  The raw-domain quotients y_raw = w * 2^-126 / s' (signed) are rescaled
+// exactly to real units and converted by the hardware E2M1 conversion (round-to-nearest-
+// even, sign kept).  That equals the exact rounding of |w| / s unless y_raw lies within 16
+// ulps of a midpoint.  The main pass only notes whether any element does; then such
+// elements are found and redone one by one with the exact midpoint test, reading the
+// weight back from `wg` (the group's 16 bf16 values in global memory).
 __device__ __forceinline__ uint2 quantize_pack(const Group& G, uint32_t c, float inv_raw, float sgk,
                                                float pw, const uint16_t* wg) {
   const float2 ir2 = make_float2(inv_raw, inv_raw);
   const float2 up2 = make_float2(0x1p126f, 0x1p126f);
   uint32_t word[2] = {0u, 0u};
-  uint32_t flagged = 0u;
+  bool any = false;
 #pragma unroll
   for (int i = 0; i < 8; ++i) {
     const float2 yr = __fmul2_rn(G.a[i], ir2);
-    flagged |= (uint32_t)(((__float_as_uint(yr.x) - 0x1FFFF0u) & 0x3FFFFFu) <= 0x20u) << (2 * i);
-    flagged |= (uint32_t)(((__float_as_uint(yr.y) - 0x1FFFF0u) & 0x3FFFFFu) <= 0x20u) << (2 * i + 1);
+    any |= e2m1_uncertain(yr.x) | e2m1_uncertain(yr.y);
     const float2 yv = __fmul2_rn(yr, up2);
-    const float y0 = __uint_as_float(__float_as_uint(yv.x) | ((G.wb[i] << 16) & 0x80000000u));
-    const float y1 = __uint_as_float(__float_as_uint(yv.y) | (G.wb[i] & 0x80000000u));
-    word[i >> 2] |= cvt_e2m1x2(y1, y0) << (8 * (i & 3));
+    word[i >> 2] |= cvt_e2m1x2(yv.y, yv.x) << (8 * (i & 3));
   }
-  if (flagged) {
+  if (any) {
+    uint32_t flagged = 0u;
+#pragma unroll
+    for (int i = 0; i < 8; ++i) {
+      const float2 yr = __fmul2_rn(G.a[i], ir2);
+      flagged |= (uint32_t)e2m1_uncertain(yr.x) << (2 * i);
+      flagged |= (uint32_t)e2m1_uncertain(yr.y) << (2 * i + 1);
+    }
     const float l = e4m3_mag(c);
     do {
       const int j = __ffs(flagged) - 1;
@@ -294,7 +301,7 @@ __device__ __forceinline__ float exact_group_mse(const Group& G, uint32_t c, flo
   float t[16];
 #pragma unroll
   for (int j = 0; j < 16; ++j) {
-    const float a = (j & 1) ? G.a[j >> 1].y : G.a[j >> 1].x;
+    const float a = fabsf((j & 1) ? G.a[j >> 1].y : G.a[j >> 1].x);
     const uint32_t k = e2m1_code(a, inv, l, sgk);
     const float r = __fmaf_rn(-__fmul_rn(e2m1_from_raw(k << 22), l), sgk, a);
     t[j] = __fmul_rn(r, r);
