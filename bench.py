@@ -59,6 +59,12 @@ def parse():
     p.add_argument("--init", choices=["rtn", "4over6", "4over6-2pass"], default="rtn",
                    help="initial codes of the search: max-abs RTN (Eq. 7), or 4over6 (Algorithm 2) "
                         "decided inside the search (one pass) or by a separate codes pass")
+    p.add_argument("--col-block", type=int, default=0,
+                   help="channels per column block of the step: each block's Hessian pass over every "
+                        "token, then that block's searches alongside the next block's Hessian pass "
+                        "(a multiple of 64).  0 (default): whole input spaces, Hessian pass in token "
+                        "chunks; on q_proj blocks of 512-2048 channels make the Hessian pass 5-38 %% "
+                        "slower (each launch reads a fraction of every row) and the step slower")
     p.add_argument("--overlap-ctas", type=int, default=4,
                    help="resident search CTAs per SM while the next input space's Hessian pass "
                         "runs alongside (0: run every search after the last Hessian pass)")
@@ -243,30 +249,56 @@ class Matrix:
         self.packed = torch.empty(self.m, self.n // 2, dtype=torch.uint8, device=device)
 
 
+def column_blocks(S: Space, col_block: int):
+    """Column blocks [c0, c1) of an input space: the whole width when col_block is 0 or
+    not smaller than n."""
+    if col_block <= 0 or col_block >= S.n:
+        return [(0, S.n)]
+    return [(c0, min(S.n, c0 + col_block)) for c0 in range(0, S.n, col_block)]
+
+
+def hessian_calls(S: Space, c0: int, c1: int):
+    """Token ranges (t0, t1) of the Hessian calls over the channels [c0, c1): the space's
+    chunks for the whole width, else launches of about a chunk's bytes."""
+    rows = S.chunk if c1 - c0 == S.n else max(S.chunk, S.chunk * S.n // (c1 - c0))
+    return [(t0, min(S.tokens, t0 + rows)) for t0 in range(0, S.tokens, rows)]
+
+
 class Work:
     """Device-resident inputs and outputs of one layer of a workload."""
 
-    def __init__(self, W: wl.Workload, rank: int, win, device, tokens=None, init="rtn"):
-        self.W, self.win, self.init = W, tuple(win), init
+    def __init__(self, W: wl.Workload, rank: int, win, device, tokens=None, init="rtn", col_block=0):
+        if col_block % 64:
+            raise SystemExit("--col-block must be a multiple of 64")
+        self.W, self.win, self.init, self.col_block = W, tuple(win), init, col_block
         self.seed = W.layer_seed(0) + 7919 * rank
         self.spaces = {name: Space(W, name, n, self.seed, device, tokens) for name, n in W.input_spaces()}
         self.mats = [Matrix(W, L, self.spaces[L.input_space], self.seed, device) for L in W.layers]
         self.groups = sum(M.groups for M in self.mats)
-        self.h_bytes = sum(2 * S.tokens * S.n + 8 * S.n * S.nchunks for S in self.spaces.values())
-        self.h_launches = sum(S.nchunks for S in self.spaces.values())
+        # pieces of the step in order: (space, c0, c1)
+        self.pieces = [(S, c0, c1) for S in self.spaces.values() for c0, c1 in column_blocks(S, col_block)]
+        calls = [(c1 - c0, t1 - t0) for S, c0, c1 in self.pieces for t0, t1 in hessian_calls(S, c0, c1)]
+        self.h_bytes = sum(2 * rows * width + 8 * width for width, rows in calls)
+        self.h_launches = len(calls)
         self.ws = None
 
 
-def hessian_phase(hs, work: Work, xs=None, only=None):
-    """For every input space (or the one named `only`): h = 0, then one
-    hscale_hessian_diag_accumulate per chunk."""
-    for S in work.spaces.values():
-        if only is not None and S.name != only:
-            continue
-        x = S.x if xs is None else xs[S.name]
-        S.h.zero_()
-        for c in range(S.nchunks):
-            hs.hscale_hessian_diag_accumulate(x[c * S.chunk:(c + 1) * S.chunk], S.h)
+def hessian_block(hs, S: Space, c0: int, c1: int):
+    """h[c0:c1] = 0, then the Hessian calls over every token of the channels [c0, c1)."""
+    h = S.h[c0:c1]
+    h.zero_()
+    for t0, t1 in hessian_calls(S, c0, c1):
+        hs.hscale_hessian_diag_accumulate(S.x[t0:t1, c0:c1], h)
+
+
+def refine_block(hs, work: Work, M, c0: int, c1: int, down, up, ctas_per_sm=0):
+    """The search of the columns [c0, c1) of one matrix, on 2-D views of W and its outputs."""
+    if (c0, c1) == (0, M.n):
+        return refine(hs, work, M, down, up, ctas_per_sm=ctas_per_sm)
+    g0, g1 = c0 // 16, c1 // 16
+    init = M.codes0[:, g0:g1] if work.init == "4over6-2pass" else None
+    hs.hscale_refine_scales_strided(M.w[:, c0:c1], M.space.h[c0:c1], M.sg, init, work.init == "4over6", down, up,
+                                    M.codes[:, g0:g1], M.packed[:, c0 // 2:c1 // 2], ctas_per_sm)
 
 
 def init_codes(hs, work: Work, M, w=None):
@@ -307,26 +339,32 @@ def scale_phase(hs, work: Work, win=None, ws=None):
 
 
 def run_step(hs, work: Work):
-    """One eager pass of the hot path on the current stream."""
-    hessian_phase(hs, work)
-    scale_phase(hs, work)
+    """One eager pass of the hot path on the current stream, piece by piece."""
+    init_phase(hs, work)
+    down, up = work.win
+    for S, c0, c1 in work.pieces:
+        hessian_block(hs, S, c0, c1)
+        for M in work.mats:
+            if M.space is S:
+                refine_block(hs, work, M, c0, c1, down, up)
 
 
 class StepGraphs:
-    """The step's launches as CUDA graphs on three streams.
+    """The step's launches as CUDA graphs on three streams.  The step is a sequence of
+    pieces: a column block [c0, c1) of one input space (a whole space when the step is
+    not blocked).
 
-    main:   the Hessian pass of each input space in turn (HBM-bound);
+    main:   the Hessian pass of each piece in turn (HBM-bound);
     side:   the weight-only calls of every matrix (s_g, 4over6 codes), alongside;
-    search: the searches of an input space's matrices (ALU-bound), started as soon as
-            that space's h is complete and the weight-only calls are done, so that they
-            run alongside the next space's Hessian pass.  Those searches keep at most
-            `overlap_ctas` CTAs resident per SM, which leaves registers for the Hessian
-            CTAs; the last space's searches fill the GPU.  overlap_ctas = 0 runs every
-            search after the last Hessian pass instead."""
+    search: the searches of a piece (the piece's columns of every matrix of its space;
+            ALU-bound), started as soon as the piece's h is complete and the weight-only
+            calls are done, so that they run alongside the next piece's Hessian pass.
+            Those searches keep at most `overlap_ctas` CTAs resident per SM, which leaves
+            registers for the Hessian CTAs; the last piece's searches fill the GPU.
+            overlap_ctas = 0 runs every search after the last Hessian pass instead."""
 
     def __init__(self, hs, work: Work, overlap_ctas: int):
         self.work, self.overlap = work, overlap_ctas > 0
-        spaces = list(work.spaces.values())
         warm = torch.cuda.Stream()
         warm.wait_stream(torch.cuda.current_stream())
         with torch.cuda.stream(warm):
@@ -335,17 +373,17 @@ class StepGraphs:
         torch.cuda.synchronize()
         down, up = work.win
         self.gh, self.gr = [], []
-        for i, S in enumerate(spaces):
+        for i, (S, c0, c1) in enumerate(work.pieces):
             g = torch.cuda.CUDAGraph()
             with torch.cuda.graph(g):
-                hessian_phase(hs, work, only=S.name)
+                hessian_block(hs, S, c0, c1)
             self.gh.append(g)
-            ctas = overlap_ctas if (self.overlap and i + 1 < len(spaces)) else 0
+            ctas = overlap_ctas if (self.overlap and i + 1 < len(work.pieces)) else 0
             g = torch.cuda.CUDAGraph()
             with torch.cuda.graph(g):
                 for M in work.mats:
                     if M.space is S:
-                        refine(hs, work, M, down, up, ctas_per_sm=ctas)
+                        refine_block(hs, work, M, c0, c1, down, up, ctas_per_sm=ctas)
             self.gr.append(g)
         self.gi = torch.cuda.CUDAGraph()
         with torch.cuda.graph(self.gi):
@@ -353,7 +391,7 @@ class StepGraphs:
         torch.cuda.synchronize()
         self.side, self.search = torch.cuda.Stream(), torch.cuda.Stream()
         self.ev_init = torch.cuda.Event()
-        self.ev_h = [torch.cuda.Event() for _ in spaces]
+        self.ev_h = [torch.cuda.Event() for _ in work.pieces]
 
     def replay(self, ev=None):
         """One step.  ev: optional (start, after the last Hessian pass, end) timing events
@@ -656,7 +694,7 @@ def gpu_arm(args, d: Dist):
     dev = torch.device("cuda", d.local)
     W = wl.WORKLOADS[args.workload]
     win = window_of(args, W)
-    work = Work(W, d.rank, win, dev, tokens=args.tokens, init=args.init)
+    work = Work(W, d.rank, win, dev, tokens=args.tokens, init=args.init, col_block=args.col_block)
     work.ws = torch.empty(hs.hscale_rtn_workspace_bytes(), dtype=torch.uint8, device=dev)
     torch.cuda.synchronize()
 
@@ -735,7 +773,9 @@ def gpu_arm(args, d: Dist):
     ms_h_launch = ms_h / work.h_launches
     h_gbs = work.h_bytes / (ms_h * 1e-3) / 1e9
     first = next(iter(work.spaces.values()))
-    traffic = profiled_traffic(W.name, first.chunk, first.n) if len(work.spaces) == 1 else None
+    _, c0, c1 = work.pieces[0]
+    t0, t1 = hessian_calls(first, c0, c1)[0]
+    traffic = profiled_traffic(W.name, t1 - t0, c1 - c0) if len(work.spaces) == 1 else None
 
     # ---- end to end through the public API with host buffers
     e2e = None if args.no_e2e else e2e_leg(hs, work, args)
@@ -750,6 +790,7 @@ def gpu_arm(args, d: Dist):
                    "matrices": [[M.name, M.m, M.n] for M in work.mats],
                    "input_spaces": [[S.name, S.tokens, S.n, S.chunk] for S in work.spaces.values()],
                    "window": list(win), "init": work.init, "groups": work.groups,
+                   "col_block": work.col_block,
                    "l2": "inputs larger than L2: %.2f GB of X streamed per step" %
                          (sum(S.tokens * S.n * 2 for S in work.spaces.values()) / 1e9),
                    "parallelism": f"independent layer per GPU x{d.world}"},
@@ -762,10 +803,13 @@ def gpu_arm(args, d: Dist):
                       "weight_only": ms_init, "refine": main["ms"]},
         "ms_per_step_eager": ms_eager,
         "timed_launch": ("CUDA graphs of the step's API calls on three streams: the Hessian pass of "
-                         "each input space; alongside it the weight-only calls (s_g, 4over6 codes); the "
-                         "searches of each input space as soon as its h is complete"
+                         + (f"each {work.col_block}-channel column block of each input space over every token"
+                            if work.col_block else "each input space in token chunks")
+                         + "; alongside it the weight-only calls (s_g, 4over6 codes); the searches of "
+                         + ("each block" if work.col_block else "each input space")
+                         + " as soon as its h is complete"
                          + (f" (at most {args.overlap_ctas} search CTAs per SM while a Hessian pass runs)"
-                            if args.overlap_ctas > 0 and len(work.spaces) > 1 else "")),
+                            if args.overlap_ctas > 0 and len(work.pieces) > 1 else "")),
         "hessian": {"gbs": h_gbs, "tokens_channels_per_s": work.h_bytes / 2 / (ms_h * 1e-3),
                     "frac_of_measured_hbm": h_gbs / hbm_peak, "frac_of_8TBs": h_gbs / HBM_SPEC_GBS},
         "search": {"groups_per_s": main["groups_per_s"], "candidates": main["candidates"],

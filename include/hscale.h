@@ -22,6 +22,7 @@
  *                                       alternative start for the refinement (Sec. 3.5)
  *      hscale_refine_scales_4over6      Algorithm 2 in one pass: those codes decided
  *                                       inside the search
+ *      hscale_refine_scales_strided     the search on 2-D views (column blocks, slices)
  *      hscale_dequant_residual          dW = W - W_hat of the packed weights (Eqs. 1-3)
  *      hscale_output_error              ||X dW^T||_F^2 on the tensor cores (Eq. 3)
  *      hscale_hessian_full_accumulate   H += X^T X on the tensor cores (Algorithm 3)
@@ -236,6 +237,35 @@ int hscale_refine_scales_ex(const void* w_bf16, const float* h, int64_t m, int64
 int hscale_refine_scales_4over6(const void* w_bf16, const float* h, int64_t m, int64_t n,
                                 const float* global_scale, int32_t down, int32_t up, uint8_t* codes_out,
                                 uint8_t* packed_out, int32_t ctas_per_sm, void* stream);
+
+/*
+ * The search on 2-D views: hscale_refine_scales_ex / hscale_refine_scales_4over6 on a
+ * block of columns (or rows) of larger arrays.  The paper has no counterpart: it lets a
+ * caller search a column block of W as soon as h of those channels is final, while the
+ * Hessian pass of the next block runs, or quantize one slice of a fused matrix.
+ *
+ * w             [m, n] bfloat16 view; row r starts at element r * ld_w.  w 16-byte
+ *               aligned, ld_w >= n, ld_w % 8 == 0 (every row 16-byte aligned).
+ * h             [n] fp32 of the view's columns, 16-byte aligned; NULL means h = 1.
+ * global_scale  device fp32 scalar s_g (of the whole matrix the view belongs to).
+ * init_codes    NULL, or [m, n/16] bytes with rows ld_init bytes apart, ld_init >= n/16
+ *               (used only when fourover6 = 0; ld_init is ignored when it is NULL).
+ * fourover6     0: initial codes from init_codes, or RTN (Eq. 7) when it is NULL;
+ *               1: Algorithm 2's 4over6 codes decided in place (init_codes must be NULL).
+ *               Other values and fourover6 = 1 with init_codes return HSCALE_ERR_ARG.
+ * codes_out     [m, n/16] bytes with rows ld_codes bytes apart (ld_codes >= n/16), written.
+ * packed_out    NULL, or [m, n/2] bytes with rows ld_packed bytes apart: 8-byte aligned,
+ *               ld_packed >= n/2 and ld_packed % 8 == 0.
+ * down, up, ctas_per_sm as for hscale_refine_scales_ex.
+ *
+ * Every group's result depends only on its 16 weights, its 16 h values, s_g and the
+ * window, so a view gives exactly the bytes the whole-matrix call writes there.
+ */
+int hscale_refine_scales_strided(const void* w_bf16, int64_t ld_w, const float* h, int64_t m, int64_t n,
+                                 const float* global_scale, const uint8_t* init_codes, int64_t ld_init,
+                                 int32_t fourover6, int32_t down, int32_t up, uint8_t* codes_out,
+                                 int64_t ld_codes, uint8_t* packed_out, int64_t ld_packed, int32_t ctas_per_sm,
+                                 void* stream);
 
 /*
  * Final FP4 quantization with given codes (Sec. 3.3 "Final re-quantization", Eq. 2):

@@ -25,7 +25,8 @@ __all__ = [
     "hscale_device_error_flags",
     "hscale_hessian_diag_accumulate", "hscale_rtn_workspace_bytes", "hscale_rtn_scales",
     "hscale_rtn_scales_noalloc",
-    "hscale_refine_scales", "hscale_refine_scales_ex", "hscale_refine_scales_4over6", "hscale_pack_nvfp4", "hscale_fourover6_codes",
+    "hscale_refine_scales", "hscale_refine_scales_ex", "hscale_refine_scales_4over6",
+    "hscale_refine_scales_strided", "hscale_pack_nvfp4", "hscale_fourover6_codes",
     "hscale_dequant_residual", "hscale_output_error_workspace_bytes", "hscale_output_error",
     "residual_ld", "hscale_selftest_bounded_wait", "hscale_hessian_full_workspace_bytes",
     "hscale_hessian_full_accumulate", "hscale_gptq_factor_workspace_bytes", "hscale_gptq_factor",
@@ -51,6 +52,8 @@ _SIGNATURES = {
     "hscale_refine_scales": (ctypes.c_int, [_P, _P, _I64, _I64, _P, _P, _I32, _I32, _P, _P, _P]),
     "hscale_refine_scales_ex": (ctypes.c_int, [_P, _P, _I64, _I64, _P, _P, _I32, _I32, _P, _P, _I32, _P]),
     "hscale_refine_scales_4over6": (ctypes.c_int, [_P, _P, _I64, _I64, _P, _I32, _I32, _P, _P, _I32, _P]),
+    "hscale_refine_scales_strided": (ctypes.c_int, [_P, _I64, _P, _I64, _I64, _P, _P, _I64, _I32, _I32, _I32,
+                                                    _P, _I64, _P, _I64, _I32, _P]),
     "hscale_pack_nvfp4": (ctypes.c_int, [_P, _I64, _I64, _P, _P, _P, _P]),
     "hscale_fourover6_codes": (ctypes.c_int, [_P, _I64, _I64, _P, _P, _P]),
     "hscale_dequant_residual": (ctypes.c_int, [_P, _I64, _I64, _P, _P, _P, _P, _I64, _P]),
@@ -255,6 +258,38 @@ def hscale_refine_scales_4over6(w: torch.Tensor, h: torch.Tensor | None, global_
            load().hscale_refine_scales_4over6(_ptr(w), _ptr(h), m, n, _ptr(global_scale), int(down), int(up),
                                               _ptr(codes_out), _ptr(packed_out), int(ctas_per_sm),
                                               _stream_ptr(stream)))
+
+
+def _row_view(t: torch.Tensor, name: str, dtype, rows: int, cols: int) -> int:
+    """Row stride (elements) of a 2-D view with unit column stride; checks its shape."""
+    _need(t, dtype, name)
+    if t.dim() != 2 or tuple(t.shape) != (rows, cols) or (cols > 1 and t.stride(1) != 1):
+        raise ValueError(f"{name} must be a [{rows}, {cols}] view with contiguous rows")
+    return t.stride(0) if rows > 1 else max(cols, t.stride(0))
+
+
+def hscale_refine_scales_strided(w: torch.Tensor, h: torch.Tensor | None, global_scale: torch.Tensor,
+                                 init_codes: torch.Tensor | None, fourover6: bool, down: int, up: int,
+                                 codes_out: torch.Tensor, packed_out: torch.Tensor | None,
+                                 ctas_per_sm: int = 0, stream=None) -> None:
+    """The search on 2-D views (e.g. ``W[:, c0:c1]``, ``codes[:, c0/16:c1/16]``,
+    ``packed[:, c0/2:c1/2]``)."""
+    if w.dim() != 2:
+        raise ValueError("w must be a 2-D view")
+    m, n = w.shape
+    ld_w = _row_view(w, "w", torch.bfloat16, m, n)
+    _need(global_scale, torch.float32, "global_scale")
+    if h is not None:
+        _need(h, torch.float32, "h")
+        if h.numel() != n or not h.is_contiguous():
+            raise ValueError("h must be a contiguous float32 vector of length n")
+    ld_c = _row_view(codes_out, "codes_out", torch.uint8, m, n // 16)
+    ld_i = 0 if init_codes is None else _row_view(init_codes, "init_codes", torch.uint8, m, n // 16)
+    ld_p = 0 if packed_out is None else _row_view(packed_out, "packed_out", torch.uint8, m, n // 2)
+    _check("hscale_refine_scales_strided",
+           load().hscale_refine_scales_strided(_ptr(w), ld_w, _ptr(h), m, n, _ptr(global_scale), _ptr(init_codes),
+                                               ld_i, int(bool(fourover6)), int(down), int(up), _ptr(codes_out), ld_c,
+                                               _ptr(packed_out), ld_p, int(ctas_per_sm), _stream_ptr(stream)))
 
 
 def hscale_pack_nvfp4(w: torch.Tensor, global_scale: torch.Tensor, codes: torch.Tensor,

@@ -129,33 +129,43 @@ int hscale_refine_scales_ex(const void* w_bf16, const float* h, int64_t m, int64
                             const float* global_scale, const uint8_t* init_codes, int32_t down,
                             int32_t up, uint8_t* codes_out, uint8_t* packed_out,
                             int32_t ctas_per_sm, void* stream) {
-  int st = check_weight(w_bf16, m, n);
-  if (st != HSCALE_OK) return st;
-  if (down < 0 || up < 0 || down > 125 || up > 125) return HSCALE_ERR_ARG;
-  if (ctas_per_sm < 0) return HSCALE_ERR_ARG;
-  if (m == 0 || n == 0) return HSCALE_OK;
-  if (global_scale == nullptr || codes_out == nullptr) return HSCALE_ERR_NULL;
-  if (!aligned(global_scale, 4)) return HSCALE_ERR_ALIGN;
-  if (h != nullptr && !aligned(h, 16)) return HSCALE_ERR_ALIGN;
-  if (packed_out != nullptr && !aligned(packed_out, 8)) return HSCALE_ERR_ALIGN;
-  return from_cuda(hscale::launch_refine(w_bf16, h, m, n, global_scale, init_codes, down, up,
-                                         codes_out, packed_out, ctas_per_sm, false, as_stream(stream)));
+  return hscale_refine_scales_strided(w_bf16, n, h, m, n, global_scale, init_codes, n / 16, 0, down, up,
+                                      codes_out, n / 16, packed_out, n / 2, ctas_per_sm, stream);
 }
 
 int hscale_refine_scales_4over6(const void* w_bf16, const float* h, int64_t m, int64_t n,
                                 const float* global_scale, int32_t down, int32_t up, uint8_t* codes_out,
                                 uint8_t* packed_out, int32_t ctas_per_sm, void* stream) {
+  return hscale_refine_scales_strided(w_bf16, n, h, m, n, global_scale, nullptr, 0, 1, down, up, codes_out,
+                                      n / 16, packed_out, n / 2, ctas_per_sm, stream);
+}
+
+int hscale_refine_scales_strided(const void* w_bf16, int64_t ld_w, const float* h, int64_t m, int64_t n,
+                                 const float* global_scale, const uint8_t* init_codes, int64_t ld_init,
+                                 int32_t fourover6, int32_t down, int32_t up, uint8_t* codes_out,
+                                 int64_t ld_codes, uint8_t* packed_out, int64_t ld_packed, int32_t ctas_per_sm,
+                                 void* stream) {
   int st = check_weight(w_bf16, m, n);
   if (st != HSCALE_OK) return st;
   if (down < 0 || up < 0 || down > 125 || up > 125) return HSCALE_ERR_ARG;
-  if (ctas_per_sm < 0) return HSCALE_ERR_ARG;
+  if (ctas_per_sm < 0 || (fourover6 != 0 && fourover6 != 1)) return HSCALE_ERR_ARG;
+  if (fourover6 && init_codes != nullptr) return HSCALE_ERR_ARG;
   if (m == 0 || n == 0) return HSCALE_OK;
+  if (ld_w < n || ld_codes < n / 16 || (packed_out != nullptr && ld_packed < n / 2) ||
+      (init_codes != nullptr && ld_init < n / 16))
+    return HSCALE_ERR_SHAPE;
+  if (ld_w > INT64_MAX / m || ld_codes > INT64_MAX / m || (packed_out != nullptr && ld_packed > INT64_MAX / m) ||
+      (init_codes != nullptr && ld_init > INT64_MAX / m))
+    return HSCALE_ERR_SHAPE;
+  if (ld_w % 8 != 0) return HSCALE_ERR_ALIGN;
   if (global_scale == nullptr || codes_out == nullptr) return HSCALE_ERR_NULL;
   if (!aligned(global_scale, 4)) return HSCALE_ERR_ALIGN;
   if (h != nullptr && !aligned(h, 16)) return HSCALE_ERR_ALIGN;
-  if (packed_out != nullptr && !aligned(packed_out, 8)) return HSCALE_ERR_ALIGN;
-  return from_cuda(hscale::launch_refine(w_bf16, h, m, n, global_scale, nullptr, down, up, codes_out,
-                                         packed_out, ctas_per_sm, true, as_stream(stream)));
+  if (packed_out != nullptr && (!aligned(packed_out, 8) || ld_packed % 8 != 0)) return HSCALE_ERR_ALIGN;
+  return from_cuda(hscale::launch_refine(w_bf16, ld_w, h, m, n, global_scale, init_codes,
+                                         init_codes ? ld_init : 0, down, up, codes_out, ld_codes, packed_out,
+                                         packed_out ? ld_packed : 0, ctas_per_sm, fourover6 != 0,
+                                         as_stream(stream)));
 }
 
 int hscale_fourover6_codes(const void* w_bf16, int64_t m, int64_t n, const float* global_scale,

@@ -110,14 +110,19 @@ struct Group {
   float2 a[8];     // w * 2^-K, elements (2i, 2i+1)
 };
 
-__device__ __forceinline__ void load_group(const uint4* w, int64_t g, float pw, Group& G) {
-  const uint4 p = ld_stream_v4(w + 2 * g);
-  const uint4 q = ld_stream_v4(w + 2 * g + 1);
+// The group whose 16 bf16 values start at wg (16-byte aligned).
+__device__ __forceinline__ void load_group_at(const uint4* wg, float pw, Group& G) {
+  const uint4 p = ld_stream_v4(wg);
+  const uint4 q = ld_stream_v4(wg + 1);
   G.wb[0] = p.x; G.wb[1] = p.y; G.wb[2] = p.z; G.wb[3] = p.w;
   G.wb[4] = q.x; G.wb[5] = q.y; G.wb[6] = q.z; G.wb[7] = q.w;
 #pragma unroll
   for (int i = 0; i < 8; ++i)
     G.a[i] = __fmul2_rn(make_float2(bf16_lo(G.wb[i]), bf16_hi(G.wb[i])), make_float2(pw, pw));
+}
+
+__device__ __forceinline__ void load_group(const uint4* w, int64_t g, float pw, Group& G) {
+  load_group_at(w + 2 * g, pw, G);
 }
 
 // Per-block table of the candidate constants of every E4M3 code c (1..126), filled once
@@ -213,11 +218,11 @@ __device__ __forceinline__ float exact_term(float a_k, float hj, uint32_t c, flo
 // The whole warp rescores the group of lane `owner` with exact rounding decisions and
 // returns its winning code (in every lane).  Lanes 0-15 take the candidates lo, lo+2,
 // ..., lanes 16-31 lo+1, lo+3, ...; lane j of each half scores element j & 15.
-__device__ __noinline__ int warp_exact_search(int owner, const uint4* w, int64_t g_own, const float* h,
+__device__ __noinline__ int warp_exact_search(int owner, const uint16_t* wg_own, const float* h,
                                  int64_t hcol_own, int c0, int lo, int hi, float sgk, float pw) {
   const int lane = threadIdx.x & 31;
   const int j = lane & 15, half = lane >> 4;
-  const uint16_t wb = reinterpret_cast<const uint16_t*>(w)[g_own * 16 + j];
+  const uint16_t wb = wg_own[j];
   const float a_k = __fmul_rn(fabsf(__uint_as_float((uint32_t)wb << 16)), pw);
   const float hj = h ? h[hcol_own * 16 + j] : 1.0f;
   const unsigned mask = 0xFFFFu << (16 * half);
@@ -343,10 +348,10 @@ __device__ __forceinline__ bool fast_winner_certain(float e1, float e2, float A)
 // The anchor choice of Algorithm 2 for one group with exact rounding decisions (the
 // group is read back from global memory); the anchor 4 code c4 wins an exact tie.  Kept
 // out of line: the search calls it only when the fast scores cannot order the anchors.
-__device__ __noinline__ uint32_t fourover6_exact_pick(const uint4* w, int64_t g, float pw, uint32_t c4,
-                                                      uint32_t c6, float sgk) {
+__device__ __noinline__ uint32_t fourover6_exact_pick(const uint4* wg, float pw, uint32_t c4, uint32_t c6,
+                                                      float sgk) {
   Group G;
-  load_group(w, g, pw, G);
+  load_group_at(wg, pw, G);
   return exact_group_mse(G, c6, sgk) < exact_group_mse(G, c4, sgk) ? c6 : c4;
 }
 
@@ -356,7 +361,7 @@ __device__ __noinline__ uint32_t fourover6_exact_pick(const uint4* w, int64_t g,
 // fast order is the order of the exact errors, and the exact fp32 sums (relative error
 // <= 7 * 2^-24, far inside the margin) order them the same way; so the result is always
 // the code fourover6_codes_kernel writes.
-__device__ __forceinline__ int fourover6_init_code(const Group& G, const uint4* w, int64_t g, const float4* tab,
+__device__ __forceinline__ int fourover6_init_code(const Group& G, const uint4* wg, const float4* tab,
                                                    float amax_k, float sgk, float pw, float inv4, float inv6) {
   const uint32_t c4 = anchored_code(amax_k, sgk, inv4, 2.0f);
   const uint32_t c6 = anchored_code(amax_k, sgk, inv6, 3.0f);
@@ -368,7 +373,7 @@ __device__ __forceinline__ int fourover6_init_code(const Group& G, const uint4* 
   for (int i = 0; i < 8; ++i) acc = __ffma2_rn(G.a[i], G.a[i], acc);
   const float A = __fadd_rn(acc.x, acc.y);
   if (fast_winner_certain(fminf(e4, e6), fmaxf(e4, e6), A)) return (int)(e6 < e4 ? c6 : c4);
-  return (int)fourover6_exact_pick(w, g, pw, c4, c6, sgk);
+  return (int)fourover6_exact_pick(wg, pw, c4, c6, sgk);
 }
 
 // ---------------------------------------------------------------- refine (Algorithm 1)
@@ -377,11 +382,14 @@ __device__ __forceinline__ int fourover6_init_code(const Group& G, const uint4* 
 // changes.  7 resident CTAs of 4 warps per SM (72 registers); the rarely taken
 // warp-cooperative rescoring is a separate call so it does not raise that.
 // kFourOverSix: the initial codes are Algorithm 2's, decided in place (init_codes unused).
+// W, the codes and the nibbles are 2-D views: row r starts at element r * ld_w of w, byte
+// r * ld_i of the initial codes, byte r * ld_c of the codes and 8-byte word r * ld_p of the
+// nibbles.
 template <bool kFourOverSix>
 __global__ void __launch_bounds__(kRefineThreads, 7)
-refine_kernel(const uint4* __restrict__ w, const float* __restrict__ h, int64_t m, int ng,
-              const float* __restrict__ global_scale, const uint8_t* init_codes,
-              int down, int up, uint8_t* codes_out, uint2* __restrict__ packed_out) {
+refine_kernel(const uint4* __restrict__ w, int64_t ld_w, const float* __restrict__ h, int64_t m, int ng,
+              const float* __restrict__ global_scale, const uint8_t* init_codes, int64_t ld_i,
+              int down, int up, uint8_t* codes_out, int64_t ld_c, uint2* __restrict__ packed_out, int64_t ld_p) {
   const int lane = threadIdx.x & 31;
   const int64_t warp_global = ((int64_t)blockIdx.x * blockDim.x + threadIdx.x) >> 5;
   const int64_t warps_total = ((int64_t)gridDim.x * blockDim.x) >> 5;
@@ -412,7 +420,7 @@ refine_kernel(const uint4* __restrict__ w, const float* __restrict__ h, int64_t 
     }
     const int gcol = chunk * 32 + lane;
     const bool active = gcol < ng;
-    const int64_t g = row * ng + gcol;
+    const int64_t wofs = row * ld_w + (int64_t)gcol * 16;  // first element of the group
 
     if (chunk != cur_chunk) {
       cur_chunk = chunk;
@@ -430,15 +438,15 @@ refine_kernel(const uint4* __restrict__ w, const float* __restrict__ h, int64_t 
     Group G;
     int c0 = 1, lo = 1, hi = 1;
     if (active) {
-      load_group(w, g, d.pw, G);
+      load_group_at(w + wofs / 8, d.pw, G);
       if (!kFourOverSix && init_codes != nullptr) {
-        c0 = init_codes[g] & 0x7F;
+        c0 = init_codes[row * ld_i + gcol] & 0x7F;
         c0 = c0 < 1 ? 1 : (c0 > (int)kE4M3MaxCode ? (int)kE4M3MaxCode : c0);
       } else {
         const uint32_t amax = group_abs_max_bits(make_uint4(G.wb[0], G.wb[1], G.wb[2], G.wb[3]),
                                                  make_uint4(G.wb[4], G.wb[5], G.wb[6], G.wb[7]));
         const float amax_k = __fmul_rn(__uint_as_float(amax << 16), d.pw);
-        c0 = kFourOverSix ? fourover6_init_code(G, w, g, tab, amax_k, d.sgk, d.pw, inv4, inv6)
+        c0 = kFourOverSix ? fourover6_init_code(G, w + wofs / 8, tab, amax_k, d.sgk, d.pw, inv4, inv6)
                           : (int)rtn_code(amax_k, d.sgk, inv6);
       }
       lo = max(1, c0 - down);
@@ -458,20 +466,21 @@ refine_kernel(const uint4* __restrict__ w, const float* __restrict__ h, int64_t 
     while (amb) {
       const int owner = __ffs(amb) - 1;
       amb &= amb - 1;
-      const int64_t g_own = __shfl_sync(0xFFFFFFFFu, g, owner);
+      const int64_t wofs_own = __shfl_sync(0xFFFFFFFFu, wofs, owner);
       const int gcol_own = __shfl_sync(0xFFFFFFFFu, gcol, owner);
       const int c0o = __shfl_sync(0xFFFFFFFFu, c0, owner);
       const int loo = __shfl_sync(0xFFFFFFFFu, lo, owner);
       const int hio = __shfl_sync(0xFFFFFFFFu, hi, owner);
-      const int bc = warp_exact_search(owner, w, g_own, h, gcol_own, c0o, loo, hio, d.sgk, d.pw);
+      const int bc = warp_exact_search(owner, reinterpret_cast<const uint16_t*>(w) + wofs_own, h, gcol_own,
+                                       c0o, loo, hio, d.sgk, d.pw);
       if (lane == owner) best = bc;
     }
 
     if (active) {
-      codes_out[g] = (uint8_t)best;
+      codes_out[row * ld_c + gcol] = (uint8_t)best;
       if (packed_out != nullptr)
-        packed_out[g] = quantize_pack(G, (uint32_t)best, __fmul_rn(tab[best].z, 0x1p-126f), d.sgk, d.pw,
-                                      reinterpret_cast<const uint16_t*>(w) + g * 16);
+        packed_out[row * ld_p + gcol] = quantize_pack(G, (uint32_t)best, __fmul_rn(tab[best].z, 0x1p-126f), d.sgk,
+                                                      d.pw, reinterpret_cast<const uint16_t*>(w) + wofs);
     }
   }
 }
@@ -561,10 +570,10 @@ cudaError_t launch_rtn_codes(const void* w, int64_t m, int64_t n, const uint32_t
   return cudaGetLastError();
 }
 
-cudaError_t launch_refine(const void* w, const float* h, int64_t m, int64_t n,
-                          const float* global_scale, const uint8_t* init_codes, int down, int up,
-                          uint8_t* codes_out, uint8_t* packed_out, int ctas_per_sm, bool fourover6,
-                          cudaStream_t stream) {
+cudaError_t launch_refine(const void* w, int64_t ld_w, const float* h, int64_t m, int64_t n,
+                          const float* global_scale, const uint8_t* init_codes, int64_t ld_init, int down,
+                          int up, uint8_t* codes_out, int64_t ld_codes, uint8_t* packed_out, int64_t ld_packed,
+                          int ctas_per_sm, bool fourover6, cudaStream_t stream) {
   DeviceInfo info;
   cudaError_t err = current_device_info(&info);
   if (err != cudaSuccess) return err;
@@ -576,9 +585,10 @@ cudaError_t launch_refine(const void* w, const float* h, int64_t m, int64_t n,
   const int64_t resident = (int64_t)info.sm_count * per_sm;
   const int64_t blocks = std::max<int64_t>(1, std::min<int64_t>((units + kWarpsPerRefineBlock - 1) / kWarpsPerRefineBlock, resident));
   auto kernel = fourover6 ? refine_kernel<true> : refine_kernel<false>;
-  kernel<<<(unsigned)blocks, kRefineThreads, 0, stream>>>(static_cast<const uint4*>(w), h, m, ng, global_scale,
-                                                          fourover6 ? nullptr : init_codes, down, up, codes_out,
-                                                          reinterpret_cast<uint2*>(packed_out));
+  kernel<<<(unsigned)blocks, kRefineThreads, 0, stream>>>(static_cast<const uint4*>(w), ld_w, h, m, ng, global_scale,
+                                                          fourover6 ? nullptr : init_codes, ld_init, down, up,
+                                                          codes_out, ld_codes, reinterpret_cast<uint2*>(packed_out),
+                                                          ld_packed / 8);
   return cudaGetLastError();
 }
 

@@ -103,6 +103,35 @@ def test_refine_ex_argument_errors(lib):
     assert f(None, None, 0, 32, None, None, 4, 4, None, None, 5, None) == OK
 
 
+def test_refine_strided_argument_errors(lib):
+    f = lib.hscale_refine_scales_strided
+    ok = (FAKE, 64, FAKE, 4, 32, FAKE, None, 0, 0, 4, 4, FAKE, 4, FAKE, 32, 0, None)
+
+    def call(**kw):
+        names = ["w", "ld_w", "h", "m", "n", "sg", "init", "ld_i", "f46", "down", "up", "codes", "ld_c",
+                 "packed", "ld_p", "ctas", "stream"]
+        args = dict(zip(names, ok))
+        args.update(kw)
+        return f(*[args[k] for k in names])
+
+    assert call(ld_w=16) == ERR_SHAPE                 # ld_w < n
+    assert call(ld_w=36) == ERR_ALIGN                 # rows not 16-byte aligned
+    assert call(ld_c=1) == ERR_SHAPE                  # ld_codes < n/16
+    assert call(ld_p=8) == ERR_SHAPE                  # ld_packed < n/2
+    assert call(ld_p=20) == ERR_ALIGN                 # ld_packed % 8
+    assert call(init=FAKE, ld_i=1) == ERR_SHAPE       # ld_init < n/16
+    assert call(f46=2) == ERR_ARG
+    assert call(f46=1, init=FAKE) == ERR_ARG          # 4over6 decides the codes itself
+    assert call(ctas=-1) == ERR_ARG
+    assert call(down=126) == ERR_ARG
+    assert call(codes=None) == ERR_NULL
+    assert call(sg=None) == ERR_NULL
+    assert call(w=MIS) == ERR_ALIGN
+    assert call(h=MIS) == ERR_ALIGN
+    assert call(n=40) == ERR_SHAPE
+    assert call(m=0, w=None, codes=None) == OK        # empty view: no-op
+
+
 def test_refine_4over6_argument_errors(lib):
     f = lib.hscale_refine_scales_4over6
     assert f(FAKE, FAKE, 4, 32, FAKE, 4, 4, FAKE, FAKE, -1, None) == ERR_ARG

@@ -525,6 +525,70 @@ def test_fused_fourover6_ragged_shapes(seed, m, n):
         compare_search(ref, codes, packed, f"fused 4over6 {m}x{n} window -{down}/+{up}")
 
 
+# ------------------------------------------------------------------ 2-D views (column blocks)
+
+@pytest.mark.parametrize("init", ["rtn", "given", "4over6"])
+def test_strided_column_blocks_match_whole_matrix(init):
+    """The search on column blocks of W (ragged last block, padded rows: ld_w > n), written
+    into column blocks of the outputs, gives the whole-matrix call's bytes, and the
+    oracle's on the block."""
+    m, n, pad = 96, 16 * 136, 64
+    w = small_layer(9, m, n)
+    h32 = oracle_h32(9, n, tokens=512)
+    buf = torch.zeros(m, n + pad, dtype=torch.bfloat16, device=dev())
+    buf[:, :n] = w.to(dev())
+    wd = buf[:, :n]
+    sg, rtn = gpu_rtn(w.to(dev()))
+    s_ref, _ = oracle.global_scale(bits(w))
+    hd = torch.from_numpy(h32).to(dev())
+    init_codes = rtn if init == "given" else None
+    codes = torch.empty(m, n // 16, dtype=torch.uint8, device=dev())
+    packed = torch.empty(m, n // 2, dtype=torch.uint8, device=dev())
+    if init == "4over6":
+        hs.hscale_refine_scales_4over6(w.to(dev()), hd, sg, 4, 4, codes, packed)
+    else:
+        hs.hscale_refine_scales(w.to(dev()), hd, sg, init_codes, 4, 4, codes, packed)
+    bc = torch.full((m, n // 16 + 8), 0xAB, dtype=torch.uint8, device=dev())
+    bp = torch.full((m, n // 2 + 16), 0xAB, dtype=torch.uint8, device=dev())
+    for c0, c1, ctas in ((0, 512, 4), (512, 1536, 2), (1536, n, 0)):
+        g0, g1 = c0 // 16, c1 // 16
+        hs.hscale_refine_scales_strided(wd[:, c0:c1], hd[c0:c1], sg,
+                                        None if init_codes is None else init_codes[:, g0:g1],
+                                        init == "4over6", 4, 4, bc[:, g0:g1], bp[:, c0 // 2:c1 // 2], ctas)
+    torch.cuda.synchronize()
+    assert torch.equal(bc[:, :n // 16], codes) and torch.equal(bp[:, :n // 2], packed)
+    assert bool((bc[:, n // 16:] == 0xAB).all()) and bool((bp[:, n // 2:] == 0xAB).all()), "wrote past the view"
+    # the middle block against the oracle on that block alone
+    c0, c1 = 512, 1536
+    wb = bits(w)[:, c0:c1]
+    if init == "4over6":
+        i_ref, nt = oracle.fourover6_codes(bits(w), s_ref)
+        i_ref, nt = i_ref[:, c0 // 16:c1 // 16], nt[:, c0 // 16:c1 // 16]
+    else:
+        i_ref, nt = oracle.rtn_codes(wb, s_ref), np.zeros((m, (c1 - c0) // 16), np.uint8)
+    ref = oracle.refine(wb, h32[c0:c1], s_ref, i_ref, 4, 4)
+    ref["near_tie"] = ref["near_tie"] | nt
+    compare_search(ref, bc[:, c0 // 16:c1 // 16].cpu().numpy(), bp[:, c0 // 2:c1 // 2].cpu().numpy(),
+                   f"strided block {c0}:{c1}, init {init}")
+
+
+def test_strided_row_slice_and_no_packed_output():
+    """A row slice (one row of a larger matrix) and a view without nibbles."""
+    m, n = 40, 1024
+    w = small_layer(10, m, n).to(dev())
+    h32 = oracle_h32(10, n, tokens=256)
+    hd = torch.from_numpy(h32).to(dev())
+    sg, _ = gpu_rtn(w)
+    codes, packed = gpu_refine(w, h32, sg, None, 9, 6)
+    c1 = torch.empty(1, n // 16, dtype=torch.uint8, device=dev())
+    hs.hscale_refine_scales_strided(w[17:18], hd, sg, None, False, 9, 6, c1, None, 0)
+    c2 = torch.empty(m, n // 16, dtype=torch.uint8, device=dev())
+    hs.hscale_refine_scales_strided(w, hd, sg, None, False, 9, 6, c2, None, 3)
+    torch.cuda.synchronize()
+    assert np.array_equal(c1.cpu().numpy()[0], codes[17])
+    assert np.array_equal(c2.cpu().numpy(), codes)
+
+
 # ------------------------------------------------------------------ output error (Eq. 3)
 
 def oracle_codes_packed(wb, h32, s_ref, window):
@@ -648,6 +712,9 @@ def test_full_size_output_error_q_proj():
 
 # ------------------------------------------------------------------ full-size workloads
 
+BLOCK = 1024  # channels per column block of `bench.py --col-block 1024`
+
+
 def full_size_check(name, sample_rows, layer_index=0, windows=None, fourover6=False):
     """A workload at its full size in the launch configuration bench.py times: h of every
     input space over every streamed chunk (all columns, against the oracle fed the same
@@ -672,6 +739,22 @@ def full_size_check(name, sample_rows, layer_index=0, windows=None, fourover6=Fa
         torch.cuda.synchronize()
         err = assert_h_close(h.cpu().numpy(), href)
         print(f"[parity] {name} {space}: h over {W.tokens} tokens x {n}: max rel err {err:.3e}")
+        # the column-blocked calls of `bench.py --col-block 1024`: every token of 1024
+        # channels per block, in launches of about a chunk's bytes
+        x_all = torch.empty(W.tokens, n, dtype=torch.bfloat16, device=dev())
+        for c in range(W.tokens // chunk):
+            wl.activation_chunk(chunk, a, wl.chunk_seed(seed, space, 1) & 0xFFFFFFFF, c,
+                                out=x_all[c * chunk:(c + 1) * chunk])
+        hb = torch.zeros(n, device=dev())
+        for c0 in range(0, n, BLOCK):
+            c1 = min(n, c0 + BLOCK)
+            rows = chunk if c1 - c0 == n else max(chunk, chunk * n // (c1 - c0))
+            for t0 in range(0, W.tokens, rows):
+                hs.hscale_hessian_diag_accumulate(x_all[t0:t0 + rows, c0:c1], hb[c0:c1])
+        torch.cuda.synchronize()
+        del x_all
+        err = assert_h_close(hb.cpu().numpy(), href)
+        print(f"[parity] {name} {space}: h in {BLOCK}-channel column blocks: max rel err {err:.3e}")
         h_ref[space] = href.astype(np.float32)
     for L in W.layers:
         m, n = L.out_features, L.in_features
@@ -700,6 +783,19 @@ def full_size_check(name, sample_rows, layer_index=0, windows=None, fourover6=Fa
                 # the one-pass form, at the launch shape the bench times it with (4 CTAs/SM)
                 codes_f, packed_f = gpu_refine_4over6(w, h_ref[L.input_space], sg, down, up, 4)
                 assert np.array_equal(codes_f, codes_g) and np.array_equal(packed_f, packed_g)
+            # the column-blocked searches of `bench.py --col-block 1024` (views, 4 CTAs/SM
+            # but the last block)
+            hd = torch.from_numpy(h_ref[L.input_space]).to(dev())
+            bc = torch.empty(m, n // 16, dtype=torch.uint8, device=dev())
+            bp = torch.empty(m, n // 2, dtype=torch.uint8, device=dev())
+            for c0 in range(0, n, BLOCK):
+                c1 = min(n, c0 + BLOCK)
+                g0, g1 = c0 // 16, c1 // 16
+                hs.hscale_refine_scales_strided(w[:, c0:c1], hd[c0:c1], sg, None if init is None else init[:, g0:g1],
+                                                False, down, up, bc[:, g0:g1], bp[:, c0 // 2:c1 // 2],
+                                                4 if c1 < n else 0)
+            torch.cuda.synchronize()
+            assert np.array_equal(bc.cpu().numpy(), codes_g) and np.array_equal(bp.cpu().numpy(), packed_g)
         del w
 
 
