@@ -14,17 +14,22 @@
 //   y_j = a_j / s' (one packed multiply by a tabulated reciprocal) and q_j = RNE_sat(y_j)
 //   from the hardware E2M1 conversion (saturation included) converted back to f16; the
 //   residual q - y is one mixed f16/f32 subtract.  That is five lane operations per
-//   element and candidate.  With y within a relative 2^-21 of the exact quotient, every
-//   element's term differs from its exact-decision term by at most
-//   4 * 2^-21 y* |q* - y*| + 8 * 2^-42 y*^2 (also where a midpoint falls between y and
-//   y*), so by Cauchy-Schwarz the fast score is within
-//        4 * 2^-21 sqrt(A E*) + 8 * 2^-42 A + 13 * 2^-24 E*    (A = sum_j h_j a_j^2)
+//   element and candidate.  The tabulated reciprocal is correctly rounded, so y (one more
+//   rounding) is within a relative eps = 2^-23 (+ 2^-48) of the exact quotient y*, and
+//   every element's term differs from its exact-decision term by at most
+//   4 eps y* |q* - y*| + 8 eps^2 y*^2 (also where a midpoint falls between y and y*:
+//   both distances to the grid are then within eps y* of half the grid gap), so by
+//   Cauchy-Schwarz the fast score is within
+//        4 eps sqrt(A E*) + 8 eps^2 A + 13 * 2^-24 E*    (A = sum_j h_j a_j^2)
 //   of the exact score E*; in terms of the fast score E that is at most
-//   4.01 * 2^-21 sqrt(A E) + 33 * 2^-42 A + 13 * 2^-24 E.  When
-//        runner-up - best > 2^-18 E2 + 2^-17 sqrt(A E2) + 2^-35 A
+//   4.01 * 2^-23 sqrt(A E) + 33 * 2^-46 A + 13 * 2^-24 E.  When
+//        runner-up - best > 2^-18 E2 + 2^-19 sqrt(A E2) + 2^-35 A
 //   (more than the two errors together, with at least 2x slack on every term) and
 //   E2 >= 2^-36 A (so the bound grows slower than the score for every other candidate),
-//   the fast winner is the exact winner.
+//   the fast winner is the exact winner.  (A quotient below the normal range carries an
+//   absolute error of half a denormal unit instead; such an element rounds to zero under
+//   every candidate, and a group made only of them has scores within rounding of A under
+//   every candidate, which the 2^-18 E2 term sends to the exact rescoring.)
 //   Otherwise the group is "ambiguous" and the whole warp rescores it cooperatively with
 //   exact rounding decisions (16 lanes per candidate, one element each, a fixed
 //   pairwise shuffle tree per error: relative error <= 8 * 2^-24), applying the tie
@@ -127,12 +132,12 @@ __device__ __forceinline__ void load_group(const uint4* w, int64_t g, float pw, 
 
 // Per-block table of the candidate constants of every E4M3 code c (1..126), filled once
 // per CTA and stored pre-splatted for the packed arithmetic: x = y = s'^2 and
-// z = w = 1 / s' (fast reciprocal), with s' = l(c) * sgk in [2^-21, 2^-2], so both are
+// z = w = 1 / s' (correctly rounded), with s' = l(c) * sgk in [2^-21, 2^-2], so both are
 // normal numbers.  One 16-byte shared load per candidate replaces a decode, a multiply
 // and a reciprocal on the candidate's critical path.
 __device__ __forceinline__ float4 candidate_constants(uint32_t c, float sgk) {
   const float sp = __fmul_rn(e4m3_mag(c), sgk);
-  const float s2 = __fmul_rn(sp, sp), inv = c ? rcp_approx(sp) : 0.0f;
+  const float s2 = __fmul_rn(sp, sp), inv = c ? __frcp_rn(sp) : 0.0f;
   return make_float4(s2, s2, inv, inv);
 }
 
@@ -335,13 +340,13 @@ __device__ __forceinline__ float fast_mse(const Group& G, float4 t) {
 // Is the fast winner (fast score e1) certainly ahead of the runner-up (e2), given the
 // energy A = sum_j h_j a_j^2 of the group?  The test of the file comment, in units of e2
 // (no underflow or overflow for 2^-36 A <= e2 <= A-ish):
-//   g = (e2 - e1) / e2 - 2^-18 - 2^-35 A / e2 > 2^-17 sqrt(A / e2), tested on squares.
+//   g = (e2 - e1) / e2 - 2^-18 - 2^-35 A / e2 > 2^-19 sqrt(A / e2), tested on squares.
 // A zero, denormal or non-finite e2 makes the reciprocal infinite or NaN and g fails.
 __device__ __forceinline__ bool fast_winner_certain(float e1, float e2, float A) {
   const float r = rcp_approx(e2);
   const float ratio = __fmul_rn(A, r);
   const float g = __fsub_rn(__fsub_rn(__fmul_rn(__fsub_rn(e2, e1), r), 0x1p-18f), __fmul_rn(0x1p-35f, ratio));
-  const bool certain = g > 0.0f && __fmul_rn(g, g) > __fmul_rn(0x1p-34f, ratio);
+  const bool certain = g > 0.0f && __fmul_rn(g, g) > __fmul_rn(0x1p-38f, ratio);
   return certain && ratio <= 0x1p36f && A > 0.0f;
 }
 
