@@ -26,10 +26,12 @@
 //        runner-up - best > 2^-18 E2 + 2^-19 sqrt(A E2) + 2^-35 A
 //   (more than the two errors together, with at least 2x slack on every term) and
 //   E2 >= 2^-36 A (so the bound grows slower than the score for every other candidate),
-//   the fast winner is the exact winner.  (A quotient below the normal range carries an
-//   absolute error of half a denormal unit instead; such an element rounds to zero under
-//   every candidate, and a group made only of them has scores within rounding of A under
-//   every candidate, which the 2^-18 E2 term sends to the exact rescoring.)
+//   the fast winner is the exact winner; the kernel puts the upper bound
+//   (sum_j h_j) max_j a_j^2 in place of A, which only widens the margin.  (A quotient
+//   below the normal range carries an absolute error of half a denormal unit instead;
+//   such an element rounds to zero under every candidate, and a group made only of them
+//   has scores within rounding of A under every candidate, which the 2^-18 E2 term sends
+//   to the exact rescoring.)
 //   Otherwise the group is "ambiguous" and the whole warp rescores it cooperatively with
 //   exact rounding decisions (16 lanes per candidate, one element each, a fixed
 //   pairwise shuffle tree per error: relative error <= 8 * 2^-24), applying the tie
@@ -173,9 +175,13 @@ __device__ __forceinline__ float fast_score(const Group& G, const float2 (&hv2)[
   return __fmul_rn(t.x, __fadd_rn(t2.x, t2.y));
 }
 
+// Running best (e1, best) and runner-up e2 (e1 <= e2); branch-free: a select and three
+// min/max.  A tie with the best makes e2 = e1 (the margin test then fails); NaN scores
+// are ignored.
 __device__ __forceinline__ void keep_best(float e, int c, float& e1, float& e2, int& best) {
-  if (e < e1) { e2 = e1; e1 = e; best = c; }
-  else if (e < e2) { e2 = e; }
+  best = e < e1 ? c : best;
+  e2 = fminf(e2, fmaxf(e1, e));
+  e1 = fminf(e1, e);
 }
 
 // Scores the codes [a, b) two at a time (independent chains interleave).
@@ -193,12 +199,12 @@ __device__ __forceinline__ void score_range(const Group& G, const float2 (&hv2)[
   if (c < b) keep_best(fast_score(G, hv2, tab[c]), c, e1, e2, best);
 }
 
-// A = sum_j h_j a_j^2 of a group (scaled domain), the scale of the fast-score error bound.
-__device__ __forceinline__ float group_energy(const Group& G, const float2 (&hv2)[8]) {
-  float2 acc = make_float2(0.f, 0.f);
-#pragma unroll
-  for (int i = 0; i < 8; ++i) acc = __ffma2_rn(hv2[i], __fmul2_rn(G.a[i], G.a[i]), acc);
-  return __fadd_rn(acc.x, acc.y);
+// Upper bound of A = sum_j h_j a_j^2, the scale of the fast-score error bound:
+// (sum_j h_j) * max_j a_j^2.  Two multiplies instead of a pass over the group; a larger A
+// only widens the margin (the rounding of the bound, a relative 2^-20 at most, is far
+// inside the margin's 2x slack).
+__device__ __forceinline__ float energy_bound(float hsum, float amax_k) {
+  return __fmul_rn(hsum, __fmul_rn(amax_k, amax_k));
 }
 
 // tie rule of the search: smaller error, then smaller |shift|, then smaller shift
@@ -338,7 +344,7 @@ __device__ __forceinline__ float fast_mse(const Group& G, float4 t) {
 }
 
 // Is the fast winner (fast score e1) certainly ahead of the runner-up (e2), given the
-// energy A = sum_j h_j a_j^2 of the group?  The test of the file comment, in units of e2
+// energy A = sum_j h_j a_j^2 of the group (or an upper bound of it)?  The test of the file comment, in units of e2
 // (no underflow or overflow for 2^-36 A <= e2 <= A-ish):
 //   g = (e2 - e1) / e2 - 2^-18 - 2^-35 A / e2 > 2^-19 sqrt(A / e2), tested on squares.
 // A zero, denormal or non-finite e2 makes the reciprocal infinite or NaN and g fails.
@@ -373,11 +379,8 @@ __device__ __forceinline__ int fourover6_init_code(const Group& G, const uint4* 
   if (c4 == c6) return (int)c4;
   const float e4 = fast_mse(G, tab[c4]);
   const float e6 = fast_mse(G, tab[c6]);
-  float2 acc = make_float2(0.f, 0.f);
-#pragma unroll
-  for (int i = 0; i < 8; ++i) acc = __ffma2_rn(G.a[i], G.a[i], acc);
-  const float A = __fadd_rn(acc.x, acc.y);
-  if (fast_winner_certain(fminf(e4, e6), fmaxf(e4, e6), A)) return (int)(e6 < e4 ? c6 : c4);
+  if (fast_winner_certain(fminf(e4, e6), fmaxf(e4, e6), energy_bound(16.0f, amax_k)))
+    return (int)(e6 < e4 ? c6 : c4);
   return (int)fourover6_exact_pick(wg, pw, c4, c6, sgk);
 }
 
@@ -412,6 +415,7 @@ refine_kernel(const uint4* __restrict__ w, int64_t ld_w, const float* __restrict
   float2 hv2[8];
 #pragma unroll
   for (int j = 0; j < 8; ++j) hv2[j] = make_float2(1.0f, 1.0f);
+  float hsum = 16.0f;  // sum of the lane's 16 h values
 
   // (row, chunk) of unit u, advanced by warps_total units per step without a division
   const int row_step = (int)(warps_total / chunks);
@@ -437,20 +441,24 @@ refine_kernel(const uint4* __restrict__ w, int64_t ld_w, const float* __restrict
           hv2[2 * i] = make_float2(t.x, t.y);
           hv2[2 * i + 1] = make_float2(t.z, t.w);
         }
+        float2 s2 = __fadd2_rn(__fadd2_rn(hv2[0], hv2[1]), __fadd2_rn(hv2[2], hv2[3]));
+        s2 = __fadd2_rn(s2, __fadd2_rn(__fadd2_rn(hv2[4], hv2[5]), __fadd2_rn(hv2[6], hv2[7])));
+        hsum = __fadd_rn(s2.x, s2.y);
       }
     }
 
     Group G;
     int c0 = 1, lo = 1, hi = 1;
+    float amax_k = 0.0f;
     if (active) {
       load_group_at(w + wofs / 8, d.pw, G);
+      const uint32_t amax = group_abs_max_bits(make_uint4(G.wb[0], G.wb[1], G.wb[2], G.wb[3]),
+                                               make_uint4(G.wb[4], G.wb[5], G.wb[6], G.wb[7]));
+      amax_k = __fmul_rn(__uint_as_float(amax << 16), d.pw);
       if (!kFourOverSix && init_codes != nullptr) {
         c0 = init_codes[row * ld_i + gcol] & 0x7F;
         c0 = c0 < 1 ? 1 : (c0 > (int)kE4M3MaxCode ? (int)kE4M3MaxCode : c0);
       } else {
-        const uint32_t amax = group_abs_max_bits(make_uint4(G.wb[0], G.wb[1], G.wb[2], G.wb[3]),
-                                                 make_uint4(G.wb[4], G.wb[5], G.wb[6], G.wb[7]));
-        const float amax_k = __fmul_rn(__uint_as_float(amax << 16), d.pw);
         c0 = kFourOverSix ? fourover6_init_code(G, w + wofs / 8, tab, amax_k, d.sgk, d.pw, inv4, inv6)
                           : (int)rtn_code(amax_k, d.sgk, inv6);
       }
@@ -466,7 +474,7 @@ refine_kernel(const uint4* __restrict__ w, int64_t ld_w, const float* __restrict
 
     // ---- is the fast winner certain?
     bool ambiguous = false;
-    if (active && hi > lo) ambiguous = !fast_winner_certain(e1, e2, group_energy(G, hv2));
+    if (active && hi > lo) ambiguous = !fast_winner_certain(e1, e2, energy_bound(hsum, amax_k));
     unsigned amb = __ballot_sync(0xFFFFFFFFu, ambiguous);
     while (amb) {
       const int owner = __ffs(amb) - 1;
