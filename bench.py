@@ -431,8 +431,9 @@ SEARCH_BYTES = {"rtn": 41, "4over6": 41, "4over6-2pass": 42}
 
 
 def kernels_per_matrix(work: Work) -> int:
-    """Library kernels per matrix and step: amax, (4over6 codes,) refine."""
-    return 3 if work.init == "4over6-2pass" else 2
+    """Library kernels per matrix and step: amax and s_g (hscale_rtn_scales), the 4over6
+    codes with the two-pass init, the search."""
+    return 4 if work.init == "4over6-2pass" else 3
 
 
 def timed(fn, reps):
