@@ -2,9 +2,13 @@
 //
 //   factor            the damped inverse-Cholesky factor U of GPTQ: dead channels (H_jj = 0)
 //                     get H_jj = 1, the diagonal gets damp * mean(diag), and U is upper
-//                     triangular with U^T U = (H + damp I)^-1.  Cholesky and the inverse come
-//                     from cuSOLVER, loaded at run time (column-major: its lower factor of
-//                     (H + damp I)^-1 is our row-major U).
+//                     triangular with U^T U = (H + damp I)^-1 = A^-1.  It is formed without
+//                     A^-1: with J the order-reversing permutation and J A J = R^T R (R upper,
+//                     Cholesky), A = (J R^T J)(J R J), so U = (J R^T J)^-1 = J R^-T J, an
+//                     upper-triangular matrix with a positive diagonal, hence the Cholesky
+//                     factor.  cuSOLVER (loaded at run time) does the Cholesky and the
+//                     triangular inverse on column-major storage; reversing the row-major
+//                     array turns A into J A J, and column-major R^-1 into row-major U.
 //   block_kernel      one thread per 16-element group of a block of B columns of the running
 //                     fp32 weights: the RTN code (Eq. 7) of the current weights, the exact
 //                     H-Scale search over the window (Algorithm 1, exact E2M1 decisions, the
@@ -16,6 +20,7 @@
 #include <algorithm>
 #include <cstdio>
 #include <mutex>
+#include <vector>
 
 #include <cusolverDn.h>
 
@@ -31,8 +36,8 @@ struct Solver {
   decltype(&cusolverDnSetStream) set_stream = nullptr;
   decltype(&cusolverDnSpotrf_bufferSize) potrf_size = nullptr;
   decltype(&cusolverDnSpotrf) potrf = nullptr;
-  decltype(&cusolverDnSpotri_bufferSize) potri_size = nullptr;
-  decltype(&cusolverDnSpotri) potri = nullptr;
+  decltype(&cusolverDnXtrtri_bufferSize) trtri_size = nullptr;
+  decltype(&cusolverDnXtrtri) trtri = nullptr;
   bool ok = false;
 };
 
@@ -50,9 +55,9 @@ const Solver& solver() {
     s.set_stream = reinterpret_cast<decltype(s.set_stream)>(dlsym(lib, "cusolverDnSetStream"));
     s.potrf_size = reinterpret_cast<decltype(s.potrf_size)>(dlsym(lib, "cusolverDnSpotrf_bufferSize"));
     s.potrf = reinterpret_cast<decltype(s.potrf)>(dlsym(lib, "cusolverDnSpotrf"));
-    s.potri_size = reinterpret_cast<decltype(s.potri_size)>(dlsym(lib, "cusolverDnSpotri_bufferSize"));
-    s.potri = reinterpret_cast<decltype(s.potri)>(dlsym(lib, "cusolverDnSpotri"));
-    s.ok = s.create && s.set_stream && s.potrf_size && s.potrf && s.potri_size && s.potri;
+    s.trtri_size = reinterpret_cast<decltype(s.trtri_size)>(dlsym(lib, "cusolverDnXtrtri_bufferSize"));
+    s.trtri = reinterpret_cast<decltype(s.trtri)>(dlsym(lib, "cusolverDnXtrtri"));
+    s.ok = s.create && s.set_stream && s.potrf_size && s.potrf && s.trtri_size && s.trtri;
   });
   return s;
 }
@@ -90,12 +95,16 @@ __global__ void __launch_bounds__(1024) damp_diagonal_kernel(float* A, int64_t n
   for (int64_t j = threadIdx.x; j < n; j += blockDim.x) A[j * n + j] += add;
 }
 
-// row-major: A[r][c] = A[c][r] for r > c (mirror the upper triangle), or zero it (zero_lower)
-__global__ void __launch_bounds__(256) lower_kernel(float* A, int64_t n, int zero_lower) {
-  const int64_t total = n * n;
-  for (int64_t e = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; e < total; e += (int64_t)gridDim.x * blockDim.x) {
-    const int64_t r = e / n, c = e - r * n;
-    if (r > c) A[e] = zero_lower ? 0.0f : A[c * n + r];
+// Reverses the n*n array A in place (A[e] <-> A[n*n - 1 - e]: row-major A becomes J A J);
+// with zero_lower, entries that land below the diagonal are set to zero.
+__global__ void __launch_bounds__(256) reverse_kernel(float* A, int64_t n, int zero_lower) {
+  const int64_t total = n * n, half = total / 2;
+  for (int64_t e = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; e < half; e += (int64_t)gridDim.x * blockDim.x) {
+    const int64_t f = total - 1 - e;
+    const float a = A[e], b = A[f];
+    const int64_t re = e / n, rf = f / n;
+    A[e] = (zero_lower && re > e - re * n) ? 0.0f : b;
+    A[f] = (zero_lower && rf > f - rf * n) ? 0.0f : a;
   }
 }
 
@@ -247,12 +256,14 @@ bool gptq_solver_available() { return solver().ok && solver_handle() != nullptr;
 
 size_t gptq_factor_solver_floats(int64_t n) {
   if (!gptq_solver_available()) return 0;
-  int a = 0, b = 0;
+  int a = 0;
+  size_t dev_bytes = 0, host_bytes = 0;
   cusolverDnHandle_t hd = solver_handle();
-  if (solver().potrf_size(hd, CUBLAS_FILL_MODE_LOWER, (int)n, nullptr, (int)n, &a) != CUSOLVER_STATUS_SUCCESS ||
-      solver().potri_size(hd, CUBLAS_FILL_MODE_LOWER, (int)n, nullptr, (int)n, &b) != CUSOLVER_STATUS_SUCCESS)
+  if (solver().potrf_size(hd, CUBLAS_FILL_MODE_UPPER, (int)n, nullptr, (int)n, &a) != CUSOLVER_STATUS_SUCCESS ||
+      solver().trtri_size(hd, CUBLAS_FILL_MODE_UPPER, CUBLAS_DIAG_NON_UNIT, n, CUDA_R_32F, nullptr, n, &dev_bytes,
+                          &host_bytes) != CUSOLVER_STATUS_SUCCESS)
     return 0;
-  return (size_t)std::max(std::max(a, b), 1);
+  return std::max<size_t>(std::max<size_t>((size_t)a, (dev_bytes + 3) / 4), 1);
 }
 
 cudaError_t launch_gptq_factor(const float* H, int64_t n, int64_t ld_h, float damp, float* Uo, uint8_t* dead,
@@ -266,18 +277,28 @@ cudaError_t launch_gptq_factor(const float* H, int64_t n, int64_t ld_h, float da
   if (err != cudaSuccess) return err;
   damp_diagonal_kernel<<<1, 1024, 0, stream>>>(Uo, n, damp, dead);
   if ((err = cudaGetLastError()) != cudaSuccess) return err;
-  const int ni = (int)n, lw = (int)work_floats;
-  if (sv.potrf(hd, CUBLAS_FILL_MODE_LOWER, ni, Uo, ni, work, lw, info) != CUSOLVER_STATUS_SUCCESS) return cudaErrorUnknown;
-  if (sv.potri(hd, CUBLAS_FILL_MODE_LOWER, ni, Uo, ni, work, lw, info + 1) != CUSOLVER_STATUS_SUCCESS)
-    return cudaErrorUnknown;
   DeviceInfo dinfo;
   if ((err = current_device_info(&dinfo)) != cudaSuccess) return err;
-  const unsigned blocks = (unsigned)std::min<int64_t>((n * n + 255) / 256, (int64_t)dinfo.sm_count * 16);
-  lower_kernel<<<blocks, 256, 0, stream>>>(Uo, n, 0);
+  const unsigned blocks = (unsigned)std::max<int64_t>(1, std::min<int64_t>((n * n / 2 + 255) / 256,
+                                                                          (int64_t)dinfo.sm_count * 16));
+  // J A J; its row-major lower triangle (column-major upper) holds A's upper triangle
+  reverse_kernel<<<blocks, 256, 0, stream>>>(Uo, n, 0);
   if ((err = cudaGetLastError()) != cudaSuccess) return err;
-  if (sv.potrf(hd, CUBLAS_FILL_MODE_LOWER, ni, Uo, ni, work, lw, info + 2) != CUSOLVER_STATUS_SUCCESS)
+  if ((err = cudaMemsetAsync(info, 0, 3 * sizeof(int32_t), stream)) != cudaSuccess) return err;
+  const int ni = (int)n, lw = (int)std::min<size_t>(work_floats, (size_t)INT32_MAX);
+  if (sv.potrf(hd, CUBLAS_FILL_MODE_UPPER, ni, Uo, ni, work, lw, info) != CUSOLVER_STATUS_SUCCESS)
     return cudaErrorUnknown;
-  lower_kernel<<<blocks, 256, 0, stream>>>(Uo, n, 1);
+  size_t dev_bytes = 0, host_bytes = 0;
+  if (sv.trtri_size(hd, CUBLAS_FILL_MODE_UPPER, CUBLAS_DIAG_NON_UNIT, n, CUDA_R_32F, Uo, n, &dev_bytes,
+                    &host_bytes) != CUSOLVER_STATUS_SUCCESS || dev_bytes > work_floats * 4)
+    return cudaErrorUnknown;
+  static thread_local std::vector<char> host_work;
+  if (host_work.size() < host_bytes) host_work.resize(host_bytes);
+  if (sv.trtri(hd, CUBLAS_FILL_MODE_UPPER, CUBLAS_DIAG_NON_UNIT, n, CUDA_R_32F, Uo, n, work, dev_bytes,
+               host_bytes ? host_work.data() : nullptr, host_bytes, info + 1) != CUSOLVER_STATUS_SUCCESS)
+    return cudaErrorUnknown;
+  // column-major R^-1 (upper) reversed is row-major U; the other triangle is cleared
+  reverse_kernel<<<blocks, 256, 0, stream>>>(Uo, n, 1);
   return cudaGetLastError();
 }
 
