@@ -437,7 +437,9 @@ def kernels_per_matrix(work: Work) -> int:
 
 
 def timed(fn, reps):
-    """Average CUDA-event time (ms) of fn over reps calls on the current stream."""
+    """Average CUDA-event time (ms) of fn over reps calls on the current stream, after one
+    untimed call (library loading, handle creation and first-use costs stay out)."""
+    fn()
     e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
     e0.record()
     for _ in range(reps):

@@ -330,11 +330,13 @@ int hscale_output_error(const void* x_bf16, int64_t tokens, int64_t n, int64_t l
  *    zeroed in step 3) and get H_jj = 1; the diagonal gets damp * mean(diag H) (GPTQ uses
  *    damp = 0.01); U [n, n] (fp32, row stride n) is upper triangular with
  *    U^T U = (H + damp I)^-1, formed from the Cholesky factor of the reversed matrix and
- *    its triangular inverse (no explicit inverse).  Both come from cuSOLVER, loaded at run
- *    time: without it the call returns HSCALE_ERR_CUDA and the rest of the library is
- *    unaffected.  info is a device int32[3]: info[0] the status of the factorization
- *    (0 = success, > 0: not positive definite), info[1] that of the triangular inverse
- *    (> 0: a zero pivot), info[2] = 0.  n < 46341.
+ *    its triangular inverse (no explicit inverse of H).  cuSOLVER (Cholesky) and cuBLAS
+ *    (triangular solve) are loaded at run time: without them the call returns
+ *    HSCALE_ERR_CUDA and the rest of the library is unaffected.  info is a device int32[3]:
+ *    info[0] the status of the factorization (0 = success, > 0: not positive definite),
+ *    info[1] = info[2] = 0.  The workspace (hscale_gptq_factor_workspace_bytes, 256-byte
+ *    aligned) holds n^2 floats for the reversed matrix and its factor plus cuSOLVER's.
+ *    n < 46341.
  *
  * 3. hscale_gptq_hscale: for each block of `block` columns (a multiple of 16 dividing n)
  *    of the running fp32 weights (W with dead columns zeroed): the RTN codes of Eq. 7 of

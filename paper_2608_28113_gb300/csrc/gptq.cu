@@ -3,12 +3,13 @@
 //   factor            the damped inverse-Cholesky factor U of GPTQ: dead channels (H_jj = 0)
 //                     get H_jj = 1, the diagonal gets damp * mean(diag), and U is upper
 //                     triangular with U^T U = (H + damp I)^-1 = A^-1.  It is formed without
-//                     A^-1: with J the order-reversing permutation and J A J = R^T R (R upper,
-//                     Cholesky), A = (J R^T J)(J R J), so U = (J R^T J)^-1 = J R^-T J, an
+//                     A^-1: with J the order-reversing permutation and J A J = L L^T (L lower,
+//                     Cholesky), A = (J L J)(J L^T J), so U = (J L J)^-1 = J L^-1 J, an
 //                     upper-triangular matrix with a positive diagonal, hence the Cholesky
-//                     factor.  cuSOLVER (loaded at run time) does the Cholesky and the
-//                     triangular inverse on column-major storage; reversing the row-major
-//                     array turns A into J A J, and column-major R^-1 into row-major U.
+//                     factor.  cuSOLVER does the Cholesky and cuBLAS the triangular solve
+//                     L^T Y = I (both loaded at run time) on column-major storage: Y = L^-T
+//                     in column-major order is (J Y J)^T = U^T after reversing the array,
+//                     i.e. row-major U.
 //   block_kernel      one thread per 16-element group of a block of B columns of the running
 //                     fp32 weights: the RTN code (Eq. 7) of the current weights, the exact
 //                     H-Scale search over the window (Algorithm 1, exact E2M1 decisions, the
@@ -22,6 +23,7 @@
 #include <mutex>
 #include <vector>
 
+#include <cublas_v2.h>
 #include <cusolverDn.h>
 
 #include "hscale_device.cuh"
@@ -36,8 +38,9 @@ struct Solver {
   decltype(&cusolverDnSetStream) set_stream = nullptr;
   decltype(&cusolverDnSpotrf_bufferSize) potrf_size = nullptr;
   decltype(&cusolverDnSpotrf) potrf = nullptr;
-  decltype(&cusolverDnXtrtri_bufferSize) trtri_size = nullptr;
-  decltype(&cusolverDnXtrtri) trtri = nullptr;
+  decltype(&cublasCreate_v2) blas_create = nullptr;
+  decltype(&cublasSetStream_v2) blas_set_stream = nullptr;
+  decltype(&cublasStrsm_v2) trsm = nullptr;
   bool ok = false;
 };
 
@@ -55,14 +58,21 @@ const Solver& solver() {
     s.set_stream = reinterpret_cast<decltype(s.set_stream)>(dlsym(lib, "cusolverDnSetStream"));
     s.potrf_size = reinterpret_cast<decltype(s.potrf_size)>(dlsym(lib, "cusolverDnSpotrf_bufferSize"));
     s.potrf = reinterpret_cast<decltype(s.potrf)>(dlsym(lib, "cusolverDnSpotrf"));
-    s.trtri_size = reinterpret_cast<decltype(s.trtri_size)>(dlsym(lib, "cusolverDnXtrtri_bufferSize"));
-    s.trtri = reinterpret_cast<decltype(s.trtri)>(dlsym(lib, "cusolverDnXtrtri"));
-    s.ok = s.create && s.set_stream && s.potrf_size && s.potrf && s.trtri_size && s.trtri;
+    void* blas = nullptr;
+    for (const char* name : {"libcublas.so.13", "libcublas.so.12", "libcublas.so"}) {
+      blas = dlopen(name, RTLD_NOW | RTLD_LOCAL);
+      if (blas) break;
+    }
+    if (!blas) return;
+    s.blas_create = reinterpret_cast<decltype(s.blas_create)>(dlsym(blas, "cublasCreate_v2"));
+    s.blas_set_stream = reinterpret_cast<decltype(s.blas_set_stream)>(dlsym(blas, "cublasSetStream_v2"));
+    s.trsm = reinterpret_cast<decltype(s.trsm)>(dlsym(blas, "cublasStrsm_v2"));
+    s.ok = s.create && s.set_stream && s.potrf_size && s.potrf && s.blas_create && s.blas_set_stream && s.trsm;
   });
   return s;
 }
 
-// one handle per device, created on first use
+// one handle of each library per device, created on first use
 cusolverDnHandle_t solver_handle() {
   static std::mutex mu;
   static cusolverDnHandle_t handles[64] = {};
@@ -70,6 +80,16 @@ cusolverDnHandle_t solver_handle() {
   if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return nullptr;
   std::lock_guard<std::mutex> lock(mu);
   if (!handles[dev] && solver().create(&handles[dev]) != CUSOLVER_STATUS_SUCCESS) handles[dev] = nullptr;
+  return handles[dev];
+}
+
+cublasHandle_t blas_handle() {
+  static std::mutex mu;
+  static cublasHandle_t handles[64] = {};
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return nullptr;
+  std::lock_guard<std::mutex> lock(mu);
+  if (!handles[dev] && solver().blas_create(&handles[dev]) != CUBLAS_STATUS_SUCCESS) handles[dev] = nullptr;
   return handles[dev];
 }
 
@@ -95,16 +115,37 @@ __global__ void __launch_bounds__(1024) damp_diagonal_kernel(float* A, int64_t n
   for (int64_t j = threadIdx.x; j < n; j += blockDim.x) A[j * n + j] += add;
 }
 
-// Reverses the n*n array A in place (A[e] <-> A[n*n - 1 - e]: row-major A becomes J A J);
-// with zero_lower, entries that land below the diagonal are set to zero.
-__global__ void __launch_bounds__(256) reverse_kernel(float* A, int64_t n, int zero_lower) {
+// B[i][j] = A[p][q] with (p, q) = (n-1-i, n-1-j) taken in the upper triangle (p <= q) of
+// row-major A: B = J A J, complete and symmetric, from A's upper triangle.
+__global__ void __launch_bounds__(256) reverse_symmetric_kernel(const float* __restrict__ A, int64_t n,
+                                                                float* __restrict__ B) {
+  const int64_t total = n * n;
+  for (int64_t e = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; e < total; e += (int64_t)gridDim.x * blockDim.x) {
+    const int64_t i = e / n, j = e - i * n;
+    const int64_t p = n - 1 - i, q = n - 1 - j;
+    B[e] = p <= q ? A[p * n + q] : A[q * n + p];
+  }
+}
+
+// Reverses the n*n array A in place (A[e] <-> A[n*n - 1 - e]) and zeroes what lands below
+// the diagonal of row-major A.
+__global__ void __launch_bounds__(256) reverse_upper_kernel(float* A, int64_t n) {
   const int64_t total = n * n, half = total / 2;
   for (int64_t e = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; e < half; e += (int64_t)gridDim.x * blockDim.x) {
     const int64_t f = total - 1 - e;
     const float a = A[e], b = A[f];
     const int64_t re = e / n, rf = f / n;
-    A[e] = (zero_lower && re > e - re * n) ? 0.0f : b;
-    A[f] = (zero_lower && rf > f - rf * n) ? 0.0f : a;
+    A[e] = re > e - re * n ? 0.0f : b;
+    A[f] = rf > f - rf * n ? 0.0f : a;
+  }
+}
+
+// the n x n identity
+__global__ void __launch_bounds__(256) identity_kernel(float* X, int64_t n) {
+  const int64_t total = n * n;
+  for (int64_t e = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; e < total; e += (int64_t)gridDim.x * blockDim.x) {
+    const int64_t r = e / n;
+    X[e] = (e - r * n == r) ? 1.0f : 0.0f;
   }
 }
 
@@ -252,18 +293,17 @@ __global__ void __launch_bounds__(256) to_fp32_kernel(const uint16_t* __restrict
 }  // namespace
 
 // ---------------------------------------------------------------- host side
-bool gptq_solver_available() { return solver().ok && solver_handle() != nullptr; }
+bool gptq_solver_available() { return solver().ok && solver_handle() != nullptr && blas_handle() != nullptr; }
 
+// The factor's workspace in floats: J A J and its Cholesky factor (n*n, rounded up to 64
+// floats), then cuSOLVER's.
 size_t gptq_factor_solver_floats(int64_t n) {
   if (!gptq_solver_available()) return 0;
   int a = 0;
-  size_t dev_bytes = 0, host_bytes = 0;
-  cusolverDnHandle_t hd = solver_handle();
-  if (solver().potrf_size(hd, CUBLAS_FILL_MODE_UPPER, (int)n, nullptr, (int)n, &a) != CUSOLVER_STATUS_SUCCESS ||
-      solver().trtri_size(hd, CUBLAS_FILL_MODE_UPPER, CUBLAS_DIAG_NON_UNIT, n, CUDA_R_32F, nullptr, n, &dev_bytes,
-                          &host_bytes) != CUSOLVER_STATUS_SUCCESS)
+  if (solver().potrf_size(solver_handle(), CUBLAS_FILL_MODE_LOWER, (int)n, nullptr, (int)n, &a) !=
+      CUSOLVER_STATUS_SUCCESS)
     return 0;
-  return std::max<size_t>(std::max<size_t>((size_t)a, (dev_bytes + 3) / 4), 1);
+  return ((size_t)n * (size_t)n + 63) / 64 * 64 + std::max(a, 1);
 }
 
 cudaError_t launch_gptq_factor(const float* H, int64_t n, int64_t ld_h, float damp, float* Uo, uint8_t* dead,
@@ -271,7 +311,13 @@ cudaError_t launch_gptq_factor(const float* H, int64_t n, int64_t ld_h, float da
   if (!gptq_solver_available()) return cudaErrorNotSupported;
   const Solver& sv = solver();
   cusolverDnHandle_t hd = solver_handle();
-  if (sv.set_stream(hd, stream) != CUSOLVER_STATUS_SUCCESS) return cudaErrorUnknown;
+  cublasHandle_t hb = blas_handle();
+  if (sv.set_stream(hd, stream) != CUSOLVER_STATUS_SUCCESS || sv.blas_set_stream(hb, stream) != CUBLAS_STATUS_SUCCESS)
+    return cudaErrorUnknown;
+  const size_t x_floats = ((size_t)n * (size_t)n + 63) / 64 * 64;
+  if (work_floats <= x_floats) return cudaErrorInvalidValue;
+  float* X = work;
+  float* solver_work = work + x_floats;
   cudaError_t err = cudaMemcpy2DAsync(Uo, (size_t)n * 4, H, (size_t)ld_h * 4, (size_t)n * 4, (size_t)n,
                                       cudaMemcpyDeviceToDevice, stream);
   if (err != cudaSuccess) return err;
@@ -279,26 +325,24 @@ cudaError_t launch_gptq_factor(const float* H, int64_t n, int64_t ld_h, float da
   if ((err = cudaGetLastError()) != cudaSuccess) return err;
   DeviceInfo dinfo;
   if ((err = current_device_info(&dinfo)) != cudaSuccess) return err;
-  const unsigned blocks = (unsigned)std::max<int64_t>(1, std::min<int64_t>((n * n / 2 + 255) / 256,
+  const unsigned blocks = (unsigned)std::max<int64_t>(1, std::min<int64_t>((n * n + 255) / 256,
                                                                           (int64_t)dinfo.sm_count * 16));
-  // J A J; its row-major lower triangle (column-major upper) holds A's upper triangle
-  reverse_kernel<<<blocks, 256, 0, stream>>>(Uo, n, 0);
+  // X = J A J, symmetric, from the upper triangle of the damped copy
+  reverse_symmetric_kernel<<<blocks, 256, 0, stream>>>(Uo, n, X);
   if ((err = cudaGetLastError()) != cudaSuccess) return err;
   if ((err = cudaMemsetAsync(info, 0, 3 * sizeof(int32_t), stream)) != cudaSuccess) return err;
-  const int ni = (int)n, lw = (int)std::min<size_t>(work_floats, (size_t)INT32_MAX);
-  if (sv.potrf(hd, CUBLAS_FILL_MODE_UPPER, ni, Uo, ni, work, lw, info) != CUSOLVER_STATUS_SUCCESS)
+  const int ni = (int)n, lw = (int)std::min<size_t>(work_floats - x_floats, (size_t)INT32_MAX);
+  if (sv.potrf(hd, CUBLAS_FILL_MODE_LOWER, ni, X, ni, solver_work, lw, info) != CUSOLVER_STATUS_SUCCESS)
     return cudaErrorUnknown;
-  size_t dev_bytes = 0, host_bytes = 0;
-  if (sv.trtri_size(hd, CUBLAS_FILL_MODE_UPPER, CUBLAS_DIAG_NON_UNIT, n, CUDA_R_32F, Uo, n, &dev_bytes,
-                    &host_bytes) != CUSOLVER_STATUS_SUCCESS || dev_bytes > work_floats * 4)
+  // L^T Y = I: Y = L^-T (upper, column-major) in U's buffer
+  identity_kernel<<<blocks, 256, 0, stream>>>(Uo, n);
+  if ((err = cudaGetLastError()) != cudaSuccess) return err;
+  const float one = 1.0f;
+  if (sv.trsm(hb, CUBLAS_SIDE_LEFT, CUBLAS_FILL_MODE_LOWER, CUBLAS_OP_T, CUBLAS_DIAG_NON_UNIT, ni, ni, &one, X, ni,
+              Uo, ni) != CUBLAS_STATUS_SUCCESS)
     return cudaErrorUnknown;
-  static thread_local std::vector<char> host_work;
-  if (host_work.size() < host_bytes) host_work.resize(host_bytes);
-  if (sv.trtri(hd, CUBLAS_FILL_MODE_UPPER, CUBLAS_DIAG_NON_UNIT, n, CUDA_R_32F, Uo, n, work, dev_bytes,
-               host_bytes ? host_work.data() : nullptr, host_bytes, info + 1) != CUSOLVER_STATUS_SUCCESS)
-    return cudaErrorUnknown;
-  // column-major R^-1 (upper) reversed is row-major U; the other triangle is cleared
-  reverse_kernel<<<blocks, 256, 0, stream>>>(Uo, n, 1);
+  // reversed, column-major Y is row-major U; the other triangle is cleared
+  reverse_upper_kernel<<<blocks, 256, 0, stream>>>(Uo, n);
   return cudaGetLastError();
 }
 
