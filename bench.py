@@ -275,12 +275,37 @@ class Work:
         self.spaces = {name: Space(W, name, n, self.seed, device, tokens) for name, n in W.input_spaces()}
         self.mats = [Matrix(W, L, self.spaces[L.input_space], self.seed, device) for L in W.layers]
         self.groups = sum(M.groups for M in self.mats)
-        # pieces of the step in order: (space, c0, c1)
-        self.pieces = [(S, c0, c1) for S in self.spaces.values() for c0, c1 in column_blocks(S, col_block)]
+        # pieces of the step in order: (space, c0, c1), spaces in flow-shop order
+        self.pieces = [(S, c0, c1) for S in self.space_order() for c0, c1 in column_blocks(S, col_block)]
         calls = [(c1 - c0, t1 - t0) for S, c0, c1 in self.pieces for t0, t1 in hessian_calls(S, c0, c1)]
         self.h_bytes = sum(2 * rows * width + 8 * width for width, rows in calls)
         self.h_launches = len(calls)
         self.ws = None
+
+    def space_order(self):
+        """The input spaces in the order the step takes them.  Each space is a two-stage
+        job: its Hessian pass (HBM-bound, about 2 bytes per token and channel) and then the
+        searches of its matrices (ALU-bound, about 80 operations per group and candidate);
+        the searches of one space run alongside the Hessian passes of the next, so
+        Johnson's rule on estimated stage times keeps both streams busy.  The estimates
+        use nominal rates (6.6 TB/s; 0.45 of 40 T lane operations per second); only their
+        ratio matters."""
+        cands = self.win[0] + self.win[1] + 1
+        jobs = []
+        for S in self.spaces.values():
+            a = 2.0 * S.tokens * S.n / 6.6e12
+            b = sum(M.groups for M in self.mats if M.space is S) * 80.0 * cands / (0.45 * 40.3e12)
+            jobs.append((S.name, a, b))
+        return [self.spaces[name] for name in johnson_order(jobs)]
+
+
+def johnson_order(jobs):
+    """Order of two-stage jobs (name, a, b) -- stage 1 (time a) before stage 2 (time b), one
+    machine per stage -- that minimises the makespan (Johnson's rule): jobs with a <= b
+    first, by increasing a; then the others, by decreasing b."""
+    first = sorted((j for j in jobs if j[1] <= j[2]), key=lambda j: j[1])
+    last = sorted((j for j in jobs if j[1] > j[2]), key=lambda j: -j[2])
+    return [j[0] for j in first + last]
 
 
 def hessian_block(hs, S: Space, c0: int, c1: int):
