@@ -341,7 +341,8 @@ int hscale_output_error(const void* x_bf16, int64_t tokens, int64_t n, int64_t l
  * 3. hscale_gptq_hscale: for each block of `block` columns (a multiple of 16 dividing n)
  *    of the running fp32 weights (W with dead columns zeroed): the RTN codes of Eq. 7 of
  *    the current block weights, the H-Scale search over the window (down, up) with the
- *    diagonal proxy h [n] (16-byte aligned) and the global scale s_g of the original W,
+ *    diagonal proxy h [n] (16-byte aligned) and the global scale s_g of the original W
+ *    (U as written by hscale_gptq_factor, 16-byte aligned),
  *    with exact E2M1 decisions and the tie rule of hscale_refine_scales; then
  *    E = (W_b - W_hat_b) / diag(U_b) and W[:, i+B:] -= E U[i:i+B, i+B:] in fp32.  Writes
  *    codes_out [m, n/16] and packed_out [m, n/2] (8-byte aligned) as hscale_refine_scales

@@ -277,7 +277,7 @@ int hscale_gptq_hscale(const void* w_bf16, int64_t m, int64_t n, const float* U,
   if (m == 0 || n == 0) return HSCALE_OK;
   if (U == nullptr || h == nullptr || global_scale == nullptr || codes_out == nullptr || packed_out == nullptr)
     return HSCALE_ERR_NULL;
-  if (!aligned(U, 4) || !aligned(h, 16) || !aligned(global_scale, 4) || !aligned(packed_out, 8))
+  if (!aligned(U, 16) || !aligned(h, 16) || !aligned(global_scale, 4) || !aligned(packed_out, 8))
     return HSCALE_ERR_ALIGN;
   if (workspace == nullptr || workspace_bytes < hscale_gptq_workspace_bytes(m, n, block) || !aligned(workspace, 256))
     return HSCALE_ERR_WORKSPACE;

@@ -232,51 +232,103 @@ __global__ void __launch_bounds__(128) block_kernel(const float* __restrict__ W,
 }
 
 // W[r, c1 + c] -= sum_k E[r, k] U[col0 + k, c1 + c], k < B; 128 x 128 tiles, 8 x 8 per thread
+// W[:, c1:] -= E U[col0:c1, c1:] (c1 = col0 + B) in fp32: 128 x 128 output tiles, 256
+// threads with 8 rows x 8 columns each (columns 4*tc..4*tc+3 and 64+4*tc..64+4*tc+3, so
+// the 128-bit shared loads of a quarter warp are contiguous), k-slices of 8 staged in shared
+// memory with the next slice prefetched into registers.  E is stored pre-splatted (each
+// value twice) so that one packed FMA updates two columns of a row: every accumulator is
+// still a chain of scalar-rounded FMAs in k order.
 constexpr int kUT = 128, kUK = 8;
-__global__ void __launch_bounds__(256) update_kernel(float* __restrict__ W, int64_t m, int64_t n, int64_t col0, int B,
+__global__ void __launch_bounds__(256, 2) update_kernel(float* __restrict__ W, int64_t m, int64_t n, int64_t col0, int B,
                                                      const float* __restrict__ E, const float* __restrict__ U) {
-  __shared__ float As[kUK][kUT];
-  __shared__ float Bs[kUK][kUT];
+  __shared__ __align__(16) float2 As[2][kUK][kUT];
+  __shared__ __align__(16) float Bs[2][kUK][kUT];
   const int64_t c1 = col0 + B;
   const int64_t row0 = (int64_t)blockIdx.y * kUT, cb = c1 + (int64_t)blockIdx.x * kUT;
-  const int tr = threadIdx.x / 16, tc = threadIdx.x % 16;
-  float acc[8][8];
+  const int tid = threadIdx.x, tr = tid / 16, tc = tid % 16;
+  // global -> register staging: E row ar, k-quad aq; U k-row bk, column quad bq
+  const int ar = tid / 2, aq = (tid % 2) * 4;
+  const int bk = tid / 32, bq = (tid % 32) * 4;
+  const int64_t arow = row0 + ar, bcol = cb + bq;
+  auto load_a = [&](int k0) -> float4 {
+    if (arow >= m) return make_float4(0.f, 0.f, 0.f, 0.f);
+    return *reinterpret_cast<const float4*>(E + arow * B + k0 + aq);
+  };
+  auto load_b = [&](int k0) -> float4 {
+    const float* src = U + (col0 + k0 + bk) * n;
+    if (bcol + 3 < n) return *reinterpret_cast<const float4*>(src + bcol);
+    float4 v = make_float4(0.f, 0.f, 0.f, 0.f);
+    if (bcol + 0 < n) v.x = src[bcol + 0];
+    if (bcol + 1 < n) v.y = src[bcol + 1];
+    if (bcol + 2 < n) v.z = src[bcol + 2];
+    return v;
+  };
+  auto store = [&](int buf, float4 a, float4 b) {
+    As[buf][aq + 0][ar] = make_float2(a.x, a.x);
+    As[buf][aq + 1][ar] = make_float2(a.y, a.y);
+    As[buf][aq + 2][ar] = make_float2(a.z, a.z);
+    As[buf][aq + 3][ar] = make_float2(a.w, a.w);
+    *reinterpret_cast<float4*>(&Bs[buf][bk][bq]) = b;
+  };
+  float2 acc[8][4];
 #pragma unroll
   for (int i = 0; i < 8; ++i)
 #pragma unroll
-    for (int j = 0; j < 8; ++j) acc[i][j] = 0.0f;
+    for (int j = 0; j < 4; ++j) acc[i][j] = make_float2(0.f, 0.f);
+
+  store(0, load_a(0), load_b(0));
+  __syncthreads();
+  int buf = 0;
   for (int k0 = 0; k0 < B; k0 += kUK) {
-    for (int e = threadIdx.x; e < kUK * kUT; e += 256) {
-      const int kk = e % kUK, rr = e / kUK;
-      const int64_t row = row0 + rr;
-      As[kk][rr] = row < m ? E[row * B + k0 + kk] : 0.0f;
-      const int cc = e % kUT, kb = e / kUT;
-      const int64_t col = cb + cc;
-      Bs[kb][cc] = col < n ? U[(col0 + k0 + kb) * n + col] : 0.0f;
+    const bool more = k0 + kUK < B;
+    float4 na = make_float4(0.f, 0.f, 0.f, 0.f), nb = na;
+    if (more) {
+      na = load_a(k0 + kUK);
+      nb = load_b(k0 + kUK);
     }
-    __syncthreads();
 #pragma unroll
     for (int kk = 0; kk < kUK; ++kk) {
-      float av[8], bv[8];
+      float2 av[8];
+      const float4* ap = reinterpret_cast<const float4*>(&As[buf][kk][tr * 8]);
 #pragma unroll
-      for (int i = 0; i < 8; ++i) av[i] = As[kk][tr * 8 + i];
-#pragma unroll
-      for (int j = 0; j < 8; ++j) bv[j] = Bs[kk][tc * 8 + j];
+      for (int i = 0; i < 4; ++i) {
+        const float4 t = ap[i];
+        av[2 * i] = make_float2(t.x, t.y);
+        av[2 * i + 1] = make_float2(t.z, t.w);
+      }
+      const float4 b0 = *reinterpret_cast<const float4*>(&Bs[buf][kk][tc * 4]);
+      const float4 b1 = *reinterpret_cast<const float4*>(&Bs[buf][kk][64 + tc * 4]);
+      const float2 bv[4] = {make_float2(b0.x, b0.y), make_float2(b0.z, b0.w), make_float2(b1.x, b1.y),
+                            make_float2(b1.z, b1.w)};
 #pragma unroll
       for (int i = 0; i < 8; ++i)
 #pragma unroll
-        for (int j = 0; j < 8; ++j) acc[i][j] = __fmaf_rn(av[i], bv[j], acc[i][j]);
+        for (int j = 0; j < 4; ++j) acc[i][j] = __ffma2_rn(av[i], bv[j], acc[i][j]);
     }
-    __syncthreads();
+    if (more) {
+      store(buf ^ 1, na, nb);
+      __syncthreads();
+      buf ^= 1;
+    }
   }
 #pragma unroll
   for (int i = 0; i < 8; ++i) {
     const int64_t row = row0 + tr * 8 + i;
     if (row >= m) continue;
 #pragma unroll
-    for (int j = 0; j < 8; ++j) {
-      const int64_t col = cb + tc * 8 + j;
-      if (col < n) W[row * n + col] -= acc[i][j];
+    for (int half = 0; half < 2; ++half) {
+      const int64_t col = cb + half * 64 + tc * 4;
+      float* dst = W + row * n + col;
+      const float2 lo = acc[i][2 * half], hi = acc[i][2 * half + 1];
+      if (col + 3 < n) {
+        float4 v = *reinterpret_cast<float4*>(dst);
+        v.x -= lo.x; v.y -= lo.y; v.z -= hi.x; v.w -= hi.y;
+        *reinterpret_cast<float4*>(dst) = v;
+      } else {
+        if (col + 0 < n) dst[0] -= lo.x;
+        if (col + 1 < n) dst[1] -= lo.y;
+        if (col + 2 < n) dst[2] -= hi.x;
+      }
     }
   }
 }
