@@ -8,7 +8,9 @@
 //                         operands, fp32 accumulation in tensor memory), fused with the sum of
 //                         squares of C: one fp64 partial per 128 x 256 tile of C
 //   reduce_kernel         the partials summed in tile order, added to the caller's scalar
-//   transpose_kernel      X [tokens, n] -> X^T [n, tokens] (tokens contiguous per channel)
+//   transpose64_kernel    X [tokens, n] -> X^T [n, tokens] (tokens contiguous per channel),
+//                         16-byte accesses; transpose_kernel is the 2-byte form for X
+//                         whose rows are not 16-byte aligned
 //   gemm_kernel<true>     H += X^T X, the full Hessian of Algorithm 3, with the same tensor-
 //                         core pipeline over K = tokens and an epilogue that adds each
 //                         128 x 256 tile of the product into H; tiles wholly below the
@@ -297,6 +299,56 @@ __global__ void __launch_bounds__(256) transpose_kernel(const uint16_t* __restri
   }
 }
 
+// The same transpose with 16-byte accesses on both sides, for X with 16-byte aligned rows:
+// a 64-token x 64-channel tile per CTA.  Each thread loads 8 channels of two consecutive
+// tokens, pairs them into eight 32-bit words (token t low, t + 1 high) with byte permutes,
+// and stores the words transposed into shared memory (64 channel rows x 32 words, 16-byte
+// word groups XOR-swizzled by the channel octet so that neither side has bank conflicts);
+// then each thread writes two 16-byte runs of 8 tokens of one channel.
+__global__ void __launch_bounds__(256) transpose64_kernel(const uint16_t* __restrict__ x, int64_t tokens, int64_t n,
+                                                          int64_t ld_x, uint16_t* __restrict__ xt, int64_t ld_t) {
+  __shared__ __align__(16) uint32_t tile[64 * 32];
+  const int64_t t0 = (int64_t)blockIdx.x * 64, c0 = (int64_t)blockIdx.y * 64;
+  const int tid = threadIdx.x;
+  {
+    const int p = tid >> 3, g = tid & 7;
+    const int64_t t = t0 + 2 * p, c = c0 + 8 * g;
+    uint4 va = make_uint4(0u, 0u, 0u, 0u), vb = va;
+    if (c + 8 <= n) {
+      if (t < tokens) va = *reinterpret_cast<const uint4*>(x + t * ld_x + c);
+      if (t + 1 < tokens) vb = *reinterpret_cast<const uint4*>(x + (t + 1) * ld_x + c);
+    } else if (c < n) {
+      uint16_t ea[8] = {0, 0, 0, 0, 0, 0, 0, 0}, eb[8] = {0, 0, 0, 0, 0, 0, 0, 0};
+      for (int j = 0; j < 8 && c + j < n; ++j) {
+        if (t < tokens) ea[j] = x[t * ld_x + c + j];
+        if (t + 1 < tokens) eb[j] = x[(t + 1) * ld_x + c + j];
+      }
+      va = make_uint4(ea[0] | (uint32_t)ea[1] << 16, ea[2] | (uint32_t)ea[3] << 16, ea[4] | (uint32_t)ea[5] << 16,
+                      ea[6] | (uint32_t)ea[7] << 16);
+      vb = make_uint4(eb[0] | (uint32_t)eb[1] << 16, eb[2] | (uint32_t)eb[3] << 16, eb[4] | (uint32_t)eb[5] << 16,
+                      eb[6] | (uint32_t)eb[7] << 16);
+    }
+    const uint32_t a[4] = {va.x, va.y, va.z, va.w}, b[4] = {vb.x, vb.y, vb.z, vb.w};
+    const int col = (((p >> 2) ^ g) << 2) | (p & 3);
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {
+      tile[(8 * g + 2 * i) * 32 + col] = __byte_perm(a[i], b[i], 0x5410);
+      tile[(8 * g + 2 * i + 1) * 32 + col] = __byte_perm(a[i], b[i], 0x7632);
+    }
+  }
+  __syncthreads();
+#pragma unroll
+  for (int it = 0; it < 2; ++it) {
+    const int item = tid + 256 * it;
+    const int c = item >> 3, q = item & 7;
+    const int64_t cg = c0 + c, tg = t0 + 8 * q;
+    if (cg < n && tg < tokens) {
+      const uint4 v = *reinterpret_cast<const uint4*>(&tile[c * 32 + ((q ^ ((c >> 3) & 7)) << 2)]);
+      *reinterpret_cast<uint4*>(xt + cg * ld_t + tg) = v;
+    }
+  }
+}
+
 // The partials summed in index order by one block (fixed tree), added to *out.
 __global__ void __launch_bounds__(256) reduce_kernel(const double* __restrict__ partials, int64_t count,
                                                      double* __restrict__ out) {
@@ -380,9 +432,15 @@ int64_t hessian_full_ld(int64_t tokens) { return (tokens + 7) / 8 * 8; }
 cudaError_t launch_hessian_full(const void* x, int64_t tokens, int64_t n, int64_t ld_x, float* H, int64_t ld_h,
                                 void* xt, cudaStream_t stream) {
   const int64_t ld_t = hessian_full_ld(tokens);
-  const dim3 tgrid((unsigned)((tokens + 31) / 32), (unsigned)((n + 31) / 32));
-  transpose_kernel<<<tgrid, 256, 0, stream>>>(static_cast<const uint16_t*>(x), tokens, n, ld_x,
-                                              static_cast<uint16_t*>(xt), ld_t);
+  if ((reinterpret_cast<uintptr_t>(x) & 15) == 0 && ld_x % 8 == 0) {
+    const dim3 tgrid((unsigned)((tokens + 63) / 64), (unsigned)((n + 63) / 64));
+    transpose64_kernel<<<tgrid, 256, 0, stream>>>(static_cast<const uint16_t*>(x), tokens, n, ld_x,
+                                                  static_cast<uint16_t*>(xt), ld_t);
+  } else {
+    const dim3 tgrid((unsigned)((tokens + 31) / 32), (unsigned)((n + 31) / 32));
+    transpose_kernel<<<tgrid, 256, 0, stream>>>(static_cast<const uint16_t*>(x), tokens, n, ld_x,
+                                                static_cast<uint16_t*>(xt), ld_t);
+  }
   cudaError_t err = cudaGetLastError();
   if (err != cudaSuccess) return err;
   EncodeTiledFn encode = nullptr;

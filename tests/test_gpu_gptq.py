@@ -51,11 +51,21 @@ def oracle_H(x, n):
     return H
 
 
-@pytest.mark.parametrize("tokens,n,chunks", [(128, 256, 1), (300, 200, 1), (1000, 520, 2)])
-def test_full_hessian_matches_oracle(tokens, n, chunks):
+@pytest.mark.parametrize("tokens,n,chunks,view", [(128, 256, 1, "whole"), (300, 200, 1, "whole"),
+                                                  (1000, 520, 2, "whole"), (77, 131, 1, "whole"),
+                                                  (200, 96, 2, "aligned slice"), (150, 72, 1, "odd slice")])
+def test_full_hessian_matches_oracle(tokens, n, chunks, view):
+    """Whole X, a ragged width (n % 8 != 0), a 16-byte aligned column slice of a wider X
+    (ld_x > n) and a slice starting at an odd column (the 2-byte transpose path)."""
     x = calib(n, tokens, 60 + n)
     ref = oracle_H(x, n)
-    xd = x.to(dev())
+    if view == "whole":
+        xd = x.to(dev())
+    else:
+        off = 8 if view == "aligned slice" else 1
+        wide = torch.zeros(tokens, n + 24, dtype=torch.bfloat16, device=dev())
+        wide[:, off:off + n] = x.to(dev())
+        xd = wide[:, off:off + n]
     H = torch.zeros(n, n, dtype=torch.float32, device=dev())
     step = (tokens + chunks - 1) // chunks
     for t0 in range(0, tokens, step):
