@@ -589,6 +589,53 @@ def test_strided_row_slice_and_no_packed_output():
     assert np.array_equal(c2.cpu().numpy(), codes)
 
 
+# ------------------------------------------------------------------ offsets past 2^31 elements
+
+def test_search_and_hessian_beyond_2_31_elements():
+    """W and X of 65600 x 32768 bf16 (2.15e9 elements, 4.3 GB each): element offsets past
+    2^31.  s_g against an exact maximum on the device; RTN codes, searched codes and nibbles
+    of rows on both sides of the 2^31 boundary against the oracle; h of sampled channels
+    against the oracle."""
+    m, n = 65600, 32768
+    assert m * n > 2 ** 31
+    W = torch.empty(m, n, dtype=torch.bfloat16, device=dev())
+    step = 4096
+    for r0 in range(0, m, step):
+        W[r0:r0 + step] = wl.weight(min(step, m - r0), n, 0.02, 900 + r0 // step, device=dev())
+    sg, rtn = gpu_rtn(W)
+    amax_bits = int((W.view(torch.int16) & 0x7FFF).max().item())
+    amax = float(np.array([amax_bits << 16], dtype=np.uint32).view(np.float32)[0])
+    s_ref = np.float32(amax / 2688.0)
+    assert sg.cpu().numpy()[0] == s_ref
+    h32 = (wl.channel_magnitudes(n, 1.0, 32, 50.0, 77).numpy().astype(np.float64) ** 2 * 1000.0).astype(np.float32)
+    hd = torch.from_numpy(h32).to(dev())
+    codes = torch.empty(m, n // 16, dtype=torch.uint8, device=dev())
+    packed = torch.empty(m, n // 2, dtype=torch.uint8, device=dev())
+    hs.hscale_refine_scales(W, hd, sg, None, 4, 4, codes, packed)
+    torch.cuda.synchronize()
+    rows = np.array([0, 65535, 65536, 65537, m - 2, m - 1])  # row 65536 starts at element 2^31
+    wb = bits(W[torch.from_numpy(rows).to(dev())])
+    assert np.array_equal(rtn[torch.from_numpy(rows).to(dev())].cpu().numpy(), oracle.rtn_codes(wb, s_ref))
+    ref = oracle.refine(wb, h32, s_ref, None, 4, 4)
+    compare_search(ref, codes[torch.from_numpy(rows).to(dev())].cpu().numpy(),
+                   packed[torch.from_numpy(rows).to(dev())].cpu().numpy(), "rows across the 2^31 element offset")
+    del W, codes, packed, rtn
+    torch.cuda.empty_cache()
+    X = torch.empty(m, n, dtype=torch.bfloat16, device=dev())
+    a = wl.channel_magnitudes(n, 1.0, 32, 50.0, 78, device=dev())
+    for r0 in range(0, m, step):
+        wl.activation_chunk(min(step, m - r0), a, 78, r0 // step, out=X[r0:r0 + step])
+    h = torch.zeros(n, device=dev())
+    hs.hscale_hessian_diag_accumulate(X, h)
+    torch.cuda.synchronize()
+    cols = torch.tensor([0, 1, 4095, 16384, n - 2, n - 1], device=dev())
+    href = np.zeros(cols.numel())
+    oracle.hessian_accumulate(bits(X[:, cols].contiguous()), href)
+    err = assert_h_close(h[cols].cpu().numpy(), href)
+    print(f"[parity] 65600 x 32768 (2.15e9 elements): h max rel err {err:.3e} on sampled channels")
+    del X
+
+
 # ------------------------------------------------------------------ output error (Eq. 3)
 
 def oracle_codes_packed(wb, h32, s_ref, window):
