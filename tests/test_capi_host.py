@@ -45,6 +45,37 @@ def test_library_exports_every_declared_symbol(lib):
     assert hs.library_path().exists()
 
 
+def test_header_is_plain_c_and_every_symbol_links(lib, tmp_path):
+    """include/hscale.h compiles as strict C99, and a C program that takes the address of
+    every declared entry point links against the in-tree library and runs (host-only
+    calls: the ABI version, a status string, an argument error)."""
+    import shutil
+    import subprocess
+    cc = shutil.which("gcc") or shutil.which("cc")
+    if cc is None:
+        pytest.skip("no C compiler")
+    names = declared_functions()
+    src = tmp_path / "abi_check.c"
+    src.write_text(
+        "#include <stdio.h>\n#include \"hscale.h\"\n"
+        "typedef void (*fn_t)(void);\n"
+        "static const fn_t every[] = {\n" + "".join(f"  (fn_t)&{n},\n" for n in names) + "};\n"
+        "int main(void) {\n"
+        "  if (sizeof every / sizeof every[0] != %d) return 2;\n" % len(names) +
+        "  printf(\"%d %s\\n\", hscale_abi_version(), hscale_status_string(HSCALE_ERR_SHAPE));\n"
+        "  return hscale_refine_scales(0, 0, 4, 40, 0, 0, 4, 4, 0, 0, 0) == HSCALE_ERR_SHAPE ? 0 : 1;\n"
+        "}\n")
+    build_dir = hs.library_path().parent
+    exe = tmp_path / "abi_check"
+    cmd = [cc, "-std=c99", "-Wall", "-Wextra", "-pedantic", "-Werror", f"-I{HEADER.parent}", str(src),
+           f"-L{build_dir}", "-lhscale", f"-Wl,-rpath,{build_dir}", "-o", str(exe)]
+    r = subprocess.run(cmd, capture_output=True, text=True)
+    assert r.returncode == 0, r.stderr
+    r = subprocess.run([str(exe)], capture_output=True, text=True)
+    assert r.returncode == 0, (r.stdout, r.stderr)
+    assert r.stdout.split()[0] == str(hs.hscale_abi_version())
+
+
 def test_status_strings(lib):
     for s in range(7):
         assert hs.hscale_status_string(s)
