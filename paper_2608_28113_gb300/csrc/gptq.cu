@@ -10,7 +10,7 @@
 //                     L^T Y = I (both loaded at run time) on column-major storage: Y = L^-T
 //                     in column-major order is (J Y J)^T = U^T after reversing the array,
 //                     i.e. row-major U.
-//   block_kernel      one thread per 16-element group of a block of B columns of the running
+//   block_kernel      four lanes per 16-element group of a block of B columns of the running
 //                     fp32 weights: the RTN code (Eq. 7) of the current weights, the exact
 //                     H-Scale search over the window (Algorithm 1, exact E2M1 decisions, the
 //                     tie rule of the search), the codes and packed nibbles, and the
@@ -176,27 +176,36 @@ __device__ float exact_group_score(const float (&a)[16], const float (&hj)[16], 
   return t[0];
 }
 
+// Four lanes (a quad) per group: each scores every fourth candidate of the window with exact
+// decisions, the quad keeps the best under the search's tie rule (a total order, so every
+// lane ends with the same code), and each lane writes the nibbles and errors of four of the
+// group's elements.
 __global__ void __launch_bounds__(128) block_kernel(const float* __restrict__ W, int64_t m, int64_t n, int64_t col0,
                                                     int B, const float* __restrict__ h, const float* __restrict__ U,
                                                     const float* __restrict__ global_scale, int down, int up,
                                                     uint8_t* __restrict__ codes, uint2* __restrict__ packed,
                                                     float* __restrict__ E) {
   const int gpb = B / 16;
-  const int64_t groups = m * gpb;
+  const int64_t total = m * gpb * 4;  // lanes
+  const int q = threadIdx.x & 3;
   const ScaleDomain d = make_scale_domain(*global_scale);
   const float inv6 = rtn_inv6_raw(d.sgk);
-  for (int64_t g = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; g < groups; g += (int64_t)gridDim.x * blockDim.x) {
+  // block-uniform trip count: every lane of a warp reaches the shuffles together
+  for (int64_t base = (int64_t)blockIdx.x * blockDim.x; base < total; base += (int64_t)gridDim.x * blockDim.x) {
+    const int64_t lane_id = base + threadIdx.x;
+    const bool active = lane_id < total;
+    const int64_t g = active ? lane_id >> 2 : 0;
     const int64_t r = g / gpb;
     const int i = (int)(g - r * gpb);
     const int64_t col = col0 + 16 * i;
     float w[16], a[16], hj[16];
     float amax = 0.0f;
 #pragma unroll
-    for (int q = 0; q < 4; ++q) {
-      const float4 v = reinterpret_cast<const float4*>(W + r * n + col)[q];
-      const float4 hv = reinterpret_cast<const float4*>(h + col)[q];
-      w[4 * q] = v.x; w[4 * q + 1] = v.y; w[4 * q + 2] = v.z; w[4 * q + 3] = v.w;
-      hj[4 * q] = hv.x; hj[4 * q + 1] = hv.y; hj[4 * q + 2] = hv.z; hj[4 * q + 3] = hv.w;
+    for (int k = 0; k < 4; ++k) {
+      const float4 v = reinterpret_cast<const float4*>(W + r * n + col)[k];
+      const float4 hv = reinterpret_cast<const float4*>(h + col)[k];
+      w[4 * k] = v.x; w[4 * k + 1] = v.y; w[4 * k + 2] = v.z; w[4 * k + 3] = v.w;
+      hj[4 * k] = hv.x; hj[4 * k + 1] = hv.y; hj[4 * k + 2] = hv.z; hj[4 * k + 3] = hv.w;
     }
 #pragma unroll
     for (int j = 0; j < 16; ++j) {
@@ -207,31 +216,48 @@ __global__ void __launch_bounds__(128) block_kernel(const float* __restrict__ W,
     const int lo = max(1, c0 - down), hi = min((int)kE4M3MaxCode, c0 + up);
     float be = 0.0f;
     int bc = -1;
-    for (int c = lo; c <= hi; ++c) {
+    for (int c = lo + q; c <= hi; c += 4) {
       const float e = exact_group_score(a, hj, (uint32_t)c, d.sgk);
       if (bc < 0 || better_code(e, c, be, bc, c0)) {
         be = e;
         bc = c;
       }
     }
+#pragma unroll
+    for (int off = 1; off < 4; off <<= 1) {
+      const float oe = __shfl_xor_sync(0xFFFFFFFFu, be, off);
+      const int oc = __shfl_xor_sync(0xFFFFFFFFu, bc, off);
+      if (oc >= 0 && (bc < 0 || better_code(oe, oc, be, bc, c0))) {
+        be = oe;
+        bc = oc;
+      }
+    }
     const float l = e4m3_mag((uint32_t)bc);
     const float inv = inv_raw_of(__fmul_rn(l, d.sgk));
-    uint32_t word[2] = {0u, 0u};
+    // this lane's elements 4q..4q+3 (read again as one vector: no dynamic register index)
+    const float4 wq = reinterpret_cast<const float4*>(W + r * n + col)[q];
+    const float wv[4] = {wq.x, wq.y, wq.z, wq.w};
+    uint32_t part = 0u;  // this lane's four nibbles in their place in the group's 32-bit word
 #pragma unroll
-    for (int j = 0; j < 16; ++j) {
-      const uint32_t k = e2m1_code(a[j], inv, l, d.sgk);
-      const uint32_t neg = signbit(w[j]) ? 1u : 0u;
-      word[j >> 3] |= ((neg << 3) | k) << (4 * (j & 7));
+    for (int t = 0; t < 4; ++t) {
+      const int j = 4 * q + t;
+      const float av = __fmul_rn(fabsf(wv[t]), d.pw);
+      const uint32_t k = e2m1_code(av, inv, l, d.sgk);
+      const uint32_t neg = signbit(wv[t]) ? 1u : 0u;
+      part |= ((neg << 3) | k) << (4 * (j & 7));
       float what = __fmul_rn(d.sg, __fmul_rn(e2m1_from_raw(k << 22), l));  // s_g (l q), l q exact
       if (neg) what = -what;
-      E[r * B + 16 * i + j] = __fdiv_rn(__fsub_rn(w[j], what), U[(col + j) * n + col + j]);
+      if (active) E[r * B + 16 * i + j] = __fdiv_rn(__fsub_rn(wv[t], what), U[(col + j) * n + col + j]);
     }
-    codes[r * (n / 16) + col / 16] = (uint8_t)bc;
-    packed[r * (n / 16) + col / 16] = make_uint2(word[0], word[1]);
+    const uint32_t word = part | __shfl_xor_sync(0xFFFFFFFFu, part, 1);  // lanes 0-1: word 0, 2-3: word 1
+    const uint32_t other = __shfl_xor_sync(0xFFFFFFFFu, word, 2);
+    if (active && q == 0) {
+      codes[r * (n / 16) + col / 16] = (uint8_t)bc;
+      packed[r * (n / 16) + col / 16] = make_uint2(word, other);
+    }
   }
 }
 
-// W[r, c1 + c] -= sum_k E[r, k] U[col0 + k, c1 + c], k < B; 128 x 128 tiles, 8 x 8 per thread
 // W[:, c1:] -= E U[col0:c1, c1:] (c1 = col0 + B) in fp32: 128 x 128 output tiles, 256
 // threads with 8 rows x 8 columns each (columns 4*tc..4*tc+3 and 64+4*tc..64+4*tc+3, so
 // the 128-bit shared loads of a quarter warp are contiguous), k-slices of 8 staged in shared
@@ -409,7 +435,7 @@ cudaError_t launch_gptq_hscale(const void* w, int64_t m, int64_t n, const float*
   if ((err = cudaGetLastError()) != cudaSuccess) return err;
   for (int64_t col0 = 0; col0 < n; col0 += block) {
     const int64_t groups = m * (block / 16);
-    const unsigned qb = (unsigned)std::min<int64_t>((groups + 127) / 128, (int64_t)info.sm_count * 16);
+    const unsigned qb = (unsigned)std::min<int64_t>((groups * 4 + 127) / 128, (int64_t)info.sm_count * 16);
     block_kernel<<<qb, 128, 0, stream>>>(Wf, m, n, col0, block, h, U, global_scale, down, up, codes,
                                          reinterpret_cast<uint2*>(packed), E);
     if ((err = cudaGetLastError()) != cudaSuccess) return err;
