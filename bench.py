@@ -498,15 +498,13 @@ def window_of(args, W: wl.Workload):
     return (k, k)
 
 
-def cpu_baseline(W: wl.Workload, win, budget_s: float = 12.0, init: str = "rtn"):
-    """Time the fp64 oracle on a bounded sample of the workload and extrapolate the
-    whole-step time: Hessian over sampled tokens of every input space, global scale +
+def _oracle_step(W: wl.Workload, win, budget_s: float, init: str, threads: int):
+    """Whole-step time of the fp64 oracle with `threads` threads, extrapolated from a
+    bounded sample: Hessian over sampled tokens of every input space, global scale +
     initial codes (RTN or 4over6) over every matrix, search over sampled rows of every
-    matrix."""
+    matrix.  Returns (seconds per step, groups, samples, token-channels)."""
     import oracle
-    oracle.build()
-    cores = len(os.sched_getaffinity(0)) if hasattr(os, "sched_getaffinity") else os.cpu_count()
-    oracle.set_threads(cores)
+    oracle.set_threads(threads)
     per_part = budget_s / (len(W.input_spaces()) + len(W.layers))
     step = 0.0
     groups = 0
@@ -553,11 +551,25 @@ def cpu_baseline(W: wl.Workload, win, budget_s: float = 12.0, init: str = "rtn")
         groups += G
         samples.append(f"search {L.name}: {done}x{rows} rows")
     step += t_rtn_total
+    return step, groups, samples, h_tc
+
+
+def cpu_baseline(W: wl.Workload, win, budget_s: float = 12.0, init: str = "rtn"):
+    """The fp64 oracle timed on the host's cores (all of them, and one thread on a shorter
+    sample), extrapolated to the whole step."""
+    import oracle
+    oracle.build()
+    cores = len(os.sched_getaffinity(0)) if hasattr(os, "sched_getaffinity") else os.cpu_count()
+    step, groups, samples, h_tc = _oracle_step(W, win, budget_s, init, cores)
+    step1, _, samples1, _ = _oracle_step(W, win, budget_s / 3, init, 1)
+    oracle.set_threads(cores)
     return {
         "value": groups / step, "unit": UNIT, "cores": cores, "kind": "oracle",
         "sample": (f"fp64 C oracle, {cores} threads, bounded sample extrapolated to the step "
                    f"({W.tokens} tokens per input space, {groups} groups, window -{win[0]}/+{win[1]}): "
                    + "; ".join(samples) + f"; global scale + {init} codes over every whole matrix"),
+        "single_thread_value": groups / step1,
+        "single_thread_sample": "; ".join(samples1),
         "seconds_per_step": step,
         "hessian_tokens_channels_per_s": h_tc / max(step, 1e-30),
     }
@@ -567,14 +579,17 @@ def reference_arm(args, d: Dist):
     """--impl reference: the CPU oracle, as it stands, on the host cores."""
     if d.rank != 0:
         return
+    import oracle
+    oracle.build()
     W = wl.WORKLOADS[args.workload]
     win = window_of(args, W)
+    cores = len(os.sched_getaffinity(0)) if hasattr(os, "sched_getaffinity") else os.cpu_count()
     vals = []
-    cb = None
+    samples = []
     for i in range(args.warmup + args.steps):
-        cb = cpu_baseline(W, win, budget_s=3.0, init=args.init)
+        step, _, samples, _ = _oracle_step(W, win, 3.0, args.init, cores)
         if i >= args.warmup:
-            vals.append(cb["seconds_per_step"])
+            vals.append(step)
     groups = sum(L.out_features * L.in_features // 16 for L in W.layers)
     sec = statistics.mean(vals)
     value = groups / sec
@@ -585,8 +600,11 @@ def reference_arm(args, d: Dist):
         "data": "synthetic",
         "config": {"workload": W.name, "matrices": [[L.name, L.out_features, L.in_features] for L in W.layers],
                    "tokens": W.tokens, "window": list(win), "init": args.init},
-        "cpu_baseline": {"value": value, "unit": UNIT, "cores": cb["cores"], "kind": "oracle",
-                         "sample": cb["sample"]},
+        "cpu_baseline": {"value": value, "unit": UNIT, "cores": cores, "kind": "oracle",
+                         "sample": (f"fp64 C oracle, {cores} threads, per step a bounded sample extrapolated "
+                                    f"to the step ({W.tokens} tokens per input space, {groups} groups, window "
+                                    f"-{win[0]}/+{win[1]}): " + "; ".join(samples)
+                                    + f"; global scale + {args.init} codes over every whole matrix")},
         "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
     }
     print(json.dumps(line), flush=True)
@@ -902,7 +920,8 @@ def gpu_arm(args, d: Dist):
         line["e2e"] = e2e
     if d.rank == 0 and d.world == 1 and not args.no_cpu_baseline:
         cb = cpu_baseline(W, win, init=args.init)
-        line["cpu_baseline"] = {k2: cb[k2] for k2 in ("value", "unit", "cores", "kind", "sample")}
+        line["cpu_baseline"] = {k2: cb[k2] for k2 in ("value", "unit", "cores", "kind", "sample",
+                                                      "single_thread_value")}
     if d.rank == 0:
         print(json.dumps(line), flush=True)
 
