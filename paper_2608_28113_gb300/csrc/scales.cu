@@ -265,6 +265,27 @@ __device__ __forceinline__ uint32_t cvt_e2m1x2(float hi, float lo) {
   return r;
 }
 
+// The anchored code of Eq. 7 (anchor c = 2 * half_c; RTN is c = 6), decided by the hardware
+// E4M3 conversion of the fast quotient r = amax_k * inv_c (inv_c ~ 1 / (c * sgk), within a
+// relative 2^-22 of the exact quotient, so r is within 2^-21 of it).  RNE of r equals RNE
+// of the exact quotient unless the quotient lies near an E4M3 midpoint: in the normal
+// range (r >= 2^-6) the midpoints are the fp32 patterns whose low 20 bits are 0x80000, and
+// r within 16 ulps of one is flagged.  Flagged quotients and the subnormal range take the
+// exact midpoint tests of anchored_code().  Saturation at 448 (code 126) is the
+// conversion's own; code 0 is clamped to 1.
+__device__ __forceinline__ uint32_t anchored_code_fast(float amax_k, float sgk, float inv_c, float inv_raw,
+                                                       float half_c) {
+  const float r = __fmul_rn(amax_k, inv_c);
+  const bool near = ((__float_as_uint(r) - 0x7FFF0u) & 0xFFFFFu) <= 0x20u;
+  if (near || !(r >= 0x1p-6f)) return anchored_code(amax_k, sgk, inv_raw, half_c);
+  uint32_t c;
+  asm("{\n\t.reg .b16 t;\n\tcvt.rn.satfinite.e4m3x2.f32 t, %1, %2;\n\tcvt.u32.u16 %0, t;\n\t}"
+      : "=r"(c)
+      : "f"(0.0f), "f"(r));
+  c &= 0xFFu;
+  return c < 1u ? 1u : c;
+}
+
 // Exact final re-quantization of one group under code c (inv_raw = 2^-126 / s'): 8 bytes of
 // packed nibbles.  The raw-domain quotients y_raw = w * 2^-126 / s' (signed) are rescaled
 // exactly to real units and converted by the hardware E2M1 conversion (round-to-nearest-
@@ -373,9 +394,10 @@ __device__ __noinline__ uint32_t fourover6_exact_pick(const uint4* wg, float pw,
 // <= 7 * 2^-24, far inside the margin) order them the same way; so the result is always
 // the code fourover6_codes_kernel writes.
 __device__ __forceinline__ int fourover6_init_code(const Group& G, const uint4* wg, const float4* tab,
-                                                   float amax_k, float sgk, float pw, float inv4, float inv6) {
-  const uint32_t c4 = anchored_code(amax_k, sgk, inv4, 2.0f);
-  const uint32_t c6 = anchored_code(amax_k, sgk, inv6, 3.0f);
+                                                   float amax_k, float sgk, float pw, float inv4, float inv6,
+                                                   float inv4r, float inv6r) {
+  const uint32_t c4 = anchored_code_fast(amax_k, sgk, inv4r, inv4, 2.0f);
+  const uint32_t c6 = anchored_code_fast(amax_k, sgk, inv6r, inv6, 3.0f);
   if (c4 == c6) return (int)c4;
   const float e4 = fast_mse(G, tab[c4]);
   const float e6 = fast_mse(G, tab[c6]);
@@ -408,6 +430,7 @@ refine_kernel(const uint4* __restrict__ w, int64_t ld_w, const float* __restrict
   const ScaleDomain d = make_scale_domain(*global_scale);
   const float inv6 = rtn_inv6_raw(d.sgk);
   const float inv4 = kFourOverSix ? anchor_inv_raw(d.sgk, 4.0f) : 0.0f;
+  const float inv6r = __frcp_rn(__fmul_rn(6.0f, d.sgk)), inv4r = __frcp_rn(__fmul_rn(4.0f, d.sgk));
   for (int c = threadIdx.x; c < 128; c += blockDim.x) tab[c] = candidate_constants((uint32_t)c, d.sgk);
   __syncthreads();
 
@@ -459,8 +482,8 @@ refine_kernel(const uint4* __restrict__ w, int64_t ld_w, const float* __restrict
         c0 = init_codes[row * ld_i + gcol] & 0x7F;
         c0 = c0 < 1 ? 1 : (c0 > (int)kE4M3MaxCode ? (int)kE4M3MaxCode : c0);
       } else {
-        c0 = kFourOverSix ? fourover6_init_code(G, w + wofs / 8, tab, amax_k, d.sgk, d.pw, inv4, inv6)
-                          : (int)rtn_code(amax_k, d.sgk, inv6);
+        c0 = kFourOverSix ? fourover6_init_code(G, w + wofs / 8, tab, amax_k, d.sgk, d.pw, inv4, inv6, inv4r, inv6r)
+                          : (int)anchored_code_fast(amax_k, d.sgk, inv6r, inv6, 3.0f);
       }
       lo = max(1, c0 - down);
       hi = min((int)kE4M3MaxCode, c0 + up);
