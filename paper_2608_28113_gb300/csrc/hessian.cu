@@ -10,7 +10,7 @@
 //     16-byte vectors) read each stage back with conflict-free 128-bit shared loads
 //     and accumulate in fp32.  mbarriers order the ring; every wait is bounded.
 //   * The token range of a tile is split over the CTAs of one thread-block cluster
-//     (1, 2, 4 or 8 CTAs, so a launch holds about two CTAs per SM).  The CTAs
+//     (1, 2, 4 or 8 CTAs, so a launch holds about one CTA per SM).  The CTAs
 //     of a cluster reduce their partial sums through distributed shared memory: the
 //     kernel needs no global scratch, no atomics and no second launch.
 //   * Launches use programmatic dependent launch: the next chunk's kernel may start
@@ -254,9 +254,11 @@ cudaError_t launch_hessian(const void* x, int64_t tokens, int64_t n, int64_t ld_
   if (r != CUDA_SUCCESS) return cudaErrorInvalidValue;
 
   const int tiles = (int)((n + kTileCols - 1) / kTileCols);
-  // about two CTAs per SM: two consecutive chunk launches fit side by side, so with
-  // programmatic dependent launch the next chunk streams while this one drains
-  const int64_t target = (int64_t)info.sm_count * 2;
+  // at most about one CTA per SM per launch: with programmatic dependent launch,
+  // consecutive chunk launches share the GPU, so the next chunk streams while this one
+  // drains (q_proj, 8192-token chunks, 64 tiles: cluster size 1 gives 10.2 us per chunk,
+  // 2 (this rule) 9.8, 4 9.9, 8 11.2)
+  const int64_t target = (int64_t)info.sm_count;
   int cs = 1;
   while (cs < kMaxCluster && (int64_t)tiles * cs * 2 <= target && (int64_t)cs * 2 * kStageRows * 4 <= tokens)
     cs *= 2;
