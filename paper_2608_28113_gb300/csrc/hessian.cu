@@ -5,7 +5,7 @@
 // Layout of the work
 //   * A CTA owns a 64-channel column tile (128 bytes of every row) and a contiguous
 //     run of tokens.  One thread streams the run into a ring of shared-memory stages
-//     with 2-D TMA tensor loads (64 channels x 128 rows = 16 KB per stage, 3 stages in
+//     with 2-D TMA tensor loads (64 channels x 128 rows = 16 KB per stage, 4 stages in
 //     flight per CTA, L2 evict-first); the CTA's 256 threads (32 row phases x 8
 //     16-byte vectors) read each stage back with conflict-free 128-bit shared loads
 //     and accumulate in fp32.  mbarriers order the ring; every wait is bounded.
@@ -50,7 +50,7 @@ constexpr int kThreads = 256;
 constexpr int kPhases = 32;                         // rows read side by side
 constexpr int kWarps = kThreads / 32;
 constexpr int kStageRows = 128;
-constexpr int kStages = 3;
+constexpr int kStages = 4;
 constexpr uint32_t kStageBytes = kStageRows * kTileCols * 2;
 constexpr size_t kRingBytes = (size_t)kStages * kStageBytes;
 constexpr int64_t kMaxRowsPerCta = 1024 * kPhases;  // <= 1024 sequential adds per thread
