@@ -199,12 +199,8 @@ hessian_colsumsq_kernel(const __grid_constant__ CUtensorMap xmap, int64_t row0, 
 template <int CS>
 cudaError_t launch_cs(const CUtensorMap& map, int64_t tokens, int n, float* h, int tiles,
                       cudaStream_t stream) {
-  static std::once_flag once;
-  static cudaError_t attr_status = cudaSuccess;
-  std::call_once(once, [] {
-    attr_status = cudaFuncSetAttribute(hessian_colsumsq_kernel<CS>,
-                                       cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kRingBytes);
-  });
+  const cudaError_t attr_status =
+      ensure_dynamic_smem(reinterpret_cast<const void*>(hessian_colsumsq_kernel<CS>), (int)kRingBytes);
   if (attr_status != cudaSuccess) return attr_status;
   const int64_t rows_per_launch = kMaxRowsPerCta * CS;
   for (int64_t t0 = 0; t0 < tokens; t0 += rows_per_launch) {
@@ -268,6 +264,26 @@ cudaError_t launch_hessian(const void* x, int64_t tokens, int64_t n, int64_t ld_
     case 4: return launch_cs<4>(map, tokens, (int)n, h, tiles, stream);
     default: return launch_cs<8>(map, tokens, (int)n, h, tiles, stream);
   }
+}
+
+cudaError_t ensure_dynamic_smem(const void* func, int bytes) {
+  static std::mutex mu;
+  static const void* done_func[256];
+  static int done_dev[256];
+  static int done_count = 0;
+  int dev = 0;
+  cudaError_t err = cudaGetDevice(&dev);
+  if (err != cudaSuccess) return err;
+  std::lock_guard<std::mutex> lock(mu);
+  for (int i = 0; i < done_count; ++i)
+    if (done_func[i] == func && done_dev[i] == dev) return cudaSuccess;
+  err = cudaFuncSetAttribute(func, cudaFuncAttributeMaxDynamicSharedMemorySize, bytes);
+  if (err == cudaSuccess && done_count < 256) {
+    done_func[done_count] = func;
+    done_dev[done_count] = dev;
+    ++done_count;
+  }
+  return err;
 }
 
 cudaError_t encode_tiled_fn(EncodeTiledFn* out) {

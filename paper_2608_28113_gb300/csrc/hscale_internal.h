@@ -48,6 +48,11 @@ using EncodeTiledFn = CUresult (*)(CUtensorMap*, CUtensorMapDataType, cuuint32_t
                                    CUtensorMapL2promotion, CUtensorMapFloatOOBfill);
 cudaError_t encode_tiled_fn(EncodeTiledFn* out);
 
+// cudaFuncAttributeMaxDynamicSharedMemorySize = bytes for kernel `func` on the current
+// device, set once per (kernel, device) and remembered, so that every GPU of a process
+// gets it (a function attribute belongs to one device's context).
+cudaError_t ensure_dynamic_smem(const void* func, int bytes);
+
 // dW = W - W_hat of packed NVFP4 weights as a bf16 pair [hi | lo] per row, rows of ld
 // elements: hi in [0, n_pad), lo in [n_pad, 2 n_pad), zero padding, n_pad = 64 * ceil(n / 64).
 cudaError_t launch_residual(const void* w, int64_t m, int64_t n, const float* global_scale,

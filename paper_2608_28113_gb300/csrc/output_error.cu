@@ -414,8 +414,8 @@ cudaError_t launch_output_error(const void* x, int64_t tokens, int64_t n, int64_
                CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) != CUDA_SUCCESS)
       return cudaErrorInvalidValue;
   }
-  static cudaError_t attr_status = cudaFuncSetAttribute(gemm_kernel<false>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                                        (int)kGemmSmemBytes);
+  const cudaError_t attr_status =
+      ensure_dynamic_smem(reinterpret_cast<const void*>(gemm_kernel<false>), (int)kGemmSmemBytes);
   if (attr_status != cudaSuccess) return attr_status;
   const int64_t tiles_n = (m + kBN - 1) / kBN;
   const int64_t tiles = output_error_tiles(tokens, m);
@@ -457,8 +457,8 @@ cudaError_t launch_hessian_full(const void* x, int64_t tokens, int64_t n, int64_
       encode(&bmap, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, xt, dims, strides, bbox, estr, CU_TENSOR_MAP_INTERLEAVE_NONE,
              CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) != CUDA_SUCCESS)
     return cudaErrorInvalidValue;
-  static cudaError_t attr_status = cudaFuncSetAttribute(gemm_kernel<true>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                                        (int)kGemmSmemBytes);
+  const cudaError_t attr_status =
+      ensure_dynamic_smem(reinterpret_cast<const void*>(gemm_kernel<true>), (int)kGemmSmemBytes);
   if (attr_status != cudaSuccess) return attr_status;
   const int64_t tiles_n = (n + kBN - 1) / kBN;
   const int64_t tiles = ((n + kBM - 1) / kBM) * tiles_n;
