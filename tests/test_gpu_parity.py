@@ -589,6 +589,37 @@ def test_strided_row_slice_and_no_packed_output():
     assert np.array_equal(c2.cpu().numpy(), codes)
 
 
+# ------------------------------------------------------------------ the fast path's margin band
+
+@pytest.mark.parametrize("down,up", [(4, 4), (9, 6)])
+def test_search_exact_in_the_margin_band(down, up):
+    """2,097,152 groups against the oracle, with the groups whose best and runner-up errors
+    differ by 1e-6 to 1e-3 relative counted separately: there the fast scores cannot
+    decide and the exact rescoring must (outside the 1e-6 near-tie band every code and
+    nibble must be the oracle's)."""
+    m, n = 4096, 8192
+    w = wl.weight(m, n, 0.02, 4242, device=dev())
+    h32 = oracle_h32(4242, n, tokens=1024)
+    sg, _ = gpu_rtn(w)
+    wb = bits(w)
+    s_ref, _ = oracle.global_scale(wb)
+    assert sg.cpu().numpy()[0] == s_ref
+    codes, packed = gpu_refine(w, h32, sg, None, down, up)
+    ref = oracle.refine(wb, h32, s_ref, None, down, up)
+    compare_search(ref, codes, packed, f"2M groups -{down}/+{up}")
+    with np.errstate(divide="ignore", invalid="ignore"):
+        gap = (ref["e_second"] - ref["e_best"]) / ref["e_second"]
+    band = (gap > 1e-6) & (gap < 1e-3)
+    assert band.sum() >= 100, f"only {band.sum()} groups in the margin band"
+    assert np.array_equal(codes[band], ref["codes"][band])
+    rows = np.nonzero(band.any(axis=1))[0]
+    for r in rows[:256]:
+        cols = np.nonzero(band[r])[0]
+        for c in cols:
+            assert np.array_equal(packed[r, 8 * c:8 * c + 8], ref["packed"][r, 8 * c:8 * c + 8])
+    print(f"[parity] margin band -{down}/+{up}: {int(band.sum())} groups with 1e-6 < gap < 1e-3, all exact")
+
+
 # ------------------------------------------------------------------ offsets past 2^31 elements
 
 def test_search_and_hessian_beyond_2_31_elements():
