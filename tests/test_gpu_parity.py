@@ -347,6 +347,31 @@ def test_pack_matches_oracle_bit_exact():
         assert np.array_equal(packed.cpu().numpy(), oracle.pack(bits(w), s_ref, c))
 
 
+def test_pack_full_size_q_proj():
+    """hscale_pack_nvfp4 over the whole 4096 x 4096 q_proj matrix: with the search's own
+    codes it reproduces the search's nibbles (every group), and with random codes (sign bit
+    set, off-ladder bytes 0 and 127-255 clamped) it matches the oracle on sampled rows."""
+    W = wl.WORKLOADS["llama8b-q_proj"]
+    L = W.layers[0]
+    m, n = L.out_features, L.in_features
+    w = wl.weight(m, n, W.sigma_w, wl.chunk_seed(W.layer_seed(0), L.name, 0) & 0xFFFFFFFF, device=dev())
+    h32 = oracle_h32(1, n, tokens=512)
+    sg, _ = gpu_rtn(w)
+    codes, packed = gpu_refine(w, h32, sg, None, 4, 4)
+    out = torch.empty(m, n // 2, dtype=torch.uint8, device=dev())
+    hs.hscale_pack_nvfp4(w, sg, torch.from_numpy(codes).to(dev()), out)
+    torch.cuda.synchronize()
+    assert np.array_equal(out.cpu().numpy(), packed)
+    rng = np.random.default_rng(33)
+    rnd = rng.integers(0, 256, size=(m, n // 16)).astype(np.uint8)
+    hs.hscale_pack_nvfp4(w, sg, torch.from_numpy(rnd).to(dev()), out)
+    torch.cuda.synchronize()
+    rows = np.sort(rng.choice(m, size=64, replace=False))
+    s_ref, _ = oracle.global_scale(bits(w))
+    wb = bits(w[torch.from_numpy(rows).to(dev())])
+    assert np.array_equal(out.cpu().numpy()[rows], oracle.pack(wb, s_ref, rnd[rows]))
+
+
 def test_refine_launch_shape_does_not_change_results():
     """hscale_refine_scales_ex with 1, 2 or 5 resident CTAs per SM (more units per warp,
     other unit-to-warp assignment) writes the same bytes as the full launch."""
