@@ -344,9 +344,11 @@ int hscale_output_error(const void* x_bf16, int64_t tokens, int64_t n, int64_t l
  *    diagonal proxy h [n] (16-byte aligned) and the global scale s_g of the original W
  *    (U as written by hscale_gptq_factor, 16-byte aligned),
  *    with exact E2M1 decisions and the tie rule of hscale_refine_scales; then
- *    E = (W_b - W_hat_b) / diag(U_b) and W[:, i+B:] -= E U[i:i+B, i+B:] in fp32.  Writes
- *    codes_out [m, n/16] and packed_out [m, n/2] (8-byte aligned) as hscale_refine_scales
- *    does.  The workspace (hscale_gptq_workspace_bytes) holds the running weights and E.
+ *    E = (W_b - W_hat_b) / diag(U_b) and W[:, i+B:] -= E U[i:i+B, i+B:] with fp32-level
+ *    accuracy (on the tensor cores: three-way bf16 splits of E and U, the six products
+ *    above 2^-24 relative, fp32 accumulation).  Writes codes_out [m, n/16] and packed_out
+ *    [m, n/2] (8-byte aligned) as hscale_refine_scales does.  The workspace
+ *    (hscale_gptq_workspace_bytes) holds the running weights, E and the split operands.
  */
 size_t hscale_hessian_full_workspace_bytes(int64_t tokens, int64_t n);
 int hscale_hessian_full_accumulate(const void* x_bf16, int64_t tokens, int64_t n, int64_t ld_x, float* H,

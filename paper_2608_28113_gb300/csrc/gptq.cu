@@ -15,7 +15,8 @@
 //                     H-Scale search over the window (Algorithm 1, exact E2M1 decisions, the
 //                     tie rule of the search), the codes and packed nibbles, and the
 //                     propagated errors E = (W - W_hat) / U_jj
-//   update_kernel     W[:, i+B:] -= E U[i:i+B, i+B:] in fp32 (register-blocked SIMT GEMM)
+//   update            W[:, i+B:] -= E U[i:i+B, i+B:] with fp32-level accuracy on the tensor
+//                     cores (three-way bf16 splits, six products, one GEMM)
 #include <dlfcn.h>
 
 #include <algorithm>
@@ -24,6 +25,7 @@
 #include <vector>
 
 #include <cublas_v2.h>
+#include <cuda_bf16.h>
 #include <cusolverDn.h>
 
 #include "hscale_device.cuh"
@@ -258,103 +260,69 @@ __global__ void __launch_bounds__(128) block_kernel(const float* __restrict__ W,
   }
 }
 
-// W[:, c1:] -= E U[col0:c1, c1:] (c1 = col0 + B) in fp32: 128 x 128 output tiles, 256
-// threads with 8 rows x 8 columns each (columns 4*tc..4*tc+3 and 64+4*tc..64+4*tc+3, so
-// the 128-bit shared loads of a quarter warp are contiguous), k-slices of 8 staged in shared
-// memory with the next slice prefetched into registers.  E is stored pre-splatted (each
-// value twice) so that one packed FMA updates two columns of a row: every accumulator is
-// still a chain of scalar-rounded FMAs in k order.
-constexpr int kUT = 128, kUK = 8;
-__global__ void __launch_bounds__(256, 2) update_kernel(float* __restrict__ W, int64_t m, int64_t n, int64_t col0, int B,
-                                                     const float* __restrict__ E, const float* __restrict__ U) {
-  __shared__ __align__(16) float2 As[2][kUK][kUT];
-  __shared__ __align__(16) float Bs[2][kUK][kUT];
-  const int64_t c1 = col0 + B;
-  const int64_t row0 = (int64_t)blockIdx.y * kUT, cb = c1 + (int64_t)blockIdx.x * kUT;
-  const int tid = threadIdx.x, tr = tid / 16, tc = tid % 16;
-  // global -> register staging: E row ar, k-quad aq; U k-row bk, column quad bq
-  const int ar = tid / 2, aq = (tid % 2) * 4;
-  const int bk = tid / 32, bq = (tid % 32) * 4;
-  const int64_t arow = row0 + ar, bcol = cb + bq;
-  auto load_a = [&](int k0) -> float4 {
-    if (arow >= m) return make_float4(0.f, 0.f, 0.f, 0.f);
-    return *reinterpret_cast<const float4*>(E + arow * B + k0 + aq);
-  };
-  auto load_b = [&](int k0) -> float4 {
-    const float* src = U + (col0 + k0 + bk) * n;
-    if (bcol + 3 < n) return *reinterpret_cast<const float4*>(src + bcol);
-    float4 v = make_float4(0.f, 0.f, 0.f, 0.f);
-    if (bcol + 0 < n) v.x = src[bcol + 0];
-    if (bcol + 1 < n) v.y = src[bcol + 1];
-    if (bcol + 2 < n) v.z = src[bcol + 2];
-    return v;
-  };
-  auto store = [&](int buf, float4 a, float4 b) {
-    As[buf][aq + 0][ar] = make_float2(a.x, a.x);
-    As[buf][aq + 1][ar] = make_float2(a.y, a.y);
-    As[buf][aq + 2][ar] = make_float2(a.z, a.z);
-    As[buf][aq + 3][ar] = make_float2(a.w, a.w);
-    *reinterpret_cast<float4*>(&Bs[buf][bk][bq]) = b;
-  };
-  float2 acc[8][4];
-#pragma unroll
-  for (int i = 0; i < 8; ++i)
-#pragma unroll
-    for (int j = 0; j < 4; ++j) acc[i][j] = make_float2(0.f, 0.f);
+// The update W[:, c1:] -= E U[col0:c1, c1:] (c1 = col0 + B) runs on the tensor cores with
+// fp32-level accuracy: every fp32 value x is split into three bf16 parts x1 + x2 + x3 (each
+// difference exact in fp32, so the parts carry x to about 2^-24 relative), and the six
+// products E1 U1, E1 U2, E2 U1, E1 U3, E2 U2, E3 U1 (every pair whose weight is above
+// 2^-24) are one bf16 GEMM over K = 6B with fp32 accumulation: A' = [-E1 | -E1 | -E2 | -E1
+// | -E2 | -E3] against B' = [U1 | U2 | U1 | U3 | U2 | U1] (the negation makes the GEMM's
+// accumulate a subtract).
+__device__ __forceinline__ void split3(float x, uint16_t (&p)[3]) {
+  const __nv_bfloat16 a = __float2bfloat16_rn(x);
+  const float r1 = __fsub_rn(x, __bfloat162float(a));
+  const __nv_bfloat16 b = __float2bfloat16_rn(r1);
+  const float r2 = __fsub_rn(r1, __bfloat162float(b));
+  const __nv_bfloat16 c = __float2bfloat16_rn(r2);
+  p[0] = __bfloat16_as_ushort(a);
+  p[1] = __bfloat16_as_ushort(b);
+  p[2] = __bfloat16_as_ushort(c);
+}
 
-  store(0, load_a(0), load_b(0));
-  __syncthreads();
-  int buf = 0;
-  for (int k0 = 0; k0 < B; k0 += kUK) {
-    const bool more = k0 + kUK < B;
-    float4 na = make_float4(0.f, 0.f, 0.f, 0.f), nb = na;
-    if (more) {
-      na = load_a(k0 + kUK);
-      nb = load_b(k0 + kUK);
-    }
-#pragma unroll
-    for (int kk = 0; kk < kUK; ++kk) {
-      float2 av[8];
-      const float4* ap = reinterpret_cast<const float4*>(&As[buf][kk][tr * 8]);
-#pragma unroll
-      for (int i = 0; i < 4; ++i) {
-        const float4 t = ap[i];
-        av[2 * i] = make_float2(t.x, t.y);
-        av[2 * i + 1] = make_float2(t.z, t.w);
-      }
-      const float4 b0 = *reinterpret_cast<const float4*>(&Bs[buf][kk][tc * 4]);
-      const float4 b1 = *reinterpret_cast<const float4*>(&Bs[buf][kk][64 + tc * 4]);
-      const float2 bv[4] = {make_float2(b0.x, b0.y), make_float2(b0.z, b0.w), make_float2(b1.x, b1.y),
-                            make_float2(b1.z, b1.w)};
-#pragma unroll
-      for (int i = 0; i < 8; ++i)
-#pragma unroll
-        for (int j = 0; j < 4; ++j) acc[i][j] = __ffma2_rn(av[i], bv[j], acc[i][j]);
-    }
-    if (more) {
-      store(buf ^ 1, na, nb);
-      __syncthreads();
-      buf ^= 1;
-    }
+// A' [m, 6B] from E [m, B] (segments -E1, -E1, -E2, -E1, -E2, -E3)
+__global__ void __launch_bounds__(256) split_e_kernel(const float* __restrict__ E, int64_t m, int B,
+                                                      uint16_t* __restrict__ A) {
+  const int64_t total = m * B;
+  for (int64_t e = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; e < total; e += (int64_t)gridDim.x * blockDim.x) {
+    const int64_t r = e / B;
+    const int k = (int)(e - r * B);
+    uint16_t p[3];
+    split3(-E[e], p);
+    uint16_t* row = A + r * 6 * B + k;
+    row[0] = p[0];
+    row[B] = p[0];
+    row[2 * B] = p[1];
+    row[3 * B] = p[0];
+    row[4 * B] = p[1];
+    row[5 * B] = p[2];
   }
-#pragma unroll
-  for (int i = 0; i < 8; ++i) {
-    const int64_t row = row0 + tr * 8 + i;
-    if (row >= m) continue;
-#pragma unroll
-    for (int half = 0; half < 2; ++half) {
-      const int64_t col = cb + half * 64 + tc * 4;
-      float* dst = W + row * n + col;
-      const float2 lo = acc[i][2 * half], hi = acc[i][2 * half + 1];
-      if (col + 3 < n) {
-        float4 v = *reinterpret_cast<float4*>(dst);
-        v.x -= lo.x; v.y -= lo.y; v.z -= hi.x; v.w -= hi.y;
-        *reinterpret_cast<float4*>(dst) = v;
-      } else {
-        if (col + 0 < n) dst[0] -= lo.x;
-        if (col + 1 < n) dst[1] -= lo.y;
-        if (col + 2 < n) dst[2] -= hi.x;
-      }
+}
+
+// B' [nn, 6B] from U[col0 + k, c1 + j] (segments U1, U2, U1, U3, U2, U1), transposed through
+// 32 x 32 shared-memory tiles so that the reads of U and the writes of B' are coalesced
+__global__ void __launch_bounds__(256) split_u_kernel(const float* __restrict__ U, int64_t n, int64_t col0, int B,
+                                                      int64_t c1, uint16_t* __restrict__ Bt) {
+  __shared__ float t[32][33];
+  const int64_t j0 = (int64_t)blockIdx.x * 32;
+  const int k0 = blockIdx.y * 32;
+  const int tx = threadIdx.x & 31, ty = threadIdx.x >> 5;
+  for (int kk = ty; kk < 32; kk += 8) {
+    const int64_t col = c1 + j0 + tx;
+    t[kk][tx] = (k0 + kk < B && col < n) ? U[(col0 + k0 + kk) * n + col] : 0.0f;
+  }
+  __syncthreads();
+  for (int jj = ty; jj < 32; jj += 8) {
+    const int64_t j = j0 + jj;
+    const int k = k0 + tx;
+    if (c1 + j < n && k < B) {
+      uint16_t p[3];
+      split3(t[tx][jj], p);
+      uint16_t* row = Bt + j * 6 * B + k;
+      row[0] = p[0];
+      row[B] = p[1];
+      row[2 * B] = p[0];
+      row[3 * B] = p[2];
+      row[4 * B] = p[1];
+      row[5 * B] = p[0];
     }
   }
 }
@@ -426,7 +394,8 @@ cudaError_t launch_gptq_factor(const float* H, int64_t n, int64_t ld_h, float da
 
 cudaError_t launch_gptq_hscale(const void* w, int64_t m, int64_t n, const float* U, const float* h,
                                const float* global_scale, const uint8_t* dead, int block, int down, int up,
-                               uint8_t* codes, uint8_t* packed, float* Wf, float* E, cudaStream_t stream) {
+                               uint8_t* codes, uint8_t* packed, float* Wf, float* E, uint16_t* A6, uint16_t* B6,
+                               cudaStream_t stream) {
   DeviceInfo info;
   cudaError_t err = current_device_info(&info);
   if (err != cudaSuccess) return err;
@@ -440,9 +409,15 @@ cudaError_t launch_gptq_hscale(const void* w, int64_t m, int64_t n, const float*
                                          reinterpret_cast<uint2*>(packed), E);
     if ((err = cudaGetLastError()) != cudaSuccess) return err;
     if (col0 + block < n) {
-      const dim3 ug((unsigned)((n - col0 - block + kUT - 1) / kUT), (unsigned)((m + kUT - 1) / kUT));
-      update_kernel<<<ug, 256, 0, stream>>>(Wf, m, n, col0, block, E, U);
+      const int64_t c1 = col0 + block, nn = n - c1;
+      const unsigned eb = (unsigned)std::min<int64_t>((m * block + 255) / 256, (int64_t)info.sm_count * 16);
+      split_e_kernel<<<eb, 256, 0, stream>>>(E, m, block, A6);
       if ((err = cudaGetLastError()) != cudaSuccess) return err;
+      split_u_kernel<<<dim3((unsigned)((nn + 31) / 32), (unsigned)((block + 31) / 32)), 256, 0, stream>>>(
+          U, n, col0, block, c1, B6);
+      if ((err = cudaGetLastError()) != cudaSuccess) return err;
+      if ((err = launch_gemm_accumulate(A6, B6, m, nn, 6 * (int64_t)block, Wf + c1, n, stream)) != cudaSuccess)
+        return err;
     }
   }
   return cudaSuccess;

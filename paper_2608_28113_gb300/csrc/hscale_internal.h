@@ -76,9 +76,15 @@ bool gptq_solver_available();
 size_t gptq_factor_solver_floats(int64_t n);  // 0 if cuSOLVER is unavailable
 cudaError_t launch_gptq_factor(const float* H, int64_t n, int64_t ld_h, float damp, float* U, uint8_t* dead,
                                int32_t* info, float* work, size_t work_floats, cudaStream_t stream);
+// C[m, nn] (row stride ld_c, fp32) += A B^T on the tensor cores, with A [m, k] and B [nn, k]
+// bf16, rows of k elements contiguous (k % 8 == 0, 16-byte aligned bases); every tile.
+cudaError_t launch_gemm_accumulate(const void* a, const void* b, int64_t m, int64_t nn, int64_t k, float* C,
+                                   int64_t ld_c, cudaStream_t stream);
+
 cudaError_t launch_gptq_hscale(const void* w, int64_t m, int64_t n, const float* U, const float* h,
                                const float* global_scale, const uint8_t* dead, int block, int down, int up,
-                               uint8_t* codes, uint8_t* packed, float* Wf, float* E, cudaStream_t stream);
+                               uint8_t* codes, uint8_t* packed, float* Wf, float* E, uint16_t* A6, uint16_t* B6,
+                               cudaStream_t stream);
 
 // Sticky device error flags of each translation unit (bit 0: a bounded wait ran out);
 // cleared on read.

@@ -11,7 +11,7 @@
 //   transpose64_kernel    X [tokens, n] -> X^T [n, tokens] (tokens contiguous per channel),
 //                         16-byte accesses; transpose_kernel is the 2-byte form for X
 //                         whose rows are not 16-byte aligned
-//   gemm_kernel<true>     H += X^T X, the full Hessian of Algorithm 3, with the same tensor-
+//   gemm_kernel<1>        H += X^T X, the full Hessian of Algorithm 3, with the same tensor-
 //                         core pipeline over K = tokens and an epilogue that adds each
 //                         128 x 256 tile of the product into H; tiles wholly below the
 //                         diagonal are skipped (the factor reads the upper triangle only)
@@ -119,10 +119,11 @@ __device__ __forceinline__ float sum_squares32(const uint32_t (&r)[32]) {
   return t[0];
 }
 
-// kAccum = false: the sum-of-squares GEMM of the output error (K runs over [X | X], kb_half
-// blocks per half).  kAccum = true: H[rows, cols] += A B^T over kb_half K blocks, both
-// operands rows of X^T.
-template <bool kAccum>
+// kMode 0: the sum-of-squares GEMM of the output error (K runs over [X | X], kb_half
+// blocks per half).  kMode 1: H[rows, cols] += A B^T over kb_half K blocks, both operands
+// rows of X^T, tiles wholly below the diagonal skipped.  kMode 2: C[rows, cols] += A B^T
+// over kb_half K blocks, every tile (the GPTQ update).
+template <int kMode>
 __global__ void __launch_bounds__(kGemmThreads, 1)
 gemm_kernel(const __grid_constant__ CUtensorMap xmap, const __grid_constant__ CUtensorMap wmap,
             int kb_half, int tiles_n, double* __restrict__ partials, float* __restrict__ H, int64_t h_rows,
@@ -140,10 +141,11 @@ gemm_kernel(const __grid_constant__ CUtensorMap xmap, const __grid_constant__ CU
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int tile_m = blockIdx.x / tiles_n, tile_n = blockIdx.x - tile_m * tiles_n;
+  constexpr bool kAccum = kMode != 0;
   const int kb_total = kAccum ? kb_half : 2 * kb_half;
   // H is symmetric and only its upper triangle is used: a tile wholly below the diagonal
   // (every column index below every row index) is skipped, uniformly for the whole CTA
-  if (kAccum && (int64_t)(tile_n + 1) * kBN <= (int64_t)tile_m * kBM) return;
+  if (kMode == 1 && (int64_t)(tile_n + 1) * kBN <= (int64_t)tile_m * kBM) return;
 
   if (threadIdx.x == 0) {
     for (int s = 0; s < kStages; ++s) {
@@ -415,11 +417,11 @@ cudaError_t launch_output_error(const void* x, int64_t tokens, int64_t n, int64_
       return cudaErrorInvalidValue;
   }
   const cudaError_t attr_status =
-      ensure_dynamic_smem(reinterpret_cast<const void*>(gemm_kernel<false>), (int)kGemmSmemBytes);
+      ensure_dynamic_smem(reinterpret_cast<const void*>(gemm_kernel<0>), (int)kGemmSmemBytes);
   if (attr_status != cudaSuccess) return attr_status;
   const int64_t tiles_n = (m + kBN - 1) / kBN;
   const int64_t tiles = output_error_tiles(tokens, m);
-  gemm_kernel<false><<<(unsigned)tiles, kGemmThreads, kGemmSmemBytes, stream>>>(
+  gemm_kernel<0><<<(unsigned)tiles, kGemmThreads, kGemmSmemBytes, stream>>>(
       xmap, wmap, (int)(n_pad / kBK), (int)tiles_n, partials, nullptr, 0, 0, 0);
   err = cudaGetLastError();
   if (err != cudaSuccess) return err;
@@ -458,12 +460,40 @@ cudaError_t launch_hessian_full(const void* x, int64_t tokens, int64_t n, int64_
              CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) != CUDA_SUCCESS)
     return cudaErrorInvalidValue;
   const cudaError_t attr_status =
-      ensure_dynamic_smem(reinterpret_cast<const void*>(gemm_kernel<true>), (int)kGemmSmemBytes);
+      ensure_dynamic_smem(reinterpret_cast<const void*>(gemm_kernel<1>), (int)kGemmSmemBytes);
   if (attr_status != cudaSuccess) return attr_status;
   const int64_t tiles_n = (n + kBN - 1) / kBN;
   const int64_t tiles = ((n + kBM - 1) / kBM) * tiles_n;
-  gemm_kernel<true><<<(unsigned)tiles, kGemmThreads, kGemmSmemBytes, stream>>>(
+  gemm_kernel<1><<<(unsigned)tiles, kGemmThreads, kGemmSmemBytes, stream>>>(
       amap, bmap, (int)((tokens + kBK - 1) / kBK), (int)tiles_n, nullptr, H, n, n, ld_h);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_gemm_accumulate(const void* a, const void* b, int64_t m, int64_t nn, int64_t k, float* C,
+                                   int64_t ld_c, cudaStream_t stream) {
+  EncodeTiledFn encode = nullptr;
+  cudaError_t err = encode_tiled_fn(&encode);
+  if (err != cudaSuccess) return err;
+  CUtensorMap amap, bmap;
+  const cuuint64_t adims[2] = {(cuuint64_t)k, (cuuint64_t)m};
+  const cuuint64_t bdims[2] = {(cuuint64_t)k, (cuuint64_t)nn};
+  const cuuint64_t strides[1] = {(cuuint64_t)k * 2};
+  const cuuint32_t estr[2] = {1, 1};
+  const cuuint32_t abox[2] = {(cuuint32_t)kBK, (cuuint32_t)kBM};
+  const cuuint32_t bbox[2] = {(cuuint32_t)kBK, (cuuint32_t)kBN};
+  if (encode(&amap, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(a), adims, strides, abox, estr,
+             CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+             CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) != CUDA_SUCCESS ||
+      encode(&bmap, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(b), bdims, strides, bbox, estr,
+             CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+             CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) != CUDA_SUCCESS)
+    return cudaErrorInvalidValue;
+  err = ensure_dynamic_smem(reinterpret_cast<const void*>(gemm_kernel<2>), (int)kGemmSmemBytes);
+  if (err != cudaSuccess) return err;
+  const int64_t tiles_n = (nn + kBN - 1) / kBN;
+  const int64_t tiles = ((m + kBM - 1) / kBM) * tiles_n;
+  gemm_kernel<2><<<(unsigned)tiles, kGemmThreads, kGemmSmemBytes, stream>>>(
+      amap, bmap, (int)((k + kBK - 1) / kBK), (int)tiles_n, nullptr, C, m, nn, ld_c);
   return cudaGetLastError();
 }
 

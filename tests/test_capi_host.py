@@ -211,7 +211,8 @@ def test_gptq_argument_errors(lib):
     assert g(FAKE, 64, 64, -1.0, FAKE, None, FAKE, FAKE, 1 << 20, None) == ERR_ARG
     assert g(FAKE, 64, 64, 0.01, None, None, FAKE, FAKE, 1 << 20, None) == ERR_NULL
     assert g(None, 0, 0, 0.01, None, None, None, None, 0, None) == OK
-    assert lib.hscale_gptq_workspace_bytes(4, 64, 32) == 1536
+    # 4x64 fp32 weights + 4x32 fp32 E + 4x192 and 64x192 bf16 split operands, each rounded to 256 B
+    assert lib.hscale_gptq_workspace_bytes(4, 64, 32) == 1024 + 512 + 1536 + 24576
     q = lib.hscale_gptq_hscale
     assert q(FAKE, 4, 64, FAKE, FAKE, FAKE, None, 24, 4, 4, FAKE, FAKE, FAKE, 1 << 20, None) == ERR_SHAPE
     assert q(FAKE, 4, 64, FAKE, FAKE, FAKE, None, 48, 4, 4, FAKE, FAKE, FAKE, 1 << 20, None) == ERR_SHAPE
