@@ -38,6 +38,7 @@
 //   rule (smaller error, then smaller |shift|, then smaller shift).  The winner's
 //   nibbles are always produced with exact round-to-nearest-even decisions.
 #include <algorithm>
+#include <atomic>
 
 #include "hscale_device.cuh"
 #include "hscale_internal.h"
@@ -565,19 +566,21 @@ __global__ void __launch_bounds__(256) fourover6_codes_kernel(const uint4* __res
   }
 }
 
+// Resident blocks per SM of kKernel at `threads` threads, queried once per device (a race
+// between threads only repeats the query: the cached value is the same either way).
 template <auto kKernel>
 int occupancy_blocks(int threads) {
-  static int cache[64] = {0};
+  static std::atomic<int> cache[64];
   int dev = 0;
   if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) dev = 0;
-  if (cache[dev] == 0) {
-    int blocks = 0;
+  int blocks = cache[dev].load(std::memory_order_relaxed);
+  if (blocks == 0) {
     if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&blocks, kKernel, threads, 0) != cudaSuccess ||
         blocks < 1)
       blocks = 1;
-    cache[dev] = blocks;
+    cache[dev].store(blocks, std::memory_order_relaxed);
   }
-  return cache[dev];
+  return blocks;
 }
 
 }  // namespace
