@@ -8,7 +8,10 @@ RTN codes (Eq. 7) and the H-Scale window search fused with the final re-quantiza
 packing (Algorithm 1).  Default workload: Llama-style 8B q_proj, W [4096, 4096] bf16,
 262144 calibration tokens of width 4096 streamed in 8192-token chunks, window k = +-4.
 Other workloads: the full 8B decoder layer (per-layer and per-model seconds), the MLP
-down_proj, and the 70B MLP block with its window sweep.
+down_proj, and the 70B MLP block with its window sweep.  The timed steps replay CUDA
+graphs on three streams; steps with several input spaces, or whose searches outweigh
+their Hessian passes, are pipelined (a step's last searches alongside the next step's
+first Hessian pass, on alternating buffer sets).
 
 value      groups quantized per second by the whole step (all ranks), inputs in HBM
 e2e        the same through the public API with host buffers: the X chunks and W copied
@@ -70,6 +73,12 @@ def parse():
                         "runs alongside (0: run every search after the last Hessian pass; -1, the "
                         "default: 5 when the step's estimated search time exceeds its Hessian time, "
                         "else 4)")
+    p.add_argument("--pipeline", choices=["auto", "on", "off"], default="auto",
+                   help="run each step's last searches alongside the next step's first Hessian pass "
+                        "(h, s_g and initial codes double-buffered).  auto (default): on when the step "
+                        "has several input spaces or its searches outweigh its Hessian passes (decoder "
+                        "layer -4 %%, 70B MLP block -5 %% per step); off for one Hessian-bound input "
+                        "space (q_proj: -1.5 %% per step, while the Hessian pass shares its SMs)")
     p.add_argument("--no-cpu-baseline", action="store_true")
     p.add_argument("--no-output-error", action="store_true",
                    help="skip the tensor-core layer-output error evaluation")
@@ -295,14 +304,27 @@ class Work:
             jobs.append((S.name, a, b))
         return jobs
 
+    def search_bound(self) -> bool:
+        """Do the step's searches take longer (estimated) than its Hessian passes?"""
+        jobs = self.stage_estimates()
+        return sum(j[2] for j in jobs) > sum(j[1] for j in jobs)
+
+    def pipelined(self, requested: str) -> bool:
+        """Whether consecutive steps overlap: as requested, or by default when the step has
+        several input spaces or is search-bound (there the last searches are a large
+        part of the step; with one Hessian-bound space they are not, and the Hessian pass
+        would share its SMs for a gain of about 1.5 %)."""
+        if requested != "auto":
+            return requested == "on"
+        return len(self.spaces) > 1 or self.search_bound()
+
     def overlap_ctas(self, requested: int) -> int:
         """Search CTAs per SM alongside a Hessian pass: the requested number, or by default
         5 when the searches outweigh the Hessian passes (they should take more of the SM)
         and 4 otherwise (measured best on the 70B MLP block and the 8B decoder layer)."""
         if requested >= 0:
             return requested
-        jobs = self.stage_estimates()
-        return 5 if sum(j[2] for j in jobs) > sum(j[1] for j in jobs) else 4
+        return 5 if self.search_bound() else 4
 
     def space_order(self):
         """The input spaces in the order the step takes them.  Each space is a two-stage
@@ -399,69 +421,121 @@ class StepGraphs:
             ALU-bound), started as soon as the piece's h is complete and the weight-only
             calls are done, so that they run alongside the next piece's Hessian pass.
             Those searches keep at most `overlap_ctas` CTAs resident per SM, which leaves
-            registers for the Hessian CTAs; the last piece's searches fill the GPU.
-            overlap_ctas = 0 runs every search after the last Hessian pass instead."""
+            registers for the Hessian CTAs.  overlap_ctas = 0 runs every search after the
+            last Hessian pass instead.
 
-    def __init__(self, hs, work: Work, overlap_ctas: int):
+    pipelined (when asked for and overlap_ctas > 0): consecutive steps overlap as well, so
+    the last piece's searches run alongside the next step's first Hessian pass.  The
+    buffers that one step's streams hand to each other -- h of every input space; s_g
+    and the two-pass 4over6 codes of every matrix -- come in two sets, taken by
+    alternate steps, and a step starts its Hessian passes and weight-only calls only
+    once the searches of the step before the previous one, which read the same set, are
+    done.  Without pipelining the last piece's searches fill the GPU and the step ends
+    when they do."""
+
+    def __init__(self, hs, work: Work, overlap_ctas: int, pipeline: bool = True):
         self.work, self.overlap = work, overlap_ctas > 0
-        warm = torch.cuda.Stream()
-        warm.wait_stream(torch.cuda.current_stream())
-        with torch.cuda.stream(warm):
-            run_step(hs, work)
-        torch.cuda.current_stream().wait_stream(warm)
-        torch.cuda.synchronize()
+        self.pipeline = pipeline and self.overlap
+        spaces = list(work.spaces.values())
+        self.sets = [({S.name: S.h for S in spaces}, {M.name: (M.sg, M.codes0) for M in work.mats})]
+        if self.pipeline:
+            self.sets.append(({S.name: torch.zeros_like(S.h) for S in spaces},
+                              {M.name: (torch.empty_like(M.sg), torch.empty_like(M.codes0))
+                               for M in work.mats}))
         down, up = work.win
-        self.gh, self.gr = [], []
-        for i, (S, c0, c1) in enumerate(work.pieces):
-            g = torch.cuda.CUDAGraph()
-            with torch.cuda.graph(g):
-                hessian_block(hs, S, c0, c1)
-            self.gh.append(g)
-            ctas = overlap_ctas if (self.overlap and i + 1 < len(work.pieces)) else 0
-            g = torch.cuda.CUDAGraph()
-            with torch.cuda.graph(g):
-                for M in work.mats:
-                    if M.space is S:
-                        refine_block(hs, work, M, c0, c1, down, up, ctas_per_sm=ctas)
-            self.gr.append(g)
-        self.gi = torch.cuda.CUDAGraph()
-        with torch.cuda.graph(self.gi):
-            init_phase(hs, work)
+        self.gh, self.gr, self.gi = [], [], []
+        for p in range(len(self.sets)):
+            self.bind(p)
+            warm = torch.cuda.Stream()
+            warm.wait_stream(torch.cuda.current_stream())
+            with torch.cuda.stream(warm):
+                run_step(hs, work)
+            torch.cuda.current_stream().wait_stream(warm)
+            torch.cuda.synchronize()
+            gh, gr = [], []
+            for i, (S, c0, c1) in enumerate(work.pieces):
+                g = torch.cuda.CUDAGraph()
+                with torch.cuda.graph(g):
+                    hessian_block(hs, S, c0, c1)
+                gh.append(g)
+                alongside = self.overlap and (self.pipeline or i + 1 < len(work.pieces))
+                g = torch.cuda.CUDAGraph()
+                with torch.cuda.graph(g):
+                    for M in work.mats:
+                        if M.space is S:
+                            refine_block(hs, work, M, c0, c1, down, up,
+                                         ctas_per_sm=overlap_ctas if alongside else 0)
+                gr.append(g)
+            gi = torch.cuda.CUDAGraph()
+            with torch.cuda.graph(gi):
+                init_phase(hs, work)
+            self.gh.append(gh)
+            self.gr.append(gr)
+            self.gi.append(gi)
+        self.bind(0)
         torch.cuda.synchronize()
         self.side, self.search = torch.cuda.Stream(), torch.cuda.Stream()
         self.ev_init = torch.cuda.Event()
         self.ev_h = [torch.cuda.Event() for _ in work.pieces]
+        self.done = [torch.cuda.Event() for _ in self.sets]
+        self.used = [False for _ in self.sets]
+        self.k = 0
+
+    def bind(self, p: int):
+        """Points the work's spaces and matrices at buffer set p."""
+        hset, mset = self.sets[p]
+        for S in self.work.spaces.values():
+            S.h = hset[S.name]
+        for M in self.work.mats:
+            M.sg, M.codes0 = mset[M.name]
 
     def replay(self, ev=None):
-        """One step.  ev: optional (start, after the last Hessian pass, end) timing events
-        recorded on the current stream, which runs the Hessian passes."""
+        """One step.  ev: optional (start, after the last Hessian pass, end of the step's
+        searches) timing events; the first two are recorded on the current stream, which
+        runs the Hessian passes, the last on the search stream when pipelined.  A
+        pipelined step may still be running when this returns: drain() joins it."""
         main = torch.cuda.current_stream()
+        p = self.k % len(self.sets)
+        self.k += 1
         if ev:
             ev[0].record()
+        if self.pipeline and self.used[p]:
+            main.wait_event(self.done[p])
         self.side.wait_stream(main)
         self.search.wait_stream(main)
         with torch.cuda.stream(self.side):
-            self.gi.replay()
+            self.gi[p].replay()
             self.ev_init.record(self.side)
         self.search.wait_event(self.ev_init)
-        for i, g in enumerate(self.gh):
+        for i, g in enumerate(self.gh[p]):
             g.replay()
             self.ev_h[i].record(main)
             if self.overlap:
                 self.search.wait_event(self.ev_h[i])
                 with torch.cuda.stream(self.search):
-                    self.gr[i].replay()
+                    self.gr[p][i].replay()
         if ev:
             ev[1].record()
         if not self.overlap:
             self.search.wait_stream(main)
             with torch.cuda.stream(self.search):
-                for g in self.gr:
+                for g in self.gr[p]:
                     g.replay()
+        if self.pipeline:
+            self.done[p].record(self.search)
+            self.used[p] = True
+            if ev:
+                ev[2].record(self.search)
+        else:
+            self.drain()
+            if ev:
+                ev[2].record()
+
+    def drain(self):
+        """Joins every stream of the steps replayed so far into the current stream."""
+        main = torch.cuda.current_stream()
         main.wait_stream(self.search)
         main.wait_stream(self.side)
-        if ev:
-            ev[2].record()
 
 
 # algorithmic bytes per group of the search: W 32, nibbles 8, code out 1, code in 1 (none
@@ -775,9 +849,10 @@ def gpu_arm(args, d: Dist):
 
     # timed region: the same launches replayed from CUDA graphs
     args.overlap_ctas = work.overlap_ctas(args.overlap_ctas)
-    graphs = StepGraphs(hs, work, args.overlap_ctas)
+    graphs = StepGraphs(hs, work, args.overlap_ctas, pipeline=work.pipelined(args.pipeline))
     for _ in range(warm):
         graphs.replay()
+    graphs.drain()
     evs = [[torch.cuda.Event(enable_timing=True) for _ in range(3)] for _ in range(args.steps)]
     d.barrier()
     torch.cuda.synchronize()
@@ -787,6 +862,7 @@ def gpu_arm(args, d: Dist):
         t0.record()
         for s in range(args.steps):
             graphs.replay(evs[s])
+        graphs.drain()
         t1.record()
         torch.cuda.synchronize()
     d.barrier()
@@ -803,7 +879,7 @@ def gpu_arm(args, d: Dist):
     fp32_peak = props.multi_processor_count * 128 * sm_max_mhz * 1e6
     reps = max(3, min(args.steps, 20))
     ms_init = sum(timed(lambda M=M: init_codes(hs, work, M), reps) for M in work.mats)
-    ms_h_alone = timed(lambda: [g.replay() for g in graphs.gh], reps)
+    ms_h_alone = timed(lambda: [g.replay() for g in graphs.gh[0]], reps)
     sweep = []
     windows = sorted(set([win] + [(kk, kk) for kk in W.window]))
     for dn, upw in windows:
@@ -881,6 +957,7 @@ def gpu_arm(args, d: Dist):
                    "input_spaces": [[S.name, S.tokens, S.n, S.chunk] for S in work.spaces.values()],
                    "window": list(win), "init": work.init, "groups": work.groups,
                    "col_block": work.col_block,
+                   "schedule": "pipelined" if graphs.pipeline else "sequential",
                    "l2": "inputs larger than L2: %.2f GB of X streamed per step" %
                          (sum(S.tokens * S.n * 2 for S in work.spaces.values()) / 1e9),
                    "parallelism": f"independent layer per GPU x{d.world}"},
@@ -895,7 +972,10 @@ def gpu_arm(args, d: Dist):
                          + ("each block" if work.col_block else "each input space")
                          + " as soon as its h is complete"
                          + (f" (at most {args.overlap_ctas} search CTAs per SM while a Hessian pass runs)"
-                            if args.overlap_ctas > 0 and len(work.pieces) > 1 else "")),
+                            if args.overlap_ctas > 0 and (len(work.pieces) > 1 or graphs.pipeline) else "")
+                         + ("; consecutive steps pipelined: each step's last searches run alongside the next "
+                            "step's first Hessian pass (h, s_g and initial codes double-buffered); the timed "
+                            "region ends when the last step's searches are done" if graphs.pipeline else "")),
         "hessian": {"gbs": h_gbs, "tokens_channels_per_s": work.h_bytes / 2 / (ms_h * 1e-3),
                     "frac_of_measured_hbm": h_gbs / hbm_peak, "frac_of_8TBs": h_gbs / HBM_SPEC_GBS},
         "search": {"groups_per_s": main["groups_per_s"], "candidates": main["candidates"],
