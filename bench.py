@@ -71,13 +71,14 @@ def parse():
     p.add_argument("--overlap-ctas", type=int, default=-1,
                    help="resident search CTAs per SM while the next input space's Hessian pass "
                         "runs alongside (0: run every search after the last Hessian pass; -1, the "
-                        "default: 5 when the step's estimated search time exceeds its Hessian time, "
-                        "else 4)")
+                        "default: when the step's estimated search time exceeds its Hessian time, 7 "
+                        "(every CTA the search kernel keeps resident) with pipelined steps and 5 "
+                        "without; else 4)")
     p.add_argument("--pipeline", choices=["auto", "on", "off"], default="auto",
                    help="run each step's last searches alongside the next step's first Hessian pass "
                         "(h, s_g and initial codes double-buffered).  auto (default): on when the step "
                         "has several input spaces or its searches outweigh its Hessian passes (decoder "
-                        "layer -4 %%, 70B MLP block -5 %% per step); off for one Hessian-bound input "
+                        "layer -4 %%, 70B MLP block -11 %% per step); off for one Hessian-bound input "
                         "space (q_proj: -1.5 %% per step, while the Hessian pass shares its SMs)")
     p.add_argument("--no-cpu-baseline", action="store_true")
     p.add_argument("--no-output-error", action="store_true",
@@ -318,13 +319,18 @@ class Work:
             return requested == "on"
         return len(self.spaces) > 1 or self.search_bound()
 
-    def overlap_ctas(self, requested: int) -> int:
+    def overlap_ctas(self, requested: int, pipelined: bool) -> int:
         """Search CTAs per SM alongside a Hessian pass: the requested number, or by default
-        5 when the searches outweigh the Hessian passes (they should take more of the SM)
-        and 4 otherwise (measured best on the 70B MLP block and the 8B decoder layer)."""
+        4 when the Hessian passes outweigh the searches (8B decoder layer: 1.31 ms, against
+        1.34 at 3 and 1.44 at 5).  When the searches outweigh them they should take more of
+        the SM: 7, every CTA the search kernel keeps resident, with pipelined steps (70B MLP
+        block: 2.14 ms, against 2.19 at 6 and 2.29 at 5), and 5 without (2.39 ms, against
+        2.54 at 4).  The launcher clamps a larger number to the kernel's occupancy."""
         if requested >= 0:
             return requested
-        return 5 if self.search_bound() else 4
+        if not self.search_bound():
+            return 4
+        return 7 if pipelined else 5
 
     def space_order(self):
         """The input spaces in the order the step takes them.  Each space is a two-stage
@@ -848,8 +854,9 @@ def gpu_arm(args, d: Dist):
     ms_eager = timed(lambda: run_step(hs, work), args.steps)
 
     # timed region: the same launches replayed from CUDA graphs
-    args.overlap_ctas = work.overlap_ctas(args.overlap_ctas)
-    graphs = StepGraphs(hs, work, args.overlap_ctas, pipeline=work.pipelined(args.pipeline))
+    pipelined = work.pipelined(args.pipeline)
+    args.overlap_ctas = work.overlap_ctas(args.overlap_ctas, pipelined)
+    graphs = StepGraphs(hs, work, args.overlap_ctas, pipeline=pipelined)
     for _ in range(warm):
         graphs.replay()
     graphs.drain()
