@@ -607,7 +607,7 @@ def _oracle_step(W: wl.Workload, win, budget_s: float, init: str, threads: int):
         step += t_tc * W.tokens * n
         h_tc += W.tokens * n
         hs_of[name] = (h / reps * (W.tokens / tok)).astype(np.float32)
-        samples.append(f"Hessian {name}: {reps} x {tok}x{n}")
+        samples.append(f"Hessian {name}: {reps} passes over one {tok}-token x {n}-channel chunk")
     t_rtn_total = 0.0
     for L in W.layers:
         m, n = L.out_features, L.in_features
@@ -629,7 +629,7 @@ def _oracle_step(W: wl.Workload, win, budget_s: float, init: str, threads: int):
         G = m * n // 16
         step += t_g * G
         groups += G
-        samples.append(f"search {L.name}: {done}x{rows} rows")
+        samples.append(f"search {L.name}: {done} batches of {rows} rows")
     step += t_rtn_total
     return step, groups, samples, h_tc
 
