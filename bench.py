@@ -740,12 +740,15 @@ def gptq_eval(hs, work: Work, peaks: dict, block: int = 128, reps: int = 3):
     n, m = M.n, M.m
     down, up = work.win
     H = torch.zeros(n, n, dtype=torch.float32, device=dev)
-    hws = torch.empty(max(256, hs.hscale_hessian_full_workspace_bytes(S.chunk, n)), dtype=torch.uint8, device=dev)
+    # calls of up to 65536 tokens: the kernel accumulates 2048-token segments whatever the
+    # call, so larger calls cost no accuracy and save per-launch work
+    call = min(S.tokens, 65536)
+    hws = torch.empty(max(256, hs.hscale_hessian_full_workspace_bytes(call, n)), dtype=torch.uint8, device=dev)
 
     def hessian():
         H.zero_()
-        for c in range(S.nchunks):
-            hs.hscale_hessian_full_accumulate(S.x[c * S.chunk:(c + 1) * S.chunk], H, hws)
+        for t0 in range(0, S.tokens, call):
+            hs.hscale_hessian_full_accumulate(S.x[t0:t0 + call], H, hws)
 
     ms_h = timed(hessian, reps)
     U = torch.empty(n, n, dtype=torch.float32, device=dev)
@@ -786,7 +789,8 @@ def gptq_eval(hs, work: Work, peaks: dict, block: int = 128, reps: int = 3):
             "hessian_full_ms": ms_h, "hessian_full_tflops": h_flop / (ms_h * 1e-3) / 1e12,
             "hessian_full_note": "dense-equivalent 2 T n^2 FLOP; tiles wholly below the diagonal are skipped, "
                                  "so the computed-tile rate below is the one to compare with the peak; the time "
-                                 "includes the transpose of every chunk",
+                                 "includes the transpose of every call's tokens",
+            "hessian_full_tokens_per_call": call,
             "hessian_full_tflops_computed": h_flop_done / (ms_h * 1e-3) / 1e12,
             "hessian_full_frac_of_measured_bf16": h_flop_done / (ms_h * 1e-3) / 1e12 / peak,
             "factor_ms": ms_f, "block_loop_ms": ms_q, "update_gemm_gflop": upd_flop / 1e9,

@@ -14,7 +14,9 @@
 //   gemm_kernel<1>        H += X^T X, the full Hessian of Algorithm 3, with the same tensor-
 //                         core pipeline over K = tokens and an epilogue that adds each
 //                         128 x 256 tile of the product into H; tiles wholly below the
-//                         diagonal are skipped (the factor reads the upper triangle only)
+//                         diagonal are skipped (the factor reads the upper triangle only).
+//                         K runs in segments of 2048 tokens, each accumulated from zero and
+//                         folded into a running sum in tensor memory
 //
 // The residual is rounded once (one FMA of the exact w - s_g * (l q)), and hi + lo carries
 // it to a relative 2^-17, so the GEMM sees dW, not a difference of two large products.
@@ -42,6 +44,15 @@ constexpr uint32_t kTileABytes = kBM * kBK * 2;  // 16 KB
 constexpr uint32_t kTileBBytes = kBN * kBK * 2;  // 32 KB
 constexpr uint32_t kStageBytes = kTileABytes + kTileBBytes;
 constexpr uint32_t kTmemCols = kBN;  // fp32 accumulator: 128 lanes x 256 columns
+// Full Hessian (mode 1): the tensor cores accumulate in fp32 with an error that grows with
+// the accumulation length (the diagonal comes out low by about 0.9 u per K = 16 step,
+// measured), so each tile's K loop is cut into segments of kSegBlocks K blocks (2048
+// tokens).  Each segment accumulates from zero in TMEM columns [0, 256); the epilogue warps
+// add it in fp32 round-to-nearest into a running sum kept in TMEM columns [256, 512), and
+// add the running sum into H after the last segment.  With H = 0 before the call the
+// result is bit for bit that of successive calls of 2048 tokens, whatever the call size.
+constexpr int kSegBlocks = 32;
+constexpr uint32_t kTmemColsSeg = 2 * kBN;
 constexpr uint32_t kGemmSmemBytes = kStages * kStageBytes + 1024 /* alignment */ + 256 /* barriers */;
 constexpr uint32_t kIdesc = idesc_bf16_f32(kBM, kBN);
 
@@ -137,7 +148,10 @@ gemm_kernel(const __grid_constant__ CUtensorMap xmap, const __grid_constant__ CU
   uint64_t* acc_ready = empty + kStages;
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(acc_ready + 1);
   uint32_t* failed = tmem_slot + 1;
+  uint64_t* seg_full = acc_ready + 2;  // mode 1: the partial of a segment is complete
+  uint64_t* seg_empty = seg_full + 1;  // mode 1: the partial has been folded into the sum
   double* warp_sum = reinterpret_cast<double*>(smem + kStages * kStageBytes + 128);
+  constexpr uint32_t kCols = kMode == 1 ? kTmemColsSeg : kTmemCols;
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int tile_m = blockIdx.x / tiles_n, tile_n = blockIdx.x - tile_m * tiles_n;
@@ -153,13 +167,15 @@ gemm_kernel(const __grid_constant__ CUtensorMap xmap, const __grid_constant__ CU
       mbar_init(&empty[s], 1);
     }
     mbar_init(acc_ready, 1);
+    mbar_init(seg_full, 1);
+    mbar_init(seg_empty, 128);  // every epilogue thread arrives
     *failed = 0u;
     mbar_fence_init();
     prefetch_tensormap(&xmap);
     prefetch_tensormap(&wmap);
   }
   if (warp == 1) {
-    tmem_alloc(smem_addr(tmem_slot), kTmemCols);
+    tmem_alloc(smem_addr(tmem_slot), kCols);
     tmem_relinquish();
   }
   tc_fence_before_sync();
@@ -186,37 +202,74 @@ gemm_kernel(const __grid_constant__ CUtensorMap xmap, const __grid_constant__ CU
     }
   } else if (warp == 1) {
     if (lane == 0) {
-      int issued = 0;
-      for (int kb = 0; kb < kb_total; ++kb) {
-        const int s = kb % kStages;
-        const uint32_t round = (uint32_t)(kb / kStages);
-        if (!mbar_wait(&full[s], round & 1u)) {
+      // mode 1: segments of kSegBlocks K blocks, each accumulated from zero; the other
+      // modes: one segment over the whole K loop
+      const int seg_blocks = kMode == 1 ? kSegBlocks : (kb_total > 0 ? kb_total : 1);
+      const int nseg = (kb_total + seg_blocks - 1) / seg_blocks;
+      bool ok = true;
+      for (int seg = 0; seg < nseg && ok; ++seg) {
+        // the previous segment's partial must have been read out of TMEM
+        if (kMode == 1 && seg >= 1 && !mbar_wait(seg_empty, (uint32_t)(seg - 1) & 1u)) {
           atomicOr(failed, 1u);
           break;
         }
         tc_fence_after_sync();
-        const uint64_t ad = smem_desc_k_sw128(smem_addr(tile_a + s * kTileABytes));
-        const uint64_t bd = smem_desc_k_sw128(smem_addr(tile_b + s * kTileBBytes));
+        const uint32_t d = tmem_d;
+        const int kb0 = seg * seg_blocks, kb1 = min(kb_total, kb0 + seg_blocks);
+        for (int kb = kb0; kb < kb1; ++kb) {
+          const int s = kb % kStages;
+          const uint32_t round = (uint32_t)(kb / kStages);
+          if (!mbar_wait(&full[s], round & 1u)) {
+            atomicOr(failed, 1u);
+            ok = false;
+            break;
+          }
+          tc_fence_after_sync();
+          const uint64_t ad = smem_desc_k_sw128(smem_addr(tile_a + s * kTileABytes));
+          const uint64_t bd = smem_desc_k_sw128(smem_addr(tile_b + s * kTileBBytes));
 #pragma unroll
-        for (int kk = 0; kk < kBK / 16; ++kk)
-          umma_bf16(tmem_d, ad + 2 * kk, bd + 2 * kk, kIdesc, (uint32_t)(issued++ > 0));
-        umma_commit(smem_addr(&empty[s]));
+          for (int kk = 0; kk < kBK / 16; ++kk)
+            umma_bf16(d, ad + 2 * kk, bd + 2 * kk, kIdesc, (uint32_t)(kb > kb0 || kk > 0));
+          umma_commit(smem_addr(&empty[s]));
+        }
+        // fires once every MMA issued above has completed
+        if (ok) umma_commit(smem_addr(kMode == 1 ? seg_full : acc_ready));
       }
-      umma_commit(smem_addr(acc_ready));  // fires once every MMA issued above has completed
     }
     __syncwarp();
   } else if (kAccum) {
-    // row of H held by this thread (TMEM lane = row of the tile), 32 columns at a time
+    // row of H held by this thread (TMEM lane = row of the tile), 32 columns at a time;
+    // mode 1 folds every segment's partial into the running sum and adds the sum into H
+    // after the last one
     const uint32_t quarter = (uint32_t)(warp & 3);
     const int64_t row = (int64_t)tile_m * kBM + quarter * 32 + lane;
     const int64_t col0 = (int64_t)tile_n * kBN;
-    if (mbar_wait(acc_ready, 0u)) {
+    const uint32_t lane_base = (quarter * 32u) << 16;
+    const int nseg = kMode == 1 ? (kb_total + kSegBlocks - 1) / kSegBlocks : 1;
+    for (int seg = 0; seg < nseg; ++seg) {
+      if (!mbar_wait(kMode == 1 ? seg_full : acc_ready, kMode == 1 ? (uint32_t)seg & 1u : 0u)) {
+        atomicOr(failed, 1u);
+        break;
+      }
       tc_fence_after_sync();
+      const bool last = seg + 1 == nseg;
 #pragma unroll 1
       for (int c0 = 0; c0 < kBN; c0 += 32) {
         uint32_t r[32];
-        tmem_ld_32x32b_x32(tmem_d + ((quarter * 32u) << 16) + (uint32_t)c0, r);
-        tmem_ld_wait();
+        tmem_ld_32x32b_x32(tmem_d + lane_base + (uint32_t)c0, r);
+        if (kMode == 1 && seg > 0) {
+          uint32_t q[32];
+          tmem_ld_32x32b_x32(tmem_d + lane_base + kBN + (uint32_t)c0, q);
+          tmem_ld_wait();
+#pragma unroll
+          for (int j = 0; j < 32; ++j) r[j] = __float_as_uint(__fadd_rn(__uint_as_float(q[j]), __uint_as_float(r[j])));
+        } else {
+          tmem_ld_wait();
+        }
+        if (kMode == 1 && !last) {
+          tmem_st_32x32b_x32(tmem_d + lane_base + kBN + (uint32_t)c0, r);
+          continue;
+        }
         if (row < h_rows) {
           float* dst = H + row * ld_h + col0 + c0;
           if (col0 + c0 + 32 <= h_cols && ((ld_h | (col0 + c0)) & 3) == 0 &&
@@ -235,8 +288,12 @@ gemm_kernel(const __grid_constant__ CUtensorMap xmap, const __grid_constant__ CU
           }
         }
       }
-    } else {
-      atomicOr(failed, 1u);
+      if (kMode == 1 && !last) {
+        // the partial has been read and the running sum written: the MMAs may go on
+        tmem_st_wait();
+        tc_fence_before_sync();
+        mbar_arrive(seg_empty);
+      }
     }
   } else {
     const uint32_t quarter = (uint32_t)(warp & 3);
@@ -279,7 +336,7 @@ gemm_kernel(const __grid_constant__ CUtensorMap xmap, const __grid_constant__ CU
   }
   if (warp == 1) {
     tc_fence_after_sync();
-    tmem_dealloc(tmem_d, kTmemCols);
+    tmem_dealloc(tmem_d, kCols);
   }
 }
 

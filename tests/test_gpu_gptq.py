@@ -53,10 +53,15 @@ def oracle_H(x, n):
 
 @pytest.mark.parametrize("tokens,n,chunks,view", [(128, 256, 1, "whole"), (300, 200, 1, "whole"),
                                                   (1000, 520, 2, "whole"), (77, 131, 1, "whole"),
-                                                  (200, 96, 2, "aligned slice"), (150, 72, 1, "odd slice")])
+                                                  (200, 96, 2, "aligned slice"), (150, 72, 1, "odd slice"),
+                                                  (4500, 136, 1, "whole"), (9000, 264, 2, "whole"),
+                                                  (65536, 256, 1, "whole")])
 def test_full_hessian_matches_oracle(tokens, n, chunks, view):
     """Whole X, a ragged width (n % 8 != 0), a 16-byte aligned column slice of a wider X
-    (ld_x > n) and a slice starting at an odd column (the 2-byte transpose path)."""
+    (ld_x > n) and a slice starting at an odd column (the 2-byte transpose path); calls
+    of several 2048-token accumulation segments with a ragged last one; and one call of
+    65536 tokens, whose error stays that of a 2048-token segment (one long fp32
+    accumulation on the tensor cores would be 30x over the bound there)."""
     x = calib(n, tokens, 60 + n)
     ref = oracle_H(x, n)
     if view == "whole":
@@ -75,6 +80,21 @@ def test_full_hessian_matches_oracle(tokens, n, chunks, view):
     scale = np.sqrt(np.outer(np.diag(ref), np.diag(ref)))
     err = np.triu(np.abs(got - ref))        # the upper triangle is the accumulated part
     assert np.all(err <= 1e-5 * scale + 1e-30), f"max scaled err {np.max(err / (scale + 1e-300)):.2e}"
+    assert hs.hscale_device_error_flags() == 0
+
+
+def test_full_hessian_one_call_equals_2048_token_calls():
+    """The kernel's accumulation segments: one call over 12,000 tokens gives, bit for bit,
+    the H of successive calls of 2048 tokens (the last one ragged)."""
+    n, tokens = 384, 12000
+    x = calib(n, tokens, 91).to(dev())
+    H1 = torch.zeros(n, n, dtype=torch.float32, device=dev())
+    H2 = torch.zeros_like(H1)
+    hs.hscale_hessian_full_accumulate(x, H1)
+    for t0 in range(0, tokens, 2048):
+        hs.hscale_hessian_full_accumulate(x[t0:t0 + 2048], H2)
+    torch.cuda.synchronize()
+    assert torch.equal(torch.triu(H1), torch.triu(H2))
     assert hs.hscale_device_error_flags() == 0
 
 
