@@ -740,15 +740,15 @@ def gptq_eval(hs, work: Work, peaks: dict, block: int = 128, reps: int = 3):
     n, m = M.n, M.m
     down, up = work.win
     H = torch.zeros(n, n, dtype=torch.float32, device=dev)
-    # calls of up to 65536 tokens: the kernel accumulates 2048-token segments whatever the
-    # call, so larger calls cost no accuracy and save per-launch work
-    call = min(S.tokens, 65536)
-    hws = torch.empty(max(256, hs.hscale_hessian_full_workspace_bytes(call, n)), dtype=torch.uint8, device=dev)
+    # one call over every token: the kernel accumulates 2048-token segments whatever the
+    # call, so a large call costs no accuracy and saves per-launch work; X's rows are
+    # 16-byte aligned, so it is read as it is (no workspace)
+    call = S.tokens
 
     def hessian():
         H.zero_()
         for t0 in range(0, S.tokens, call):
-            hs.hscale_hessian_full_accumulate(S.x[t0:t0 + call], H, hws)
+            hs.hscale_hessian_full_accumulate(S.x[t0:t0 + call], H)
 
     ms_h = timed(hessian, reps)
     U = torch.empty(n, n, dtype=torch.float32, device=dev)
@@ -788,8 +788,8 @@ def gptq_eval(hs, work: Work, peaks: dict, block: int = 128, reps: int = 3):
     return {"matrix": M.name, "block": block, "window": [down, up], "tokens": S.tokens,
             "hessian_full_ms": ms_h, "hessian_full_tflops": h_flop / (ms_h * 1e-3) / 1e12,
             "hessian_full_note": "dense-equivalent 2 T n^2 FLOP; tiles wholly below the diagonal are skipped, "
-                                 "so the computed-tile rate below is the one to compare with the peak; the time "
-                                 "includes the transpose of every call's tokens",
+                                 "so the computed-tile rate below is the one to compare with the peak; X is read "
+                                 "as it is (MN-major operand tiles, no transpose)",
             "hessian_full_tokens_per_call": call,
             "hessian_full_tflops_computed": h_flop_done / (ms_h * 1e-3) / 1e12,
             "hessian_full_frac_of_measured_bf16": h_flop_done / (ms_h * 1e-3) / 1e12 / peak,

@@ -326,8 +326,10 @@ int hscale_output_error(const void* x_bf16, int64_t tokens, int64_t n, int64_t l
  *    a zeroed H equals successive 2048-token calls bit for bit.  Large calls are faster.  H is symmetric and only its upper triangle (j >= i) is
  *    accumulated and read later: 128 x 256 tiles wholly below the diagonal are not
  *    written, those crossing it are written in full.  x is [tokens, ld_x] bf16 row-major
- *    (2-byte aligned); the workspace (hscale_hessian_full_workspace_bytes, 256-byte
- *    aligned) holds X^T.
+ *    (2-byte aligned).  When x is 16-byte aligned and ld_x a multiple of 8 the tensor
+ *    cores read X as it is (MN-major operand tiles) and the workspace may be NULL; other X
+ *    is first transposed into the workspace (hscale_hessian_full_workspace_bytes, 256-byte
+ *    aligned), which then must be given.
  *
  * 2. hscale_gptq_factor: the damped inverse-Cholesky factor, formed as GPTQ forms it.
  *    Only the upper triangle of H (j >= i) is read.  Channels with H_jj = 0 are dead (dead[j] = 1 if dead is not NULL; their weights are

@@ -375,17 +375,22 @@ def _workspace(nbytes: int, device) -> torch.Tensor:
 
 def hscale_hessian_full_accumulate(x: torch.Tensor, H: torch.Tensor, workspace: torch.Tensor | None = None,
                                    stream=None) -> None:
-    """Upper triangle of H (fp32 [n, n]) += X^T X for x [tokens, n] bf16 on the tensor cores."""
+    """Upper triangle of H (fp32 [n, n]) += X^T X for x [tokens, n] bf16 on the tensor cores.
+    A workspace is needed (and allocated here if not given) only for x whose rows are not
+    16-byte aligned."""
     _need(x, torch.bfloat16, "x")
     _need(H, torch.float32, "H")
     if x.dim() != 2 or x.stride(1) != 1 or H.dim() != 2 or H.stride(1) != 1:
         raise ValueError("x and H must be 2-D with unit column stride")
     tokens, n = x.shape
-    if workspace is None:
+    direct = x.data_ptr() % 16 == 0 and x.stride(0) % 8 == 0
+    if workspace is None and not direct:
         workspace = _workspace(load().hscale_hessian_full_workspace_bytes(tokens, n), x.device)
     _check("hscale_hessian_full_accumulate",
-           load().hscale_hessian_full_accumulate(_ptr(x), tokens, n, x.stride(0), _ptr(H), H.stride(0), _ptr(workspace),
-                                                 workspace.numel(), _stream_ptr(stream)))
+           load().hscale_hessian_full_accumulate(_ptr(x), tokens, n, x.stride(0), _ptr(H), H.stride(0),
+                                                 _ptr(workspace) if workspace is not None else None,
+                                                 workspace.numel() if workspace is not None else 0,
+                                                 _stream_ptr(stream)))
 
 
 def hscale_gptq_factor(H: torch.Tensor, damp: float, U: torch.Tensor, dead: torch.Tensor | None,

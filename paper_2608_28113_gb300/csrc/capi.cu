@@ -234,8 +234,10 @@ int hscale_hessian_full_accumulate(const void* x_bf16, int64_t tokens, int64_t n
   if (tokens > INT32_MAX || n > INT32_MAX || tokens > INT64_MAX / ld_x || n > INT64_MAX / ld_h) return HSCALE_ERR_SHAPE;
   if (x_bf16 == nullptr || H == nullptr) return HSCALE_ERR_NULL;
   if (!aligned(x_bf16, 2) || !aligned(H, 4)) return HSCALE_ERR_ALIGN;
-  if (workspace == nullptr || workspace_bytes < hscale_hessian_full_workspace_bytes(tokens, n) ||
-      !aligned(workspace, 256))
+  // X with 16-byte aligned rows is read as it is; other X is transposed into the workspace
+  const bool direct = aligned(x_bf16, 16) && ld_x % 8 == 0;
+  if (!direct && (workspace == nullptr || workspace_bytes < hscale_hessian_full_workspace_bytes(tokens, n) ||
+                  !aligned(workspace, 256)))
     return HSCALE_ERR_WORKSPACE;
   return from_cuda(hscale::launch_hessian_full(x_bf16, tokens, n, ld_x, H, ld_h, workspace, as_stream(stream)));
 }

@@ -8,15 +8,16 @@
 //                         operands, fp32 accumulation in tensor memory), fused with the sum of
 //                         squares of C: one fp64 partial per 128 x 256 tile of C
 //   reduce_kernel         the partials summed in tile order, added to the caller's scalar
-//   transpose64_kernel    X [tokens, n] -> X^T [n, tokens] (tokens contiguous per channel),
-//                         16-byte accesses; transpose_kernel is the 2-byte form for X
-//                         whose rows are not 16-byte aligned
-//   gemm_kernel<1>        H += X^T X, the full Hessian of Algorithm 3, with the same tensor-
-//                         core pipeline over K = tokens and an epilogue that adds each
-//                         128 x 256 tile of the product into H; tiles wholly below the
-//                         diagonal are skipped (the factor reads the upper triangle only).
-//                         K runs in segments of 2048 tokens, each accumulated from zero and
-//                         folded into a running sum in tensor memory
+//   gemm_kernel<3>        H += X^T X, the full Hessian of Algorithm 3, with the same tensor-
+//                         core pipeline over K = tokens, reading X as it is (both operands
+//                         MN-major), and an epilogue that adds each 128 x 256 tile of the
+//                         product into H; tiles wholly below the diagonal are skipped (the
+//                         factor reads the upper triangle only).  K runs in segments of 2048
+//                         tokens, each accumulated from zero and folded into a running sum
+//                         in tensor memory
+//   transpose_kernel,     the same for X whose rows are not 16-byte aligned (no TMA): X is
+//   gemm_kernel<1>        transposed into the workspace (tokens contiguous per channel)
+//                         and both operands are K-major
 //
 // The residual is rounded once (one FMA of the exact w - s_g * (l q)), and hi + lo carries
 // it to a relative 2^-17, so the GEMM sees dW, not a difference of two large products.
@@ -55,6 +56,8 @@ constexpr int kSegBlocks = 32;
 constexpr uint32_t kTmemColsSeg = 2 * kBN;
 constexpr uint32_t kGemmSmemBytes = kStages * kStageBytes + 1024 /* alignment */ + 256 /* barriers */;
 constexpr uint32_t kIdesc = idesc_bf16_f32(kBM, kBN);
+constexpr uint32_t kIdescMN = idesc_bf16_f32_mn(kBM, kBN);
+constexpr uint32_t kBoxBytes = 64 * kBK * 2;  // mode 3: one 64-channel x 64-token TMA box
 
 __device__ uint32_t g_output_error_flags = 0;
 
@@ -133,7 +136,9 @@ __device__ __forceinline__ float sum_squares32(const uint32_t (&r)[32]) {
 // kMode 0: the sum-of-squares GEMM of the output error (K runs over [X | X], kb_half
 // blocks per half).  kMode 1: H[rows, cols] += A B^T over kb_half K blocks, both operands
 // rows of X^T, tiles wholly below the diagonal skipped.  kMode 2: C[rows, cols] += A B^T
-// over kb_half K blocks, every tile (the GPTQ update).
+// over kb_half K blocks, every tile (the GPTQ update).  kMode 3: kMode 1 read from X itself
+// ([tokens, n], channels contiguous): each stage loads 64-channel x 64-token boxes and
+// the MMAs take both operands MN-major, so no transpose is needed.
 template <int kMode>
 __global__ void __launch_bounds__(kGemmThreads, 1)
 gemm_kernel(const __grid_constant__ CUtensorMap xmap, const __grid_constant__ CUtensorMap wmap,
@@ -151,7 +156,8 @@ gemm_kernel(const __grid_constant__ CUtensorMap xmap, const __grid_constant__ CU
   uint64_t* seg_full = acc_ready + 2;  // mode 1: the partial of a segment is complete
   uint64_t* seg_empty = seg_full + 1;  // mode 1: the partial has been folded into the sum
   double* warp_sum = reinterpret_cast<double*>(smem + kStages * kStageBytes + 128);
-  constexpr uint32_t kCols = kMode == 1 ? kTmemColsSeg : kTmemCols;
+  constexpr bool kHessian = kMode == 1 || kMode == 3;
+  constexpr uint32_t kCols = kHessian ? kTmemColsSeg : kTmemCols;
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int tile_m = blockIdx.x / tiles_n, tile_n = blockIdx.x - tile_m * tiles_n;
@@ -159,7 +165,7 @@ gemm_kernel(const __grid_constant__ CUtensorMap xmap, const __grid_constant__ CU
   const int kb_total = kAccum ? kb_half : 2 * kb_half;
   // H is symmetric and only its upper triangle is used: a tile wholly below the diagonal
   // (every column index below every row index) is skipped, uniformly for the whole CTA
-  if (kMode == 1 && (int64_t)(tile_n + 1) * kBN <= (int64_t)tile_m * kBM) return;
+  if (kHessian && (int64_t)(tile_n + 1) * kBN <= (int64_t)tile_m * kBM) return;
 
   if (threadIdx.x == 0) {
     for (int s = 0; s < kStages; ++s) {
@@ -195,21 +201,32 @@ gemm_kernel(const __grid_constant__ CUtensorMap xmap, const __grid_constant__ CU
           break;
         }
         mbar_arrive_expect_tx(&full[s], kStageBytes);
-        const int xk = (kAccum || kb < kb_half ? kb : kb - kb_half) * kBK;
-        tma_load_2d(tile_a + s * kTileABytes, &xmap, xk, tile_m * kBM, &full[s], policy);
-        tma_load_2d(tile_b + s * kTileBBytes, &wmap, kb * kBK, tile_n * kBN, &full[s], policy);
+        if (kMode == 3) {
+#pragma unroll
+          for (int j = 0; j < kBM / 64; ++j)
+            tma_load_2d(tile_a + s * kTileABytes + j * kBoxBytes, &xmap, tile_m * kBM + 64 * j, kb * kBK, &full[s],
+                        policy);
+#pragma unroll
+          for (int j = 0; j < kBN / 64; ++j)
+            tma_load_2d(tile_b + s * kTileBBytes + j * kBoxBytes, &wmap, tile_n * kBN + 64 * j, kb * kBK, &full[s],
+                        policy);
+        } else {
+          const int xk = (kAccum || kb < kb_half ? kb : kb - kb_half) * kBK;
+          tma_load_2d(tile_a + s * kTileABytes, &xmap, xk, tile_m * kBM, &full[s], policy);
+          tma_load_2d(tile_b + s * kTileBBytes, &wmap, kb * kBK, tile_n * kBN, &full[s], policy);
+        }
       }
     }
   } else if (warp == 1) {
     if (lane == 0) {
       // mode 1: segments of kSegBlocks K blocks, each accumulated from zero; the other
       // modes: one segment over the whole K loop
-      const int seg_blocks = kMode == 1 ? kSegBlocks : (kb_total > 0 ? kb_total : 1);
+      const int seg_blocks = kHessian ? kSegBlocks : (kb_total > 0 ? kb_total : 1);
       const int nseg = (kb_total + seg_blocks - 1) / seg_blocks;
       bool ok = true;
       for (int seg = 0; seg < nseg && ok; ++seg) {
         // the previous segment's partial must have been read out of TMEM
-        if (kMode == 1 && seg >= 1 && !mbar_wait(seg_empty, (uint32_t)(seg - 1) & 1u)) {
+        if (kHessian && seg >= 1 && !mbar_wait(seg_empty, (uint32_t)(seg - 1) & 1u)) {
           atomicOr(failed, 1u);
           break;
         }
@@ -225,15 +242,24 @@ gemm_kernel(const __grid_constant__ CUtensorMap xmap, const __grid_constant__ CU
             break;
           }
           tc_fence_after_sync();
-          const uint64_t ad = smem_desc_k_sw128(smem_addr(tile_a + s * kTileABytes));
-          const uint64_t bd = smem_desc_k_sw128(smem_addr(tile_b + s * kTileBBytes));
+          if (kMode == 3) {
+            // MN-major: 16 K rows are two 1024-byte swizzle atoms further
+            const uint64_t ad = smem_desc_mn_sw128(smem_addr(tile_a + s * kTileABytes), kBoxBytes);
+            const uint64_t bd = smem_desc_mn_sw128(smem_addr(tile_b + s * kTileBBytes), kBoxBytes);
 #pragma unroll
-          for (int kk = 0; kk < kBK / 16; ++kk)
-            umma_bf16(d, ad + 2 * kk, bd + 2 * kk, kIdesc, (uint32_t)(kb > kb0 || kk > 0));
+            for (int kk = 0; kk < kBK / 16; ++kk)
+              umma_bf16(d, ad + 128 * kk, bd + 128 * kk, kIdescMN, (uint32_t)(kb > kb0 || kk > 0));
+          } else {
+            const uint64_t ad = smem_desc_k_sw128(smem_addr(tile_a + s * kTileABytes));
+            const uint64_t bd = smem_desc_k_sw128(smem_addr(tile_b + s * kTileBBytes));
+#pragma unroll
+            for (int kk = 0; kk < kBK / 16; ++kk)
+              umma_bf16(d, ad + 2 * kk, bd + 2 * kk, kIdesc, (uint32_t)(kb > kb0 || kk > 0));
+          }
           umma_commit(smem_addr(&empty[s]));
         }
         // fires once every MMA issued above has completed
-        if (ok) umma_commit(smem_addr(kMode == 1 ? seg_full : acc_ready));
+        if (ok) umma_commit(smem_addr(kHessian ? seg_full : acc_ready));
       }
     }
     __syncwarp();
@@ -245,9 +271,9 @@ gemm_kernel(const __grid_constant__ CUtensorMap xmap, const __grid_constant__ CU
     const int64_t row = (int64_t)tile_m * kBM + quarter * 32 + lane;
     const int64_t col0 = (int64_t)tile_n * kBN;
     const uint32_t lane_base = (quarter * 32u) << 16;
-    const int nseg = kMode == 1 ? (kb_total + kSegBlocks - 1) / kSegBlocks : 1;
+    const int nseg = kHessian ? (kb_total + kSegBlocks - 1) / kSegBlocks : 1;
     for (int seg = 0; seg < nseg; ++seg) {
-      if (!mbar_wait(kMode == 1 ? seg_full : acc_ready, kMode == 1 ? (uint32_t)seg & 1u : 0u)) {
+      if (!mbar_wait(kHessian ? seg_full : acc_ready, kHessian ? (uint32_t)seg & 1u : 0u)) {
         atomicOr(failed, 1u);
         break;
       }
@@ -257,7 +283,7 @@ gemm_kernel(const __grid_constant__ CUtensorMap xmap, const __grid_constant__ CU
       for (int c0 = 0; c0 < kBN; c0 += 32) {
         uint32_t r[32];
         tmem_ld_32x32b_x32(tmem_d + lane_base + (uint32_t)c0, r);
-        if (kMode == 1 && seg > 0) {
+        if (kHessian && seg > 0) {
           uint32_t q[32];
           tmem_ld_32x32b_x32(tmem_d + lane_base + kBN + (uint32_t)c0, q);
           tmem_ld_wait();
@@ -266,7 +292,7 @@ gemm_kernel(const __grid_constant__ CUtensorMap xmap, const __grid_constant__ CU
         } else {
           tmem_ld_wait();
         }
-        if (kMode == 1 && !last) {
+        if (kHessian && !last) {
           tmem_st_32x32b_x32(tmem_d + lane_base + kBN + (uint32_t)c0, r);
           continue;
         }
@@ -288,7 +314,7 @@ gemm_kernel(const __grid_constant__ CUtensorMap xmap, const __grid_constant__ CU
           }
         }
       }
-      if (kMode == 1 && !last) {
+      if (kHessian && !last) {
         // the partial has been read and the running sum written: the MMAs may go on
         tmem_st_wait();
         tc_fence_before_sync();
@@ -355,56 +381,6 @@ __global__ void __launch_bounds__(256) transpose_kernel(const uint16_t* __restri
   for (int k = ty; k < 32; k += 8) {
     const int64_t c = c0 + k, t = t0 + tx;
     if (c < n && t < tokens) xt[c * ld_t + t] = tile[tx][k];
-  }
-}
-
-// The same transpose with 16-byte accesses on both sides, for X with 16-byte aligned rows:
-// a 64-token x 64-channel tile per CTA.  Each thread loads 8 channels of two consecutive
-// tokens, pairs them into eight 32-bit words (token t low, t + 1 high) with byte permutes,
-// and stores the words transposed into shared memory (64 channel rows x 32 words, 16-byte
-// word groups XOR-swizzled by the channel octet so that neither side has bank conflicts);
-// then each thread writes two 16-byte runs of 8 tokens of one channel.
-__global__ void __launch_bounds__(256) transpose64_kernel(const uint16_t* __restrict__ x, int64_t tokens, int64_t n,
-                                                          int64_t ld_x, uint16_t* __restrict__ xt, int64_t ld_t) {
-  __shared__ __align__(16) uint32_t tile[64 * 32];
-  const int64_t t0 = (int64_t)blockIdx.x * 64, c0 = (int64_t)blockIdx.y * 64;
-  const int tid = threadIdx.x;
-  {
-    const int p = tid >> 3, g = tid & 7;
-    const int64_t t = t0 + 2 * p, c = c0 + 8 * g;
-    uint4 va = make_uint4(0u, 0u, 0u, 0u), vb = va;
-    if (c + 8 <= n) {
-      if (t < tokens) va = *reinterpret_cast<const uint4*>(x + t * ld_x + c);
-      if (t + 1 < tokens) vb = *reinterpret_cast<const uint4*>(x + (t + 1) * ld_x + c);
-    } else if (c < n) {
-      uint16_t ea[8] = {0, 0, 0, 0, 0, 0, 0, 0}, eb[8] = {0, 0, 0, 0, 0, 0, 0, 0};
-      for (int j = 0; j < 8 && c + j < n; ++j) {
-        if (t < tokens) ea[j] = x[t * ld_x + c + j];
-        if (t + 1 < tokens) eb[j] = x[(t + 1) * ld_x + c + j];
-      }
-      va = make_uint4(ea[0] | (uint32_t)ea[1] << 16, ea[2] | (uint32_t)ea[3] << 16, ea[4] | (uint32_t)ea[5] << 16,
-                      ea[6] | (uint32_t)ea[7] << 16);
-      vb = make_uint4(eb[0] | (uint32_t)eb[1] << 16, eb[2] | (uint32_t)eb[3] << 16, eb[4] | (uint32_t)eb[5] << 16,
-                      eb[6] | (uint32_t)eb[7] << 16);
-    }
-    const uint32_t a[4] = {va.x, va.y, va.z, va.w}, b[4] = {vb.x, vb.y, vb.z, vb.w};
-    const int col = (((p >> 2) ^ g) << 2) | (p & 3);
-#pragma unroll
-    for (int i = 0; i < 4; ++i) {
-      tile[(8 * g + 2 * i) * 32 + col] = __byte_perm(a[i], b[i], 0x5410);
-      tile[(8 * g + 2 * i + 1) * 32 + col] = __byte_perm(a[i], b[i], 0x7632);
-    }
-  }
-  __syncthreads();
-#pragma unroll
-  for (int it = 0; it < 2; ++it) {
-    const int item = tid + 256 * it;
-    const int c = item >> 3, q = item & 7;
-    const int64_t cg = c0 + c, tg = t0 + 8 * q;
-    if (cg < n && tg < tokens) {
-      const uint4 v = *reinterpret_cast<const uint4*>(&tile[c * 32 + ((q ^ ((c >> 3) & 7)) << 2)]);
-      *reinterpret_cast<uint4*>(xt + cg * ld_t + tg) = v;
-    }
   }
 }
 
@@ -490,20 +466,35 @@ int64_t hessian_full_ld(int64_t tokens) { return (tokens + 7) / 8 * 8; }
 
 cudaError_t launch_hessian_full(const void* x, int64_t tokens, int64_t n, int64_t ld_x, float* H, int64_t ld_h,
                                 void* xt, cudaStream_t stream) {
-  const int64_t ld_t = hessian_full_ld(tokens);
-  if ((reinterpret_cast<uintptr_t>(x) & 15) == 0 && ld_x % 8 == 0) {
-    const dim3 tgrid((unsigned)((tokens + 63) / 64), (unsigned)((n + 63) / 64));
-    transpose64_kernel<<<tgrid, 256, 0, stream>>>(static_cast<const uint16_t*>(x), tokens, n, ld_x,
-                                                  static_cast<uint16_t*>(xt), ld_t);
-  } else {
-    const dim3 tgrid((unsigned)((tokens + 31) / 32), (unsigned)((n + 31) / 32));
-    transpose_kernel<<<tgrid, 256, 0, stream>>>(static_cast<const uint16_t*>(x), tokens, n, ld_x,
-                                                static_cast<uint16_t*>(xt), ld_t);
-  }
-  cudaError_t err = cudaGetLastError();
-  if (err != cudaSuccess) return err;
   EncodeTiledFn encode = nullptr;
-  err = encode_tiled_fn(&encode);
+  cudaError_t err = encode_tiled_fn(&encode);
+  if (err != cudaSuccess) return err;
+  const int64_t tiles_n = (n + kBN - 1) / kBN;
+  const int64_t tiles = ((n + kBM - 1) / kBM) * tiles_n;
+  if ((reinterpret_cast<uintptr_t>(x) & 15) == 0 && ld_x % 8 == 0) {
+    // X read as it is: 64-channel x 64-token boxes, MN-major operands (kMode 3)
+    CUtensorMap map;
+    const cuuint64_t dims[2] = {(cuuint64_t)n, (cuuint64_t)tokens};
+    const cuuint64_t strides[1] = {(cuuint64_t)ld_x * 2};
+    const cuuint32_t box[2] = {64, (cuuint32_t)kBK};
+    const cuuint32_t estr[2] = {1, 1};
+    if (encode(&map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(x), dims, strides, box, estr,
+               CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+               CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) != CUDA_SUCCESS)
+      return cudaErrorInvalidValue;
+    err = ensure_dynamic_smem(reinterpret_cast<const void*>(gemm_kernel<3>), (int)kGemmSmemBytes);
+    if (err != cudaSuccess) return err;
+    gemm_kernel<3><<<(unsigned)tiles, kGemmThreads, kGemmSmemBytes, stream>>>(
+        map, map, (int)((tokens + kBK - 1) / kBK), (int)tiles_n, nullptr, H, n, n, ld_h);
+    return cudaGetLastError();
+  }
+  // X with rows that are not 16-byte aligned: transposed first (tokens contiguous per
+  // channel), then both operands K-major (kMode 1)
+  const int64_t ld_t = hessian_full_ld(tokens);
+  const dim3 tgrid((unsigned)((tokens + 31) / 32), (unsigned)((n + 31) / 32));
+  transpose_kernel<<<tgrid, 256, 0, stream>>>(static_cast<const uint16_t*>(x), tokens, n, ld_x,
+                                              static_cast<uint16_t*>(xt), ld_t);
+  err = cudaGetLastError();
   if (err != cudaSuccess) return err;
   CUtensorMap amap, bmap;
   const cuuint64_t dims[2] = {(cuuint64_t)tokens, (cuuint64_t)n};
@@ -519,8 +510,6 @@ cudaError_t launch_hessian_full(const void* x, int64_t tokens, int64_t n, int64_
   const cudaError_t attr_status =
       ensure_dynamic_smem(reinterpret_cast<const void*>(gemm_kernel<1>), (int)kGemmSmemBytes);
   if (attr_status != cudaSuccess) return attr_status;
-  const int64_t tiles_n = (n + kBN - 1) / kBN;
-  const int64_t tiles = ((n + kBM - 1) / kBM) * tiles_n;
   gemm_kernel<1><<<(unsigned)tiles, kGemmThreads, kGemmSmemBytes, stream>>>(
       amap, bmap, (int)((tokens + kBK - 1) / kBK), (int)tiles_n, nullptr, H, n, n, ld_h);
   return cudaGetLastError();

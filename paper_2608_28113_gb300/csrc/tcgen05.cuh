@@ -44,12 +44,32 @@ __device__ __forceinline__ uint64_t smem_desc_k_sw128(uint32_t saddr) {
   return d;
 }
 
+// Shared-memory matrix descriptor of an MN-major operand tile (M or N contiguous) written
+// by TMA with 128-byte swizzling: each TMA box holds 64 MN elements (one 128-byte row) for
+// each of its K rows, in 8-row (1024-byte) swizzle atoms.
+//   bits 16-29  leading-dimension byte offset >> 4: between 64-element groups along M/N
+//               (one TMA box further)
+//   bits 32-45  stride-dimension byte offset >> 4: between 8-row groups along K (1024)
+// Stepping K by 16 rows adds 2048 bytes to the start address.
+__device__ __forceinline__ uint64_t smem_desc_mn_sw128(uint32_t saddr, uint32_t mn_group_bytes) {
+  uint64_t d = (uint64_t)((saddr & 0x3FFFFu) >> 4);
+  d |= (uint64_t)((mn_group_bytes >> 4) & 0x3FFFu) << 16;
+  d |= (uint64_t)(1024u >> 4) << 32;
+  d |= (uint64_t)1 << 46;
+  d |= (uint64_t)2 << 61;
+  return d;
+}
+
 // Instruction descriptor of tcgen05.mma kind::f16 with bf16 A and B (both K-major) and
 // an fp32 accumulator, M x N per instruction:
 //   bits 4-5 D format (1 = f32), 7-9 A format (1 = bf16), 10-12 B format (1 = bf16),
 //   15/16 A/B major (0 = K-major), 17-22 N >> 3, 24-28 M >> 4.
 __host__ __device__ constexpr uint32_t idesc_bf16_f32(uint32_t M, uint32_t N) {
   return (1u << 4) | (1u << 7) | (1u << 10) | ((N >> 3) << 17) | ((M >> 4) << 24);
+}
+// The same with both A and B MN-major (bits 15 and 16).
+__host__ __device__ constexpr uint32_t idesc_bf16_f32_mn(uint32_t M, uint32_t N) {
+  return idesc_bf16_f32(M, N) | (1u << 15) | (1u << 16);
 }
 
 // ---------------------------------------------------------------- MMA

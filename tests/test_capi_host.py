@@ -204,7 +204,9 @@ def test_gptq_argument_errors(lib):
     f = lib.hscale_hessian_full_accumulate
     assert f(FAKE, 100, 64, 32, FAKE, 64, FAKE, 1 << 20, None) == ERR_SHAPE      # ld_x < n
     assert f(FAKE, 100, 64, 64, None, 64, FAKE, 1 << 20, None) == ERR_NULL
-    assert f(FAKE, 100, 64, 64, FAKE, 64, FAKE, 16, None) == ERR_WS
+    # X whose rows are not 16-byte aligned (ld_x % 8 != 0) is transposed: a workspace is needed
+    assert f(FAKE, 100, 64, 66, FAKE, 64, FAKE, 16, None) == ERR_WS
+    assert f(FAKE, 100, 64, 66, FAKE, 64, None, 0, None) == ERR_WS
     assert f(None, 0, 64, 64, None, 64, None, 0, None) == OK
     g = lib.hscale_gptq_factor
     assert g(FAKE, 64, 32, 0.01, FAKE, None, FAKE, FAKE, 1 << 20, None) == ERR_SHAPE   # ld < n
