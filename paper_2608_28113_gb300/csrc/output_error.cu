@@ -24,9 +24,9 @@
 //
 // GEMM tile: 128 tokens x 256 outputs, K in steps of 64 bf16 (one 128-byte swizzle atom
 // per row), a 4-stage ring of TMA loads (48 KB per stage).  Warp 0 issues the loads, warp 1
-// owns the tensor memory and issues the MMAs (M = 128, N = 256, K = 16 each), warps 2-5
-// read the 128 x 256 fp32 accumulator back (each warp its 32-lane quarter) and square and
-// sum it.  Every wait is bounded; one that runs out sets the error flag and the tile's
+// owns the tensor memory and issues the MMAs (M = 128, N = 256, K = 16 each), warps 2-9
+// read the 128 x 256 fp32 accumulator back (each warp half the columns of its 32-lane
+// quarter) and square and sum it.  Every wait is bounded; one that runs out sets the error flag and the tile's
 // partial becomes NaN.
 #include <algorithm>
 #include <cuda_bf16.h>
@@ -40,18 +40,20 @@ namespace hscale {
 namespace {
 
 constexpr int kBM = 128, kBN = 256, kBK = 64, kStages = 4;
-constexpr int kGemmThreads = 192;
+constexpr int kGemmThreads = 320;  // TMA warp, MMA warp, 8 epilogue warps
 constexpr uint32_t kTileABytes = kBM * kBK * 2;  // 16 KB
 constexpr uint32_t kTileBBytes = kBN * kBK * 2;  // 32 KB
 constexpr uint32_t kStageBytes = kTileABytes + kTileBBytes;
 constexpr uint32_t kTmemCols = kBN;  // fp32 accumulator: 128 lanes x 256 columns
-// Full Hessian (mode 1): the tensor cores accumulate in fp32 with an error that grows with
-// the accumulation length (the diagonal comes out low by about 0.9 u per K = 16 step,
-// measured), so each tile's K loop is cut into segments of kSegBlocks K blocks (2048
-// tokens).  Each segment accumulates from zero in TMEM columns [0, 256); the epilogue warps
-// add it in fp32 round-to-nearest into a running sum kept in TMEM columns [256, 512), and
-// add the running sum into H after the last segment.  With H = 0 before the call the
-// result is bit for bit that of successive calls of 2048 tokens, whatever the call size.
+// Full Hessian (modes 1, 3) and output error (mode 0): the tensor cores accumulate in fp32
+// with an error that grows with the accumulation length (the Hessian's diagonal comes out
+// low by about 0.9 u per K = 16 step, measured), so each tile's K loop is cut into
+// segments of kSegBlocks K blocks (2048 tokens, or 2048 of the 2 n channels of [X | X]).
+// Each segment accumulates from zero in TMEM columns [0, 256); the epilogue warps add it in
+// fp32 round-to-nearest into a running sum kept in TMEM columns [256, 512) and, after the
+// last segment, add the running sum into H (or square and sum it).  With H = 0 before the
+// call the Hessian is bit for bit that of successive calls of 2048 tokens, whatever the
+// call size.
 constexpr int kSegBlocks = 32;
 constexpr uint32_t kTmemColsSeg = 2 * kBN;
 constexpr uint32_t kGemmSmemBytes = kStages * kStageBytes + 1024 /* alignment */ + 256 /* barriers */;
@@ -157,7 +159,10 @@ gemm_kernel(const __grid_constant__ CUtensorMap xmap, const __grid_constant__ CU
   uint64_t* seg_empty = seg_full + 1;  // mode 1: the partial has been folded into the sum
   double* warp_sum = reinterpret_cast<double*>(smem + kStages * kStageBytes + 128);
   constexpr bool kHessian = kMode == 1 || kMode == 3;
-  constexpr uint32_t kCols = kHessian ? kTmemColsSeg : kTmemCols;
+  // K loops cut into accumulation segments folded in TMEM: the Hessian (K = tokens) and the
+  // output error (K = 2 n); the GPTQ update's K = 6 B is a single segment anyway
+  constexpr bool kSegmented = kMode != 2;
+  constexpr uint32_t kCols = kSegmented ? kTmemColsSeg : kTmemCols;
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int tile_m = blockIdx.x / tiles_n, tile_n = blockIdx.x - tile_m * tiles_n;
@@ -174,7 +179,7 @@ gemm_kernel(const __grid_constant__ CUtensorMap xmap, const __grid_constant__ CU
     }
     mbar_init(acc_ready, 1);
     mbar_init(seg_full, 1);
-    mbar_init(seg_empty, 128);  // every epilogue thread arrives
+    mbar_init(seg_empty, 256);  // every epilogue thread arrives
     *failed = 0u;
     mbar_fence_init();
     prefetch_tensormap(&xmap);
@@ -221,12 +226,12 @@ gemm_kernel(const __grid_constant__ CUtensorMap xmap, const __grid_constant__ CU
     if (lane == 0) {
       // mode 1: segments of kSegBlocks K blocks, each accumulated from zero; the other
       // modes: one segment over the whole K loop
-      const int seg_blocks = kHessian ? kSegBlocks : (kb_total > 0 ? kb_total : 1);
+      const int seg_blocks = kSegmented ? kSegBlocks : (kb_total > 0 ? kb_total : 1);
       const int nseg = (kb_total + seg_blocks - 1) / seg_blocks;
       bool ok = true;
       for (int seg = 0; seg < nseg && ok; ++seg) {
         // the previous segment's partial must have been read out of TMEM
-        if (kHessian && seg >= 1 && !mbar_wait(seg_empty, (uint32_t)(seg - 1) & 1u)) {
+        if (kSegmented && seg >= 1 && !mbar_wait(seg_empty, (uint32_t)(seg - 1) & 1u)) {
           atomicOr(failed, 1u);
           break;
         }
@@ -259,86 +264,88 @@ gemm_kernel(const __grid_constant__ CUtensorMap xmap, const __grid_constant__ CU
           umma_commit(smem_addr(&empty[s]));
         }
         // fires once every MMA issued above has completed
-        if (ok) umma_commit(smem_addr(kHessian ? seg_full : acc_ready));
+        if (ok) umma_commit(smem_addr(kSegmented ? seg_full : acc_ready));
       }
     }
     __syncwarp();
-  } else if (kAccum) {
-    // row of H held by this thread (TMEM lane = row of the tile), 32 columns at a time;
-    // mode 1 folds every segment's partial into the running sum and adds the sum into H
-    // after the last one
+  } else {
+    // epilogue warps 2-9: TMEM lane quarter warp % 4 (a warp may only touch that quarter),
+    // column half (warp - 2) / 4; each thread holds one tile row's half of the partial
+    constexpr int kHalf = kBN / 2;
     const uint32_t quarter = (uint32_t)(warp & 3);
-    const int64_t row = (int64_t)tile_m * kBM + quarter * 32 + lane;
-    const int64_t col0 = (int64_t)tile_n * kBN;
+    const uint32_t cbase = (uint32_t)((warp - 2) >> 2) * kHalf;
     const uint32_t lane_base = (quarter * 32u) << 16;
-    const int nseg = kHessian ? (kb_total + kSegBlocks - 1) / kSegBlocks : 1;
+    const int64_t row = (int64_t)tile_m * kBM + quarter * 32 + lane;
+    const int64_t col0 = (int64_t)tile_n * kBN + cbase;
+    const int nseg = kSegmented ? (kb_total + kSegBlocks - 1) / kSegBlocks : 1;
+    double acc = 0.0;
     for (int seg = 0; seg < nseg; ++seg) {
-      if (!mbar_wait(kHessian ? seg_full : acc_ready, kHessian ? (uint32_t)seg & 1u : 0u)) {
+      if (!mbar_wait(kSegmented ? seg_full : acc_ready, kSegmented ? (uint32_t)seg & 1u : 0u)) {
         atomicOr(failed, 1u);
         break;
       }
       tc_fence_after_sync();
       const bool last = seg + 1 == nseg;
-#pragma unroll 1
-      for (int c0 = 0; c0 < kBN; c0 += 32) {
-        uint32_t r[32];
-        tmem_ld_32x32b_x32(tmem_d + lane_base + (uint32_t)c0, r);
-        if (kHessian && seg > 0) {
-          uint32_t q[32];
-          tmem_ld_32x32b_x32(tmem_d + lane_base + kBN + (uint32_t)c0, q);
-          tmem_ld_wait();
+      uint32_t p[kHalf];
 #pragma unroll
-          for (int j = 0; j < 32; ++j) r[j] = __float_as_uint(__fadd_rn(__uint_as_float(q[j]), __uint_as_float(r[j])));
-        } else {
-          tmem_ld_wait();
-        }
-        if (kHessian && !last) {
-          tmem_st_32x32b_x32(tmem_d + lane_base + kBN + (uint32_t)c0, r);
-          continue;
-        }
-        if (row < h_rows) {
-          float* dst = H + row * ld_h + col0 + c0;
-          if (col0 + c0 + 32 <= h_cols && ((ld_h | (col0 + c0)) & 3) == 0 &&
-              (reinterpret_cast<uintptr_t>(H) & 15) == 0) {
-#pragma unroll
-            for (int q = 0; q < 8; ++q) {
-              float4 v = reinterpret_cast<float4*>(dst)[q];
-              v.x += __uint_as_float(r[4 * q]);
-              v.y += __uint_as_float(r[4 * q + 1]);
-              v.z += __uint_as_float(r[4 * q + 2]);
-              v.w += __uint_as_float(r[4 * q + 3]);
-              reinterpret_cast<float4*>(dst)[q] = v;
-            }
-          } else {
-            for (int q = 0; q < 32 && col0 + c0 + q < h_cols; ++q) dst[q] += __uint_as_float(r[q]);
-          }
-        }
-      }
-      if (kHessian && !last) {
-        // the partial has been read and the running sum written: the MMAs may go on
-        tmem_st_wait();
+      for (int c = 0; c < kHalf; c += 32)
+        tmem_ld_32x32b_x32(tmem_d + lane_base + cbase + (uint32_t)c, *reinterpret_cast<uint32_t(*)[32]>(p + c));
+      tmem_ld_wait();
+      if (kSegmented && !last) {
+        // the partial is in registers: the MMAs may go on with the next segment
         tc_fence_before_sync();
         mbar_arrive(seg_empty);
       }
-    }
-  } else {
-    const uint32_t quarter = (uint32_t)(warp & 3);
-    double acc = 0.0;
-    if (mbar_wait(acc_ready, 0u)) {
-      tc_fence_after_sync();
-#pragma unroll 1
-      for (int c0 = 0; c0 < kBN; c0 += 32) {
-        uint32_t r[32];
-        tmem_ld_32x32b_x32(tmem_d + ((quarter * 32u) << 16) + (uint32_t)c0, r);
-        tmem_ld_wait();
-        acc += (double)sum_squares32(r);
-      }
-    } else {
-      atomicOr(failed, 1u);
-    }
+      if (kSegmented && seg > 0) {
+        // fold into the running sum (TMEM columns [256, 512)), fp32 round-to-nearest
 #pragma unroll
-    for (int off = 16; off > 0; off >>= 1) acc += __shfl_xor_sync(0xFFFFFFFFu, acc, off);
-    if (lane == 0) warp_sum[quarter] = acc;
+        for (int c = 0; c < kHalf; c += 32) {
+          uint32_t q[32];
+          tmem_ld_32x32b_x32(tmem_d + lane_base + kBN + cbase + (uint32_t)c, q);
+          tmem_ld_wait();
+#pragma unroll
+          for (int j = 0; j < 32; ++j)
+            p[c + j] = __float_as_uint(__fadd_rn(__uint_as_float(q[j]), __uint_as_float(p[c + j])));
+        }
+      }
+      if (kSegmented && !last) {
+#pragma unroll
+        for (int c = 0; c < kHalf; c += 32)
+          tmem_st_32x32b_x32(tmem_d + lane_base + kBN + cbase + (uint32_t)c, *reinterpret_cast<uint32_t(*)[32]>(p + c));
+        tmem_st_wait();
+        continue;
+      }
+      if (!kAccum) {
+        // the output error: the sum of squares of the complete tile
+#pragma unroll
+        for (int c = 0; c < kHalf; c += 32) acc += (double)sum_squares32(*reinterpret_cast<uint32_t(*)[32]>(p + c));
+        continue;
+      }
+      // the Hessian and the GPTQ update: the tile row added into H (C)
+      if (row < h_rows) {
+        float* dst = H + row * ld_h + col0;
+        if (col0 + kHalf <= h_cols && ((ld_h | col0) & 3) == 0 && (reinterpret_cast<uintptr_t>(H) & 15) == 0) {
+#pragma unroll
+          for (int q = 0; q < kHalf / 4; ++q) {
+            float4 v = reinterpret_cast<float4*>(dst)[q];
+            v.x += __uint_as_float(p[4 * q]);
+            v.y += __uint_as_float(p[4 * q + 1]);
+            v.z += __uint_as_float(p[4 * q + 2]);
+            v.w += __uint_as_float(p[4 * q + 3]);
+            reinterpret_cast<float4*>(dst)[q] = v;
+          }
+        } else {
+#pragma unroll
+          for (int q = 0; q < kHalf; ++q)
+            if (col0 + q < h_cols) dst[q] += __uint_as_float(p[q]);
+        }
+      }
+    }
+    if (!kAccum) {
+#pragma unroll
+      for (int off = 16; off > 0; off >>= 1) acc += __shfl_xor_sync(0xFFFFFFFFu, acc, off);
+      if (lane == 0) warp_sum[warp - 2] = acc;
+    }
   }
   tc_fence_before_sync();
   __syncthreads();
@@ -347,13 +354,14 @@ gemm_kernel(const __grid_constant__ CUtensorMap xmap, const __grid_constant__ CU
     if (*failed && warp >= 2) {
       const uint32_t quarter = (uint32_t)(warp & 3);
       const int64_t row = (int64_t)tile_m * kBM + quarter * 32 + lane;
+      const int64_t c0 = (int64_t)tile_n * kBN + ((warp - 2) >> 2) * (kBN / 2);
       if (row < h_rows)
-        for (int64_t c = (int64_t)tile_n * kBN; c < (int64_t)(tile_n + 1) * kBN && c < h_cols; ++c)
-          H[row * ld_h + c] = __int_as_float(0x7FC00000);
+        for (int64_t c = c0; c < c0 + kBN / 2 && c < h_cols; ++c) H[row * ld_h + c] = __int_as_float(0x7FC00000);
       if (threadIdx.x == 64) atomicOr(&g_output_error_flags, kErrMbarTimeout);
     }
   } else if (threadIdx.x == 0) {
-    double total = (warp_sum[0] + warp_sum[1]) + (warp_sum[2] + warp_sum[3]);
+    double total = ((warp_sum[0] + warp_sum[1]) + (warp_sum[2] + warp_sum[3])) +
+                   ((warp_sum[4] + warp_sum[5]) + (warp_sum[6] + warp_sum[7]));
     if (*failed) {
       atomicOr(&g_output_error_flags, kErrMbarTimeout);
       total = __longlong_as_double(0x7FF8000000000000ll);
