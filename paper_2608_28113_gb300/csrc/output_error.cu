@@ -144,8 +144,8 @@ __device__ __forceinline__ float sum_squares32(const uint32_t (&r)[32]) {
 template <int kMode>
 __global__ void __launch_bounds__(kGemmThreads, 1)
 gemm_kernel(const __grid_constant__ CUtensorMap xmap, const __grid_constant__ CUtensorMap wmap,
-            int kb_half, int tiles_n, double* __restrict__ partials, float* __restrict__ H, int64_t h_rows,
-            int64_t h_cols, int64_t ld_h) {
+            int kb_half, int tiles_n, int tiles_total, double* __restrict__ partials, float* __restrict__ H,
+            int64_t h_rows, int64_t h_cols, int64_t ld_h) {
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
   uint8_t* tile_a = smem;
@@ -157,14 +157,22 @@ gemm_kernel(const __grid_constant__ CUtensorMap xmap, const __grid_constant__ CU
   uint32_t* failed = tmem_slot + 1;
   uint64_t* seg_full = acc_ready + 2;  // mode 1: the partial of a segment is complete
   uint64_t* seg_empty = seg_full + 1;  // mode 1: the partial has been folded into the sum
+  uint64_t* tacc_full = seg_empty + 1;  // mode 2: accumulator a holds a finished tile
+  uint64_t* tacc_empty = tacc_full + 2;  // mode 2: accumulator a has been read out
   double* warp_sum = reinterpret_cast<double*>(smem + kStages * kStageBytes + 128);
   constexpr bool kHessian = kMode == 1 || kMode == 3;
   // K loops cut into accumulation segments folded in TMEM: the Hessian (K = tokens) and the
   // output error (K = 2 n); the GPTQ update's K = 6 B is a single segment anyway
   constexpr bool kSegmented = kMode != 2;
-  constexpr uint32_t kCols = kSegmented ? kTmemColsSeg : kTmemCols;
+  // The GPTQ update is persistent: a CTA takes tiles blockIdx.x, + gridDim.x, ... and
+  // alternates two 256-column accumulators, so a tile's epilogue (the read-modify-write of
+  // the running weights) runs alongside the next tile's loads and MMAs.  The other modes
+  // take one tile per CTA.
+  constexpr bool kPersistent = kMode == 2;
+  constexpr uint32_t kCols = (kSegmented || kPersistent) ? kTmemColsSeg : kTmemCols;
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int ntiles = kPersistent ? (tiles_total - (int)blockIdx.x + (int)gridDim.x - 1) / (int)gridDim.x : 1;
   const int tile_m = blockIdx.x / tiles_n, tile_n = blockIdx.x - tile_m * tiles_n;
   constexpr bool kAccum = kMode != 0;
   const int kb_total = kAccum ? kb_half : 2 * kb_half;
@@ -180,6 +188,10 @@ gemm_kernel(const __grid_constant__ CUtensorMap xmap, const __grid_constant__ CU
     mbar_init(acc_ready, 1);
     mbar_init(seg_full, 1);
     mbar_init(seg_empty, 256);  // every epilogue thread arrives
+    for (int a = 0; a < 2; ++a) {
+      mbar_init(&tacc_full[a], 1);
+      mbar_init(&tacc_empty[a], 256);
+    }
     *failed = 0u;
     mbar_fence_init();
     prefetch_tensormap(&xmap);
@@ -198,73 +210,91 @@ gemm_kernel(const __grid_constant__ CUtensorMap xmap, const __grid_constant__ CU
     if (lane == 0) {
       uint64_t policy;
       asm volatile("createpolicy.fractional.L2::evict_last.b64 %0, 1.0;" : "=l"(policy));
-      for (int kb = 0; kb < kb_total; ++kb) {
-        const int s = kb % kStages;
-        const uint32_t round = (uint32_t)(kb / kStages);
-        if (!mbar_wait(&empty[s], (round & 1u) ^ 1u)) {
-          atomicOr(failed, 1u);
-          break;
-        }
-        mbar_arrive_expect_tx(&full[s], kStageBytes);
-        if (kMode == 3) {
+      bool go = true;
+      for (int i = 0; i < ntiles && go; ++i) {
+        const int t = (int)blockIdx.x + i * (int)gridDim.x;
+        const int tm = t / tiles_n, tn = t - tm * tiles_n;
+        for (int kb = 0; kb < kb_total; ++kb) {
+          // the ring's position counts K blocks over all of the CTA's tiles
+          const int g = i * kb_total + kb;
+          const int s = g % kStages;
+          const uint32_t round = (uint32_t)(g / kStages);
+          if (!mbar_wait(&empty[s], (round & 1u) ^ 1u)) {
+            atomicOr(failed, 1u);
+            go = false;
+            break;
+          }
+          mbar_arrive_expect_tx(&full[s], kStageBytes);
+          if (kMode == 3) {
 #pragma unroll
-          for (int j = 0; j < kBM / 64; ++j)
-            tma_load_2d(tile_a + s * kTileABytes + j * kBoxBytes, &xmap, tile_m * kBM + 64 * j, kb * kBK, &full[s],
-                        policy);
+            for (int j = 0; j < kBM / 64; ++j)
+              tma_load_2d(tile_a + s * kTileABytes + j * kBoxBytes, &xmap, tm * kBM + 64 * j, kb * kBK, &full[s],
+                          policy);
 #pragma unroll
-          for (int j = 0; j < kBN / 64; ++j)
-            tma_load_2d(tile_b + s * kTileBBytes + j * kBoxBytes, &wmap, tile_n * kBN + 64 * j, kb * kBK, &full[s],
-                        policy);
-        } else {
-          const int xk = (kAccum || kb < kb_half ? kb : kb - kb_half) * kBK;
-          tma_load_2d(tile_a + s * kTileABytes, &xmap, xk, tile_m * kBM, &full[s], policy);
-          tma_load_2d(tile_b + s * kTileBBytes, &wmap, kb * kBK, tile_n * kBN, &full[s], policy);
+            for (int j = 0; j < kBN / 64; ++j)
+              tma_load_2d(tile_b + s * kTileBBytes + j * kBoxBytes, &wmap, tn * kBN + 64 * j, kb * kBK, &full[s],
+                          policy);
+          } else {
+            const int xk = (kAccum || kb < kb_half ? kb : kb - kb_half) * kBK;
+            tma_load_2d(tile_a + s * kTileABytes, &xmap, xk, tm * kBM, &full[s], policy);
+            tma_load_2d(tile_b + s * kTileBBytes, &wmap, kb * kBK, tn * kBN, &full[s], policy);
+          }
         }
       }
     }
   } else if (warp == 1) {
     if (lane == 0) {
-      // mode 1: segments of kSegBlocks K blocks, each accumulated from zero; the other
-      // modes: one segment over the whole K loop
+      // the segmented modes: segments of kSegBlocks K blocks, each accumulated from zero;
+      // the GPTQ update: one segment over its short K loop, per tile
       const int seg_blocks = kSegmented ? kSegBlocks : (kb_total > 0 ? kb_total : 1);
       const int nseg = (kb_total + seg_blocks - 1) / seg_blocks;
       bool ok = true;
-      for (int seg = 0; seg < nseg && ok; ++seg) {
-        // the previous segment's partial must have been read out of TMEM
-        if (kSegmented && seg >= 1 && !mbar_wait(seg_empty, (uint32_t)(seg - 1) & 1u)) {
+      for (int i = 0; i < ntiles && ok; ++i) {
+        const uint32_t acc = kPersistent ? (uint32_t)(i & 1) : 0u;
+        // the accumulator's previous tile (two back) must have been read out of TMEM
+        if (kPersistent && i >= 2 && !mbar_wait(&tacc_empty[acc], (uint32_t)((i >> 1) - 1) & 1u)) {
           atomicOr(failed, 1u);
           break;
         }
-        tc_fence_after_sync();
-        const uint32_t d = tmem_d;
-        const int kb0 = seg * seg_blocks, kb1 = min(kb_total, kb0 + seg_blocks);
-        for (int kb = kb0; kb < kb1; ++kb) {
-          const int s = kb % kStages;
-          const uint32_t round = (uint32_t)(kb / kStages);
-          if (!mbar_wait(&full[s], round & 1u)) {
+        for (int seg = 0; seg < nseg && ok; ++seg) {
+          // the previous segment's partial must have been read out of TMEM
+          if (kSegmented && seg >= 1 && !mbar_wait(seg_empty, (uint32_t)(seg - 1) & 1u)) {
             atomicOr(failed, 1u);
             ok = false;
             break;
           }
           tc_fence_after_sync();
-          if (kMode == 3) {
-            // MN-major: 16 K rows are two 1024-byte swizzle atoms further
-            const uint64_t ad = smem_desc_mn_sw128(smem_addr(tile_a + s * kTileABytes), kBoxBytes);
-            const uint64_t bd = smem_desc_mn_sw128(smem_addr(tile_b + s * kTileBBytes), kBoxBytes);
+          const uint32_t d = tmem_d + acc * kBN;
+          const int kb0 = seg * seg_blocks, kb1 = min(kb_total, kb0 + seg_blocks);
+          for (int kb = kb0; kb < kb1; ++kb) {
+            const int g = i * kb_total + kb;
+            const int s = g % kStages;
+            const uint32_t round = (uint32_t)(g / kStages);
+            if (!mbar_wait(&full[s], round & 1u)) {
+              atomicOr(failed, 1u);
+              ok = false;
+              break;
+            }
+            tc_fence_after_sync();
+            if (kMode == 3) {
+              // MN-major: 16 K rows are two 1024-byte swizzle atoms further
+              const uint64_t ad = smem_desc_mn_sw128(smem_addr(tile_a + s * kTileABytes), kBoxBytes);
+              const uint64_t bd = smem_desc_mn_sw128(smem_addr(tile_b + s * kTileBBytes), kBoxBytes);
 #pragma unroll
-            for (int kk = 0; kk < kBK / 16; ++kk)
-              umma_bf16(d, ad + 128 * kk, bd + 128 * kk, kIdescMN, (uint32_t)(kb > kb0 || kk > 0));
-          } else {
-            const uint64_t ad = smem_desc_k_sw128(smem_addr(tile_a + s * kTileABytes));
-            const uint64_t bd = smem_desc_k_sw128(smem_addr(tile_b + s * kTileBBytes));
+              for (int kk = 0; kk < kBK / 16; ++kk)
+                umma_bf16(d, ad + 128 * kk, bd + 128 * kk, kIdescMN, (uint32_t)(kb > kb0 || kk > 0));
+            } else {
+              const uint64_t ad = smem_desc_k_sw128(smem_addr(tile_a + s * kTileABytes));
+              const uint64_t bd = smem_desc_k_sw128(smem_addr(tile_b + s * kTileBBytes));
 #pragma unroll
-            for (int kk = 0; kk < kBK / 16; ++kk)
-              umma_bf16(d, ad + 2 * kk, bd + 2 * kk, kIdesc, (uint32_t)(kb > kb0 || kk > 0));
+              for (int kk = 0; kk < kBK / 16; ++kk)
+                umma_bf16(d, ad + 2 * kk, bd + 2 * kk, kIdesc, (uint32_t)(kb > kb0 || kk > 0));
+            }
+            umma_commit(smem_addr(&empty[s]));
           }
-          umma_commit(smem_addr(&empty[s]));
+          // fires once every MMA issued above has completed
+          if (ok) umma_commit(smem_addr(kSegmented ? seg_full : (kPersistent ? &tacc_full[acc] : acc_ready)));
         }
-        // fires once every MMA issued above has completed
-        if (ok) umma_commit(smem_addr(kSegmented ? seg_full : acc_ready));
       }
     }
     __syncwarp();
@@ -275,69 +305,80 @@ gemm_kernel(const __grid_constant__ CUtensorMap xmap, const __grid_constant__ CU
     const uint32_t quarter = (uint32_t)(warp & 3);
     const uint32_t cbase = (uint32_t)((warp - 2) >> 2) * kHalf;
     const uint32_t lane_base = (quarter * 32u) << 16;
-    const int64_t row = (int64_t)tile_m * kBM + quarter * 32 + lane;
-    const int64_t col0 = (int64_t)tile_n * kBN + cbase;
     const int nseg = kSegmented ? (kb_total + kSegBlocks - 1) / kSegBlocks : 1;
     double acc = 0.0;
-    for (int seg = 0; seg < nseg; ++seg) {
-      if (!mbar_wait(kSegmented ? seg_full : acc_ready, kSegmented ? (uint32_t)seg & 1u : 0u)) {
-        atomicOr(failed, 1u);
-        break;
-      }
-      tc_fence_after_sync();
-      const bool last = seg + 1 == nseg;
-      uint32_t p[kHalf];
-#pragma unroll
-      for (int c = 0; c < kHalf; c += 32)
-        tmem_ld_32x32b_x32(tmem_d + lane_base + cbase + (uint32_t)c, *reinterpret_cast<uint32_t(*)[32]>(p + c));
-      tmem_ld_wait();
-      if (kSegmented && !last) {
-        // the partial is in registers: the MMAs may go on with the next segment
-        tc_fence_before_sync();
-        mbar_arrive(seg_empty);
-      }
-      if (kSegmented && seg > 0) {
-        // fold into the running sum (TMEM columns [256, 512)), fp32 round-to-nearest
-#pragma unroll
-        for (int c = 0; c < kHalf; c += 32) {
-          uint32_t q[32];
-          tmem_ld_32x32b_x32(tmem_d + lane_base + kBN + cbase + (uint32_t)c, q);
-          tmem_ld_wait();
-#pragma unroll
-          for (int j = 0; j < 32; ++j)
-            p[c + j] = __float_as_uint(__fadd_rn(__uint_as_float(q[j]), __uint_as_float(p[c + j])));
+    bool alive = true;
+    for (int i = 0; i < ntiles && alive; ++i) {
+      const int t = (int)blockIdx.x + i * (int)gridDim.x;
+      const int tm = t / tiles_n, tn = t - tm * tiles_n;
+      const int64_t row = (int64_t)tm * kBM + quarter * 32 + lane;
+      const int64_t col0 = (int64_t)tn * kBN + cbase;
+      const uint32_t tacc = kPersistent ? (uint32_t)(i & 1) : 0u;
+      for (int seg = 0; seg < nseg; ++seg) {
+        uint64_t* ready = kSegmented ? seg_full : (kPersistent ? &tacc_full[tacc] : acc_ready);
+        const uint32_t parity = kSegmented ? (uint32_t)seg & 1u : (kPersistent ? (uint32_t)(i >> 1) & 1u : 0u);
+        if (!mbar_wait(ready, parity)) {
+          atomicOr(failed, 1u);
+          alive = false;
+          break;
         }
-      }
-      if (kSegmented && !last) {
+        tc_fence_after_sync();
+        const bool last = seg + 1 == nseg;
+        uint32_t p[kHalf];
 #pragma unroll
         for (int c = 0; c < kHalf; c += 32)
-          tmem_st_32x32b_x32(tmem_d + lane_base + kBN + cbase + (uint32_t)c, *reinterpret_cast<uint32_t(*)[32]>(p + c));
-        tmem_st_wait();
-        continue;
-      }
-      if (!kAccum) {
-        // the output error: the sum of squares of the complete tile
+          tmem_ld_32x32b_x32(tmem_d + tacc * kBN + lane_base + cbase + (uint32_t)c,
+                             *reinterpret_cast<uint32_t(*)[32]>(p + c));
+        tmem_ld_wait();
+        if ((kSegmented && !last) || kPersistent) {
+          // the partial is in registers: the MMAs may go on with the next segment (or the
+          // tile after next may use this accumulator)
+          tc_fence_before_sync();
+          mbar_arrive(kPersistent ? &tacc_empty[tacc] : seg_empty);
+        }
+        if (kSegmented && seg > 0) {
+          // fold into the running sum (TMEM columns [256, 512)), fp32 round-to-nearest
 #pragma unroll
-        for (int c = 0; c < kHalf; c += 32) acc += (double)sum_squares32(*reinterpret_cast<uint32_t(*)[32]>(p + c));
-        continue;
-      }
-      // the Hessian and the GPTQ update: the tile row added into H (C)
-      if (row < h_rows) {
-        float* dst = H + row * ld_h + col0;
-        if (col0 + kHalf <= h_cols && ((ld_h | col0) & 3) == 0 && (reinterpret_cast<uintptr_t>(H) & 15) == 0) {
+          for (int c = 0; c < kHalf; c += 32) {
+            uint32_t q[32];
+            tmem_ld_32x32b_x32(tmem_d + lane_base + kBN + cbase + (uint32_t)c, q);
+            tmem_ld_wait();
 #pragma unroll
-          for (int q = 0; q < kHalf / 4; ++q) {
-            float4 v = reinterpret_cast<float4*>(dst)[q];
-            v.x += __uint_as_float(p[4 * q]);
-            v.y += __uint_as_float(p[4 * q + 1]);
-            v.z += __uint_as_float(p[4 * q + 2]);
-            v.w += __uint_as_float(p[4 * q + 3]);
-            reinterpret_cast<float4*>(dst)[q] = v;
+            for (int j = 0; j < 32; ++j)
+              p[c + j] = __float_as_uint(__fadd_rn(__uint_as_float(q[j]), __uint_as_float(p[c + j])));
           }
-        } else {
+        }
+        if (kSegmented && !last) {
 #pragma unroll
-          for (int q = 0; q < kHalf; ++q)
-            if (col0 + q < h_cols) dst[q] += __uint_as_float(p[q]);
+          for (int c = 0; c < kHalf; c += 32)
+            tmem_st_32x32b_x32(tmem_d + lane_base + kBN + cbase + (uint32_t)c, *reinterpret_cast<uint32_t(*)[32]>(p + c));
+          tmem_st_wait();
+          continue;
+        }
+        if (!kAccum) {
+          // the output error: the sum of squares of the complete tile
+#pragma unroll
+          for (int c = 0; c < kHalf; c += 32) acc += (double)sum_squares32(*reinterpret_cast<uint32_t(*)[32]>(p + c));
+          continue;
+        }
+        // the Hessian and the GPTQ update: the tile row added into H (C)
+        if (row < h_rows) {
+          float* dst = H + row * ld_h + col0;
+          if (col0 + kHalf <= h_cols && ((ld_h | col0) & 3) == 0 && (reinterpret_cast<uintptr_t>(H) & 15) == 0) {
+#pragma unroll
+            for (int q = 0; q < kHalf / 4; ++q) {
+              float4 v = reinterpret_cast<float4*>(dst)[q];
+              v.x += __uint_as_float(p[4 * q]);
+              v.y += __uint_as_float(p[4 * q + 1]);
+              v.z += __uint_as_float(p[4 * q + 2]);
+              v.w += __uint_as_float(p[4 * q + 3]);
+              reinterpret_cast<float4*>(dst)[q] = v;
+            }
+          } else {
+#pragma unroll
+            for (int q = 0; q < kHalf; ++q)
+              if (col0 + q < h_cols) dst[q] += __uint_as_float(p[q]);
+          }
         }
       }
     }
@@ -353,10 +394,14 @@ gemm_kernel(const __grid_constant__ CUtensorMap xmap, const __grid_constant__ CU
     // a wait that ran out makes the whole tile NaN (written after the partial sums above)
     if (*failed && warp >= 2) {
       const uint32_t quarter = (uint32_t)(warp & 3);
-      const int64_t row = (int64_t)tile_m * kBM + quarter * 32 + lane;
-      const int64_t c0 = (int64_t)tile_n * kBN + ((warp - 2) >> 2) * (kBN / 2);
-      if (row < h_rows)
-        for (int64_t c = c0; c < c0 + kBN / 2 && c < h_cols; ++c) H[row * ld_h + c] = __int_as_float(0x7FC00000);
+      for (int i = 0; i < ntiles; ++i) {
+        const int t = (int)blockIdx.x + i * (int)gridDim.x;
+        const int tm = t / tiles_n, tn = t - tm * tiles_n;
+        const int64_t row = (int64_t)tm * kBM + quarter * 32 + lane;
+        const int64_t c0 = (int64_t)tn * kBN + ((warp - 2) >> 2) * (kBN / 2);
+        if (row < h_rows)
+          for (int64_t c = c0; c < c0 + kBN / 2 && c < h_cols; ++c) H[row * ld_h + c] = __int_as_float(0x7FC00000);
+      }
       if (threadIdx.x == 64) atomicOr(&g_output_error_flags, kErrMbarTimeout);
     }
   } else if (threadIdx.x == 0) {
@@ -463,7 +508,7 @@ cudaError_t launch_output_error(const void* x, int64_t tokens, int64_t n, int64_
   const int64_t tiles_n = (m + kBN - 1) / kBN;
   const int64_t tiles = output_error_tiles(tokens, m);
   gemm_kernel<0><<<(unsigned)tiles, kGemmThreads, kGemmSmemBytes, stream>>>(
-      xmap, wmap, (int)(n_pad / kBK), (int)tiles_n, partials, nullptr, 0, 0, 0);
+      xmap, wmap, (int)(n_pad / kBK), (int)tiles_n, (int)tiles, partials, nullptr, 0, 0, 0);
   err = cudaGetLastError();
   if (err != cudaSuccess) return err;
   reduce_kernel<<<1, 256, 0, stream>>>(partials, tiles, out);
@@ -493,7 +538,7 @@ cudaError_t launch_hessian_full(const void* x, int64_t tokens, int64_t n, int64_
     err = ensure_dynamic_smem(reinterpret_cast<const void*>(gemm_kernel<3>), (int)kGemmSmemBytes);
     if (err != cudaSuccess) return err;
     gemm_kernel<3><<<(unsigned)tiles, kGemmThreads, kGemmSmemBytes, stream>>>(
-        map, map, (int)((tokens + kBK - 1) / kBK), (int)tiles_n, nullptr, H, n, n, ld_h);
+        map, map, (int)((tokens + kBK - 1) / kBK), (int)tiles_n, (int)tiles, nullptr, H, n, n, ld_h);
     return cudaGetLastError();
   }
   // X with rows that are not 16-byte aligned: transposed first (tokens contiguous per
@@ -519,7 +564,7 @@ cudaError_t launch_hessian_full(const void* x, int64_t tokens, int64_t n, int64_
       ensure_dynamic_smem(reinterpret_cast<const void*>(gemm_kernel<1>), (int)kGemmSmemBytes);
   if (attr_status != cudaSuccess) return attr_status;
   gemm_kernel<1><<<(unsigned)tiles, kGemmThreads, kGemmSmemBytes, stream>>>(
-      amap, bmap, (int)((tokens + kBK - 1) / kBK), (int)tiles_n, nullptr, H, n, n, ld_h);
+      amap, bmap, (int)((tokens + kBK - 1) / kBK), (int)tiles_n, (int)tiles, nullptr, H, n, n, ld_h);
   return cudaGetLastError();
 }
 
@@ -546,8 +591,12 @@ cudaError_t launch_gemm_accumulate(const void* a, const void* b, int64_t m, int6
   if (err != cudaSuccess) return err;
   const int64_t tiles_n = (nn + kBN - 1) / kBN;
   const int64_t tiles = ((m + kBM - 1) / kBM) * tiles_n;
-  gemm_kernel<2><<<(unsigned)tiles, kGemmThreads, kGemmSmemBytes, stream>>>(
-      amap, bmap, (int)((k + kBK - 1) / kBK), (int)tiles_n, nullptr, C, m, nn, ld_c);
+  // persistent: one CTA per SM (the shared-memory ring allows no more), tiles strided
+  DeviceInfo info;
+  if ((err = current_device_info(&info)) != cudaSuccess) return err;
+  const int64_t grid = std::max<int64_t>(1, std::min<int64_t>(tiles, info.sm_count));
+  gemm_kernel<2><<<(unsigned)grid, kGemmThreads, kGemmSmemBytes, stream>>>(
+      amap, bmap, (int)((k + kBK - 1) / kBK), (int)tiles_n, (int)tiles, nullptr, C, m, nn, ld_c);
   return cudaGetLastError();
 }
 
