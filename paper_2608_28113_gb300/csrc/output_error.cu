@@ -57,11 +57,37 @@ constexpr uint32_t kTmemCols = kBN;  // fp32 accumulator: 128 lanes x 256 column
 constexpr int kSegBlocks = 32;
 constexpr uint32_t kTmemColsSeg = 2 * kBN;
 constexpr uint32_t kGemmSmemBytes = kStages * kStageBytes + 1024 /* alignment */ + 256 /* barriers */;
+// the GPTQ update also stages its epilogue: barriers in a 1 KB block (keeping the staging
+// buffers 1 KB aligned for the 128-byte swizzle), then 4 KB per epilogue warp
+constexpr uint32_t kUpdateSmemBytes = kStages * kStageBytes + 1024 /* alignment */ + 1024 + 8 * 4096;
 constexpr uint32_t kIdesc = idesc_bf16_f32(kBM, kBN);
 constexpr uint32_t kIdescMN = idesc_bf16_f32_mn(kBM, kBN);
 constexpr uint32_t kBoxBytes = 64 * kBK * 2;  // mode 3: one 64-channel x 64-token TMA box
 
 __device__ uint32_t g_output_error_flags = 0;
+
+// ---------------------------------------------------------------- TMA reduce-add
+// The GPTQ update's epilogue adds each tile into the running weights with TMA: a warp
+// stages 32 rows x 32 fp32 columns (4 KB, 128-byte swizzled, as the tensor map says) and
+// one lane issues a bulk reduce-add, which the L2 applies in fp32 round-to-nearest without
+// the SM reading the weights.  The coordinates are (column, row), column a multiple of 4.
+constexpr uint32_t kStageRows = 32, kStageCols = 32;
+constexpr uint32_t kStageBufBytes = kStageRows * kStageCols * 4;  // per epilogue warp
+
+__device__ __forceinline__ void tma_reduce_add_2d(const CUtensorMap* map, const void* src, int32_t c0, int32_t c1) {
+  asm volatile("cp.reduce.async.bulk.tensor.2d.global.shared::cta.add.tile.bulk_group [%0, {%1, %2}], [%3];" ::"l"(
+                   reinterpret_cast<uint64_t>(map)),
+               "r"(c0), "r"(c1), "r"(smem_addr(src))
+               : "memory");
+}
+__device__ __forceinline__ void bulk_commit() { asm volatile("cp.async.bulk.commit_group;" ::: "memory"); }
+// every committed bulk operation has finished reading shared memory
+__device__ __forceinline__ void bulk_wait_read() { asm volatile("cp.async.bulk.wait_group.read 0;" ::: "memory"); }
+// every committed bulk operation has completed
+__device__ __forceinline__ void bulk_wait_all() { asm volatile("cp.async.bulk.wait_group 0;" ::: "memory"); }
+__device__ __forceinline__ void fence_proxy_async_smem() {
+  asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+}
 
 // ---------------------------------------------------------------- residual
 __device__ __forceinline__ uint32_t bf16x2_pack(__nv_bfloat16 lo, __nv_bfloat16 hi) {
@@ -144,7 +170,7 @@ __device__ __forceinline__ float sum_squares32(const uint32_t (&r)[32]) {
 template <int kMode>
 __global__ void __launch_bounds__(kGemmThreads, 1)
 gemm_kernel(const __grid_constant__ CUtensorMap xmap, const __grid_constant__ CUtensorMap wmap,
-            int kb_half, int tiles_n, int tiles_total, double* __restrict__ partials, float* __restrict__ H,
+            const __grid_constant__ CUtensorMap cmap, int kb_half, int tiles_n, int tiles_total, double* __restrict__ partials, float* __restrict__ H,
             int64_t h_rows, int64_t h_cols, int64_t ld_h) {
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
@@ -361,7 +387,32 @@ gemm_kernel(const __grid_constant__ CUtensorMap xmap, const __grid_constant__ CU
           for (int c = 0; c < kHalf; c += 32) acc += (double)sum_squares32(*reinterpret_cast<uint32_t(*)[32]>(p + c));
           continue;
         }
-        // the Hessian and the GPTQ update: the tile row added into H (C)
+        if (kPersistent) {
+          // the GPTQ update: staged 32 x 32 boxes reduce-added into C by TMA.  Row `lane`
+          // of a box holds 128 bytes; the 128-byte swizzle puts its 16-byte chunk k at
+          // k ^ (lane & 7), so a warp's stores hit every bank once.
+          uint8_t* stage = smem + kStages * kStageBytes + 1024 + (uint32_t)(warp - 2) * kStageBufBytes;
+          const int64_t row0 = (int64_t)tm * kBM + quarter * 32;
+#pragma unroll
+          for (int c = 0; c < kHalf; c += 32) {
+            // the previous box must have been read out of the buffer
+            if (lane == 0) bulk_wait_read();
+            __syncwarp();
+            float4* rowp = reinterpret_cast<float4*>(stage + lane * 128);
+#pragma unroll
+            for (int k = 0; k < 8; ++k)
+              rowp[k ^ (lane & 7)] = make_float4(__uint_as_float(p[c + 4 * k]), __uint_as_float(p[c + 4 * k + 1]),
+                                                 __uint_as_float(p[c + 4 * k + 2]), __uint_as_float(p[c + 4 * k + 3]));
+            fence_proxy_async_smem();
+            __syncwarp();
+            if (lane == 0 && row0 < h_rows && col0 + c < h_cols) {
+              tma_reduce_add_2d(&cmap, stage, (int32_t)(col0 + c), (int32_t)row0);
+              bulk_commit();
+            }
+          }
+          continue;
+        }
+        // the Hessian: the tile row added into H
         if (row < h_rows) {
           float* dst = H + row * ld_h + col0;
           if (col0 + kHalf <= h_cols && ((ld_h | col0) & 3) == 0 && (reinterpret_cast<uintptr_t>(H) & 15) == 0) {
@@ -382,6 +433,8 @@ gemm_kernel(const __grid_constant__ CUtensorMap xmap, const __grid_constant__ CU
         }
       }
     }
+    // the update's reduce-adds complete before the CTA ends
+    if (kPersistent && lane == 0) bulk_wait_all();
     if (!kAccum) {
 #pragma unroll
       for (int off = 16; off > 0; off >>= 1) acc += __shfl_xor_sync(0xFFFFFFFFu, acc, off);
@@ -508,7 +561,7 @@ cudaError_t launch_output_error(const void* x, int64_t tokens, int64_t n, int64_
   const int64_t tiles_n = (m + kBN - 1) / kBN;
   const int64_t tiles = output_error_tiles(tokens, m);
   gemm_kernel<0><<<(unsigned)tiles, kGemmThreads, kGemmSmemBytes, stream>>>(
-      xmap, wmap, (int)(n_pad / kBK), (int)tiles_n, (int)tiles, partials, nullptr, 0, 0, 0);
+      xmap, wmap, wmap, (int)(n_pad / kBK), (int)tiles_n, (int)tiles, partials, nullptr, 0, 0, 0);
   err = cudaGetLastError();
   if (err != cudaSuccess) return err;
   reduce_kernel<<<1, 256, 0, stream>>>(partials, tiles, out);
@@ -538,7 +591,7 @@ cudaError_t launch_hessian_full(const void* x, int64_t tokens, int64_t n, int64_
     err = ensure_dynamic_smem(reinterpret_cast<const void*>(gemm_kernel<3>), (int)kGemmSmemBytes);
     if (err != cudaSuccess) return err;
     gemm_kernel<3><<<(unsigned)tiles, kGemmThreads, kGemmSmemBytes, stream>>>(
-        map, map, (int)((tokens + kBK - 1) / kBK), (int)tiles_n, (int)tiles, nullptr, H, n, n, ld_h);
+        map, map, map, (int)((tokens + kBK - 1) / kBK), (int)tiles_n, (int)tiles, nullptr, H, n, n, ld_h);
     return cudaGetLastError();
   }
   // X with rows that are not 16-byte aligned: transposed first (tokens contiguous per
@@ -564,7 +617,7 @@ cudaError_t launch_hessian_full(const void* x, int64_t tokens, int64_t n, int64_
       ensure_dynamic_smem(reinterpret_cast<const void*>(gemm_kernel<1>), (int)kGemmSmemBytes);
   if (attr_status != cudaSuccess) return attr_status;
   gemm_kernel<1><<<(unsigned)tiles, kGemmThreads, kGemmSmemBytes, stream>>>(
-      amap, bmap, (int)((tokens + kBK - 1) / kBK), (int)tiles_n, (int)tiles, nullptr, H, n, n, ld_h);
+      amap, bmap, bmap, (int)((tokens + kBK - 1) / kBK), (int)tiles_n, (int)tiles, nullptr, H, n, n, ld_h);
   return cudaGetLastError();
 }
 
@@ -573,7 +626,7 @@ cudaError_t launch_gemm_accumulate(const void* a, const void* b, int64_t m, int6
   EncodeTiledFn encode = nullptr;
   cudaError_t err = encode_tiled_fn(&encode);
   if (err != cudaSuccess) return err;
-  CUtensorMap amap, bmap;
+  CUtensorMap amap, bmap, cmap;
   const cuuint64_t adims[2] = {(cuuint64_t)k, (cuuint64_t)m};
   const cuuint64_t bdims[2] = {(cuuint64_t)k, (cuuint64_t)nn};
   const cuuint64_t strides[1] = {(cuuint64_t)k * 2};
@@ -587,7 +640,16 @@ cudaError_t launch_gemm_accumulate(const void* a, const void* b, int64_t m, int6
              CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
              CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) != CUDA_SUCCESS)
     return cudaErrorInvalidValue;
-  err = ensure_dynamic_smem(reinterpret_cast<const void*>(gemm_kernel<2>), (int)kGemmSmemBytes);
+  // C [m, nn] fp32 (row stride ld_c), reduce-added in 32 x 32 boxes
+  const cuuint64_t cdims[2] = {(cuuint64_t)nn, (cuuint64_t)m};
+  const cuuint64_t cstrides[1] = {(cuuint64_t)ld_c * 4};
+  const cuuint32_t cbox[2] = {kStageCols, kStageRows};
+  if ((reinterpret_cast<uintptr_t>(C) & 15) != 0 || (ld_c * 4) % 16 != 0) return cudaErrorInvalidValue;
+  if (encode(&cmap, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, 2, C, cdims, cstrides, cbox, estr, CU_TENSOR_MAP_INTERLEAVE_NONE,
+             CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) !=
+      CUDA_SUCCESS)
+    return cudaErrorInvalidValue;
+  err = ensure_dynamic_smem(reinterpret_cast<const void*>(gemm_kernel<2>), (int)kUpdateSmemBytes);
   if (err != cudaSuccess) return err;
   const int64_t tiles_n = (nn + kBN - 1) / kBN;
   const int64_t tiles = ((m + kBM - 1) / kBM) * tiles_n;
@@ -595,8 +657,8 @@ cudaError_t launch_gemm_accumulate(const void* a, const void* b, int64_t m, int6
   DeviceInfo info;
   if ((err = current_device_info(&info)) != cudaSuccess) return err;
   const int64_t grid = std::max<int64_t>(1, std::min<int64_t>(tiles, info.sm_count));
-  gemm_kernel<2><<<(unsigned)grid, kGemmThreads, kGemmSmemBytes, stream>>>(
-      amap, bmap, (int)((k + kBK - 1) / kBK), (int)tiles_n, (int)tiles, nullptr, C, m, nn, ld_c);
+  gemm_kernel<2><<<(unsigned)grid, kGemmThreads, kUpdateSmemBytes, stream>>>(
+      amap, bmap, cmap, (int)((k + kBK - 1) / kBK), (int)tiles_n, (int)tiles, nullptr, C, m, nn, ld_c);
   return cudaGetLastError();
 }
 
