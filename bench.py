@@ -558,14 +558,16 @@ def kernels_per_matrix(work: Work) -> int:
 def timed(fn, reps, flush=None):
     """Average CUDA-event time (ms) of fn over reps calls on the current stream, after one
     untimed call (library loading, handle creation and first-use costs stay out).  With
-    `flush` (a device buffer larger than L2), each call is timed on its own after the
-    buffer is rewritten outside the timed window, so inputs smaller than L2 (a weight
-    matrix) are read from HBM every time."""
+    `flush` (two device buffers, each larger than L2), each call is timed on its own after
+    the first buffer is rewritten and the second read, outside the timed window, so inputs
+    smaller than L2 (a weight matrix) are read from HBM every time, and the flush's dirty
+    lines have been written back before the call starts."""
     fn()
     if flush is not None:
         total = 0.0
         for _ in range(reps):
-            flush.fill_(1.0)
+            flush[0].fill_(1.0)
+            flush[1].sum()
             e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
             e0.record()
             fn()
@@ -904,9 +906,10 @@ def gpu_arm(args, d: Dist):
     fp32_peak = props.multi_processor_count * 128 * sm_max_mhz * 1e6
     reps = max(3, min(args.steps, 20))
     # W of a matrix can be smaller than L2: its kernels are timed after an L2 flush (twice
-    # the L2 size written between calls, outside the timed window)
+    # the L2 size written, then another twice read, between calls, outside the timed window)
     l2 = int(getattr(props, "L2_cache_size", 0) or (126 << 20))
-    flush = torch.empty(2 * l2 // 4, dtype=torch.float32, device=dev)
+    flush = (torch.empty(2 * l2 // 4, dtype=torch.float32, device=dev),
+             torch.zeros(2 * l2 // 4, dtype=torch.float32, device=dev))
     ms_init = sum(timed(lambda M=M: init_codes(hs, work, M), reps, flush) for M in work.mats)
     ms_h_alone = timed(lambda: [g.replay() for g in graphs.gh[0]], reps)
     sweep = []

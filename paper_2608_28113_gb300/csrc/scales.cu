@@ -441,6 +441,7 @@ refine_kernel(const uint4* __restrict__ w, int64_t ld_w, const float* __restrict
   for (int j = 0; j < 8; ++j) hv2[j] = make_float2(1.0f, 1.0f);
   float hsum = 16.0f;  // sum of the lane's 16 h values
 
+  const bool linear_units = ld_w == (int64_t)ng * 16 && ng % 32 == 0;
   // (row, chunk) of unit u, advanced by warps_total units per step without a division
   const int row_step = (int)(warps_total / chunks);
   const int chunk_step = (int)(warps_total - (int64_t)row_step * chunks);
@@ -454,6 +455,11 @@ refine_kernel(const uint4* __restrict__ w, int64_t ld_w, const float* __restrict
     const int gcol = chunk * 32 + lane;
     const bool active = gcol < ng;
     const int64_t wofs = row * ld_w + (int64_t)gcol * 16;  // first element of the group
+    // the warp's next unit (1 KB of W) requested into L2 while this one is scored, so a W
+    // that is not in L2 yet is not waited for unit by unit.  With contiguous rows of whole
+    // units, unit u holds the elements [512 u, 512 u + 512); one lane per 128 bytes.
+    if (linear_units && (lane & 3) == 0 && u + warps_total < units)
+      asm volatile("prefetch.global.L2 [%0];" ::"l"(w + ((u + warps_total) * 512 + lane * 16) / 8));
 
     if (chunk != cur_chunk) {
       cur_chunk = chunk;
