@@ -170,8 +170,8 @@ __device__ __forceinline__ float sum_squares32(const uint32_t (&r)[32]) {
 template <int kMode>
 __global__ void __launch_bounds__(kGemmThreads, 1)
 gemm_kernel(const __grid_constant__ CUtensorMap xmap, const __grid_constant__ CUtensorMap wmap,
-            const __grid_constant__ CUtensorMap cmap, int kb_half, int tiles_n, int tiles_total, double* __restrict__ partials, float* __restrict__ H,
-            int64_t h_rows, int64_t h_cols, int64_t ld_h) {
+            const __grid_constant__ CUtensorMap cmap, int kb_half, int tiles_n, int tiles_total,
+            double* __restrict__ partials, float* __restrict__ H, int64_t h_rows, int64_t h_cols, int64_t ld_h) {
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
   uint8_t* tile_a = smem;
@@ -181,8 +181,8 @@ gemm_kernel(const __grid_constant__ CUtensorMap xmap, const __grid_constant__ CU
   uint64_t* acc_ready = empty + kStages;
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(acc_ready + 1);
   uint32_t* failed = tmem_slot + 1;
-  uint64_t* seg_full = acc_ready + 2;  // mode 1: the partial of a segment is complete
-  uint64_t* seg_empty = seg_full + 1;  // mode 1: the partial has been folded into the sum
+  uint64_t* seg_full = acc_ready + 2;  // segmented modes: a segment's partial is complete
+  uint64_t* seg_empty = seg_full + 1;  // segmented modes: the partial has been read out
   uint64_t* tacc_full = seg_empty + 1;  // mode 2: accumulator a holds a finished tile
   uint64_t* tacc_empty = tacc_full + 2;  // mode 2: accumulator a has been read out
   double* warp_sum = reinterpret_cast<double*>(smem + kStages * kStageBytes + 128);
@@ -191,7 +191,7 @@ gemm_kernel(const __grid_constant__ CUtensorMap xmap, const __grid_constant__ CU
   // output error (K = 2 n); the GPTQ update's K = 6 B is a single segment anyway
   constexpr bool kSegmented = kMode != 2;
   // The GPTQ update is persistent: a CTA takes tiles blockIdx.x, + gridDim.x, ... and
-  // alternates two 256-column accumulators, so a tile's epilogue (the read-modify-write of
+  // alternates two 256-column accumulators, so a tile's epilogue (the TMA reduce-add into
   // the running weights) runs alongside the next tile's loads and MMAs.  The other modes
   // take one tile per CTA.
   constexpr bool kPersistent = kMode == 2;
