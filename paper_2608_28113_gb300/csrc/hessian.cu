@@ -56,17 +56,22 @@ constexpr size_t kRingBytes = (size_t)kStages * kStageBytes;
 constexpr int64_t kMaxRowsPerCta = 1024 * kPhases;  // <= 1024 sequential adds per thread
 constexpr int kMaxCluster = 8;
 
+// acc += x^2 for the two bf16 values of a 32-bit word, taken straight from its halves by
+// the mixed-precision FMA (a bf16 x bf16 product is exact in fp32; the add rounds once, as
+// an fp32 FMA of the widened values would): one instruction per element, no unpacking.
+__device__ __forceinline__ void accum_sq2(float& lo_acc, float& hi_acc, uint32_t pair) {
+  asm("{\n\t.reg .b16 l, h;\n\tmov.b32 {l, h}, %2;\n\t"
+      "fma.rn.f32.bf16 %0, l, l, %0;\n\t"
+      "fma.rn.f32.bf16 %1, h, h, %1;\n\t}"
+      : "+f"(lo_acc), "+f"(hi_acc)
+      : "r"(pair));
+}
+
 __device__ __forceinline__ void accum_sq8(float (&acc)[8], const uint4& v) {
-  const float f0 = bf16_lo(v.x), f1 = bf16_hi(v.x), f2 = bf16_lo(v.y), f3 = bf16_hi(v.y);
-  const float f4 = bf16_lo(v.z), f5 = bf16_hi(v.z), f6 = bf16_lo(v.w), f7 = bf16_hi(v.w);
-  acc[0] = __fmaf_rn(f0, f0, acc[0]);
-  acc[1] = __fmaf_rn(f1, f1, acc[1]);
-  acc[2] = __fmaf_rn(f2, f2, acc[2]);
-  acc[3] = __fmaf_rn(f3, f3, acc[3]);
-  acc[4] = __fmaf_rn(f4, f4, acc[4]);
-  acc[5] = __fmaf_rn(f5, f5, acc[5]);
-  acc[6] = __fmaf_rn(f6, f6, acc[6]);
-  acc[7] = __fmaf_rn(f7, f7, acc[7]);
+  accum_sq2(acc[0], acc[1], v.x);
+  accum_sq2(acc[2], acc[3], v.y);
+  accum_sq2(acc[4], acc[5], v.z);
+  accum_sq2(acc[6], acc[7], v.w);
 }
 
 template <int CS>
