@@ -53,7 +53,12 @@ def parse():
     p.add_argument("--steps", type=int, default=50)
     p.add_argument("--warmup", type=int, default=3)
     p.add_argument("--impl", choices=["hscale", "reference"], default="hscale")
-    p.add_argument("--workload", default="llama8b-q_proj", choices=sorted(wl.WORKLOADS))
+    p.add_argument("--workload", default="llama8b-decoder", choices=sorted(wl.WORKLOADS),
+                   help="the step's workload (default: one layer of the full 8B decoder, the largest "
+                        "single-GPU configuration; per-model time = 32 layers)")
+    p.add_argument("--extra-workload", default="llama70b-mlp", choices=["none"] + sorted(wl.WORKLOADS),
+                   help="a second workload measured in the same process and reported under its own key "
+                        "(default: the 70B MLP block with its window sweep k = 1, 2, 4, 8, 16)")
     p.add_argument("--k", type=int, default=None, help="symmetric window half-width (default: workload's first)")
     p.add_argument("--window", default=None,
                    help="asymmetric window 'D,U' (codes c0-D .. c0+U); e.g. 9,6 is the paper's K = 16 default")
@@ -81,6 +86,9 @@ def parse():
                         "layer -4 %%, 70B MLP block -11 %% per step); off for one Hessian-bound input "
                         "space (q_proj: -1.5 %% per step, while the Hessian pass shares its SMs)")
     p.add_argument("--no-cpu-baseline", action="store_true")
+    p.add_argument("--cpu-baseline", choices=["full", "sample"], default="full",
+                   help="full (default): the oracle over the step's whole layer on all host cores, "
+                        "verified against the GPU outputs; sample: a bounded sample extrapolated")
     p.add_argument("--no-output-error", action="store_true",
                    help="skip the tensor-core layer-output error evaluation")
     p.add_argument("--no-gptq", action="store_true",
@@ -137,11 +145,13 @@ def measured_peaks():
         return FALLBACK_HBM_GBS, "fallback", {}
 
 
-def profiled_traffic(workload: str, chunk: int, n: int):
-    """DRAM bytes per Hessian launch from the committed ncu summary, if the kernel's sources
-    are unchanged since that capture and the launch shape matches; else None."""
+def step_traffic(work) -> float | None:
+    """DRAM bytes per Hessian launch of the step (the mean over its launches), from the
+    committed ncu summary of the workload: one figure per launch shape (chunk tokens,
+    channels).  None when the kernel's sources changed since that capture, or a launch
+    shape of the step was not captured."""
     import hashlib
-    path = os.path.join(ROOT, "profiles", f"hessian_colsumsq_{workload}.traffic.json")
+    path = os.path.join(ROOT, "profiles", f"hessian_colsumsq_{work.W.name}.traffic.json")
     try:
         with open(path) as f:
             d = json.load(f)
@@ -149,9 +159,18 @@ def profiled_traffic(workload: str, chunk: int, n: int):
         for src in d["kernel_sources"]:
             with open(os.path.join(ROOT, src), "rb") as f:
                 h.update(f.read())
-        if h.hexdigest() != d["kernel_sources_sha256"] or d["chunk_tokens"] != chunk or d["n"] != n:
+        if h.hexdigest() != d["kernel_sources_sha256"]:
             return None
-        return int(d["dram_bytes_per_launch"])
+        per_shape = {(int(e["chunk_tokens"]), int(e["n"])): float(e["dram_bytes_per_launch"]) for e in d["shapes"]}
+        total, launches = 0.0, 0
+        for S, c0, c1 in work.pieces:
+            for t0, t1 in hessian_calls(S, c0, c1):
+                key = (t1 - t0, c1 - c0)
+                if key not in per_shape:
+                    return None
+                total += per_shape[key]
+                launches += 1
+        return total / launches if launches else None
     except Exception:
         return None
 
@@ -355,7 +374,8 @@ def hessian_block(hs, S: Space, c0: int, c1: int):
     h = S.h[c0:c1]
     h.zero_()
     for t0, t1 in hessian_calls(S, c0, c1):
-        hs.hscale_hessian_diag_accumulate(S.x[t0:t1, c0:c1], h)
+        # X is resident and complete before the step starts: the chunk kernels may overlap
+        hs.hscale_hessian_diag_accumulate_ex(S.x[t0:t1, c0:c1], h, hs.HSCALE_HESSIAN_X_READY)
 
 
 def refine_block(hs, work: Work, M, c0: int, c1: int, down, up, ctas_per_sm=0):
@@ -652,7 +672,7 @@ def _oracle_step(W: wl.Workload, win, budget_s: float, init: str, threads: int):
 
 def cpu_baseline(W: wl.Workload, win, budget_s: float = 12.0, init: str = "rtn"):
     """The fp64 oracle timed on the host's cores (all of them, and one thread on a shorter
-    sample), extrapolated to the whole step."""
+    sample), extrapolated to the whole step from a bounded sample."""
     import oracle
     oracle.build()
     cores = len(os.sched_getaffinity(0)) if hasattr(os, "sched_getaffinity") else os.cpu_count()
@@ -668,6 +688,98 @@ def cpu_baseline(W: wl.Workload, win, budget_s: float = 12.0, init: str = "rtn")
         "single_thread_sample": "; ".join(samples1),
         "seconds_per_step": step,
         "hessian_tokens_channels_per_s": h_tc / max(step, 1e-30),
+    }
+
+
+def cpu_baseline_full(work: Work, win, single_thread_budget_s: float = 4.0) -> dict:
+    """The fp64 oracle over the step's whole layer on all host cores, timed part by part
+    (steady clock): the Hessian pass over every calibration chunk of every input space,
+    then per matrix the global scale, the initial codes and the search with packing.  Each
+    result is checked against the GPU's outputs of the step: h within 1e-4 relative; s_g
+    bit for bit; codes and nibbles bit for bit in every group that is not an oracle near-tie
+    (the search takes the GPU's fp32 h, so both sides search the same input).  X and W are
+    copied to the host outside the timed parts.  One thread is timed on a bounded sample."""
+    import oracle
+    oracle.build()
+    cores = len(os.sched_getaffinity(0)) if hasattr(os, "sched_getaffinity") else os.cpu_count()
+    oracle.set_threads(cores)
+    down, up = win
+    t_h = t_init = t_search = 0.0
+    h_rel = 0.0
+    tok_ch = 0
+    for S in work.spaces.values():
+        h_ref = np.zeros(S.n)
+        for c in range(S.nchunks):
+            xb = wl.bf16_bits(S.x[c * S.chunk:(c + 1) * S.chunk])
+            t0 = time.perf_counter()
+            oracle.hessian_accumulate(xb, h_ref)
+            t_h += time.perf_counter() - t0
+        tok_ch += S.tokens * S.n
+        hg = S.h.double().cpu().numpy()
+        h_rel = max(h_rel, float(np.max(np.abs(hg - h_ref) / np.maximum(h_ref, 1e-300))))
+    mism = ties = groups = 0
+    sg_ok = True
+    for M in work.mats:
+        wb = wl.bf16_bits(M.w)
+        hg = M.space.h.cpu().numpy().astype(np.float32)
+        t0 = time.perf_counter()
+        s_g, _ = oracle.global_scale(wb)
+        c0 = oracle.fourover6_codes(wb, s_g)[0] if work.init.startswith("4over6") else oracle.rtn_codes(wb, s_g)
+        t_init += time.perf_counter() - t0
+        t0 = time.perf_counter()
+        ref = oracle.refine(wb, hg, s_g, c0, down, up)
+        t_search += time.perf_counter() - t0
+        sg_ok &= bool(np.float32(s_g) == np.float32(M.sg.item()))
+        ok = ref["near_tie"] == 0
+        codes = M.codes.cpu().numpy()
+        packed = M.packed.cpu().numpy().reshape(M.m, M.n // 16, 8)
+        bad = (codes != ref["codes"]) | np.any(packed != ref["packed"].reshape(M.m, M.n // 16, 8), axis=2)
+        mism += int(np.count_nonzero(bad & ok))
+        ties += int(np.count_nonzero(~ok))
+        groups += M.groups
+        del ref, wb
+    total = t_h + t_init + t_search
+    # one thread, bounded: the first chunk of the first input space and the first 64 rows of
+    # every matrix, scaled to the whole layer by tokens and by rows
+    oracle.set_threads(1)
+    t1 = 0.0
+    S0 = next(iter(work.spaces.values()))
+    xb = wl.bf16_bits(S0.x[:S0.chunk])
+    h1 = np.zeros(S0.n)
+    t0 = time.perf_counter()
+    oracle.hessian_accumulate(xb, h1)
+    per_tc = (time.perf_counter() - t0) / (S0.chunk * S0.n)
+    t1 += per_tc * tok_ch
+    for M in work.mats:
+        rows = min(M.m, 64)
+        wb = wl.bf16_bits(M.w[:rows])
+        s_g = np.float32(M.sg.item())
+        t0 = time.perf_counter()
+        c0 = oracle.rtn_codes(wb, s_g)
+        oracle.refine(wb, M.space.h.cpu().numpy().astype(np.float32), s_g, c0, down, up)
+        t1 += (time.perf_counter() - t0) * M.m / rows
+    oracle.set_threads(cores)
+    n_layers = work.W.n_layers
+    return {
+        "value": work.groups / total, "unit": UNIT, "cores": cores, "kind": "oracle",
+        "sample": (f"full: the fp64 C oracle over the whole layer ({work.W.name} layer 0: {work.groups} groups, "
+                   f"{tok_ch} token-channels of X, window -{down}/+{up}, {work.init} start) on {cores} threads, "
+                   f"steady-clock timed: Hessian pass {t_h:.2f} s, global scale + initial codes {t_init:.2f} s, "
+                   f"search + pack {t_search:.2f} s"
+                   + (f"; per model {n_layers} layers, extrapolated x{n_layers}: {total * n_layers:.1f} s"
+                      if n_layers > 1 else "")),
+        "seconds_per_layer": total,
+        "seconds_per_model": total * n_layers if n_layers > 1 else None,
+        "seconds_per_model_note": f"extrapolated x{n_layers} from layer 0" if n_layers > 1 else None,
+        "phases_s": {"hessian": t_h, "init": t_init, "search": t_search},
+        "hessian_tokens_channels_per_s": tok_ch / t_h if t_h > 0 else None,
+        "search_groups_per_s": groups / t_search if t_search > 0 else None,
+        "verified": {"h_max_rel_err": h_rel, "h_ok": h_rel <= 1e-4, "global_scale_bit_exact": sg_ok,
+                     "groups": groups, "near_ties": ties, "mismatches_outside_near_ties": mism},
+        "single_thread_value": work.groups / t1,
+        "single_thread_sample": ("one thread on a bounded sample extrapolated to the layer: the first "
+                                 f"{S0.chunk}-token chunk of {S0.name} (scaled by token-channels) and the "
+                                 "first 64 rows of every matrix (scaled by rows)"),
     }
 
 
@@ -854,14 +966,12 @@ def shift_statistics(work: Work, win, sample_rows: int = 16):
 
 
 # ------------------------------------------------------------------ GPU arm
-def gpu_arm(args, d: Dist):
-    import paper_2608_28113_gb300 as hs
-    hs.load()
-    torch.cuda.set_device(d.local)
-    dev = torch.device("cuda", d.local)
-    W = wl.WORKLOADS[args.workload]
-    win = window_of(args, W)
-    work = Work(W, d.rank, win, dev, tokens=args.tokens, init=args.init, col_block=args.col_block)
+def measure_workload(hs, d: Dist, args, W: wl.Workload, win, dev, overlap_ctas: int, pipeline: str,
+                     tokens=None, init="rtn", col_block=0):
+    """One workload's timed steps (CUDA graphs, max over ranks), the Hessian and search
+    figures, and the search over every window of the workload timed per kernel.  Returns
+    (result dict, work); the work keeps the step's outputs."""
+    work = Work(W, d.rank, win, dev, tokens=tokens, init=init, col_block=col_block)
     work.ws = torch.empty(hs.hscale_rtn_workspace_bytes(), dtype=torch.uint8, device=dev)
     torch.cuda.synchronize()
 
@@ -874,9 +984,9 @@ def gpu_arm(args, d: Dist):
     ms_eager = timed(lambda: run_step(hs, work), args.steps)
 
     # timed region: the same launches replayed from CUDA graphs
-    pipelined = work.pipelined(args.pipeline)
-    args.overlap_ctas = work.overlap_ctas(args.overlap_ctas, pipelined)
-    graphs = StepGraphs(hs, work, args.overlap_ctas, pipeline=pipelined)
+    pipelined = work.pipelined(pipeline)
+    overlap = work.overlap_ctas(overlap_ctas, pipelined)
+    graphs = StepGraphs(hs, work, overlap, pipeline=pipelined)
     for _ in range(warm):
         graphs.replay()
     graphs.drain()
@@ -897,7 +1007,6 @@ def gpu_arm(args, d: Dist):
     ms_h = sum(e[0].elapsed_time(e[1]) for e in evs) / args.steps
     ms_sc = sum(e[1].elapsed_time(e[2]) for e in evs) / args.steps
     ms_step = d.max(ms_total / args.steps)
-    value = work.groups * d.world / (ms_step * 1e-3)
 
     # ---- per-kernel times of the scale phase, every matrix, every window of the workload
     hbm_peak, peak_kind, peaks = measured_peaks()
@@ -913,7 +1022,7 @@ def gpu_arm(args, d: Dist):
     ms_init = sum(timed(lambda M=M: init_codes(hs, work, M), reps, flush) for M in work.mats)
     ms_h_alone = timed(lambda: [g.replay() for g in graphs.gh[0]], reps)
     sweep = []
-    windows = sorted(set([win] + [(kk, kk) for kk in W.window]))
+    windows = sorted(set([tuple(win)] + [(kk, kk) for kk in W.window]))
     for dn, upw in windows:
         ms_ref = 0.0
         for M in work.mats:
@@ -936,53 +1045,110 @@ def gpu_arm(args, d: Dist):
             hs.hscale_fourover6_codes(M.w, M.sg, M.codes0)
     torch.cuda.synchronize()
     main = [s for s in sweep if tuple(s["window"]) == tuple(win)][0]
+
+    # ---- roofline of the Hessian pass: algorithmic bytes over the launches' event time
+    h_bytes_launch = work.h_bytes / work.h_launches
+    ms_h_launch = ms_h / work.h_launches
+    h_gbs = work.h_bytes / (ms_h * 1e-3) / 1e9
+    traffic = step_traffic(work)
+    hess_roof = {"bound": "hbm", "kernel": "hessian_colsumsq", "achieved": h_gbs,
+                 "peak": hbm_peak, "unit": "GB/s", "frac": h_gbs / hbm_peak,
+                 "peak_kind": f"{peak_kind} HBM copy bandwidth",
+                 "frac_of_8TBs_spec": h_gbs / HBM_SPEC_GBS, "traffic": traffic,
+                 "bytes_per_launch": h_bytes_launch, "ms_per_launch": ms_h_launch}
+    # ---- roofline of the search (its own window, W read from HBM after an L2 flush)
+    if main["bound"] == "alu":
+        ops = 80.0 * main["candidates"] * work.groups
+        search_roof = {"bound": "alu", "kernel": "refine_kernel", "achieved": ops / (main["ms"] * 1e-3) / 1e12,
+                       "peak": fp32_peak / 1e12, "unit": "Tops/s", "frac": main["frac"],
+                       "peak_kind": "SMs x 128 fp32 lanes x max SM clock; 5 lane operations per element "
+                                    "and candidate", "candidates": main["candidates"], "traffic": None,
+                       "ops_per_launch": ops / len(work.mats), "ms_per_launch": main["ms"] / len(work.mats)}
+    else:
+        b = SEARCH_BYTES[work.init] * work.groups
+        search_roof = {"bound": "hbm", "kernel": "refine_kernel", "achieved": b / (main["ms"] * 1e-3) / 1e9,
+                       "peak": hbm_peak, "unit": "GB/s", "frac": b / (main["ms"] * 1e-3) / 1e9 / hbm_peak,
+                       "peak_kind": f"{peak_kind} HBM copy bandwidth", "candidates": main["candidates"],
+                       "traffic": None, "bytes_per_launch": b / len(work.mats),
+                       "ms_per_launch": main["ms"] / len(work.mats)}
+    # the dominant kernel of the step: the Hessian pass, unless the searches take longer
+    # than the Hessian passes do alone (e.g. the 70B MLP block)
+    dominant = search_roof if main["ms"] > ms_h_alone else hess_roof
+    res = {
+        "work": work, "graphs": graphs, "ms_step": ms_step, "ms_eager": ms_eager, "warm": warm,
+        "value": work.groups * d.world / (ms_step * 1e-3), "overlap_ctas": overlap,
+        "roofline": dominant, "roofline_hessian": hess_roof, "roofline_search": search_roof,
+        "phases_ms": {"hessian": ms_h, "after_hessian": ms_sc, "hessian_alone": ms_h_alone,
+                      "weight_only": ms_init, "refine": main["ms"]},
+        "hessian": {"gbs": h_gbs, "tokens_channels_per_s": work.h_bytes / 2 / (ms_h * 1e-3),
+                    "frac_of_measured_hbm": h_gbs / hbm_peak, "frac_of_8TBs": h_gbs / HBM_SPEC_GBS},
+        "search": {"groups_per_s": main["groups_per_s"], "candidates": main["candidates"],
+                   "bound": main["bound"], "roofline_s": main["roofline_ms"] * 1e-3, "frac": main["frac"],
+                   "fp32_peak_ops": fp32_peak, "sm_count": props.multi_processor_count,
+                   "clock_mhz_for_peak": sm_max_mhz},
+        "sweep": sweep, "clocks": clk.summary(), "peaks": peaks,
+    }
+    return res, work
+
+
+def compact_roofline(r: dict) -> dict:
+    """The figures of a roofline object that a one-line summary needs."""
+    return {k: r[k] for k in ("kernel", "bound", "achieved", "peak", "unit", "frac") if k in r}
+
+
+def extra_workload(hs, d: Dist, args, name: str, dev) -> dict:
+    """A second workload measured in the same process (its own timed steps and its search
+    over every window of the workload): per-step time, the step's rate and both rooflines,
+    and the window sweep."""
+    W = wl.WORKLOADS[name]
+    res, work = measure_workload(hs, d, args, W, (W.window[0], W.window[0]), dev, -1, "auto")
+    out = {"workload": W.name, "matrices": [[M.name, M.m, M.n] for M in work.mats],
+           "input_spaces": [[S.name, S.tokens, S.n, S.chunk] for S in work.spaces.values()],
+           "window": [W.window[0], W.window[0]], "groups": work.groups,
+           "ms_per_step": res["ms_step"], "value": res["value"], "unit": UNIT,
+           "schedule": "pipelined" if res["graphs"].pipeline else "sequential",
+           "roofline_hessian": compact_roofline(res["roofline_hessian"]),
+           "roofline_search": compact_roofline(res["roofline_search"]),
+           "phases_ms": res["phases_ms"], "clocks": res["clocks"],
+           "search_sweep": [{k: s[k] for k in ("window", "candidates", "ms", "groups_per_s", "bound", "frac")}
+                            for s in res["sweep"]]}
+    del res, work
+    torch.cuda.synchronize()
+    torch.cuda.empty_cache()
+    return out
+
+
+def gpu_arm(args, d: Dist):
+    import paper_2608_28113_gb300 as hs
+    hs.load()
+    torch.cuda.set_device(d.local)
+    dev = torch.device("cuda", d.local)
+    W = wl.WORKLOADS[args.workload]
+    win = window_of(args, W)
+    res, work = measure_workload(hs, d, args, W, win, dev, args.overlap_ctas, args.pipeline,
+                                 tokens=args.tokens, init=args.init, col_block=args.col_block)
+    graphs, peaks, ms_step = res["graphs"], res["peaks"], res["ms_step"]
     shifts = shift_statistics(work, win)
     out_err = None if args.no_output_error else output_error_eval(hs, work, peaks)
     gptq = None
     if not args.no_gptq:
         try:
             gptq = gptq_eval(hs, work, peaks)
-        except Exception as e:  # e.g. no cuSOLVER on the machine: report, keep the bench line
+        except Exception as e:  # report, keep the bench line
             gptq = {"unavailable": f"{type(e).__name__}: {e}"}
-
-    # ---- roofline of the dominant kernel (the Hessian pass)
-    h_bytes_launch = work.h_bytes / work.h_launches
-    ms_h_launch = ms_h / work.h_launches
-    h_gbs = work.h_bytes / (ms_h * 1e-3) / 1e9
-    first = next(iter(work.spaces.values()))
-    _, c0, c1 = work.pieces[0]
-    t0, t1 = hessian_calls(first, c0, c1)[0]
-    traffic = profiled_traffic(W.name, t1 - t0, c1 - c0) if len(work.spaces) == 1 else None
-
-    # the dominant kernel of the step: the Hessian pass, unless the searches take longer
-    # than the Hessian passes do alone (e.g. the 70B MLP block)
-    roofline = {"bound": "hbm", "kernel": "hessian_colsumsq", "achieved": h_gbs,
-                "peak": hbm_peak, "unit": "GB/s", "frac": h_gbs / hbm_peak,
-                "peak_kind": f"{peak_kind} HBM copy bandwidth",
-                "frac_of_8TBs_spec": h_gbs / HBM_SPEC_GBS, "traffic": traffic,
-                "bytes_per_launch": h_bytes_launch, "ms_per_launch": ms_h_launch}
-    if main["ms"] > ms_h_alone:
-        if main["bound"] == "alu":
-            ops = 80.0 * main["candidates"] * work.groups
-            roofline = {"bound": "alu", "kernel": "refine_kernel", "achieved": ops / (main["ms"] * 1e-3) / 1e12,
-                        "peak": fp32_peak / 1e12, "unit": "Tops/s", "frac": main["frac"],
-                        "peak_kind": "SMs x 128 fp32 lanes x max SM clock; 5 lane operations per element "
-                                     "and candidate", "traffic": None,
-                        "ops_per_launch": ops / len(work.mats), "ms_per_launch": main["ms"] / len(work.mats)}
-        else:
-            b = SEARCH_BYTES[work.init] * work.groups
-            roofline = {"bound": "hbm", "kernel": "refine_kernel", "achieved": b / (main["ms"] * 1e-3) / 1e9,
-                        "peak": hbm_peak, "unit": "GB/s", "frac": b / (main["ms"] * 1e-3) / 1e9 / hbm_peak,
-                        "peak_kind": f"{peak_kind} HBM copy bandwidth", "traffic": None,
-                        "bytes_per_launch": b / len(work.mats), "ms_per_launch": main["ms"] / len(work.mats)}
 
     # ---- end to end through the public API with host buffers
     e2e = None if args.no_e2e else e2e_leg(hs, work, args)
 
     n_layers = W.n_layers
+    roofline = dict(res["roofline"])
+    # the other kernel's roofline in the same object, so a reader of the standard keys sees
+    # both targets of the path
+    other = res["roofline_search"] if roofline["kernel"] == "hessian_colsumsq" else res["roofline_hessian"]
+    roofline["other"] = compact_roofline(other)
     line = {
-        "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": d.world, "steps": args.steps,
-        "warmup": warm, "ms_per_step": ms_step, "higher_is_better": True,
+        "metric": METRIC, "value": res["value"], "unit": UNIT, "n_gpus": d.world, "steps": args.steps,
+        "warmup": res["warm"], "ms_per_step": ms_step, "higher_is_better": True,
         "scaling": "weak", "vs_baseline": None, "dtype": "f32", "input_dtype": "bf16",
         "data": "synthetic",
         "config": {"workload": W.name,
@@ -995,46 +1161,54 @@ def gpu_arm(args, d: Dist):
                          (sum(S.tokens * S.n * 2 for S in work.spaces.values()) / 1e9),
                    "parallelism": f"independent layer per GPU x{d.world}"},
         "roofline": roofline,
-        "phases_ms": {"hessian": ms_h, "after_hessian": ms_sc, "hessian_alone": ms_h_alone,
-                      "weight_only": ms_init, "refine": main["ms"]},
-        "ms_per_step_eager": ms_eager,
+        "roofline_search": res["roofline_search"],
+        "roofline_hessian": res["roofline_hessian"],
+        "seconds_per_layer": ms_step * 1e-3,
+    }
+    if n_layers > 1:
+        line["seconds_per_model"] = ms_step * 1e-3 * n_layers
+        line["seconds_per_model_note"] = f"{n_layers} layers of identical shapes: per-layer step x {n_layers}"
+    line.update({
+        "phases_ms": res["phases_ms"],
+        "ms_per_step_eager": res["ms_eager"],
         "timed_launch": ("CUDA graphs of the step's API calls on three streams: the Hessian pass of "
                          + (f"each {work.col_block}-channel column block of each input space over every token"
                             if work.col_block else "each input space in token chunks")
                          + "; alongside it the weight-only calls (s_g, 4over6 codes); the searches of "
                          + ("each block" if work.col_block else "each input space")
                          + " as soon as its h is complete"
-                         + (f" (at most {args.overlap_ctas} search CTAs per SM while a Hessian pass runs)"
-                            if args.overlap_ctas > 0 and (len(work.pieces) > 1 or graphs.pipeline) else "")
+                         + (f" (at most {res['overlap_ctas']} search CTAs per SM while a Hessian pass runs)"
+                            if res["overlap_ctas"] > 0 and (len(work.pieces) > 1 or graphs.pipeline) else "")
                          + ("; consecutive steps pipelined: each step's last searches run alongside the next "
                             "step's first Hessian pass (h, s_g and initial codes double-buffered); the timed "
                             "region ends when the last step's searches are done" if graphs.pipeline else "")),
-        "hessian": {"gbs": h_gbs, "tokens_channels_per_s": work.h_bytes / 2 / (ms_h * 1e-3),
-                    "frac_of_measured_hbm": h_gbs / hbm_peak, "frac_of_8TBs": h_gbs / HBM_SPEC_GBS},
-        "search": {"groups_per_s": main["groups_per_s"], "candidates": main["candidates"],
-                   "bound": main["bound"], "roofline_s": main["roofline_ms"] * 1e-3, "frac": main["frac"],
-                   "fp32_peak_ops": fp32_peak, "sm_count": props.multi_processor_count,
-                   "clock_mhz_for_peak": sm_max_mhz},
-        "seconds_per_layer": ms_step * 1e-3,
-        "clocks": clk.summary(),
+        "hessian": res["hessian"],
+        "search": res["search"],
+        "clocks": res["clocks"],
         "gpu_launches": args.steps * (work.h_launches + kernels_per_matrix(work) * len(work.mats)),
-    }
-    if len(sweep) > 1:
-        line["search_sweep"] = sweep
+    })
+    if len(res["sweep"]) > 1:
+        line["search_sweep"] = res["sweep"]
     line["shift_statistics"] = shifts
     if out_err:
         line["output_error"] = out_err
     if gptq:
         line["gptq_hscale"] = gptq
-    if n_layers > 1:
-        line["seconds_per_model"] = ms_step * 1e-3 * n_layers
-        line["seconds_per_model_note"] = f"{n_layers} layers of identical shapes: per-layer step x {n_layers}"
     if e2e:
         line["e2e"] = e2e
     if d.rank == 0 and d.world == 1 and not args.no_cpu_baseline:
-        cb = cpu_baseline(W, win, init=args.init)
-        line["cpu_baseline"] = {k2: cb[k2] for k2 in ("value", "unit", "cores", "kind", "sample",
-                                                      "single_thread_value")}
+        if args.cpu_baseline == "full" and work.col_block == 0:
+            line["cpu_baseline"] = cpu_baseline_full(work, win)
+        else:
+            cb = cpu_baseline(W, win, init=args.init)
+            line["cpu_baseline"] = {k2: cb[k2] for k2 in ("value", "unit", "cores", "kind", "sample",
+                                                          "single_thread_value")}
+    # a second workload from the same process (the 70B MLP block with its window sweep)
+    if args.extra_workload != "none" and args.extra_workload != W.name:
+        del graphs, res, work
+        torch.cuda.synchronize()
+        torch.cuda.empty_cache()
+        line[args.extra_workload.replace("-", "_")] = extra_workload(hs, d, args, args.extra_workload, dev)
     if d.rank == 0:
         print(json.dumps(line), flush=True)
 

@@ -7,7 +7,9 @@
  * hot path has two parts, both exposed here:
  *
  *   1. hscale_hessian_diag_accumulate   h_j += sum_t x_tj^2 over a token chunk
- *                                       (Sec. 3.2, Eq. 4: h = diag(X^T X))
+ *                                       (Sec. 3.2, Eq. 4: h = diag(X^T X));
+ *                                       _ex: the same, overlapping the previous kernel
+ *                                       when X is known to be complete
  *   2. hscale_rtn_scales                global scale s_g and the RTN local-scale codes
  *                                       (Sec. 3.3 "Initialization", Eq. 7)
  *      hscale_refine_scales             Algorithm 1: walk the E4M3 ladder around the
@@ -114,12 +116,31 @@ int hscale_selftest_bounded_wait(uint32_t polls, void* stream);
  * Arithmetic: x^2 is exact in fp32; sums are fp32 in a fixed order (per-thread runs of
  * at most 1024 tokens, then fixed-order trees inside the CTA and across a thread-block
  * cluster), so each call adds a relative error of at most about 1100 * 2^-24 to h.
- * Nothing else is touched: the call needs no workspace.  Consecutive calls on one
- * stream overlap (programmatic dependent launch): a call starts reading its chunk
- * while the previous one finishes, and waits for it before it updates h.
+ * Nothing else is touched: the call needs no workspace.  The call's kernel is launched
+ * with programmatic dependent launch; it waits for the kernel before it on the stream
+ * to finish (and for its writes to be visible) before it reads X, so X may be the output
+ * of any earlier work on the stream, including a kernel that lets its dependents start
+ * early.  hscale_hessian_diag_accumulate_ex lets a caller whose X is already complete
+ * skip that wait.
  */
 int hscale_hessian_diag_accumulate(const void* x_bf16, int64_t tokens, int64_t n, int64_t ld_x,
                                    float* h, void* stream);
+
+/*
+ * hscale_hessian_diag_accumulate with flags (the paper has no counterpart: a scheduling
+ * option of the library).  Same arguments, results and status codes, plus:
+ *
+ * flags  0, or HSCALE_HESSIAN_X_READY: the caller guarantees that X is complete, i.e.
+ *        nothing that may still be running on the GPU when this call's kernel starts
+ *        writes X (for instance calibration chunks resident in device memory, streamed
+ *        by successive calls).  The kernel then starts streaming X while the previous
+ *        kernel on the stream finishes, and waits for it only before it reads and
+ *        updates h; successive chunk calls overlap.  Without the guarantee this flag can
+ *        read stale or partly written X.  Other bits return HSCALE_ERR_ARG.
+ */
+#define HSCALE_HESSIAN_X_READY 1u
+int hscale_hessian_diag_accumulate_ex(const void* x_bf16, int64_t tokens, int64_t n, int64_t ld_x,
+                                      float* h, uint32_t flags, void* stream);
 
 /*
  * Global scale and RTN local-scale codes (Sec. 3.3 "Initialization", Eq. 7).
@@ -150,7 +171,9 @@ int hscale_rtn_scales(const void* w_bf16, int64_t m, int64_t n, float* global_sc
  * into the library, which every GPU that loads the library holds until the process exits.
  *
  * - The first call on each device looks up that array's device address (a synchronous
- *   runtime query) and caches it; make that first call before any stream capture.
+ *   runtime query) and caches it with the id of the device's context; make that first
+ *   call before any stream capture.  A call in a new context of the device (after
+ *   cudaDeviceReset) looks the address up again, so it is then a first call too.
  * - Every call on a device shares the array: each call clears the part it uses on its
  *   stream before use, and calls whose work overlaps on the GPU (different streams,
  *   different threads) race with each other.  Serialise them.

@@ -23,7 +23,8 @@ import torch
 __all__ = [
     "HScaleError", "load", "library_path", "hscale_status_string", "hscale_abi_version",
     "hscale_device_error_flags",
-    "hscale_hessian_diag_accumulate", "hscale_rtn_workspace_bytes", "hscale_rtn_scales",
+    "hscale_hessian_diag_accumulate", "hscale_hessian_diag_accumulate_ex", "HSCALE_HESSIAN_X_READY",
+    "hscale_rtn_workspace_bytes", "hscale_rtn_scales",
     "hscale_rtn_scales_noalloc",
     "hscale_refine_scales", "hscale_refine_scales_ex", "hscale_refine_scales_4over6",
     "hscale_refine_scales_strided", "hscale_pack_nvfp4", "hscale_fourover6_codes",
@@ -46,6 +47,7 @@ _SIGNATURES = {
     "hscale_device_error_flags": (ctypes.c_int, [_P]),
     "hscale_selftest_bounded_wait": (ctypes.c_int, [ctypes.c_uint32, _P]),
     "hscale_hessian_diag_accumulate": (ctypes.c_int, [_P, _I64, _I64, _I64, _P, _P]),
+    "hscale_hessian_diag_accumulate_ex": (ctypes.c_int, [_P, _I64, _I64, _I64, _P, ctypes.c_uint32, _P]),
     "hscale_rtn_workspace_bytes": (_SZ, []),
     "hscale_rtn_scales": (ctypes.c_int, [_P, _I64, _I64, _P, _P, _P, _SZ, _P]),
     "hscale_rtn_scales_noalloc": (ctypes.c_int, [_P, _I64, _I64, _P, _P, _P]),
@@ -141,8 +143,18 @@ def _need(t: torch.Tensor, dtype, name: str):
         raise TypeError(f"{name} must be a CUDA tensor of dtype {dtype}")
 
 
+HSCALE_HESSIAN_X_READY = 1
+
+
 def hscale_hessian_diag_accumulate(x: torch.Tensor, h: torch.Tensor, stream=None) -> torch.Tensor:
     """h[j] += sum_t x[t, j]^2 for a bf16 chunk x [tokens, n] (row stride >= n)."""
+    return hscale_hessian_diag_accumulate_ex(x, h, 0, stream)
+
+
+def hscale_hessian_diag_accumulate_ex(x: torch.Tensor, h: torch.Tensor, flags: int = 0,
+                                      stream=None) -> torch.Tensor:
+    """hscale_hessian_diag_accumulate with flags; HSCALE_HESSIAN_X_READY declares that nothing
+    still running writes x, so the kernel may overlap the previous kernel on the stream."""
     _need(x, torch.bfloat16, "x")
     _need(h, torch.float32, "h")
     if x.dim() != 2 or x.stride(1) != 1:
@@ -151,8 +163,9 @@ def hscale_hessian_diag_accumulate(x: torch.Tensor, h: torch.Tensor, stream=None
     if h.numel() != n or not h.is_contiguous():
         raise ValueError("h must be a contiguous float32 vector of length n")
     ld = x.stride(0) if tokens > 1 else n
-    _check("hscale_hessian_diag_accumulate",
-           load().hscale_hessian_diag_accumulate(_ptr(x), tokens, n, ld, _ptr(h), _stream_ptr(stream)))
+    _check("hscale_hessian_diag_accumulate_ex",
+           load().hscale_hessian_diag_accumulate_ex(_ptr(x), tokens, n, ld, _ptr(h), int(flags),
+                                                    _stream_ptr(stream)))
     return h
 
 

@@ -69,7 +69,7 @@ const char* hscale_status_string(int status) {
   }
 }
 
-int hscale_abi_version(void) { return 1; }
+int hscale_abi_version(void) { return 2; }
 
 int hscale_device_error_flags(uint32_t* flags) {
   if (flags == nullptr) return HSCALE_ERR_NULL;
@@ -87,6 +87,12 @@ int hscale_selftest_bounded_wait(uint32_t polls, void* stream) {
 
 int hscale_hessian_diag_accumulate(const void* x_bf16, int64_t tokens, int64_t n, int64_t ld_x,
                                    float* h, void* stream) {
+  return hscale_hessian_diag_accumulate_ex(x_bf16, tokens, n, ld_x, h, 0u, stream);
+}
+
+int hscale_hessian_diag_accumulate_ex(const void* x_bf16, int64_t tokens, int64_t n, int64_t ld_x,
+                                      float* h, uint32_t flags, void* stream) {
+  if ((flags & ~(uint32_t)HSCALE_HESSIAN_X_READY) != 0) return HSCALE_ERR_ARG;
   if (tokens < 0 || n < 0 || ld_x < n) return HSCALE_ERR_SHAPE;
   if (n % 8 != 0) return HSCALE_ERR_SHAPE;
   if (n > (int64_t)65535 * 64) return HSCALE_ERR_SHAPE;  // 64-channel tiles on grid.y
@@ -95,7 +101,8 @@ int hscale_hessian_diag_accumulate(const void* x_bf16, int64_t tokens, int64_t n
   if (ld_x % 8 != 0) return HSCALE_ERR_ALIGN;
   if (!aligned(x_bf16, 16) || !aligned(h, 4)) return HSCALE_ERR_ALIGN;
   if (tokens > INT32_MAX || tokens > INT64_MAX / ld_x) return HSCALE_ERR_SHAPE;
-  return from_cuda(hscale::launch_hessian(x_bf16, tokens, n, ld_x, h, as_stream(stream)));
+  return from_cuda(hscale::launch_hessian(x_bf16, tokens, n, ld_x, h, (flags & HSCALE_HESSIAN_X_READY) != 0,
+                                          as_stream(stream)));
 }
 
 size_t hscale_rtn_workspace_bytes(void) { return 256; }

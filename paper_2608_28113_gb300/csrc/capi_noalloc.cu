@@ -7,6 +7,7 @@
 // the small workspace hscale_rtn_scales needs for its amax word.  This entry point keeps
 // that word in a fixed array of this file that lives in every GPU's memory from the
 // moment the library is loaded there until the process exits.
+#include <cuda.h>
 #include <cuda_runtime.h>
 
 #include <cstdint>
@@ -24,22 +25,63 @@ static __device__ __align__(256) uint8_t g_noalloc_scratch[HSCALE_NOALLOC_SCRATC
 
 constexpr int kMaxDevices = 64;
 
-// Device address of g_noalloc_scratch on the current device, resolved on the first call
-// for that device (with that device current) and cached.
+using CtxGetCurrentFn = CUresult (*)(CUcontext*);
+using CtxGetIdFn = CUresult (*)(CUcontext, unsigned long long*);
+
+// Unique id of the calling thread's current context, or 0 when it has none yet.  A
+// context destroyed and created again (cudaDeviceReset) gets a new id; its module, and
+// with it the array, may then sit at another address.
+cudaError_t current_context_id(unsigned long long* id) {
+  static std::once_flag once;
+  static CtxGetCurrentFn get_current = nullptr;
+  static CtxGetIdFn get_id = nullptr;
+  std::call_once(once, [] {
+    void* p = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    if (cudaGetDriverEntryPointByVersion("cuCtxGetCurrent", &p, 12000, cudaEnableDefault, &q) == cudaSuccess &&
+        q == cudaDriverEntryPointSuccess)
+      get_current = reinterpret_cast<CtxGetCurrentFn>(p);
+    p = nullptr;
+    if (cudaGetDriverEntryPointByVersion("cuCtxGetId", &p, 12000, cudaEnableDefault, &q) == cudaSuccess &&
+        q == cudaDriverEntryPointSuccess)
+      get_id = reinterpret_cast<CtxGetIdFn>(p);
+  });
+  if (get_current == nullptr || get_id == nullptr) return cudaErrorNotSupported;
+  CUcontext ctx = nullptr;
+  if (get_current(&ctx) != CUDA_SUCCESS) return cudaErrorDeviceUninitialized;
+  *id = 0;
+  if (ctx == nullptr) return cudaSuccess;
+  return get_id(ctx, id) == CUDA_SUCCESS ? cudaSuccess : cudaErrorDeviceUninitialized;
+}
+
+// Device address of g_noalloc_scratch in the current device's context, resolved on the
+// first call in that context (with that device current) and cached per device together
+// with the context's id: a call in a new context of the same device (after
+// cudaDeviceReset) resolves it again instead of using a stale address.
 cudaError_t scratch_address(uint32_t** out) {
   static std::mutex mu;
   static void* addr[kMaxDevices] = {nullptr};
+  static unsigned long long ctx_of[kMaxDevices] = {0};
   int dev = 0;
   cudaError_t err = cudaGetDevice(&dev);
   if (err != cudaSuccess) return err;
   if (dev < 0 || dev >= kMaxDevices) return cudaErrorInvalidDevice;
   std::lock_guard<std::mutex> lock(mu);
-  if (addr[dev] == nullptr) {
+  unsigned long long id = 0;
+  err = current_context_id(&id);
+  if (err != cudaSuccess) return err;
+  if (id == 0 || addr[dev] == nullptr || ctx_of[dev] != id) {
+    // the lookup also makes the runtime bind the device's primary context to the thread
+    // when it has none yet, so the context id is read (again) after it
     void* p = nullptr;
     err = cudaGetSymbolAddress(&p, g_noalloc_scratch);
     if (err != cudaSuccess) return err;
     if (p == nullptr) return cudaErrorInvalidSymbol;
+    err = current_context_id(&id);
+    if (err != cudaSuccess) return err;
+    if (id == 0) return cudaErrorDeviceUninitialized;
     addr[dev] = p;
+    ctx_of[dev] = id;
   }
   *out = static_cast<uint32_t*>(addr[dev]);
   return cudaSuccess;

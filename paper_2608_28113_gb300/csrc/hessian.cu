@@ -13,9 +13,13 @@
 //     (1, 2, 4 or 8 CTAs, so a launch holds about one CTA per SM).  The CTAs
 //     of a cluster reduce their partial sums through distributed shared memory: the
 //     kernel needs no global scratch, no atomics and no second launch.
-//   * Launches use programmatic dependent launch: the next chunk's kernel may start
-//     streaming X while this one finishes; it waits (griddepcontrol.wait) only before
-//     it reads and writes h.
+//   * Launches use programmatic dependent launch.  By default a call's kernel waits
+//     (griddepcontrol.wait) for the kernel before it on the stream before it reads X, so
+//     X may come from a kernel that lets its dependents start early; it then lets its
+//     own dependents start.  When the caller declares X complete (nothing still running
+//     writes it), and for the second and later launches of one call (whose predecessor
+//     is this call's own launch), the kernel streams X at once, while the previous
+//     kernel finishes, and waits only before it reads and writes h.
 //   * Rows past the end of the chunk read as zero (TMA out-of-bounds fill), so ragged
 //     chunks and ragged column tiles need no special cases.
 // Determinism and accuracy
@@ -77,7 +81,7 @@ __device__ __forceinline__ void accum_sq8(float (&acc)[8], const uint4& v) {
 template <int CS>
 __global__ void __launch_bounds__(kThreads, 4)
 hessian_colsumsq_kernel(const __grid_constant__ CUtensorMap xmap, int64_t row0, int64_t rows,
-                        int n, float* __restrict__ h, int64_t rows_per_cta) {
+                        int n, float* __restrict__ h, int64_t rows_per_cta, int x_ready) {
   extern __shared__ __align__(1024) uint8_t ring[];
   __shared__ __align__(8) uint64_t full_bar[kStages];
   __shared__ __align__(8) uint64_t empty_bar[kStages];
@@ -106,6 +110,9 @@ hessian_colsumsq_kernel(const __grid_constant__ CUtensorMap xmap, int64_t row0, 
     s_bad = 0;
   }
   __syncthreads();
+  // X may still be being written by the previous kernel on the stream: read it only once
+  // that kernel has finished and its writes are visible
+  if (!x_ready) pdl_wait_primary();
   if (tid == 0) {
     policy = l2_evict_first_policy();
     for (; issued < kStages && issued < nst; ++issued) {
@@ -202,7 +209,7 @@ hessian_colsumsq_kernel(const __grid_constant__ CUtensorMap xmap, int64_t row0, 
 
 // ---------------------------------------------------------------- host side
 template <int CS>
-cudaError_t launch_cs(const CUtensorMap& map, int64_t tokens, int n, float* h, int tiles,
+cudaError_t launch_cs(const CUtensorMap& map, int64_t tokens, int n, float* h, int tiles, bool x_ready,
                       cudaStream_t stream) {
   const cudaError_t attr_status =
       ensure_dynamic_smem(reinterpret_cast<const void*>(hessian_colsumsq_kernel<CS>), (int)kRingBytes);
@@ -226,8 +233,10 @@ cudaError_t launch_cs(const CUtensorMap& map, int64_t tokens, int n, float* h, i
     attr[1].val.programmaticStreamSerializationAllowed = 1;
     cfg.attrs = attr;
     cfg.numAttrs = 2;
+    // a later launch of this call follows this call's own launch, which reads X only
+    const int ready = (x_ready || t0 > 0) ? 1 : 0;
     cudaError_t err = cudaLaunchKernelEx(&cfg, hessian_colsumsq_kernel<CS>, map, t0, t, n, h,
-                                         rows_per_cta);
+                                         rows_per_cta, ready);
     if (err != cudaSuccess) return err;
   }
   return cudaGetLastError();
@@ -235,7 +244,7 @@ cudaError_t launch_cs(const CUtensorMap& map, int64_t tokens, int n, float* h, i
 
 }  // namespace
 
-cudaError_t launch_hessian(const void* x, int64_t tokens, int64_t n, int64_t ld_x, float* h,
+cudaError_t launch_hessian(const void* x, int64_t tokens, int64_t n, int64_t ld_x, float* h, bool x_ready,
                            cudaStream_t stream) {
   DeviceInfo info;
   cudaError_t err = current_device_info(&info);
@@ -264,10 +273,10 @@ cudaError_t launch_hessian(const void* x, int64_t tokens, int64_t n, int64_t ld_
   while (cs < kMaxCluster && (int64_t)tiles * cs * 2 <= target && (int64_t)cs * 2 * kStageRows * 4 <= tokens)
     cs *= 2;
   switch (cs) {
-    case 1: return launch_cs<1>(map, tokens, (int)n, h, tiles, stream);
-    case 2: return launch_cs<2>(map, tokens, (int)n, h, tiles, stream);
-    case 4: return launch_cs<4>(map, tokens, (int)n, h, tiles, stream);
-    default: return launch_cs<8>(map, tokens, (int)n, h, tiles, stream);
+    case 1: return launch_cs<1>(map, tokens, (int)n, h, tiles, x_ready, stream);
+    case 2: return launch_cs<2>(map, tokens, (int)n, h, tiles, x_ready, stream);
+    case 4: return launch_cs<4>(map, tokens, (int)n, h, tiles, x_ready, stream);
+    default: return launch_cs<8>(map, tokens, (int)n, h, tiles, x_ready, stream);
   }
 }
 

@@ -15,8 +15,10 @@ struct DeviceInfo {
 // SM count of the current device (cached per device).
 cudaError_t current_device_info(DeviceInfo* out);
 
-// h[j] += sum_t x[t, j]^2.  Arguments already validated; tokens, n > 0.
-cudaError_t launch_hessian(const void* x, int64_t tokens, int64_t n, int64_t ld_x, float* h,
+// h[j] += sum_t x[t, j]^2.  Arguments already validated; tokens, n > 0.  x_ready: nothing
+// that may still be running writes X, so the kernel may read it before the previous
+// kernel on the stream has finished.
+cudaError_t launch_hessian(const void* x, int64_t tokens, int64_t n, int64_t ld_x, float* h, bool x_ready,
                            cudaStream_t stream);
 
 // amax over W into *amax_bits (16-bit |bf16| pattern, zero-extended); *amax_bits must be 0.

@@ -41,7 +41,7 @@ def test_header_declares_the_boundary():
 def test_library_exports_every_declared_symbol(lib):
     for name in declared_functions():
         assert hasattr(lib, name), name
-    assert hs.hscale_abi_version() == 1
+    assert hs.hscale_abi_version() == 2
     assert hs.library_path().exists()
 
 
@@ -97,6 +97,12 @@ def test_hessian_argument_errors(lib):
     assert f(MIS, 4, 64, 64, FAKE, None) == ERR_ALIGN
     assert f(FAKE, 0, 64, 64, FAKE, None) == OK               # empty chunk: no-op
     assert f(None, 0, 0, 0, None, None) == OK
+    fx = lib.hscale_hessian_diag_accumulate_ex
+    assert fx(FAKE, 4, 64, 64, FAKE, 2, None) == ERR_ARG     # unknown flag bit
+    assert fx(FAKE, 4, 64, 64, FAKE, 0xFFFFFFFF, None) == ERR_ARG
+    assert fx(None, 4, 64, 64, FAKE, hs.HSCALE_HESSIAN_X_READY, None) == ERR_NULL
+    assert fx(FAKE, 4, 60, 64, FAKE, hs.HSCALE_HESSIAN_X_READY, None) == ERR_SHAPE
+    assert fx(FAKE, 0, 64, 64, FAKE, hs.HSCALE_HESSIAN_X_READY, None) == OK
 
 
 def test_rtn_argument_errors(lib):

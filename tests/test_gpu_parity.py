@@ -162,6 +162,32 @@ def test_hessian_closed_forms_and_empty_chunk():
     assert torch.all(h == 12.0)
 
 
+def test_hessian_x_ready_flag_gives_the_same_bits():
+    """The chunk stream with and without HSCALE_HESSIAN_X_READY (early X reads overlapping the
+    previous chunk's kernel) gives the same h bit for bit, and a chunk written by the kernel
+    just before the call on the same stream is read after that kernel is done."""
+    g = torch.Generator().manual_seed(11)
+    x = (torch.randn(8 * 4096, 1024, generator=g) * 2).to(torch.bfloat16).to(dev())
+    hs_default = torch.zeros(1024, device=dev())
+    hs_ready = torch.zeros(1024, device=dev())
+    for c in range(8):
+        hs.hscale_hessian_diag_accumulate(x[c * 4096:(c + 1) * 4096], hs_default)
+    for c in range(8):
+        hs.hscale_hessian_diag_accumulate_ex(x[c * 4096:(c + 1) * 4096], hs_ready, hs.HSCALE_HESSIAN_X_READY)
+    torch.cuda.synchronize()
+    assert torch.equal(hs_default, hs_ready)
+    # producer kernel immediately before the call on the same stream
+    y = torch.empty_like(x)
+    h1 = torch.zeros(1024, device=dev())
+    for c in range(8):
+        blk = y[c * 4096:(c + 1) * 4096]
+        torch.mul(x[c * 4096:(c + 1) * 4096], 1.0, out=blk)
+        hs.hscale_hessian_diag_accumulate(blk, h1)
+    torch.cuda.synchronize()
+    assert torch.equal(h1, hs_default)
+    assert hs.hscale_device_error_flags() == 0
+
+
 def test_hessian_is_deterministic():
     g = torch.Generator().manual_seed(5)
     x = (torch.randn(20000, 4096, generator=g) * 3).to(torch.bfloat16).to(dev())

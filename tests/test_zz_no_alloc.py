@@ -44,3 +44,25 @@ def test_noalloc_matches_workspace_entry_point_on_two_calls():
         assert sg.cpu().numpy().tobytes() == ref_sg.cpu().numpy().tobytes()
         assert np.array_equal(codes.cpu().numpy(), ref_codes.cpu().numpy())
     assert hs.hscale_device_error_flags() == 0
+
+
+def test_noalloc_allocates_no_device_memory():
+    """After a first call (which resolves the scratch address and loads the kernels), further
+    calls change neither torch's allocator nor the device's free memory."""
+    if not torch.cuda.is_available():
+        pytest.skip("no CUDA device")
+    hs.load()
+    dev = torch.device("cuda", 0)
+    w = wl.weight(512, 1024, 0.02, seed=23).to(dev)
+    sg = torch.empty(1, dtype=torch.float32, device=dev)
+    codes = torch.empty(512, 1024 // 16, dtype=torch.uint8, device=dev)
+    hs.hscale_rtn_scales_noalloc(w, sg, codes)
+    torch.cuda.synchronize()
+    allocated = torch.cuda.memory_allocated(dev)
+    free_before, _ = torch.cuda.mem_get_info(dev)
+    for _ in range(3):
+        hs.hscale_rtn_scales_noalloc(w, sg, codes)
+    torch.cuda.synchronize()
+    free_after, _ = torch.cuda.mem_get_info(dev)
+    assert torch.cuda.memory_allocated(dev) == allocated
+    assert free_after == free_before
