@@ -112,9 +112,11 @@ __device__ __forceinline__ uint32_t rtn_code(float amax_k, float sgk, float inv6
   return anchored_code(amax_k, sgk, inv6_raw, 3.0f);
 }
 
-// 2^-120 / (c sgk): the factor anchored_code multiplies amax_k by (a normal number).
+// ~2^-120 / (c sgk): the factor anchored_code multiplies amax_k by (a normal number).  Only
+// an estimate is needed (anchored_code checks both neighbouring midpoints exactly), so it is
+// the correctly rounded reciprocal of the rounded product (c sgk) 2^120, within 2^-23.
 __device__ __forceinline__ float anchor_inv_raw(float sgk, float c) {
-  return __fdiv_rn(0x1p-120f, __fmul_rn(c, sgk));
+  return __frcp_rn(__fmul_rn(__fmul_rn(c, sgk), 0x1p120f));
 }
 __device__ __forceinline__ float rtn_inv6_raw(float sgk) { return anchor_inv_raw(sgk, 6.0f); }
 
@@ -149,6 +151,19 @@ __device__ __forceinline__ uint32_t e2m1_exact_code(float y_raw, float a_k, floa
   else if (t < 0.0f) k = klo;
   else k = (klo & 1u) ? klo + 1 : klo;  // tie: even code
   return min(k, 7u);
+}
+
+// Exact round-to-nearest-even magnitude code of a_k / (l sgk) (a_k >= 0) when the quotient
+// is known to lie between the grid points of codes klo and klo + 1 (klo < 7): the midpoint
+// is compared exactly with one FMA; a tie goes to the even code.
+__device__ __forceinline__ uint32_t e2m1_code_between(float a_k, uint32_t klo, float l, float sgk) {
+  const float vlo = e2m1_from_raw(klo << 22);
+  const float vhi = e2m1_from_raw((klo + 1) << 22);
+  const float mid = __fmul_rn(0.5f, __fadd_rn(vlo, vhi));
+  const float t = __fmaf_rn(-__fmul_rn(mid, l), sgk, a_k);
+  if (t > 0.0f) return klo + 1;
+  if (t < 0.0f) return klo;
+  return (klo & 1u) ? klo + 1 : klo;
 }
 
 // Exact magnitude code of a_k / (l sgk): fast path plus the exact fix when flagged.

@@ -42,6 +42,7 @@
 
 #include "hscale_device.cuh"
 #include "hscale_internal.h"
+#include "tma.cuh"
 
 namespace hscale {
 namespace {
@@ -114,19 +115,21 @@ __global__ void __launch_bounds__(256) rtn_codes_kernel(const uint4* __restrict_
 // saturation are symmetric, and only squares of residuals enter), so the search pays
 // nothing for the sign, and the pack converts the signed quotients directly.
 struct Group {
-  uint32_t wb[8];  // raw bf16 pairs (element 2i in the low half of wb[i])
   float2 a[8];     // w * 2^-K, elements (2i, 2i+1)
 };
 
-// The group whose 16 bf16 values start at wg (16-byte aligned).
-__device__ __forceinline__ void load_group_at(const uint4* wg, float pw, Group& G) {
-  const uint4 p = ld_stream_v4(wg);
-  const uint4 q = ld_stream_v4(wg + 1);
-  G.wb[0] = p.x; G.wb[1] = p.y; G.wb[2] = p.z; G.wb[3] = p.w;
-  G.wb[4] = q.x; G.wb[5] = q.y; G.wb[6] = q.z; G.wb[7] = q.w;
+// The group's 16 bf16 values, given as two 16-byte words (element 2i in the low half of
+// word i), unpacked and scaled.
+__device__ __forceinline__ void unpack_group(const uint4& p, const uint4& q, float pw, Group& G) {
+  const uint32_t wb[8] = {p.x, p.y, p.z, p.w, q.x, q.y, q.z, q.w};
 #pragma unroll
   for (int i = 0; i < 8; ++i)
-    G.a[i] = __fmul2_rn(make_float2(bf16_lo(G.wb[i]), bf16_hi(G.wb[i])), make_float2(pw, pw));
+    G.a[i] = __fmul2_rn(make_float2(bf16_lo(wb[i]), bf16_hi(wb[i])), make_float2(pw, pw));
+}
+
+// The group whose 16 bf16 values start at wg (16-byte aligned).
+__device__ __forceinline__ void load_group_at(const uint4* wg, float pw, Group& G) {
+  unpack_group(ld_stream_v4(wg), ld_stream_v4(wg + 1), pw, G);
 }
 
 __device__ __forceinline__ void load_group(const uint4* w, int64_t g, float pw, Group& G) {
@@ -267,66 +270,92 @@ __device__ __forceinline__ uint32_t cvt_e2m1x2(float hi, float lo) {
 }
 
 // The anchored code of Eq. 7 (anchor c = 2 * half_c; RTN is c = 6), decided by the hardware
-// E4M3 conversion of the fast quotient r = amax_k * inv_c (inv_c ~ 1 / (c * sgk), within a
-// relative 2^-22 of the exact quotient, so r is within 2^-21 of it).  RNE of r equals RNE
-// of the exact quotient unless the quotient lies near an E4M3 midpoint: in the normal
-// range (r >= 2^-6) the midpoints are the fp32 patterns whose low 20 bits are 0x80000, and
-// r within 16 ulps of one is flagged.  Flagged quotients and the subnormal range take the
-// exact midpoint tests of anchored_code().  Saturation at 448 (code 126) is the
-// conversion's own; code 0 is clamped to 1.
-__device__ __forceinline__ uint32_t anchored_code_fast(float amax_k, float sgk, float inv_c, float inv_raw,
-                                                       float half_c) {
-  const float r = __fmul_rn(amax_k, inv_c);
-  const bool near = ((__float_as_uint(r) - 0x7FFF0u) & 0xFFFFFu) <= 0x20u;
-  if (near || !(r >= 0x1p-6f)) return anchored_code(amax_k, sgk, inv_raw, half_c);
-  uint32_t c;
+// E4M3 conversion (round-to-nearest-even, saturating at 448) of two bracketing quotients
+// r_lo = amax_k * inv_lo and r_hi = amax_k * inv_hi, with inv_lo and inv_hi the reciprocal
+// 1 / (c sgk) (relative error <= 2^-23) scaled by 1 -+ 2^-20: r_lo lies below the exact
+// quotient amax_g / (c s_g) and r_hi above it, so where the two conversions (one
+// instruction for the pair) agree, that code is the exact rounding; otherwise an E4M3
+// midpoint lies between them and the exact midpoint tests of anchored_code() decide.
+// Quotients below the fp32 normal range convert to code 0 under both.  Code 0 is clamped
+// to 1.
+__device__ __forceinline__ uint32_t anchored_code_fast(float amax_k, float sgk, float inv_lo, float inv_hi,
+                                                       float inv_raw, float half_c) {
+  const float rl = __fmul_rn(amax_k, inv_lo), rh = __fmul_rn(amax_k, inv_hi);
+  uint32_t p;
   asm("{\n\t.reg .b16 t;\n\tcvt.rn.satfinite.e4m3x2.f32 t, %1, %2;\n\tcvt.u32.u16 %0, t;\n\t}"
-      : "=r"(c)
-      : "f"(0.0f), "f"(r));
-  c &= 0xFFu;
+      : "=r"(p)
+      : "f"(rh), "f"(rl));
+  uint32_t c = p & 0xFFu;
+  if (c != (p >> 8)) c = anchored_code(amax_k, sgk, inv_raw, half_c);
   return c < 1u ? 1u : c;
 }
 
-// Exact final re-quantization of one group under code c (inv_raw = 2^-126 / s'): 8 bytes of
-// packed nibbles.  The raw-domain quotients y_raw = w * 2^-126 / s' (signed) are rescaled
-// exactly to real units and converted by the hardware E2M1 conversion (round-to-nearest-
-// even, sign kept).  That equals the exact rounding of |w| / s unless y_raw lies within 16
-// ulps of a midpoint.  The main pass only notes whether any element does; then such
-// elements are found and redone one by one with the exact midpoint test, reading the
-// weight back from `wg` (the group's 16 bf16 values in global memory).
-__device__ __forceinline__ uint2 quantize_pack(const Group& G, uint32_t c, float inv_raw, float sgk,
-                                               float pw, const uint16_t* wg) {
-  const float2 ir2 = make_float2(inv_raw, inv_raw);
-  const float2 up2 = make_float2(0x1p126f, 0x1p126f);
-  uint32_t word[2] = {0u, 0u};
-  bool any = false;
+// Bracketing factors of a reciprocal (see quantize_pack): 1 -+ 2^-20.
+constexpr float kBracketLo = 1.0f - 0x1p-20f;
+constexpr float kBracketHi = 1.0f + 0x1p-20f;
+
+// Exact final re-quantization of one group under code c: 8 bytes of packed nibbles.
+// inv ~ 1 / s' is the correctly rounded reciprocal of s' = l(c) sgk (the candidate
+// table's), so y = a * inv is within a relative 2^-23 (+ 2^-48) of the exact quotient
+// y* = a / s'.  The quotients are formed under two bracketing reciprocals,
+// inv (1 - 2^-20) and inv (1 + 2^-20), each rounded once more: the one is below |y*| and
+// the other above it by at least 2^-21 |y*| - 4 * 2^-24 |y*| > 0.  Round-to-nearest-even
+// is monotone, so where the hardware conversions (RNE, saturation, sign kept also for a
+// zero) of the two agree, that is the exact rounding of y*; the two differ only where a
+// midpoint of the grid lies between them (an exact tie among them), and those elements are
+// decided exactly with the one-FMA midpoint test of e2m1_exact_code, reading the weight back
+// from `wg` (the group's 16 bf16 values): the lower conversion gives the lower of the two
+// grid points.  A quotient below the normal range is far below the first midpoint 0.25 and
+// converts to a signed zero under both reciprocals.
+// Four element pairs (real-unit quotients) converted to E2M1 nibble pairs and packed into
+// one 32-bit word, pair i in byte i.
+__device__ __forceinline__ uint32_t cvt_e2m1x8(float2 y0, float2 y1, float2 y2, float2 y3) {
+  uint32_t r;
+  asm("{\n\t.reg .b8 b0, b1, b2, b3;\n\t"
+      "cvt.rn.satfinite.e2m1x2.f32 b0, %2, %1;\n\t"
+      "cvt.rn.satfinite.e2m1x2.f32 b1, %4, %3;\n\t"
+      "cvt.rn.satfinite.e2m1x2.f32 b2, %6, %5;\n\t"
+      "cvt.rn.satfinite.e2m1x2.f32 b3, %8, %7;\n\t"
+      "mov.b32 %0, {b0, b1, b2, b3};\n\t}"
+      : "=r"(r)
+      : "f"(y0.x), "f"(y0.y), "f"(y1.x), "f"(y1.y), "f"(y2.x), "f"(y2.y), "f"(y3.x), "f"(y3.y));
+  return r;
+}
+
+// Bit 4j of the result is set iff nibble j of x is non-zero.
+__device__ __forceinline__ uint32_t nonzero_nibbles(uint32_t x) {
+  x |= x >> 1;
+  x |= x >> 2;
+  return x & 0x11111111u;
+}
+
+__device__ __forceinline__ uint2 quantize_pack(const Group& G, uint32_t c, float inv, float sgk, float pw,
+                                               const uint16_t* wg) {
+  const float ilo = __fmul_rn(inv, kBracketLo), ihi = __fmul_rn(inv, kBracketHi);
+  const float2 il2 = make_float2(ilo, ilo), ih2 = make_float2(ihi, ihi);
+  uint32_t lo[2], hi[2];
 #pragma unroll
-  for (int i = 0; i < 8; ++i) {
-    const float2 yr = __fmul2_rn(G.a[i], ir2);
-    any |= e2m1_uncertain(yr.x) | e2m1_uncertain(yr.y);
-    const float2 yv = __fmul2_rn(yr, up2);
-    word[i >> 2] |= cvt_e2m1x2(yv.y, yv.x) << (8 * (i & 3));
+  for (int wd = 0; wd < 2; ++wd) {
+    const float2* a = G.a + 4 * wd;
+    lo[wd] = cvt_e2m1x8(__fmul2_rn(a[0], il2), __fmul2_rn(a[1], il2), __fmul2_rn(a[2], il2), __fmul2_rn(a[3], il2));
+    hi[wd] = cvt_e2m1x8(__fmul2_rn(a[0], ih2), __fmul2_rn(a[1], ih2), __fmul2_rn(a[2], ih2), __fmul2_rn(a[3], ih2));
   }
-  if (any) {
-    uint32_t flagged = 0u;
-#pragma unroll
-    for (int i = 0; i < 8; ++i) {
-      const float2 yr = __fmul2_rn(G.a[i], ir2);
-      flagged |= (uint32_t)e2m1_uncertain(yr.x) << (2 * i);
-      flagged |= (uint32_t)e2m1_uncertain(yr.y) << (2 * i + 1);
-    }
+  if ((lo[0] ^ hi[0]) | (lo[1] ^ hi[1])) {
     const float l = e4m3_mag(c);
-    do {
-      const int j = __ffs(flagged) - 1;
-      flagged &= flagged - 1;
-      const uint32_t b = wg[j];
-      const float a = __fmul_rn(__uint_as_float((b & 0x7FFFu) << 16), pw);
-      const uint32_t k = e2m1_exact_code(__fmul_rn(a, inv_raw), a, l, sgk);
-      const int sh = 4 * (j & 7);
-      word[j >> 3] = (word[j >> 3] & ~(0xFu << sh)) | ((((b >> 15) << 3) | k) << sh);
-    } while (flagged);
+#pragma unroll
+    for (int wd = 0; wd < 2; ++wd) {
+      uint32_t flagged = nonzero_nibbles(lo[wd] ^ hi[wd]);
+      while (flagged) {
+        const int sh = __ffs(flagged) - 1;  // 4 * (element index within the word)
+        flagged &= flagged - 1;
+        const uint32_t nib = (lo[wd] >> sh) & 0xFu;  // the lower magnitude code, with the sign
+        const float a = __fmul_rn(__uint_as_float(((uint32_t)wg[8 * wd + (sh >> 2)] & 0x7FFFu) << 16), pw);
+        const uint32_t k = e2m1_code_between(a, nib & 7u, l, sgk);
+        lo[wd] = (lo[wd] & ~(0xFu << sh)) | (((nib & 8u) | k) << sh);
+      }
+    }
   }
-  return make_uint2(word[0], word[1]);
+  return make_uint2(lo[0], lo[1]);
 }
 
 // ---------------------------------------------------------------- 4over6 scores (Algorithm 2)
@@ -396,9 +425,9 @@ __device__ __noinline__ uint32_t fourover6_exact_pick(const uint4* wg, float pw,
 // the code fourover6_codes_kernel writes.
 __device__ __forceinline__ int fourover6_init_code(const Group& G, const uint4* wg, const float4* tab,
                                                    float amax_k, float sgk, float pw, float inv4, float inv6,
-                                                   float inv4r, float inv6r) {
-  const uint32_t c4 = anchored_code_fast(amax_k, sgk, inv4r, inv4, 2.0f);
-  const uint32_t c6 = anchored_code_fast(amax_k, sgk, inv6r, inv6, 3.0f);
+                                                   const float2& b4, const float2& b6) {
+  const uint32_t c4 = anchored_code_fast(amax_k, sgk, b4.x, b4.y, inv4, 2.0f);
+  const uint32_t c6 = anchored_code_fast(amax_k, sgk, b6.x, b6.y, inv6, 3.0f);
   if (c4 == c6) return (int)c4;
   const float e4 = fast_mse(G, tab[c4]);
   const float e6 = fast_mse(G, tab[c6]);
@@ -408,10 +437,27 @@ __device__ __forceinline__ int fourover6_init_code(const Group& G, const uint4* 
 }
 
 // ---------------------------------------------------------------- refine (Algorithm 1)
-// Work unit: one warp, 32 consecutive groups of one row (a "row chunk"); warps stride
-// over (row, chunk) units so the h slice of a lane is reloaded only when its chunk
-// changes.  7 resident CTAs of 4 warps per SM (72 registers); the rarely taken
-// warp-cooperative rescoring is a separate call so it does not raise that.
+// 16-byte asynchronous copy global -> shared (L1 bypassed), and the wait for all but the
+// latest `n` groups of this thread's copies.
+__device__ __forceinline__ void cp_async16(void* smem, const void* gmem) {
+  asm volatile("cp.async.cg.shared.global [%0], [%1], 16;" ::"r"(smem_addr(smem)), "l"(gmem) : "memory");
+}
+__device__ __forceinline__ void cp_async_commit() { asm volatile("cp.async.commit_group;" ::: "memory"); }
+__device__ __forceinline__ void cp_async_wait_1() { asm volatile("cp.async.wait_group 1;" ::: "memory"); }
+
+// Reciprocal 1 / (c sgk) scaled by the bracketing factors (lo, hi) of anchored_code_fast.
+__device__ __forceinline__ float2 anchor_brackets(float sgk, float c) {
+  const float r = __frcp_rn(__fmul_rn(c, sgk));
+  return make_float2(__fmul_rn(r, kBracketLo), __fmul_rn(r, kBracketHi));
+}
+
+// Work unit: one warp, 32 consecutive groups of one row (a "row chunk", 1 KB of W); warps
+// stride over (row, chunk) units so the h slice of a lane is reloaded only when its chunk
+// changes.  Each lane copies its group of the warp's next unit into a per-warp staging
+// buffer in shared memory (cp.async, two buffers) while the current unit is scored, so the
+// scoring never waits for W; a lane reads back only what it copied itself.  7 resident
+// CTAs of 4 warps per SM; the rarely taken warp-cooperative rescoring is a separate call so
+// it does not raise the register count.
 // kFourOverSix: the initial codes are Algorithm 2's, decided in place (init_codes unused).
 // W, the codes and the nibbles are 2-D views: row r starts at element r * ld_w of w, byte
 // r * ld_i of the initial codes, byte r * ld_c of the codes and 8-byte word r * ld_p of the
@@ -422,18 +468,22 @@ refine_kernel(const uint4* __restrict__ w, int64_t ld_w, const float* __restrict
               const float* __restrict__ global_scale, const uint8_t* init_codes, int64_t ld_i,
               int down, int up, uint8_t* codes_out, int64_t ld_c, uint2* __restrict__ packed_out, int64_t ld_p) {
   const int lane = threadIdx.x & 31;
+  const int warp = threadIdx.x >> 5;
   const int64_t warp_global = ((int64_t)blockIdx.x * blockDim.x + threadIdx.x) >> 5;
   const int64_t warps_total = ((int64_t)gridDim.x * blockDim.x) >> 5;
   const int chunks = (ng + 31) / 32;
   const int64_t units = m * chunks;
 
   __shared__ float4 tab[128];
+  // per warp, two buffers of one unit: the first 16 bytes of every lane's group, then the
+  // second 16 bytes (consecutive lanes, consecutive 16-byte words: conflict-free)
+  __shared__ __align__(16) uint4 stage[kWarpsPerRefineBlock][2][64];
   const ScaleDomain d = make_scale_domain(*global_scale);
   const float inv6 = rtn_inv6_raw(d.sgk);
   const float inv4 = kFourOverSix ? anchor_inv_raw(d.sgk, 4.0f) : 0.0f;
-  const float inv6r = __frcp_rn(__fmul_rn(6.0f, d.sgk)), inv4r = __frcp_rn(__fmul_rn(4.0f, d.sgk));
+  const float2 b6 = anchor_brackets(d.sgk, 6.0f);
+  const float2 b4 = kFourOverSix ? anchor_brackets(d.sgk, 4.0f) : make_float2(0.f, 0.f);
   for (int c = threadIdx.x; c < 128; c += blockDim.x) tab[c] = candidate_constants((uint32_t)c, d.sgk);
-  __syncthreads();
 
   int cur_chunk = -1;
   float2 hv2[8];
@@ -441,25 +491,38 @@ refine_kernel(const uint4* __restrict__ w, int64_t ld_w, const float* __restrict
   for (int j = 0; j < 8; ++j) hv2[j] = make_float2(1.0f, 1.0f);
   float hsum = 16.0f;  // sum of the lane's 16 h values
 
-  const bool linear_units = ld_w == (int64_t)ng * 16 && ng % 32 == 0;
   // (row, chunk) of unit u, advanced by warps_total units per step without a division
   const int row_step = (int)(warps_total / chunks);
   const int chunk_step = (int)(warps_total - (int64_t)row_step * chunks);
   int64_t row = warp_global / chunks;
   int chunk = (int)(warp_global - row * chunks);
-  for (int64_t u = warp_global; u < units; u += warps_total, row += row_step, chunk += chunk_step) {
-    if (chunk >= chunks) {
-      chunk -= chunks;
-      ++row;
+
+  // the copy of unit (r, ch), if it exists, into buffer `buf`; always one commit group
+  auto stage_unit = [&](int64_t uu, int64_t r, int ch, int buf) {
+    const int gc = ch * 32 + lane;
+    if (uu < units && gc < ng) {
+      const uint4* src = w + (r * ld_w + (int64_t)gc * 16) / 8;
+      cp_async16(&stage[warp][buf][lane], src);
+      cp_async16(&stage[warp][buf][32 + lane], src + 1);
     }
+    cp_async_commit();
+  };
+  stage_unit(warp_global, row, chunk, 0);
+  __syncthreads();  // the candidate table
+
+  int buf = 0;
+  for (int64_t u = warp_global; u < units; u += warps_total, buf ^= 1) {
     const int gcol = chunk * 32 + lane;
     const bool active = gcol < ng;
     const int64_t wofs = row * ld_w + (int64_t)gcol * 16;  // first element of the group
-    // the warp's next unit (1 KB of W) requested into L2 while this one is scored, so a W
-    // that is not in L2 yet is not waited for unit by unit.  With contiguous rows of whole
-    // units, unit u holds the elements [512 u, 512 u + 512); one lane per 128 bytes.
-    if (linear_units && (lane & 3) == 0 && u + warps_total < units)
-      asm volatile("prefetch.global.L2 [%0];" ::"l"(w + ((u + warps_total) * 512 + lane * 16) / 8));
+    // (row, chunk) of the warp's next unit, whose copy starts now
+    int64_t nrow = row + row_step;
+    int nchunk = chunk + chunk_step;
+    if (nchunk >= chunks) {
+      nchunk -= chunks;
+      ++nrow;
+    }
+    stage_unit(u + warps_total, nrow, nchunk, buf ^ 1);
 
     if (chunk != cur_chunk) {
       cur_chunk = chunk;
@@ -480,17 +543,18 @@ refine_kernel(const uint4* __restrict__ w, int64_t ld_w, const float* __restrict
     Group G;
     int c0 = 1, lo = 1, hi = 1;
     float amax_k = 0.0f;
+    cp_async_wait_1();  // this lane's copy of the current unit has landed
     if (active) {
-      load_group_at(w + wofs / 8, d.pw, G);
-      const uint32_t amax = group_abs_max_bits(make_uint4(G.wb[0], G.wb[1], G.wb[2], G.wb[3]),
-                                               make_uint4(G.wb[4], G.wb[5], G.wb[6], G.wb[7]));
-      amax_k = __fmul_rn(__uint_as_float(amax << 16), d.pw);
+      const uint4 p = stage[warp][buf][lane];
+      const uint4 q = stage[warp][buf][32 + lane];
+      amax_k = __fmul_rn(__uint_as_float(group_abs_max_bits(p, q) << 16), d.pw);
+      unpack_group(p, q, d.pw, G);
       if (!kFourOverSix && init_codes != nullptr) {
         c0 = init_codes[row * ld_i + gcol] & 0x7F;
         c0 = c0 < 1 ? 1 : (c0 > (int)kE4M3MaxCode ? (int)kE4M3MaxCode : c0);
       } else {
-        c0 = kFourOverSix ? fourover6_init_code(G, w + wofs / 8, tab, amax_k, d.sgk, d.pw, inv4, inv6, inv4r, inv6r)
-                          : (int)anchored_code_fast(amax_k, d.sgk, inv6r, inv6, 3.0f);
+        c0 = kFourOverSix ? fourover6_init_code(G, w + wofs / 8, tab, amax_k, d.sgk, d.pw, inv4, inv6, b4, b6)
+                          : (int)anchored_code_fast(amax_k, d.sgk, b6.x, b6.y, inv6, 3.0f);
       }
       lo = max(1, c0 - down);
       hi = min((int)kE4M3MaxCode, c0 + up);
@@ -522,9 +586,129 @@ refine_kernel(const uint4* __restrict__ w, int64_t ld_w, const float* __restrict
     if (active) {
       codes_out[row * ld_c + gcol] = (uint8_t)best;
       if (packed_out != nullptr)
-        packed_out[row * ld_p + gcol] = quantize_pack(G, (uint32_t)best, __fmul_rn(tab[best].z, 0x1p-126f), d.sgk,
-                                                      d.pw, reinterpret_cast<const uint16_t*>(w) + wofs);
+        packed_out[row * ld_p + gcol] = quantize_pack(G, (uint32_t)best, tab[best].z, d.sgk, d.pw,
+                                                      reinterpret_cast<const uint16_t*>(w) + wofs);
     }
+    row = nrow;
+    chunk = nchunk;
+  }
+}
+
+// The search over a contiguous W [m, n] with n a multiple of 512 (every unit a full row
+// chunk) and contiguous outputs: the same work as refine_kernel per group, with the walk
+// reduced to pointer increments.  Unit u is groups [32 u, 32 u + 32), i.e. the 1 KB of W at
+// uint4 offset 64 u, code bytes [32 u, 32 u + 32) and nibble words [32 u, 32 u + 32); every
+// lane of every unit is active.
+template <bool kFourOverSix>
+__global__ void __launch_bounds__(kRefineThreads, 7)
+refine_linear_kernel(const uint4* __restrict__ w, const float* __restrict__ h, int64_t units, int chunks,
+                     const float* __restrict__ global_scale, const uint8_t* init_codes, int down, int up,
+                     uint8_t* codes_out, uint2* __restrict__ packed_out) {
+  const int lane = threadIdx.x & 31;
+  const int warp = threadIdx.x >> 5;
+  const int64_t warp_global = ((int64_t)blockIdx.x * blockDim.x + threadIdx.x) >> 5;
+  const int64_t warps_total = ((int64_t)gridDim.x * blockDim.x) >> 5;
+
+  __shared__ float4 tab[128];
+  __shared__ __align__(16) uint4 stage[kWarpsPerRefineBlock][2][64];
+  const ScaleDomain d = make_scale_domain(*global_scale);
+  const float inv6 = rtn_inv6_raw(d.sgk);
+  const float inv4 = kFourOverSix ? anchor_inv_raw(d.sgk, 4.0f) : 0.0f;
+  const float2 b6 = anchor_brackets(d.sgk, 6.0f);
+  const float2 b4 = kFourOverSix ? anchor_brackets(d.sgk, 4.0f) : make_float2(0.f, 0.f);
+  for (int c = threadIdx.x; c < 128; c += blockDim.x) tab[c] = candidate_constants((uint32_t)c, d.sgk);
+
+  // this lane's group of unit u: uint4 words 64 u + 2 lane and the one after
+  const int64_t wstep = warps_total * 64;
+  const uint4* wp = w + warp_global * 64 + 2 * lane;
+  const int64_t ostep = warps_total * 32;
+  int64_t go = warp_global * 32 + lane;  // this lane's group index
+  // the grid holds at most 2^31 warps, so 32-bit remainders suffice
+  int chunk = (int)((uint32_t)warp_global % (uint32_t)chunks);
+  const int chunk_step = (int)((uint32_t)warps_total % (uint32_t)chunks);
+  uint4* const st0 = &stage[warp][0][lane];
+  uint4* const st1 = &stage[warp][1][lane];
+
+  if (warp_global < units) {
+    cp_async16(st0, wp);
+    cp_async16(st0 + 32, wp + 1);
+  }
+  cp_async_commit();
+  __syncthreads();  // the candidate table
+
+  float2 hv2[8];
+  float hsum = 16.0f;
+  int cur_chunk = -1;
+#pragma unroll
+  for (int j = 0; j < 8; ++j) hv2[j] = make_float2(1.0f, 1.0f);
+
+  int buf = 0;
+  for (int64_t u = warp_global; u < units; u += warps_total, buf ^= 1) {
+    // the copy of the warp's next unit starts now
+    if (u + warps_total < units) {
+      uint4* dst = buf ? st0 : st1;
+      cp_async16(dst, wp + wstep);
+      cp_async16(dst + 32, wp + wstep + 1);
+    }
+    cp_async_commit();
+
+    if (h != nullptr && chunk != cur_chunk) {
+      cur_chunk = chunk;
+      const float4* hp = reinterpret_cast<const float4*>(h + ((int64_t)chunk * 32 + lane) * 16);
+#pragma unroll
+      for (int i = 0; i < 4; ++i) {
+        const float4 t = hp[i];
+        hv2[2 * i] = make_float2(t.x, t.y);
+        hv2[2 * i + 1] = make_float2(t.z, t.w);
+      }
+      float2 s2 = __fadd2_rn(__fadd2_rn(hv2[0], hv2[1]), __fadd2_rn(hv2[2], hv2[3]));
+      s2 = __fadd2_rn(s2, __fadd2_rn(__fadd2_rn(hv2[4], hv2[5]), __fadd2_rn(hv2[6], hv2[7])));
+      hsum = __fadd_rn(s2.x, s2.y);
+    }
+
+    cp_async_wait_1();  // this lane's copy of the current unit has landed
+    const uint4* cur = buf ? st1 : st0;
+    const uint4 p = cur[0], q = cur[32];
+    const float amax_k = __fmul_rn(__uint_as_float(group_abs_max_bits(p, q) << 16), d.pw);
+    Group G;
+    unpack_group(p, q, d.pw, G);
+    int c0;
+    if (!kFourOverSix && init_codes != nullptr) {
+      c0 = init_codes[go] & 0x7F;
+      c0 = c0 < 1 ? 1 : (c0 > (int)kE4M3MaxCode ? (int)kE4M3MaxCode : c0);
+    } else {
+      c0 = kFourOverSix ? fourover6_init_code(G, wp, tab, amax_k, d.sgk, d.pw, inv4, inv6, b4, b6)
+                        : (int)anchored_code_fast(amax_k, d.sgk, b6.x, b6.y, inv6, 3.0f);
+    }
+    const int lo = max(1, c0 - down);
+    const int hi = min((int)kE4M3MaxCode, c0 + up);
+
+    float e1 = kInf, e2 = kInf;
+    int best = c0;
+    score_range(G, hv2, tab, lo, hi + 1, e1, e2, best);
+
+    const bool ambiguous = hi > lo && !fast_winner_certain(e1, e2, energy_bound(hsum, amax_k));
+    unsigned amb = __ballot_sync(0xFFFFFFFFu, ambiguous);
+    while (amb) {
+      const int owner = __ffs(amb) - 1;
+      amb &= amb - 1;
+      const int64_t g_own = __shfl_sync(0xFFFFFFFFu, go, owner);
+      const int c0o = __shfl_sync(0xFFFFFFFFu, c0, owner);
+      const int loo = __shfl_sync(0xFFFFFFFFu, lo, owner);
+      const int hio = __shfl_sync(0xFFFFFFFFu, hi, owner);
+      const int bc = warp_exact_search(owner, reinterpret_cast<const uint16_t*>(w) + g_own * 16, h,
+                                       chunk * 32 + owner, c0o, loo, hio, d.sgk, d.pw);
+      if (lane == owner) best = bc;
+    }
+
+    codes_out[go] = (uint8_t)best;
+    if (packed_out != nullptr)
+      packed_out[go] = quantize_pack(G, (uint32_t)best, tab[best].z, d.sgk, d.pw,
+                                     reinterpret_cast<const uint16_t*>(wp));
+    wp += wstep;
+    go += ostep;
+    chunk += chunk_step;
+    if (chunk >= chunks) chunk -= chunks;
   }
 }
 
@@ -540,7 +724,7 @@ __global__ void __launch_bounds__(256) pack_kernel(const uint4* __restrict__ w, 
     load_group(w, g, d.pw, G);
     uint32_t c = codes[g] & 0x7Fu;
     c = c < 1 ? 1u : (c > kE4M3MaxCode ? kE4M3MaxCode : c);
-    packed_out[g] = quantize_pack(G, c, inv_raw_of(__fmul_rn(e4m3_mag(c), d.sgk)), d.sgk, d.pw,
+    packed_out[g] = quantize_pack(G, c, __frcp_rn(__fmul_rn(e4m3_mag(c), d.sgk)), d.sgk, d.pw,
                                   reinterpret_cast<const uint16_t*>(w) + g * 16);
   }
 }
@@ -560,10 +744,9 @@ __global__ void __launch_bounds__(256) fourover6_codes_kernel(const uint4* __res
   const int64_t stride = (int64_t)gridDim.x * blockDim.x;
   for (int64_t g = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; g < groups; g += stride) {
     Group G;
-    load_group(w, g, d.pw, G);
-    const uint32_t amax = group_abs_max_bits(make_uint4(G.wb[0], G.wb[1], G.wb[2], G.wb[3]),
-                                             make_uint4(G.wb[4], G.wb[5], G.wb[6], G.wb[7]));
-    const float amax_k = __fmul_rn(__uint_as_float(amax << 16), d.pw);
+    const uint4 p = ld_stream_v4(w + 2 * g), q = ld_stream_v4(w + 2 * g + 1);
+    unpack_group(p, q, d.pw, G);
+    const float amax_k = __fmul_rn(__uint_as_float(group_abs_max_bits(p, q) << 16), d.pw);
     const uint32_t c4 = anchored_code(amax_k, d.sgk, inv4, 2.0f);
     const uint32_t c6 = anchored_code(amax_k, d.sgk, inv6, 3.0f);
     uint32_t c = c4;
@@ -624,11 +807,23 @@ cudaError_t launch_refine(const void* w, int64_t ld_w, const float* h, int64_t m
   if (err != cudaSuccess) return err;
   const int ng = (int)(n / 16);
   const int64_t units = m * ((ng + 31) / 32);
-  int per_sm = fourover6 ? occupancy_blocks<refine_kernel<true>>(kRefineThreads)
-                         : occupancy_blocks<refine_kernel<false>>(kRefineThreads);
+  // contiguous W and outputs with whole row chunks: the pointer-walk kernel
+  const bool linear = ld_w == n && ng % 32 == 0 && ld_codes == ng && (packed_out == nullptr || ld_packed == n / 2) &&
+                      (init_codes == nullptr || ld_init == ng);
+  int per_sm = linear ? (fourover6 ? occupancy_blocks<refine_linear_kernel<true>>(kRefineThreads)
+                                   : occupancy_blocks<refine_linear_kernel<false>>(kRefineThreads))
+                      : (fourover6 ? occupancy_blocks<refine_kernel<true>>(kRefineThreads)
+                                   : occupancy_blocks<refine_kernel<false>>(kRefineThreads));
   if (ctas_per_sm > 0) per_sm = std::min(per_sm, ctas_per_sm);
   const int64_t resident = (int64_t)info.sm_count * per_sm;
   const int64_t blocks = std::max<int64_t>(1, std::min<int64_t>((units + kWarpsPerRefineBlock - 1) / kWarpsPerRefineBlock, resident));
+  if (linear) {
+    auto lk = fourover6 ? refine_linear_kernel<true> : refine_linear_kernel<false>;
+    lk<<<(unsigned)blocks, kRefineThreads, 0, stream>>>(static_cast<const uint4*>(w), h, units, (ng + 31) / 32,
+                                                         global_scale, fourover6 ? nullptr : init_codes, down, up,
+                                                         codes_out, reinterpret_cast<uint2*>(packed_out));
+    return cudaGetLastError();
+  }
   auto kernel = fourover6 ? refine_kernel<true> : refine_kernel<false>;
   kernel<<<(unsigned)blocks, kRefineThreads, 0, stream>>>(static_cast<const uint4*>(w), ld_w, h, m, ng, global_scale,
                                                           fourover6 ? nullptr : init_codes, ld_init, down, up,

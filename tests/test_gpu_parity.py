@@ -323,6 +323,47 @@ def test_refine_edge_groups():
         assert codes[5, 6] == ref["codes"][5, 6]
 
 
+def test_refine_inline_rtn_on_exact_e4m3_ties():
+    """The search's own RTN start (init_codes = NULL) on groups whose max sits exactly on every
+    E4M3 ladder value and midpoint (s_g = 2^-10): exact ties are decided half-to-even, as in
+    hscale_rtn_scales; the codes below 8 (E4M3 subnormals) are included."""
+    w = exact_tie_matrix()
+    b = bits(w)
+    m, n = w.shape
+    h32 = oracle_h32(12, n)
+    wd = w.to(dev())
+    sg, rtn = gpu_rtn(wd)
+    s_ref, _ = oracle.global_scale(b)
+    assert np.array_equal(rtn.cpu().numpy(), oracle.rtn_codes(b, s_ref))
+    for down, up in ((0, 0), (4, 4), (9, 6)):
+        ref = oracle.refine(b, h32, s_ref, None, down, up)
+        codes, packed = gpu_refine(wd, h32, sg, None, down, up)
+        compare_search(ref, codes, packed, f"exact E4M3 ties -{down}/+{up}")
+        if down == up == 0:
+            assert np.array_equal(codes, rtn.cpu().numpy())
+
+
+def test_refine_group_magnitudes_across_the_ladder():
+    """Groups scaled over 2^-12 .. 2^0 of the tensor's amax, so their RTN codes cover the E4M3
+    subnormals, every binade and the clipped walk at both ends of the ladder."""
+    rng = np.random.default_rng(13)
+    m, n = 96, 512
+    w = (rng.standard_t(4, size=(m, n)) * 0.02).astype(np.float32)
+    scale = 2.0 ** rng.uniform(-12, 0, size=(m, n // 16))
+    w *= np.repeat(scale, 16, axis=1).astype(np.float32)
+    w[0, 0] = 3.0
+    wb = torch.from_numpy(w).to(torch.bfloat16)
+    h32 = oracle_h32(14, n)
+    wd = wb.to(dev())
+    sg, _ = gpu_rtn(wd)
+    s_ref, _ = oracle.global_scale(bits(wb))
+    for down, up in ((4, 4), (9, 6), (16, 16)):
+        ref = oracle.refine(bits(wb), h32, s_ref, None, down, up)
+        codes, packed = gpu_refine(wd, h32, sg, None, down, up)
+        compare_search(ref, codes, packed, f"magnitudes across the ladder -{down}/+{up}")
+        assert (ref["codes"] < 8).any()
+
+
 @pytest.mark.parametrize("m,n", [(1, 16), (3, 48), (33, 16 * 33), (1, 4096 * 4)])
 def test_refine_tiny_and_ragged_shapes(m, n):
     w = wl.weight(m, n, 0.02, m * 1000 + n)
