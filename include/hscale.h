@@ -359,13 +359,16 @@ int hscale_output_error(const void* x_bf16, int64_t tokens, int64_t n, int64_t l
  *    zeroed in step 3) and get H_jj = 1; the diagonal gets damp * mean(diag H) (GPTQ uses
  *    damp = 0.01); U [n, n] (fp32, row stride n) is upper triangular with
  *    U^T U = (H + damp I)^-1, formed from the Cholesky factor of the reversed matrix and
- *    its triangular inverse (no explicit inverse of H).  cuSOLVER (Cholesky) and cuBLAS
- *    (triangular solve) are loaded at run time: without them the call returns
- *    HSCALE_ERR_CUDA and the rest of the library is unaffected.  info is a device int32[3]:
- *    info[0] the status of the factorization (0 = success, > 0: not positive definite),
- *    info[1] = info[2] = 0.  The workspace (hscale_gptq_factor_workspace_bytes, 256-byte
- *    aligned) holds n^2 floats for the reversed matrix and its factor plus cuSOLVER's.
- *    n < 46341.
+ *    its triangular inverse (no explicit inverse of H), by the library's own kernels: a
+ *    blocked Cholesky in 128-wide block columns with the triangular inverse built in the same
+ *    sweep, the diagonal blocks on CUDA cores and the trailing updates on the tensor cores
+ *    with fp32-level accuracy (three-way bf16 splits).  info is a device int32[3]: info[0] the
+ *    status of the factorization (0 = success; > 0: a pivot was not positive, the damped
+ *    matrix is not positive definite, and U is unspecified), info[1] = info[2] = 0.  The
+ *    workspace (hscale_gptq_factor_workspace_bytes, 256-byte aligned) holds the reversed
+ *    matrix and the inverse side by side (2 n_pad^2 floats, n_pad = 128 ceil(n / 128)) and
+ *    the split operands of the updates.  U's buffer also serves as scratch for the damped
+ *    copy of H during the call.  n <= 65536.
  *
  * 3. hscale_gptq_hscale: for each block of `block` columns (a multiple of 16 dividing n)
  *    of the running fp32 weights (W with dead columns zeroed): the RTN codes of Eq. 7 of

@@ -62,7 +62,7 @@ def build(force: bool = False, verbose: bool = False) -> pathlib.Path:
         results = list(ex.map(compile_one, sources()))
     (BUILD / "ptxas.log").write_text("".join(log for _, log in results))
     tmp = BUILD / f"libhscale.{os.getpid()}.so"
-    cmd = [nvcc, *ARCH, "-shared", "-o", str(tmp), *[str(o) for o, _ in results], "-ldl"]
+    cmd = [nvcc, *ARCH, "-shared", "-o", str(tmp), *[str(o) for o, _ in results]]
     r = subprocess.run(cmd, capture_output=True, text=True)
     if r.returncode != 0:
         raise RuntimeError(f"link failed:\n{r.stdout}\n{r.stderr}")

@@ -250,24 +250,20 @@ int hscale_hessian_full_accumulate(const void* x_bf16, int64_t tokens, int64_t n
 }
 
 size_t hscale_gptq_factor_workspace_bytes(int64_t n) {
-  if (n <= 0 || n > INT32_MAX) return 0;
-  const size_t floats = hscale::gptq_factor_solver_floats(n);
-  return floats ? (floats * 4 + 255) / 256 * 256 : 0;
+  if (n <= 0 || n > 65536) return 0;
+  return hscale::gptq_factor_workspace(n);
 }
 
 int hscale_gptq_factor(const float* H, int64_t n, int64_t ld_h, float damp, float* U, uint8_t* dead,
                        int32_t* info, void* workspace, size_t workspace_bytes, void* stream) {
-  if (n < 0 || ld_h < n || n > 46340) return HSCALE_ERR_SHAPE;  // n^2 < 2^31 (cuSOLVER's int sizes)
+  if (n < 0 || ld_h < n || n > 65536) return HSCALE_ERR_SHAPE;
   if (!(damp >= 0.0f)) return HSCALE_ERR_ARG;
   if (n == 0) return HSCALE_OK;
   if (H == nullptr || U == nullptr || info == nullptr) return HSCALE_ERR_NULL;
   if (!aligned(H, 4) || !aligned(U, 4) || !aligned(info, 4)) return HSCALE_ERR_ALIGN;
-  if (!hscale::gptq_solver_available()) return HSCALE_ERR_CUDA;
-  const size_t need = hscale_gptq_factor_workspace_bytes(n);
-  if (workspace == nullptr || need == 0 || workspace_bytes < need || !aligned(workspace, 256))
+  if (workspace == nullptr || workspace_bytes < hscale_gptq_factor_workspace_bytes(n) || !aligned(workspace, 256))
     return HSCALE_ERR_WORKSPACE;
-  return from_cuda(hscale::launch_gptq_factor(H, n, ld_h, damp, U, dead, info, static_cast<float*>(workspace),
-                                              workspace_bytes / 4, as_stream(stream)));
+  return from_cuda(hscale::launch_gptq_factor(H, n, ld_h, damp, U, dead, info, workspace, as_stream(stream)));
 }
 
 namespace {

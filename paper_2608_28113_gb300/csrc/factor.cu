@@ -1,0 +1,586 @@
+// factor.cu -- the damped inverse-Cholesky factor of GPTQ (Algorithm 3) on sm_103a.
+//
+// U is upper triangular with U^T U = A^-1 for the damped Hessian A = H + damp * mean(diag H) I
+// (dead channels, H_jj = 0, get H_jj = 1 first).  With J the order-reversing permutation and
+// B = J A J = L L^T (L lower, Cholesky), A = (J L J)(J L^T J), so U = (J L J)^-1 = J L^-1 J:
+// upper triangular with a positive diagonal, hence the Cholesky factor of A^-1.  No inverse of
+// A is formed.
+//
+// B is padded to n_pad = 128 * ceil(n / 128) with an identity block, whose factor and inverse
+// are the identity.  B (then L, lower) and X (R, then X = L^-1, lower) sit side by side in one
+// [n_pad, 2 n_pad] buffer, so that the two updates of a step are one GEMM over contiguous
+// columns.  The sweep takes 128-wide block columns j = 0, 1, ...  (right-looking):
+//   diag     the CTA of factor_diag_kernel factors the (updated) diagonal block,
+//            B_jj = L_jj L_jj^T, in shared memory and inverts it, Z_jj = L_jj^-1, into the
+//            inverse's diagonal block (32-wide tiles: one warp factors and inverts each 32 x 32
+//            tile on the diagonal, the CTA's warps update the other tiles);
+//   strips   panel L_ij = B_ij Z_jj^T (i > j) and the inverse's row X_j,c = Z_jj R_j,c (c < j),
+//            in 64-wide strips on CUDA cores (factor_strip_kernel);
+//   updates  B_ik -= L_ij L_kj^T over the trailing square, and R_ic -= L_ij X_jc for i > j,
+//            c <= j: for the rows below the diagonal block, the columns from the trailing
+//            square's first to the inverse's block j are contiguous in the buffer, n_pad of
+//            them, and both updates are one product -L_:j [L_:j ; X_j,:]^T.  It runs on the
+//            tensor cores: the tcgen05 GEMM with three-way bf16 splits of both operands (the
+//            six products above 2^-24 relative, one GEMM over K = 6 * 128), which carries
+//            fp32-level accuracy.
+// X = L^-1 is built alongside: row blocks below the diagonal accumulate
+// R_ic = -sum_k L_ik X_kc as the sweep passes, and X_ic = Z_ii R_ic once row block i is reached.
+// A last kernel writes U_ij = X_{n-1-i, n-1-j}.
+//
+// A pivot that is not positive (the damped matrix is then not positive definite) is recorded
+// in info[0] as its 1-based order in B and replaced by 1, so the sweep ends with finite values;
+// U is then unspecified.
+#include <cuda_bf16.h>
+
+#include <algorithm>
+
+#include "hscale_internal.h"
+
+namespace hscale {
+namespace {
+
+constexpr int kNb = 128;                  // block of the sweep
+constexpr int kSub = 32;                  // sub-block of the diagonal factor (one warp)
+constexpr int kLd = kNb + 4;              // padded shared-memory row (16-byte multiple)
+constexpr int kDiagThreads = 512;
+constexpr int kDiagSmemBytes = (3 * kNb * kLd + 2 * kSub) * 4;
+constexpr int kStripRows = 32;            // rows (or columns) of one strip
+constexpr int kStripThreads = 256;
+constexpr int kStripSmemBytes = (kNb * (kNb + 4) + kNb * (kStripRows + 4)) * 4;
+constexpr int kSplitK = 6 * kNb;          // K of the split update GEMMs
+
+// ---------------------------------------------------------------- set-up
+// One block: dead channels, the mean of the diagonal, and the damping added to it.  A is the
+// n x n copy of H (row stride n).
+__global__ void __launch_bounds__(1024) damp_diagonal_kernel(float* A, int64_t n, float damp, uint8_t* dead) {
+  __shared__ double part[1024];
+  double s = 0.0;
+  for (int64_t j = threadIdx.x; j < n; j += blockDim.x) {
+    float d = A[j * n + j];
+    const bool is_dead = (d == 0.0f);
+    if (is_dead) A[j * n + j] = d = 1.0f;
+    if (dead) dead[j] = (uint8_t)is_dead;
+    s += (double)d;
+  }
+  part[threadIdx.x] = s;
+  __syncthreads();
+  for (int step = 512; step > 0; step >>= 1) {
+    if ((int)threadIdx.x < step) part[threadIdx.x] += part[threadIdx.x + step];
+    __syncthreads();
+  }
+  const float add = (float)((double)damp * part[0] / (double)n);
+  for (int64_t j = threadIdx.x; j < n; j += blockDim.x) A[j * n + j] += add;
+}
+
+// W2 [n_pad, 2 n_pad]: the left half B_ij = A_{n-1-i, n-1-j} (taken from A's upper triangle)
+// for i, j < n and the identity beyond, the right half (X) zero.
+__global__ void __launch_bounds__(256) reverse_pad_kernel(const float* __restrict__ A, int64_t n, int64_t n_pad,
+                                                          float* __restrict__ W2) {
+  const int64_t total = n_pad * n_pad;
+  for (int64_t e = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; e < total; e += (int64_t)gridDim.x * blockDim.x) {
+    const int64_t i = e / n_pad, j = e - i * n_pad;
+    float v;
+    if (i < n && j < n) {
+      const int64_t p = n - 1 - i, q = n - 1 - j;
+      v = p <= q ? A[p * n + q] : A[q * n + p];
+    } else {
+      v = (i == j) ? 1.0f : 0.0f;
+    }
+    W2[i * 2 * n_pad + j] = v;
+    W2[i * 2 * n_pad + n_pad + j] = 0.0f;
+  }
+}
+
+// U_ij = X_{n-1-i, n-1-j} for j >= i, 0 below the diagonal (U row stride n; X row stride ld).
+__global__ void __launch_bounds__(256) reverse_out_kernel(const float* __restrict__ Xw, int64_t ld, int64_t n,
+                                                          float* __restrict__ U) {
+  const int64_t total = n * n;
+  for (int64_t e = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; e < total; e += (int64_t)gridDim.x * blockDim.x) {
+    const int64_t i = e / n, j = e - i * n;
+    U[e] = j >= i ? Xw[(n - 1 - i) * ld + (n - 1 - j)] : 0.0f;
+  }
+}
+
+// ---------------------------------------------------------------- diagonal block
+__device__ __forceinline__ void record_failure(int32_t* info, int32_t order) {
+  atomicCAS(reinterpret_cast<int*>(info), 0, order);
+}
+
+__device__ __forceinline__ float rsqrt_approx(float x) {
+  float r;
+  asm("rsqrt.approx.f32 %0, %1;" : "=f"(r) : "f"(x));
+  return r;
+}
+__device__ __forceinline__ float rcp_approx_f(float x) {
+  float r;
+  asm("rcp.approx.f32 %0, %1;" : "=f"(r) : "f"(x));
+  return r;
+}
+
+// One warp factors the 32 x 32 block at A (row stride kLd, lower triangle) in place,
+// A = L L^T, and writes Z = L^-1 (lower, zeros above) at Zo and its transpose at Zt (row
+// stride kLd each); col is a 64-float scratch.  Lane i holds row i of the block in registers
+// (every loop has a constant trip count and every register index is a constant, so the row
+// stays in registers; kept out of line: inlined into the block kernel, the compiler moves the
+// row to local memory).  Two columns are eliminated per step: the 2 x 2 pivot block gives
+// L_jj, L_j+1,j and L_j+1,j+1, every lane scales its two entries, the pairs (L_kj, L_k,j+1)
+// go to shared memory and come back four rows per 16-byte broadcast load, and each lane
+// updates its row.  Entries above the diagonal are updated too (harmlessly) and zeroed at the
+// end.  The square roots and reciprocals come from the approximate hardware instructions
+// (relative error about 2^-22), which keeps the serial chain of pivots short.  Then lane c
+// computes column c of Z by forward substitution, reading L from shared memory (a broadcast).
+__device__ __noinline__ void factor_sub32(float* A, float* Zo, float* Zt, float* col, int lane, int32_t* info,
+                                          int32_t base) {
+  const unsigned full = 0xFFFFFFFFu;
+  float r[kSub];
+#pragma unroll
+  for (int k = 0; k < kSub; ++k) r[k] = A[lane * kLd + k];
+  float2* col2 = reinterpret_cast<float2*>(col);
+#pragma unroll
+  for (int j = 0; j < kSub; j += 2) {
+    float a = __shfl_sync(full, r[j], j);
+    const float b = __shfl_sync(full, r[j], j + 1);
+    float c = __shfl_sync(full, r[j + 1], j + 1);
+    if (!(a > 0.0f)) {
+      if (lane == 0) record_failure(info, base + j + 1);
+      a = 1.0f;
+    }
+    const float ra = rsqrt_approx(a);
+    const float l00 = __fmul_rn(a, ra), l10 = __fmul_rn(b, ra);
+    float c2 = __fmaf_rn(-l10, l10, c);
+    if (!(c2 > 0.0f)) {
+      if (lane == 0) record_failure(info, base + j + 2);
+      c2 = 1.0f;
+    }
+    const float rc = rsqrt_approx(c2);
+    const float l11 = __fmul_rn(c2, rc);
+    // this lane's entries of columns j and j + 1
+    const float x0 = __fmul_rn(r[j], ra);
+    const float x1 = __fmul_rn(__fmaf_rn(-x0, l10, r[j + 1]), rc);
+    const float v0 = lane == j ? l00 : (lane == j + 1 ? l10 : (lane > j + 1 ? x0 : 0.0f));
+    const float v1 = lane == j + 1 ? l11 : (lane > j + 1 ? x1 : 0.0f);
+    r[j] = v0;
+    r[j + 1] = v1;
+    if (j + 2 < kSub) {
+      col2[lane] = make_float2(v0, v1);
+      __syncwarp();
+#pragma unroll
+      for (int k = j + 2; k < kSub; k += 2) {
+        const float4 q = *reinterpret_cast<const float4*>(col + 2 * k);  // (L_kj, L_k,j+1, L_k+1,j, L_k+1,j+1)
+        r[k] = __fmaf_rn(-v0, q.x, __fmaf_rn(-v1, q.y, r[k]));
+        r[k + 1] = __fmaf_rn(-v0, q.z, __fmaf_rn(-v1, q.w, r[k + 1]));
+      }
+      __syncwarp();
+    }
+  }
+#pragma unroll
+  for (int k = 0; k < kSub; ++k) A[lane * kLd + k] = k <= lane ? r[k] : 0.0f;
+  __syncwarp();
+  float x[kSub];
+#pragma unroll
+  for (int i = 0; i < kSub; ++i) {
+    float acc0 = 0.0f, acc1 = 0.0f, acc2 = 0.0f, acc3 = 0.0f;
+#pragma unroll
+    for (int m = 0; m + 3 < i; m += 4) {
+      const float4 l = *reinterpret_cast<const float4*>(A + i * kLd + m);
+      acc0 = __fmaf_rn(l.x, x[m], acc0);
+      acc1 = __fmaf_rn(l.y, x[m + 1], acc1);
+      acc2 = __fmaf_rn(l.z, x[m + 2], acc2);
+      acc3 = __fmaf_rn(l.w, x[m + 3], acc3);
+    }
+#pragma unroll
+    for (int m = i & ~3; m < i; ++m) acc0 = __fmaf_rn(A[i * kLd + m], x[m], acc0);
+    const float invl = rcp_approx_f(A[i * kLd + i]);
+    const float v = -__fmul_rn(__fadd_rn(__fadd_rn(acc0, acc1), __fadd_rn(acc2, acc3)), invl);
+    x[i] = lane == i ? invl : (lane < i ? v : 0.0f);
+  }
+#pragma unroll
+  for (int i = 0; i < kSub; ++i) {
+    Zo[i * kLd + lane] = x[i];
+    Zt[lane * kLd + i] = x[i];
+  }
+}
+
+// Warp-tile products on 32 x 32 tiles in shared memory (row stride kLd, a multiple of 4): a
+// warp computes kR rows of the output tile, lane c column c, in acc[0..kR) (independent
+// accumulators).  A's rows are read four entries at a time (the same address in every lane: a
+// broadcast), B's row m at column c (consecutive lanes, consecutive words).
+//   acc[r] += sum_m A[r][m] B[m][c]   (acc[r] -= ... with kNeg), rows r of A from A's row 0
+template <int kR, bool kNeg = false>
+__device__ __forceinline__ void tile_nn(float (&acc)[kR], const float* A, const float* B, int lane) {
+#pragma unroll 2
+  for (int m = 0; m < kSub; m += 4) {
+    float b0 = B[m * kLd + lane], b1 = B[(m + 1) * kLd + lane];
+    float b2 = B[(m + 2) * kLd + lane], b3 = B[(m + 3) * kLd + lane];
+    if (kNeg) {
+      b0 = -b0;
+      b1 = -b1;
+      b2 = -b2;
+      b3 = -b3;
+    }
+#pragma unroll
+    for (int r = 0; r < kR; ++r) {
+      const float4 a = *reinterpret_cast<const float4*>(A + r * kLd + m);
+      acc[r] = __fmaf_rn(a.x, b0, acc[r]);
+      acc[r] = __fmaf_rn(a.y, b1, acc[r]);
+      acc[r] = __fmaf_rn(a.z, b2, acc[r]);
+      acc[r] = __fmaf_rn(a.w, b3, acc[r]);
+    }
+  }
+}
+template <int kR>
+__device__ __forceinline__ void tile_zero(float (&acc)[kR]) {
+#pragma unroll
+  for (int r = 0; r < kR; ++r) acc[r] = 0.0f;
+}
+template <int kR>
+__device__ __forceinline__ void tile_load(float (&acc)[kR], const float* T, int lane) {
+#pragma unroll
+  for (int r = 0; r < kR; ++r) acc[r] = T[r * kLd + lane];
+}
+template <int kR>
+__device__ __forceinline__ void tile_store(const float (&acc)[kR], float* T, int lane, float sign) {
+#pragma unroll
+  for (int r = 0; r < kR; ++r) T[r * kLd + lane] = sign * acc[r];
+}
+
+constexpr int kQ = 8;                     // rows of a tile per warp (four warps per tile)
+
+// Factor the 128 x 128 diagonal block at (j0, j0) of Bw and invert the factor: Z_jj = L_jj^-1
+// into Xw's diagonal block (zeros above the diagonal).  The block is a 4 x 4 grid of 32 x 32
+// tiles, taken in tile columns p = 0..3:
+//   (a) warp 0 factors the tile on the diagonal and inverts it (factor_sub32);
+//   (b) the tiles below it: L_ip = B_ip Z_p^T, one warp per tile;
+//   (c) the tiles of the rest of the block: B_ik -= L_ip L_kp^T, one warp per tile.
+// Then the inverse of the block, tile row q = 1..3: T_qr = sum_{m=r}^{q-1} L_qm X_mr and
+// X_qr = -Z_q T_qr, one warp per tile.  The transposes a tile product needs (Z_p^T, L_kp^T)
+// are written next to the tiles.
+__global__ void __launch_bounds__(kDiagThreads, 1)
+factor_diag_kernel(const float* __restrict__ Bw, int64_t ld, int64_t j0, float* __restrict__ Xw,
+                   int32_t* __restrict__ info) {
+  extern __shared__ __align__(16) float sm[];
+  float* S = sm;                 // [128][kLd] the block, then L (lower)
+  float* X = S + kNb * kLd;      // [128][kLd] the inverse (lower)
+  float* St = X + kNb * kLd;     // [128][kLd] transposes: Z_p^T in its diagonal tile, L^T
+  float* col = St + kNb * kLd;   // [64] the pivot columns of factor_sub32
+  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+  const int part = warp & 3;     // which 8 rows of its tile a warp computes
+  const int unit = warp >> 2;    // which tile (of up to four at a time)
+
+  const float* blk = Bw + j0 * ld + j0;
+  // independent 16-byte loads per thread in flight
+#pragma unroll 4
+  for (int t = 0; t < kNb * kNb / 4 / kDiagThreads; ++t) {
+    const int e = tid + t * kDiagThreads;
+    const int r = e >> 5, c = (e & 31) * 4;
+    *reinterpret_cast<float4*>(S + r * kLd + c) = *reinterpret_cast<const float4*>(blk + r * ld + c);
+    *reinterpret_cast<float4*>(X + r * kLd + c) = make_float4(0.f, 0.f, 0.f, 0.f);
+  }
+  __syncthreads();
+
+  for (int p = 0; p < kNb / kSub; ++p) {
+    const int c0 = p * kSub;
+    if (warp == 0)
+      factor_sub32(S + c0 * kLd + c0, X + c0 * kLd + c0, St + c0 * kLd + c0, col, lane, info, (int32_t)(j0 + c0));
+    __syncthreads();
+    // (b) tiles below: L_ip = B_ip Z_p^T, four warps per tile
+    const int below = kNb / kSub - 1 - p;
+    if (unit < below) {
+      const int i0 = c0 + kSub * (1 + unit) + kQ * part;  // this warp's first row
+      float acc[kQ];
+      tile_zero(acc);
+      tile_nn<kQ>(acc, S + i0 * kLd + c0, St + c0 * kLd + c0, lane);
+      __syncwarp();
+      tile_store(acc, S + i0 * kLd + c0, lane, 1.0f);
+      // the transpose L_ip^T, for (c): St[c0 + c][i0 + r] = L_ip[r][c]
+      *reinterpret_cast<float4*>(St + (c0 + lane) * kLd + i0) = make_float4(acc[0], acc[1], acc[2], acc[3]);
+      *reinterpret_cast<float4*>(St + (c0 + lane) * kLd + i0 + 4) = make_float4(acc[4], acc[5], acc[6], acc[7]);
+    }
+    __syncthreads();
+    // (c) tiles (i, k), p < k <= i: B_ik -= L_ip L_kp^T = L_ip (L_kp^T), four warps per tile;
+    // up to six tiles, so the sixteen warps take them in two rounds
+    for (int round = 0; round < 2; ++round) {
+      int t = unit + 4 * round, i = p + 1;
+      while (i < kNb / kSub && t > i - (p + 1)) {
+        t -= i - p;
+        ++i;
+      }
+      if (i < kNb / kSub) {
+        const int k0 = (p + 1 + t) * kSub, i0 = i * kSub + kQ * part;
+        float acc[kQ];
+        tile_load(acc, S + i0 * kLd + k0, lane);
+        tile_nn<kQ, true>(acc, S + i0 * kLd + c0, St + c0 * kLd + k0, lane);
+        tile_store(acc, S + i0 * kLd + k0, lane, 1.0f);
+      }
+    }
+    __syncthreads();
+  }
+
+  // inverse of the whole block, tile row q = 1..3; T tiles kept in St's first tile row
+  for (int q = 1; q < kNb / kSub; ++q) {
+    const int q0 = q * kSub;
+    if (unit < q) {
+      const int r0 = unit * kSub, i0 = kQ * part;
+      float acc[kQ];
+      tile_zero(acc);
+      for (int m = unit; m < q; ++m)
+        tile_nn<kQ>(acc, S + (q0 + i0) * kLd + m * kSub, X + m * kSub * kLd + r0, lane);
+      tile_store(acc, St + i0 * kLd + r0, lane, 1.0f);
+    }
+    __syncthreads();
+    if (unit < q) {
+      const int r0 = unit * kSub, i0 = kQ * part;
+      float acc[kQ];
+      tile_zero(acc);
+      tile_nn<kQ>(acc, X + (q0 + i0) * kLd + q0, St + r0, lane);
+      tile_store(acc, X + (q0 + i0) * kLd + r0, lane, -1.0f);
+    }
+    __syncthreads();
+  }
+
+  // write-out: Z into Xw's diagonal block (16-byte words).  L_jj itself is not needed again:
+  // the panel uses Z_jj, and the rest of the sweep reads only the blocks below the diagonal.
+  float* xo = Xw + j0 * ld + j0;
+#pragma unroll 4
+  for (int t = 0; t < kNb * kNb / 4 / kDiagThreads; ++t) {
+    const int e = tid + t * kDiagThreads;
+    const int r = e >> 5, c = (e & 31) * 4;
+    *reinterpret_cast<float4*>(xo + r * ld + c) = *reinterpret_cast<const float4*>(X + r * kLd + c);
+  }
+}
+
+// ---------------------------------------------------------------- strips (CUDA cores)
+// Blocks [0, panel_strips): the panel below the diagonal block, 32 rows each:
+//   P[i][c] = sum_{m <= c} B[i][j0 + m] Z[c][m]        (L_ij = B_ij Z_jj^T, rows i of B)
+// written to P (row stride 128, rows relative to r_first).
+// Blocks [panel_strips, ...): the inverse's row j, 32 columns each, in place in Xw:
+//   X[j0 + r][c] = sum_{m <= r} Z[r][m] R[j0 + m][c]   (X_jc = Z_jj R_jc, c < j0)
+// Z = Z_jj is Xw's diagonal block.  256 threads; each computes 4 x 4 outputs over K = 128 from
+// shared memory.  The panel's columns c = tx + 32 k take Z's rows at a stride of 129 words
+// (consecutive lanes, distinct banks); the row's columns are one 16-byte word.  The staging
+// loads are unrolled so that each thread has several in flight.
+__global__ void __launch_bounds__(kStripThreads)
+factor_strip_kernel(const float* __restrict__ Bw, float* __restrict__ Xw, int64_t ld, int64_t j0,
+                    float* __restrict__ P, int panel_strips, int64_t r_first) {
+  extern __shared__ __align__(16) float sm[];
+  constexpr int kZl = kNb + 4;       // row-major Z for the row strips (16-byte rows)
+  constexpr int kZp = kNb + 1;       // row-major Z for the panel (column reads across lanes)
+  constexpr int kRl = kStripRows + 4;
+  const int tid = threadIdx.x;
+  const bool panel = (int)blockIdx.x < panel_strips;
+  const int sb = panel ? (int)blockIdx.x : (int)blockIdx.x - panel_strips;
+  float* Zs = sm;                    // 128 x (kZl or kZp)
+  float* Ss = sm + kNb * kZl;        // panel: B rows (i, m), 32 x kZl; row: R (m, c), 128 x kRl
+  const float* zsrc = Xw + j0 * ld + j0;
+  float acc[4][4];
+#pragma unroll
+  for (int a = 0; a < 4; ++a)
+#pragma unroll
+    for (int b = 0; b < 4; ++b) acc[a][b] = 0.0f;
+  if (panel) {
+#pragma unroll 16
+    for (int e = tid; e < kNb * kNb / 4; e += kStripThreads) {
+      const int r = e >> 5, c = (e & 31) * 4;
+      const float4 v = *reinterpret_cast<const float4*>(zsrc + r * ld + c);
+      Zs[r * kZp + c] = v.x;
+      Zs[r * kZp + c + 1] = v.y;
+      Zs[r * kZp + c + 2] = v.z;
+      Zs[r * kZp + c + 3] = v.w;
+    }
+    const int64_t row0 = r_first + (int64_t)sb * kStripRows;
+#pragma unroll 4
+    for (int e = tid; e < kStripRows * kNb / 4; e += kStripThreads) {
+      const int i = e >> 5, m = (e & 31) * 4;
+      *reinterpret_cast<float4*>(Ss + i * kZl + m) = *reinterpret_cast<const float4*>(Bw + (row0 + i) * ld + j0 + m);
+    }
+    __syncthreads();
+    // outputs 32 rows x 128 columns: rows 4 ty .. +3, columns tx + 32 k (k < 4)
+    const int ty = tid >> 5, tx = tid & 31;
+#pragma unroll 4
+    for (int m = 0; m < kNb; ++m) {
+      float bv[4];
+#pragma unroll
+      for (int k = 0; k < 4; ++k) bv[k] = Zs[(tx + 32 * k) * kZp + m];
+#pragma unroll
+      for (int a = 0; a < 4; ++a) {
+        const float av = Ss[(4 * ty + a) * kZl + m];
+#pragma unroll
+        for (int k = 0; k < 4; ++k) acc[a][k] = __fmaf_rn(av, bv[k], acc[a][k]);
+      }
+    }
+#pragma unroll
+    for (int a = 0; a < 4; ++a)
+#pragma unroll
+      for (int k = 0; k < 4; ++k) P[((int64_t)sb * kStripRows + 4 * ty + a) * kNb + tx + 32 * k] = acc[a][k];
+  } else {
+#pragma unroll 16
+    for (int e = tid; e < kNb * kNb / 4; e += kStripThreads) {
+      const int r = e >> 5, c = (e & 31) * 4;
+      *reinterpret_cast<float4*>(Zs + r * kZl + c) = *reinterpret_cast<const float4*>(zsrc + r * ld + c);
+    }
+    const int64_t col0 = (int64_t)sb * kStripRows;
+#pragma unroll 4
+    for (int e = tid; e < kNb * kStripRows / 4; e += kStripThreads) {
+      const int m = e >> 3, c = (e & 7) * 4;
+      *reinterpret_cast<float4*>(Ss + m * kRl + c) = *reinterpret_cast<const float4*>(Xw + (j0 + m) * ld + col0 + c);
+    }
+    __syncthreads();
+    // outputs 128 rows x 32 columns: rows 4 ty .. +3, columns 4 tx .. +3
+    const int ty = tid >> 3, tx = tid & 7;
+#pragma unroll 4
+    for (int m = 0; m < kNb; ++m) {
+      const float4 bv = *reinterpret_cast<const float4*>(Ss + m * kRl + 4 * tx);
+#pragma unroll
+      for (int a = 0; a < 4; ++a) {
+        const float av = Zs[(4 * ty + a) * kZl + m];
+        acc[a][0] = __fmaf_rn(av, bv.x, acc[a][0]);
+        acc[a][1] = __fmaf_rn(av, bv.y, acc[a][1]);
+        acc[a][2] = __fmaf_rn(av, bv.z, acc[a][2]);
+        acc[a][3] = __fmaf_rn(av, bv.w, acc[a][3]);
+      }
+    }
+    __syncthreads();  // every thread has read its R entries before any is overwritten
+#pragma unroll
+    for (int a = 0; a < 4; ++a)
+      *reinterpret_cast<float4*>(Xw + (j0 + 4 * ty + a) * ld + col0 + 4 * tx) =
+          make_float4(acc[a][0], acc[a][1], acc[a][2], acc[a][3]);
+  }
+}
+
+// ---------------------------------------------------------------- three-way bf16 splits
+// x = x1 + x2 + x3 with bf16 parts, each difference exact in fp32: the parts carry x to
+// about 2^-24 relative.
+__device__ __forceinline__ void split3(float x, uint16_t (&p)[3]) {
+  const __nv_bfloat16 a = __float2bfloat16_rn(x);
+  const float r1 = __fsub_rn(x, __bfloat162float(a));
+  const __nv_bfloat16 b = __float2bfloat16_rn(r1);
+  const float r2 = __fsub_rn(r1, __bfloat162float(b));
+  const __nv_bfloat16 c = __float2bfloat16_rn(r2);
+  p[0] = __bfloat16_as_ushort(a);
+  p[1] = __bfloat16_as_ushort(b);
+  p[2] = __bfloat16_as_ushort(c);
+}
+
+// The panel P [rows, 128] (fp32) into its place in Bw (rows r_first.., columns j0..) and as
+// the two operands of the updates: An = [-P1 | -P1 | -P2 | -P1 | -P2 | -P3] and
+// Bp = [P1 | P2 | P1 | P3 | P2 | P1] (rows of 6 * 128 bf16), so that An Bp^T = -P P^T to fp32
+// accuracy (the six products E1U1, E1U2, E2U1, E1U3, E2U2, E3U1).
+__global__ void __launch_bounds__(256) factor_split_panel_kernel(const float* __restrict__ P, int64_t rows,
+                                                                 float* __restrict__ Bw, int64_t ld, int64_t r_first,
+                                                                 int64_t j0, uint16_t* __restrict__ An,
+                                                                 uint16_t* __restrict__ Bp) {
+  const int64_t total = rows * kNb;
+  for (int64_t e = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; e < total; e += (int64_t)gridDim.x * blockDim.x) {
+    const int64_t i = e >> 7;
+    const int k = (int)(e & (kNb - 1));
+    const float x = P[e];
+    Bw[(r_first + i) * ld + j0 + k] = x;
+    uint16_t p[3], q[3];
+    split3(x, p);
+    split3(-x, q);
+    uint16_t* a = An + i * kSplitK + k;
+    uint16_t* b = Bp + i * kSplitK + k;
+    a[0] = q[0]; a[kNb] = q[0]; a[2 * kNb] = q[1]; a[3 * kNb] = q[0]; a[4 * kNb] = q[1]; a[5 * kNb] = q[2];
+    b[0] = p[0]; b[kNb] = p[1]; b[2 * kNb] = p[0]; b[3 * kNb] = p[2]; b[4 * kNb] = p[1]; b[5 * kNb] = p[0];
+  }
+}
+
+// The inverse's row block j (Xw rows j0..j0+127, columns 0..cols-1) transposed, as the B
+// operand of the R update: Bx[c] = [X1 | X2 | X1 | X3 | X2 | X1] of column c of the row block,
+// through 32 x 32 shared-memory tiles (coalesced reads along c, writes along the row index).
+__global__ void __launch_bounds__(256) factor_split_row_kernel(const float* __restrict__ Xw, int64_t ld, int64_t j0,
+                                                               int64_t cols, uint16_t* __restrict__ Bx) {
+  __shared__ float t[32][33];
+  const int64_t c0 = (int64_t)blockIdx.x * 32;
+  const int m0 = blockIdx.y * 32;
+  const int tx = threadIdx.x & 31, ty = threadIdx.x >> 5;
+  for (int mm = ty; mm < 32; mm += 8) t[mm][tx] = c0 + tx < cols ? Xw[(j0 + m0 + mm) * ld + c0 + tx] : 0.0f;
+  __syncthreads();
+  for (int cc = ty; cc < 32; cc += 8) {
+    const int64_t c = c0 + cc;
+    if (c >= cols) continue;
+    uint16_t p[3];
+    split3(t[tx][cc], p);
+    uint16_t* b = Bx + c * kSplitK + m0 + tx;
+    b[0] = p[0]; b[kNb] = p[1]; b[2 * kNb] = p[0]; b[3 * kNb] = p[2]; b[4 * kNb] = p[1]; b[5 * kNb] = p[0];
+  }
+}
+
+inline int64_t round256(int64_t bytes) { return (bytes + 255) / 256 * 256; }
+
+}  // namespace
+
+int64_t gptq_factor_padded(int64_t n) { return (n + kNb - 1) / kNb * kNb; }
+
+// W2 = [B | X] (n_pad x 2 n_pad fp32), the panel (n_pad x 128 fp32) and the split operands (A: n_pad x 768 bf16; B: [L_:j ; X_j,:], n_pad x 768 bf16), each region
+// 256-byte aligned.
+size_t gptq_factor_workspace(int64_t n) {
+  const int64_t np = gptq_factor_padded(n);
+  return (size_t)(round256(2 * np * np * 4) + round256(np * kNb * 4) + 2 * round256(np * kSplitK * 2));
+}
+
+cudaError_t launch_gptq_factor(const float* H, int64_t n, int64_t ld_h, float damp, float* Uo, uint8_t* dead,
+                               int32_t* info, void* workspace, cudaStream_t stream) {
+  DeviceInfo dinfo;
+  cudaError_t err = current_device_info(&dinfo);
+  if (err != cudaSuccess) return err;
+  const int64_t np = gptq_factor_padded(n);
+  const int64_t ld = 2 * np;
+  uint8_t* base = static_cast<uint8_t*>(workspace);
+  float* Bw = reinterpret_cast<float*>(base);  // left half of W2; X = Bw + np
+  float* Xw = Bw + np;
+  float* P = reinterpret_cast<float*>(base + round256(2 * np * np * 4));
+  uint8_t* ops = base + round256(2 * np * np * 4) + round256(np * kNb * 4);
+  uint16_t* An = reinterpret_cast<uint16_t*>(ops);
+  uint16_t* Bo = reinterpret_cast<uint16_t*>(ops + round256(np * kSplitK * 2));
+
+  if ((err = cudaMemsetAsync(info, 0, 3 * sizeof(int32_t), stream)) != cudaSuccess) return err;
+  // the damped copy of H in U's buffer (n x n, row stride n)
+  if ((err = cudaMemcpy2DAsync(Uo, (size_t)n * 4, H, (size_t)ld_h * 4, (size_t)n * 4, (size_t)n,
+                               cudaMemcpyDeviceToDevice, stream)) != cudaSuccess)
+    return err;
+  damp_diagonal_kernel<<<1, 1024, 0, stream>>>(Uo, n, damp, dead);
+  if ((err = cudaGetLastError()) != cudaSuccess) return err;
+  const unsigned eblocks = (unsigned)std::max<int64_t>(1, std::min<int64_t>((np * np + 255) / 256,
+                                                                           (int64_t)dinfo.sm_count * 16));
+  reverse_pad_kernel<<<eblocks, 256, 0, stream>>>(Uo, n, np, Bw);
+  if ((err = cudaGetLastError()) != cudaSuccess) return err;
+  if ((err = ensure_dynamic_smem(reinterpret_cast<const void*>(factor_diag_kernel), kDiagSmemBytes)) != cudaSuccess)
+    return err;
+  if ((err = ensure_dynamic_smem(reinterpret_cast<const void*>(factor_strip_kernel), kStripSmemBytes)) != cudaSuccess)
+    return err;
+
+  const int64_t nblk = np / kNb;
+  for (int64_t jb = 0; jb < nblk; ++jb) {
+    const int64_t j0 = jb * kNb;
+    const int64_t r_first = j0 + kNb;          // first row below the diagonal block
+    const int64_t rows = np - r_first;         // rows of the panel
+    factor_diag_kernel<<<1, kDiagThreads, kDiagSmemBytes, stream>>>(Bw, ld, j0, Xw, info);
+    if ((err = cudaGetLastError()) != cudaSuccess) return err;
+    const int panel_strips = (int)(rows / kStripRows);
+    const int row_strips = (int)(j0 / kStripRows);
+    if (panel_strips + row_strips > 0) {
+      factor_strip_kernel<<<(unsigned)(panel_strips + row_strips), kStripThreads, kStripSmemBytes, stream>>>(
+          Bw, Xw, ld, j0, P, panel_strips, r_first);
+      if ((err = cudaGetLastError()) != cudaSuccess) return err;
+    }
+    if (rows == 0) break;
+    const unsigned sblocks = (unsigned)std::max<int64_t>(1, std::min<int64_t>((rows * kNb + 255) / 256,
+                                                                             (int64_t)dinfo.sm_count * 8));
+    factor_split_panel_kernel<<<sblocks, 256, 0, stream>>>(P, rows, Bw, ld, r_first, j0, An, Bo);
+    if ((err = cudaGetLastError()) != cudaSuccess) return err;
+    const int64_t xcols = j0 + kNb;            // columns of the inverse's row block j, diagonal included
+    factor_split_row_kernel<<<dim3((unsigned)((xcols + 31) / 32), kNb / 32), 256, 0, stream>>>(
+        Xw, ld, j0, xcols, Bo + rows * kSplitK);
+    if ((err = cudaGetLastError()) != cudaSuccess) return err;
+    // rows below the diagonal block, columns r_first .. np + xcols of W2 (rows + xcols = np):
+    // the trailing square and the inverse's rows, -= L_:j [L_:j ; X_j,:]^T
+    if ((err = launch_gemm_accumulate(An, Bo, rows, rows + xcols, kSplitK, Bw + r_first * ld + r_first, ld,
+                                      stream)) != cudaSuccess)
+      return err;
+  }
+  reverse_out_kernel<<<eblocks, 256, 0, stream>>>(Xw, ld, n, Uo);
+  return cudaGetLastError();
+}
+
+}  // namespace hscale

@@ -1,15 +1,6 @@
 // gptq.cu -- GPTQ with H-Scale as the local quantizer (Algorithm 3) on sm_103a.
 //
-//   factor            the damped inverse-Cholesky factor U of GPTQ: dead channels (H_jj = 0)
-//                     get H_jj = 1, the diagonal gets damp * mean(diag), and U is upper
-//                     triangular with U^T U = (H + damp I)^-1 = A^-1.  It is formed without
-//                     A^-1: with J the order-reversing permutation and J A J = L L^T (L lower,
-//                     Cholesky), A = (J L J)(J L^T J), so U = (J L J)^-1 = J L^-1 J, an
-//                     upper-triangular matrix with a positive diagonal, hence the Cholesky
-//                     factor.  cuSOLVER does the Cholesky and cuBLAS the triangular solve
-//                     L^T Y = I (both loaded at run time) on column-major storage: Y = L^-T
-//                     in column-major order is (J Y J)^T = U^T after reversing the array,
-//                     i.e. row-major U.
+//   (the damped inverse-Cholesky factor U is formed in factor.cu)
 //   block_kernel      four lanes per 16-element group of a block of B columns of the running
 //                     fp32 weights: the RTN code (Eq. 7) of the current weights, the exact
 //                     H-Scale search over the window (Algorithm 1, exact E2M1 decisions, the
@@ -17,139 +8,18 @@
 //                     propagated errors E = (W - W_hat) / U_jj
 //   update            W[:, i+B:] -= E U[i:i+B, i+B:] with fp32-level accuracy on the tensor
 //                     cores (three-way bf16 splits, six products, one GEMM)
-#include <dlfcn.h>
-
 #include <algorithm>
 #include <cstdio>
 #include <mutex>
 #include <vector>
 
-#include <cublas_v2.h>
 #include <cuda_bf16.h>
-#include <cusolverDn.h>
 
 #include "hscale_device.cuh"
 #include "hscale_internal.h"
 
 namespace hscale {
 namespace {
-
-// ---------------------------------------------------------------- cuSOLVER at run time
-struct Solver {
-  decltype(&cusolverDnCreate) create = nullptr;
-  decltype(&cusolverDnSetStream) set_stream = nullptr;
-  decltype(&cusolverDnSpotrf_bufferSize) potrf_size = nullptr;
-  decltype(&cusolverDnSpotrf) potrf = nullptr;
-  decltype(&cublasCreate_v2) blas_create = nullptr;
-  decltype(&cublasSetStream_v2) blas_set_stream = nullptr;
-  decltype(&cublasStrsm_v2) trsm = nullptr;
-  bool ok = false;
-};
-
-const Solver& solver() {
-  static Solver s;
-  static std::once_flag once;
-  std::call_once(once, [] {
-    void* lib = nullptr;
-    for (const char* name : {"libcusolver.so.12", "libcusolver.so.11", "libcusolver.so"}) {
-      lib = dlopen(name, RTLD_NOW | RTLD_LOCAL);
-      if (lib) break;
-    }
-    if (!lib) return;
-    s.create = reinterpret_cast<decltype(s.create)>(dlsym(lib, "cusolverDnCreate"));
-    s.set_stream = reinterpret_cast<decltype(s.set_stream)>(dlsym(lib, "cusolverDnSetStream"));
-    s.potrf_size = reinterpret_cast<decltype(s.potrf_size)>(dlsym(lib, "cusolverDnSpotrf_bufferSize"));
-    s.potrf = reinterpret_cast<decltype(s.potrf)>(dlsym(lib, "cusolverDnSpotrf"));
-    void* blas = nullptr;
-    for (const char* name : {"libcublas.so.13", "libcublas.so.12", "libcublas.so"}) {
-      blas = dlopen(name, RTLD_NOW | RTLD_LOCAL);
-      if (blas) break;
-    }
-    if (!blas) return;
-    s.blas_create = reinterpret_cast<decltype(s.blas_create)>(dlsym(blas, "cublasCreate_v2"));
-    s.blas_set_stream = reinterpret_cast<decltype(s.blas_set_stream)>(dlsym(blas, "cublasSetStream_v2"));
-    s.trsm = reinterpret_cast<decltype(s.trsm)>(dlsym(blas, "cublasStrsm_v2"));
-    s.ok = s.create && s.set_stream && s.potrf_size && s.potrf && s.blas_create && s.blas_set_stream && s.trsm;
-  });
-  return s;
-}
-
-// one handle of each library per device, created on first use
-cusolverDnHandle_t solver_handle() {
-  static std::mutex mu;
-  static cusolverDnHandle_t handles[64] = {};
-  int dev = 0;
-  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return nullptr;
-  std::lock_guard<std::mutex> lock(mu);
-  if (!handles[dev] && solver().create(&handles[dev]) != CUSOLVER_STATUS_SUCCESS) handles[dev] = nullptr;
-  return handles[dev];
-}
-
-cublasHandle_t blas_handle() {
-  static std::mutex mu;
-  static cublasHandle_t handles[64] = {};
-  int dev = 0;
-  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return nullptr;
-  std::lock_guard<std::mutex> lock(mu);
-  if (!handles[dev] && solver().blas_create(&handles[dev]) != CUBLAS_STATUS_SUCCESS) handles[dev] = nullptr;
-  return handles[dev];
-}
-
-// ---------------------------------------------------------------- factor helpers
-// One block: dead channels, the mean of the diagonal, and the damping added to it.
-__global__ void __launch_bounds__(1024) damp_diagonal_kernel(float* A, int64_t n, float damp, uint8_t* dead) {
-  __shared__ double part[1024];
-  double s = 0.0;
-  for (int64_t j = threadIdx.x; j < n; j += blockDim.x) {
-    float d = A[j * n + j];
-    const bool is_dead = (d == 0.0f);
-    if (is_dead) A[j * n + j] = d = 1.0f;
-    if (dead) dead[j] = (uint8_t)is_dead;
-    s += (double)d;
-  }
-  part[threadIdx.x] = s;
-  __syncthreads();
-  for (int step = 512; step > 0; step >>= 1) {
-    if ((int)threadIdx.x < step) part[threadIdx.x] += part[threadIdx.x + step];
-    __syncthreads();
-  }
-  const float add = (float)((double)damp * part[0] / (double)n);
-  for (int64_t j = threadIdx.x; j < n; j += blockDim.x) A[j * n + j] += add;
-}
-
-// B[i][j] = A[p][q] with (p, q) = (n-1-i, n-1-j) taken in the upper triangle (p <= q) of
-// row-major A: B = J A J, complete and symmetric, from A's upper triangle.
-__global__ void __launch_bounds__(256) reverse_symmetric_kernel(const float* __restrict__ A, int64_t n,
-                                                                float* __restrict__ B) {
-  const int64_t total = n * n;
-  for (int64_t e = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; e < total; e += (int64_t)gridDim.x * blockDim.x) {
-    const int64_t i = e / n, j = e - i * n;
-    const int64_t p = n - 1 - i, q = n - 1 - j;
-    B[e] = p <= q ? A[p * n + q] : A[q * n + p];
-  }
-}
-
-// Reverses the n*n array A in place (A[e] <-> A[n*n - 1 - e]) and zeroes what lands below
-// the diagonal of row-major A.
-__global__ void __launch_bounds__(256) reverse_upper_kernel(float* A, int64_t n) {
-  const int64_t total = n * n, half = total / 2;
-  for (int64_t e = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; e < half; e += (int64_t)gridDim.x * blockDim.x) {
-    const int64_t f = total - 1 - e;
-    const float a = A[e], b = A[f];
-    const int64_t re = e / n, rf = f / n;
-    A[e] = re > e - re * n ? 0.0f : b;
-    A[f] = rf > f - rf * n ? 0.0f : a;
-  }
-}
-
-// the n x n identity
-__global__ void __launch_bounds__(256) identity_kernel(float* X, int64_t n) {
-  const int64_t total = n * n;
-  for (int64_t e = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; e < total; e += (int64_t)gridDim.x * blockDim.x) {
-    const int64_t r = e / n;
-    X[e] = (e - r * n == r) ? 1.0f : 0.0f;
-  }
-}
 
 // ---------------------------------------------------------------- block quantizer
 __device__ __forceinline__ bool better_code(float e, int c, float be, int bc, int c0) {
@@ -339,59 +209,6 @@ __global__ void __launch_bounds__(256) to_fp32_kernel(const uint16_t* __restrict
 }  // namespace
 
 // ---------------------------------------------------------------- host side
-bool gptq_solver_available() { return solver().ok && solver_handle() != nullptr && blas_handle() != nullptr; }
-
-// The factor's workspace in floats: J A J and its Cholesky factor (n*n, rounded up to 64
-// floats), then cuSOLVER's.
-size_t gptq_factor_solver_floats(int64_t n) {
-  if (!gptq_solver_available()) return 0;
-  int a = 0;
-  if (solver().potrf_size(solver_handle(), CUBLAS_FILL_MODE_LOWER, (int)n, nullptr, (int)n, &a) !=
-      CUSOLVER_STATUS_SUCCESS)
-    return 0;
-  return ((size_t)n * (size_t)n + 63) / 64 * 64 + std::max(a, 1);
-}
-
-cudaError_t launch_gptq_factor(const float* H, int64_t n, int64_t ld_h, float damp, float* Uo, uint8_t* dead,
-                               int32_t* info, float* work, size_t work_floats, cudaStream_t stream) {
-  if (!gptq_solver_available()) return cudaErrorNotSupported;
-  const Solver& sv = solver();
-  cusolverDnHandle_t hd = solver_handle();
-  cublasHandle_t hb = blas_handle();
-  if (sv.set_stream(hd, stream) != CUSOLVER_STATUS_SUCCESS || sv.blas_set_stream(hb, stream) != CUBLAS_STATUS_SUCCESS)
-    return cudaErrorUnknown;
-  const size_t x_floats = ((size_t)n * (size_t)n + 63) / 64 * 64;
-  if (work_floats <= x_floats) return cudaErrorInvalidValue;
-  float* X = work;
-  float* solver_work = work + x_floats;
-  cudaError_t err = cudaMemcpy2DAsync(Uo, (size_t)n * 4, H, (size_t)ld_h * 4, (size_t)n * 4, (size_t)n,
-                                      cudaMemcpyDeviceToDevice, stream);
-  if (err != cudaSuccess) return err;
-  damp_diagonal_kernel<<<1, 1024, 0, stream>>>(Uo, n, damp, dead);
-  if ((err = cudaGetLastError()) != cudaSuccess) return err;
-  DeviceInfo dinfo;
-  if ((err = current_device_info(&dinfo)) != cudaSuccess) return err;
-  const unsigned blocks = (unsigned)std::max<int64_t>(1, std::min<int64_t>((n * n + 255) / 256,
-                                                                          (int64_t)dinfo.sm_count * 16));
-  // X = J A J, symmetric, from the upper triangle of the damped copy
-  reverse_symmetric_kernel<<<blocks, 256, 0, stream>>>(Uo, n, X);
-  if ((err = cudaGetLastError()) != cudaSuccess) return err;
-  if ((err = cudaMemsetAsync(info, 0, 3 * sizeof(int32_t), stream)) != cudaSuccess) return err;
-  const int ni = (int)n, lw = (int)std::min<size_t>(work_floats - x_floats, (size_t)INT32_MAX);
-  if (sv.potrf(hd, CUBLAS_FILL_MODE_LOWER, ni, X, ni, solver_work, lw, info) != CUSOLVER_STATUS_SUCCESS)
-    return cudaErrorUnknown;
-  // L^T Y = I: Y = L^-T (upper, column-major) in U's buffer
-  identity_kernel<<<blocks, 256, 0, stream>>>(Uo, n);
-  if ((err = cudaGetLastError()) != cudaSuccess) return err;
-  const float one = 1.0f;
-  if (sv.trsm(hb, CUBLAS_SIDE_LEFT, CUBLAS_FILL_MODE_LOWER, CUBLAS_OP_T, CUBLAS_DIAG_NON_UNIT, ni, ni, &one, X, ni,
-              Uo, ni) != CUBLAS_STATUS_SUCCESS)
-    return cudaErrorUnknown;
-  // reversed, column-major Y is row-major U; the other triangle is cleared
-  reverse_upper_kernel<<<blocks, 256, 0, stream>>>(Uo, n);
-  return cudaGetLastError();
-}
-
 cudaError_t launch_gptq_hscale(const void* w, int64_t m, int64_t n, const float* U, const float* h,
                                const float* global_scale, const uint8_t* dead, int block, int down, int up,
                                uint8_t* codes, uint8_t* packed, float* Wf, float* E, uint16_t* A6, uint16_t* B6,

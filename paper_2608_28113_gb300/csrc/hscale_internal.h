@@ -73,11 +73,12 @@ int64_t hessian_full_ld(int64_t tokens);
 cudaError_t launch_hessian_full(const void* x, int64_t tokens, int64_t n, int64_t ld_x, float* H, int64_t ld_h,
                                 void* xt, cudaStream_t stream);
 
-// Algorithm 3 (GPTQ + H-Scale).  The factor needs cuSOLVER, loaded at run time.
-bool gptq_solver_available();
-size_t gptq_factor_solver_floats(int64_t n);  // 0 if cuSOLVER is unavailable
+// Algorithm 3 (GPTQ + H-Scale).  The factor's workspace (bytes) and the factor itself; U is
+// also used as scratch for the damped copy of H.
+int64_t gptq_factor_padded(int64_t n);
+size_t gptq_factor_workspace(int64_t n);
 cudaError_t launch_gptq_factor(const float* H, int64_t n, int64_t ld_h, float damp, float* U, uint8_t* dead,
-                               int32_t* info, float* work, size_t work_floats, cudaStream_t stream);
+                               int32_t* info, void* workspace, cudaStream_t stream);
 // C[m, nn] (row stride ld_c, fp32) += A B^T on the tensor cores, with A [m, k] and B [nn, k]
 // bf16, rows of k elements contiguous (k % 8 == 0, 16-byte aligned bases); every tile.
 cudaError_t launch_gemm_accumulate(const void* a, const void* b, int64_t m, int64_t nn, int64_t k, float* C,

@@ -219,6 +219,14 @@ def test_gptq_argument_errors(lib):
     assert g(FAKE, 64, 64, -1.0, FAKE, None, FAKE, FAKE, 1 << 20, None) == ERR_ARG
     assert g(FAKE, 64, 64, 0.01, None, None, FAKE, FAKE, 1 << 20, None) == ERR_NULL
     assert g(None, 0, 0, 0.01, None, None, None, None, 0, None) == OK
+    # the factor's workspace: the 128 x 256 fp32 pair [B | X] (n = 64 pads to one block), the
+    # 128 x 128 panel and two 128 x 768 bf16 split operands
+    wsf = lib.hscale_gptq_factor_workspace_bytes
+    assert wsf(64) == 131072 + 65536 + 2 * 196608
+    assert wsf(0) == 0 and wsf(65537) == 0
+    assert g(FAKE, 64, 64, 0.01, FAKE, None, FAKE, FAKE, wsf(64) - 256, None) == ERR_WS
+    assert g(FAKE, 64, 64, 0.01, FAKE, None, FAKE, None, wsf(64), None) == ERR_WS
+    assert g(FAKE, 65537, 65537, 0.01, FAKE, None, FAKE, FAKE, 1 << 20, None) == ERR_SHAPE
     # 4x64 fp32 weights + 4x32 fp32 E + 4x192 and 64x192 bf16 split operands, each rounded to 256 B
     assert lib.hscale_gptq_workspace_bytes(4, 64, 32) == 1024 + 512 + 1536 + 24576
     q = lib.hscale_gptq_hscale
@@ -228,6 +236,16 @@ def test_gptq_argument_errors(lib):
     assert q(FAKE, 4, 64, None, FAKE, FAKE, None, 32, 4, 4, FAKE, FAKE, FAKE, 1 << 20, None) == ERR_NULL
     assert q(FAKE, 4, 64, FAKE, FAKE, FAKE, None, 32, 4, 4, FAKE, FAKE, FAKE, 64, None) == ERR_WS
     assert q(None, 0, 64, None, None, None, None, 32, 4, 4, None, None, None, 0, None) == OK
+
+
+def test_library_sources_load_no_other_library_at_run_time():
+    """Every kernel of the path is the library's own: nothing is looked up with dlopen (the
+    factor of Algorithm 3 no longer calls a solver library)."""
+    csrc = pathlib.Path(hs.__file__).resolve().parent / "csrc"
+    for src in csrc.iterdir():
+        text = src.read_text()
+        for word in ("dlopen", "cusolver", "cublas"):
+            assert word not in text.lower(), (src.name, word)
 
 
 def test_pack_argument_errors(lib):

@@ -3,7 +3,8 @@
 Pass rules:
   * H = X^T X on the tensor cores: |H_gpu - H| <= 1e-5 * sqrt(H_ii H_jj) (bf16 products are
     exact; fp32 accumulation over the tokens).
-  * the factor U (fp32 cuSOLVER Cholesky of a 1 %-damped H): relative Frobenius error
+  * the factor U (the library's blocked fp32 Cholesky of the reversed 1 %-damped H and its
+    triangular inverse, updates on the tensor cores in three-way bf16 splits): relative Frobenius error
     <= 1e-3 against numpy's fp64 factor of the same fp32 H; identical dead channels.
   * the block loop, fed the same fp32 U, h and s_g as the oracle: the first block's codes and
     nibbles bit-exact outside the oracle's near-ties; one block (B = n) and a diagonal U (no
@@ -123,6 +124,36 @@ def test_factor_matches_oracle_with_a_dead_channel():
     assert rel <= 1e-3
 
 
+@pytest.mark.parametrize("n,tokens", [(72, 300), (128, 400), (131, 500), (200, 600), (384, 1200), (1000, 3000)])
+def test_factor_sizes_across_block_boundaries(n, tokens):
+    """Widths below one 128-wide block, exactly one, ragged (padded with an identity block) and
+    several blocks (trailing and inverse updates on the tensor cores)."""
+    x = calib(n, tokens, 700 + n)
+    H32 = oracle_H(x, n).astype(np.float32)
+    U, dead, info = gpu_factor(H32)
+    Uref, dref = oracle.gptq_factor(H32.astype(np.float64))
+    assert np.all(info == 0), info
+    assert np.array_equal(dead, dref)
+    assert np.all(np.tril(U, -1) == 0)
+    rel = np.linalg.norm(U - Uref) / np.linalg.norm(Uref)
+    print(f"[parity] gptq factor n={n}: rel Frobenius err {rel:.2e}")
+    assert rel <= 1e-4
+    assert hs.hscale_device_error_flags() == 0
+
+
+def test_factor_reports_a_matrix_that_is_not_positive_definite():
+    """A symmetric matrix with a negative eigenvalue that the damping does not lift: info[0]
+    names a failed pivot (1-based, in the reversed order); U is then unspecified."""
+    n = 300
+    rng = np.random.default_rng(5)
+    Q, _ = np.linalg.qr(rng.standard_normal((n, n)))
+    ev = np.linspace(1.0, 2.0, n)
+    ev[7] = -50.0
+    H32 = ((Q * ev) @ Q.T).astype(np.float32)
+    U, dead, info = gpu_factor(H32)
+    assert 1 <= info[0] <= n and info[1] == 0 and info[2] == 0
+
+
 def gpu_gptq(w, U32, h32, s_g, block, down, up, dead=None):
     m, n = w.shape
     codes = torch.empty(m, n // 16, dtype=torch.uint8, device=dev())
@@ -188,7 +219,7 @@ def test_gptq_one_block_and_diagonal_factor_reduce_to_the_search():
 
 def test_full_size_gptq_q_proj_slice():
     """A 1024 x 4096 slice of the q_proj layer at full width with the full pipeline on the
-    GPU (H on the tensor cores, cuSOLVER factor, block loop of 128 columns, k = 4) against
+    GPU (H on the tensor cores, the factor, block loop of 128 columns, k = 4) against
     the oracle fed the GPU-independent inputs; output errors of GPTQ + H-Scale, H-Scale and
     RTN are reported."""
     W = wl.WORKLOADS["llama8b-q_proj"]
