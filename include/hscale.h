@@ -143,6 +143,46 @@ int hscale_hessian_diag_accumulate_ex(const void* x_bf16, int64_t tokens, int64_
                                       float* h, uint32_t flags, void* stream);
 
 /*
+ * Rank-order sum of partial Hessian diagonals (Sec. 3.2, Eq. 4, with the calibration tokens
+ * split across ranks: h = sum over the ranks' token shares of sum_t x_tj^2).  The paper has
+ * no counterpart; it is the reduction step of a token-sharded calibration pass.
+ *
+ *   h[j] = (((p_0[j] + p_1[j]) + p_2[j]) + ...) + p_{parts-1}[j]      for j < n
+ *
+ * partials  [parts, ld] fp32 device array, row r = rank r's partial h (its own
+ *           hscale_hessian_diag_accumulate calls into a zeroed vector); ld >= n.
+ * h         [n] fp32, written (not accumulated).  The adds are fp32 round-to-nearest in rank
+ *           order, so every rank that sums the same gathered partials gets the same bits,
+ *           and repeated runs give the same bits; against one rank's pass over every token,
+ *           the result differs only by the order of the additions (relative error of the
+ *           same bound).
+ * parts = 0 or n = 0 is a no-op.
+ */
+int hscale_hessian_sum_partials(const float* partials, int64_t parts, int64_t n, int64_t ld, float* h,
+                                void* stream);
+
+/*
+ * The global amax of W as an integer word, for a global scale over a matrix whose rows are
+ * split across ranks (the paper has no counterpart).  The global scale of Sec. 3.3 needs the
+ * amax of the whole matrix: each rank computes the word of its rows, the ranks take the
+ * maximum of the words (an all-reduce with MAX on a 32-bit integer), and
+ * hscale_global_scale_from_amax turns the result into s_g.
+ *
+ * amax_bits  device uint32, written: the bf16 bit pattern of max|w| over the m x n bf16
+ *            matrix w (16-byte aligned, n % 16 == 0), zero-extended; 0 for an empty or all-zero
+ *            matrix.  Bit patterns of non-negative bf16 values order as the values do, so the
+ *            maximum of the ranks' words is the word of the whole matrix.
+ */
+int hscale_amax_bits(const void* w_bf16, int64_t m, int64_t n, uint32_t* amax_bits, void* stream);
+
+/*
+ * s_g = fl32(amax / (6 * 448)) from an amax word of hscale_amax_bits (1.0 when it is 0):
+ * the global scale hscale_rtn_scales writes for a matrix of that amax, bit for bit.
+ * amax_bits and global_scale are device pointers (4-byte aligned).
+ */
+int hscale_global_scale_from_amax(const uint32_t* amax_bits, float* global_scale, void* stream);
+
+/*
  * Global scale and RTN local-scale codes (Sec. 3.3 "Initialization", Eq. 7).
  *
  *   s_g      = fl32(amax|W| / (6 * 448))          (1.0 when W is all zero)

@@ -24,6 +24,7 @@ __all__ = [
     "HScaleError", "load", "library_path", "hscale_status_string", "hscale_abi_version",
     "hscale_device_error_flags",
     "hscale_hessian_diag_accumulate", "hscale_hessian_diag_accumulate_ex", "HSCALE_HESSIAN_X_READY",
+    "hscale_hessian_sum_partials", "hscale_amax_bits", "hscale_global_scale_from_amax",
     "hscale_rtn_workspace_bytes", "hscale_rtn_scales",
     "hscale_rtn_scales_noalloc",
     "hscale_refine_scales", "hscale_refine_scales_ex", "hscale_refine_scales_4over6",
@@ -48,6 +49,9 @@ _SIGNATURES = {
     "hscale_selftest_bounded_wait": (ctypes.c_int, [ctypes.c_uint32, _P]),
     "hscale_hessian_diag_accumulate": (ctypes.c_int, [_P, _I64, _I64, _I64, _P, _P]),
     "hscale_hessian_diag_accumulate_ex": (ctypes.c_int, [_P, _I64, _I64, _I64, _P, ctypes.c_uint32, _P]),
+    "hscale_hessian_sum_partials": (ctypes.c_int, [_P, _I64, _I64, _I64, _P, _P]),
+    "hscale_amax_bits": (ctypes.c_int, [_P, _I64, _I64, _P, _P]),
+    "hscale_global_scale_from_amax": (ctypes.c_int, [_P, _P, _P]),
     "hscale_rtn_workspace_bytes": (_SZ, []),
     "hscale_rtn_scales": (ctypes.c_int, [_P, _I64, _I64, _P, _P, _P, _SZ, _P]),
     "hscale_rtn_scales_noalloc": (ctypes.c_int, [_P, _I64, _I64, _P, _P, _P]),
@@ -167,6 +171,40 @@ def hscale_hessian_diag_accumulate_ex(x: torch.Tensor, h: torch.Tensor, flags: i
            load().hscale_hessian_diag_accumulate_ex(_ptr(x), tokens, n, ld, _ptr(h), int(flags),
                                                     _stream_ptr(stream)))
     return h
+
+
+def hscale_hessian_sum_partials(partials: torch.Tensor, h: torch.Tensor, stream=None) -> torch.Tensor:
+    """h = rank-order fp32 sum of the rows of partials [parts, n] (each a rank's partial h)."""
+    _need(partials, torch.float32, "partials")
+    _need(h, torch.float32, "h")
+    if partials.dim() != 2 or partials.stride(1) != 1:
+        raise ValueError("partials must be 2-D [parts, n] with unit column stride")
+    parts, n = partials.shape
+    if h.numel() != n or not h.is_contiguous():
+        raise ValueError("h must be a contiguous float32 vector of length n")
+    ld = partials.stride(0) if parts > 1 else n
+    _check("hscale_hessian_sum_partials",
+           load().hscale_hessian_sum_partials(_ptr(partials), parts, n, ld, _ptr(h), _stream_ptr(stream)))
+    return h
+
+
+def hscale_amax_bits(w: torch.Tensor, amax_bits: torch.Tensor, stream=None) -> torch.Tensor:
+    """amax_bits (int32 [1], device) = bf16 bit pattern of max|W| (for an all-reduce MAX)."""
+    _need(w, torch.bfloat16, "w")
+    _need(amax_bits, torch.int32, "amax_bits")
+    if not w.is_contiguous() or w.dim() != 2:
+        raise ValueError("w must be a contiguous 2-D tensor")
+    m, n = w.shape
+    _check("hscale_amax_bits", load().hscale_amax_bits(_ptr(w), m, n, _ptr(amax_bits), _stream_ptr(stream)))
+    return amax_bits
+
+
+def hscale_global_scale_from_amax(amax_bits: torch.Tensor, global_scale: torch.Tensor, stream=None) -> None:
+    """global_scale[0] = s_g of a matrix whose amax word is amax_bits[0]."""
+    _need(amax_bits, torch.int32, "amax_bits")
+    _need(global_scale, torch.float32, "global_scale")
+    _check("hscale_global_scale_from_amax",
+           load().hscale_global_scale_from_amax(_ptr(amax_bits), _ptr(global_scale), _stream_ptr(stream)))
 
 
 def hscale_rtn_workspace_bytes() -> int:

@@ -69,7 +69,7 @@ const char* hscale_status_string(int status) {
   }
 }
 
-int hscale_abi_version(void) { return 2; }
+int hscale_abi_version(void) { return 3; }
 
 int hscale_device_error_flags(uint32_t* flags) {
   if (flags == nullptr) return HSCALE_ERR_NULL;
@@ -103,6 +103,34 @@ int hscale_hessian_diag_accumulate_ex(const void* x_bf16, int64_t tokens, int64_
   if (tokens > INT32_MAX || tokens > INT64_MAX / ld_x) return HSCALE_ERR_SHAPE;
   return from_cuda(hscale::launch_hessian(x_bf16, tokens, n, ld_x, h, (flags & HSCALE_HESSIAN_X_READY) != 0,
                                           as_stream(stream)));
+}
+
+int hscale_hessian_sum_partials(const float* partials, int64_t parts, int64_t n, int64_t ld, float* h,
+                                void* stream) {
+  if (parts < 0 || n < 0 || (parts > 0 && ld < n)) return HSCALE_ERR_SHAPE;
+  if (parts == 0 || n == 0) return HSCALE_OK;
+  if (parts > 1 && ld > INT64_MAX / parts) return HSCALE_ERR_SHAPE;
+  if (partials == nullptr || h == nullptr) return HSCALE_ERR_NULL;
+  if (!aligned(partials, 4) || !aligned(h, 4)) return HSCALE_ERR_ALIGN;
+  return from_cuda(hscale::launch_sum_partials(partials, parts, n, ld, h, as_stream(stream)));
+}
+
+int hscale_amax_bits(const void* w_bf16, int64_t m, int64_t n, uint32_t* amax_bits, void* stream) {
+  int st = check_weight(w_bf16, m, n);
+  if (st != HSCALE_OK) return st;
+  if (amax_bits == nullptr) return HSCALE_ERR_NULL;
+  if (!aligned(amax_bits, 4)) return HSCALE_ERR_ALIGN;
+  cudaStream_t s = as_stream(stream);
+  // an empty matrix has amax 0: the word is cleared either way
+  if (cudaMemsetAsync(amax_bits, 0, sizeof(uint32_t), s) != cudaSuccess) return HSCALE_ERR_CUDA;
+  if (m == 0 || n == 0) return HSCALE_OK;
+  return from_cuda(hscale::launch_amax(w_bf16, m * n, amax_bits, s));
+}
+
+int hscale_global_scale_from_amax(const uint32_t* amax_bits, float* global_scale, void* stream) {
+  if (amax_bits == nullptr || global_scale == nullptr) return HSCALE_ERR_NULL;
+  if (!aligned(amax_bits, 4) || !aligned(global_scale, 4)) return HSCALE_ERR_ALIGN;
+  return from_cuda(hscale::launch_rtn_codes(nullptr, 0, 16, amax_bits, global_scale, nullptr, as_stream(stream)));
 }
 
 size_t hscale_rtn_workspace_bytes(void) { return 256; }

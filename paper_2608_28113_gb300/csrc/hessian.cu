@@ -280,6 +280,29 @@ cudaError_t launch_hessian(const void* x, int64_t tokens, int64_t n, int64_t ld_
   }
 }
 
+// h[j] = (((p_0[j] + p_1[j]) + p_2[j]) + ...) + p_{parts-1}[j]: the partial sums of the ranks
+// that each took a share of the calibration tokens, added in rank order with fp32 round-to-
+// nearest adds, so every rank that runs this on the gathered partials gets the same bits.
+__global__ void __launch_bounds__(256) sum_partials_kernel(const float* __restrict__ partials, int64_t parts,
+                                                           int64_t n, int64_t ld, float* __restrict__ h) {
+  const int64_t stride = (int64_t)gridDim.x * blockDim.x;
+  for (int64_t j = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; j < n; j += stride) {
+    float s = partials[j];
+    for (int64_t r = 1; r < parts; ++r) s = __fadd_rn(s, partials[r * ld + j]);
+    h[j] = s;
+  }
+}
+
+cudaError_t launch_sum_partials(const float* partials, int64_t parts, int64_t n, int64_t ld, float* h,
+                                cudaStream_t stream) {
+  DeviceInfo info;
+  cudaError_t err = current_device_info(&info);
+  if (err != cudaSuccess) return err;
+  const int64_t blocks = std::max<int64_t>(1, std::min<int64_t>((n + 255) / 256, (int64_t)info.sm_count * 8));
+  sum_partials_kernel<<<(unsigned)blocks, 256, 0, stream>>>(partials, parts, n, ld, h);
+  return cudaGetLastError();
+}
+
 cudaError_t ensure_dynamic_smem(const void* func, int bytes) {
   static std::mutex mu;
   static const void* done_func[256];

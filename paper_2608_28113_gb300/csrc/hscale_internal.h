@@ -21,6 +21,10 @@ cudaError_t current_device_info(DeviceInfo* out);
 cudaError_t launch_hessian(const void* x, int64_t tokens, int64_t n, int64_t ld_x, float* h, bool x_ready,
                            cudaStream_t stream);
 
+// h[j] = sum of the parts' partial sums p_r[j] (row r at partials + r * ld) in rank order.
+cudaError_t launch_sum_partials(const float* partials, int64_t parts, int64_t n, int64_t ld, float* h,
+                                cudaStream_t stream);
+
 // amax over W into *amax_bits (16-bit |bf16| pattern, zero-extended); *amax_bits must be 0.
 cudaError_t launch_amax(const void* w, int64_t count, uint32_t* amax_bits, cudaStream_t stream);
 

@@ -41,7 +41,7 @@ def test_header_declares_the_boundary():
 def test_library_exports_every_declared_symbol(lib):
     for name in declared_functions():
         assert hasattr(lib, name), name
-    assert hs.hscale_abi_version() == 2
+    assert hs.hscale_abi_version() == 3
     assert hs.library_path().exists()
 
 
@@ -103,6 +103,24 @@ def test_hessian_argument_errors(lib):
     assert fx(None, 4, 64, 64, FAKE, hs.HSCALE_HESSIAN_X_READY, None) == ERR_NULL
     assert fx(FAKE, 4, 60, 64, FAKE, hs.HSCALE_HESSIAN_X_READY, None) == ERR_SHAPE
     assert fx(FAKE, 0, 64, 64, FAKE, hs.HSCALE_HESSIAN_X_READY, None) == OK
+
+
+def test_sharding_entry_point_argument_errors(lib):
+    f = lib.hscale_hessian_sum_partials
+    assert f(FAKE, 2, 64, 32, FAKE, None) == ERR_SHAPE        # ld < n
+    assert f(FAKE, -1, 64, 64, FAKE, None) == ERR_SHAPE
+    assert f(None, 2, 64, 64, FAKE, None) == ERR_NULL
+    assert f(FAKE, 2, 64, 64, None, None) == ERR_NULL
+    assert f(MIS, 2, 64, 64, FAKE, None) == ERR_ALIGN
+    assert f(None, 0, 64, 64, None, None) == OK               # no parts: no-op
+    g = lib.hscale_amax_bits
+    assert g(FAKE, 4, 24, FAKE, None) == ERR_SHAPE            # n % 16
+    assert g(FAKE, 4, 32, None, None) == ERR_NULL
+    assert g(MIS, 4, 32, FAKE, None) == ERR_ALIGN
+    assert g(FAKE, 4, 32, MIS, None) == ERR_ALIGN
+    q = lib.hscale_global_scale_from_amax
+    assert q(None, FAKE, None) == ERR_NULL and q(FAKE, None, None) == ERR_NULL
+    assert q(MIS, FAKE, None) == ERR_ALIGN
 
 
 def test_rtn_argument_errors(lib):
