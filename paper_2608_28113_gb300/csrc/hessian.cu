@@ -4,9 +4,10 @@
 //
 // Layout of the work
 //   * A CTA owns a 64-channel column tile (128 bytes of every row) and a contiguous
-//     run of tokens.  One thread streams the run into a ring of shared-memory stages
-//     with 2-D TMA tensor loads (64 channels x 128 rows = 16 KB per stage, 4 stages in
-//     flight per CTA, L2 evict-first); the CTA's 256 threads (32 row phases x 8
+//     run of tokens.  A producer warp (one thread) streams the run into a ring of
+//     shared-memory stages with 2-D TMA tensor loads (64 channels x 128 rows = 16 KB per
+//     stage, 4 stages in flight per CTA, L2 evict-first), refilling each stage as soon as
+//     the consumers release it; the CTA's 256 consumer threads (32 row phases x 8
 //     16-byte vectors) read each stage back with conflict-free 128-bit shared loads
 //     and accumulate in fp32.  mbarriers order the ring; every wait is bounded.
 //   * The token range of a tile is split over the CTAs of one thread-block cluster
@@ -50,9 +51,9 @@ __device__ uint32_t g_device_error = 0;
 namespace {
 
 constexpr int kTileCols = 64;                       // channels per CTA tile (128 bytes)
-constexpr int kThreads = 256;
+constexpr int kWarps = 8;                           // consumer warps
+constexpr int kThreads = (kWarps + 1) * 32;         // and one producer warp
 constexpr int kPhases = 32;                         // rows read side by side
-constexpr int kWarps = kThreads / 32;
 constexpr int kStageRows = 128;
 constexpr int kStages = 4;
 constexpr uint32_t kStageBytes = kStageRows * kTileCols * 2;
@@ -98,8 +99,6 @@ hessian_colsumsq_kernel(const __grid_constant__ CUtensorMap xmap, int64_t row0, 
   const int nst = r1 > r0 ? (int)((r1 - r0 + kStageRows - 1) / kStageRows) : 0;
   const int x0 = blockIdx.y * kTileCols;
 
-  uint64_t policy = 0;
-  int issued = 0;
   if (tid == 0) {
     prefetch_tensormap(&xmap);
     for (int s = 0; s < kStages; ++s) {
@@ -113,50 +112,52 @@ hessian_colsumsq_kernel(const __grid_constant__ CUtensorMap xmap, int64_t row0, 
   // X may still be being written by the previous kernel on the stream: read it only once
   // that kernel has finished and its writes are visible
   if (!x_ready) pdl_wait_primary();
-  if (tid == 0) {
-    policy = l2_evict_first_policy();
-    for (; issued < kStages && issued < nst; ++issued) {
-      mbar_arrive_expect_tx(&full_bar[issued], kStageBytes);
-      tma_load_2d(ring + (size_t)issued * kStageBytes, &xmap, x0, (int32_t)(r0 + issued * kStageRows),
-                  &full_bar[issued], policy);
-    }
-  }
   pdl_launch_dependents();
 
   float acc[8] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};
-  int waited = 0;  // tid 0: stages whose full barrier it has seen complete
-  for (int i = 0; i < nst; ++i) {
-    const int s = i % kStages;
-    const uint32_t par = (uint32_t)(i / kStages) & 1u;
-    bool ok = !*(volatile int*)&s_bad;
-    if (ok && !mbar_wait(&full_bar[s], par)) {
-      ok = false;
-      s_bad = 1;
-    }
-    if (ok) {
-      if (tid == 0) waited = i + 1;
-      const uint8_t* st = ring + (size_t)s * kStageBytes + p * 128 + v * 16;
-#pragma unroll
-      for (int rr = 0; rr < kStageRows / kPhases; ++rr)
-        accum_sq8(acc, *reinterpret_cast<const uint4*>(st + rr * kPhases * 128));
-    }
-    __syncwarp();
-    if (lane == 0) mbar_arrive(&empty_bar[s]);
-    if (tid == 0 && issued < nst && issued == i + kStages) {
-      if (!*(volatile int*)&s_bad && mbar_wait(&empty_bar[s], par)) {
+  if (warp == kWarps) {
+    // producer: one thread refills each stage as soon as the consumers have released it, so
+    // a consumer warp that is slow to be scheduled delays no other stage's load
+    if (lane == 0) {
+      const uint64_t policy = l2_evict_first_policy();
+      int issued = 0;
+      for (; issued < nst; ++issued) {
+        const int s = issued % kStages;
+        if (issued >= kStages &&
+            (*(volatile int*)&s_bad || !mbar_wait(&empty_bar[s], (uint32_t)(issued / kStages - 1) & 1u))) {
+          s_bad = 1;
+          break;
+        }
         mbar_arrive_expect_tx(&full_bar[s], kStageBytes);
-        tma_load_2d(ring + (size_t)s * kStageBytes, &xmap, x0, (int32_t)(r0 + issued * kStageRows),
-                    &full_bar[s], policy);
-        ++issued;
-      } else {
-        s_bad = 1;
+        tma_load_2d(ring + (size_t)s * kStageBytes, &xmap, x0, (int32_t)(r0 + issued * kStageRows), &full_bar[s],
+                    policy);
+      }
+      if (*(volatile int*)&s_bad) {
+        // let the copies still in flight land before the CTA's shared memory goes away (the
+        // loads of earlier uses of a stage completed before the stage was refilled)
+        for (int j = issued > kStages ? issued - kStages : 0; j < issued; ++j)
+          mbar_wait(&full_bar[j % kStages], (uint32_t)(j / kStages) & 1u);
+        atomicOr(&g_device_error, kErrMbarTimeout);
       }
     }
-  }
-  if (tid == 0 && s_bad) {
-    // let copies still in flight land before the CTA's shared memory goes away
-    for (int j = waited; j < issued; ++j) mbar_wait(&full_bar[j % kStages], (uint32_t)(j / kStages) & 1u);
-    atomicOr(&g_device_error, kErrMbarTimeout);
+  } else {
+    for (int i = 0; i < nst; ++i) {
+      const int s = i % kStages;
+      const uint32_t par = (uint32_t)(i / kStages) & 1u;
+      bool ok = !*(volatile int*)&s_bad;
+      if (ok && !mbar_wait(&full_bar[s], par)) {
+        ok = false;
+        s_bad = 1;
+      }
+      if (ok) {
+        const uint8_t* st = ring + (size_t)s * kStageBytes + p * 128 + v * 16;
+#pragma unroll
+        for (int rr = 0; rr < kStageRows / kPhases; ++rr)
+          accum_sq8(acc, *reinterpret_cast<const uint4*>(st + rr * kPhases * 128));
+      }
+      __syncwarp();
+      if (lane == 0) mbar_arrive(&empty_bar[s]);
+    }
   }
 
   // phases 4w..4w+3 of a warp: lane bit 3 is phase bit 0, lane bit 4 is phase bit 1
@@ -167,7 +168,7 @@ hessian_colsumsq_kernel(const __grid_constant__ CUtensorMap xmap, int64_t row0, 
     t = __fadd_rn(t, __shfl_xor_sync(0xFFFFFFFFu, t, 16));
     acc[k] = t;
   }
-  if (lane < 8) {
+  if (lane < 8 && warp < kWarps) {
 #pragma unroll
     for (int k = 0; k < 8; ++k) warp_part[warp][lane * 8 + k] = acc[k];
   }
