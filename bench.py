@@ -147,32 +147,35 @@ def measured_peaks():
 
 def step_traffic(work) -> float | None:
     """DRAM bytes per Hessian launch of the step (the mean over its launches), from the
-    committed ncu summary of the workload: one figure per launch shape (chunk tokens,
-    channels).  None when the kernel's sources changed since that capture, or a launch
-    shape of the step was not captured."""
+    committed ncu summaries (profiles/hessian_colsumsq_*.traffic.json): one figure per
+    launch shape (chunk tokens, channels), taken from any summary whose kernel sources hash
+    to the current ones.  None when no such summary covers every launch shape of the step."""
+    import glob
     import hashlib
-    path = os.path.join(ROOT, "profiles", f"hessian_colsumsq_{work.W.name}.traffic.json")
-    try:
-        with open(path) as f:
-            d = json.load(f)
-        h = hashlib.sha256()
-        for src in d["kernel_sources"]:
-            with open(os.path.join(ROOT, src), "rb") as f:
-                h.update(f.read())
-        if h.hexdigest() != d["kernel_sources_sha256"]:
-            return None
-        per_shape = {(int(e["chunk_tokens"]), int(e["n"])): float(e["dram_bytes_per_launch"]) for e in d["shapes"]}
-        total, launches = 0.0, 0
-        for S, c0, c1 in work.pieces:
-            for t0, t1 in hessian_calls(S, c0, c1):
-                key = (t1 - t0, c1 - c0)
-                if key not in per_shape:
-                    return None
-                total += per_shape[key]
-                launches += 1
-        return total / launches if launches else None
-    except Exception:
-        return None
+    per_shape = {}
+    for path in sorted(glob.glob(os.path.join(ROOT, "profiles", "hessian_colsumsq_*.traffic.json"))):
+        try:
+            with open(path) as f:
+                d = json.load(f)
+            h = hashlib.sha256()
+            for src in d["kernel_sources"]:
+                with open(os.path.join(ROOT, src), "rb") as f:
+                    h.update(f.read())
+            if h.hexdigest() != d["kernel_sources_sha256"]:
+                continue
+            for e in d["shapes"]:
+                per_shape[(int(e["chunk_tokens"]), int(e["n"]))] = float(e["dram_bytes_per_launch"])
+        except Exception:
+            continue
+    total, launches = 0.0, 0
+    for S, c0, c1 in work.pieces:
+        for t0, t1 in hessian_calls(S, c0, c1):
+            key = (t1 - t0, c1 - c0)
+            if key not in per_shape:
+                return None
+            total += per_shape[key]
+            launches += 1
+    return total / launches if launches else None
 
 
 class ClockSampler:
