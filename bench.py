@@ -77,14 +77,12 @@ def parse():
                    help="resident search CTAs per SM while the next input space's Hessian pass "
                         "runs alongside (0: run every search after the last Hessian pass; -1, the "
                         "default: when the step's estimated search time exceeds its Hessian time, 7 "
-                        "(every CTA the search kernel keeps resident) with pipelined steps and 5 "
-                        "without; else 4)")
+                        "(every CTA the search kernel keeps resident); else 4)")
     p.add_argument("--pipeline", choices=["auto", "on", "off"], default="auto",
                    help="run each step's last searches alongside the next step's first Hessian pass "
-                        "(h, s_g and initial codes double-buffered).  auto (default): on when the step "
-                        "has several input spaces or its searches outweigh its Hessian passes (decoder "
-                        "layer -4 %%, 70B MLP block -11 %% per step); off for one Hessian-bound input "
-                        "space (q_proj: -1.5 %% per step, while the Hessian pass shares its SMs)")
+                        "(h, s_g and initial codes double-buffered).  auto (default) and on: pipelined "
+                        "(decoder layer -4 %%, 70B MLP block -9 %%, q_proj -8 %% per step); off: each "
+                        "step ends when its last searches do")
     p.add_argument("--no-cpu-baseline", action="store_true")
     p.add_argument("--cpu-baseline", choices=["full", "sample"], default="full",
                    help="full (default): the oracle over the step's whole layer on all host cores, "
@@ -333,26 +331,23 @@ class Work:
         return sum(j[2] for j in jobs) > sum(j[1] for j in jobs)
 
     def pipelined(self, requested: str) -> bool:
-        """Whether consecutive steps overlap: as requested, or by default when the step has
-        several input spaces or is search-bound (there the last searches are a large
-        part of the step; with one Hessian-bound space they are not, and the Hessian pass
-        would share its SMs for a gain of about 1.5 %)."""
-        if requested != "auto":
-            return requested == "on"
-        return len(self.spaces) > 1 or self.search_bound()
+        """Whether consecutive steps overlap: unless asked not to.  With the Hessian pass's
+        squares on the tensor cores it shares its SMs with the searches well enough that
+        overlapping pays on every workload measured (1 GB300): decoder layer 1.217 against
+        1.271 ms per step, 70B MLP block 1.866 against 2.057 ms, q_proj 0.318 against
+        0.345 ms."""
+        return requested != "off"
 
     def overlap_ctas(self, requested: int, pipelined: bool) -> int:
         """Search CTAs per SM alongside a Hessian pass: the requested number, or by default
-        4 when the Hessian passes outweigh the searches (8B decoder layer: 1.31 ms, against
-        1.34 at 3 and 1.44 at 5).  When the searches outweigh them they should take more of
-        the SM: 7, every CTA the search kernel keeps resident, with pipelined steps (70B MLP
-        block: 2.14 ms, against 2.19 at 6 and 2.29 at 5), and 5 without (2.39 ms, against
-        2.54 at 4).  The launcher clamps a larger number to the kernel's occupancy."""
+        4 when the Hessian passes outweigh the searches (decoder layer, pipelined: 1.217 ms,
+        against 1.252 at 3 and 1.224 at 5; q_proj 0.318 ms).  When the searches outweigh
+        them they take 7, every CTA the search kernel keeps resident (70B MLP block: 1.866 ms
+        pipelined, against 1.995 at 6 and 2.089 at 5; 2.057 ms at 7 without pipelining,
+        2.084 at 5).  The launcher clamps a larger number to the kernel's occupancy."""
         if requested >= 0:
             return requested
-        if not self.search_bound():
-            return 4
-        return 7 if pipelined else 5
+        return 7 if self.search_bound() else 4
 
     def space_order(self):
         """The input spaces in the order the step takes them.  Each space is a two-stage

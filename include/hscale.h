@@ -113,9 +113,11 @@ int hscale_selftest_bounded_wait(uint32_t polls, void* stream);
  * h      [n] fp32, read and written (accumulated in place).  Zero it before the first
  *        chunk; streaming a calibration set is one call per chunk on the same h.
  * n      multiple of 8; ld_x >= n and a multiple of 8.
- * Arithmetic: x^2 is exact in fp32; sums are fp32 in a fixed order (per-thread runs of
- * at most 1024 tokens, then fixed-order trees inside the CTA and across a thread-block
- * cluster), so each call adds a relative error of at most about 1100 * 2^-24 to h.
+ * Arithmetic: x^2 is exact in fp32; the squares are summed on the tensor cores in fp32
+ * over runs of 1024 tokens (their accumulation is measured low by about 0.9 units in the
+ * last place per 16 tokens, so about 2^-18 relative per run at most), then the runs'
+ * sums and a thread-block cluster's partial sums meet in fp32 round-to-nearest adds in
+ * a fixed order.  Every run of a call gives the same bits.
  * Nothing else is touched: the call needs no workspace.  The call's kernel is launched
  * with programmatic dependent launch; it waits for the kernel before it on the stream
  * to finish (and for its writes to be visible) before it reads X, so X may be the output

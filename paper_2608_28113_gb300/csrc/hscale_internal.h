@@ -54,9 +54,10 @@ using EncodeTiledFn = CUresult (*)(CUtensorMap*, CUtensorMapDataType, cuuint32_t
                                    CUtensorMapL2promotion, CUtensorMapFloatOOBfill);
 cudaError_t encode_tiled_fn(EncodeTiledFn* out);
 
-// cudaFuncAttributeMaxDynamicSharedMemorySize = bytes for kernel `func` on the current
-// device, set once per (kernel, device) and remembered, so that every GPU of a process
-// gets it (a function attribute belongs to one device's context).
+// cudaFuncAttributeMaxDynamicSharedMemorySize = bytes and the maximum shared-memory
+// carveout for kernel `func` on the current device, set once per (kernel, device) and
+// remembered, so that every GPU of a process gets it (a function attribute belongs to one
+// device's context).
 cudaError_t ensure_dynamic_smem(const void* func, int bytes);
 
 // dW = W - W_hat of packed NVFP4 weights as a bf16 pair [hi | lo] per row, rows of ld

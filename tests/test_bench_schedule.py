@@ -62,11 +62,11 @@ def fake_work(spaces, mats, win=(4, 4)):
 
 
 def test_pipelining_and_overlap_policies():
-    # one Hessian-bound input space (q_proj): sequential steps, 4 search CTAs alongside
+    # one Hessian-bound input space (q_proj): pipelined unless asked not to, 4 search CTAs
     q = fake_work({"x": (262144, 4096)}, [(4096 * 4096 // 16, "x")])
     assert not q.search_bound()
-    assert not q.pipelined("auto") and q.pipelined("on") and not q.pipelined("off")
-    assert q.overlap_ctas(-1, False) == 4 and q.overlap_ctas(2, False) == 2
+    assert q.pipelined("auto") and q.pipelined("on") and not q.pipelined("off")
+    assert q.overlap_ctas(-1, True) == 4 and q.overlap_ctas(-1, False) == 4 and q.overlap_ctas(2, False) == 2
     # several input spaces (decoder layer): pipelined
     dec = fake_work({"qkv": (131072, 4096), "o": (131072, 4096), "mlp": (131072, 4096),
                      "down": (131072, 14336)},
@@ -75,10 +75,10 @@ def test_pipelining_and_overlap_policies():
     assert not dec.search_bound() and dec.pipelined("auto") and dec.overlap_ctas(-1, True) == 4
     assert not dec.pipelined("off")
     # one input space but search-bound (a wide window over a large matrix): pipelined, the
-    # searches fill the SMs (5 CTAs per SM when not pipelined)
+    # searches fill the SMs
     wide = fake_work({"x": (65536, 8192)}, [(28672 * 8192 // 16, "x")] * 2, win=(16, 16))
     assert wide.search_bound() and wide.pipelined("auto")
-    assert wide.overlap_ctas(-1, True) == 7 and wide.overlap_ctas(-1, False) == 5
+    assert wide.overlap_ctas(-1, True) == 7 and wide.overlap_ctas(-1, False) == 7
 
 
 @pytest.mark.gpu
