@@ -579,13 +579,17 @@ def timed(fn, reps, flush=None):
     `flush` (two device buffers, each larger than L2), each call is timed on its own after
     the first buffer is rewritten and the second read, outside the timed window, so inputs
     smaller than L2 (a weight matrix) are read from HBM every time, and the flush's dirty
-    lines have been written back before the call starts."""
+    lines have been written back before the call starts.  The start event follows a short
+    device-side spin (about 50 us), queued before the host makes the call, so the window
+    holds the call's kernels and not the host's time to enqueue them."""
     fn()
     if flush is not None:
         total = 0.0
         for _ in range(reps):
             flush[0].fill_(1.0)
             flush[1].sum()
+            torch.cuda.synchronize()
+            torch.cuda._sleep(SPIN_CYCLES)
             e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
             e0.record()
             fn()
@@ -593,6 +597,8 @@ def timed(fn, reps, flush=None):
             torch.cuda.synchronize()
             total += e0.elapsed_time(e1)
         return total / reps
+    torch.cuda.synchronize()
+    torch.cuda._sleep(SPIN_CYCLES)
     e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
     e0.record()
     for _ in range(reps):
@@ -600,6 +606,10 @@ def timed(fn, reps, flush=None):
     e1.record()
     torch.cuda.synchronize()
     return e0.elapsed_time(e1) / reps
+
+
+# device-side spin before a timed window: ~50 us at 2 GHz, longer than one host call
+SPIN_CYCLES = 100_000
 
 
 # ------------------------------------------------------------------ CPU oracle baseline
