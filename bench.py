@@ -1067,14 +1067,14 @@ def measure_workload(hs, d: Dist, args, W: wl.Workload, win, dev, overlap_ctas: 
     # ---- roofline of the search (its own window, W read from HBM after an L2 flush)
     if main["bound"] == "alu":
         ops = 80.0 * main["candidates"] * work.groups
-        search_roof = {"bound": "alu", "kernel": "refine_kernel", "achieved": ops / (main["ms"] * 1e-3) / 1e12,
+        search_roof = {"bound": "alu", "kernel": "refine_linear_kernel", "achieved": ops / (main["ms"] * 1e-3) / 1e12,
                        "peak": fp32_peak / 1e12, "unit": "Tops/s", "frac": main["frac"],
                        "peak_kind": "SMs x 128 fp32 lanes x max SM clock; 5 lane operations per element "
                                     "and candidate", "candidates": main["candidates"], "traffic": None,
                        "ops_per_launch": ops / len(work.mats), "ms_per_launch": main["ms"] / len(work.mats)}
     else:
         b = SEARCH_BYTES[work.init] * work.groups
-        search_roof = {"bound": "hbm", "kernel": "refine_kernel", "achieved": b / (main["ms"] * 1e-3) / 1e9,
+        search_roof = {"bound": "hbm", "kernel": "refine_linear_kernel", "achieved": b / (main["ms"] * 1e-3) / 1e9,
                        "peak": hbm_peak, "unit": "GB/s", "frac": b / (main["ms"] * 1e-3) / 1e9 / hbm_peak,
                        "peak_kind": f"{peak_kind} HBM copy bandwidth", "candidates": main["candidates"],
                        "traffic": None, "bytes_per_launch": b / len(work.mats),
