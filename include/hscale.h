@@ -422,7 +422,15 @@ int hscale_output_error(const void* x_bf16, int64_t tokens, int64_t n, int64_t l
  *    accuracy (on the tensor cores: three-way bf16 splits of E and U, the six products
  *    above 2^-24 relative, fp32 accumulation).  Writes codes_out [m, n/16] and packed_out
  *    [m, n/2] (8-byte aligned) as hscale_refine_scales does.  The workspace
- *    (hscale_gptq_workspace_bytes) holds the running weights, E and the split operands.
+ *    (hscale_gptq_workspace_bytes) holds the running weights, E and two buffers of each
+ *    split operand.  With more than one block the call works ahead: the update of the
+ *    next block's columns runs on `stream` and the rest of each update on a second stream
+ *    of the library, alongside the next block's quantization; events order the two, every
+ *    weight receives its updates in block order (the same bits on every run), and the
+ *    call's work on `stream` ends after all of it.  The library creates that stream and
+ *    its events on the first such call in each device context and keeps them; a first
+ *    call made while `stream` is being captured (which may not create them) runs every
+ *    block on `stream` instead, with the same results.  Calls are enqueued one at a time.
  */
 size_t hscale_hessian_full_workspace_bytes(int64_t tokens, int64_t n);
 int hscale_hessian_full_accumulate(const void* x_bf16, int64_t tokens, int64_t n, int64_t ld_x, float* H,

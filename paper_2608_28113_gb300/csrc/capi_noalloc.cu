@@ -16,22 +16,15 @@
 #include "../../include/hscale.h"
 #include "hscale_internal.h"
 
-namespace {
-
-// The fixed scratch of hscale_rtn_scales_noalloc (HSCALE_NOALLOC_SCRATCH_BYTES bytes per
-// GPU).  Host code must not pass this name to a kernel: on the host it is only a stand-in
-// for the symbol, so its device address is looked up once per device below.
-static __device__ __align__(256) uint8_t g_noalloc_scratch[HSCALE_NOALLOC_SCRATCH_BYTES];
-
-constexpr int kMaxDevices = 64;
-
-using CtxGetCurrentFn = CUresult (*)(CUcontext*);
-using CtxGetIdFn = CUresult (*)(CUcontext, unsigned long long*);
+namespace hscale {
 
 // Unique id of the calling thread's current context, or 0 when it has none yet.  A
 // context destroyed and created again (cudaDeviceReset) gets a new id; its module, and
-// with it the array, may then sit at another address.
+// with it the array below, may then sit at another address, and its streams and events
+// are gone.
 cudaError_t current_context_id(unsigned long long* id) {
+  using CtxGetCurrentFn = CUresult (*)(CUcontext*);
+  using CtxGetIdFn = CUresult (*)(CUcontext, unsigned long long*);
   static std::once_flag once;
   static CtxGetCurrentFn get_current = nullptr;
   static CtxGetIdFn get_id = nullptr;
@@ -53,6 +46,19 @@ cudaError_t current_context_id(unsigned long long* id) {
   if (ctx == nullptr) return cudaSuccess;
   return get_id(ctx, id) == CUDA_SUCCESS ? cudaSuccess : cudaErrorDeviceUninitialized;
 }
+
+}  // namespace hscale
+
+namespace {
+
+using hscale::current_context_id;
+
+// The fixed scratch of hscale_rtn_scales_noalloc (HSCALE_NOALLOC_SCRATCH_BYTES bytes per
+// GPU).  Host code must not pass this name to a kernel: on the host it is only a stand-in
+// for the symbol, so its device address is looked up once per device below.
+static __device__ __align__(256) uint8_t g_noalloc_scratch[HSCALE_NOALLOC_SCRATCH_BYTES];
+
+constexpr int kMaxDevices = 64;
 
 // Device address of g_noalloc_scratch in the current device's context, resolved on the
 // first call in that context (with that device current) and cached per device together

@@ -209,6 +209,67 @@ __global__ void __launch_bounds__(256) to_fp32_kernel(const uint16_t* __restrict
 }  // namespace
 
 // ---------------------------------------------------------------- host side
+namespace {
+
+// ---------------------------------------------------------------- the look-ahead stream
+// The block loop runs most of each block's update on a second stream, alongside the next
+// block's quantization.  The stream and its events are created once per device context
+// and reused; a mutex keeps calls from enqueuing at the same time, so one call's events
+// are never re-recorded while another call still has waits to enqueue on them.
+constexpr int kLookEvents = 10;
+struct LookAhead {
+  cudaStream_t side = nullptr;
+  cudaEvent_t ev[kLookEvents] = {};
+  unsigned long long ctx = 0;
+};
+constexpr int kMaxLookDevices = 64;
+std::mutex g_look_mu;
+LookAhead g_look[kMaxLookDevices];
+
+// The current device's stream and events (caller holds g_look_mu).  nullptr in *out when
+// they do not exist yet and `stream` is being captured: creating them then is not allowed,
+// and the caller takes the one-stream loop.
+cudaError_t look_ahead(cudaStream_t stream, LookAhead** out) {
+  *out = nullptr;
+  int dev = 0;
+  cudaError_t err = cudaGetDevice(&dev);
+  if (err != cudaSuccess) return err;
+  if (dev < 0 || dev >= kMaxLookDevices) return cudaSuccess;
+  unsigned long long id = 0;
+  if ((err = current_context_id(&id)) != cudaSuccess) return err;
+  LookAhead& L = g_look[dev];
+  if (L.side == nullptr || L.ctx != id) {
+    cudaStreamCaptureStatus cap = cudaStreamCaptureStatusNone;
+    if ((err = cudaStreamIsCapturing(stream, &cap)) != cudaSuccess) return err;
+    if (cap != cudaStreamCaptureStatusNone) return cudaSuccess;
+    L = LookAhead{};  // the handles of an earlier context went with it
+    if ((err = cudaStreamCreateWithFlags(&L.side, cudaStreamNonBlocking)) != cudaSuccess) return err;
+    for (cudaEvent_t& e : L.ev)
+      if ((err = cudaEventCreateWithFlags(&e, cudaEventDisableTiming)) != cudaSuccess) return err;
+    L.ctx = id;
+  }
+  *out = &L;
+  return cudaSuccess;
+}
+
+}  // namespace
+
+// Algorithm 3's block loop.  Per block of B columns: the quantizer (block_kernel) writes
+// the block's codes, nibbles and scaled errors E; then the running weights right of the
+// block take the update W[:, c1:] += (-E) U[block, c1:] as one tcgen05 GEMM over the
+// three-way bf16 splits of E and U (split_e_kernel, split_u_kernel; K = 6 B).
+//
+// Look-ahead: the update is split into the next block's B columns (on the caller's
+// stream, right after the block) and the rest (on a second stream).  The next block's
+// quantization needs only the former, so it runs alongside the latter; U's split for a
+// block is made one block ahead on the second stream.  Events order the two streams:
+//   - block b reads its columns after the second stream's update of block b - 2;
+//   - the next-columns update of block b follows the second stream's update of block
+//     b - 1, which adds into the same columns, so every weight receives its updates in
+//     block order, as in a one-stream loop, and every run gives the same bits;
+//   - the split operands are double-buffered (A' and B' of block b in buffer b % 2) and
+//     each buffer is rewritten only after both updates that read it.
+// A6 and B6 hold two buffers each: A' [m, 6 B] and B' [n, 6 B] bf16.
 cudaError_t launch_gptq_hscale(const void* w, int64_t m, int64_t n, const float* U, const float* h,
                                const float* global_scale, const uint8_t* dead, int block, int down, int up,
                                uint8_t* codes, uint8_t* packed, float* Wf, float* E, uint16_t* A6, uint16_t* B6,
@@ -216,28 +277,84 @@ cudaError_t launch_gptq_hscale(const void* w, int64_t m, int64_t n, const float*
   DeviceInfo info;
   cudaError_t err = current_device_info(&info);
   if (err != cudaSuccess) return err;
+  const int64_t B = block, nb = n / block;
   const unsigned cvt_blocks = (unsigned)std::min<int64_t>((m * n + 255) / 256, (int64_t)info.sm_count * 16);
   to_fp32_kernel<<<cvt_blocks, 256, 0, stream>>>(static_cast<const uint16_t*>(w), m, n, dead, Wf);
   if ((err = cudaGetLastError()) != cudaSuccess) return err;
-  for (int64_t col0 = 0; col0 < n; col0 += block) {
-    const int64_t groups = m * (block / 16);
-    const unsigned qb = (unsigned)std::min<int64_t>((groups * 4 + 127) / 128, (int64_t)info.sm_count * 16);
-    block_kernel<<<qb, 128, 0, stream>>>(Wf, m, n, col0, block, h, U, global_scale, down, up, codes,
-                                         reinterpret_cast<uint2*>(packed), E);
-    if ((err = cudaGetLastError()) != cudaSuccess) return err;
-    if (col0 + block < n) {
-      const int64_t c1 = col0 + block, nn = n - c1;
-      const unsigned eb = (unsigned)std::min<int64_t>((m * block + 255) / 256, (int64_t)info.sm_count * 16);
-      split_e_kernel<<<eb, 256, 0, stream>>>(E, m, block, A6);
+  const int64_t groups = m * (B / 16);
+  const unsigned qb = (unsigned)std::min<int64_t>((groups * 4 + 127) / 128, (int64_t)info.sm_count * 16);
+  const unsigned eb = (unsigned)std::min<int64_t>((m * B + 255) / 256, (int64_t)info.sm_count * 16);
+  uint16_t* Abuf[2] = {A6, A6 + m * 6 * B};
+  uint16_t* Bbuf[2] = {B6, B6 + n * 6 * B};
+  auto quantize = [&](int64_t col0, cudaStream_t s) {
+    block_kernel<<<qb, 128, 0, s>>>(Wf, m, n, col0, block, h, U, global_scale, down, up, codes,
+                                    reinterpret_cast<uint2*>(packed), E);
+    return cudaGetLastError();
+  };
+  auto split_u = [&](int64_t b, cudaStream_t s) {
+    const int64_t c1 = (b + 1) * B, nn = n - c1;
+    split_u_kernel<<<dim3((unsigned)((nn + 31) / 32), (unsigned)((B + 31) / 32)), 256, 0, s>>>(U, n, b * B, block, c1,
+                                                                                                Bbuf[b & 1]);
+    return cudaGetLastError();
+  };
+
+  std::unique_lock<std::mutex> lock(g_look_mu);
+  LookAhead* L = nullptr;
+  if (nb > 1 && (err = look_ahead(stream, &L)) != cudaSuccess) return err;
+  if (L == nullptr) {
+    // one stream: quantize, split, update, block after block
+    lock.unlock();
+    for (int64_t b = 0; b < nb; ++b) {
+      if ((err = quantize(b * B, stream)) != cudaSuccess) return err;
+      if (b + 1 == nb) break;
+      const int64_t c1 = (b + 1) * B, nn = n - c1;
+      split_e_kernel<<<eb, 256, 0, stream>>>(E, m, block, Abuf[0]);
       if ((err = cudaGetLastError()) != cudaSuccess) return err;
-      split_u_kernel<<<dim3((unsigned)((nn + 31) / 32), (unsigned)((block + 31) / 32)), 256, 0, stream>>>(
-          U, n, col0, block, c1, B6);
-      if ((err = cudaGetLastError()) != cudaSuccess) return err;
-      if ((err = launch_gemm_accumulate(A6, B6, m, nn, 6 * (int64_t)block, Wf + c1, n, stream)) != cudaSuccess)
+      if ((err = split_u(b, stream)) != cudaSuccess) return err;  // into buffer b % 2
+      if ((err = launch_gemm_accumulate(Abuf[0], Bbuf[b & 1], m, nn, 6 * B, Wf + c1, n, stream)) != cudaSuccess)
         return err;
     }
+    return cudaSuccess;
   }
-  return cudaSuccess;
+
+  cudaStream_t side = L->side;
+  cudaEvent_t fork = L->ev[0], join = L->ev[1];
+  cudaEvent_t ev_se[2] = {L->ev[2], L->ev[3]}, ev_su[2] = {L->ev[4], L->ev[5]};
+  cudaEvent_t ev_ga[2] = {L->ev[6], L->ev[7]}, ev_gb[2] = {L->ev[8], L->ev[9]};
+  if ((err = cudaEventRecord(fork, stream)) != cudaSuccess) return err;
+  if ((err = cudaStreamWaitEvent(side, fork, 0)) != cudaSuccess) return err;
+  if ((err = split_u(0, side)) != cudaSuccess) return err;
+  if ((err = cudaEventRecord(ev_su[0], side)) != cudaSuccess) return err;
+  for (int64_t b = 0; b < nb; ++b) {
+    const int x = (int)(b & 1);
+    const int64_t c1 = (b + 1) * B, nn = n - c1;
+    // ---- the caller's stream
+    if (b >= 2 && (err = cudaStreamWaitEvent(stream, ev_gb[x], 0)) != cudaSuccess) return err;
+    if ((err = quantize(b * B, stream)) != cudaSuccess) return err;
+    if (b + 1 == nb) break;
+    split_e_kernel<<<eb, 256, 0, stream>>>(E, m, block, Abuf[x]);
+    if ((err = cudaGetLastError()) != cudaSuccess) return err;
+    if ((err = cudaEventRecord(ev_se[x], stream)) != cudaSuccess) return err;
+    if ((err = cudaStreamWaitEvent(stream, ev_su[x], 0)) != cudaSuccess) return err;
+    if (b >= 1 && (err = cudaStreamWaitEvent(stream, ev_gb[x ^ 1], 0)) != cudaSuccess) return err;
+    if ((err = launch_gemm_accumulate(Abuf[x], Bbuf[x], m, std::min<int64_t>(B, nn), 6 * B, Wf + c1, n, stream)) !=
+        cudaSuccess)
+      return err;
+    if ((err = cudaEventRecord(ev_ga[x], stream)) != cudaSuccess) return err;
+    // ---- the second stream
+    if ((err = cudaStreamWaitEvent(side, ev_se[x], 0)) != cudaSuccess) return err;
+    if (nn > B && (err = launch_gemm_accumulate(Abuf[x], Bbuf[x] + B * 6 * B, m, nn - B, 6 * B, Wf + c1 + B, n,
+                                                side)) != cudaSuccess)
+      return err;
+    if ((err = cudaEventRecord(ev_gb[x], side)) != cudaSuccess) return err;
+    if (b + 2 < nb) {  // U's split for the next block, once both updates of block b - 1 have read its buffer
+      if (b >= 1 && (err = cudaStreamWaitEvent(side, ev_ga[x ^ 1], 0)) != cudaSuccess) return err;
+      if ((err = split_u(b + 1, side)) != cudaSuccess) return err;
+      if ((err = cudaEventRecord(ev_su[x ^ 1], side)) != cudaSuccess) return err;
+    }
+  }
+  if ((err = cudaEventRecord(join, side)) != cudaSuccess) return err;
+  return cudaStreamWaitEvent(stream, join, 0);
 }
 
 }  // namespace hscale

@@ -54,6 +54,10 @@ using EncodeTiledFn = CUresult (*)(CUtensorMap*, CUtensorMapDataType, cuuint32_t
                                    CUtensorMapL2promotion, CUtensorMapFloatOOBfill);
 cudaError_t encode_tiled_fn(EncodeTiledFn* out);
 
+// Unique id of the calling thread's current context (0 when it has none yet); a context
+// created again after cudaDeviceReset gets a new id.
+cudaError_t current_context_id(unsigned long long* id);
+
 // cudaFuncAttributeMaxDynamicSharedMemorySize = bytes and the maximum shared-memory
 // carveout for kernel `func` on the current device, set once per (kernel, device) and
 // remembered, so that every GPU of a process gets it (a function attribute belongs to one
