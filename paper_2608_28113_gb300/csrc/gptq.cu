@@ -212,25 +212,24 @@ __global__ void __launch_bounds__(256) to_fp32_kernel(const uint16_t* __restrict
 namespace {
 
 // ---------------------------------------------------------------- the look-ahead stream
-// The block loop runs most of each block's update on a second stream, alongside the next
-// block's quantization.  The stream and its events are created once per device context
-// and reused; a mutex keeps calls from enqueuing at the same time, so one call's events
-// are never re-recorded while another call still has waits to enqueue on them.
-constexpr int kLookEvents = 10;
+// Calls that work ahead (the block loop, the factor) run part of their work on a second
+// stream.  The stream and its events are created once per device context and reused; a
+// mutex keeps calls from enqueuing at the same time, so one call's events are never
+// re-recorded while another call still has waits to enqueue on them.
 struct LookAhead {
   cudaStream_t side = nullptr;
-  cudaEvent_t ev[kLookEvents] = {};
+  cudaEvent_t ev[kLookAheadEvents] = {};
   unsigned long long ctx = 0;
 };
 constexpr int kMaxLookDevices = 64;
 std::mutex g_look_mu;
 LookAhead g_look[kMaxLookDevices];
 
-// The current device's stream and events (caller holds g_look_mu).  nullptr in *out when
-// they do not exist yet and `stream` is being captured: creating them then is not allowed,
-// and the caller takes the one-stream loop.
-cudaError_t look_ahead(cudaStream_t stream, LookAhead** out) {
-  *out = nullptr;
+}  // namespace
+
+cudaError_t acquire_look_ahead(cudaStream_t stream, LookAheadLease* lease) {
+  lease->lock = std::unique_lock<std::mutex>(g_look_mu);
+  lease->side = nullptr;
   int dev = 0;
   cudaError_t err = cudaGetDevice(&dev);
   if (err != cudaSuccess) return err;
@@ -239,6 +238,7 @@ cudaError_t look_ahead(cudaStream_t stream, LookAhead** out) {
   if ((err = current_context_id(&id)) != cudaSuccess) return err;
   LookAhead& L = g_look[dev];
   if (L.side == nullptr || L.ctx != id) {
+    // creating them is not allowed while the stream is being captured
     cudaStreamCaptureStatus cap = cudaStreamCaptureStatusNone;
     if ((err = cudaStreamIsCapturing(stream, &cap)) != cudaSuccess) return err;
     if (cap != cudaStreamCaptureStatusNone) return cudaSuccess;
@@ -248,11 +248,10 @@ cudaError_t look_ahead(cudaStream_t stream, LookAhead** out) {
       if ((err = cudaEventCreateWithFlags(&e, cudaEventDisableTiming)) != cudaSuccess) return err;
     L.ctx = id;
   }
-  *out = &L;
+  lease->side = L.side;
+  for (int i = 0; i < kLookAheadEvents; ++i) lease->ev[i] = L.ev[i];
   return cudaSuccess;
 }
-
-}  // namespace
 
 // Algorithm 3's block loop.  Per block of B columns: the quantizer (block_kernel) writes
 // the block's codes, nibbles and scaled errors E; then the running weights right of the
@@ -298,12 +297,11 @@ cudaError_t launch_gptq_hscale(const void* w, int64_t m, int64_t n, const float*
     return cudaGetLastError();
   };
 
-  std::unique_lock<std::mutex> lock(g_look_mu);
-  LookAhead* L = nullptr;
-  if (nb > 1 && (err = look_ahead(stream, &L)) != cudaSuccess) return err;
-  if (L == nullptr) {
+  LookAheadLease L;
+  if (nb > 1 && (err = acquire_look_ahead(stream, &L)) != cudaSuccess) return err;
+  if (L.side == nullptr) {
     // one stream: quantize, split, update, block after block
-    lock.unlock();
+    if (L.lock.owns_lock()) L.lock.unlock();
     for (int64_t b = 0; b < nb; ++b) {
       if ((err = quantize(b * B, stream)) != cudaSuccess) return err;
       if (b + 1 == nb) break;
@@ -317,10 +315,10 @@ cudaError_t launch_gptq_hscale(const void* w, int64_t m, int64_t n, const float*
     return cudaSuccess;
   }
 
-  cudaStream_t side = L->side;
-  cudaEvent_t fork = L->ev[0], join = L->ev[1];
-  cudaEvent_t ev_se[2] = {L->ev[2], L->ev[3]}, ev_su[2] = {L->ev[4], L->ev[5]};
-  cudaEvent_t ev_ga[2] = {L->ev[6], L->ev[7]}, ev_gb[2] = {L->ev[8], L->ev[9]};
+  cudaStream_t side = L.side;
+  cudaEvent_t fork = L.ev[0], join = L.ev[1];
+  cudaEvent_t ev_se[2] = {L.ev[2], L.ev[3]}, ev_su[2] = {L.ev[4], L.ev[5]};
+  cudaEvent_t ev_ga[2] = {L.ev[6], L.ev[7]}, ev_gb[2] = {L.ev[8], L.ev[9]};
   if ((err = cudaEventRecord(fork, stream)) != cudaSuccess) return err;
   if ((err = cudaStreamWaitEvent(side, fork, 0)) != cudaSuccess) return err;
   if ((err = split_u(0, side)) != cudaSuccess) return err;

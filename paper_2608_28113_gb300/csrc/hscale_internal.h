@@ -5,6 +5,8 @@
 #include <cuda.h>
 #include <cuda_runtime.h>
 
+#include <mutex>
+
 namespace hscale {
 
 struct DeviceInfo {
@@ -57,6 +59,19 @@ cudaError_t encode_tiled_fn(EncodeTiledFn* out);
 // Unique id of the calling thread's current context (0 when it has none yet); a context
 // created again after cudaDeviceReset gets a new id.
 cudaError_t current_context_id(unsigned long long* id);
+
+// The library's second stream and its events in the current device context, for calls that
+// work ahead on it (created on first use and kept).  The lease holds the library's mutex:
+// release it (destroy the lease) only after the call has enqueued all its work.  side is
+// null when they do not exist yet and `stream` is being captured (they may not be created
+// then): the call then runs on `stream` alone.
+constexpr int kLookAheadEvents = 10;
+struct LookAheadLease {
+  std::unique_lock<std::mutex> lock;
+  cudaStream_t side = nullptr;
+  cudaEvent_t ev[kLookAheadEvents] = {};
+};
+cudaError_t acquire_look_ahead(cudaStream_t stream, LookAheadLease* lease);
 
 // cudaFuncAttributeMaxDynamicSharedMemorySize = bytes and the maximum shared-memory
 // carveout for kernel `func` on the current device, set once per (kernel, device) and

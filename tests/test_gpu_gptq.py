@@ -293,3 +293,27 @@ def test_gptq_look_ahead_is_deterministic_and_capturable():
     assert np.array_equal(packed.cpu().numpy(), runs[0][1])
     ref = oracle.gptq_hscale(wb, U32.astype(np.float64), h32, s_g, block, 4, 4, dead=dead)
     assert float(np.mean(runs[0][0] == ref["codes"])) >= 0.98
+
+
+def test_factor_is_deterministic_and_capturable():
+    """The factor gives the same bits on every run and when captured into a CUDA graph and
+    replayed (the bench times it that way)."""
+    n = 1000
+    g = np.random.default_rng(31)
+    A = g.standard_normal((n, n)) / np.sqrt(n)
+    H32 = (A @ A.T + 0.1 * np.eye(n)).astype(np.float32)
+    outs = [gpu_factor(H32) for _ in range(2)]
+    assert np.array_equal(outs[0][0], outs[1][0]) and np.all(outs[0][2] == 0)
+    Hd = torch.from_numpy(H32).to(dev())
+    U = torch.zeros(n, n, dtype=torch.float32, device=dev())
+    dead = torch.empty(n, dtype=torch.uint8, device=dev())
+    info = torch.zeros(3, dtype=torch.int32, device=dev())
+    ws = torch.empty(hs.hscale_gptq_factor_workspace_bytes(n), dtype=torch.uint8, device=dev())
+    s = torch.cuda.Stream()
+    s.wait_stream(torch.cuda.current_stream())
+    gr = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(gr, stream=s):
+        hs.hscale_gptq_factor(Hd, 0.01, U, dead, info, ws)
+    gr.replay()
+    torch.cuda.synchronize()
+    assert np.array_equal(U.cpu().numpy(), outs[0][0]) and int(info.abs().sum()) == 0
