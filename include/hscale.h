@@ -422,7 +422,7 @@ int hscale_output_error(const void* x_bf16, int64_t tokens, int64_t n, int64_t l
  *    accuracy (on the tensor cores: three-way bf16 splits of E and U, the six products
  *    above 2^-24 relative, fp32 accumulation).  Writes codes_out [m, n/16] and packed_out
  *    [m, n/2] (8-byte aligned) as hscale_refine_scales does.  The workspace
- *    (hscale_gptq_workspace_bytes) holds the running weights, E and two buffers of each
+ *    (hscale_gptq_workspace_bytes) holds the running weights and two buffers of each
  *    split operand.  With more than one block the call works ahead: the update of the
  *    next block's columns runs on `stream` and the rest of each update on a second stream
  *    of the library, alongside the next block's quantization; events order the two, every

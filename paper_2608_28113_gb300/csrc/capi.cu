@@ -298,13 +298,12 @@ namespace {
 inline int64_t round256(int64_t bytes) { return (bytes + 255) / 256 * 256; }
 }  // namespace
 
-// running weights (fp32 m x n), E (fp32 m x block), and two buffers each of the bf16 split
-// operands of the update GEMM: A' (m x 6 block) and B' (n x 6 block)
+// running weights (fp32 m x n) and two buffers each of the bf16 split operands of the
+// update GEMM: A' (m x 6 block) and B' (n x 6 block)
 size_t hscale_gptq_workspace_bytes(int64_t m, int64_t n, int32_t block) {
   if (m <= 0 || n <= 0 || block <= 0) return 0;
   const int64_t b = block;
-  return (size_t)(round256(m * n * 4) + round256(m * b * 4) + round256(2 * m * 6 * b * 2) +
-                  round256(2 * n * 6 * b * 2));
+  return (size_t)(round256(m * n * 4) + round256(2 * m * 6 * b * 2) + round256(2 * n * 6 * b * 2));
 }
 
 int hscale_gptq_hscale(const void* w_bf16, int64_t m, int64_t n, const float* U, const float* h,
@@ -325,12 +324,10 @@ int hscale_gptq_hscale(const void* w_bf16, int64_t m, int64_t n, const float* U,
   uint8_t* base = static_cast<uint8_t*>(workspace);
   const int64_t b = block;
   float* Wf = reinterpret_cast<float*>(base);
-  float* E = reinterpret_cast<float*>(base + round256(m * n * 4));
-  uint16_t* A6 = reinterpret_cast<uint16_t*>(base + round256(m * n * 4) + round256(m * b * 4));
-  uint16_t* B6 = reinterpret_cast<uint16_t*>(base + round256(m * n * 4) + round256(m * b * 4) +
-                                             round256(2 * m * 6 * b * 2));
+  uint16_t* A6 = reinterpret_cast<uint16_t*>(base + round256(m * n * 4));
+  uint16_t* B6 = reinterpret_cast<uint16_t*>(base + round256(m * n * 4) + round256(2 * m * 6 * b * 2));
   return from_cuda(hscale::launch_gptq_hscale(w_bf16, m, n, U, h, global_scale, dead, block, down, up, codes_out,
-                                              packed_out, Wf, E, A6, B6, as_stream(stream)));
+                                              packed_out, Wf, A6, B6, as_stream(stream)));
 }
 
 int hscale_pack_nvfp4(const void* w_bf16, int64_t m, int64_t n, const float* global_scale,

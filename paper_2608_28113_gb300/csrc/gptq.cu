@@ -48,15 +48,34 @@ __device__ float exact_group_score(const float (&a)[16], const float (&hj)[16], 
   return t[0];
 }
 
+// The update W[:, c1:] -= E U[col0:c1, c1:] (c1 = col0 + B) runs on the tensor cores with
+// fp32-level accuracy: every fp32 value x is split into three bf16 parts x1 + x2 + x3 (each
+// difference exact in fp32, so the parts carry x to about 2^-24 relative), and the six
+// products E1 U1, E1 U2, E2 U1, E1 U3, E2 U2, E3 U1 (every pair whose weight is above
+// 2^-24) are one bf16 GEMM over K = 6B with fp32 accumulation: A' = [-E1 | -E1 | -E2 | -E1
+// | -E2 | -E3] against B' = [U1 | U2 | U1 | U3 | U2 | U1] (the negation makes the GEMM's
+// accumulate a subtract).
+__device__ __forceinline__ void split3(float x, uint16_t (&p)[3]) {
+  const __nv_bfloat16 a = __float2bfloat16_rn(x);
+  const float r1 = __fsub_rn(x, __bfloat162float(a));
+  const __nv_bfloat16 b = __float2bfloat16_rn(r1);
+  const float r2 = __fsub_rn(r1, __bfloat162float(b));
+  const __nv_bfloat16 c = __float2bfloat16_rn(r2);
+  p[0] = __bfloat16_as_ushort(a);
+  p[1] = __bfloat16_as_ushort(b);
+  p[2] = __bfloat16_as_ushort(c);
+}
+
 // Four lanes (a quad) per group: each scores every fourth candidate of the window with exact
 // decisions, the quad keeps the best under the search's tie rule (a total order, so every
-// lane ends with the same code), and each lane writes the nibbles and errors of four of the
-// group's elements.
+// lane ends with the same code), and each lane writes the nibbles of four of the group's
+// elements and their scaled errors E = (w - w_hat) / U_jj, split, into the update's A
+// operand [m, 6B]: A' = [-E1 | -E1 | -E2 | -E1 | -E2 | -E3], four bf16 (8 bytes) per segment.
 __global__ void __launch_bounds__(128) block_kernel(const float* __restrict__ W, int64_t m, int64_t n, int64_t col0,
                                                     int B, const float* __restrict__ h, const float* __restrict__ U,
                                                     const float* __restrict__ global_scale, int down, int up,
                                                     uint8_t* __restrict__ codes, uint2* __restrict__ packed,
-                                                    float* __restrict__ E) {
+                                                    uint16_t* __restrict__ A) {
   const int gpb = B / 16;
   const int64_t total = m * gpb * 4;  // lanes
   const int q = threadIdx.x & 3;
@@ -110,6 +129,7 @@ __global__ void __launch_bounds__(128) block_kernel(const float* __restrict__ W,
     const float4 wq = reinterpret_cast<const float4*>(W + r * n + col)[q];
     const float wv[4] = {wq.x, wq.y, wq.z, wq.w};
     uint32_t part = 0u;  // this lane's four nibbles in their place in the group's 32-bit word
+    uint16_t ep[3][4];   // the three bf16 parts of -E for this lane's four elements
 #pragma unroll
     for (int t = 0; t < 4; ++t) {
       const int j = 4 * q + t;
@@ -119,7 +139,27 @@ __global__ void __launch_bounds__(128) block_kernel(const float* __restrict__ W,
       part |= ((neg << 3) | k) << (4 * (j & 7));
       float what = __fmul_rn(d.sg, __fmul_rn(e2m1_from_raw(k << 22), l));  // s_g (l q), l q exact
       if (neg) what = -what;
-      if (active) E[r * B + 16 * i + j] = __fdiv_rn(__fsub_rn(wv[t], what), U[(col + j) * n + col + j]);
+      const float e = __fdiv_rn(__fsub_rn(wv[t], what), U[(col + j) * n + col + j]);
+      uint16_t pp[3];
+      split3(-e, pp);
+      ep[0][t] = pp[0];
+      ep[1][t] = pp[1];
+      ep[2][t] = pp[2];
+    }
+    if (active) {
+      uint2 v[3];
+#pragma unroll
+      for (int p3 = 0; p3 < 3; ++p3)
+        v[p3] = make_uint2((uint32_t)ep[p3][0] | ((uint32_t)ep[p3][1] << 16),
+                           (uint32_t)ep[p3][2] | ((uint32_t)ep[p3][3] << 16));
+      uint2* row = reinterpret_cast<uint2*>(A + r * 6 * (int64_t)B + 16 * i + 4 * q);
+      const int seg = B / 4;  // one segment, in 8-byte words
+      row[0] = v[0];
+      row[seg] = v[0];
+      row[2 * seg] = v[1];
+      row[3 * seg] = v[0];
+      row[4 * seg] = v[1];
+      row[5 * seg] = v[2];
     }
     const uint32_t word = part | __shfl_xor_sync(0xFFFFFFFFu, part, 1);  // lanes 0-1: word 0, 2-3: word 1
     const uint32_t other = __shfl_xor_sync(0xFFFFFFFFu, word, 2);
@@ -127,43 +167,6 @@ __global__ void __launch_bounds__(128) block_kernel(const float* __restrict__ W,
       codes[r * (n / 16) + col / 16] = (uint8_t)bc;
       packed[r * (n / 16) + col / 16] = make_uint2(word, other);
     }
-  }
-}
-
-// The update W[:, c1:] -= E U[col0:c1, c1:] (c1 = col0 + B) runs on the tensor cores with
-// fp32-level accuracy: every fp32 value x is split into three bf16 parts x1 + x2 + x3 (each
-// difference exact in fp32, so the parts carry x to about 2^-24 relative), and the six
-// products E1 U1, E1 U2, E2 U1, E1 U3, E2 U2, E3 U1 (every pair whose weight is above
-// 2^-24) are one bf16 GEMM over K = 6B with fp32 accumulation: A' = [-E1 | -E1 | -E2 | -E1
-// | -E2 | -E3] against B' = [U1 | U2 | U1 | U3 | U2 | U1] (the negation makes the GEMM's
-// accumulate a subtract).
-__device__ __forceinline__ void split3(float x, uint16_t (&p)[3]) {
-  const __nv_bfloat16 a = __float2bfloat16_rn(x);
-  const float r1 = __fsub_rn(x, __bfloat162float(a));
-  const __nv_bfloat16 b = __float2bfloat16_rn(r1);
-  const float r2 = __fsub_rn(r1, __bfloat162float(b));
-  const __nv_bfloat16 c = __float2bfloat16_rn(r2);
-  p[0] = __bfloat16_as_ushort(a);
-  p[1] = __bfloat16_as_ushort(b);
-  p[2] = __bfloat16_as_ushort(c);
-}
-
-// A' [m, 6B] from E [m, B] (segments -E1, -E1, -E2, -E1, -E2, -E3)
-__global__ void __launch_bounds__(256) split_e_kernel(const float* __restrict__ E, int64_t m, int B,
-                                                      uint16_t* __restrict__ A) {
-  const int64_t total = m * B;
-  for (int64_t e = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; e < total; e += (int64_t)gridDim.x * blockDim.x) {
-    const int64_t r = e / B;
-    const int k = (int)(e - r * B);
-    uint16_t p[3];
-    split3(-E[e], p);
-    uint16_t* row = A + r * 6 * B + k;
-    row[0] = p[0];
-    row[B] = p[0];
-    row[2 * B] = p[1];
-    row[3 * B] = p[0];
-    row[4 * B] = p[1];
-    row[5 * B] = p[2];
   }
 }
 
@@ -254,9 +257,10 @@ cudaError_t acquire_look_ahead(cudaStream_t stream, LookAheadLease* lease) {
 }
 
 // Algorithm 3's block loop.  Per block of B columns: the quantizer (block_kernel) writes
-// the block's codes, nibbles and scaled errors E; then the running weights right of the
-// block take the update W[:, c1:] += (-E) U[block, c1:] as one tcgen05 GEMM over the
-// three-way bf16 splits of E and U (split_e_kernel, split_u_kernel; K = 6 B).
+// the block's codes and nibbles and its scaled errors E, split into the update's A operand
+// A'; then the running weights right of the block take the update W[:, c1:] += (-E)
+// U[block, c1:] as one tcgen05 GEMM over the three-way bf16 splits of E and U
+// (split_u_kernel writes U's, B'; K = 6 B).
 //
 // Look-ahead: the update is split into the next block's B columns (on the caller's
 // stream, right after the block) and the rest (on a second stream).  The next block's
@@ -271,7 +275,7 @@ cudaError_t acquire_look_ahead(cudaStream_t stream, LookAheadLease* lease) {
 // A6 and B6 hold two buffers each: A' [m, 6 B] and B' [n, 6 B] bf16.
 cudaError_t launch_gptq_hscale(const void* w, int64_t m, int64_t n, const float* U, const float* h,
                                const float* global_scale, const uint8_t* dead, int block, int down, int up,
-                               uint8_t* codes, uint8_t* packed, float* Wf, float* E, uint16_t* A6, uint16_t* B6,
+                               uint8_t* codes, uint8_t* packed, float* Wf, uint16_t* A6, uint16_t* B6,
                                cudaStream_t stream) {
   DeviceInfo info;
   cudaError_t err = current_device_info(&info);
@@ -282,12 +286,11 @@ cudaError_t launch_gptq_hscale(const void* w, int64_t m, int64_t n, const float*
   if ((err = cudaGetLastError()) != cudaSuccess) return err;
   const int64_t groups = m * (B / 16);
   const unsigned qb = (unsigned)std::min<int64_t>((groups * 4 + 127) / 128, (int64_t)info.sm_count * 16);
-  const unsigned eb = (unsigned)std::min<int64_t>((m * B + 255) / 256, (int64_t)info.sm_count * 16);
   uint16_t* Abuf[2] = {A6, A6 + m * 6 * B};
   uint16_t* Bbuf[2] = {B6, B6 + n * 6 * B};
-  auto quantize = [&](int64_t col0, cudaStream_t s) {
-    block_kernel<<<qb, 128, 0, s>>>(Wf, m, n, col0, block, h, U, global_scale, down, up, codes,
-                                    reinterpret_cast<uint2*>(packed), E);
+  auto quantize = [&](int64_t b, cudaStream_t s) {
+    block_kernel<<<qb, 128, 0, s>>>(Wf, m, n, b * B, block, h, U, global_scale, down, up, codes,
+                                    reinterpret_cast<uint2*>(packed), Abuf[b & 1]);
     return cudaGetLastError();
   };
   auto split_u = [&](int64_t b, cudaStream_t s) {
@@ -303,13 +306,11 @@ cudaError_t launch_gptq_hscale(const void* w, int64_t m, int64_t n, const float*
     // one stream: quantize, split, update, block after block
     if (L.lock.owns_lock()) L.lock.unlock();
     for (int64_t b = 0; b < nb; ++b) {
-      if ((err = quantize(b * B, stream)) != cudaSuccess) return err;
+      if ((err = quantize(b, stream)) != cudaSuccess) return err;
       if (b + 1 == nb) break;
       const int64_t c1 = (b + 1) * B, nn = n - c1;
-      split_e_kernel<<<eb, 256, 0, stream>>>(E, m, block, Abuf[0]);
-      if ((err = cudaGetLastError()) != cudaSuccess) return err;
-      if ((err = split_u(b, stream)) != cudaSuccess) return err;  // into buffer b % 2
-      if ((err = launch_gemm_accumulate(Abuf[0], Bbuf[b & 1], m, nn, 6 * B, Wf + c1, n, stream)) != cudaSuccess)
+      if ((err = split_u(b, stream)) != cudaSuccess) return err;
+      if ((err = launch_gemm_accumulate(Abuf[b & 1], Bbuf[b & 1], m, nn, 6 * B, Wf + c1, n, stream)) != cudaSuccess)
         return err;
     }
     return cudaSuccess;
@@ -317,7 +318,7 @@ cudaError_t launch_gptq_hscale(const void* w, int64_t m, int64_t n, const float*
 
   cudaStream_t side = L.side;
   cudaEvent_t fork = L.ev[0], join = L.ev[1];
-  cudaEvent_t ev_se[2] = {L.ev[2], L.ev[3]}, ev_su[2] = {L.ev[4], L.ev[5]};
+  cudaEvent_t ev_q[2] = {L.ev[2], L.ev[3]}, ev_su[2] = {L.ev[4], L.ev[5]};
   cudaEvent_t ev_ga[2] = {L.ev[6], L.ev[7]}, ev_gb[2] = {L.ev[8], L.ev[9]};
   if ((err = cudaEventRecord(fork, stream)) != cudaSuccess) return err;
   if ((err = cudaStreamWaitEvent(side, fork, 0)) != cudaSuccess) return err;
@@ -327,12 +328,11 @@ cudaError_t launch_gptq_hscale(const void* w, int64_t m, int64_t n, const float*
     const int x = (int)(b & 1);
     const int64_t c1 = (b + 1) * B, nn = n - c1;
     // ---- the caller's stream
+    // block b reads its columns, and its A' buffer was last read, by block b - 2's update
     if (b >= 2 && (err = cudaStreamWaitEvent(stream, ev_gb[x], 0)) != cudaSuccess) return err;
-    if ((err = quantize(b * B, stream)) != cudaSuccess) return err;
+    if ((err = quantize(b, stream)) != cudaSuccess) return err;
     if (b + 1 == nb) break;
-    split_e_kernel<<<eb, 256, 0, stream>>>(E, m, block, Abuf[x]);
-    if ((err = cudaGetLastError()) != cudaSuccess) return err;
-    if ((err = cudaEventRecord(ev_se[x], stream)) != cudaSuccess) return err;
+    if ((err = cudaEventRecord(ev_q[x], stream)) != cudaSuccess) return err;
     if ((err = cudaStreamWaitEvent(stream, ev_su[x], 0)) != cudaSuccess) return err;
     if (b >= 1 && (err = cudaStreamWaitEvent(stream, ev_gb[x ^ 1], 0)) != cudaSuccess) return err;
     if ((err = launch_gemm_accumulate(Abuf[x], Bbuf[x], m, std::min<int64_t>(B, nn), 6 * B, Wf + c1, n, stream)) !=
@@ -340,7 +340,7 @@ cudaError_t launch_gptq_hscale(const void* w, int64_t m, int64_t n, const float*
       return err;
     if ((err = cudaEventRecord(ev_ga[x], stream)) != cudaSuccess) return err;
     // ---- the second stream
-    if ((err = cudaStreamWaitEvent(side, ev_se[x], 0)) != cudaSuccess) return err;
+    if ((err = cudaStreamWaitEvent(side, ev_q[x], 0)) != cudaSuccess) return err;
     if (nn > B && (err = launch_gemm_accumulate(Abuf[x], Bbuf[x] + B * 6 * B, m, nn - B, 6 * B, Wf + c1 + B, n,
                                                 side)) != cudaSuccess)
       return err;

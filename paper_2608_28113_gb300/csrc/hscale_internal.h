@@ -110,7 +110,7 @@ cudaError_t launch_gemm_accumulate(const void* a, const void* b, int64_t m, int6
 
 cudaError_t launch_gptq_hscale(const void* w, int64_t m, int64_t n, const float* U, const float* h,
                                const float* global_scale, const uint8_t* dead, int block, int down, int up,
-                               uint8_t* codes, uint8_t* packed, float* Wf, float* E, uint16_t* A6, uint16_t* B6,
+                               uint8_t* codes, uint8_t* packed, float* Wf, uint16_t* A6, uint16_t* B6,
                                cudaStream_t stream);
 
 // Sticky device error flags of each translation unit (bit 0: a bounded wait ran out);

@@ -246,7 +246,7 @@ def test_gptq_argument_errors(lib):
     assert g(FAKE, 64, 64, 0.01, FAKE, None, FAKE, None, wsf(64), None) == ERR_WS
     assert g(FAKE, 65537, 65537, 0.01, FAKE, None, FAKE, FAKE, 1 << 20, None) == ERR_SHAPE
     # 4x64 fp32 weights + 4x32 fp32 E + 4x192 and 64x192 bf16 split operands, each rounded to 256 B
-    assert lib.hscale_gptq_workspace_bytes(4, 64, 32) == 1024 + 512 + 2 * 1536 + 2 * 24576
+    assert lib.hscale_gptq_workspace_bytes(4, 64, 32) == 1024 + 2 * 1536 + 2 * 24576
     q = lib.hscale_gptq_hscale
     assert q(FAKE, 4, 64, FAKE, FAKE, FAKE, None, 24, 4, 4, FAKE, FAKE, FAKE, 1 << 20, None) == ERR_SHAPE
     assert q(FAKE, 4, 64, FAKE, FAKE, FAKE, None, 48, 4, 4, FAKE, FAKE, FAKE, 1 << 20, None) == ERR_SHAPE
