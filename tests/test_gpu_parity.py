@@ -129,6 +129,9 @@ def test_hessian_single_chunk_small_layer():
     (8, 3, 3, 8),              # minimum width, strided rows (ld = 16)
     (4096, 777, 256, 64),      # wide rows, ld = n + 64, ragged last chunk
     (14336, 4096, 4096, 0),    # MLP width
+    (200, 9000, 4500, 8),      # last 128-channel tile 72 wide: second 64-channel box partly past n
+    (136, 1000, 333, 0),       # last tile 8 wide: its second box wholly past n (not loaded)
+    (4096, 8256, 8256, 0),     # chunk not a multiple of a 64-token stage per cluster CTA
 ])
 def test_hessian_chunking_ragged_and_strided(n, tokens, chunk, pad):
     g = torch.Generator().manual_seed(n * 7 + tokens)
