@@ -37,7 +37,8 @@
  * Conventions shared by every entry point
  * ---------------------------------------
  * - All pointers except `stream` are DEVICE pointers owned by the caller; the
- *   library allocates and frees nothing.  Work is enqueued on `stream` (a
+ *   library allocates and frees no memory (hscale_gptq_hscale keeps one stream and a
+ *   few events per device context, see there).  Work is enqueued on `stream` (a
  *   cudaStream_t passed as void*, NULL = legacy default stream) and nothing
  *   synchronises: results are ready when the stream reaches them.
  * - Matrices are row-major.  W is [m, n] bfloat16 with contiguous rows; groups of 16
