@@ -127,14 +127,21 @@ __device__ __forceinline__ float rcp_approx_f(float x) {
 // go to shared memory and come back four rows per 16-byte broadcast load, and each lane
 // updates its row.  Entries above the diagonal are updated too (harmlessly) and zeroed at the
 // end.  The square roots and reciprocals come from the approximate hardware instructions
-// (relative error about 2^-22), which keeps the serial chain of pivots short.  Then lane c
-// computes column c of Z by forward substitution, reading L from shared memory (a broadcast).
+// (relative error about 2^-22), which keeps the serial chain of pivots short.
+// The inverse is built in the same sweep: lane c also holds column c of Z, as partial sums
+// s_i = delta_ic - sum_{m < j} L_im Z_mc over the rows not yet final.  When columns j and
+// j + 1 of L are known, Z_jc = s_j / L_jj and Z_j+1,c = (s_j+1 - L_j+1,j Z_jc) / L_j+1,j+1
+// (forward substitution), and the later rows take s_k -= L_kj Z_jc + L_k,j+1 Z_j+1,c with
+// the same broadcast loads as the factor's update, so no second serial pass is needed.
 __device__ __noinline__ void factor_sub32(float* A, float* Zo, float* Zt, float* col, int lane, int32_t* info,
                                           int32_t base) {
   const unsigned full = 0xFFFFFFFFu;
-  float r[kSub];
+  float r[kSub], z[kSub];
 #pragma unroll
-  for (int k = 0; k < kSub; ++k) r[k] = A[lane * kLd + k];
+  for (int k = 0; k < kSub; ++k) {
+    r[k] = A[lane * kLd + k];
+    z[k] = k == lane ? 1.0f : 0.0f;
+  }
   float2* col2 = reinterpret_cast<float2*>(col);
 #pragma unroll
   for (int j = 0; j < kSub; j += 2) {
@@ -161,6 +168,11 @@ __device__ __noinline__ void factor_sub32(float* A, float* Zo, float* Zt, float*
     const float v1 = lane == j + 1 ? l11 : (lane > j + 1 ? x1 : 0.0f);
     r[j] = v0;
     r[j + 1] = v1;
+    // rows j and j + 1 of Z in this lane's column (1 / L_jj = ra, 1 / L_j+1,j+1 = rc)
+    const float zj = __fmul_rn(z[j], ra);
+    const float zj1 = __fmul_rn(__fmaf_rn(-l10, zj, z[j + 1]), rc);
+    z[j] = zj;
+    z[j + 1] = zj1;
     if (j + 2 < kSub) {
       col2[lane] = make_float2(v0, v1);
       __syncwarp();
@@ -169,35 +181,20 @@ __device__ __noinline__ void factor_sub32(float* A, float* Zo, float* Zt, float*
         const float4 q = *reinterpret_cast<const float4*>(col + 2 * k);  // (L_kj, L_k,j+1, L_k+1,j, L_k+1,j+1)
         r[k] = __fmaf_rn(-v0, q.x, __fmaf_rn(-v1, q.y, r[k]));
         r[k + 1] = __fmaf_rn(-v0, q.z, __fmaf_rn(-v1, q.w, r[k + 1]));
+        z[k] = __fmaf_rn(-q.x, zj, __fmaf_rn(-q.y, zj1, z[k]));
+        z[k + 1] = __fmaf_rn(-q.z, zj, __fmaf_rn(-q.w, zj1, z[k + 1]));
       }
       __syncwarp();
     }
   }
 #pragma unroll
   for (int k = 0; k < kSub; ++k) A[lane * kLd + k] = k <= lane ? r[k] : 0.0f;
-  __syncwarp();
-  float x[kSub];
+  // lane c holds column c of Z: row i is zero above the diagonal (i < c)
 #pragma unroll
   for (int i = 0; i < kSub; ++i) {
-    float acc0 = 0.0f, acc1 = 0.0f, acc2 = 0.0f, acc3 = 0.0f;
-#pragma unroll
-    for (int m = 0; m + 3 < i; m += 4) {
-      const float4 l = *reinterpret_cast<const float4*>(A + i * kLd + m);
-      acc0 = __fmaf_rn(l.x, x[m], acc0);
-      acc1 = __fmaf_rn(l.y, x[m + 1], acc1);
-      acc2 = __fmaf_rn(l.z, x[m + 2], acc2);
-      acc3 = __fmaf_rn(l.w, x[m + 3], acc3);
-    }
-#pragma unroll
-    for (int m = i & ~3; m < i; ++m) acc0 = __fmaf_rn(A[i * kLd + m], x[m], acc0);
-    const float invl = rcp_approx_f(A[i * kLd + i]);
-    const float v = -__fmul_rn(__fadd_rn(__fadd_rn(acc0, acc1), __fadd_rn(acc2, acc3)), invl);
-    x[i] = lane == i ? invl : (lane < i ? v : 0.0f);
-  }
-#pragma unroll
-  for (int i = 0; i < kSub; ++i) {
-    Zo[i * kLd + lane] = x[i];
-    Zt[lane * kLd + i] = x[i];
+    const float x = i >= lane ? z[i] : 0.0f;
+    Zo[i * kLd + lane] = x;
+    Zt[lane * kLd + i] = x;
   }
 }
 
