@@ -1,4 +1,4 @@
-"""Sharding of the hot path across ranks (SURVEY §8(e) shape), tested on CPU with gloo ranks.
+"""Sharding of the hot path across ranks (calibration tokens for h, rows of W for the search), tested on CPU with gloo ranks.
 
 The orchestration in paper_2608_28113_gb300.sharded -- token shares for the Hessian pass,
 the all-gather of the partials and their rank-order sum, the all-reduce with MAX of the amax
