@@ -43,7 +43,7 @@ constexpr int kNb = 128;                  // block of the sweep
 constexpr int kSub = 32;                  // sub-block of the diagonal factor (one warp)
 constexpr int kLd = kNb + 4;              // padded shared-memory row (16-byte multiple)
 constexpr int kDiagThreads = 512;
-constexpr int kDiagSmemBytes = (3 * kNb * kLd + 2 * kSub) * 4;
+constexpr int kDiagSmemBytes = (3 * kNb * kLd + 4 * kSub) * 4;
 constexpr int kStripRows = 32;            // rows (or columns) of one strip
 constexpr int kStripThreads = 256;
 constexpr int kStripSmemBytes = (kNb * (kNb + 4) + kNb * (kStripRows + 4)) * 4;
@@ -111,91 +111,122 @@ __device__ __forceinline__ float rsqrt_approx(float x) {
   asm("rsqrt.approx.f32 %0, %1;" : "=f"(r) : "f"(x));
   return r;
 }
-__device__ __forceinline__ float rcp_approx_f(float x) {
-  float r;
-  asm("rcp.approx.f32 %0, %1;" : "=f"(r) : "f"(x));
-  return r;
-}
 
 // One warp factors the 32 x 32 block at A (row stride kLd, lower triangle) in place,
 // A = L L^T, and writes Z = L^-1 (lower, zeros above) at Zo and its transpose at Zt (row
-// stride kLd each); col is a 64-float scratch.  Lane i holds row i of the block in registers
-// (every loop has a constant trip count and every register index is a constant, so the row
-// stays in registers; kept out of line: inlined into the block kernel, the compiler moves the
-// row to local memory).  Two columns are eliminated per step: the 2 x 2 pivot block gives
-// L_jj, L_j+1,j and L_j+1,j+1, every lane scales its two entries, the pairs (L_kj, L_k,j+1)
-// go to shared memory and come back four rows per 16-byte broadcast load, and each lane
-// updates its row.  Entries above the diagonal are updated too (harmlessly) and zeroed at the
-// end.  The square roots and reciprocals come from the approximate hardware instructions
-// (relative error about 2^-22), which keeps the serial chain of pivots short.
+// stride kLd each); col is a 128-float scratch (two 64-float buffers).  Lane i holds row i of
+// the block in registers (every loop has a constant trip count and every register index is a
+// constant, so the row stays in registers; kept out of line: inlined into the block kernel,
+// the compiler moves the row to local memory).  Two columns are eliminated per step: the
+// 2 x 2 pivot block gives L_jj, L_j+1,j and L_j+1,j+1, every lane scales its two entries, the
+// pairs (L_kj, L_k,j+1) go to shared memory and come back four rows per 16-byte broadcast
+// load, and each lane updates its row.  Entries above the diagonal are updated too
+// (harmlessly) and zeroed at the end.  The square roots come from the approximate hardware
+// instruction (relative error about 2^-22), which keeps the serial chain of pivots short.
 // The inverse is built in the same sweep: lane c also holds column c of Z, as partial sums
 // s_i = delta_ic - sum_{m < j} L_im Z_mc over the rows not yet final.  When columns j and
 // j + 1 of L are known, Z_jc = s_j / L_jj and Z_j+1,c = (s_j+1 - L_j+1,j Z_jc) / L_j+1,j+1
 // (forward substitution), and the later rows take s_k -= L_kj Z_jc + L_k,j+1 Z_j+1,c with
 // the same broadcast loads as the factor's update, so no second serial pass is needed.
+// Each step updates the next pivot pair's two rows first and computes that pair's pivots
+// before the rest of its update, so the serial chain of the next step can run alongside this
+// step's bulk of independent FMAs; the pivot columns alternate between the two scratch
+// buffers, so one __syncwarp per step orders them.  A pivot that is not positive is kept in a
+// register (the first one) and recorded once at the end, so no step branches.  Every value
+// takes the same operations in the same order as a plain right-looking sweep.
+
+// The pivot pair (j, j + 1) from the current rows (the 2 x 2 block comes from lanes j and
+// j + 1): this lane's entries v0 = L_lane,j and v1 = L_lane,j+1 (zero above the diagonal),
+// rows j and j + 1 of Z in this lane's column (1 / L_jj = ra, 1 / L_j+1,j+1 = rc), all four
+// written back into r and z.
+__device__ __forceinline__ void pivot_pair(float (&r)[kSub], float (&z)[kSub], const int j, int lane,
+                                           int32_t base, int32_t& fail, float& v0, float& v1, float& zj,
+                                           float& zj1) {
+  const unsigned full = 0xFFFFFFFFu;
+  float a = __shfl_sync(full, r[j], j);
+  const float b = __shfl_sync(full, r[j], j + 1);
+  const float c = __shfl_sync(full, r[j + 1], j + 1);
+  const bool bad_a = !(a > 0.0f);
+  fail = (fail == 0 && bad_a) ? base + j + 1 : fail;
+  a = bad_a ? 1.0f : a;
+  const float ra = rsqrt_approx(a);
+  const float l00 = __fmul_rn(a, ra), l10 = __fmul_rn(b, ra);
+  float c2 = __fmaf_rn(-l10, l10, c);
+  const bool bad_c = !(c2 > 0.0f);
+  fail = (fail == 0 && bad_c) ? base + j + 2 : fail;
+  c2 = bad_c ? 1.0f : c2;
+  const float rc = rsqrt_approx(c2);
+  const float l11 = __fmul_rn(c2, rc);
+  const float x0 = __fmul_rn(r[j], ra);
+  const float x1 = __fmul_rn(__fmaf_rn(-x0, l10, r[j + 1]), rc);
+  v0 = lane == j ? l00 : (lane == j + 1 ? l10 : (lane > j + 1 ? x0 : 0.0f));
+  v1 = lane == j + 1 ? l11 : (lane > j + 1 ? x1 : 0.0f);
+  r[j] = v0;
+  r[j + 1] = v1;
+  zj = __fmul_rn(z[j], ra);
+  zj1 = __fmul_rn(__fmaf_rn(-l10, zj, z[j + 1]), rc);
+  z[j] = zj;
+  z[j + 1] = zj1;
+}
+
+// Rows k and k + 1 of this lane's row and Z column take the pivot pair's update; cb holds
+// the pairs (L_kj, L_k,j+1) of every row.
+__device__ __forceinline__ void update_pair(float (&r)[kSub], float (&z)[kSub], const int k, const float* cb,
+                                            float v0, float v1, float zj, float zj1) {
+  const float4 q = *reinterpret_cast<const float4*>(cb + 2 * k);  // (L_kj, L_k,j+1, L_k+1,j, L_k+1,j+1)
+  r[k] = __fmaf_rn(-v0, q.x, __fmaf_rn(-v1, q.y, r[k]));
+  r[k + 1] = __fmaf_rn(-v0, q.z, __fmaf_rn(-v1, q.w, r[k + 1]));
+  z[k] = __fmaf_rn(-q.x, zj, __fmaf_rn(-q.y, zj1, z[k]));
+  z[k + 1] = __fmaf_rn(-q.z, zj, __fmaf_rn(-q.w, zj1, z[k + 1]));
+}
+
 __device__ __noinline__ void factor_sub32(float* A, float* Zo, float* Zt, float* col, int lane, int32_t* info,
                                           int32_t base) {
-  const unsigned full = 0xFFFFFFFFu;
   float r[kSub], z[kSub];
 #pragma unroll
-  for (int k = 0; k < kSub; ++k) {
-    r[k] = A[lane * kLd + k];
-    z[k] = k == lane ? 1.0f : 0.0f;
-  }
-  float2* col2 = reinterpret_cast<float2*>(col);
-#pragma unroll
-  for (int j = 0; j < kSub; j += 2) {
-    float a = __shfl_sync(full, r[j], j);
-    const float b = __shfl_sync(full, r[j], j + 1);
-    float c = __shfl_sync(full, r[j + 1], j + 1);
-    if (!(a > 0.0f)) {
-      if (lane == 0) record_failure(info, base + j + 1);
-      a = 1.0f;
-    }
-    const float ra = rsqrt_approx(a);
-    const float l00 = __fmul_rn(a, ra), l10 = __fmul_rn(b, ra);
-    float c2 = __fmaf_rn(-l10, l10, c);
-    if (!(c2 > 0.0f)) {
-      if (lane == 0) record_failure(info, base + j + 2);
-      c2 = 1.0f;
-    }
-    const float rc = rsqrt_approx(c2);
-    const float l11 = __fmul_rn(c2, rc);
-    // this lane's entries of columns j and j + 1
-    const float x0 = __fmul_rn(r[j], ra);
-    const float x1 = __fmul_rn(__fmaf_rn(-x0, l10, r[j + 1]), rc);
-    const float v0 = lane == j ? l00 : (lane == j + 1 ? l10 : (lane > j + 1 ? x0 : 0.0f));
-    const float v1 = lane == j + 1 ? l11 : (lane > j + 1 ? x1 : 0.0f);
-    r[j] = v0;
-    r[j + 1] = v1;
-    // rows j and j + 1 of Z in this lane's column (1 / L_jj = ra, 1 / L_j+1,j+1 = rc)
-    const float zj = __fmul_rn(z[j], ra);
-    const float zj1 = __fmul_rn(__fmaf_rn(-l10, zj, z[j + 1]), rc);
-    z[j] = zj;
-    z[j + 1] = zj1;
-    if (j + 2 < kSub) {
-      col2[lane] = make_float2(v0, v1);
-      __syncwarp();
-#pragma unroll
-      for (int k = j + 2; k < kSub; k += 2) {
-        const float4 q = *reinterpret_cast<const float4*>(col + 2 * k);  // (L_kj, L_k,j+1, L_k+1,j, L_k+1,j+1)
-        r[k] = __fmaf_rn(-v0, q.x, __fmaf_rn(-v1, q.y, r[k]));
-        r[k + 1] = __fmaf_rn(-v0, q.z, __fmaf_rn(-v1, q.w, r[k + 1]));
-        z[k] = __fmaf_rn(-q.x, zj, __fmaf_rn(-q.y, zj1, z[k]));
-        z[k + 1] = __fmaf_rn(-q.z, zj, __fmaf_rn(-q.w, zj1, z[k + 1]));
-      }
-      __syncwarp();
-    }
+  for (int k = 0; k < kSub; k += 4) {
+    const float4 a = *reinterpret_cast<const float4*>(A + lane * kLd + k);
+    r[k] = a.x;
+    r[k + 1] = a.y;
+    r[k + 2] = a.z;
+    r[k + 3] = a.w;
   }
 #pragma unroll
-  for (int k = 0; k < kSub; ++k) A[lane * kLd + k] = k <= lane ? r[k] : 0.0f;
+  for (int k = 0; k < kSub; ++k) z[k] = k == lane ? 1.0f : 0.0f;
+  int32_t fail = 0;
+  float v0, v1, zj, zj1;
+  pivot_pair(r, z, 0, lane, base, fail, v0, v1, zj, zj1);
+#pragma unroll
+  for (int j = 0; j + 2 < kSub; j += 2) {
+    float* cb = col + ((j >> 1) & 1) * (2 * kSub);
+    reinterpret_cast<float2*>(cb)[lane] = make_float2(v0, v1);
+    __syncwarp();
+    update_pair(r, z, j + 2, cb, v0, v1, zj, zj1);
+    float n0, n1, nz0, nz1;
+    pivot_pair(r, z, j + 2, lane, base, fail, n0, n1, nz0, nz1);
+#pragma unroll
+    for (int k = j + 4; k < kSub; k += 2) update_pair(r, z, k, cb, v0, v1, zj, zj1);
+    v0 = n0;
+    v1 = n1;
+    zj = nz0;
+    zj1 = nz1;
+  }
+  if (fail != 0 && lane == 0) record_failure(info, fail);
+#pragma unroll
+  for (int k = 0; k < kSub; k += 4)
+    *reinterpret_cast<float4*>(A + lane * kLd + k) =
+        make_float4(k <= lane ? r[k] : 0.0f, k + 1 <= lane ? r[k + 1] : 0.0f, k + 2 <= lane ? r[k + 2] : 0.0f,
+                    k + 3 <= lane ? r[k + 3] : 0.0f);
   // lane c holds column c of Z: row i is zero above the diagonal (i < c)
 #pragma unroll
   for (int i = 0; i < kSub; ++i) {
     const float x = i >= lane ? z[i] : 0.0f;
+    z[i] = x;
     Zo[i * kLd + lane] = x;
-    Zt[lane * kLd + i] = x;
   }
+#pragma unroll
+  for (int i = 0; i < kSub; i += 4)
+    *reinterpret_cast<float4*>(Zt + lane * kLd + i) = make_float4(z[i], z[i + 1], z[i + 2], z[i + 3]);
 }
 
 // Warp-tile products on 32 x 32 tiles in shared memory (row stride kLd, a multiple of 4): a
@@ -249,9 +280,12 @@ constexpr int kQ = 8;                     // rows of a tile per warp (four warps
 //   (a) warp 0 factors the tile on the diagonal and inverts it (factor_sub32);
 //   (b) the tiles below it: L_ip = B_ip Z_p^T, one warp per tile;
 //   (c) the tiles of the rest of the block: B_ik -= L_ip L_kp^T, one warp per tile.
-// Then the inverse of the block, tile row q = 1..3: T_qr = sum_{m=r}^{q-1} L_qm X_mr and
-// X_qr = -Z_q T_qr, one warp per tile.  The transposes a tile product needs (Z_p^T, L_kp^T)
-// are written next to the tiles.
+// The inverse of the block is built by tile rows q = 1..3, X_qr = -Z_q T_qr with
+// T_qr = sum_{m=r}^{q-1} L_qm X_mr (r < q), on warps 4..15 while warp 0 runs (a): T_qr needs
+// only the tile columns m < q, and X_qr only Z_q besides, so during (a) of step p they form
+// row p - 1 (its X) and then row p (its T); row 3's X follows the sweep.  The T tiles sit in
+// St's first tile row, which step 0 alone uses otherwise.  The transposes a tile product
+// needs (Z_p^T, L_kp^T) are written next to the tiles.
 __global__ void __launch_bounds__(kDiagThreads, 1)
 factor_diag_kernel(const float* __restrict__ Bw, int64_t ld, int64_t j0, float* __restrict__ Xw,
                    int32_t* __restrict__ info) {
@@ -259,7 +293,7 @@ factor_diag_kernel(const float* __restrict__ Bw, int64_t ld, int64_t j0, float* 
   float* S = sm;                 // [128][kLd] the block, then L (lower)
   float* X = S + kNb * kLd;      // [128][kLd] the inverse (lower)
   float* St = X + kNb * kLd;     // [128][kLd] transposes: Z_p^T in its diagonal tile, L^T
-  float* col = St + kNb * kLd;   // [64] the pivot columns of factor_sub32
+  float* col = St + kNb * kLd;   // [128] the pivot columns of factor_sub32
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
   const int part = warp & 3;     // which 8 rows of its tile a warp computes
   const int unit = warp >> 2;    // which tile (of up to four at a time)
@@ -275,24 +309,48 @@ factor_diag_kernel(const float* __restrict__ Bw, int64_t ld, int64_t j0, float* 
   }
   __syncthreads();
 
+  const int i0 = kQ * part;      // this warp's first row within its tile
   for (int p = 0; p < kNb / kSub; ++p) {
     const int c0 = p * kSub;
-    if (warp == 0)
+    if (warp == 0) {
       factor_sub32(S + c0 * kLd + c0, X + c0 * kLd + c0, St + c0 * kLd + c0, col, lane, info, (int32_t)(j0 + c0));
+    } else if (unit >= 1 && p >= 1) {
+      const int u = unit - 1;    // the tile column r = u of the inverse's row
+      if (p >= 2) {
+        // X_qr = -Z_q T_qr for q = p - 1
+        const int q0 = (p - 1) * kSub;
+        if (u < p - 1) {
+          float acc[kQ];
+          tile_zero(acc);
+          tile_nn<kQ>(acc, X + (q0 + i0) * kLd + q0, St + u * kSub, lane);
+          tile_store(acc, X + (q0 + i0) * kLd + u * kSub, lane, -1.0f);
+        }
+        asm volatile("bar.sync 1, 384;" ::: "memory");  // warps 4..15: X_q done, T tiles free
+      }
+      // T_pr = sum_{m=r}^{p-1} L_pm X_mr
+      if (u < p) {
+        float acc[kQ];
+        tile_zero(acc);
+        for (int m = u; m < p; ++m)
+          tile_nn<kQ>(acc, S + (c0 + i0) * kLd + m * kSub, X + m * kSub * kLd + u * kSub, lane);
+        tile_store(acc, St + i0 * kLd + u * kSub, lane, 1.0f);
+      }
+    }
     __syncthreads();
     // (b) tiles below: L_ip = B_ip Z_p^T, four warps per tile
     const int below = kNb / kSub - 1 - p;
     if (unit < below) {
-      const int i0 = c0 + kSub * (1 + unit) + kQ * part;  // this warp's first row
+      const int r0 = c0 + kSub * (1 + unit) + i0;  // this warp's first row
       float acc[kQ];
       tile_zero(acc);
-      tile_nn<kQ>(acc, S + i0 * kLd + c0, St + c0 * kLd + c0, lane);
+      tile_nn<kQ>(acc, S + r0 * kLd + c0, St + c0 * kLd + c0, lane);
       __syncwarp();
-      tile_store(acc, S + i0 * kLd + c0, lane, 1.0f);
-      // the transpose L_ip^T, for (c): St[c0 + c][i0 + r] = L_ip[r][c]
-      *reinterpret_cast<float4*>(St + (c0 + lane) * kLd + i0) = make_float4(acc[0], acc[1], acc[2], acc[3]);
-      *reinterpret_cast<float4*>(St + (c0 + lane) * kLd + i0 + 4) = make_float4(acc[4], acc[5], acc[6], acc[7]);
+      tile_store(acc, S + r0 * kLd + c0, lane, 1.0f);
+      // the transpose L_ip^T, for (c): St[c0 + c][r0 + r] = L_ip[r][c]
+      *reinterpret_cast<float4*>(St + (c0 + lane) * kLd + r0) = make_float4(acc[0], acc[1], acc[2], acc[3]);
+      *reinterpret_cast<float4*>(St + (c0 + lane) * kLd + r0 + 4) = make_float4(acc[4], acc[5], acc[6], acc[7]);
     }
+    if (below == 0) break;
     __syncthreads();
     // (c) tiles (i, k), p < k <= i: B_ik -= L_ip L_kp^T = L_ip (L_kp^T), four warps per tile;
     // up to six tiles, so the sixteen warps take them in two rounds
@@ -303,37 +361,25 @@ factor_diag_kernel(const float* __restrict__ Bw, int64_t ld, int64_t j0, float* 
         ++i;
       }
       if (i < kNb / kSub) {
-        const int k0 = (p + 1 + t) * kSub, i0 = i * kSub + kQ * part;
+        const int k0 = (p + 1 + t) * kSub, r0 = i * kSub + i0;
         float acc[kQ];
-        tile_load(acc, S + i0 * kLd + k0, lane);
-        tile_nn<kQ, true>(acc, S + i0 * kLd + c0, St + c0 * kLd + k0, lane);
-        tile_store(acc, S + i0 * kLd + k0, lane, 1.0f);
+        tile_load(acc, S + r0 * kLd + k0, lane);
+        tile_nn<kQ, true>(acc, S + r0 * kLd + c0, St + c0 * kLd + k0, lane);
+        tile_store(acc, S + r0 * kLd + k0, lane, 1.0f);
       }
     }
     __syncthreads();
   }
 
-  // inverse of the whole block, tile row q = 1..3; T tiles kept in St's first tile row
-  for (int q = 1; q < kNb / kSub; ++q) {
-    const int q0 = q * kSub;
-    if (unit < q) {
-      const int r0 = unit * kSub, i0 = kQ * part;
-      float acc[kQ];
-      tile_zero(acc);
-      for (int m = unit; m < q; ++m)
-        tile_nn<kQ>(acc, S + (q0 + i0) * kLd + m * kSub, X + m * kSub * kLd + r0, lane);
-      tile_store(acc, St + i0 * kLd + r0, lane, 1.0f);
-    }
-    __syncthreads();
-    if (unit < q) {
-      const int r0 = unit * kSub, i0 = kQ * part;
-      float acc[kQ];
-      tile_zero(acc);
-      tile_nn<kQ>(acc, X + (q0 + i0) * kLd + q0, St + r0, lane);
-      tile_store(acc, X + (q0 + i0) * kLd + r0, lane, -1.0f);
-    }
-    __syncthreads();
+  // the inverse's last tile row: X_3r = -Z_3 T_3r
+  if (unit < kNb / kSub - 1) {
+    const int q0 = kNb - kSub;
+    float acc[kQ];
+    tile_zero(acc);
+    tile_nn<kQ>(acc, X + (q0 + i0) * kLd + q0, St + unit * kSub, lane);
+    tile_store(acc, X + (q0 + i0) * kLd + unit * kSub, lane, -1.0f);
   }
+  __syncthreads();
 
   // write-out: Z into Xw's diagonal block (16-byte words).  L_jj itself is not needed again:
   // the panel uses Z_jj, and the rest of the sweep reads only the blocks below the diagonal.
