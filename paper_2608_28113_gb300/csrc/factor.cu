@@ -504,38 +504,42 @@ __device__ __forceinline__ void split3(float x, uint16_t (&p)[3]) {
   p[2] = __bfloat16_as_ushort(c);
 }
 
-// The panel P [rows, 128] (fp32) into its place in Bw (rows r_first.., columns j0..) and as
-// the two operands of the updates: An = [-P1 | -P1 | -P2 | -P1 | -P2 | -P3] and
+// Both split operands of a step's update in one launch.  Blocks [0, panel_blocks): the panel
+// P [rows, 128] (fp32) into its place in Bw (rows r_first.., columns j0..) and as the two
+// operands of the updates: An = [-P1 | -P1 | -P2 | -P1 | -P2 | -P3] and
 // Bp = [P1 | P2 | P1 | P3 | P2 | P1] (rows of 6 * 128 bf16), so that An Bp^T = -P P^T to fp32
-// accuracy (the six products E1U1, E1U2, E2U1, E1U3, E2U2, E3U1).
-__global__ void __launch_bounds__(256) factor_split_panel_kernel(const float* __restrict__ P, int64_t rows,
-                                                                 float* __restrict__ Bw, int64_t ld, int64_t r_first,
-                                                                 int64_t j0, uint16_t* __restrict__ An,
-                                                                 uint16_t* __restrict__ Bp) {
-  const int64_t total = rows * kNb;
-  for (int64_t e = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; e < total; e += (int64_t)gridDim.x * blockDim.x) {
-    const int64_t i = e >> 7;
-    const int k = (int)(e & (kNb - 1));
-    const float x = P[e];
-    Bw[(r_first + i) * ld + j0 + k] = x;
-    uint16_t p[3], q[3];
-    split3(x, p);
-    split3(-x, q);
-    uint16_t* a = An + i * kSplitK + k;
-    uint16_t* b = Bp + i * kSplitK + k;
-    a[0] = q[0]; a[kNb] = q[0]; a[2 * kNb] = q[1]; a[3 * kNb] = q[0]; a[4 * kNb] = q[1]; a[5 * kNb] = q[2];
-    b[0] = p[0]; b[kNb] = p[1]; b[2 * kNb] = p[0]; b[3 * kNb] = p[2]; b[4 * kNb] = p[1]; b[5 * kNb] = p[0];
+// accuracy (the six products E1U1, E1U2, E2U1, E1U3, E2U2, E3U1).  The blocks after them: the
+// inverse's row block j (Xw rows j0..j0+127, columns 0..cols-1) transposed, as the B operand
+// of the R update: Bx[c] = [X1 | X2 | X1 | X3 | X2 | X1] of column c of the row block, one
+// 32 x 32 tile per block (4 tiles per 32 columns) through shared memory (coalesced reads
+// along c, writes along the row index).  The two parts are independent.
+__global__ void __launch_bounds__(256) factor_split_kernel(const float* __restrict__ P, int64_t rows,
+                                                           float* __restrict__ Bw, const float* __restrict__ Xw,
+                                                           int64_t ld, int64_t r_first, int64_t j0, int64_t cols,
+                                                           int panel_blocks, uint16_t* __restrict__ An,
+                                                           uint16_t* __restrict__ Bp, uint16_t* __restrict__ Bx) {
+  if ((int)blockIdx.x < panel_blocks) {
+    const int64_t total = rows * kNb;
+    for (int64_t e = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; e < total;
+         e += (int64_t)panel_blocks * blockDim.x) {
+      const int64_t i = e >> 7;
+      const int k = (int)(e & (kNb - 1));
+      const float x = P[e];
+      Bw[(r_first + i) * ld + j0 + k] = x;
+      uint16_t p[3], q[3];
+      split3(x, p);
+      split3(-x, q);
+      uint16_t* a = An + i * kSplitK + k;
+      uint16_t* b = Bp + i * kSplitK + k;
+      a[0] = q[0]; a[kNb] = q[0]; a[2 * kNb] = q[1]; a[3 * kNb] = q[0]; a[4 * kNb] = q[1]; a[5 * kNb] = q[2];
+      b[0] = p[0]; b[kNb] = p[1]; b[2 * kNb] = p[0]; b[3 * kNb] = p[2]; b[4 * kNb] = p[1]; b[5 * kNb] = p[0];
+    }
+    return;
   }
-}
-
-// The inverse's row block j (Xw rows j0..j0+127, columns 0..cols-1) transposed, as the B
-// operand of the R update: Bx[c] = [X1 | X2 | X1 | X3 | X2 | X1] of column c of the row block,
-// through 32 x 32 shared-memory tiles (coalesced reads along c, writes along the row index).
-__global__ void __launch_bounds__(256) factor_split_row_kernel(const float* __restrict__ Xw, int64_t ld, int64_t j0,
-                                                               int64_t cols, uint16_t* __restrict__ Bx) {
   __shared__ float t[32][33];
-  const int64_t c0 = (int64_t)blockIdx.x * 32;
-  const int m0 = blockIdx.y * 32;
+  const int rb = (int)blockIdx.x - panel_blocks;
+  const int64_t c0 = (int64_t)(rb >> 2) * 32;
+  const int m0 = (rb & 3) * 32;
   const int tx = threadIdx.x & 31, ty = threadIdx.x >> 5;
   for (int mm = ty; mm < 32; mm += 8) t[mm][tx] = c0 + tx < cols ? Xw[(j0 + m0 + mm) * ld + c0 + tx] : 0.0f;
   __syncthreads();
@@ -608,13 +612,12 @@ cudaError_t launch_gptq_factor(const float* H, int64_t n, int64_t ld_h, float da
       if ((err = cudaGetLastError()) != cudaSuccess) return err;
     }
     if (rows == 0) break;
-    const unsigned sblocks = (unsigned)std::max<int64_t>(1, std::min<int64_t>((rows * kNb + 255) / 256,
-                                                                             (int64_t)dinfo.sm_count * 8));
-    factor_split_panel_kernel<<<sblocks, 256, 0, stream>>>(P, rows, Bw, ld, r_first, j0, An, Bo);
-    if ((err = cudaGetLastError()) != cudaSuccess) return err;
+    const int sblocks = (int)std::max<int64_t>(1, std::min<int64_t>((rows * kNb + 255) / 256,
+                                                                    (int64_t)dinfo.sm_count * 8));
     const int64_t xcols = j0 + kNb;            // columns of the inverse's row block j, diagonal included
-    factor_split_row_kernel<<<dim3((unsigned)((xcols + 31) / 32), kNb / 32), 256, 0, stream>>>(
-        Xw, ld, j0, xcols, Bo + rows * kSplitK);
+    const int64_t rblocks = (xcols + 31) / 32 * (kNb / 32);
+    factor_split_kernel<<<(unsigned)(sblocks + rblocks), 256, 0, stream>>>(P, rows, Bw, Xw, ld, r_first, j0, xcols,
+                                                                           sblocks, An, Bo, Bo + rows * kSplitK);
     if ((err = cudaGetLastError()) != cudaSuccess) return err;
     // rows below the diagonal block, columns r_first .. np + xcols of W2 (rows + xcols = np):
     // the trailing square and the inverse's rows, -= L_:j [L_:j ; X_j,:]^T
