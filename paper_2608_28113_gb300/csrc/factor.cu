@@ -35,6 +35,7 @@
 #include <algorithm>
 
 #include "hscale_internal.h"
+#include "tma.cuh"
 
 namespace hscale {
 namespace {
@@ -298,6 +299,10 @@ factor_diag_kernel(const float* __restrict__ Bw, int64_t ld, int64_t j0, float* 
   const int part = warp & 3;     // which 8 rows of its tile a warp computes
   const int unit = warp >> 2;    // which tile (of up to four at a time)
 
+  // programmatic dependent launch: the strips may be scheduled now; the previous step's update
+  // must have finished before the block is read
+  pdl_launch_dependents();
+  pdl_wait_primary();
   const float* blk = Bw + j0 * ld + j0;
   // independent 16-byte loads per thread in flight
 #pragma unroll 4
@@ -405,6 +410,9 @@ factor_diag_kernel(const float* __restrict__ Bw, int64_t ld, int64_t j0, float* 
 __global__ void __launch_bounds__(kStripThreads)
 factor_strip_kernel(const float* __restrict__ Bw, float* __restrict__ Xw, int64_t ld, int64_t j0,
                     float* __restrict__ P, int panel_strips, int64_t r_first) {
+  // launched in stream order (scheduled early, beside the diagonal block's CTA, the strips ran
+  // slower); lets the split kernel be scheduled
+  pdl_launch_dependents();
   extern __shared__ __align__(16) float sm[];
   constexpr int kZl = kNb + 4;       // row-major Z for the row strips (16-byte rows)
   constexpr int kZp = kNb + 1;       // row-major Z for the panel (column reads across lanes)
@@ -518,6 +526,8 @@ __global__ void __launch_bounds__(256) factor_split_kernel(const float* __restri
                                                            int64_t ld, int64_t r_first, int64_t j0, int64_t cols,
                                                            int panel_blocks, uint16_t* __restrict__ An,
                                                            uint16_t* __restrict__ Bp, uint16_t* __restrict__ Bx) {
+  pdl_launch_dependents();
+  pdl_wait_primary();  // the strips' panel and row (programmatic dependent launch)
   if ((int)blockIdx.x < panel_blocks) {
     const int64_t total = rows * kNb;
     for (int64_t e = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; e < total;
@@ -554,6 +564,29 @@ __global__ void __launch_bounds__(256) factor_split_kernel(const float* __restri
 }
 
 inline int64_t round256(int64_t bytes) { return (bytes + 255) / 256 * 256; }
+
+// The diagonal block, split and update kernels are launched with programmatic dependent launch:
+// the kernel before each lets it be scheduled as soon as it starts, and it waits for that
+// kernel's writes before its first read, so those launches do not each wait out a launch's
+// latency (n = 4096: 1.92 -> 1.88 ms).  The strips are launched in stream order: scheduled
+// early, beside the diagonal block, they made the sweep 4 % slower.
+template <typename... KArgs, typename... Args>
+cudaError_t launch_chained(void (*kernel)(KArgs...), unsigned grid, unsigned block, int smem, cudaStream_t stream,
+                           Args... args) {
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3(grid, 1, 1);
+  cfg.blockDim = dim3(block, 1, 1);
+  cfg.dynamicSmemBytes = (size_t)smem;
+  cfg.stream = stream;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  cudaError_t err = cudaLaunchKernelEx(&cfg, kernel, static_cast<KArgs>(args)...);
+  if (err != cudaSuccess) return err;
+  return cudaGetLastError();
+}
 
 }  // namespace
 
@@ -602,8 +635,9 @@ cudaError_t launch_gptq_factor(const float* H, int64_t n, int64_t ld_h, float da
     const int64_t j0 = jb * kNb;
     const int64_t r_first = j0 + kNb;          // first row below the diagonal block
     const int64_t rows = np - r_first;         // rows of the panel
-    factor_diag_kernel<<<1, kDiagThreads, kDiagSmemBytes, stream>>>(Bw, ld, j0, Xw, info);
-    if ((err = cudaGetLastError()) != cudaSuccess) return err;
+    if ((err = launch_chained(factor_diag_kernel, 1, kDiagThreads, kDiagSmemBytes, stream, (const float*)Bw, ld, j0,
+                              Xw, info)) != cudaSuccess)
+      return err;
     const int panel_strips = (int)(rows / kStripRows);
     const int row_strips = (int)(j0 / kStripRows);
     if (panel_strips + row_strips > 0) {
@@ -616,13 +650,14 @@ cudaError_t launch_gptq_factor(const float* H, int64_t n, int64_t ld_h, float da
                                                                     (int64_t)dinfo.sm_count * 8));
     const int64_t xcols = j0 + kNb;            // columns of the inverse's row block j, diagonal included
     const int64_t rblocks = (xcols + 31) / 32 * (kNb / 32);
-    factor_split_kernel<<<(unsigned)(sblocks + rblocks), 256, 0, stream>>>(P, rows, Bw, Xw, ld, r_first, j0, xcols,
-                                                                           sblocks, An, Bo, Bo + rows * kSplitK);
-    if ((err = cudaGetLastError()) != cudaSuccess) return err;
+    if ((err = launch_chained(factor_split_kernel, (unsigned)(sblocks + rblocks), 256, 0, stream, (const float*)P, rows,
+                              Bw, (const float*)Xw, ld, r_first, j0, xcols, sblocks, An, Bo, Bo + rows * kSplitK)) !=
+        cudaSuccess)
+      return err;
     // rows below the diagonal block, columns r_first .. np + xcols of W2 (rows + xcols = np):
     // the trailing square and the inverse's rows, -= L_:j [L_:j ; X_j,:]^T
-    if ((err = launch_gemm_accumulate(An, Bo, rows, rows + xcols, kSplitK, Bw + r_first * ld + r_first, ld,
-                                      stream)) != cudaSuccess)
+    if ((err = launch_gemm_accumulate(An, Bo, rows, rows + xcols, kSplitK, Bw + r_first * ld + r_first, ld, stream,
+                                      true)) != cudaSuccess)
       return err;
   }
   reverse_out_kernel<<<eblocks, 256, 0, stream>>>(Xw, ld, n, Uo);

@@ -105,8 +105,10 @@ cudaError_t launch_gptq_factor(const float* H, int64_t n, int64_t ld_h, float da
                                int32_t* info, void* workspace, cudaStream_t stream);
 // C[m, nn] (row stride ld_c, fp32) += A B^T on the tensor cores, with A [m, k] and B [nn, k]
 // bf16, rows of k elements contiguous (k % 8 == 0, 16-byte aligned bases); every tile.
+// programmatic: launched with programmatic dependent launch (the kernel waits for the
+// previous kernel on the stream before its first load, and lets the next one be scheduled).
 cudaError_t launch_gemm_accumulate(const void* a, const void* b, int64_t m, int64_t nn, int64_t k, float* C,
-                                   int64_t ld_c, cudaStream_t stream);
+                                   int64_t ld_c, cudaStream_t stream, bool programmatic = false);
 
 cudaError_t launch_gptq_hscale(const void* w, int64_t m, int64_t n, const float* U, const float* h,
                                const float* global_scale, const uint8_t* dead, int block, int down, int up,

@@ -231,6 +231,13 @@ gemm_kernel(const __grid_constant__ CUtensorMap xmap, const __grid_constant__ CU
   __syncthreads();
   tc_fence_after_sync();
   const uint32_t tmem_d = *tmem_slot;
+  if (kMode == 2) {
+    // launched with programmatic dependent launch by the factor's sweep: let the next kernel
+    // be scheduled (after the TMEM allocation), then wait for the previous one's writes
+    // before the first load; without the launch attribute both are no-ops
+    pdl_launch_dependents();
+    pdl_wait_primary();
+  }
 
   if (warp == 0) {
     if (lane == 0) {
@@ -622,7 +629,7 @@ cudaError_t launch_hessian_full(const void* x, int64_t tokens, int64_t n, int64_
 }
 
 cudaError_t launch_gemm_accumulate(const void* a, const void* b, int64_t m, int64_t nn, int64_t k, float* C,
-                                   int64_t ld_c, cudaStream_t stream) {
+                                   int64_t ld_c, cudaStream_t stream, bool programmatic) {
   EncodeTiledFn encode = nullptr;
   cudaError_t err = encode_tiled_fn(&encode);
   if (err != cudaSuccess) return err;
@@ -657,8 +664,19 @@ cudaError_t launch_gemm_accumulate(const void* a, const void* b, int64_t m, int6
   DeviceInfo info;
   if ((err = current_device_info(&info)) != cudaSuccess) return err;
   const int64_t grid = std::max<int64_t>(1, std::min<int64_t>(tiles, info.sm_count));
-  gemm_kernel<2><<<(unsigned)grid, kGemmThreads, kUpdateSmemBytes, stream>>>(
-      amap, bmap, cmap, (int)((k + kBK - 1) / kBK), (int)tiles_n, (int)tiles, nullptr, C, m, nn, ld_c);
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3((unsigned)grid, 1, 1);
+  cfg.blockDim = dim3(kGemmThreads, 1, 1);
+  cfg.dynamicSmemBytes = kUpdateSmemBytes;
+  cfg.stream = stream;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = programmatic ? 1 : 0;
+  err = cudaLaunchKernelEx(&cfg, gemm_kernel<2>, amap, bmap, cmap, (int)((k + kBK - 1) / kBK), (int)tiles_n,
+                           (int)tiles, (double*)nullptr, C, m, nn, ld_c);
+  if (err != cudaSuccess) return err;
   return cudaGetLastError();
 }
 
