@@ -410,8 +410,8 @@ int hscale_output_error(const void* x_bf16, int64_t tokens, int64_t n, int64_t l
  *    matrix is not positive definite, and U is unspecified), info[1] = info[2] = 0.  The
  *    workspace (hscale_gptq_factor_workspace_bytes, 256-byte aligned) holds the reversed
  *    matrix and the inverse side by side (2 n_pad^2 floats, n_pad = 128 ceil(n / 128)) and
- *    the split operands of the updates.  U's buffer also serves as scratch for the damped
- *    copy of H during the call.  n <= 65536.
+ *    the split operands of the updates.  U is written only at the end of the call.
+ *    n <= 65536.
  *
  * 3. hscale_gptq_hscale: for each block of `block` columns (a multiple of 16 dividing n)
  *    of the running fp32 weights (W with dead columns zeroed): the RTN codes of Eq. 7 of

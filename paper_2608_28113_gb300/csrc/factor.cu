@@ -51,16 +51,20 @@ constexpr int kStripSmemBytes = (kNb * (kNb + 4) + kNb * (kStripRows + 4)) * 4;
 constexpr int kSplitK = 6 * kNb;          // K of the split update GEMMs
 
 // ---------------------------------------------------------------- set-up
-// One block: dead channels, the mean of the diagonal, and the damping added to it.  A is the
-// n x n copy of H (row stride n).
-__global__ void __launch_bounds__(1024) damp_diagonal_kernel(float* A, int64_t n, float damp, uint8_t* dead) {
+// One block: dead channels (H_jj = 0) and the damped diagonal dd_j = d_j + damp * mean(d),
+// d_j = H_jj, or 1 for a dead channel (fp32; the mean in fp64).
+__global__ void __launch_bounds__(1024) damp_diagonal_kernel(const float* __restrict__ H, int64_t n, int64_t ld_h,
+                                                             float damp, uint8_t* __restrict__ dead,
+                                                             float* __restrict__ dd) {
   __shared__ double part[1024];
   double s = 0.0;
+#pragma unroll 4
   for (int64_t j = threadIdx.x; j < n; j += blockDim.x) {
-    float d = A[j * n + j];
+    float d = H[j * ld_h + j];
     const bool is_dead = (d == 0.0f);
-    if (is_dead) A[j * n + j] = d = 1.0f;
+    if (is_dead) d = 1.0f;
     if (dead) dead[j] = (uint8_t)is_dead;
+    dd[j] = d;
     s += (double)d;
   }
   part[threadIdx.x] = s;
@@ -70,36 +74,60 @@ __global__ void __launch_bounds__(1024) damp_diagonal_kernel(float* A, int64_t n
     __syncthreads();
   }
   const float add = (float)((double)damp * part[0] / (double)n);
-  for (int64_t j = threadIdx.x; j < n; j += blockDim.x) A[j * n + j] += add;
+  for (int64_t j = threadIdx.x; j < n; j += blockDim.x) dd[j] = dd[j] + add;
 }
 
-// W2 [n_pad, 2 n_pad]: the left half B_ij = A_{n-1-i, n-1-j} (taken from A's upper triangle)
-// for i, j < n and the identity beyond, the right half (X) zero.
-__global__ void __launch_bounds__(256) reverse_pad_kernel(const float* __restrict__ A, int64_t n, int64_t n_pad,
+// W2 [n_pad, 2 n_pad]: the left half B_ij = A_{n-1-i, n-1-j} for i, j < n, A the damped H
+// (read from H's upper triangle, row stride ld_h, and the damped diagonal dd), the identity
+// beyond n; the right half (X) zero where the sweep accumulates into it, strictly below the
+// 128-block diagonal (nothing reads X above it).  One 32 x 32 tile of each half per block.
+// Every read and write runs along a row: a tile of B below the diagonal reads H's rows
+// (reversed), a tile above it reads the mirrored tile of H and transposes it in shared
+// memory, and a tile on the diagonal reads the entries on and below it and takes the rest
+// from its own transpose.
+__global__ void __launch_bounds__(256) reverse_pad_kernel(const float* __restrict__ H, int64_t n, int64_t ld_h,
+                                                          const float* __restrict__ dd, int64_t n_pad,
                                                           float* __restrict__ W2) {
-  const int64_t total = n_pad * n_pad;
-  for (int64_t e = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; e < total; e += (int64_t)gridDim.x * blockDim.x) {
-    const int64_t i = e / n_pad, j = e - i * n_pad;
-    float v;
-    if (i < n && j < n) {
-      const int64_t p = n - 1 - i, q = n - 1 - j;
-      v = p <= q ? A[p * n + q] : A[q * n + p];
-    } else {
-      v = (i == j) ? 1.0f : 0.0f;
+  __shared__ float t[32][33];
+  const int bi = (int)blockIdx.y, bj = (int)blockIdx.x;
+  const int64_t i0 = 32 * (int64_t)bi, j0 = 32 * (int64_t)bj, ld = 2 * n_pad;
+  const int tx = threadIdx.x & 31, ty = threadIdx.x >> 5;
+  if (bi < bj) {
+    // B_ij = A_{n-1-j, n-1-i}: t[jj][ii]
+    for (int jj = ty; jj < 32; jj += 8) {
+      const int64_t j = j0 + jj, i = i0 + tx;
+      t[jj][tx] = (i < n && j < n) ? H[(n - 1 - j) * ld_h + (n - 1 - i)] : 0.0f;
     }
-    W2[i * 2 * n_pad + j] = v;
-    W2[i * 2 * n_pad + n_pad + j] = 0.0f;
+    __syncthreads();
+    for (int ii = ty; ii < 32; ii += 8) W2[(i0 + ii) * ld + j0 + tx] = t[tx][ii];  // i < j: 0 beyond n
+  } else {
+    // B_ij = A_{n-1-i, n-1-j} for i >= j: t[ii][jj]
+    for (int ii = ty; ii < 32; ii += 8) {
+      const int64_t i = i0 + ii, j = j0 + tx;
+      t[ii][tx] = (i < n && j < n && i >= j) ? H[(n - 1 - i) * ld_h + (n - 1 - j)] : 0.0f;
+    }
+    __syncthreads();
+    for (int ii = ty; ii < 32; ii += 8) {
+      const int64_t i = i0 + ii, j = j0 + tx;
+      float v;
+      if (i < n && j < n)
+        v = i == j ? dd[n - 1 - i] : (i > j ? t[ii][tx] : t[tx][ii]);
+      else
+        v = i == j ? 1.0f : 0.0f;
+      W2[i * ld + j] = v;
+    }
   }
+  if (bi / (kNb / 32) > bj / (kNb / 32))
+    for (int ii = ty; ii < 32; ii += 8) W2[(i0 + ii) * ld + n_pad + j0 + tx] = 0.0f;
 }
 
-// U_ij = X_{n-1-i, n-1-j} for j >= i, 0 below the diagonal (U row stride n; X row stride ld).
+// U_ij = X_{n-1-i, n-1-j} for j >= i, 0 below the diagonal (U row stride n; X row stride ld);
+// rows i = blockIdx.y, + gridDim.y, ...
 __global__ void __launch_bounds__(256) reverse_out_kernel(const float* __restrict__ Xw, int64_t ld, int64_t n,
                                                           float* __restrict__ U) {
-  const int64_t total = n * n;
-  for (int64_t e = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; e < total; e += (int64_t)gridDim.x * blockDim.x) {
-    const int64_t i = e / n, j = e - i * n;
-    U[e] = j >= i ? Xw[(n - 1 - i) * ld + (n - 1 - j)] : 0.0f;
-  }
+  const int64_t j = (int64_t)blockIdx.x * 256 + threadIdx.x;
+  if (j >= n) return;
+  for (int64_t i = blockIdx.y; i < n; i += gridDim.y) U[i * n + j] = j >= i ? Xw[(n - 1 - i) * ld + (n - 1 - j)] : 0.0f;
 }
 
 // ---------------------------------------------------------------- diagonal block
@@ -615,15 +643,11 @@ cudaError_t launch_gptq_factor(const float* H, int64_t n, int64_t ld_h, float da
   uint16_t* Bo = reinterpret_cast<uint16_t*>(ops + round256(np * kSplitK * 2));
 
   if ((err = cudaMemsetAsync(info, 0, 3 * sizeof(int32_t), stream)) != cudaSuccess) return err;
-  // the damped copy of H in U's buffer (n x n, row stride n)
-  if ((err = cudaMemcpy2DAsync(Uo, (size_t)n * 4, H, (size_t)ld_h * 4, (size_t)n * 4, (size_t)n,
-                               cudaMemcpyDeviceToDevice, stream)) != cudaSuccess)
-    return err;
-  damp_diagonal_kernel<<<1, 1024, 0, stream>>>(Uo, n, damp, dead);
+  // the damped diagonal, in the panel's buffer until the sweep writes the first panel
+  float* dd = P;
+  damp_diagonal_kernel<<<1, 1024, 0, stream>>>(H, n, ld_h, damp, dead, dd);
   if ((err = cudaGetLastError()) != cudaSuccess) return err;
-  const unsigned eblocks = (unsigned)std::max<int64_t>(1, std::min<int64_t>((np * np + 255) / 256,
-                                                                           (int64_t)dinfo.sm_count * 16));
-  reverse_pad_kernel<<<eblocks, 256, 0, stream>>>(Uo, n, np, Bw);
+  reverse_pad_kernel<<<dim3((unsigned)(np / 32), (unsigned)(np / 32)), 256, 0, stream>>>(H, n, ld_h, dd, np, Bw);
   if ((err = cudaGetLastError()) != cudaSuccess) return err;
   if ((err = ensure_dynamic_smem(reinterpret_cast<const void*>(factor_diag_kernel), kDiagSmemBytes)) != cudaSuccess)
     return err;
@@ -660,7 +684,8 @@ cudaError_t launch_gptq_factor(const float* H, int64_t n, int64_t ld_h, float da
                                       true)) != cudaSuccess)
       return err;
   }
-  reverse_out_kernel<<<eblocks, 256, 0, stream>>>(Xw, ld, n, Uo);
+  reverse_out_kernel<<<dim3((unsigned)((n + 255) / 256), (unsigned)std::min<int64_t>(n, 65535)), 256, 0, stream>>>(
+      Xw, ld, n, Uo);
   return cudaGetLastError();
 }
 
