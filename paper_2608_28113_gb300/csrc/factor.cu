@@ -127,6 +127,7 @@ __global__ void __launch_bounds__(256) reverse_out_kernel(const float* __restric
                                                           float* __restrict__ U) {
   const int64_t j = (int64_t)blockIdx.x * 256 + threadIdx.x;
   if (j >= n) return;
+#pragma unroll 4
   for (int64_t i = blockIdx.y; i < n; i += gridDim.y) U[i * n + j] = j >= i ? Xw[(n - 1 - i) * ld + (n - 1 - j)] : 0.0f;
 }
 
@@ -432,9 +433,11 @@ factor_diag_kernel(const float* __restrict__ Bw, int64_t ld, int64_t j0, float* 
 // Blocks [panel_strips, ...): the inverse's row j, 32 columns each, in place in Xw:
 //   X[j0 + r][c] = sum_{m <= r} Z[r][m] R[j0 + m][c]   (X_jc = Z_jj R_jc, c < j0)
 // Z = Z_jj is Xw's diagonal block.  256 threads; each computes 4 x 4 outputs over K = 128 from
-// shared memory.  The panel's columns c = tx + 32 k take Z's rows at a stride of 129 words
-// (consecutive lanes, distinct banks); the row's columns are one 16-byte word.  The staging
-// loads are unrolled so that each thread has several in flight.
+// shared memory, reading four consecutive m per 16-byte load: the panel's columns
+// c = tx + 32 k take Z's rows 132 words apart (each load spans every bank in four
+// wavefronts), the shared operand of a warp is a broadcast, and the row's columns are one
+// 16-byte word.  The sums run over m in order.  The staging loads are unrolled so that each
+// thread has several in flight.
 __global__ void __launch_bounds__(kStripThreads)
 factor_strip_kernel(const float* __restrict__ Bw, float* __restrict__ Xw, int64_t ld, int64_t j0,
                     float* __restrict__ P, int panel_strips, int64_t r_first) {
@@ -442,13 +445,12 @@ factor_strip_kernel(const float* __restrict__ Bw, float* __restrict__ Xw, int64_
   // slower); lets the split kernel be scheduled
   pdl_launch_dependents();
   extern __shared__ __align__(16) float sm[];
-  constexpr int kZl = kNb + 4;       // row-major Z for the row strips (16-byte rows)
-  constexpr int kZp = kNb + 1;       // row-major Z for the panel (column reads across lanes)
+  constexpr int kZl = kNb + 4;       // row-major Z (16-byte rows; rows 4 banks apart)
   constexpr int kRl = kStripRows + 4;
   const int tid = threadIdx.x;
   const bool panel = (int)blockIdx.x < panel_strips;
   const int sb = panel ? (int)blockIdx.x : (int)blockIdx.x - panel_strips;
-  float* Zs = sm;                    // 128 x (kZl or kZp)
+  float* Zs = sm;                    // 128 x kZl
   float* Ss = sm + kNb * kZl;        // panel: B rows (i, m), 32 x kZl; row: R (m, c), 128 x kRl
   const float* zsrc = Xw + j0 * ld + j0;
   float acc[4][4];
@@ -456,16 +458,14 @@ factor_strip_kernel(const float* __restrict__ Bw, float* __restrict__ Xw, int64_
   for (int a = 0; a < 4; ++a)
 #pragma unroll
     for (int b = 0; b < 4; ++b) acc[a][b] = 0.0f;
-  if (panel) {
 #pragma unroll 16
-    for (int e = tid; e < kNb * kNb / 4; e += kStripThreads) {
-      const int r = e >> 5, c = (e & 31) * 4;
-      const float4 v = *reinterpret_cast<const float4*>(zsrc + r * ld + c);
-      Zs[r * kZp + c] = v.x;
-      Zs[r * kZp + c + 1] = v.y;
-      Zs[r * kZp + c + 2] = v.z;
-      Zs[r * kZp + c + 3] = v.w;
-    }
+  for (int e = tid; e < kNb * kNb / 4; e += kStripThreads) {
+    const int r = e >> 5, c = (e & 31) * 4;
+    *reinterpret_cast<float4*>(Zs + r * kZl + c) = *reinterpret_cast<const float4*>(zsrc + r * ld + c);
+  }
+  // Both products run over m in order, four m per step: 16-byte loads of four consecutive m
+  // (the same address across a warp where the operand is shared: a broadcast).
+  if (panel) {
     const int64_t row0 = r_first + (int64_t)sb * kStripRows;
 #pragma unroll 4
     for (int e = tid; e < kStripRows * kNb / 4; e += kStripThreads) {
@@ -473,18 +473,24 @@ factor_strip_kernel(const float* __restrict__ Bw, float* __restrict__ Xw, int64_
       *reinterpret_cast<float4*>(Ss + i * kZl + m) = *reinterpret_cast<const float4*>(Bw + (row0 + i) * ld + j0 + m);
     }
     __syncthreads();
-    // outputs 32 rows x 128 columns: rows 4 ty .. +3, columns tx + 32 k (k < 4)
+    // outputs 32 rows x 128 columns: rows 4 ty .. +3, columns tx + 32 k (k < 4); Z's rows
+    // tx + 32 k are read four m at a time (lanes 4 banks apart: four wavefronts per load)
     const int ty = tid >> 5, tx = tid & 31;
-#pragma unroll 4
-    for (int m = 0; m < kNb; ++m) {
-      float bv[4];
+#pragma unroll 2
+    for (int m = 0; m < kNb; m += 4) {
+      float4 bv[4];
 #pragma unroll
-      for (int k = 0; k < 4; ++k) bv[k] = Zs[(tx + 32 * k) * kZp + m];
+      for (int k = 0; k < 4; ++k) bv[k] = *reinterpret_cast<const float4*>(Zs + (tx + 32 * k) * kZl + m);
 #pragma unroll
       for (int a = 0; a < 4; ++a) {
-        const float av = Ss[(4 * ty + a) * kZl + m];
+        const float4 av = *reinterpret_cast<const float4*>(Ss + (4 * ty + a) * kZl + m);
 #pragma unroll
-        for (int k = 0; k < 4; ++k) acc[a][k] = __fmaf_rn(av, bv[k], acc[a][k]);
+        for (int k = 0; k < 4; ++k) {
+          acc[a][k] = __fmaf_rn(av.x, bv[k].x, acc[a][k]);
+          acc[a][k] = __fmaf_rn(av.y, bv[k].y, acc[a][k]);
+          acc[a][k] = __fmaf_rn(av.z, bv[k].z, acc[a][k]);
+          acc[a][k] = __fmaf_rn(av.w, bv[k].w, acc[a][k]);
+        }
       }
     }
 #pragma unroll
@@ -492,11 +498,6 @@ factor_strip_kernel(const float* __restrict__ Bw, float* __restrict__ Xw, int64_
 #pragma unroll
       for (int k = 0; k < 4; ++k) P[((int64_t)sb * kStripRows + 4 * ty + a) * kNb + tx + 32 * k] = acc[a][k];
   } else {
-#pragma unroll 16
-    for (int e = tid; e < kNb * kNb / 4; e += kStripThreads) {
-      const int r = e >> 5, c = (e & 31) * 4;
-      *reinterpret_cast<float4*>(Zs + r * kZl + c) = *reinterpret_cast<const float4*>(zsrc + r * ld + c);
-    }
     const int64_t col0 = (int64_t)sb * kStripRows;
 #pragma unroll 4
     for (int e = tid; e < kNb * kStripRows / 4; e += kStripThreads) {
@@ -506,19 +507,26 @@ factor_strip_kernel(const float* __restrict__ Bw, float* __restrict__ Xw, int64_
     __syncthreads();
     // outputs 128 rows x 32 columns: rows 4 ty .. +3, columns 4 tx .. +3
     const int ty = tid >> 3, tx = tid & 7;
-#pragma unroll 4
-    for (int m = 0; m < kNb; ++m) {
-      const float4 bv = *reinterpret_cast<const float4*>(Ss + m * kRl + 4 * tx);
+#pragma unroll 2
+    for (int m = 0; m < kNb; m += 4) {
+      float4 av[4], bv[4];
+#pragma unroll
+      for (int a = 0; a < 4; ++a) av[a] = *reinterpret_cast<const float4*>(Zs + (4 * ty + a) * kZl + m);
+#pragma unroll
+      for (int q = 0; q < 4; ++q) bv[q] = *reinterpret_cast<const float4*>(Ss + (m + q) * kRl + 4 * tx);
 #pragma unroll
       for (int a = 0; a < 4; ++a) {
-        const float av = Zs[(4 * ty + a) * kZl + m];
-        acc[a][0] = __fmaf_rn(av, bv.x, acc[a][0]);
-        acc[a][1] = __fmaf_rn(av, bv.y, acc[a][1]);
-        acc[a][2] = __fmaf_rn(av, bv.z, acc[a][2]);
-        acc[a][3] = __fmaf_rn(av, bv.w, acc[a][3]);
+        const float am[4] = {av[a].x, av[a].y, av[a].z, av[a].w};
+#pragma unroll
+        for (int q = 0; q < 4; ++q) {
+          acc[a][0] = __fmaf_rn(am[q], bv[q].x, acc[a][0]);
+          acc[a][1] = __fmaf_rn(am[q], bv[q].y, acc[a][1]);
+          acc[a][2] = __fmaf_rn(am[q], bv[q].z, acc[a][2]);
+          acc[a][3] = __fmaf_rn(am[q], bv[q].w, acc[a][3]);
+        }
       }
     }
-    __syncthreads();  // every thread has read its R entries before any is overwritten
+    // R was staged into shared memory before the first barrier, so the outputs may overwrite it
 #pragma unroll
     for (int a = 0; a < 4; ++a)
       *reinterpret_cast<float4*>(Xw + (j0 + 4 * ty + a) * ld + col0 + 4 * tx) =
@@ -684,7 +692,8 @@ cudaError_t launch_gptq_factor(const float* H, int64_t n, int64_t ld_h, float da
                                       true)) != cudaSuccess)
       return err;
   }
-  reverse_out_kernel<<<dim3((unsigned)((n + 255) / 256), (unsigned)std::min<int64_t>(n, 65535)), 256, 0, stream>>>(
+  // 256 columns per block, rows strided over 512 blocks (several independent rows per thread)
+  reverse_out_kernel<<<dim3((unsigned)((n + 255) / 256), (unsigned)std::min<int64_t>(n, 512)), 256, 0, stream>>>(
       Xw, ld, n, Uo);
   return cudaGetLastError();
 }
