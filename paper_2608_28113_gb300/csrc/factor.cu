@@ -44,7 +44,7 @@ constexpr int kNb = 128;                  // block of the sweep
 constexpr int kSub = 32;                  // sub-block of the diagonal factor (one warp)
 constexpr int kLd = kNb + 4;              // padded shared-memory row (16-byte multiple)
 constexpr int kDiagThreads = 512;
-constexpr int kDiagSmemBytes = (3 * kNb * kLd + 4 * kSub) * 4;
+constexpr int kDiagSmemBytes = (2 * kNb * kLd + kSub * kLd + 4 * kSub) * 4;
 constexpr int kStripRows = 32;            // rows (or columns) of one strip
 constexpr int kStripThreads = 256;
 constexpr int kStripSmemBytes = (kNb * (kNb + 4) + kNb * (kStripRows + 4)) * 4;
@@ -143,8 +143,7 @@ __device__ __forceinline__ float rsqrt_approx(float x) {
 }
 
 // One warp factors the 32 x 32 block at A (row stride kLd, lower triangle) in place,
-// A = L L^T, and writes Z = L^-1 (lower, zeros above) at Zo and its transpose at Zt (row
-// stride kLd each); col is a 128-float scratch (two 64-float buffers).  Lane i holds row i of
+// A = L L^T, and writes Z = L^-1 (lower, zeros above) at Zo (row stride kLd); col is a 128-float scratch (two 64-float buffers).  Lane i holds row i of
 // the block in registers (every loop has a constant trip count and every register index is a
 // constant, so the row stays in registers; kept out of line: inlined into the block kernel,
 // the compiler moves the row to local memory).  Two columns are eliminated per step: the
@@ -210,7 +209,7 @@ __device__ __forceinline__ void update_pair(float (&r)[kSub], float (&z)[kSub], 
   z[k + 1] = __fmaf_rn(-q.z, zj, __fmaf_rn(-q.w, zj1, z[k + 1]));
 }
 
-__device__ __noinline__ void factor_sub32(float* A, float* Zo, float* Zt, float* col, int lane, int32_t* info,
+__device__ __noinline__ void factor_sub32(float* A, float* Zo, float* col, int lane, int32_t* info,
                                           int32_t base) {
   float r[kSub], z[kSub];
 #pragma unroll
@@ -249,84 +248,102 @@ __device__ __noinline__ void factor_sub32(float* A, float* Zo, float* Zt, float*
                     k + 3 <= lane ? r[k + 3] : 0.0f);
   // lane c holds column c of Z: row i is zero above the diagonal (i < c)
 #pragma unroll
-  for (int i = 0; i < kSub; ++i) {
-    const float x = i >= lane ? z[i] : 0.0f;
-    z[i] = x;
-    Zo[i * kLd + lane] = x;
-  }
-#pragma unroll
-  for (int i = 0; i < kSub; i += 4)
-    *reinterpret_cast<float4*>(Zt + lane * kLd + i) = make_float4(z[i], z[i + 1], z[i + 2], z[i + 3]);
+  for (int i = 0; i < kSub; ++i) Zo[i * kLd + lane] = i >= lane ? z[i] : 0.0f;
 }
 
-// Warp-tile products on 32 x 32 tiles in shared memory (row stride kLd, a multiple of 4): a
-// warp computes kR rows of the output tile, lane c column c, in acc[0..kR) (independent
-// accumulators).  A's rows are read four entries at a time (the same address in every lane: a
-// broadcast), B's row m at column c (consecutive lanes, consecutive words).
-//   acc[r] += sum_m A[r][m] B[m][c]   (acc[r] -= ... with kNeg), rows r of A from A's row 0
-template <int kR, bool kNeg = false>
-__device__ __forceinline__ void tile_nn(float (&acc)[kR], const float* A, const float* B, int lane) {
+// Warp-tile products on 32 x 32 tiles in shared memory (row stride kLd = 4 mod 32 words, a
+// multiple of 4).  A warp computes 16 rows of the output tile: lane (h = lane / 16,
+// cl = lane % 16) holds rows h + 2 r (r < 8) and columns cl, cl + 16 in acc[r][0..1]
+// (independent accumulators).  Per four m, A's rows are read as 16-byte words (two rows per
+// warp, four banks apart: one wavefront), and B either row by row (kNT false: B[m][c] at
+// B + m kLd + c; consecutive lanes, consecutive words) or, for a transposed operand, in place
+// from its rows (kNT true: B[m][c] at B + c kLd + m; lanes cl read rows cl and cl + 16 as
+// 16-byte words, four banks apart: two wavefronts each), so no transposed copy is needed.
+//   acc[r][q] += sum_m A[h + 2 r][m] B[m][cl + 16 q]   (-= with kNeg), over m in order
+template <bool kNT, bool kNeg = false>
+__device__ __forceinline__ void tile_mma(float (&acc)[8][2], const float* A, const float* B, int lane) {
+  const int h = lane >> 4, cl = lane & 15;
 #pragma unroll 2
   for (int m = 0; m < kSub; m += 4) {
-    float b0 = B[m * kLd + lane], b1 = B[(m + 1) * kLd + lane];
-    float b2 = B[(m + 2) * kLd + lane], b3 = B[(m + 3) * kLd + lane];
+    float b[4][2];
+    if (kNT) {
+      const float4 u = *reinterpret_cast<const float4*>(B + cl * kLd + m);
+      const float4 v = *reinterpret_cast<const float4*>(B + (cl + 16) * kLd + m);
+      b[0][0] = u.x; b[1][0] = u.y; b[2][0] = u.z; b[3][0] = u.w;
+      b[0][1] = v.x; b[1][1] = v.y; b[2][1] = v.z; b[3][1] = v.w;
+    } else {
+#pragma unroll
+      for (int q = 0; q < 4; ++q) {
+        b[q][0] = B[(m + q) * kLd + cl];
+        b[q][1] = B[(m + q) * kLd + cl + 16];
+      }
+    }
     if (kNeg) {
-      b0 = -b0;
-      b1 = -b1;
-      b2 = -b2;
-      b3 = -b3;
+#pragma unroll
+      for (int q = 0; q < 4; ++q) {
+        b[q][0] = -b[q][0];
+        b[q][1] = -b[q][1];
+      }
     }
 #pragma unroll
-    for (int r = 0; r < kR; ++r) {
-      const float4 a = *reinterpret_cast<const float4*>(A + r * kLd + m);
-      acc[r] = __fmaf_rn(a.x, b0, acc[r]);
-      acc[r] = __fmaf_rn(a.y, b1, acc[r]);
-      acc[r] = __fmaf_rn(a.z, b2, acc[r]);
-      acc[r] = __fmaf_rn(a.w, b3, acc[r]);
+    for (int r = 0; r < 8; ++r) {
+      const float4 a = *reinterpret_cast<const float4*>(A + (h + 2 * r) * kLd + m);
+#pragma unroll
+      for (int q = 0; q < 2; ++q) {
+        acc[r][q] = __fmaf_rn(a.x, b[0][q], acc[r][q]);
+        acc[r][q] = __fmaf_rn(a.y, b[1][q], acc[r][q]);
+        acc[r][q] = __fmaf_rn(a.z, b[2][q], acc[r][q]);
+        acc[r][q] = __fmaf_rn(a.w, b[3][q], acc[r][q]);
+      }
     }
   }
 }
-template <int kR>
-__device__ __forceinline__ void tile_zero(float (&acc)[kR]) {
+__device__ __forceinline__ void tile_zero(float (&acc)[8][2]) {
 #pragma unroll
-  for (int r = 0; r < kR; ++r) acc[r] = 0.0f;
+  for (int r = 0; r < 8; ++r) acc[r][0] = acc[r][1] = 0.0f;
 }
-template <int kR>
-__device__ __forceinline__ void tile_load(float (&acc)[kR], const float* T, int lane) {
+__device__ __forceinline__ void tile_load(float (&acc)[8][2], const float* T, int lane) {
+  const int h = lane >> 4, cl = lane & 15;
 #pragma unroll
-  for (int r = 0; r < kR; ++r) acc[r] = T[r * kLd + lane];
+  for (int r = 0; r < 8; ++r) {
+    acc[r][0] = T[(h + 2 * r) * kLd + cl];
+    acc[r][1] = T[(h + 2 * r) * kLd + cl + 16];
+  }
 }
-template <int kR>
-__device__ __forceinline__ void tile_store(const float (&acc)[kR], float* T, int lane, float sign) {
+__device__ __forceinline__ void tile_store(const float (&acc)[8][2], float* T, int lane, float sign) {
+  const int h = lane >> 4, cl = lane & 15;
 #pragma unroll
-  for (int r = 0; r < kR; ++r) T[r * kLd + lane] = sign * acc[r];
+  for (int r = 0; r < 8; ++r) {
+    T[(h + 2 * r) * kLd + cl] = sign * acc[r][0];
+    T[(h + 2 * r) * kLd + cl + 16] = sign * acc[r][1];
+  }
 }
 
-constexpr int kQ = 8;                     // rows of a tile per warp (four warps per tile)
+constexpr int kHalf = kSub / 2;           // rows of a tile per warp (two warps per tile)
 
 // Factor the 128 x 128 diagonal block at (j0, j0) of Bw and invert the factor: Z_jj = L_jj^-1
 // into Xw's diagonal block (zeros above the diagonal).  The block is a 4 x 4 grid of 32 x 32
 // tiles, taken in tile columns p = 0..3:
 //   (a) warp 0 factors the tile on the diagonal and inverts it (factor_sub32);
-//   (b) the tiles below it: L_ip = B_ip Z_p^T, one warp per tile;
-//   (c) the tiles of the rest of the block: B_ik -= L_ip L_kp^T, one warp per tile.
-// The inverse of the block is built by tile rows q = 1..3, X_qr = -Z_q T_qr with
-// T_qr = sum_{m=r}^{q-1} L_qm X_mr (r < q), on warps 4..15 while warp 0 runs (a): T_qr needs
+//   (b) the tiles below it: L_ip = B_ip Z_p^T, two warps per tile;
+//   (c) the tiles of the rest of the block: B_ik -= L_ip L_kp^T, two warps per tile (at most
+//       six tiles: one round of the sixteen warps).
+// Z_p^T and L_kp^T are read in place (the transposed form of the tile product).  The inverse
+// of the block is built by tile rows q = 1..3, X_qr = -Z_q T_qr with
+// T_qr = sum_{m=r}^{q-1} L_qm X_mr (r < q), on warps 4..9 while warp 0 runs (a): T_qr needs
 // only the tile columns m < q, and X_qr only Z_q besides, so during (a) of step p they form
-// row p - 1 (its X) and then row p (its T); row 3's X follows the sweep.  The T tiles sit in
-// St's first tile row, which step 0 alone uses otherwise.  The transposes a tile product
-// needs (Z_p^T, L_kp^T) are written next to the tiles.
+// row p - 1 (its X) and then row p (its T); row 3's X follows the sweep.
 __global__ void __launch_bounds__(kDiagThreads, 1)
 factor_diag_kernel(const float* __restrict__ Bw, int64_t ld, int64_t j0, float* __restrict__ Xw,
                    int32_t* __restrict__ info) {
   extern __shared__ __align__(16) float sm[];
   float* S = sm;                 // [128][kLd] the block, then L (lower)
   float* X = S + kNb * kLd;      // [128][kLd] the inverse (lower)
-  float* St = X + kNb * kLd;     // [128][kLd] transposes: Z_p^T in its diagonal tile, L^T
-  float* col = St + kNb * kLd;   // [128] the pivot columns of factor_sub32
+  float* T = X + kNb * kLd;      // [32][kLd] the T tiles of the inverse's current row
+  float* col = T + kSub * kLd;   // [128] the pivot columns of factor_sub32
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
-  const int part = warp & 3;     // which 8 rows of its tile a warp computes
-  const int unit = warp >> 2;    // which tile (of up to four at a time)
+  const int h0 = kHalf * (warp & 1);  // the first of a warp's 16 rows within its tile
+  const int pair = warp >> 1;         // which tile a warp works on (of up to eight at a time)
 
   // programmatic dependent launch: the strips may be scheduled now; the previous step's update
   // must have finished before the block is read
@@ -343,62 +360,57 @@ factor_diag_kernel(const float* __restrict__ Bw, int64_t ld, int64_t j0, float* 
   }
   __syncthreads();
 
-  const int i0 = kQ * part;      // this warp's first row within its tile
   for (int p = 0; p < kNb / kSub; ++p) {
     const int c0 = p * kSub;
     if (warp == 0) {
-      factor_sub32(S + c0 * kLd + c0, X + c0 * kLd + c0, St + c0 * kLd + c0, col, lane, info, (int32_t)(j0 + c0));
-    } else if (unit >= 1 && p >= 1) {
-      const int u = unit - 1;    // the tile column r = u of the inverse's row
+      factor_sub32(S + c0 * kLd + c0, X + c0 * kLd + c0, col, lane, info, (int32_t)(j0 + c0));
+    } else if (warp >= 4 && warp < 10 && p >= 1) {
+      const int u = (warp - 4) >> 1;  // the tile column r = u of the inverse's row
       if (p >= 2) {
         // X_qr = -Z_q T_qr for q = p - 1
         const int q0 = (p - 1) * kSub;
         if (u < p - 1) {
-          float acc[kQ];
+          float acc[8][2];
           tile_zero(acc);
-          tile_nn<kQ>(acc, X + (q0 + i0) * kLd + q0, St + u * kSub, lane);
-          tile_store(acc, X + (q0 + i0) * kLd + u * kSub, lane, -1.0f);
+          tile_mma<false>(acc, X + (q0 + h0) * kLd + q0, T + u * kSub, lane);
+          tile_store(acc, X + (q0 + h0) * kLd + u * kSub, lane, -1.0f);
         }
-        asm volatile("bar.sync 1, 384;" ::: "memory");  // warps 4..15: X_q done, T tiles free
+        asm volatile("bar.sync 1, 192;" ::: "memory");  // warps 4..9: X_q done, T tiles free
       }
       // T_pr = sum_{m=r}^{p-1} L_pm X_mr
       if (u < p) {
-        float acc[kQ];
+        float acc[8][2];
         tile_zero(acc);
         for (int m = u; m < p; ++m)
-          tile_nn<kQ>(acc, S + (c0 + i0) * kLd + m * kSub, X + m * kSub * kLd + u * kSub, lane);
-        tile_store(acc, St + i0 * kLd + u * kSub, lane, 1.0f);
+          tile_mma<false>(acc, S + (c0 + h0) * kLd + m * kSub, X + m * kSub * kLd + u * kSub, lane);
+        tile_store(acc, T + h0 * kLd + u * kSub, lane, 1.0f);
       }
     }
     __syncthreads();
-    // (b) tiles below: L_ip = B_ip Z_p^T, four warps per tile
+    // (b) tiles below: L_ip = B_ip Z_p^T
     const int below = kNb / kSub - 1 - p;
-    if (unit < below) {
-      const int r0 = c0 + kSub * (1 + unit) + i0;  // this warp's first row
-      float acc[kQ];
+    if (below == 0) break;
+    if (pair < below) {
+      const int r0 = c0 + kSub * (1 + pair) + h0;  // this warp's first row
+      float acc[8][2];
       tile_zero(acc);
-      tile_nn<kQ>(acc, S + r0 * kLd + c0, St + c0 * kLd + c0, lane);
+      tile_mma<true>(acc, S + r0 * kLd + c0, X + c0 * kLd + c0, lane);
       __syncwarp();
       tile_store(acc, S + r0 * kLd + c0, lane, 1.0f);
-      // the transpose L_ip^T, for (c): St[c0 + c][r0 + r] = L_ip[r][c]
-      *reinterpret_cast<float4*>(St + (c0 + lane) * kLd + r0) = make_float4(acc[0], acc[1], acc[2], acc[3]);
-      *reinterpret_cast<float4*>(St + (c0 + lane) * kLd + r0 + 4) = make_float4(acc[4], acc[5], acc[6], acc[7]);
     }
-    if (below == 0) break;
     __syncthreads();
-    // (c) tiles (i, k), p < k <= i: B_ik -= L_ip L_kp^T = L_ip (L_kp^T), four warps per tile;
-    // up to six tiles, so the sixteen warps take them in two rounds
-    for (int round = 0; round < 2; ++round) {
-      int t = unit + 4 * round, i = p + 1;
+    // (c) tiles (i, k), p < k <= i: B_ik -= L_ip L_kp^T
+    {
+      int t = pair, i = p + 1;
       while (i < kNb / kSub && t > i - (p + 1)) {
         t -= i - p;
         ++i;
       }
       if (i < kNb / kSub) {
-        const int k0 = (p + 1 + t) * kSub, r0 = i * kSub + i0;
-        float acc[kQ];
+        const int k0 = (p + 1 + t) * kSub, r0 = i * kSub + h0;
+        float acc[8][2];
         tile_load(acc, S + r0 * kLd + k0, lane);
-        tile_nn<kQ, true>(acc, S + r0 * kLd + c0, St + c0 * kLd + k0, lane);
+        tile_mma<true, true>(acc, S + r0 * kLd + c0, S + k0 * kLd + c0, lane);
         tile_store(acc, S + r0 * kLd + k0, lane, 1.0f);
       }
     }
@@ -406,12 +418,12 @@ factor_diag_kernel(const float* __restrict__ Bw, int64_t ld, int64_t j0, float* 
   }
 
   // the inverse's last tile row: X_3r = -Z_3 T_3r
-  if (unit < kNb / kSub - 1) {
+  if (pair < kNb / kSub - 1) {
     const int q0 = kNb - kSub;
-    float acc[kQ];
+    float acc[8][2];
     tile_zero(acc);
-    tile_nn<kQ>(acc, X + (q0 + i0) * kLd + q0, St + unit * kSub, lane);
-    tile_store(acc, X + (q0 + i0) * kLd + unit * kSub, lane, -1.0f);
+    tile_mma<false>(acc, X + (q0 + h0) * kLd + q0, T + pair * kSub, lane);
+    tile_store(acc, X + (q0 + h0) * kLd + pair * kSub, lane, -1.0f);
   }
   __syncthreads();
 
