@@ -330,9 +330,11 @@ constexpr int kHalf = kSub / 2;           // rows of a tile per warp (two warps 
 //       six tiles: one round of the sixteen warps).
 // Z_p^T and L_kp^T are read in place (the transposed form of the tile product).  The inverse
 // of the block is built by tile rows q = 1..3, X_qr = -Z_q T_qr with
-// T_qr = sum_{m=r}^{q-1} L_qm X_mr (r < q), on warps 4..9 while warp 0 runs (a): T_qr needs
+// T_qr = sum_{m=r}^{q-1} L_qm X_mr (r < q), on six warps while warp 0 runs (a): T_qr needs
 // only the tile columns m < q, and X_qr only Z_q besides, so during (a) of step p they form
-// row p - 1 (its X) and then row p (its T); row 3's X follows the sweep.
+// row p - 1 (its X) and then row p (its T); row 3's X follows the sweep.  Those six warps
+// (2, 3, 6, 7, 10, 11) sit on the two schedulers that warp 0 does not use: sharing warp 0's
+// scheduler, they slowed its serial sweep (n = 4096: 1.69 against 1.65 ms).
 __global__ void __launch_bounds__(kDiagThreads, 1)
 factor_diag_kernel(const float* __restrict__ Bw, int64_t ld, int64_t j0, float* __restrict__ Xw,
                    int32_t* __restrict__ info) {
@@ -364,8 +366,9 @@ factor_diag_kernel(const float* __restrict__ Bw, int64_t ld, int64_t j0, float* 
     const int c0 = p * kSub;
     if (warp == 0) {
       factor_sub32(S + c0 * kLd + c0, X + c0 * kLd + c0, col, lane, info, (int32_t)(j0 + c0));
-    } else if (warp >= 4 && warp < 10 && p >= 1) {
-      const int u = (warp - 4) >> 1;  // the tile column r = u of the inverse's row
+    } else if ((warp & 2) != 0 && warp < 12 && p >= 1) {
+      // warps 2, 3, 6, 7, 10, 11: the schedulers that warp 0 does not use
+      const int u = warp >> 2;        // the tile column r = u of the inverse's row
       if (p >= 2) {
         // X_qr = -Z_q T_qr for q = p - 1
         const int q0 = (p - 1) * kSub;
@@ -375,7 +378,7 @@ factor_diag_kernel(const float* __restrict__ Bw, int64_t ld, int64_t j0, float* 
           tile_mma<false>(acc, X + (q0 + h0) * kLd + q0, T + u * kSub, lane);
           tile_store(acc, X + (q0 + h0) * kLd + u * kSub, lane, -1.0f);
         }
-        asm volatile("bar.sync 1, 192;" ::: "memory");  // warps 4..9: X_q done, T tiles free
+        asm volatile("bar.sync 1, 192;" ::: "memory");  // these six warps: X_q done, T tiles free
       }
       // T_pr = sum_{m=r}^{p-1} L_pm X_mr
       if (u < p) {
