@@ -167,6 +167,20 @@ __device__ __forceinline__ float sum_squares32(const uint32_t (&r)[32]) {
 // over kb_half K blocks, every tile (the GPTQ update).  kMode 3: kMode 1 read from X itself
 // ([tokens, n], channels contiguous): each stage loads 64-channel x 64-token boxes and
 // the MMAs take both operands MN-major, so no transpose is needed.
+// Tile t of a persistent GEMM's sequence (tiles_n column tiles per row of tiles) in groups of
+// kRasterRows rows of tiles, column-major within a group: the tiles in flight at once (about
+// one per SM) then cover a few row strips of A and a part of B's column strips, rather than
+// every column strip of B for one or two row strips, so their operands stay in L2.
+constexpr int kRasterRows = 8;
+__device__ __forceinline__ void raster_tile(int t, int tiles_n, int tiles_total, int& tm, int& tn) {
+  const int tiles_m = tiles_total / tiles_n;
+  const int first = t / (kRasterRows * tiles_n) * kRasterRows;
+  const int rows = min(kRasterRows, tiles_m - first);
+  const int within = t - first * tiles_n;
+  tm = first + within % rows;
+  tn = within / rows;
+}
+
 template <int kMode>
 __global__ void __launch_bounds__(kGemmThreads, 1)
 gemm_kernel(const __grid_constant__ CUtensorMap xmap, const __grid_constant__ CUtensorMap wmap,
@@ -190,11 +204,15 @@ gemm_kernel(const __grid_constant__ CUtensorMap xmap, const __grid_constant__ CU
   // K loops cut into accumulation segments folded in TMEM: the Hessian (K = tokens) and the
   // output error (K = 2 n); the GPTQ update's K = 6 B is a single segment anyway
   constexpr bool kSegmented = kMode != 2;
-  // The GPTQ update is persistent: a CTA takes tiles blockIdx.x, + gridDim.x, ... and
-  // alternates two 256-column accumulators, so a tile's epilogue (the TMA reduce-add into
-  // the running weights) runs alongside the next tile's loads and MMAs.  The other modes
+  // The GPTQ update and the output error are persistent: a CTA takes tiles blockIdx.x,
+  // + gridDim.x, ...  The update alternates two 256-column accumulators, so a tile's
+  // epilogue (the TMA reduce-add into the running weights) runs alongside the next tile's
+  // loads and MMAs.  The output error's segments run on across its tiles (one segment
+  // counter), so the MMAs of a tile's first segment start as soon as the previous tile's
+  // last partial has been read out, alongside that tile's sum of squares.  The Hessian modes
   // take one tile per CTA.
-  constexpr bool kPersistent = kMode == 2;
+  constexpr bool kPersistent = kMode == 2 || kMode == 0;
+  constexpr bool kTwoAcc = kMode == 2;
   constexpr uint32_t kCols = (kSegmented || kPersistent) ? kTmemColsSeg : kTmemCols;
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
@@ -246,7 +264,8 @@ gemm_kernel(const __grid_constant__ CUtensorMap xmap, const __grid_constant__ CU
       bool go = true;
       for (int i = 0; i < ntiles && go; ++i) {
         const int t = (int)blockIdx.x + i * (int)gridDim.x;
-        const int tm = t / tiles_n, tn = t - tm * tiles_n;
+        int tm = t / tiles_n, tn = t - tm * tiles_n;
+        if (kMode == 0) raster_tile(t, tiles_n, tiles_total, tm, tn);
         for (int kb = 0; kb < kb_total; ++kb) {
           // the ring's position counts K blocks over all of the CTA's tiles
           const int g = i * kb_total + kb;
@@ -283,15 +302,17 @@ gemm_kernel(const __grid_constant__ CUtensorMap xmap, const __grid_constant__ CU
       const int nseg = (kb_total + seg_blocks - 1) / seg_blocks;
       bool ok = true;
       for (int i = 0; i < ntiles && ok; ++i) {
-        const uint32_t acc = kPersistent ? (uint32_t)(i & 1) : 0u;
+        const uint32_t acc = kTwoAcc ? (uint32_t)(i & 1) : 0u;
         // the accumulator's previous tile (two back) must have been read out of TMEM
-        if (kPersistent && i >= 2 && !mbar_wait(&tacc_empty[acc], (uint32_t)((i >> 1) - 1) & 1u)) {
+        if (kTwoAcc && i >= 2 && !mbar_wait(&tacc_empty[acc], (uint32_t)((i >> 1) - 1) & 1u)) {
           atomicOr(failed, 1u);
           break;
         }
         for (int seg = 0; seg < nseg && ok; ++seg) {
-          // the previous segment's partial must have been read out of TMEM
-          if (kSegmented && seg >= 1 && !mbar_wait(seg_empty, (uint32_t)(seg - 1) & 1u)) {
+          // the previous segment's partial (of this tile or the one before) must have been
+          // read out of TMEM
+          const int gs = i * nseg + seg;
+          if (kSegmented && gs >= 1 && !mbar_wait(seg_empty, (uint32_t)(gs - 1) & 1u)) {
             atomicOr(failed, 1u);
             ok = false;
             break;
@@ -326,7 +347,7 @@ gemm_kernel(const __grid_constant__ CUtensorMap xmap, const __grid_constant__ CU
             umma_commit(smem_addr(&empty[s]));
           }
           // fires once every MMA issued above has completed
-          if (ok) umma_commit(smem_addr(kSegmented ? seg_full : (kPersistent ? &tacc_full[acc] : acc_ready)));
+          if (ok) umma_commit(smem_addr(kSegmented ? seg_full : (kTwoAcc ? &tacc_full[acc] : acc_ready)));
         }
       }
     }
@@ -346,10 +367,11 @@ gemm_kernel(const __grid_constant__ CUtensorMap xmap, const __grid_constant__ CU
       const int tm = t / tiles_n, tn = t - tm * tiles_n;
       const int64_t row = (int64_t)tm * kBM + quarter * 32 + lane;
       const int64_t col0 = (int64_t)tn * kBN + cbase;
-      const uint32_t tacc = kPersistent ? (uint32_t)(i & 1) : 0u;
+      const uint32_t tacc = kTwoAcc ? (uint32_t)(i & 1) : 0u;
       for (int seg = 0; seg < nseg; ++seg) {
-        uint64_t* ready = kSegmented ? seg_full : (kPersistent ? &tacc_full[tacc] : acc_ready);
-        const uint32_t parity = kSegmented ? (uint32_t)seg & 1u : (kPersistent ? (uint32_t)(i >> 1) & 1u : 0u);
+        uint64_t* ready = kSegmented ? seg_full : (kTwoAcc ? &tacc_full[tacc] : acc_ready);
+        const uint32_t parity =
+            kSegmented ? (uint32_t)(i * nseg + seg) & 1u : (kTwoAcc ? (uint32_t)(i >> 1) & 1u : 0u);
         if (!mbar_wait(ready, parity)) {
           atomicOr(failed, 1u);
           alive = false;
@@ -363,11 +385,11 @@ gemm_kernel(const __grid_constant__ CUtensorMap xmap, const __grid_constant__ CU
           tmem_ld_32x32b_x32(tmem_d + tacc * kBN + lane_base + cbase + (uint32_t)c,
                              *reinterpret_cast<uint32_t(*)[32]>(p + c));
         tmem_ld_wait();
-        if ((kSegmented && !last) || kPersistent) {
-          // the partial is in registers: the MMAs may go on with the next segment (or the
-          // tile after next may use this accumulator)
+        if ((kSegmented && (!last || kPersistent)) || kTwoAcc) {
+          // the partial is in registers: the MMAs may go on with the next segment (of this
+          // tile or the next), or the tile after next may use this accumulator
           tc_fence_before_sync();
-          mbar_arrive(kPersistent ? &tacc_empty[tacc] : seg_empty);
+          mbar_arrive(kTwoAcc ? &tacc_empty[tacc] : seg_empty);
         }
         if (kSegmented && seg > 0) {
           // fold into the running sum (TMEM columns [256, 512)), fp32 round-to-nearest
@@ -394,7 +416,7 @@ gemm_kernel(const __grid_constant__ CUtensorMap xmap, const __grid_constant__ CU
           for (int c = 0; c < kHalf; c += 32) acc += (double)sum_squares32(*reinterpret_cast<uint32_t(*)[32]>(p + c));
           continue;
         }
-        if (kPersistent) {
+        if (kTwoAcc) {
           // the GPTQ update: staged 32 x 32 boxes reduce-added into C by TMA.  Row `lane`
           // of a box holds 128 bytes; the 128-byte swizzle puts its 16-byte chunk k at
           // k ^ (lane & 7), so a warp's stores hit every bank once.
@@ -441,7 +463,7 @@ gemm_kernel(const __grid_constant__ CUtensorMap xmap, const __grid_constant__ CU
       }
     }
     // the update's reduce-adds complete before the CTA ends
-    if (kPersistent && lane == 0) bulk_wait_all();
+    if (kTwoAcc && lane == 0) bulk_wait_all();
     if (!kAccum) {
 #pragma unroll
       for (int off = 16; off > 0; off >>= 1) acc += __shfl_xor_sync(0xFFFFFFFFu, acc, off);
@@ -567,11 +589,16 @@ cudaError_t launch_output_error(const void* x, int64_t tokens, int64_t n, int64_
   if (attr_status != cudaSuccess) return attr_status;
   const int64_t tiles_n = (m + kBN - 1) / kBN;
   const int64_t tiles = output_error_tiles(tokens, m);
-  gemm_kernel<0><<<(unsigned)tiles, kGemmThreads, kGemmSmemBytes, stream>>>(
+  // persistent: one CTA per SM (the shared-memory ring and the 512 TMEM columns allow no
+  // more), tiles strided; one partial per CTA
+  DeviceInfo info;
+  if ((err = current_device_info(&info)) != cudaSuccess) return err;
+  const int64_t grid = std::max<int64_t>(1, std::min<int64_t>(tiles, info.sm_count));
+  gemm_kernel<0><<<(unsigned)grid, kGemmThreads, kGemmSmemBytes, stream>>>(
       xmap, wmap, wmap, (int)(n_pad / kBK), (int)tiles_n, (int)tiles, partials, nullptr, 0, 0, 0);
   err = cudaGetLastError();
   if (err != cudaSuccess) return err;
-  reduce_kernel<<<1, 256, 0, stream>>>(partials, tiles, out);
+  reduce_kernel<<<1, 256, 0, stream>>>(partials, grid, out);
   return cudaGetLastError();
 }
 
