@@ -812,13 +812,15 @@ OUTPUT_ERROR_RTOL = 1e-4
 
 
 @pytest.mark.parametrize("tokens,m,n", [(128, 256, 64), (300, 300, 80), (512, 512, 1024), (1000, 40, 4096),
-                                        (256, 256, 14336)])
+                                        (256, 256, 14336), (2600, 2048, 64)])
 def test_output_error_matches_oracle(tokens, m, n):
     """||X dW^T||_F^2 on the tensor cores against the fp64 oracle: ragged tokens, outputs
-    and K (n not a multiple of 64), one tile and many, and down_proj's width (K = 28672,
+    and K (n not a multiple of 64), one tile and many, down_proj's width (K = 28672,
     14 accumulation segments; one fp32 accumulation over the whole K would drift about 2x
-    past the bound there).  Tolerance: the bf16 split of dW (2^-17 relative per element)
-    plus fp32 accumulation over 2048-long segments."""
+    past the bound there), and more tiles than SMs (21 x 8 = 168 tiles of 128 x 256: CTAs
+    with two tiles, and tile-order groups of 8, 8 and 5 rows of tiles).  Tolerance: the bf16
+    split of dW (2^-17 relative per element) plus fp32 accumulation over 2048-long
+    segments."""
     w = wl.weight(m, n, 0.02, 50 + n)
     wb = bits(w)
     s_ref, _ = oracle.global_scale(wb)
