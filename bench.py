@@ -565,6 +565,20 @@ class StepGraphs:
 # algorithmic bytes per group of the search: W 32, nibbles 8, code out 1, code in 1 (none
 # when the search decides the initial codes itself)
 SEARCH_BYTES = {"rtn": 41, "4over6": 41, "4over6-2pass": 42}
+# algorithmic bytes per group of the weight-only calls: W 32 for the global amax, and with
+# the two-pass 4over6 init W 32 again and the code written 1
+WEIGHT_BYTES = {"rtn": 32, "4over6": 32, "4over6-2pass": 65}
+
+
+def step_hbm(work, ms_step: float, hbm_peak: float, peak_kind: str) -> dict:
+    """The whole step against HBM: every byte the step has to move (X once for the Hessian
+    passes, W for the global amax and again in the search, the codes and nibbles written),
+    over the step's time, against the copy bandwidth."""
+    b = work.h_bytes + (WEIGHT_BYTES[work.init] + SEARCH_BYTES[work.init]) * work.groups
+    gbs = b / (ms_step * 1e-3) / 1e9
+    return {"bytes": b, "achieved": gbs, "peak": hbm_peak, "unit": "GB/s", "frac": gbs / hbm_peak,
+            "peak_kind": f"{peak_kind} HBM copy bandwidth",
+            "note": "X once, W twice (global amax, search), codes and nibbles out, over the whole step"}
 
 
 def kernels_per_matrix(work: Work) -> int:
@@ -1111,6 +1125,7 @@ def measure_workload(hs, d: Dist, args, W: wl.Workload, win, dev, overlap_ctas: 
         "work": work, "graphs": graphs, "ms_step": ms_step, "ms_eager": ms_eager, "warm": warm,
         "value": work.groups * d.world / (ms_step * 1e-3), "overlap_ctas": overlap,
         "roofline": dominant, "roofline_hessian": hess_roof, "roofline_search": search_roof,
+        "step_hbm": step_hbm(work, ms_step, hbm_peak, peak_kind),
         "phases_ms": {"hessian": ms_h, "after_hessian": ms_sc, "hessian_alone": ms_h_alone,
                       "weight_only": ms_init, "refine": main["ms"]},
         "hessian": {"gbs": h_gbs, "tokens_channels_per_s": work.h_bytes / 2 / (ms_h * 1e-3),
@@ -1142,6 +1157,7 @@ def extra_workload(hs, d: Dist, args, name: str, dev) -> dict:
            "schedule": "pipelined" if res["graphs"].pipeline else "sequential",
            "roofline_hessian": compact_roofline(res["roofline_hessian"]),
            "roofline_search": compact_roofline(res["roofline_search"]),
+           "step_hbm": {k: res["step_hbm"][k] for k in ("bytes", "achieved", "peak", "unit", "frac")},
            "phases_ms": res["phases_ms"], "clocks": res["clocks"],
            "search_sweep": [{k: s[k] for k in ("window", "candidates", "ms", "groups_per_s", "bound", "frac")}
                             for s in res["sweep"]]}
@@ -1196,6 +1212,7 @@ def gpu_arm(args, d: Dist):
         "roofline": roofline,
         "roofline_search": res["roofline_search"],
         "roofline_hessian": res["roofline_hessian"],
+        "step_hbm": res["step_hbm"],
         "seconds_per_layer": ms_step * 1e-3,
     }
     if n_layers > 1:

@@ -129,3 +129,16 @@ def test_step_graphs_reproduce_the_eager_step(workload, pipeline):
         for M, (_, _, sg) in zip(work.mats, ref, strict=True):
             assert torch.equal(M.sg, sg)
     graphs.bind(0)
+
+
+def test_step_hbm_counts_every_byte_of_the_step():
+    """The whole-step HBM figure: X's bytes of the Hessian passes, W once for the global
+    amax and once in the search (again for the two-pass 4over6 codes), and the codes and
+    nibbles written; per group 32 + 41, or 65 + 42 with the two-pass init."""
+    work = SimpleNamespace(h_bytes=6_000_000, groups=1000, init="rtn")
+    r = bench.step_hbm(work, ms_step=1.0, hbm_peak=6000.0, peak_kind="measured")
+    assert r["bytes"] == 6_000_000 + 73 * 1000
+    assert abs(r["achieved"] - r["bytes"] / 1e-3 / 1e9) < 1e-9
+    assert abs(r["frac"] - r["achieved"] / 6000.0) < 1e-12
+    work.init = "4over6-2pass"
+    assert bench.step_hbm(work, 1.0, 6000.0, "measured")["bytes"] == 6_000_000 + 107 * 1000
