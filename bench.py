@@ -78,6 +78,10 @@ def parse():
                         "runs alongside (0: run every search after the last Hessian pass; -1, the "
                         "default: when the step's estimated search time exceeds its Hessian time, 7 "
                         "(every CTA the search kernel keeps resident); else 4)")
+    p.add_argument("--search-schedule", choices=["auto", "shared", "static"], default="auto",
+                   help="the search's unit schedule: 'shared' passes hscale_refine_scales_ws a workspace "
+                        "(units shared out at run time in long searches), 'static' passes none; 'auto' "
+                        "shares except in searches that fill the SMs beside a Hessian pass")
     p.add_argument("--pipeline", choices=["auto", "on", "off"], default="auto",
                    help="run each step's last searches alongside the next step's first Hessian pass "
                         "(h, s_g and initial codes double-buffered).  auto (default) and on: pipelined "
@@ -279,6 +283,9 @@ class Matrix:
         self.codes0 = torch.empty(self.m, self.n // 16, dtype=torch.uint8, device=device)
         self.codes = torch.empty_like(self.codes0)
         self.packed = torch.empty(self.m, self.n // 2, dtype=torch.uint8, device=device)
+        # the search's work-sharing counter (hscale_refine_workspace_bytes(); the calls of one
+        # matrix never overlap on the GPU)
+        self.sched = torch.zeros(16, dtype=torch.uint8, device=device)
 
 
 def column_blocks(S: Space, col_block: int):
@@ -313,6 +320,7 @@ class Work:
         self.h_bytes = sum(2 * rows * width + 8 * width for width, rows in calls)
         self.h_launches = len(calls)
         self.ws = None
+        self.search_schedule = "auto"
 
     def stage_estimates(self):
         """(name, Hessian seconds, search seconds) per input space, from nominal rates
@@ -404,11 +412,19 @@ def init_phase(hs, work: Work, ws=None):
 def refine(hs, work: Work, M, down, up, w=None, ctas_per_sm=0):
     """The H-Scale search with packing of one matrix over the window (down, up)."""
     w = M.w if w is None else w
-    if work.init == "4over6":
-        hs.hscale_refine_scales_4over6(w, M.space.h, M.sg, down, up, M.codes, M.packed, ctas_per_sm)
-    else:
-        init = M.codes0 if work.init == "4over6-2pass" else None
-        hs.hscale_refine_scales_ex(w, M.space.h, M.sg, init, down, up, M.codes, M.packed, ctas_per_sm)
+    init = M.codes0 if work.init == "4over6-2pass" else None
+    hs.hscale_refine_scales_ws(w, M.space.h, M.sg, init, int(work.init == "4over6"), down, up, M.codes, M.packed,
+                               ctas_per_sm, M.sched if shares(work, ctas_per_sm) else None)
+
+
+def shares(work: Work, ctas_per_sm: int) -> bool:
+    """Whether a search call gets the work-sharing workspace.  With 'auto' every call does
+    except one that fills the SMs (7 CTAs each) beside a Hessian pass: a static deal lets
+    its first CTAs finish midway and make room for the Hessian pass's CTAs, while shared
+    units keep every CTA resident to the end."""
+    if work.search_schedule == "auto":
+        return not 7 <= ctas_per_sm
+    return work.search_schedule == "shared"
 
 
 def refine_phase(hs, work: Work, win=None, ws=None):
@@ -585,6 +601,10 @@ def kernels_per_matrix(work: Work) -> int:
     """Library kernels per matrix and step: amax and s_g (hscale_rtn_scales), the 4over6
     codes with the two-pass init, the search."""
     return 4 if work.init == "4over6-2pass" else 3
+
+
+# the search kernels: the static deal, and the work-shared one for long searches
+SEARCH_KERNELS = "refine_linear_kernel|refine_shared_kernel"
 
 
 def timed(fn, reps, flush=None):
@@ -1019,6 +1039,7 @@ def measure_workload(hs, d: Dist, args, W: wl.Workload, win, dev, overlap_ctas: 
     figures, and the search over every window of the workload timed per kernel.  Returns
     (result dict, work); the work keeps the step's outputs."""
     work = Work(W, d.rank, win, dev, tokens=tokens, init=init, col_block=col_block)
+    work.search_schedule = args.search_schedule
     work.ws = torch.empty(hs.hscale_rtn_workspace_bytes(), dtype=torch.uint8, device=dev)
     torch.cuda.synchronize()
 
@@ -1106,14 +1127,14 @@ def measure_workload(hs, d: Dist, args, W: wl.Workload, win, dev, overlap_ctas: 
     # ---- roofline of the search (its own window, W read from HBM after an L2 flush)
     if main["bound"] == "alu":
         ops = 80.0 * main["candidates"] * work.groups
-        search_roof = {"bound": "alu", "kernel": "refine_linear_kernel", "achieved": ops / (main["ms"] * 1e-3) / 1e12,
+        search_roof = {"bound": "alu", "kernel": SEARCH_KERNELS, "achieved": ops / (main["ms"] * 1e-3) / 1e12,
                        "peak": fp32_peak / 1e12, "unit": "Tops/s", "frac": main["frac"],
                        "peak_kind": "SMs x 128 fp32 lanes x max SM clock; 5 lane operations per element "
                                     "and candidate", "candidates": main["candidates"], "traffic": None,
                        "ops_per_launch": ops / len(work.mats), "ms_per_launch": main["ms"] / len(work.mats)}
     else:
         b = SEARCH_BYTES[work.init] * work.groups
-        search_roof = {"bound": "hbm", "kernel": "refine_linear_kernel", "achieved": b / (main["ms"] * 1e-3) / 1e9,
+        search_roof = {"bound": "hbm", "kernel": SEARCH_KERNELS, "achieved": b / (main["ms"] * 1e-3) / 1e9,
                        "peak": hbm_peak, "unit": "GB/s", "frac": b / (main["ms"] * 1e-3) / 1e9 / hbm_peak,
                        "peak_kind": f"{peak_kind} HBM copy bandwidth", "candidates": main["candidates"],
                        "traffic": None, "bytes_per_launch": b / len(work.mats),
@@ -1124,6 +1145,7 @@ def measure_workload(hs, d: Dist, args, W: wl.Workload, win, dev, overlap_ctas: 
     res = {
         "work": work, "graphs": graphs, "ms_step": ms_step, "ms_eager": ms_eager, "warm": warm,
         "value": work.groups * d.world / (ms_step * 1e-3), "overlap_ctas": overlap,
+        "search_schedule": work.search_schedule,
         "roofline": dominant, "roofline_hessian": hess_roof, "roofline_search": search_roof,
         "step_hbm": step_hbm(work, ms_step, hbm_peak, peak_kind),
         "phases_ms": {"hessian": ms_h, "after_hessian": ms_sc, "hessian_alone": ms_h_alone,

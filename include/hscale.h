@@ -25,6 +25,8 @@
  *      hscale_refine_scales_4over6      Algorithm 2 in one pass: those codes decided
  *                                       inside the search
  *      hscale_refine_scales_strided     the search on 2-D views (column blocks, slices)
+ *      hscale_refine_scales_ws          the search with its units shared out at run time
+ *                                       (a 16-byte workspace; same results)
  *      hscale_dequant_residual          dW = W - W_hat of the packed weights (Eqs. 1-3)
  *      hscale_output_error              ||X dW^T||_F^2 on the tensor cores (Eq. 3)
  *      hscale_hessian_full_accumulate   H += X^T X on the tensor cores (Algorithm 3)
@@ -303,6 +305,38 @@ int hscale_refine_scales_ex(const void* w_bf16, const float* h, int64_t m, int64
 int hscale_refine_scales_4over6(const void* w_bf16, const float* h, int64_t m, int64_t n,
                                 const float* global_scale, int32_t down, int32_t up, uint8_t* codes_out,
                                 uint8_t* packed_out, int32_t ctas_per_sm, void* stream);
+
+/*
+ * Bytes of device workspace hscale_refine_scales_ws takes: 16.
+ */
+size_t hscale_refine_workspace_bytes(void);
+
+/*
+ * hscale_refine_scales_ex (fourover6 = 0) or hscale_refine_scales_4over6 (fourover6 = 1)
+ * with the units of long searches shared out at run time; the results are identical.
+ * The paper has no counterpart: this is a schedule.  The GPU's warp schedulers favour the
+ * warps that became resident first, so when every warp is dealt an equal share up front,
+ * the late ones run on alone at the end of a long call; here warps take small batches of
+ * units from a counter in `workspace` instead.  The library uses it when each warp would
+ * otherwise get at least about 512 units x candidates (e.g. a 28672 x 8192 matrix at
+ * k = 4, or a 14336 x 4096 one at k = 16); shorter searches take the static deal.
+ *
+ * w, h, m, n, global_scale, init_codes, down, up, codes_out, packed_out, ctas_per_sm as for
+ * hscale_refine_scales_ex; fourover6 as for hscale_refine_scales_strided (0 or 1; 1 with
+ * init_codes returns HSCALE_ERR_ARG).
+ * workspace        device memory of at least hscale_refine_workspace_bytes() bytes,
+ *                  16-byte aligned, owned by the caller; or NULL for the static deal.  The
+ *                  call zeroes its first 4 bytes on `stream` before the kernel and the
+ *                  kernel counts in them, so calls that may run at the same time on the
+ *                  GPU need distinct workspaces.  Nothing needs to persist between calls.
+ * workspace_bytes  its size; below hscale_refine_workspace_bytes() returns
+ *                  HSCALE_ERR_WORKSPACE (a misaligned workspace returns HSCALE_ERR_ALIGN).
+ * The other status codes are those of hscale_refine_scales_strided.
+ */
+int hscale_refine_scales_ws(const void* w_bf16, const float* h, int64_t m, int64_t n, const float* global_scale,
+                            const uint8_t* init_codes, int32_t fourover6, int32_t down, int32_t up,
+                            uint8_t* codes_out, uint8_t* packed_out, int32_t ctas_per_sm, void* workspace,
+                            size_t workspace_bytes, void* stream);
 
 /*
  * The search on 2-D views: hscale_refine_scales_ex / hscale_refine_scales_4over6 on a

@@ -28,7 +28,8 @@ __all__ = [
     "hscale_rtn_workspace_bytes", "hscale_rtn_scales",
     "hscale_rtn_scales_noalloc",
     "hscale_refine_scales", "hscale_refine_scales_ex", "hscale_refine_scales_4over6",
-    "hscale_refine_scales_strided", "hscale_pack_nvfp4", "hscale_fourover6_codes",
+    "hscale_refine_scales_strided", "hscale_refine_workspace_bytes", "hscale_refine_scales_ws",
+    "hscale_pack_nvfp4", "hscale_fourover6_codes",
     "hscale_dequant_residual", "hscale_output_error_workspace_bytes", "hscale_output_error",
     "residual_ld", "hscale_selftest_bounded_wait", "hscale_hessian_full_workspace_bytes",
     "hscale_hessian_full_accumulate", "hscale_gptq_factor_workspace_bytes", "hscale_gptq_factor",
@@ -60,6 +61,9 @@ _SIGNATURES = {
     "hscale_refine_scales_4over6": (ctypes.c_int, [_P, _P, _I64, _I64, _P, _I32, _I32, _P, _P, _I32, _P]),
     "hscale_refine_scales_strided": (ctypes.c_int, [_P, _I64, _P, _I64, _I64, _P, _P, _I64, _I32, _I32, _I32,
                                                     _P, _I64, _P, _I64, _I32, _P]),
+    "hscale_refine_workspace_bytes": (_SZ, []),
+    "hscale_refine_scales_ws": (ctypes.c_int, [_P, _P, _I64, _I64, _P, _P, _I32, _I32, _I32, _P, _P, _I32, _P, _SZ,
+                                               _P]),
     "hscale_pack_nvfp4": (ctypes.c_int, [_P, _I64, _I64, _P, _P, _P, _P]),
     "hscale_fourover6_codes": (ctypes.c_int, [_P, _I64, _I64, _P, _P, _P]),
     "hscale_dequant_residual": (ctypes.c_int, [_P, _I64, _I64, _P, _P, _P, _P, _I64, _P]),
@@ -283,6 +287,44 @@ def hscale_refine_scales_ex(w: torch.Tensor, h: torch.Tensor | None, global_scal
            load().hscale_refine_scales_ex(_ptr(w), _ptr(h), m, n, _ptr(global_scale), _ptr(init_codes),
                                           int(down), int(up), _ptr(codes_out), _ptr(packed_out),
                                           int(ctas_per_sm), _stream_ptr(stream)))
+
+
+def hscale_refine_workspace_bytes() -> int:
+    return int(load().hscale_refine_workspace_bytes())
+
+
+def hscale_refine_scales_ws(w: torch.Tensor, h: torch.Tensor | None, global_scale: torch.Tensor,
+                            init_codes: torch.Tensor | None, fourover6: int, down: int, up: int,
+                            codes_out: torch.Tensor, packed_out: torch.Tensor | None, ctas_per_sm: int,
+                            workspace: torch.Tensor | None, stream=None) -> None:
+    """hscale_refine_scales_ex (fourover6 = 0) or _4over6 (fourover6 = 1) with long searches'
+    units shared out at run time through ``workspace`` (a device uint8 tensor of at least
+    hscale_refine_workspace_bytes() bytes, or None for the static deal)."""
+    _need(w, torch.bfloat16, "w")
+    _need(global_scale, torch.float32, "global_scale")
+    _need(codes_out, torch.uint8, "codes_out")
+    if not w.is_contiguous() or w.dim() != 2:
+        raise ValueError("w must be a contiguous 2-D tensor")
+    m, n = w.shape
+    if h is not None:
+        _need(h, torch.float32, "h")
+        if h.numel() != n or not h.is_contiguous():
+            raise ValueError("h must be a contiguous float32 vector of length n")
+    for name, t, size in (("init_codes", init_codes, m * (n // 16)),
+                          ("codes_out", codes_out, m * (n // 16)),
+                          ("packed_out", packed_out, m * (n // 2))):
+        if t is not None:
+            _need(t, torch.uint8, name)
+            if t.numel() != size or not t.is_contiguous():
+                raise ValueError(f"{name} must be contiguous with {size} bytes")
+    nbytes = 0
+    if workspace is not None:
+        _need(workspace, torch.uint8, "workspace")
+        nbytes = workspace.numel()
+    _check("hscale_refine_scales_ws",
+           load().hscale_refine_scales_ws(_ptr(w), _ptr(h), m, n, _ptr(global_scale), _ptr(init_codes),
+                                          int(fourover6), int(down), int(up), _ptr(codes_out), _ptr(packed_out),
+                                          int(ctas_per_sm), _ptr(workspace), nbytes, _stream_ptr(stream)))
 
 
 def hscale_refine_scales_4over6(w: torch.Tensor, h: torch.Tensor | None, global_scale: torch.Tensor,

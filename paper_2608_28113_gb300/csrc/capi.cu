@@ -69,7 +69,7 @@ const char* hscale_status_string(int status) {
   }
 }
 
-int hscale_abi_version(void) { return 3; }
+int hscale_abi_version(void) { return 4; }
 
 int hscale_device_error_flags(uint32_t* flags) {
   if (flags == nullptr) return HSCALE_ERR_NULL;
@@ -175,11 +175,13 @@ int hscale_refine_scales_4over6(const void* w_bf16, const float* h, int64_t m, i
                                       n / 16, packed_out, n / 2, ctas_per_sm, stream);
 }
 
-int hscale_refine_scales_strided(const void* w_bf16, int64_t ld_w, const float* h, int64_t m, int64_t n,
-                                 const float* global_scale, const uint8_t* init_codes, int64_t ld_init,
-                                 int32_t fourover6, int32_t down, int32_t up, uint8_t* codes_out,
-                                 int64_t ld_codes, uint8_t* packed_out, int64_t ld_packed, int32_t ctas_per_sm,
-                                 void* stream) {
+namespace {
+
+// Argument checks and launch shared by the refine entry points.
+int refine_checked(const void* w_bf16, int64_t ld_w, const float* h, int64_t m, int64_t n,
+                   const float* global_scale, const uint8_t* init_codes, int64_t ld_init, int32_t fourover6,
+                   int32_t down, int32_t up, uint8_t* codes_out, int64_t ld_codes, uint8_t* packed_out,
+                   int64_t ld_packed, int32_t ctas_per_sm, unsigned* share_counter, void* stream) {
   int st = check_weight(w_bf16, m, n);
   if (st != HSCALE_OK) return st;
   if (down < 0 || up < 0 || down > 125 || up > 125) return HSCALE_ERR_ARG;
@@ -199,8 +201,33 @@ int hscale_refine_scales_strided(const void* w_bf16, int64_t ld_w, const float* 
   if (packed_out != nullptr && (!aligned(packed_out, 8) || ld_packed % 8 != 0)) return HSCALE_ERR_ALIGN;
   return from_cuda(hscale::launch_refine(w_bf16, ld_w, h, m, n, global_scale, init_codes,
                                          init_codes ? ld_init : 0, down, up, codes_out, ld_codes, packed_out,
-                                         packed_out ? ld_packed : 0, ctas_per_sm, fourover6 != 0,
+                                         packed_out ? ld_packed : 0, ctas_per_sm, fourover6 != 0, share_counter,
                                          as_stream(stream)));
+}
+
+}  // namespace
+
+int hscale_refine_scales_strided(const void* w_bf16, int64_t ld_w, const float* h, int64_t m, int64_t n,
+                                 const float* global_scale, const uint8_t* init_codes, int64_t ld_init,
+                                 int32_t fourover6, int32_t down, int32_t up, uint8_t* codes_out,
+                                 int64_t ld_codes, uint8_t* packed_out, int64_t ld_packed, int32_t ctas_per_sm,
+                                 void* stream) {
+  return refine_checked(w_bf16, ld_w, h, m, n, global_scale, init_codes, ld_init, fourover6, down, up, codes_out,
+                        ld_codes, packed_out, ld_packed, ctas_per_sm, nullptr, stream);
+}
+
+size_t hscale_refine_workspace_bytes(void) { return 16; }
+
+int hscale_refine_scales_ws(const void* w_bf16, const float* h, int64_t m, int64_t n, const float* global_scale,
+                            const uint8_t* init_codes, int32_t fourover6, int32_t down, int32_t up,
+                            uint8_t* codes_out, uint8_t* packed_out, int32_t ctas_per_sm, void* workspace,
+                            size_t workspace_bytes, void* stream) {
+  if (workspace != nullptr) {
+    if (workspace_bytes < hscale_refine_workspace_bytes()) return HSCALE_ERR_WORKSPACE;
+    if (!aligned(workspace, 16)) return HSCALE_ERR_ALIGN;
+  }
+  return refine_checked(w_bf16, n, h, m, n, global_scale, init_codes, n / 16, fourover6, down, up, codes_out,
+                        n / 16, packed_out, n / 2, ctas_per_sm, static_cast<unsigned*>(workspace), stream);
 }
 
 int hscale_fourover6_codes(const void* w_bf16, int64_t m, int64_t n, const float* global_scale,

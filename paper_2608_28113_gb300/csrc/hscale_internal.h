@@ -39,11 +39,13 @@ cudaError_t launch_rtn_codes(const void* w, int64_t m, int64_t n, const uint32_t
 // apart (ld_packed % 8 == 0).  ctas_per_sm > 0
 // caps the grid at that many resident CTAs per SM (room for a concurrent kernel); 0 fills
 // every SM.  fourover6: the initial codes are Algorithm 2's, decided in the search kernel
-// (init_codes is then ignored).
+// (init_codes is then ignored).  share_counter: 4 bytes of device memory for the
+// work-shared schedule of long contiguous searches (zeroed on the stream first), or
+// nullptr for the static deal; the results are the same either way.
 cudaError_t launch_refine(const void* w, int64_t ld_w, const float* h, int64_t m, int64_t n,
                           const float* global_scale, const uint8_t* init_codes, int64_t ld_init, int down,
                           int up, uint8_t* codes_out, int64_t ld_codes, uint8_t* packed_out, int64_t ld_packed,
-                          int ctas_per_sm, bool fourover6, cudaStream_t stream);
+                          int ctas_per_sm, bool fourover6, unsigned* share_counter, cudaStream_t stream);
 
 // Algorithm 2's initial codes (the better of the anchors m/4, m/6 by plain MSE).
 cudaError_t launch_fourover6(const void* w, int64_t m, int64_t n, const float* global_scale,

@@ -211,6 +211,18 @@ __device__ __forceinline__ float energy_bound(float hsum, float amax_k) {
   return __fmul_rn(hsum, __fmul_rn(amax_k, amax_k));
 }
 
+// A = sum_j h_j a_j^2 itself (scaled domain), for the search's margin test.  (sum h) amax^2
+// can exceed it many times over (one large weight, or h concentrated on small ones), and
+// the margin's dominant term grows with sqrt(A), so the tighter value sends several times
+// fewer groups to the exact rescoring.  The fp32 sum of non-negative terms is within a
+// relative 12 * 2^-24 of A; the factor 1 + 2^-19 makes the result an upper bound.
+__device__ __forceinline__ float group_energy(const Group& G, const float2 (&hv2)[8]) {
+  float2 acc = __fmul2_rn(hv2[0], __fmul2_rn(G.a[0], G.a[0]));
+#pragma unroll
+  for (int i = 1; i < 8; ++i) acc = __ffma2_rn(hv2[i], __fmul2_rn(G.a[i], G.a[i]), acc);
+  return __fmul_rn(__fadd_rn(acc.x, acc.y), 1.0f + 0x1p-19f);
+}
+
 // tie rule of the search: smaller error, then smaller |shift|, then smaller shift
 __device__ __forceinline__ bool better(float e, int c, float be, int bc, int c0) {
   if (e != be) return e < be;
@@ -489,7 +501,6 @@ refine_kernel(const uint4* __restrict__ w, int64_t ld_w, const float* __restrict
   float2 hv2[8];
 #pragma unroll
   for (int j = 0; j < 8; ++j) hv2[j] = make_float2(1.0f, 1.0f);
-  float hsum = 16.0f;  // sum of the lane's 16 h values
 
   // (row, chunk) of unit u, advanced by warps_total units per step without a division
   const int row_step = (int)(warps_total / chunks);
@@ -534,9 +545,6 @@ refine_kernel(const uint4* __restrict__ w, int64_t ld_w, const float* __restrict
           hv2[2 * i] = make_float2(t.x, t.y);
           hv2[2 * i + 1] = make_float2(t.z, t.w);
         }
-        float2 s2 = __fadd2_rn(__fadd2_rn(hv2[0], hv2[1]), __fadd2_rn(hv2[2], hv2[3]));
-        s2 = __fadd2_rn(s2, __fadd2_rn(__fadd2_rn(hv2[4], hv2[5]), __fadd2_rn(hv2[6], hv2[7])));
-        hsum = __fadd_rn(s2.x, s2.y);
       }
     }
 
@@ -568,7 +576,7 @@ refine_kernel(const uint4* __restrict__ w, int64_t ld_w, const float* __restrict
 
     // ---- is the fast winner certain?
     bool ambiguous = false;
-    if (active && hi > lo) ambiguous = !fast_winner_certain(e1, e2, energy_bound(hsum, amax_k));
+    if (active && hi > lo) ambiguous = !fast_winner_certain(e1, e2, group_energy(G, hv2));
     unsigned amb = __ballot_sync(0xFFFFFFFFu, ambiguous);
     while (amb) {
       const int owner = __ffs(amb) - 1;
@@ -594,11 +602,88 @@ refine_kernel(const uint4* __restrict__ w, int64_t ld_w, const float* __restrict
   }
 }
 
+// Constants of one search call shared by every group.
+struct SearchConsts {
+  float inv6, inv4;  // anchored_code's reciprocals for the anchors 6 and 4
+  float2 b6, b4;     // their bracketing pairs (anchored_code_fast)
+};
+
+__device__ __forceinline__ SearchConsts search_consts(const ScaleDomain& d, bool fourover6) {
+  SearchConsts k;
+  k.inv6 = rtn_inv6_raw(d.sgk);
+  k.inv4 = fourover6 ? anchor_inv_raw(d.sgk, 4.0f) : 0.0f;
+  k.b6 = anchor_brackets(d.sgk, 6.0f);
+  k.b4 = fourover6 ? anchor_brackets(d.sgk, 4.0f) : make_float2(0.f, 0.f);
+  return k;
+}
+
+// One unit of the contiguous layout: every lane searches its group g (index `go`, whose 16
+// bf16 values are p, q and sit at wg in W; h slice hv2 of column group hcol = chunk * 32 +
+// lane) and writes code byte go and nibble word go.  All 32 lanes take part (the warp
+// rescores ambiguous groups together).
+template <bool kFourOverSix>
+__device__ __forceinline__ void search_unit(const uint4& p, const uint4& q, const uint4* wg, int64_t go, int64_t chunk,
+                                            const float2 (&hv2)[8], const uint4* __restrict__ w,
+                                            const float* __restrict__ h, const float4* tab, const ScaleDomain& d,
+                                            const SearchConsts& k, const uint8_t* init_codes, int down, int up,
+                                            uint8_t* codes_out, uint2* __restrict__ packed_out) {
+  const int lane = threadIdx.x & 31;
+  const float amax_k = __fmul_rn(__uint_as_float(group_abs_max_bits(p, q) << 16), d.pw);
+  Group G;
+  unpack_group(p, q, d.pw, G);
+  int c0;
+  if (!kFourOverSix && init_codes != nullptr) {
+    c0 = init_codes[go] & 0x7F;
+    c0 = c0 < 1 ? 1 : (c0 > (int)kE4M3MaxCode ? (int)kE4M3MaxCode : c0);
+  } else {
+    c0 = kFourOverSix ? fourover6_init_code(G, wg, tab, amax_k, d.sgk, d.pw, k.inv4, k.inv6, k.b4, k.b6)
+                      : (int)anchored_code_fast(amax_k, d.sgk, k.b6.x, k.b6.y, k.inv6, 3.0f);
+  }
+  const float A = group_energy(G, hv2);
+  const int lo = max(1, c0 - down);
+  const int hi = min((int)kE4M3MaxCode, c0 + up);
+
+  float e1 = kInf, e2 = kInf;
+  int best = c0;
+  score_range(G, hv2, tab, lo, hi + 1, e1, e2, best);
+
+  const bool ambiguous = hi > lo && !fast_winner_certain(e1, e2, A);
+  unsigned amb = __ballot_sync(0xFFFFFFFFu, ambiguous);
+  while (amb) {
+    const int owner = __ffs(amb) - 1;
+    amb &= amb - 1;
+    const int64_t g_own = __shfl_sync(0xFFFFFFFFu, go, owner);
+    const int c0o = __shfl_sync(0xFFFFFFFFu, c0, owner);
+    const int loo = __shfl_sync(0xFFFFFFFFu, lo, owner);
+    const int hio = __shfl_sync(0xFFFFFFFFu, hi, owner);
+    const int bc = warp_exact_search(owner, reinterpret_cast<const uint16_t*>(w) + g_own * 16, h,
+                                     chunk * 32 + owner, c0o, loo, hio, d.sgk, d.pw);
+    if (lane == owner) best = bc;
+  }
+
+  codes_out[go] = (uint8_t)best;
+  if (packed_out != nullptr)
+    packed_out[go] = quantize_pack(G, (uint32_t)best, tab[best].z, d.sgk, d.pw,
+                                   reinterpret_cast<const uint16_t*>(wg));
+}
+
+// Loads the h slice of column chunk `chunk` (this lane's 16 values).
+__device__ __forceinline__ void load_h_slice(const float* __restrict__ h, int64_t chunk, float2 (&hv2)[8]) {
+  const int lane = threadIdx.x & 31;
+  const float4* hp = reinterpret_cast<const float4*>(h + (chunk * 32 + lane) * 16);
+#pragma unroll
+  for (int i = 0; i < 4; ++i) {
+    const float4 t = hp[i];
+    hv2[2 * i] = make_float2(t.x, t.y);
+    hv2[2 * i + 1] = make_float2(t.z, t.w);
+  }
+}
+
 // The search over a contiguous W [m, n] with n a multiple of 512 (every unit a full row
 // chunk) and contiguous outputs: the same work as refine_kernel per group, with the walk
 // reduced to pointer increments.  Unit u is groups [32 u, 32 u + 32), i.e. the 1 KB of W at
 // uint4 offset 64 u, code bytes [32 u, 32 u + 32) and nibble words [32 u, 32 u + 32); every
-// lane of every unit is active.
+// lane of every unit is active.  Warps take every warps_total-th unit (a static deal).
 template <bool kFourOverSix>
 __global__ void __launch_bounds__(kRefineThreads, 7)
 refine_linear_kernel(const uint4* __restrict__ w, const float* __restrict__ h, int64_t units, int chunks,
@@ -612,10 +697,7 @@ refine_linear_kernel(const uint4* __restrict__ w, const float* __restrict__ h, i
   __shared__ float4 tab[128];
   __shared__ __align__(16) uint4 stage[kWarpsPerRefineBlock][2][64];
   const ScaleDomain d = make_scale_domain(*global_scale);
-  const float inv6 = rtn_inv6_raw(d.sgk);
-  const float inv4 = kFourOverSix ? anchor_inv_raw(d.sgk, 4.0f) : 0.0f;
-  const float2 b6 = anchor_brackets(d.sgk, 6.0f);
-  const float2 b4 = kFourOverSix ? anchor_brackets(d.sgk, 4.0f) : make_float2(0.f, 0.f);
+  const SearchConsts k = search_consts(d, kFourOverSix);
   for (int c = threadIdx.x; c < 128; c += blockDim.x) tab[c] = candidate_constants((uint32_t)c, d.sgk);
 
   // this lane's group of unit u: uint4 words 64 u + 2 lane and the one after
@@ -637,7 +719,6 @@ refine_linear_kernel(const uint4* __restrict__ w, const float* __restrict__ h, i
   __syncthreads();  // the candidate table
 
   float2 hv2[8];
-  float hsum = 16.0f;
   int cur_chunk = -1;
 #pragma unroll
   for (int j = 0; j < 8; ++j) hv2[j] = make_float2(1.0f, 1.0f);
@@ -654,61 +735,112 @@ refine_linear_kernel(const uint4* __restrict__ w, const float* __restrict__ h, i
 
     if (h != nullptr && chunk != cur_chunk) {
       cur_chunk = chunk;
-      const float4* hp = reinterpret_cast<const float4*>(h + ((int64_t)chunk * 32 + lane) * 16);
-#pragma unroll
-      for (int i = 0; i < 4; ++i) {
-        const float4 t = hp[i];
-        hv2[2 * i] = make_float2(t.x, t.y);
-        hv2[2 * i + 1] = make_float2(t.z, t.w);
-      }
-      float2 s2 = __fadd2_rn(__fadd2_rn(hv2[0], hv2[1]), __fadd2_rn(hv2[2], hv2[3]));
-      s2 = __fadd2_rn(s2, __fadd2_rn(__fadd2_rn(hv2[4], hv2[5]), __fadd2_rn(hv2[6], hv2[7])));
-      hsum = __fadd_rn(s2.x, s2.y);
+      load_h_slice(h, chunk, hv2);
     }
 
     cp_async_wait_1();  // this lane's copy of the current unit has landed
     const uint4* cur = buf ? st1 : st0;
-    const uint4 p = cur[0], q = cur[32];
-    const float amax_k = __fmul_rn(__uint_as_float(group_abs_max_bits(p, q) << 16), d.pw);
-    Group G;
-    unpack_group(p, q, d.pw, G);
-    int c0;
-    if (!kFourOverSix && init_codes != nullptr) {
-      c0 = init_codes[go] & 0x7F;
-      c0 = c0 < 1 ? 1 : (c0 > (int)kE4M3MaxCode ? (int)kE4M3MaxCode : c0);
-    } else {
-      c0 = kFourOverSix ? fourover6_init_code(G, wp, tab, amax_k, d.sgk, d.pw, inv4, inv6, b4, b6)
-                        : (int)anchored_code_fast(amax_k, d.sgk, b6.x, b6.y, inv6, 3.0f);
-    }
-    const int lo = max(1, c0 - down);
-    const int hi = min((int)kE4M3MaxCode, c0 + up);
-
-    float e1 = kInf, e2 = kInf;
-    int best = c0;
-    score_range(G, hv2, tab, lo, hi + 1, e1, e2, best);
-
-    const bool ambiguous = hi > lo && !fast_winner_certain(e1, e2, energy_bound(hsum, amax_k));
-    unsigned amb = __ballot_sync(0xFFFFFFFFu, ambiguous);
-    while (amb) {
-      const int owner = __ffs(amb) - 1;
-      amb &= amb - 1;
-      const int64_t g_own = __shfl_sync(0xFFFFFFFFu, go, owner);
-      const int c0o = __shfl_sync(0xFFFFFFFFu, c0, owner);
-      const int loo = __shfl_sync(0xFFFFFFFFu, lo, owner);
-      const int hio = __shfl_sync(0xFFFFFFFFu, hi, owner);
-      const int bc = warp_exact_search(owner, reinterpret_cast<const uint16_t*>(w) + g_own * 16, h,
-                                       chunk * 32 + owner, c0o, loo, hio, d.sgk, d.pw);
-      if (lane == owner) best = bc;
-    }
-
-    codes_out[go] = (uint8_t)best;
-    if (packed_out != nullptr)
-      packed_out[go] = quantize_pack(G, (uint32_t)best, tab[best].z, d.sgk, d.pw,
-                                     reinterpret_cast<const uint16_t*>(wp));
+    search_unit<kFourOverSix>(cur[0], cur[32], wp, go, chunk, hv2, w, h, tab, d, k, init_codes, down, up,
+                              codes_out, packed_out);
     wp += wstep;
     go += ostep;
     chunk += chunk_step;
     if (chunk >= chunks) chunk -= chunks;
+  }
+}
+
+// Units per batch of the work-shared search.
+constexpr uint32_t kShareBatch = 2;
+
+// The same search with the units shared out at run time.  The warp schedulers favour the
+// warps of the CTAs that became resident first, so with a static deal those warps finish
+// early and the last CTAs to arrive run on alone at the end of a long call (on a
+// 28672 x 8192 matrix, k = 4, warps finished between 246 and 489 us).  Here warps take
+// batches of kShareBatch units from a counter in global memory (*next, zero at launch), so
+// the faster warps simply take more of them.  Batches run down the rows of one column chunk
+// (unit v is row v % m of chunk v / m), so a warp's h slice mostly stays put.  The first
+// batch of each warp is its index; the counter hands out the rest, one batch ahead, so the
+// atomic's latency stays hidden.  Same per-group work and bytes as refine_linear_kernel.
+template <bool kFourOverSix>
+__global__ void __launch_bounds__(kRefineThreads, 7)
+refine_shared_kernel(const uint4* __restrict__ w, const float* __restrict__ h, uint32_t m, uint32_t units,
+                     int64_t row_words, int64_t ng, const float* __restrict__ global_scale,
+                     const uint8_t* init_codes, int down, int up, uint8_t* codes_out,
+                     uint2* __restrict__ packed_out, unsigned* __restrict__ next) {
+  const int lane = threadIdx.x & 31;
+  const int warp = threadIdx.x >> 5;
+  const uint32_t warp_global = (blockIdx.x * blockDim.x + threadIdx.x) >> 5;
+  const uint32_t warps_total = (gridDim.x * blockDim.x) >> 5;
+
+  __shared__ float4 tab[128];
+  __shared__ __align__(16) uint4 stage[kWarpsPerRefineBlock][2][64];
+  const ScaleDomain d = make_scale_domain(*global_scale);
+  const SearchConsts k = search_consts(d, kFourOverSix);
+  for (int c = threadIdx.x; c < 128; c += blockDim.x) tab[c] = candidate_constants((uint32_t)c, d.sgk);
+
+  // the current unit v = (row, chunk) and the end of its batch; lane 0 holds the index of
+  // the warp's following batch
+  uint32_t v = warp_global * kShareBatch;
+  uint32_t vend = min(v + kShareBatch, units);
+  uint32_t chunk = v < units ? v / m : 0, row = v - chunk * m;
+  uint32_t batch_after = 0;
+  if (lane == 0) batch_after = warps_total + atomicAdd(next, 1u);
+  auto group_of = [&](uint32_t r, uint32_t c) { return w + (int64_t)r * row_words + (int64_t)c * 64 + 2 * lane; };
+  uint4* const st0 = &stage[warp][0][lane];
+  uint4* const st1 = &stage[warp][1][lane];
+  if (v < units) {
+    const uint4* s = group_of(row, chunk);
+    cp_async16(st0, s);
+    cp_async16(st0 + 32, s + 1);
+  }
+  cp_async_commit();
+  __syncthreads();  // the candidate table
+
+  float2 hv2[8];
+  uint32_t cur_chunk = 0xFFFFFFFFu;
+#pragma unroll
+  for (int j = 0; j < 8; ++j) hv2[j] = make_float2(1.0f, 1.0f);
+
+  int buf = 0;
+  while (v < units) {
+    // the warp's next unit: the next row of this batch, else the first of the next batch;
+    // its copy starts now
+    uint32_t v2 = v + 1, row2 = row + 1, chunk2 = chunk;
+    if (row2 == m) {
+      row2 = 0;
+      ++chunk2;
+    }
+    if (v2 >= vend) {
+      const uint32_t b = __shfl_sync(0xFFFFFFFFu, batch_after, 0);
+      if (lane == 0) batch_after = warps_total + atomicAdd(next, 1u);
+      v2 = b < units / kShareBatch + 1 ? b * kShareBatch : units;
+      vend = min(v2 + kShareBatch, units);
+      if (v2 < units) {
+        chunk2 = v2 / m;
+        row2 = v2 - chunk2 * m;
+      }
+    }
+    if (v2 < units) {
+      uint4* dst = buf ? st0 : st1;
+      const uint4* s = group_of(row2, chunk2);
+      cp_async16(dst, s);
+      cp_async16(dst + 32, s + 1);
+    }
+    cp_async_commit();
+
+    if (h != nullptr && chunk != cur_chunk) {
+      cur_chunk = chunk;
+      load_h_slice(h, chunk, hv2);
+    }
+
+    cp_async_wait_1();  // this lane's copy of the current unit has landed
+    const uint4* cur = buf ? st1 : st0;
+    search_unit<kFourOverSix>(cur[0], cur[32], group_of(row, chunk), (int64_t)row * ng + (int64_t)chunk * 32 + lane,
+                              chunk, hv2, w, h, tab, d, k, init_codes, down, up, codes_out, packed_out);
+    v = v2;
+    row = row2;
+    chunk = chunk2;
+    buf ^= 1;
   }
 }
 
@@ -808,7 +940,7 @@ cudaError_t launch_rtn_codes(const void* w, int64_t m, int64_t n, const uint32_t
 cudaError_t launch_refine(const void* w, int64_t ld_w, const float* h, int64_t m, int64_t n,
                           const float* global_scale, const uint8_t* init_codes, int64_t ld_init, int down,
                           int up, uint8_t* codes_out, int64_t ld_codes, uint8_t* packed_out, int64_t ld_packed,
-                          int ctas_per_sm, bool fourover6, cudaStream_t stream) {
+                          int ctas_per_sm, bool fourover6, unsigned* share_counter, cudaStream_t stream) {
   DeviceInfo info;
   cudaError_t err = current_device_info(&info);
   if (err != cudaSuccess) return err;
@@ -824,6 +956,25 @@ cudaError_t launch_refine(const void* w, int64_t ld_w, const float* h, int64_t m
   if (ctas_per_sm > 0) per_sm = std::min(per_sm, ctas_per_sm);
   const int64_t resident = (int64_t)info.sm_count * per_sm;
   const int64_t blocks = std::max<int64_t>(1, std::min<int64_t>((units + kWarpsPerRefineBlock - 1) / kWarpsPerRefineBlock, resident));
+  // Work sharing pays once a warp's static share is long (its spread in finishing times
+  // grows with it): from about 512 units x candidates per warp on (measured on 1 GB300:
+  // a 28672 x 8192 matrix gains 5 % at k = 4 and 12 % at k = 16, a 14336 x 4096 one nothing
+  // at k = 4 and 7 % at k = 16, and 4096 x 4096 matrices lose to the counter's cost).
+  const int64_t candidates = std::min(down + up + 1, (int)kE4M3MaxCode);
+  if (linear && share_counter != nullptr && units < (int64_t(1) << 30) && m < (int64_t(1) << 30) &&
+      units * candidates >= 512 * (resident * kWarpsPerRefineBlock)) {
+    err = cudaMemsetAsync(share_counter, 0, sizeof(unsigned), stream);
+    if (err != cudaSuccess) return err;
+    auto sk = fourover6 ? refine_shared_kernel<true> : refine_shared_kernel<false>;
+    const int64_t batches = (units + kShareBatch - 1) / kShareBatch;
+    const int64_t sblocks =
+        std::max<int64_t>(1, std::min<int64_t>((batches + kWarpsPerRefineBlock - 1) / kWarpsPerRefineBlock, resident));
+    sk<<<(unsigned)sblocks, kRefineThreads, 0, stream>>>(static_cast<const uint4*>(w), h, (uint32_t)m,
+                                                         (uint32_t)units, n / 8, ng, global_scale,
+                                                         fourover6 ? nullptr : init_codes, down, up, codes_out,
+                                                         reinterpret_cast<uint2*>(packed_out), share_counter);
+    return cudaGetLastError();
+  }
   if (linear) {
     auto lk = fourover6 ? refine_linear_kernel<true> : refine_linear_kernel<false>;
     lk<<<(unsigned)blocks, kRefineThreads, 0, stream>>>(static_cast<const uint4*>(w), h, units, (ng + 31) / 32,

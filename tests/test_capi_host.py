@@ -41,7 +41,7 @@ def test_header_declares_the_boundary():
 def test_library_exports_every_declared_symbol(lib):
     for name in declared_functions():
         assert hasattr(lib, name), name
-    assert hs.hscale_abi_version() == 3
+    assert hs.hscale_abi_version() == 4
     assert hs.library_path().exists()
 
 
@@ -185,6 +185,32 @@ def test_refine_strided_argument_errors(lib):
     assert call(h=MIS) == ERR_ALIGN
     assert call(n=40) == ERR_SHAPE
     assert call(m=0, w=None, codes=None) == OK        # empty view: no-op
+
+
+def test_refine_ws_argument_errors(lib):
+    assert lib.hscale_refine_workspace_bytes() == 16
+    f = lib.hscale_refine_scales_ws
+    ok = (FAKE, FAKE, 4, 32, FAKE, None, 0, 4, 4, FAKE, FAKE, 0, FAKE, 16, None)
+
+    def call(**kw):
+        names = ["w", "h", "m", "n", "sg", "init", "f46", "down", "up", "codes", "packed", "ctas", "ws", "wsb",
+                 "stream"]
+        args = dict(zip(names, ok))
+        args.update(kw)
+        return f(*[args[k] for k in names])
+
+    assert call(wsb=15) == ERR_WS                     # smaller than the query
+    assert call(ws=ctypes.c_void_p(0x10008)) == ERR_ALIGN
+    assert call(f46=2) == ERR_ARG
+    assert call(f46=1, init=FAKE) == ERR_ARG          # 4over6 decides the codes itself
+    assert call(ctas=-1) == ERR_ARG
+    assert call(down=126) == ERR_ARG
+    assert call(n=40) == ERR_SHAPE
+    assert call(codes=None) == ERR_NULL
+    assert call(sg=None) == ERR_NULL
+    assert call(h=MIS) == ERR_ALIGN
+    assert call(m=0, w=None, codes=None) == OK        # empty: no-op
+    assert call(m=0, w=None, codes=None, ws=None, wsb=0) == OK
 
 
 def test_refine_4over6_argument_errors(lib):

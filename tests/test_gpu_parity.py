@@ -460,6 +460,69 @@ def test_refine_launch_shape_does_not_change_results():
         assert torch.equal(c, outs[0][0]) and torch.equal(p, outs[0][1])
 
 
+def gpu_refine_ws(w, h, sg, init, fourover6, down, up, ctas_per_sm, ws):
+    m, n = w.shape
+    codes = torch.empty(m, n // 16, dtype=torch.uint8, device=dev())
+    packed = torch.empty(m, n // 2, dtype=torch.uint8, device=dev())
+    hs.hscale_refine_scales_ws(w, h, sg, init, fourover6, down, up, codes, packed, ctas_per_sm, ws)
+    torch.cuda.synchronize()
+    return codes.cpu().numpy(), packed.cpu().numpy()
+
+
+def shared_schedule_ran(ws):
+    """The work-shared kernel zeroes the workspace's first word and counts batches in it;
+    the static deal leaves the workspace as it was (filled with 0xAB here)."""
+    word = ws[:4].cpu().numpy()
+    return not np.all(word == 0xAB)
+
+
+@pytest.mark.parametrize("init", ["rtn", "given", "4over6"])
+def test_shared_schedule_matches_oracle(init):
+    """hscale_refine_scales_ws with a long search per warp (one resident CTA per SM, k = 8:
+    the work-shared schedule runs) against the oracle on every group, with an odd row
+    count so that batches straddle the end of a column chunk; then the same bytes as the
+    static deal, and again with the workspace reused."""
+    m, n, down, up = 4095, 4096, 8, 8
+    w = wl.weight(m, n, 0.02, 21, device="cpu")
+    h32 = oracle_h32(21, n, sigma_a=1.5)
+    wd, hd = w.to(dev()), torch.from_numpy(h32).to(dev())
+    sg, rtn = gpu_rtn(wd)
+    wb = bits(w)
+    s_ref, _ = oracle.global_scale(wb)
+    init_d = init_ref = None
+    exclude = np.zeros((m, n // 16), np.uint8)
+    if init == "given":
+        init_d = rtn
+        init_d[::7] = 200   # off-ladder bytes are clamped the same way on both sides
+        init_ref = init_d.cpu().numpy()
+    elif init == "4over6":
+        init_ref, nt = oracle.fourover6_codes(wb, s_ref)
+        exclude = nt.astype(np.uint8)
+    ws = torch.full((hs.hscale_refine_workspace_bytes(),), 0xAB, dtype=torch.uint8, device=dev())
+    codes, packed = gpu_refine_ws(wd, hd, sg, init_d, int(init == "4over6"), down, up, 1, ws)
+    assert shared_schedule_ran(ws)
+    ref = oracle.refine(wb, h32, s_ref, init_ref, down, up)
+    ref["near_tie"] = ref["near_tie"] | exclude
+    compare_search(ref, codes, packed, f"shared schedule {m}x{n} init {init}")
+    codes2, packed2 = gpu_refine_ws(wd, hd, sg, init_d, int(init == "4over6"), down, up, 1, ws)
+    assert np.array_equal(codes2, codes) and np.array_equal(packed2, packed)
+    ws_none = gpu_refine_ws(wd, hd, sg, init_d, int(init == "4over6"), down, up, 1, None)
+    assert np.array_equal(ws_none[0], codes) and np.array_equal(ws_none[1], packed)
+
+
+def test_shared_schedule_only_for_long_searches():
+    """A short search (4096 x 4096 at k = 4 over every SM) keeps the static deal and leaves
+    the workspace untouched; the bytes equal hscale_refine_scales'."""
+    w = wl.weight(4096, 4096, 0.02, 22, device=dev())
+    h = torch.from_numpy(oracle_h32(22, 4096)).to(dev())
+    sg, _ = gpu_rtn(w)
+    ws = torch.full((16,), 0xAB, dtype=torch.uint8, device=dev())
+    codes, packed = gpu_refine_ws(w, h, sg, None, 0, 4, 4, 0, ws)
+    assert not shared_schedule_ran(ws)
+    ref = gpu_refine(w, h.cpu().numpy(), sg, None, 4, 4)
+    assert np.array_equal(ref[0], codes) and np.array_equal(ref[1], packed)
+
+
 def test_refine_is_deterministic():
     w = small_layer(3, 512, 1024)
     h32 = oracle_h32(3, 1024)
@@ -961,6 +1024,13 @@ def full_size_check(name, sample_rows, layer_index=0, windows=None, fourover6=Fa
                 # the one-pass form, at the launch shape the bench times it with (4 CTAs/SM)
                 codes_f, packed_f = gpu_refine_4over6(w, h_ref[L.input_space], sg, down, up, 4)
                 assert np.array_equal(codes_f, codes_g) and np.array_equal(packed_f, packed_g)
+            # the entry point bench.py calls (work-shared schedule where the search is long),
+            # alone and at 4 CTAs per SM
+            hd32 = torch.from_numpy(h_ref[L.input_space]).to(dev())
+            ws = torch.zeros(hs.hscale_refine_workspace_bytes(), dtype=torch.uint8, device=dev())
+            for ctas in (0, 4):
+                codes_w, packed_w = gpu_refine_ws(w, hd32, sg, init, 0, down, up, ctas, ws)
+                assert np.array_equal(codes_w, codes_g) and np.array_equal(packed_w, packed_g)
             # the column-blocked searches of `bench.py --col-block 1024` (views, 4 CTAs/SM
             # but the last block)
             hd = torch.from_numpy(h_ref[L.input_space]).to(dev())
