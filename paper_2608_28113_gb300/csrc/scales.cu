@@ -20,14 +20,14 @@
 //   4 eps y* |q* - y*| + 8 eps^2 y*^2 (also where a midpoint falls between y and y*:
 //   both distances to the grid are then within eps y* of half the grid gap), so by
 //   Cauchy-Schwarz the fast score is within
-//        4 eps sqrt(A E*) + 8 eps^2 A + 13 * 2^-24 E*    (A = sum_j h_j a_j^2)
+//        4 eps sqrt(A E*) + 8 eps^2 A + 14 * 2^-24 E*    (A = sum_j h_j a_j^2)
 //   of the exact score E*; in terms of the fast score E that is at most
-//   4.01 * 2^-23 sqrt(A E) + 33 * 2^-46 A + 13 * 2^-24 E.  When
+//   4.01 * 2^-23 sqrt(A E) + 33 * 2^-46 A + 15 * 2^-24 E.  When
 //        runner-up - best > 2^-18 E2 + 2^-19 sqrt(A E2) + 2^-35 A
 //   (more than the two errors together, with at least 2x slack on every term) and
 //   E2 >= 2^-36 A (so the bound grows slower than the score for every other candidate),
-//   the fast winner is the exact winner; the kernel puts the upper bound
-//   (sum_j h_j) max_j a_j^2 in place of A, which only widens the margin.  (A quotient
+//   the fast winner is the exact winner; the kernel puts an upper bound of A in its place
+//   (the fp32 sum times 1 + 2^-19; a larger A only widens the margin).  (A quotient
 //   below the normal range carries an absolute error of half a denormal unit instead;
 //   such an element rounds to zero under every candidate, and a group made only of them
 //   has scores within rounding of A under every candidate, which the 2^-18 E2 term sends
@@ -80,15 +80,20 @@ __device__ __forceinline__ float global_scale_of(uint32_t amax_bits) {
   return amax == 0.0f ? 1.0f : __fdiv_rn(amax, 2688.0f);  // 6 * 448
 }
 
+// max(|x|, |y|) of two bf16 pairs, half by half (the sign of each half is the product of
+// the inputs' signs; finite inputs).  One of the inputs' magnitudes is returned exactly.
+__device__ __forceinline__ uint32_t bf16x2_absmax(uint32_t x, uint32_t y) {
+  uint32_t r;
+  asm("max.xorsign.abs.bf16x2 %0, %1, %2;" : "=r"(r) : "r"(x), "r"(y));
+  return r;
+}
+
+// The 16-bit |bf16| pattern of the group's largest magnitude (for finite values the order
+// of magnitudes is the order of their patterns).
 __device__ __forceinline__ uint32_t group_abs_max_bits(const uint4& a, const uint4& b) {
-  uint32_t m = __vmaxu2(a.x & 0x7FFF7FFFu, a.y & 0x7FFF7FFFu);
-  m = __vmaxu2(m, a.z & 0x7FFF7FFFu);
-  m = __vmaxu2(m, a.w & 0x7FFF7FFFu);
-  m = __vmaxu2(m, b.x & 0x7FFF7FFFu);
-  m = __vmaxu2(m, b.y & 0x7FFF7FFFu);
-  m = __vmaxu2(m, b.z & 0x7FFF7FFFu);
-  m = __vmaxu2(m, b.w & 0x7FFF7FFFu);
-  return max(m & 0xFFFFu, m >> 16);
+  const uint32_t m = bf16x2_absmax(bf16x2_absmax(bf16x2_absmax(a.x, a.y), bf16x2_absmax(a.z, a.w)),
+                                   bf16x2_absmax(bf16x2_absmax(b.x, b.y), bf16x2_absmax(b.z, b.w)));
+  return bf16x2_absmax(m, __byte_perm(m, 0, 0x1032)) & 0x7FFFu;
 }
 
 // ---------------------------------------------------------------- RTN codes
@@ -164,19 +169,18 @@ __device__ __forceinline__ float2 e2m1_residual2(float2 y) {
 
 // Fast score of one candidate from its table entry t (see the file comment): per pair of
 // elements one packed multiply for the quotients, the hardware rounding and residuals,
-// a packed square and a packed FMA into the h-weighted sum; then one multiply by s'^2.
+// a packed square and a packed FMA into the h-weighted sum (one chain per half of the
+// pair: the candidates scored side by side give the independent work); then the halves'
+// sum and one multiply by s'^2.
 __device__ __forceinline__ float fast_score(const Group& G, const float2 (&hv2)[8], float4 t) {
   const float2 inv2 = make_float2(t.z, t.w);
-  float2 acc0 = make_float2(0.f, 0.f), acc1 = make_float2(0.f, 0.f);
+  float2 acc = make_float2(0.f, 0.f);
 #pragma unroll
   for (int i = 0; i < 8; ++i) {
     const float2 d = e2m1_residual2(__fmul2_rn(G.a[i], inv2));
-    const float2 dd = __fmul2_rn(d, d);
-    if (i & 1) acc1 = __ffma2_rn(hv2[i], dd, acc1);
-    else acc0 = __ffma2_rn(hv2[i], dd, acc0);
+    acc = __ffma2_rn(hv2[i], __fmul2_rn(d, d), acc);
   }
-  const float2 t2 = __fadd2_rn(acc0, acc1);
-  return __fmul_rn(t.x, __fadd_rn(t2.x, t2.y));
+  return __fmul_rn(t.x, __fadd_rn(acc.x, acc.y));
 }
 
 // Running best (e1, best) and runner-up e2 (e1 <= e2); branch-free: a select and three

@@ -326,6 +326,37 @@ def test_refine_edge_groups():
         assert codes[5, 6] == ref["codes"][5, 6]
 
 
+def test_group_amax_over_bf16_subnormals_and_signs():
+    """The group amax (a packed bf16 max of magnitudes) where it decides the RTN code: every
+    value a bf16 subnormal of either sign, +-0 mixes, a negative largest magnitude, under
+    s_g = 2^-126 (the tensor's amax 21 * 2^-119, the smallest normal s_g), so that the
+    codes of subnormal groups vary with their amax.  RTN codes, the search's own RTN start
+    and the packed nibbles against the oracle."""
+    rng = np.random.default_rng(17)
+    m, n = 64, 512
+    b = rng.integers(1, 0x80, size=(m, n), dtype=np.uint16)          # |w| subnormal
+    b |= (rng.integers(0, 2, size=(m, n), dtype=np.uint16) << 15)   # random signs
+    b[0, 0] = 0x0628                                                # 21 * 2^-119: the amax
+    b[1, :16] = 0x8000                                              # all -0
+    b[2, 16:32] = 0x0000
+    b[2, 20] = 0x8045                                               # one negative subnormal
+    b[3, 32:48] = 0x807F                                            # equal magnitudes, negative
+    b[3, 40] = 0x007F
+    for r in range(4, m):                                           # largest magnitude negative
+        g = (r * 5) % (n // 16)
+        b[r, 16 * g + (r % 16)] = 0x807F
+    w = from_bits(b)
+    wd = w.to(dev())
+    sg, codes = gpu_rtn(wd)
+    s_ref, _ = oracle.global_scale(b)
+    assert s_ref == np.float32(2.0 ** -126) and sg.cpu().numpy()[0] == s_ref
+    assert np.array_equal(codes.cpu().numpy(), oracle.rtn_codes(b, s_ref))
+    h32 = oracle_h32(17, n)
+    ref = oracle.refine(b, h32, s_ref, None, 4, 4)
+    codes_g, packed_g = gpu_refine(wd, h32, sg, None, 4, 4)
+    compare_search(ref, codes_g, packed_g, "bf16 subnormal groups")
+
+
 def test_refine_inline_rtn_on_exact_e4m3_ties():
     """The search's own RTN start (init_codes = NULL) on groups whose max sits exactly on every
     E4M3 ladder value and midpoint (s_g = 2^-10): exact ties are decided half-to-even, as in
