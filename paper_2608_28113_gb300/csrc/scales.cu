@@ -227,6 +227,16 @@ __device__ __forceinline__ float group_energy(const Group& G, const float2 (&hv2
   return __fmul_rn(__fadd_rn(acc.x, acc.y), 1.0f + 0x1p-19f);
 }
 
+// A sufficient condition for fast_winner_certain that costs five operations: a relative
+// gap above 2^-9 with A <= 2^18 E2 (A_bound any upper bound of A, here (sum h) amax^2)
+// gives a margin of at most (2^-18 + 2^-19 2^9 + 2^-35 2^18) E2 < 2^-9 E2, and
+// E2 >= 2^-36 A.  (The fp32 rounding of the gap and of A_bound is a few units of 2^-24,
+// far inside the factor of two between 2^-9 and the margin.)  A zero, infinite or NaN
+// runner-up fails it.
+__device__ __forceinline__ bool fast_winner_clear(float e1, float e2, float A_bound) {
+  return __fsub_rn(e2, e1) > __fmul_rn(0x1p-9f, e2) && A_bound <= __fmul_rn(0x1p18f, e2);
+}
+
 // tie rule of the search: smaller error, then smaller |shift|, then smaller shift
 __device__ __forceinline__ bool better(float e, int c, float be, int bc, int c0) {
   if (e != be) return e < be;
@@ -627,7 +637,7 @@ __device__ __forceinline__ SearchConsts search_consts(const ScaleDomain& d, bool
 // rescores ambiguous groups together).
 template <bool kFourOverSix>
 __device__ __forceinline__ void search_unit(const uint4& p, const uint4& q, const uint4* wg, int64_t go, int64_t chunk,
-                                            const float2 (&hv2)[8], const uint4* __restrict__ w,
+                                            const float2 (&hv2)[8], float hsum, const uint4* __restrict__ w,
                                             const float* __restrict__ h, const float4* tab, const ScaleDomain& d,
                                             const SearchConsts& k, const uint8_t* init_codes, int down, int up,
                                             uint8_t* codes_out, uint2* __restrict__ packed_out) {
@@ -643,7 +653,6 @@ __device__ __forceinline__ void search_unit(const uint4& p, const uint4& q, cons
     c0 = kFourOverSix ? fourover6_init_code(G, wg, tab, amax_k, d.sgk, d.pw, k.inv4, k.inv6, k.b4, k.b6)
                       : (int)anchored_code_fast(amax_k, d.sgk, k.b6.x, k.b6.y, k.inv6, 3.0f);
   }
-  const float A = group_energy(G, hv2);
   const int lo = max(1, c0 - down);
   const int hi = min((int)kE4M3MaxCode, c0 + up);
 
@@ -651,7 +660,10 @@ __device__ __forceinline__ void search_unit(const uint4& p, const uint4& q, cons
   int best = c0;
   score_range(G, hv2, tab, lo, hi + 1, e1, e2, best);
 
-  const bool ambiguous = hi > lo && !fast_winner_certain(e1, e2, A);
+  // the cheap sufficient test with the loose energy bound first; the exact energy and the
+  // full test only for the groups it cannot clear
+  bool ambiguous = hi > lo && !fast_winner_clear(e1, e2, energy_bound(hsum, amax_k));
+  if (ambiguous) ambiguous = !fast_winner_certain(e1, e2, group_energy(G, hv2));
   unsigned amb = __ballot_sync(0xFFFFFFFFu, ambiguous);
   while (amb) {
     const int owner = __ffs(amb) - 1;
@@ -671,8 +683,9 @@ __device__ __forceinline__ void search_unit(const uint4& p, const uint4& q, cons
                                    reinterpret_cast<const uint16_t*>(wg));
 }
 
-// Loads the h slice of column chunk `chunk` (this lane's 16 values).
-__device__ __forceinline__ void load_h_slice(const float* __restrict__ h, int64_t chunk, float2 (&hv2)[8]) {
+// Loads the h slice of column chunk `chunk` (this lane's 16 values) and its sum.
+__device__ __forceinline__ void load_h_slice(const float* __restrict__ h, int64_t chunk, float2 (&hv2)[8],
+                                             float& hsum) {
   const int lane = threadIdx.x & 31;
   const float4* hp = reinterpret_cast<const float4*>(h + (chunk * 32 + lane) * 16);
 #pragma unroll
@@ -681,6 +694,9 @@ __device__ __forceinline__ void load_h_slice(const float* __restrict__ h, int64_
     hv2[2 * i] = make_float2(t.x, t.y);
     hv2[2 * i + 1] = make_float2(t.z, t.w);
   }
+  float2 s2 = __fadd2_rn(__fadd2_rn(hv2[0], hv2[1]), __fadd2_rn(hv2[2], hv2[3]));
+  s2 = __fadd2_rn(s2, __fadd2_rn(__fadd2_rn(hv2[4], hv2[5]), __fadd2_rn(hv2[6], hv2[7])));
+  hsum = __fadd_rn(s2.x, s2.y);
 }
 
 // The search over a contiguous W [m, n] with n a multiple of 512 (every unit a full row
@@ -723,6 +739,7 @@ refine_linear_kernel(const uint4* __restrict__ w, const float* __restrict__ h, i
   __syncthreads();  // the candidate table
 
   float2 hv2[8];
+  float hsum = 16.0f;  // sum of the lane's 16 h values (h = 1 without h)
   int cur_chunk = -1;
 #pragma unroll
   for (int j = 0; j < 8; ++j) hv2[j] = make_float2(1.0f, 1.0f);
@@ -739,12 +756,12 @@ refine_linear_kernel(const uint4* __restrict__ w, const float* __restrict__ h, i
 
     if (h != nullptr && chunk != cur_chunk) {
       cur_chunk = chunk;
-      load_h_slice(h, chunk, hv2);
+      load_h_slice(h, chunk, hv2, hsum);
     }
 
     cp_async_wait_1();  // this lane's copy of the current unit has landed
     const uint4* cur = buf ? st1 : st0;
-    search_unit<kFourOverSix>(cur[0], cur[32], wp, go, chunk, hv2, w, h, tab, d, k, init_codes, down, up,
+    search_unit<kFourOverSix>(cur[0], cur[32], wp, go, chunk, hv2, hsum, w, h, tab, d, k, init_codes, down, up,
                               codes_out, packed_out);
     wp += wstep;
     go += ostep;
@@ -801,6 +818,7 @@ refine_shared_kernel(const uint4* __restrict__ w, const float* __restrict__ h, u
   __syncthreads();  // the candidate table
 
   float2 hv2[8];
+  float hsum = 16.0f;
   uint32_t cur_chunk = 0xFFFFFFFFu;
 #pragma unroll
   for (int j = 0; j < 8; ++j) hv2[j] = make_float2(1.0f, 1.0f);
@@ -834,13 +852,13 @@ refine_shared_kernel(const uint4* __restrict__ w, const float* __restrict__ h, u
 
     if (h != nullptr && chunk != cur_chunk) {
       cur_chunk = chunk;
-      load_h_slice(h, chunk, hv2);
+      load_h_slice(h, chunk, hv2, hsum);
     }
 
     cp_async_wait_1();  // this lane's copy of the current unit has landed
     const uint4* cur = buf ? st1 : st0;
     search_unit<kFourOverSix>(cur[0], cur[32], group_of(row, chunk), (int64_t)row * ng + (int64_t)chunk * 32 + lane,
-                              chunk, hv2, w, h, tab, d, k, init_codes, down, up, codes_out, packed_out);
+                              chunk, hv2, hsum, w, h, tab, d, k, init_codes, down, up, codes_out, packed_out);
     v = v2;
     row = row2;
     chunk = chunk2;
