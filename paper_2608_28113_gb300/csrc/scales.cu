@@ -866,6 +866,92 @@ refine_shared_kernel(const uint4* __restrict__ w, const float* __restrict__ h, u
   }
 }
 
+// Warps of refine_sm_kernel's CTA: 7 x 4, the search warps one SM holds at 72 registers.
+constexpr int kSmWarps = 28;
+
+// The search of a matrix alone on the GPU, one CTA per SM: the CTA takes an equal share
+// of the (column-major) units and its warps share them out through a counter in shared
+// memory, one unit at a time.  Warps of one CTA all became resident together, but the
+// schedulers still favour some of them; here the favoured ones simply take more units, so
+// every warp of the SM finishes within about one unit of the others.  The SMs' shares are
+// equal, which suits a search that has the GPU to itself (refine_shared_kernel's global
+// counter balances the SMs as well, for long searches).  Same per-group work and bytes as
+// refine_linear_kernel.
+template <bool kFourOverSix>
+__global__ void __launch_bounds__(kSmWarps * 32, 1)
+refine_sm_kernel(const uint4* __restrict__ w, const float* __restrict__ h, uint32_t m, uint32_t units,
+                 int64_t row_words, int64_t ng, const float* __restrict__ global_scale,
+                 const uint8_t* init_codes, int down, int up, uint8_t* codes_out,
+                 uint2* __restrict__ packed_out) {
+  const int lane = threadIdx.x & 31;
+  const int warp = threadIdx.x >> 5;
+  __shared__ float4 tab[128];
+  __shared__ __align__(16) uint4 stage[kSmWarps][2][64];
+  __shared__ unsigned next_unit;
+  const ScaleDomain d = make_scale_domain(*global_scale);
+  const SearchConsts k = search_consts(d, kFourOverSix);
+  for (int c = threadIdx.x; c < 128; c += blockDim.x) tab[c] = candidate_constants((uint32_t)c, d.sgk);
+
+  // this CTA's units [vbeg, vlim); unit v is row v % m of column chunk v / m
+  const uint32_t vbeg = (uint32_t)(((uint64_t)units * blockIdx.x) / gridDim.x);
+  const uint32_t vlim = (uint32_t)(((uint64_t)units * (blockIdx.x + 1)) / gridDim.x);
+  if (threadIdx.x == 0) next_unit = vbeg + kSmWarps;  // the first kSmWarps units go to warps in order
+  auto group_of = [&](uint32_t r, uint32_t c) { return w + (int64_t)r * row_words + (int64_t)c * 64 + 2 * lane; };
+  uint4* const st0 = &stage[warp][0][lane];
+  uint4* const st1 = &stage[warp][1][lane];
+  uint32_t v = vbeg + warp;
+  uint32_t chunk = v < vlim ? v / m : 0, row = v - chunk * m;
+  if (v < vlim) {
+    const uint4* s = group_of(row, chunk);
+    cp_async16(st0, s);
+    cp_async16(st0 + 32, s + 1);
+  }
+  cp_async_commit();
+  __syncthreads();  // the candidate table and the counter
+
+  float2 hv2[8];
+  float hsum = 16.0f;
+  uint32_t cur_chunk = 0xFFFFFFFFu;
+#pragma unroll
+  for (int j = 0; j < 8; ++j) hv2[j] = make_float2(1.0f, 1.0f);
+
+  int buf = 0;
+  while (v < vlim) {
+    // the warp's next unit (counter values grow, so its chunk is at or after this one's);
+    // its copy starts now
+    uint32_t v2 = 0;
+    if (lane == 0) v2 = atomicAdd(&next_unit, 1u);
+    v2 = __shfl_sync(0xFFFFFFFFu, v2, 0);
+    uint32_t chunk2 = chunk, row2 = 0;
+    if (v2 < vlim) {
+      row2 = v2 - chunk * m;
+      while (row2 >= m) {
+        ++chunk2;
+        row2 -= m;
+      }
+      uint4* dst = buf ? st0 : st1;
+      const uint4* s = group_of(row2, chunk2);
+      cp_async16(dst, s);
+      cp_async16(dst + 32, s + 1);
+    }
+    cp_async_commit();
+
+    if (h != nullptr && chunk != cur_chunk) {
+      cur_chunk = chunk;
+      load_h_slice(h, chunk, hv2, hsum);
+    }
+
+    cp_async_wait_1();  // this lane's copy of the current unit has landed
+    const uint4* cur = buf ? st1 : st0;
+    search_unit<kFourOverSix>(cur[0], cur[32], group_of(row, chunk), (int64_t)row * ng + (int64_t)chunk * 32 + lane,
+                              chunk, hv2, hsum, w, h, tab, d, k, init_codes, down, up, codes_out, packed_out);
+    v = v2;
+    row = row2;
+    chunk = chunk2;
+    buf ^= 1;
+  }
+}
+
 // ---------------------------------------------------------------- pack with given codes
 __global__ void __launch_bounds__(256) pack_kernel(const uint4* __restrict__ w, int64_t groups,
                                                    const float* __restrict__ global_scale,
@@ -996,6 +1082,22 @@ cudaError_t launch_refine(const void* w, int64_t ld_w, const float* h, int64_t m
                                                          fourover6 ? nullptr : init_codes, down, up, codes_out,
                                                          reinterpret_cast<uint2*>(packed_out), share_counter);
     return cudaGetLastError();
+  }
+  // A search alone on the GPU with at least two units per warp: one CTA per SM sharing its
+  // units out in shared memory (1 GB300, k = 4: 14336 x 4096 127.6 -> 115.4 us, 4096 x 4096
+  // 41.6 -> 39.6 us; 1024 x 4096, one or two units per warp, keeps the static deal).
+  if (linear && ctas_per_sm == 0 && units >= 2 * (int64_t)info.sm_count * kSmWarps && units < (int64_t(1) << 30) &&
+      m < (int64_t(1) << 30)) {
+    auto qk = fourover6 ? refine_sm_kernel<true> : refine_sm_kernel<false>;
+    const int fits = fourover6 ? occupancy_blocks<refine_sm_kernel<true>>(kSmWarps * 32)
+                               : occupancy_blocks<refine_sm_kernel<false>>(kSmWarps * 32);
+    if (fits >= 1) {
+      qk<<<(unsigned)info.sm_count, kSmWarps * 32, 0, stream>>>(static_cast<const uint4*>(w), h, (uint32_t)m,
+                                                               (uint32_t)units, n / 8, ng, global_scale,
+                                                               fourover6 ? nullptr : init_codes, down, up, codes_out,
+                                                               reinterpret_cast<uint2*>(packed_out));
+      return cudaGetLastError();
+    }
   }
   if (linear) {
     auto lk = fourover6 ? refine_linear_kernel<true> : refine_linear_kernel<false>;

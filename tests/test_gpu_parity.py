@@ -508,11 +508,13 @@ def shared_schedule_ran(ws):
 
 
 @pytest.mark.parametrize("init", ["rtn", "given", "4over6"])
-def test_shared_schedule_matches_oracle(init):
-    """hscale_refine_scales_ws with a long search per warp (one resident CTA per SM, k = 8:
-    the work-shared schedule runs) against the oracle on every group, with an odd row
-    count so that batches straddle the end of a column chunk; then the same bytes as the
-    static deal, and again with the workspace reused."""
+def test_search_schedules_match_oracle(init):
+    """The three deals of the contiguous search on one matrix, each against the oracle on
+    every group: the global work-sharing counter (hscale_refine_scales_ws, one resident CTA
+    per SM, k = 8: a long search per warp), the per-SM queue (the matrix alone on the GPU,
+    no workspace) and the static deal (CTAs capped at 7 per SM).  An odd row count makes
+    units of consecutive queue positions straddle the end of a column chunk.  The
+    workspace is reused for a second call, and all three write the same bytes."""
     m, n, down, up = 4095, 4096, 8, 8
     w = wl.weight(m, n, 0.02, 21, device="cpu")
     h32 = oracle_h32(21, n, sigma_a=1.5)
@@ -524,21 +526,24 @@ def test_shared_schedule_matches_oracle(init):
     exclude = np.zeros((m, n // 16), np.uint8)
     if init == "given":
         init_d = rtn
-        init_d[::7] = 200   # off-ladder bytes are clamped the same way on both sides
+        init_d[::7] = 200   # other starting codes (the sign bit is cleared on both sides)
         init_ref = init_d.cpu().numpy()
     elif init == "4over6":
         init_ref, nt = oracle.fourover6_codes(wb, s_ref)
         exclude = nt.astype(np.uint8)
-    ws = torch.full((hs.hscale_refine_workspace_bytes(),), 0xAB, dtype=torch.uint8, device=dev())
-    codes, packed = gpu_refine_ws(wd, hd, sg, init_d, int(init == "4over6"), down, up, 1, ws)
-    assert shared_schedule_ran(ws)
+    f46 = int(init == "4over6")
     ref = oracle.refine(wb, h32, s_ref, init_ref, down, up)
     ref["near_tie"] = ref["near_tie"] | exclude
-    compare_search(ref, codes, packed, f"shared schedule {m}x{n} init {init}")
-    codes2, packed2 = gpu_refine_ws(wd, hd, sg, init_d, int(init == "4over6"), down, up, 1, ws)
-    assert np.array_equal(codes2, codes) and np.array_equal(packed2, packed)
-    ws_none = gpu_refine_ws(wd, hd, sg, init_d, int(init == "4over6"), down, up, 1, None)
-    assert np.array_equal(ws_none[0], codes) and np.array_equal(ws_none[1], packed)
+    ws = torch.full((hs.hscale_refine_workspace_bytes(),), 0xAB, dtype=torch.uint8, device=dev())
+    shared = gpu_refine_ws(wd, hd, sg, init_d, f46, down, up, 1, ws)
+    assert shared_schedule_ran(ws)
+    compare_search(ref, *shared, f"global counter {m}x{n} init {init}")
+    again = gpu_refine_ws(wd, hd, sg, init_d, f46, down, up, 1, ws)
+    queue = gpu_refine_ws(wd, hd, sg, init_d, f46, down, up, 0, None)
+    compare_search(ref, *queue, f"per-SM queue {m}x{n} init {init}")
+    static = gpu_refine_ws(wd, hd, sg, init_d, f46, down, up, 7, None)
+    for other in (again, queue, static):
+        assert np.array_equal(other[0], shared[0]) and np.array_equal(other[1], shared[1])
 
 
 def test_shared_schedule_only_for_long_searches():
