@@ -917,17 +917,17 @@ refine_sm_kernel(const uint4* __restrict__ w, const float* __restrict__ h, uint3
 
   int buf = 0;
   while (v < vlim) {
-    // the warp's next unit (counter values grow, so its chunk is at or after this one's);
-    // its copy starts now
+    // the warp's next unit (counter values grow, so its chunk is at or after this one's;
+    // a division only when it leaves this chunk); its copy starts now
     uint32_t v2 = 0;
     if (lane == 0) v2 = atomicAdd(&next_unit, 1u);
     v2 = __shfl_sync(0xFFFFFFFFu, v2, 0);
     uint32_t chunk2 = chunk, row2 = 0;
     if (v2 < vlim) {
       row2 = v2 - chunk * m;
-      while (row2 >= m) {
-        ++chunk2;
-        row2 -= m;
+      if (row2 >= m) {
+        chunk2 = v2 / m;
+        row2 = v2 - chunk2 * m;
       }
       uint4* dst = buf ? st0 : st1;
       const uint4* s = group_of(row2, chunk2);

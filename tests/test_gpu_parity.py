@@ -546,6 +546,33 @@ def test_search_schedules_match_oracle(init):
         assert np.array_equal(other[0], shared[0]) and np.array_equal(other[1], shared[1])
 
 
+@pytest.mark.parametrize("m,n", [(1, 512 * 20000), (20000, 512)])
+def test_search_schedules_on_extreme_shapes(m, n):
+    """The per-SM queue (matrix alone, no workspace) and the global counter (workspace, one
+    CTA per SM) where units are one row long and every unit is a new column chunk, or one
+    chunk wide: against the oracle, and the same bytes as the static deal."""
+    w = wl.weight(m, n, 0.02, 23, device="cpu")
+    # h of 2048 tokens with the workload's channel magnitudes, in expectation (X itself would
+    # be 2048 x n)
+    a = wl.channel_magnitudes(n, 1.0, 8, 50.0, 23)
+    h32 = (a.double() ** 2 * 2048.0).float().numpy()
+    wd, hd = w.to(dev()), torch.from_numpy(h32).to(dev())
+    sg, _ = gpu_rtn(wd)
+    wb = bits(w)
+    s_ref, _ = oracle.global_scale(wb)
+    queue = gpu_refine_ws(wd, hd, sg, None, 0, 8, 8, 0, None)
+    # the oracle parallelises over rows: on the single row, its first 65536 columns
+    cols = n if m > 1 else 65536
+    ref = oracle.refine(np.ascontiguousarray(wb[:, :cols]), h32[:cols], s_ref, None, 8, 8)
+    compare_search(ref, queue[0][:, :cols // 16], queue[1][:, :cols // 2], f"per-SM queue {m}x{n} ({cols} columns)")
+    ws = torch.full((16,), 0xAB, dtype=torch.uint8, device=dev())
+    shared = gpu_refine_ws(wd, hd, sg, None, 0, 8, 8, 1, ws)
+    assert shared_schedule_ran(ws)
+    static = gpu_refine_ws(wd, hd, sg, None, 0, 8, 8, 7, None)
+    for other in (shared, static):
+        assert np.array_equal(other[0], queue[0]) and np.array_equal(other[1], queue[1])
+
+
 def test_shared_schedule_only_for_long_searches():
     """A short search (4096 x 4096 at k = 4 over every SM) keeps the static deal and leaves
     the workspace untouched; the bytes equal hscale_refine_scales'."""
