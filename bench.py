@@ -82,6 +82,10 @@ def parse():
                    help="the search's unit schedule: 'shared' passes hscale_refine_scales_ws a workspace "
                         "(units shared out at run time in long searches), 'static' passes none; 'auto' "
                         "shares except in searches that fill the SMs beside a Hessian pass")
+    p.add_argument("--weight-pass", choices=["early", "with-search"], default="early",
+                   help="where the graphs put each matrix's weight-only calls (s_g): 'early' on a side "
+                        "stream alongside the first Hessian pass; 'with-search' on the search stream "
+                        "right before the matrix's search (its W may still be in L2)")
     p.add_argument("--pipeline", choices=["auto", "on", "off"], default="auto",
                    help="run each step's last searches alongside the next step's first Hessian pass "
                         "(h, s_g and initial codes double-buffered).  auto (default) and on: pipelined "
@@ -321,6 +325,7 @@ class Work:
         self.h_launches = len(calls)
         self.ws = None
         self.search_schedule = "auto"
+        self.weight_pass = "early"
 
     def stage_estimates(self):
         """(name, Hessian seconds, search seconds) per input space, from nominal rates
@@ -503,12 +508,16 @@ class StepGraphs:
                 with torch.cuda.graph(g):
                     for M in work.mats:
                         if M.space is S:
+                            if work.weight_pass == "with-search" and c0 == 0:
+                                init_codes(hs, work, M)
                             refine_block(hs, work, M, c0, c1, down, up,
                                          ctas_per_sm=overlap_ctas if alongside else 0)
                 gr.append(g)
-            gi = torch.cuda.CUDAGraph()
-            with torch.cuda.graph(gi):
-                init_phase(hs, work)
+            gi = None
+            if work.weight_pass == "early":
+                gi = torch.cuda.CUDAGraph()
+                with torch.cuda.graph(gi):
+                    init_phase(hs, work)
             self.gh.append(gh)
             self.gr.append(gr)
             self.gi.append(gi)
@@ -543,10 +552,11 @@ class StepGraphs:
             main.wait_event(self.done[p])
         self.side.wait_stream(main)
         self.search.wait_stream(main)
-        with torch.cuda.stream(self.side):
-            self.gi[p].replay()
-            self.ev_init.record(self.side)
-        self.search.wait_event(self.ev_init)
+        if self.gi[p] is not None:
+            with torch.cuda.stream(self.side):
+                self.gi[p].replay()
+                self.ev_init.record(self.side)
+            self.search.wait_event(self.ev_init)
         for i, g in enumerate(self.gh[p]):
             g.replay()
             self.ev_h[i].record(main)
@@ -1040,6 +1050,7 @@ def measure_workload(hs, d: Dist, args, W: wl.Workload, win, dev, overlap_ctas: 
     (result dict, work); the work keeps the step's outputs."""
     work = Work(W, d.rank, win, dev, tokens=tokens, init=init, col_block=col_block)
     work.search_schedule = args.search_schedule
+    work.weight_pass = args.weight_pass
     work.ws = torch.empty(hs.hscale_rtn_workspace_bytes(), dtype=torch.uint8, device=dev)
     torch.cuda.synchronize()
 
@@ -1177,6 +1188,7 @@ def extra_workload(hs, d: Dist, args, name: str, dev) -> dict:
            "window": [W.window[0], W.window[0]], "groups": work.groups,
            "ms_per_step": res["ms_step"], "value": res["value"], "unit": UNIT,
            "schedule": "pipelined" if res["graphs"].pipeline else "sequential",
+           "weight_pass": res["work"].weight_pass,
            "roofline_hessian": compact_roofline(res["roofline_hessian"]),
            "roofline_search": compact_roofline(res["roofline_search"]),
            "step_hbm": {k: res["step_hbm"][k] for k in ("bytes", "achieved", "peak", "unit", "frac")},
@@ -1228,6 +1240,7 @@ def gpu_arm(args, d: Dist):
                    "window": list(win), "init": work.init, "groups": work.groups,
                    "col_block": work.col_block,
                    "schedule": "pipelined" if graphs.pipeline else "sequential",
+                   "weight_pass": work.weight_pass,
                    "l2": "inputs larger than L2: %.2f GB of X streamed per step" %
                          (sum(S.tokens * S.n * 2 for S in work.spaces.values()) / 1e9),
                    "parallelism": f"independent layer per GPU x{d.world}"},
