@@ -2,10 +2,18 @@
 //
 //   amax_kernel         amax|W| (integer max of |bf16| bit patterns; order-free)
 //   rtn_codes_kernel    s_g = amax / 2688 and the RTN code of every group (Eq. 7)
-//   refine_kernel       Algorithm 1: per group, every distinct E4M3 code in the window
+//   refine_*_kernel     Algorithm 1: per group, every distinct E4M3 code in the window
 //                       (Eqs. 8-11) is scored by sum_j h_j (|w_j| - s q_j)^2 (Eqs. 6, 12,
-//                       13); the best code is re-quantized exactly and packed.  Its
-//                       4over6 instance decides Algorithm 2's initial code in place
+//                       13); the best code is re-quantized exactly and packed.  Their
+//                       4over6 instances decide Algorithm 2's initial code in place.  One
+//                       per-group body (search_unit) under four deals of the units:
+//                         refine_kernel         2-D views, ragged rows (static)
+//                         refine_linear_kernel  contiguous W, static (a search beside
+//                                               another kernel, or a tiny one)
+//                         refine_sm_kernel      contiguous W alone on the GPU: one CTA per
+//                                               SM, units shared through shared memory
+//                         refine_shared_kernel  contiguous W, long searches: units shared
+//                                               through a counter in a caller workspace
 //   fourover6_codes_kernel  Algorithm 2's initial codes as a separate pass
 //   pack_kernel         exact FP4 quantization with given codes (Eq. 2)
 //
