@@ -276,9 +276,11 @@ int hscale_refine_scales(const void* w_bf16, const float* h, int64_t m, int64_t 
  * hscale_refine_scales with an explicit launch shape; the results are identical.
  * The paper has no counterpart: this is a scheduling knob for callers that run the
  * search alongside another kernel (e.g. the next input space's Hessian pass on another
- * stream).  ctas_per_sm = 0 fills every SM as hscale_refine_scales does; k > 0 keeps at
- * most k of the search's CTAs (128 threads, 72 registers each) resident per SM, leaving
- * the rest of the register file to concurrent work.  Negative values return
+ * stream).  ctas_per_sm = 0 fills every SM as hscale_refine_scales does (a search with at
+ * least two 32-group units per warp then runs as one CTA of 28 warps per SM whose warps
+ * share its units at run time; a smaller one as up to 7 CTAs of 4 warps per SM); k > 0
+ * keeps at most k of the search's CTAs (128 threads, 72 registers each) resident per SM,
+ * leaving the rest of the register file to concurrent work.  Negative values return
  * HSCALE_ERR_ARG.
  */
 int hscale_refine_scales_ex(const void* w_bf16, const float* h, int64_t m, int64_t n,
