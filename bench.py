@@ -613,8 +613,9 @@ def kernels_per_matrix(work: Work) -> int:
     return 4 if work.init == "4over6-2pass" else 3
 
 
-# the search kernels: the static deal, and the work-shared one for long searches
-SEARCH_KERNELS = "refine_linear_kernel|refine_shared_kernel"
+# the search kernels: one CTA per SM with a shared-memory queue (a matrix alone on the GPU),
+# the global work counter (long searches), the static deal (tiny searches)
+SEARCH_KERNELS = "refine_sm_kernel|refine_shared_kernel|refine_linear_kernel"
 
 
 def timed(fn, reps, flush=None):
