@@ -131,6 +131,19 @@ def test_step_graphs_reproduce_the_eager_step(workload, pipeline):
     graphs.bind(0)
 
 
+def test_search_schedule_policy():
+    """--search-schedule: 'auto' passes the work-sharing workspace to every search except
+    one that fills the SMs (7 CTAs each) beside a Hessian pass; 'shared' and 'static'
+    always and never."""
+    w = SimpleNamespace(search_schedule="auto")
+    assert bench.shares(w, 0) and bench.shares(w, 4) and bench.shares(w, 6)
+    assert not bench.shares(w, 7) and not bench.shares(w, 8)
+    w.search_schedule = "shared"
+    assert all(bench.shares(w, c) for c in (0, 4, 7))
+    w.search_schedule = "static"
+    assert not any(bench.shares(w, c) for c in (0, 4, 7))
+
+
 def test_step_hbm_counts_every_byte_of_the_step():
     """The whole-step HBM figure: X's bytes of the Hessian passes, W once for the global
     amax and once in the search (again for the two-pass 4over6 codes), and the codes and
