@@ -327,10 +327,12 @@ size_t hscale_refine_workspace_bytes(void);
  * hscale_refine_scales_ex; fourover6 as for hscale_refine_scales_strided (0 or 1; 1 with
  * init_codes returns HSCALE_ERR_ARG).
  * workspace        device memory of at least hscale_refine_workspace_bytes() bytes,
- *                  16-byte aligned, owned by the caller; or NULL for the static deal.  The
- *                  call zeroes its first 4 bytes on `stream` before the kernel and the
- *                  kernel counts in them, so calls that may run at the same time on the
- *                  GPU need distinct workspaces.  Nothing needs to persist between calls.
+ *                  16-byte aligned, owned by the caller; or NULL (no work sharing through
+ *                  it).  When the call shares units through it, it zeroes the first 4 bytes
+ *                  on `stream` before the kernel and the kernel counts in them, so calls
+ *                  that may run at the same time on the GPU need distinct workspaces; a
+ *                  short search leaves it untouched.  Nothing needs to persist between
+ *                  calls.
  * workspace_bytes  its size; below hscale_refine_workspace_bytes() returns
  *                  HSCALE_ERR_WORKSPACE (a misaligned workspace returns HSCALE_ERR_ALIGN).
  * The other status codes are those of hscale_refine_scales_strided.
