@@ -307,6 +307,11 @@ def test_binding_refuses_cpu_tensors(lib):
     h = torch.zeros(16)
     with pytest.raises(TypeError):
         hs.hscale_hessian_diag_accumulate(x, h)
+    w = torch.zeros(4, 512, dtype=torch.bfloat16)
+    sg = torch.ones(1)
+    codes = torch.zeros(4 * 32, dtype=torch.uint8)
+    with pytest.raises(TypeError):   # host tensors, before any call into the library
+        hs.hscale_refine_scales_ws(w, None, sg, None, 0, 4, 4, codes, None, 0, torch.zeros(16, dtype=torch.uint8))
 
 
 def test_build_flags_target_sm103a_only():
