@@ -235,14 +235,16 @@ __device__ __forceinline__ float group_energy(const Group& G, const float2 (&hv2
   return __fmul_rn(__fadd_rn(acc.x, acc.y), 1.0f + 0x1p-19f);
 }
 
-// A sufficient condition for fast_winner_certain that costs five operations: a relative
+// A sufficient condition for fast_winner_certain that costs six operations: a relative
 // gap above 2^-9 with A <= 2^18 E2 (A_bound any upper bound of A, here (sum h) amax^2)
 // gives a margin of at most (2^-18 + 2^-19 2^9 + 2^-35 2^18) E2 < 2^-9 E2, and
 // E2 >= 2^-36 A.  (The fp32 rounding of the gap and of A_bound is a few units of 2^-24,
-// far inside the factor of two between 2^-9 and the margin.)  A zero, infinite or NaN
-// runner-up fails it.
+// far inside the factor of two between 2^-9 and the margin.)  The scores' error bound
+// holds for results in the normal range, so a runner-up below 2^-100 is left to
+// fast_winner_certain (which sends denormal ones to the exact rescoring); a zero,
+// infinite or NaN runner-up fails it too.
 __device__ __forceinline__ bool fast_winner_clear(float e1, float e2, float A_bound) {
-  return __fsub_rn(e2, e1) > __fmul_rn(0x1p-9f, e2) && A_bound <= __fmul_rn(0x1p18f, e2);
+  return e2 >= 0x1p-100f && __fsub_rn(e2, e1) > __fmul_rn(0x1p-9f, e2) && A_bound <= __fmul_rn(0x1p18f, e2);
 }
 
 // tie rule of the search: smaller error, then smaller |shift|, then smaller shift
