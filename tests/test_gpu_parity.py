@@ -573,6 +573,27 @@ def test_search_schedules_on_extreme_shapes(m, n):
         assert np.array_equal(other[0], queue[0]) and np.array_equal(other[1], queue[1])
 
 
+def test_search_schedules_without_h():
+    """h = NULL (the plain weight-MSE search of the h = 1 special case) under the three
+    deals: the per-SM queue, the global counter and the static deal, against the oracle's
+    unweighted search."""
+    m, n, down, up = 4095, 4096, 8, 8
+    w = wl.weight(m, n, 0.02, 24, device="cpu")
+    wd = w.to(dev())
+    sg, _ = gpu_rtn(wd)
+    wb = bits(w)
+    s_ref, _ = oracle.global_scale(wb)
+    ref = oracle.refine(wb, None, s_ref, None, down, up)
+    queue = gpu_refine_ws(wd, None, sg, None, 0, down, up, 0, None)
+    compare_search(ref, *queue, f"per-SM queue {m}x{n} h = NULL")
+    ws = torch.full((16,), 0xAB, dtype=torch.uint8, device=dev())
+    shared = gpu_refine_ws(wd, None, sg, None, 0, down, up, 1, ws)
+    assert shared_schedule_ran(ws)
+    static = gpu_refine_ws(wd, None, sg, None, 0, down, up, 7, None)
+    for other in (shared, static):
+        assert np.array_equal(other[0], queue[0]) and np.array_equal(other[1], queue[1])
+
+
 def test_shared_schedule_only_for_long_searches():
     """A short search (4096 x 4096 at k = 4 over every SM) keeps the static deal and leaves
     the workspace untouched; the bytes equal hscale_refine_scales'."""
